@@ -1,0 +1,302 @@
+/*
+ * FOCUS oracle: plain, slow, fp64 CPU statement of what the compressed-context
+ * attention path computes (arXiv 2511.14694, Appendix A).
+ *
+ * TEST INFRASTRUCTURE ONLY. The test suite, the smoke check and the benchmark's
+ * CPU-baseline leg are the only users. The CUDA library never includes, links
+ * or calls this file, and this file shares nothing with it.
+ *
+ * Conventions
+ *   - Nucleotide ids are 0..3 (A, C, G, T); the reserved summary-token id is 4
+ *     (Table "Full configuration": "Special FOCUS token: reserved").
+ *   - Indices are 0-based. Window w covers bases [w*W, min((w+1)*W, N)), the
+ *     0-based form of I_w = [(w-1)W+1, wW] ∩ [1, L]  (App. A, first display).
+ *   - Q/K/V arrive as raw bf16 bit patterns (uint16) exactly as the GPU sees
+ *     them; each is widened to fp64 here (bf16 -> fp32 is exact, fp32 -> fp64
+ *     is exact). All arithmetic after that is fp64.
+ *   - Softmax scale is a caller argument; LSE is the natural log of the sum of
+ *     exponentials of the scaled scores.
+ *
+ * Every loop below runs in the order the paper states the operation; nothing is
+ * blocked, fused or reordered.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define FO_SUMMARY_TOKEN 4
+
+static double bf16_to_f64(uint16_t bits) {
+    uint32_t u = ((uint32_t)bits) << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Token layout (App. A: windows I_w, M = ceil(L/W), B_w = ceil(|I_w|/k),     */
+/* one FOCUS token per k real bases at the right boundary of its k-mer,       */
+/* each FOCUS token occupying a real sequence position).                      */
+/* ------------------------------------------------------------------------- */
+
+/* Does a summary follow the base at in-window offset o (0-based) of a window
+ * holding n bases with cadence k? A summary closes every full k-mer, and the
+ * partial k-mer at the window's end when `close_partial` is set (the ceil in
+ * B_w = ceil(|I_w|/k)). k == 0 means "no summaries" (compression disabled). */
+static int summary_after(int64_t o, int64_t n, int32_t k, int close_partial) {
+    if (k <= 0) return 0;
+    if ((o + 1) % k == 0) return 1;
+    return (o == n - 1) && close_partial;
+}
+
+/* Sizes of the augmented layout. Returns T (augmented length) and writes R
+ * (retained summaries after the last window). Returns -1 on bad arguments. */
+int64_t fo_layout_size(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
+                       int32_t close_tail, int64_t* R_out) {
+    if (N < 0 || W <= 0) return -1;
+    int64_t M_expect = (N + W - 1) / W;
+    if (M != M_expect) return -1;
+    int64_t T = 0, R = 0;
+    for (int32_t w = 0; w < M; ++w) {
+        int64_t start = (int64_t)w * W;
+        int64_t n = (N - start < W) ? (N - start) : W;
+        int close = (w < M - 1) || close_tail;
+        for (int64_t o = 0; o < n; ++o) {
+            T += 1;
+            if (summary_after(o, n, k_sched[w], close)) { T += 1; R += 1; }
+        }
+    }
+    if (R_out) *R_out = R;
+    return T;
+}
+
+/* Full layout walk. For every augmented index t:
+ *   kind[t]  0 = ordinary base, 1 = FOCUS summary
+ *   src[t]   nucleotide index of the base (for a summary: its k-mer's last base)
+ *   pos[t]   position id = t (a summary occupies a real sequence position)
+ *   win[t]   window id w
+ *   tok[b*T + t]  nucleotide id nt[b*N + src] for bases, 4 for summaries
+ *                 (written only when nt and tok are both non-NULL)
+ * plus win_off[M+1] (first augmented index of each window, win_off[M] = T),
+ * ring_off[M+1] (summaries retained before each window, ring_off[M] = R) and
+ * sum_idx[R] (augmented index of each summary, in order).
+ * Returns T, or -1 on bad arguments. */
+int64_t fo_layout(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
+                  int32_t close_tail, int32_t B, const uint8_t* nt,
+                  uint8_t* kind, int32_t* src, int32_t* pos, int32_t* win,
+                  uint8_t* tok, int32_t* win_off, int32_t* ring_off,
+                  int32_t* sum_idx) {
+    int64_t R_total = 0;
+    int64_t T_total = fo_layout_size(N, W, M, k_sched, close_tail, &R_total);
+    if (T_total < 0) return -1;
+    int64_t t = 0, r = 0;
+    for (int32_t w = 0; w < M; ++w) {
+        int64_t start = (int64_t)w * W;
+        int64_t n = (N - start < W) ? (N - start) : W;
+        int close = (w < M - 1) || close_tail;
+        win_off[w] = (int32_t)t;
+        ring_off[w] = (int32_t)r;
+        for (int64_t o = 0; o < n; ++o) {
+            int64_t base = start + o;
+            kind[t] = 0; src[t] = (int32_t)base; pos[t] = (int32_t)t; win[t] = w;
+            if (nt && tok)
+                for (int32_t b = 0; b < B; ++b) tok[(int64_t)b * T_total + t] = nt[(int64_t)b * N + base];
+            t += 1;
+            if (summary_after(o, n, k_sched[w], close)) {
+                kind[t] = 1; src[t] = (int32_t)base; pos[t] = (int32_t)t; win[t] = w;
+                if (nt && tok)
+                    for (int32_t b = 0; b < B; ++b) tok[(int64_t)b * T_total + t] = FO_SUMMARY_TOKEN;
+                sum_idx[r] = (int32_t)t;
+                r += 1;
+                t += 1;
+            }
+        }
+    }
+    win_off[M] = (int32_t)t;
+    ring_off[M] = (int32_t)r;
+    return t;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Softmax attention of one query row over an explicit, ordered list of key   */
+/* rows: s_j = scale * <q, k_j>, m = max s, l = sum exp(s_j - m),             */
+/* o = sum exp(s_j - m) v_j / l, LSE = m + ln l.                              */
+/* ------------------------------------------------------------------------- */
+static void softmax_row(int32_t d, const uint16_t* q, int64_t n_keys,
+                        const uint16_t* const* krows, const uint16_t* const* vrows,
+                        double scale, double* o, double* lse) {
+    double* qd = (double*)malloc(sizeof(double) * (size_t)d);
+    double* s = (double*)malloc(sizeof(double) * (size_t)(n_keys > 0 ? n_keys : 1));
+    for (int32_t c = 0; c < d; ++c) qd[c] = bf16_to_f64(q[c]);
+    double m = -INFINITY;
+    for (int64_t j = 0; j < n_keys; ++j) {
+        double dot = 0.0;
+        for (int32_t c = 0; c < d; ++c) dot += qd[c] * bf16_to_f64(krows[j][c]);
+        s[j] = scale * dot;
+        if (s[j] > m) m = s[j];
+    }
+    double l = 0.0;
+    for (int32_t c = 0; c < d; ++c) o[c] = 0.0;
+    for (int64_t j = 0; j < n_keys; ++j) {
+        double p = exp(s[j] - m);
+        l += p;
+        for (int32_t c = 0; c < d; ++c) o[c] += p * bf16_to_f64(vrows[j][c]);
+    }
+    for (int32_t c = 0; c < d; ++c) o[c] /= l;
+    *lse = m + log(l);
+    free(s);
+    free(qd);
+}
+
+/* ------------------------------------------------------------------------- */
+/* Masked-parallel form (App. A.1, "Cross-window consistency" (ii), with the  */
+/* visible set of Eq. focus-attn / C(t)): row i sees key j iff j <= i and     */
+/* (j is in the same window as i, or j is a FOCUS token).                     */
+/*                                                                            */
+/* q, k, v: [n_heads][T][d] bf16 bits. Computes the requested rows only:     */
+/* row r is (head row_head[r], augmented index row_idx[r]). Outputs o[r][d],  */
+/* lse[r].                                                                    */
+/* ------------------------------------------------------------------------- */
+void fo_attn_rows(int64_t T, int32_t d, const uint8_t* kind, const int32_t* win,
+                  const uint16_t* q, const uint16_t* k, const uint16_t* v,
+                  double scale, int64_t n_rows, const int64_t* row_head,
+                  const int64_t* row_idx, double* o, double* lse) {
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t r = 0; r < n_rows; ++r) {
+        int64_t h = row_head[r], i = row_idx[r];
+        const uint16_t* kh = k + (size_t)h * (size_t)T * (size_t)d;
+        const uint16_t* vh = v + (size_t)h * (size_t)T * (size_t)d;
+        const uint16_t** kr = (const uint16_t**)malloc(sizeof(void*) * (size_t)(i + 1));
+        const uint16_t** vr = (const uint16_t**)malloc(sizeof(void*) * (size_t)(i + 1));
+        int64_t n = 0;
+        for (int64_t j = 0; j <= i; ++j) {
+            int visible = (win[j] == win[i]) || (kind[j] == 1);
+            if (!visible) continue;
+            kr[n] = kh + (size_t)j * d;
+            vr[n] = vh + (size_t)j * d;
+            n += 1;
+        }
+        softmax_row(d, q + ((size_t)h * (size_t)T + (size_t)i) * d, n, kr, vr, scale,
+                    o + (size_t)r * d, lse + r);
+        free(kr);
+        free(vr);
+    }
+}
+
+/* ------------------------------------------------------------------------- */
+/* Sequential form (App. A.1 (i); App. A.2 "Streaming with controlled         */
+/* memory"): windows in order; each row of window w attends to the retained   */
+/* FOCUS KV of earlier windows and to the rows of window w up to itself;      */
+/* after window w its ordinary KV is dropped and its FOCUS KV is appended to   */
+/* the retained set (App. A, "KV compression and budget").                    */
+/*                                                                            */
+/* One head: q, k, v are [T][d] bf16 bits; win_off[M+1] gives window rows;    */
+/* kind[T] marks FOCUS rows. want[M] (NULL = all) selects the windows whose    */
+/* outputs are computed; retention runs for every window regardless. Writes   */
+/* o[T][d], lse[T] for computed windows (others untouched) and the retained   */
+/* KV (ring_k/ring_v, [ring_cap][d]) with its length in *R_out.               */
+/* Returns 0, or -1 if ring_cap is too small.                                 */
+/* ------------------------------------------------------------------------- */
+int32_t fo_prefill_sequential(int32_t d, int32_t M, const int32_t* win_off,
+                              const uint8_t* kind, const uint16_t* q,
+                              const uint16_t* k, const uint16_t* v, double scale,
+                              const uint8_t* want, double* o, double* lse,
+                              uint16_t* ring_k, uint16_t* ring_v, int64_t ring_cap,
+                              int64_t* R_out) {
+    int64_t R = 0;
+    for (int32_t w = 0; w < M; ++w) {
+        int64_t a = win_off[w], e = win_off[w + 1];
+        if (!want || want[w]) {
+#pragma omp parallel for schedule(dynamic, 8)
+            for (int64_t i = a; i < e; ++i) {
+                int64_t nk = R + (i - a + 1);
+                const uint16_t** kr = (const uint16_t**)malloc(sizeof(void*) * (size_t)nk);
+                const uint16_t** vr = (const uint16_t**)malloc(sizeof(void*) * (size_t)nk);
+                int64_t n = 0;
+                for (int64_t j = 0; j < R; ++j) {          /* retained history */
+                    kr[n] = ring_k + (size_t)j * d;
+                    vr[n] = ring_v + (size_t)j * d;
+                    n += 1;
+                }
+                for (int64_t j = a; j <= i; ++j) {          /* current window, causal */
+                    kr[n] = k + (size_t)j * d;
+                    vr[n] = v + (size_t)j * d;
+                    n += 1;
+                }
+                softmax_row(d, q + (size_t)i * d, n, kr, vr, scale, o + (size_t)i * d, lse + i);
+                free(kr);
+                free(vr);
+            }
+        }
+        /* window finished: keep FOCUS KV, drop ordinary KV */
+        for (int64_t j = a; j < e; ++j) {
+            if (kind[j] != 1) continue;
+            if (R >= ring_cap) return -1;
+            memcpy(ring_k + (size_t)R * d, k + (size_t)j * d, sizeof(uint16_t) * (size_t)d);
+            memcpy(ring_v + (size_t)R * d, v + (size_t)j * d, sizeof(uint16_t) * (size_t)d);
+            R += 1;
+        }
+    }
+    *R_out = R;
+    return 0;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Decode (App. A.2): one new token per sequence. Its K/V are appended to the */
+/* current window; its query attends to the retained FOCUS KV (ring, R rows)  */
+/* and to the current window's rows up to and including itself.              */
+/*                                                                            */
+/* Batched over n independent (sequence, head) streams: stream s has          */
+/* ring_k/ring_v rows [s*ring_stride, +R[s]) and window rows                   */
+/* [s*win_stride, +fill[s]) (fill BEFORE the append). q/k_new/v_new: [n][d].  */
+/* The append itself is the caller's (this routine reads k_new/v_new as the   */
+/* last visible row). Outputs o[n][d], lse[n].                                */
+/* ------------------------------------------------------------------------- */
+void fo_decode(int32_t d, int64_t n, const uint16_t* ring_k, const uint16_t* ring_v,
+               int64_t ring_stride, const int64_t* R, const uint16_t* win_k,
+               const uint16_t* win_v, int64_t win_stride, const int64_t* fill,
+               const uint16_t* q, const uint16_t* k_new, const uint16_t* v_new,
+               double scale, double* o, double* lse) {
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t s = 0; s < n; ++s) {
+        int64_t nk = R[s] + fill[s] + 1;
+        const uint16_t** kr = (const uint16_t**)malloc(sizeof(void*) * (size_t)nk);
+        const uint16_t** vr = (const uint16_t**)malloc(sizeof(void*) * (size_t)nk);
+        int64_t c = 0;
+        for (int64_t j = 0; j < R[s]; ++j) {
+            kr[c] = ring_k + ((size_t)s * ring_stride + (size_t)j) * d;
+            vr[c] = ring_v + ((size_t)s * ring_stride + (size_t)j) * d;
+            c += 1;
+        }
+        for (int64_t j = 0; j < fill[s]; ++j) {
+            kr[c] = win_k + ((size_t)s * win_stride + (size_t)j) * d;
+            vr[c] = win_v + ((size_t)s * win_stride + (size_t)j) * d;
+            c += 1;
+        }
+        kr[c] = k_new + (size_t)s * d;
+        vr[c] = v_new + (size_t)s * d;
+        c += 1;
+        softmax_row(d, q + (size_t)s * d, c, kr, vr, scale, o + (size_t)s * d, lse + s);
+        free(kr);
+        free(vr);
+    }
+}
+
+/* In-window offsets (augmented, 0-based) of the FOCUS rows of one window of n
+ * bases with cadence k, i.e. which rows KV retention keeps (App. A, "KV
+ * compression and budget"). Writes up to cap offsets; returns their count. */
+int32_t fo_window_summary_rows(int64_t n, int32_t k, int32_t close_partial,
+                               int32_t* out, int32_t cap) {
+    int64_t t = 0;
+    int32_t c = 0;
+    for (int64_t o = 0; o < n; ++o) {
+        t += 1;
+        if (summary_after(o, n, k, close_partial)) {
+            if (c < cap) out[c] = (int32_t)t;
+            c += 1;
+            t += 1;
+        }
+    }
+    return c;
+}

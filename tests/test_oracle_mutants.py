@@ -1,0 +1,59 @@
+"""Plant plausible mistakes in a copy of the oracle (on the CPU) and check that
+the pins in test_oracle_pins.py fail for each one: a pin that no mistake can
+trip pins nothing."""
+import os
+import subprocess
+
+import pytest
+
+from oracle import focus_oracle as fo
+import test_oracle_pins as pins
+
+SRC = os.path.join(os.path.dirname(fo.__file__), "focus_oracle.c")
+
+# (name, exact text in focus_oracle.c, replacement, pin functions that must fail)
+MUTANTS = [
+    ("ring_dropped", "int visible = (win[j] == win[i]) || (kind[j] == 1);",
+     "int visible = (win[j] == win[i]);",
+     [lambda: pins.test_lse_of_zero_scores_counts_visible_keys(),
+      lambda: pins.test_attn_matches_streaming_simulation(40, 7, [2], 2, 16)]),
+    ("all_past_visible", "int visible = (win[j] == win[i]) || (kind[j] == 1);",
+     "int visible = 1;",
+     [lambda: pins.test_lse_of_zero_scores_counts_visible_keys()]),
+    ("strict_causal", "for (int64_t j = 0; j <= i; ++j) {\n            int visible",
+     "for (int64_t j = 0; j < i; ++j) {\n            int visible",
+     [lambda: pins.test_no_compression_is_plain_causal()]),
+    ("exp_sign", "double p = exp(s[j] - m);", "double p = exp(m - s[j]);",
+     [lambda: pins.test_no_compression_is_plain_causal()]),
+    ("k_for_v", "dot += qd[c] * bf16_to_f64(krows[j][c]);", "dot += qd[c] * bf16_to_f64(vrows[j][c]);",
+     [lambda: pins.test_no_compression_is_plain_causal()]),
+    ("scale_dropped", "s[j] = scale * dot;", "s[j] = dot;",
+     [lambda: pins.test_no_compression_is_plain_causal()]),
+    ("lse_no_max", "*lse = m + log(l);", "*lse = log(l);",
+     [lambda: pins.test_first_row_sees_only_itself()]),
+    ("summary_before_boundary", "if ((o + 1) % k == 0) return 1;", "if (o % k == 0) return 1;",
+     [lambda: pins.test_layout_positions_closed_form(10), lambda: pins.test_layout_fig1_golden()]),
+    ("partial_kmer_open", "return (o == n - 1) && close_partial;", "return 0;",
+     [lambda: pins.test_layout_fig1_golden(),
+      lambda: pins.test_layout_sizes_closed_form(5_000, 1_024, [100])]),
+    ("retain_ordinary", "if (kind[j] != 1) continue;\n            if (R >= ring_cap)",
+     "if (kind[j] != 0) continue;\n            if (R >= ring_cap)",
+     [lambda: pins.test_sequential_equals_masked_parallel(700, 100, [10])]),
+    ("decode_skips_self", "        kr[c] = k_new + (size_t)s * d;\n        vr[c] = v_new + (size_t)s * d;\n        c += 1;\n",
+     "", [lambda: pins.test_decode_equals_prefill_row()]),
+]
+
+
+@pytest.mark.parametrize("name,old,new,checks", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_pins_catch_planted_mistake(tmp_path, name, old, new, checks):
+    src = open(SRC).read()
+    assert src.count(old) == 1, f"mutation site for {name} not unique/found"
+    mut = tmp_path / f"mut_{name}.c"
+    mut.write_text(src.replace(old, new))
+    so = tmp_path / f"libmut_{name}.so"
+    subprocess.run(["gcc", "-O2", "-std=c11", "-fopenmp", "-fPIC", "-shared", str(mut), "-o", str(so), "-lm"],
+                   check=True)
+    with fo.use_library(str(so)):
+        for check in checks:
+            with pytest.raises((AssertionError, ValueError, IndexError)):
+                check()

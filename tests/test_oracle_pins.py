@@ -1,0 +1,319 @@
+"""Pins the fp64 oracle to facts fixed by the paper and by mathematics, not to
+itself: closed forms of the layout (App. A), a hand-spelled Fig. 1 layout, an
+independent string construction, a KV-retention simulation that builds the
+visible sets from the streaming process (App. A.2) instead of the visibility
+predicate, exact reductions to causal attention (library SDPA), invariants
+(rows of P sum to one, LSE of zero scores counts the visible set), the
+sequential == masked-parallel equivalence (App. A.1) and decode == prefill.
+"""
+import math
+import os
+
+import numpy as np
+import pytest
+import scipy.special
+import torch
+
+from oracle import focus_oracle as fo
+from paper_2511_14694_gb300 import inputs
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _ceil(a, b):
+    return -(-a // b)
+
+
+# ----------------------------------------------------------------------------- layout
+
+LAYOUT_CASES = [
+    (4_000, 1_000, [100]),
+    (1_000, 1_024, [100]),          # one partial window, W mod k != 0 (Table: W=1024, k=100)
+    (5_000, 1_024, [100]),
+    (10, 4, [3]),                    # Fig. 1 shape
+    (37, 7, [1]),
+    (37, 7, [7]),
+    (37, 7, [9]),                    # k > W: one summary per window
+    (50, 50, [0]),                   # compression disabled
+    (2_500, 1_000, [10, 25, 200]),   # per-window cadence
+]
+
+
+@pytest.mark.parametrize("N,W,ks", LAYOUT_CASES)
+def test_layout_sizes_closed_form(N, W, ks):
+    M = _ceil(N, W)
+    k = inputs.k_schedule(M, ks, seed=3)
+    T, R, M2 = fo.layout_size(N, W, k)
+    assert M2 == M
+    n_w = [min(W, N - w * W) for w in range(M)]
+    B_w = [(_ceil(n, int(kk)) if kk > 0 else 0) for n, kk in zip(n_w, k)]   # B_w = ceil(|I_w|/k)
+    assert R == sum(B_w)
+    assert T == N + sum(B_w)                                                  # N' = N + #summaries
+    # KV budget, eq. kv-budget: R_kept <= sum_w ceil(W/k_w) + W
+    assert R <= sum(_ceil(W, int(kk)) if kk > 0 else 0 for kk in k) + W
+
+
+@pytest.mark.parametrize("k", [1, 4, 10, 100])
+def test_layout_positions_closed_form(k):
+    """k | W, full windows: base i sits at i + floor(i/k); summary j at (j+1)(k+1)-1;
+    after n windows the retained count is n*W/k."""
+    W, n = 100, 7
+    if W % k:
+        pytest.skip("needs k | W")
+    N = n * W
+    L = fo.layout(N, W, [k])
+    base_pos = L["pos"][L["kind"] == 0]
+    assert np.array_equal(base_pos, np.arange(N) + np.arange(N) // k)
+    assert np.array_equal(L["sum_idx"], (np.arange(N // k) + 1) * (k + 1) - 1)
+    assert np.array_equal(L["ring_off"], np.arange(n + 1) * (W // k))
+    assert np.array_equal(L["pos"], np.arange(L["T"]))
+    assert np.array_equal(L["win_off"], np.arange(n + 1) * (W + W // k))
+
+
+def _string_layout(seq, W, ks, close_tail=True):
+    """Independent construction: cut the base string into windows, each window
+    into k-chunks, and write 'S' after every chunk (the last chunk of the final
+    window only if close_tail)."""
+    out = []
+    M = _ceil(len(seq), W)
+    for w in range(M):
+        chunk = seq[w * W:(w + 1) * W]
+        k = int(ks[w])
+        if k == 0:
+            out.append(chunk)
+            continue
+        pieces = [chunk[i:i + k] for i in range(0, len(chunk), k)]
+        for pi, p in enumerate(pieces):
+            last = pi == len(pieces) - 1
+            closes = len(p) == k or w < M - 1 or close_tail
+            out.append(p + ("S" if (not last or closes) else ""))
+    return "".join(out)
+
+
+@pytest.mark.parametrize("N,W,ks", LAYOUT_CASES)
+@pytest.mark.parametrize("close_tail", [True, False])
+def test_layout_matches_string_construction(N, W, ks, close_tail):
+    M = _ceil(N, W)
+    k = inputs.k_schedule(M, ks, seed=5)
+    nt = inputs.nucleotides(2, N, seed=11).numpy()
+    L = fo.layout(N, W, k, nt=nt, close_tail=close_tail)
+    for b in range(2):
+        seq = "".join("ACGT"[x] for x in nt[b])
+        expect = _string_layout(seq, W, k, close_tail)
+        got = "".join("ACGTS"[x] for x in L["tok"][b])
+        assert got == expect
+    assert "".join("BS"[x] for x in L["kind"]) == "".join("S" if c == "S" else "B" for c in expect)
+
+
+def test_layout_fig1_golden():
+    rows = []
+    with open(os.path.join(GOLDEN, "fig1_layout_k3_W4.txt")) as f:
+        for line in f:
+            if line.strip() and not line.startswith("#"):
+                t, kind, src, w = line.split()
+                rows.append((int(t), kind, int(src), int(w)))
+    L = fo.layout(10, 4, [3])
+    assert L["T"] == len(rows)
+    for t, kind, src, w in rows:
+        assert L["pos"][t] == t
+        assert "BS"[L["kind"][t]] == kind
+        assert L["src"][t] == src
+        assert L["win"][t] == w
+    assert list(L["win_off"]) == [0, 6, 12, 15]
+    assert list(L["ring_off"]) == [0, 2, 4, 5]
+
+
+def test_window_summary_rows_match_layout():
+    for n, k in [(1000, 100), (1024, 100), (4, 3), (7, 9), (5, 1)]:
+        L = fo.layout(n, n, [k])
+        assert np.array_equal(fo.window_summary_rows(n, k), np.nonzero(L["kind"] == 1)[0])
+
+
+# ----------------------------------------------------------------------------- attention
+
+
+def _rand_case(N, W, ks, H, d, seed, std=1.0):
+    M = _ceil(N, W)
+    k = inputs.k_schedule(M, ks, seed=seed)
+    L = fo.layout(N, W, k)
+    q, kk, v = inputs.qkv((H, L["T"], d), std=std, seed=seed)
+    return L, q, kk, v
+
+
+def _visible_sets_by_streaming(L):
+    """KV-retention simulation (App. A.2): process windows in order; a row sees
+    the retained set plus the current window up to itself; after the window,
+    only FOCUS rows join the retained set."""
+    retained, vis = [], {}
+    for w in range(L["M"]):
+        a, e = L["win_off"][w], L["win_off"][w + 1]
+        for i in range(a, e):
+            vis[i] = list(retained) + list(range(a, i + 1))
+        retained += [j for j in range(a, e) if L["kind"][j] == 1]
+    return vis
+
+
+def _f64(x):
+    return x.to(torch.float64).numpy()
+
+
+ATTN_CASES = [
+    (10, 4, [3], 2, 8),       # Fig. 1 shape
+    (40, 7, [2], 2, 16),
+    (64, 64, [5], 1, 8),      # W >= N with summaries
+    (64, 9, [1], 1, 8),       # every base summarised
+    (60, 10, [20], 2, 8),     # k > W
+    (63, 8, [1, 2, 3, 9], 2, 16),
+]
+
+
+@pytest.mark.parametrize("N,W,ks,H,d", ATTN_CASES)
+def test_attn_matches_streaming_simulation(N, W, ks, H, d):
+    L, q, k, v = _rand_case(N, W, ks, H, d, seed=N + W)
+    T = L["T"]
+    scale = 1.0 / math.sqrt(d)
+    heads = np.repeat(np.arange(H), T)
+    rows = np.tile(np.arange(T), H)
+    o, lse = fo.attn_rows(q, k, v, L["kind"], L["win"], scale, heads, rows)
+    vis = _visible_sets_by_streaming(L)
+    qd, kd, vd = _f64(q), _f64(k), _f64(v)
+    for r, (h, i) in enumerate(zip(heads, rows)):
+        j = np.array(vis[i])
+        s = scale * (kd[h, j] @ qd[h, i])
+        p = scipy.special.softmax(s)
+        np.testing.assert_allclose(o[r], p @ vd[h, j], rtol=0, atol=1e-12)
+        assert abs(lse[r] - scipy.special.logsumexp(s)) <= 1e-12 * max(1.0, abs(lse[r]))
+
+
+def test_no_compression_is_plain_causal():
+    """k = 0 and W >= N: exactly causal attention (App. A.2: the interface reduces
+    to the base decoder), checked against torch's SDPA in fp64."""
+    N, H, d = 96, 3, 32
+    L, q, k, v = _rand_case(N, N, [0], H, d, seed=1)
+    assert L["T"] == N and L["R"] == 0
+    heads = np.repeat(np.arange(H), N)
+    rows = np.tile(np.arange(N), H)
+    o, lse = fo.attn_rows(q, k, v, L["kind"], L["win"], 1.0 / math.sqrt(d), heads, rows)
+    qd, kd, vd = (x.to(torch.float64) for x in (q, k, v))
+    ref = torch.nn.functional.scaled_dot_product_attention(qd, kd, vd, is_causal=True)
+    np.testing.assert_allclose(o.reshape(H, N, d), ref.numpy(), rtol=0, atol=1e-12)
+    s = (qd @ kd.transpose(-1, -2)) / math.sqrt(d)
+    s = s.masked_fill(torch.triu(torch.ones(N, N, dtype=torch.bool), 1), float("-inf"))
+    np.testing.assert_allclose(lse.reshape(H, N), torch.logsumexp(s, -1).numpy(), rtol=1e-13, atol=0)
+
+
+def test_single_window_with_summaries_is_causal_over_augmented():
+    N, H, d = 50, 2, 16
+    L, q, k, v = _rand_case(N, 64, [4], H, d, seed=2)
+    T = L["T"]
+    heads = np.repeat(np.arange(H), T)
+    rows = np.tile(np.arange(T), H)
+    o, _ = fo.attn_rows(q, k, v, L["kind"], L["win"], 0.3, heads, rows)
+    ref = torch.nn.functional.scaled_dot_product_attention(
+        *(x.to(torch.float64) for x in (q, k, v)), is_causal=True, scale=0.3)
+    np.testing.assert_allclose(o.reshape(H, T, d), ref.numpy(), rtol=0, atol=1e-12)
+
+
+def test_softmax_rows_sum_to_one():
+    """V = 1 everywhere => every output is sum(p)/l = 1 (rows of P sum to 1)."""
+    L, q, k, _ = _rand_case(300, 40, [7], 2, 16, seed=4, std=3.0)
+    v = torch.ones_like(k)
+    T = L["T"]
+    heads = np.repeat(np.arange(2), T)
+    rows = np.tile(np.arange(T), 2)
+    o, _ = fo.attn_rows(q, k, v, L["kind"], L["win"], 1.0, heads, rows)
+    assert np.abs(o - 1.0).max() <= 1e-12
+
+
+def test_lse_of_zero_scores_counts_visible_keys():
+    """q = 0 => all scores 0 => LSE_i = ln |visible(i)| = ln(R_w + a + 1), with R_w
+    the summaries retained before window w and a the in-window offset of row i."""
+    N, W, ks = 500, 60, [1, 7, 13, 60, 100]
+    M = _ceil(N, W)
+    kk = inputs.k_schedule(M, ks, seed=8)
+    L = fo.layout(N, W, kk)
+    T = L["T"]
+    q = torch.zeros((1, T, 8), dtype=torch.bfloat16)
+    _, k, v = inputs.qkv((1, T, 8), seed=9)
+    o, lse = fo.attn_rows(q, k, v, L["kind"], L["win"], 1.0, np.zeros(T, np.int64), np.arange(T))
+    w = L["win"]
+    count = L["ring_off"][w] + (np.arange(T) - L["win_off"][w]) + 1
+    np.testing.assert_allclose(lse, np.log(count), rtol=0, atol=1e-12)
+
+
+def test_first_row_sees_only_itself():
+    L, q, k, v = _rand_case(30, 10, [3], 1, 8, seed=6)
+    o, lse = fo.attn_rows(q, k, v, L["kind"], L["win"], 0.5, [0], [0])
+    assert np.array_equal(o[0], _f64(v)[0, 0])
+    assert lse[0] == pytest.approx(0.5 * float(_f64(q)[0, 0] @ _f64(k)[0, 0]), abs=1e-14)
+
+
+# ----------------------------------------------------------------------------- retention / sequential
+
+
+@pytest.mark.parametrize("N,W,ks", [(700, 100, [10]), (1024, 100, [7, 30, 100]), (333, 50, [1, 51]),
+                                    (90, 200, [4])])
+def test_sequential_equals_masked_parallel(N, W, ks):
+    """App. A.1: sequential windows with KV dropping == masked-parallel."""
+    H, d = 2, 16
+    L, q, k, v = _rand_case(N, W, ks, H, d, seed=N)
+    T = L["T"]
+    for h in range(H):
+        o_s, lse_s, rk, rv = fo.prefill_sequential(q[h], k[h], v[h], L["win_off"], L["kind"], 0.25)
+        o_p, lse_p = fo.attn_rows(q, k, v, L["kind"], L["win"], 0.25, np.full(T, h), np.arange(T))
+        np.testing.assert_allclose(o_s, o_p, rtol=0, atol=1e-12)
+        np.testing.assert_allclose(lse_s, lse_p, rtol=0, atol=1e-12)
+        # retained KV == the FOCUS rows, bit for bit, count == sum_w B_w
+        kb = k[h].view(torch.int16).numpy().view(np.uint16)
+        vb = v[h].view(torch.int16).numpy().view(np.uint16)
+        assert rk.shape[0] == L["R"]
+        assert np.array_equal(rk, kb[L["sum_idx"]]) and np.array_equal(rv, vb[L["sum_idx"]])
+
+
+def test_retained_count_after_n_windows():
+    """After n full windows with k | W the ring holds n*W/k summaries per head."""
+    W, k, H, d = 200, 20, 1, 8
+    for n in (1, 2, 5):
+        L, q, kk, v = _rand_case(n * W, W, [k], H, d, seed=n)
+        _, _, rk, _ = fo.prefill_sequential(q[0], kk[0], v[0], L["win_off"], L["kind"], 1.0,
+                                            want=np.zeros(L["M"]))
+        assert rk.shape[0] == n * W // k
+
+
+# ----------------------------------------------------------------------------- decode
+
+
+def test_decode_equals_prefill_row():
+    """A decode step with the ring = retained summaries of earlier windows and the
+    window buffer = earlier rows of the current window reproduces prefill row t."""
+    N, W, ks, H, d = 900, 100, [9], 2, 16
+    L, q, k, v = _rand_case(N, W, ks, H, d, seed=12)
+    rng = np.random.default_rng(0)
+    ts = rng.integers(0, L["T"], size=24)
+    for h in range(H):
+        o_p, lse_p = fo.attn_rows(q, k, v, L["kind"], L["win"], 0.2, np.full(ts.size, h), ts)
+        for r, t in enumerate(ts):
+            w = L["win"][t]
+            ring_rows = L["sum_idx"][: L["ring_off"][w]]
+            a = L["win_off"][w]
+            ring_k = k[h][ring_rows][None] if ring_rows.size else torch.zeros((1, 1, d), dtype=torch.bfloat16)
+            ring_v = v[h][ring_rows][None] if ring_rows.size else torch.zeros((1, 1, d), dtype=torch.bfloat16)
+            wk = k[h][a:t][None] if t > a else torch.zeros((1, 1, d), dtype=torch.bfloat16)
+            wv = v[h][a:t][None] if t > a else torch.zeros((1, 1, d), dtype=torch.bfloat16)
+            o_d, lse_d = fo.decode(q[h][t][None], k[h][t][None], v[h][t][None], ring_k, ring_v,
+                                   [ring_rows.size], wk, wv, [t - a], 0.2)
+            np.testing.assert_allclose(o_d[0], o_p[r], rtol=0, atol=1e-12)
+            assert abs(lse_d[0] - lse_p[r]) <= 1e-12
+
+
+def test_decode_ring_order_is_irrelevant():
+    n, R, F, d = 3, 57, 11, 32
+    g = torch.Generator().manual_seed(1)
+    ring_k, ring_v = (torch.randn((n, R, d), generator=g).bfloat16() for _ in range(2))
+    win_k, win_v = (torch.randn((n, F, d), generator=g).bfloat16() for _ in range(2))
+    q, kn, vn = (torch.randn((n, d), generator=g).bfloat16() for _ in range(3))
+    o1, l1 = fo.decode(q, kn, vn, ring_k, ring_v, [R] * n, win_k, win_v, [F] * n, 0.3)
+    perm = torch.randperm(R, generator=g)
+    o2, l2 = fo.decode(q, kn, vn, ring_k[:, perm], ring_v[:, perm], [R] * n, win_k, win_v, [F] * n, 0.3)
+    np.testing.assert_allclose(o1, o2, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(l1, l2, rtol=0, atol=1e-12)
