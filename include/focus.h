@@ -1,0 +1,219 @@
+/*
+ * focus.h — C ABI of the GB300 FOCUS compressed-context attention library
+ * (libfocus.so). FOCUS: arXiv 2511.14694.
+ *
+ * What the library computes
+ *   A DNA sequence of N bases is cut into windows of W bases (App. A, I_w and
+ *   M = ceil(N/W)). Inside each window a FOCUS summary token is inserted after
+ *   every k_w bases, and after the partial k-mer that ends a window
+ *   (B_w = ceil(|I_w|/k_w), App. A; Sec. 3.2 "Setup and tokens"). Each inserted
+ *   token occupies a real sequence position. Row i of window w attends to
+ *   (a) the retained FOCUS K/V of all earlier windows and (b) the rows of
+ *   window w up to and including itself (Eq. focus-attn's visible set and the
+ *   context C(t) of App. A.1). After window w only its FOCUS K/V is kept
+ *   (App. A, "KV compression and budget"; App. A.2 streaming inference).
+ *
+ * Conventions for every entry point
+ *   - Ownership: the caller allocates and owns every buffer. Pointers named
+ *     d_* or documented as "device" are CUDA device pointers; "host" pointers
+ *     are ordinary host memory. The library never allocates device memory.
+ *   - Layouts are row-major with the head dimension d fastest. K/V/Q/O are
+ *     bf16 (raw 16-bit storage, passed as void*). All device pointers to bf16
+ *     tensors must be 16-byte aligned.
+ *   - Calls are asynchronous on the given stream (0 = legacy default stream)
+ *     unless stated otherwise. The return value reports argument errors found
+ *     on the host (nothing is launched then) and CUDA launch errors.
+ *   - Errors found by a kernel (a window buffer or ring overflowing, layout
+ *     sizes that disagree with the caller's) set a sticky per-device status
+ *     word; the affected work is skipped, never trapped. Read and clear it with
+ *     focus_get_device_status().
+ *   - Supported head dimensions: d = 64 and d = 128.
+ */
+#ifndef FOCUS_H_
+#define FOCUS_H_
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum focus_status {
+    FOCUS_OK = 0,
+    FOCUS_ERR_INVALID_ARG = 1,   /* null pointer, negative size, inconsistent shapes */
+    FOCUS_ERR_UNSUPPORTED = 2,   /* head dim not 64/128, misaligned pointer */
+    FOCUS_ERR_CAPACITY = 3,      /* ring or window buffer too small (host check or device word) */
+    FOCUS_ERR_CUDA = 4,          /* a CUDA call failed */
+    FOCUS_ERR_TIMEOUT = 5,       /* a bounded device wait gave up (device word only) */
+    FOCUS_ERR_LAYOUT = 6         /* device-computed layout disagrees with the caller's sizes */
+} focus_status;
+
+/* Summary token id written into the token stream (the reserved special token of
+ * Table "Full configuration"); nucleotide ids are 0..3 for A, C, G, T. */
+#define FOCUS_SUMMARY_TOKEN 4
+
+/* Layout flag: also close the partial k-mer at the end of the LAST window with a
+ * summary (App. A's ceil). Without it, the final partial k-mer stays open, which is
+ * what a caller that will continue the sequence by decoding wants. */
+#define FOCUS_LAYOUT_CLOSE_TAIL 1u
+
+/* ------------------------------------------------------------------------ */
+/* Library information                                                      */
+/* ------------------------------------------------------------------------ */
+
+/* Version of this ABI (major*10000 + minor*100 + patch). */
+int32_t focus_version(void);
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char* focus_status_string(focus_status s);
+
+/* Read the calling thread's current device's sticky status word into
+ * *host_status (FOCUS_OK if no kernel reported an error) and, if clear != 0,
+ * reset it to FOCUS_OK. Synchronises `stream` first (blocking). */
+focus_status focus_get_device_status(int32_t* host_status, int32_t clear, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------ */
+/* focus_layout — summary-token insertion and position ids                  */
+/* Sec. 3.2 "Setup and tokens"; App. A (I_w, M, B_w; FOCUS tokens occupy     */
+/* real sequence positions); Sec. 3.3 (augmented sequence y_1..y_N').       */
+/* ------------------------------------------------------------------------ */
+
+/* Host-only arithmetic: sizes of the augmented layout.
+ *   n_nt        N >= 0 bases
+ *   W           window length in bases, W >= 1
+ *   n_windows   M; must equal ceil(N/W)
+ *   h_k         HOST array [M]: cadence k_w >= 0 per window (0 = no summaries)
+ *   flags       FOCUS_LAYOUT_CLOSE_TAIL or 0
+ * Outputs (any may be NULL): *T augmented length N + sum_w B_w, *R summaries,
+ * *max_rows the largest per-window augmented row count. */
+focus_status focus_layout_size(int64_t n_nt, int32_t W, int32_t n_windows, const int32_t* h_k,
+                               uint32_t flags, int64_t* T, int64_t* R, int32_t* max_rows);
+
+/* Device arrays written by focus_layout. All are caller-allocated. */
+typedef struct focus_layout_out {
+    int64_t  T;          /* capacity/expected augmented length (from focus_layout_size) */
+    int64_t  R;          /* expected number of summaries (from focus_layout_size) */
+    uint8_t* kind;       /* [T] 0 = base, 1 = FOCUS summary */
+    int32_t* src;        /* [T] nucleotide index; a summary names the last base of its k-mer */
+    int32_t* pos;        /* [T] position id (0-based augmented index) */
+    int32_t* win;        /* [T] window id */
+    uint8_t* tok;        /* [B][T] token ids (nt id 0..3, summary FOCUS_SUMMARY_TOKEN); may be NULL */
+    int32_t* win_off;    /* [M+1] first augmented row of each window; win_off[M] = T */
+    int32_t* ring_off;   /* [M+1] summaries before each window; ring_off[M] = R */
+    int32_t* sum_idx;    /* [R] augmented index of each summary, in order (the compaction gather list) */
+} focus_layout_out;
+
+/* Device layout builder. d_k: DEVICE array [M] of cadences (same values as the
+ * host array given to focus_layout_size). d_nt: DEVICE uint8 [B][N] nucleotide ids
+ * (may be NULL, then tok is not written). If the device-computed T or R differs
+ * from out->T / out->R the device status word is set to FOCUS_ERR_LAYOUT. */
+focus_status focus_layout(int64_t n_nt, int32_t W, int32_t n_windows, const int32_t* d_k,
+                          uint32_t flags, int32_t B, const uint8_t* d_nt,
+                          const focus_layout_out* out, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------ */
+/* Compressed KV cache (caller-owned). App. A.2 "Streaming with controlled   */
+/* memory": a per-(sequence, head) contiguous ring of retained FOCUS K/V     */
+/* plus the current window's K/V buffer.                                   */
+/* ------------------------------------------------------------------------ */
+typedef struct focus_cache {
+    void*    ring_k;          /* device bf16 [B][H][C_ring][d] retained FOCUS keys */
+    void*    ring_v;          /* device bf16 [B][H][C_ring][d] retained FOCUS values */
+    void*    win_k;           /* device bf16 [B][H][C_win][d] current-window keys (decode) */
+    void*    win_v;           /* device bf16 [B][H][C_win][d] current-window values (decode) */
+    int32_t* ring_len;        /* device [B] retained rows R_b */
+    int32_t* win_fill;        /* device [B] rows in the current window buffer */
+    int32_t* win_idx;         /* device [B] index of the current window (selects k_w) */
+    const int32_t* k_per_window; /* device [n_windows] cadence schedule */
+    int32_t  n_windows;
+    int32_t  W;               /* window length in bases */
+    int32_t  B, H, d;
+    int32_t  C_ring, C_win;   /* capacities in rows */
+} focus_cache;
+
+/* ------------------------------------------------------------------------ */
+/* focus_attn_prefill — windowed attention over the compressed context      */
+/* Eq. focus-attn with visible set I_w-past ∪ retained FOCUS KV; App. A.1    */
+/* "Cross-window consistency" (sequential or masked-parallel); App. A.2.    */
+/* ------------------------------------------------------------------------ */
+typedef struct focus_prefill_args {
+    const void* q;            /* device bf16 [B][H][T_span][d] rows of windows [w_begin, w_end) */
+    const void* k;            /* device bf16 [B][H][T_span][d] */
+    const void* v;            /* device bf16 [B][H][T_span][d] */
+    void*       o;            /* device bf16 [B][H][T_span][d] output */
+    float*      lse;          /* device fp32 [B][H][T_span] natural-log sum-exp of scaled scores; may be NULL */
+    int64_t     T_span;       /* = win_off[w_end] - win_off[w_begin] */
+    const int32_t* d_win_off; /* device [M+1] from focus_layout */
+    const int32_t* d_ring_off;/* device [M+1] from focus_layout */
+    int32_t     n_windows;    /* M (the offsets arrays hold M+1 entries) */
+    int32_t     w_begin, w_end;   /* 0 <= w_begin < w_end <= M */
+    int32_t     max_rows;     /* >= every window's augmented row count in the span */
+    float       scale;        /* softmax scale, usually 1/sqrt(d) */
+    uint32_t    flags;        /* FOCUS_PREFILL_* */
+} focus_prefill_args;
+
+/* Use the legacy mma.sync kernel instead of the tcgen05/TMEM kernel (kept as the
+ * comparison baseline; same results within rounding). */
+#define FOCUS_PREFILL_LEGACY_MMA 1u
+
+/* Row a of window w (a = in-window augmented offset) gets
+ *   o = softmax_j(scale * q·k_j) v_j over j ∈ ring[0, ring_off[w]) ∪ window rows [0, a]
+ * and lse = ln Σ_j exp(scale * q·k_j). The ring rows are cache->ring_k/ring_v of the
+ * same (b, h); ring_off[w] <= C_ring is required for every window of the span.
+ * Masked-parallel use: bulk-compact all summaries first, then one call over all
+ * windows. Streaming use: one call per window, then compact that window. */
+focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_args* args,
+                                cudaStream_t stream);
+
+/* ------------------------------------------------------------------------ */
+/* focus_attn_decode — one new token per sequence against the compressed    */
+/* cache (App. A.2; the decode interface "identical to the base decoder").  */
+/* ------------------------------------------------------------------------ */
+
+/* Bytes of device workspace focus_attn_decode needs for this cache shape. */
+size_t focus_decode_workspace_size(const focus_cache* cache);
+
+/* For each (b, h): append k_new/v_new at window row win_fill[b], then
+ *   o = softmax over ring[0, ring_len[b]) ∪ window[0, win_fill[b]] (itself included),
+ * and increment win_fill[b]. q/k_new/v_new/o: device bf16 [B][H][d]; lse: device fp32
+ * [B][H] or NULL. workspace: device, >= focus_decode_workspace_size(cache) bytes,
+ * 16-byte aligned; its contents need no initialisation and are scratch afterwards.
+ * If the window buffer of sequence b is already full (win_fill[b] == that window's
+ * augmented size, or == C_win) the sequence is skipped and the status word is set to
+ * FOCUS_ERR_CAPACITY: call focus_kv_compact between steps. */
+focus_status focus_attn_decode(const focus_cache* cache, const void* q, const void* k_new,
+                               const void* v_new, float scale, void* o, float* lse,
+                               void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------ */
+/* focus_kv_compact — KV retention after a window (App. A, "KV compression  */
+/* and budget"; Sec. 3.2 "KV retention and memory profile").               */
+/* ------------------------------------------------------------------------ */
+typedef struct focus_compact_args {
+    /* Bulk mode (src_k != NULL): gather the FOCUS rows of windows [w_begin, w_end)
+     * from an augmented K/V tensor into ring rows [ring_off[w_begin], ring_off[w_end])
+     * of every (b, h), then set ring_len[b] = ring_off[w_end] for all b. */
+    const void* src_k;        /* device bf16 [B][H][src_T][d]; NULL selects window mode */
+    const void* src_v;        /* device bf16 [B][H][src_T][d] */
+    int64_t     src_T;        /* rows per (b, h) in src */
+    int64_t     src_row0;     /* augmented index of src row 0 (e.g. win_off[w_begin]) */
+    const int32_t* d_sum_idx; /* device [R] from focus_layout */
+    const int32_t* d_ring_off;/* device [M+1] from focus_layout */
+    int32_t     n_windows;    /* M (the offsets arrays hold M+1 entries) */
+    int32_t     w_begin, w_end;   /* 0 <= w_begin <= w_end <= M */
+    /* Window mode (src_k == NULL): for each sequence b whose window buffer is full
+     * (win_fill[b] == W + ceil(W / k_{win_idx[b]})), append that window's FOCUS rows
+     * to the ring at ring_len[b], advance ring_len[b], reset win_fill[b] to 0 and
+     * increment win_idx[b]. Sequences with a partly filled window are untouched. */
+} focus_compact_args;
+
+focus_status focus_kv_compact(const focus_cache* cache, const focus_compact_args* args,
+                              cudaStream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FOCUS_H_ */

@@ -1,0 +1,181 @@
+// C ABI of libfocus.so (declared in include/focus.h): host-side argument
+// checks, the per-device sticky status word, and dispatch to the kernels.
+#include <math.h>
+#include <mutex>
+
+#include "common.cuh"
+
+namespace {
+
+// Sticky status word written by kernels (first error wins). One copy per device
+// that loads the library; its device address is looked up once per device.
+__device__ int32_t g_focus_status;
+
+constexpr int kMaxDevices = 64;
+int32_t* g_status_ptr[kMaxDevices];
+std::mutex g_status_mu;
+
+focus_status status_ptr(int32_t** out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return FOCUS_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(g_status_mu);
+    if (!g_status_ptr[dev]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_focus_status) != cudaSuccess) return FOCUS_ERR_CUDA;
+        g_status_ptr[dev] = static_cast<int32_t*>(p);
+    }
+    *out = g_status_ptr[dev];
+    return FOCUS_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+focus_status from_cuda(cudaError_t e) { return e == cudaSuccess ? FOCUS_OK : FOCUS_ERR_CUDA; }
+
+focus_status check_cache(const focus_cache* c, bool need_window) {
+    if (!c) return FOCUS_ERR_INVALID_ARG;
+    if (c->B <= 0 || c->H <= 0 || c->C_ring < 0 || c->C_win < 0) return FOCUS_ERR_INVALID_ARG;
+    if (c->d != 64 && c->d != 128) return FOCUS_ERR_UNSUPPORTED;
+    if ((int64_t)c->B > 65535 || (int64_t)c->H > 65535) return FOCUS_ERR_UNSUPPORTED;
+    if (c->C_ring > 0 && (!c->ring_k || !c->ring_v)) return FOCUS_ERR_INVALID_ARG;
+    if (c->ring_k && (!aligned16(c->ring_k) || !aligned16(c->ring_v))) return FOCUS_ERR_UNSUPPORTED;
+    if (need_window) {
+        if (!c->win_k || !c->win_v || !c->ring_len || !c->win_fill || !c->win_idx || !c->k_per_window)
+            return FOCUS_ERR_INVALID_ARG;
+        if (c->W <= 0 || c->n_windows <= 0 || c->C_win <= 0) return FOCUS_ERR_INVALID_ARG;
+        if (!aligned16(c->win_k) || !aligned16(c->win_v)) return FOCUS_ERR_UNSUPPORTED;
+    }
+    return FOCUS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t focus_version(void) { return 100; }
+
+const char* focus_status_string(focus_status s) {
+    switch (s) {
+        case FOCUS_OK: return "ok";
+        case FOCUS_ERR_INVALID_ARG: return "invalid argument";
+        case FOCUS_ERR_UNSUPPORTED: return "unsupported shape, dtype or alignment";
+        case FOCUS_ERR_CAPACITY: return "ring or window buffer capacity exceeded";
+        case FOCUS_ERR_CUDA: return "CUDA error";
+        case FOCUS_ERR_TIMEOUT: return "bounded device wait timed out";
+        case FOCUS_ERR_LAYOUT: return "device layout disagrees with the given sizes";
+    }
+    return "unknown status";
+}
+
+focus_status focus_get_device_status(int32_t* host_status, int32_t clear, cudaStream_t stream) {
+    if (!host_status) return FOCUS_ERR_INVALID_ARG;
+    int32_t* p = nullptr;
+    focus_status st = status_ptr(&p);
+    if (st != FOCUS_OK) return st;
+    if (cudaStreamSynchronize(stream) != cudaSuccess) return FOCUS_ERR_CUDA;
+    if (cudaMemcpy(host_status, p, sizeof(int32_t), cudaMemcpyDeviceToHost) != cudaSuccess) return FOCUS_ERR_CUDA;
+    if (clear) {
+        if (cudaMemsetAsync(p, 0, sizeof(int32_t), stream) != cudaSuccess) return FOCUS_ERR_CUDA;
+        if (cudaStreamSynchronize(stream) != cudaSuccess) return FOCUS_ERR_CUDA;
+    }
+    return FOCUS_OK;
+}
+
+focus_status focus_layout_size(int64_t n_nt, int32_t W, int32_t n_windows, const int32_t* h_k, uint32_t flags,
+                               int64_t* T, int64_t* R, int32_t* max_rows) {
+    if (n_nt < 0 || W <= 0 || (n_nt > 0 && !h_k)) return FOCUS_ERR_INVALID_ARG;
+    if ((int64_t)n_windows != focus::ceil_div64(n_nt, W)) return FOCUS_ERR_INVALID_ARG;
+    const bool close_tail = (flags & FOCUS_LAYOUT_CLOSE_TAIL) != 0;
+    int64_t t = 0, r = 0, mx = 0;
+    for (int32_t w = 0; w < n_windows; ++w) {
+        if (h_k[w] < 0) return FOCUS_ERR_INVALID_ARG;
+        int64_t n = n_nt - (int64_t)w * W;
+        if (n > W) n = W;
+        const int64_t rows = focus::window_rows(n, h_k[w], (w < n_windows - 1) || close_tail);
+        t += rows;
+        r += rows - n;
+        if (rows > mx) mx = rows;
+    }
+    if (t > INT32_MAX) return FOCUS_ERR_UNSUPPORTED;   // offsets are int32
+    if (T) *T = t;
+    if (R) *R = r;
+    if (max_rows) *max_rows = (int32_t)mx;
+    return FOCUS_OK;
+}
+
+focus_status focus_layout(int64_t n_nt, int32_t W, int32_t n_windows, const int32_t* d_k, uint32_t flags,
+                          int32_t B, const uint8_t* d_nt, const focus_layout_out* out, cudaStream_t stream) {
+    if (!out || n_nt < 0 || W <= 0 || B < 0) return FOCUS_ERR_INVALID_ARG;
+    if ((int64_t)n_windows != focus::ceil_div64(n_nt, W) || n_windows <= 0 || !d_k) return FOCUS_ERR_INVALID_ARG;
+    if (out->T < 0 || out->R < 0 || out->T > INT32_MAX) return FOCUS_ERR_INVALID_ARG;
+    if (!out->win_off || !out->ring_off) return FOCUS_ERR_INVALID_ARG;
+    if (out->T > 0 && (!out->kind || !out->src || !out->pos || !out->win)) return FOCUS_ERR_INVALID_ARG;
+    if (out->R > 0 && !out->sum_idx) return FOCUS_ERR_INVALID_ARG;
+    if (out->tok && (!d_nt || B <= 0)) return FOCUS_ERR_INVALID_ARG;
+    int32_t* st = nullptr;
+    focus_status s = status_ptr(&st);
+    if (s != FOCUS_OK) return s;
+    return from_cuda(focus::launch_layout(n_nt, W, n_windows, d_k, (flags & FOCUS_LAYOUT_CLOSE_TAIL) != 0, B, d_nt,
+                                          *out, st, stream));
+}
+
+focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_args* a, cudaStream_t stream) {
+    focus_status s = check_cache(cache, false);
+    if (s != FOCUS_OK) return s;
+    if (!a || !a->q || !a->k || !a->v || !a->o || !a->d_win_off || !a->d_ring_off) return FOCUS_ERR_INVALID_ARG;
+    if (a->w_begin < 0 || a->w_end <= a->w_begin || a->w_end > a->n_windows || a->T_span < 0 || a->max_rows <= 0)
+        return FOCUS_ERR_INVALID_ARG;
+    if (!isfinite(a->scale)) return FOCUS_ERR_INVALID_ARG;
+    if (!aligned16(a->q) || !aligned16(a->k) || !aligned16(a->v) || !aligned16(a->o)) return FOCUS_ERR_UNSUPPORTED;
+    if (a->T_span == 0) return FOCUS_OK;
+    const int64_t tiles = focus::ceil_div64(a->max_rows, 64) * (int64_t)(a->w_end - a->w_begin);
+    if (tiles > INT32_MAX) return FOCUS_ERR_UNSUPPORTED;
+    int32_t* st = nullptr;
+    s = status_ptr(&st);
+    if (s != FOCUS_OK) return s;
+    return from_cuda(focus::launch_prefill_mma(*cache, *a, st, stream));
+}
+
+size_t focus_decode_workspace_size(const focus_cache* cache) {
+    if (check_cache(cache, false) != FOCUS_OK) return 0;
+    const int64_t ns = focus::decode_num_splits(*cache);
+    return (size_t)((int64_t)cache->B * cache->H * ns * (2 + cache->d)) * sizeof(float);
+}
+
+focus_status focus_attn_decode(const focus_cache* cache, const void* q, const void* k_new, const void* v_new,
+                               float scale, void* o, float* lse, void* workspace, size_t workspace_bytes,
+                               cudaStream_t stream) {
+    focus_status s = check_cache(cache, true);
+    if (s != FOCUS_OK) return s;
+    if (!q || !k_new || !v_new || !o || !workspace || !isfinite(scale)) return FOCUS_ERR_INVALID_ARG;
+    if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(o) || !aligned16(workspace))
+        return FOCUS_ERR_UNSUPPORTED;
+    if (workspace_bytes < focus_decode_workspace_size(cache)) return FOCUS_ERR_CAPACITY;
+    if (cache->C_ring > 0 && (!cache->ring_k || !cache->ring_v)) return FOCUS_ERR_INVALID_ARG;
+    int32_t* st = nullptr;
+    s = status_ptr(&st);
+    if (s != FOCUS_OK) return s;
+    return from_cuda(focus::launch_decode(*cache, q, k_new, v_new, scale, o, lse, workspace, st, stream));
+}
+
+focus_status focus_kv_compact(const focus_cache* cache, const focus_compact_args* a, cudaStream_t stream) {
+    if (!a) return FOCUS_ERR_INVALID_ARG;
+    const bool bulk = a->src_k != nullptr;
+    focus_status s = check_cache(cache, !bulk);
+    if (s != FOCUS_OK) return s;
+    if (!cache->ring_k || !cache->ring_v || !cache->ring_len) return FOCUS_ERR_INVALID_ARG;
+    int32_t* st = nullptr;
+    s = status_ptr(&st);
+    if (s != FOCUS_OK) return s;
+    if (bulk) {
+        if (!a->src_v || !a->d_sum_idx || !a->d_ring_off || a->src_T < 0 || a->w_begin < 0 || a->w_end < a->w_begin ||
+            a->w_end > a->n_windows)
+            return FOCUS_ERR_INVALID_ARG;
+        if (!aligned16(a->src_k) || !aligned16(a->src_v)) return FOCUS_ERR_UNSUPPORTED;
+        if (a->w_end == a->w_begin) return FOCUS_OK;
+        return from_cuda(focus::launch_compact_bulk(*cache, *a, st, stream));
+    }
+    return from_cuda(focus::launch_compact_window(*cache, st, stream));
+}
+
+}  // extern "C"

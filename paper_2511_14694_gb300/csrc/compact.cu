@@ -1,0 +1,111 @@
+// KV retention / compaction (App. A, "KV compression and budget"; Sec. 3.2
+// "KV retention and memory profile"): after a window, only the FOCUS rows' K/V
+// are kept, appended to the per-(sequence, head) ring. Ordinary rows are simply
+// not copied. Pure data movement, bit-exact; 16-byte vector loads and stores.
+#include "common.cuh"
+
+namespace focus {
+namespace {
+
+// Bulk mode: ring[b,h, r] <- src[b,h, sum_idx[r] - src_row0] for r in
+// [ring_off[w_begin], ring_off[w_end]). One thread moves one 16-byte chunk of
+// K and the same chunk of V; grid-stride over all chunks.
+__global__ void __launch_bounds__(256) compact_bulk_kernel(
+        uint4* __restrict__ ring_k, uint4* __restrict__ ring_v, const uint4* __restrict__ src_k,
+        const uint4* __restrict__ src_v, int32_t BH, int32_t B, int32_t chunks_per_row, int32_t C_ring,
+        int64_t src_T, int64_t src_row0, const int32_t* __restrict__ sum_idx,
+        const int32_t* __restrict__ ring_off, int32_t w_begin, int32_t w_end,
+        int32_t* __restrict__ ring_len, int32_t* status) {
+    const int32_t r0 = ring_off[w_begin], r1 = ring_off[w_end];
+    const int64_t rows = r1 - r0;
+    if (r1 > C_ring) {
+        if (blockIdx.x == 0 && threadIdx.x == 0) report(status, FOCUS_ERR_CAPACITY);
+        return;
+    }
+    const int64_t total = (int64_t)BH * rows * chunks_per_row;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int32_t c = (int32_t)(i % chunks_per_row);
+        const int64_t rest = i / chunks_per_row;
+        const int64_t r = r0 + rest % rows;
+        const int64_t bh = rest / rows;
+        const int64_t srow = (int64_t)sum_idx[r] - src_row0;
+        if (srow < 0 || srow >= src_T) {
+            report(status, FOCUS_ERR_INVALID_ARG);
+            continue;
+        }
+        const int64_t so = (bh * src_T + srow) * chunks_per_row + c;
+        const int64_t d_o = (bh * C_ring + r) * chunks_per_row + c;
+        ring_k[d_o] = src_k[so];
+        ring_v[d_o] = src_v[so];
+    }
+    if (blockIdx.x == 0)
+        for (int32_t b = threadIdx.x; b < B; b += blockDim.x) ring_len[b] = r1;
+}
+
+// Window mode: one CTA per sequence. If the current window buffer holds the
+// whole window (W bases + its summaries), append its FOCUS rows to the ring and
+// start the next window.
+__global__ void __launch_bounds__(256) compact_window_kernel(
+        uint4* __restrict__ ring_k, uint4* __restrict__ ring_v, const uint4* __restrict__ win_k,
+        const uint4* __restrict__ win_v, int32_t* __restrict__ ring_len, int32_t* __restrict__ win_fill,
+        int32_t* __restrict__ win_idx, const int32_t* __restrict__ ks, int32_t n_windows, int32_t W,
+        int32_t H, int32_t chunks_per_row, int32_t C_ring, int32_t C_win, int32_t* status) {
+    const int32_t b = blockIdx.x;
+    const int32_t fill = win_fill[b], widx = win_idx[b], R = ring_len[b];
+    if (widx < 0 || widx >= n_windows) {
+        if (threadIdx.x == 0) report(status, FOCUS_ERR_CAPACITY);
+        return;
+    }
+    const int32_t k = ks[widx];
+    const int32_t Tw = (int32_t)window_rows(W, k, true);
+    if (fill != Tw) return;                  // window not complete yet
+    const int32_t Bw = Tw - W;
+    if (R + Bw > C_ring || Tw > C_win) {
+        if (threadIdx.x == 0) report(status, FOCUS_ERR_CAPACITY);
+        return;
+    }
+    const int64_t total = (int64_t)H * Bw * chunks_per_row;
+    for (int64_t i = threadIdx.x; i < total; i += blockDim.x) {
+        const int32_t c = (int32_t)(i % chunks_per_row);
+        const int64_t rest = i / chunks_per_row;
+        const int32_t j = (int32_t)(rest % Bw);
+        const int64_t h = rest / Bw;
+        const int64_t bh = (int64_t)b * H + h;
+        const int32_t row = window_summary_row(j, W, k);
+        const int64_t so = (bh * C_win + row) * chunks_per_row + c;
+        const int64_t d_o = (bh * C_ring + R + j) * chunks_per_row + c;
+        ring_k[d_o] = win_k[so];
+        ring_v[d_o] = win_v[so];
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        ring_len[b] = R + Bw;
+        win_fill[b] = 0;
+        win_idx[b] = widx + 1;
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_compact_bulk(const focus_cache& c, const focus_compact_args& a, int32_t* status,
+                                cudaStream_t stream) {
+    int dev = 0, sms = 152;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int32_t cpr = c.d / 8;
+    compact_bulk_kernel<<<sms * 4, 256, 0, stream>>>(
+        (uint4*)c.ring_k, (uint4*)c.ring_v, (const uint4*)a.src_k, (const uint4*)a.src_v, c.B * c.H, c.B,
+        cpr, c.C_ring, a.src_T, a.src_row0, a.d_sum_idx, a.d_ring_off, a.w_begin, a.w_end, c.ring_len,
+        status);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_compact_window(const focus_cache& c, int32_t* status, cudaStream_t stream) {
+    compact_window_kernel<<<c.B, 256, 0, stream>>>(
+        (uint4*)c.ring_k, (uint4*)c.ring_v, (const uint4*)c.win_k, (const uint4*)c.win_v, c.ring_len,
+        c.win_fill, c.win_idx, c.k_per_window, c.n_windows, c.W, c.H, c.d / 8, c.C_ring, c.C_win, status);
+    return cudaGetLastError();
+}
+
+}  // namespace focus

@@ -1,0 +1,240 @@
+// Single-token decode against the compressed KV cache (App. A.2, streaming
+// inference: the retained FOCUS K/V of earlier windows are the history, the
+// current window's rows are attended causally; the new row sees itself).
+//
+// HBM-bound: every K/V row of the ring and of the window buffer is read once.
+// Split-K over keys: grid (split, head, sequence); each CTA streams a chunk of
+// keys with 16-byte loads (d/8 lanes per key row, several rows in flight per
+// thread), keeps a per-lane-group online softmax in registers, merges the
+// groups through shared memory and writes one partial (m, l, o) per split. A
+// second small kernel merges the splits with their log-sum-exp weights and
+// advances win_fill.
+#include "common.cuh"
+
+namespace focus {
+namespace {
+
+constexpr int kDecodeChunk = 1024;   // keys per split
+constexpr int kDecodeThreads = 128;
+constexpr int kUnroll = 8;           // key rows in flight per lane group
+
+__device__ __forceinline__ void bf16x8_to_f32(const uint4& u, float* f) {
+    const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        float2 x = __bfloat1622float2(p[i]);
+        f[2 * i] = x.x;
+        f[2 * i + 1] = x.y;
+    }
+}
+
+__device__ __forceinline__ bool decode_state_ok(int32_t R, int32_t fill, int32_t widx, const int32_t* ks,
+                                                int32_t n_windows, int32_t W, int32_t C_ring, int32_t C_win,
+                                                int32_t* Tw_out) {
+    if (widx < 0 || widx >= n_windows || R < 0 || R > C_ring) return false;
+    const int32_t Tw = (int32_t)window_rows(W, ks[widx], true);
+    *Tw_out = Tw;
+    return fill >= 0 && fill < Tw && fill < C_win;
+}
+
+template <int D>
+__global__ void __launch_bounds__(kDecodeThreads) decode_split_kernel(
+        const uint4* __restrict__ ring_k, const uint4* __restrict__ ring_v, uint4* __restrict__ win_k,
+        uint4* __restrict__ win_v, const int32_t* __restrict__ ring_len, const int32_t* __restrict__ win_fill,
+        const int32_t* __restrict__ win_idx, const int32_t* __restrict__ ks, int32_t n_windows, int32_t W,
+        int32_t H, int32_t C_ring, int32_t C_win, const uint4* __restrict__ q, const uint4* __restrict__ k_new,
+        const uint4* __restrict__ v_new, float scale_log2, float2* __restrict__ ws_ml, float* __restrict__ ws_o,
+        int32_t n_splits, int32_t* status) {
+    constexpr int CPR = D / 8;          // 16-byte chunks per row = lanes per key
+    constexpr int GPW = 32 / CPR;       // key groups per warp
+    constexpr int NG = (kDecodeThreads / 32) * GPW;
+    const int b = blockIdx.z, h = blockIdx.y, split = blockIdx.x;
+    const int64_t bh = (int64_t)b * H + h;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int sub = lane % CPR;
+    const int grp_in_warp = lane / CPR;
+
+    const int32_t R = ring_len[b], fill = win_fill[b], widx = win_idx[b];
+    int32_t Tw = 0;
+    float2* ml = ws_ml + bh * n_splits + split;
+    float* wo = ws_o + (bh * n_splits + split) * D;
+    if (!decode_state_ok(R, fill, widx, ks, n_windows, W, C_ring, C_win, &Tw)) {
+        if (split == 0 && h == 0 && tid == 0) report(status, FOCUS_ERR_CAPACITY);
+        for (int c = tid; c < D; c += blockDim.x) wo[c] = 0.f;
+        if (tid == 0) *ml = make_float2(-INFINITY, 0.f);
+        return;
+    }
+    const int64_t total = (int64_t)R + fill + 1;
+    const int64_t s0 = (int64_t)split * kDecodeChunk;
+    const int64_t s1 = min(total, s0 + kDecodeChunk);
+
+    if (split == 0 && tid < CPR) {      // append the new row to the window buffer
+        win_k[(bh * C_win + fill) * CPR + tid] = k_new[bh * CPR + tid];
+        win_v[(bh * C_win + fill) * CPR + tid] = v_new[bh * CPR + tid];
+    }
+
+    float qf[8];
+    bf16x8_to_f32(q[bh * CPR + sub], qf);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) qf[e] *= scale_log2;
+
+    float m = -INFINITY, l = 0.f, acc[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) acc[e] = 0.f;
+
+    const uint4* rk = ring_k + bh * (int64_t)C_ring * CPR + sub;
+    const uint4* rv = ring_v + bh * (int64_t)C_ring * CPR + sub;
+    const uint4* wk = win_k + bh * (int64_t)C_win * CPR + sub;
+    const uint4* wv = win_v + bh * (int64_t)C_win * CPR + sub;
+    const uint4* nk = k_new + bh * CPR + sub;
+    const uint4* nv = v_new + bh * CPR + sub;
+
+    // Warp-uniform loop: every lane runs the same trip count so the shuffles
+    // below always have the full warp.
+    for (int64_t wbase = s0 + warp * GPW; wbase < s1; wbase += (int64_t)NG * kUnroll) {
+        uint4 kr[kUnroll], vr[kUnroll];
+        float s[kUnroll];
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            const int64_t j = wbase + grp_in_warp + (int64_t)u * NG;
+            if (j < s1) {
+                const uint4 *kp, *vp;
+                if (j < R) { kp = rk + j * CPR; vp = rv + j * CPR; }
+                else if (j < (int64_t)R + fill) { kp = wk + (j - R) * CPR; vp = wv + (j - R) * CPR; }
+                else { kp = nk; vp = nv; }
+                kr[u] = __ldg(kp);
+                vr[u] = __ldg(vp);
+            } else {
+                kr[u] = make_uint4(0, 0, 0, 0);
+                vr[u] = make_uint4(0, 0, 0, 0);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            float kf[8];
+            bf16x8_to_f32(kr[u], kf);
+            float d0 = 0.f;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) d0 = fmaf(qf[e], kf[e], d0);
+            s[u] = d0;
+        }
+#pragma unroll
+        for (int off = CPR / 2; off >= 1; off >>= 1) {
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) s[u] += __shfl_xor_sync(0xffffffffu, s[u], off);
+        }
+        float mb = -INFINITY;
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            const int64_t j = wbase + grp_in_warp + (int64_t)u * NG;
+            if (j >= s1) s[u] = -INFINITY;
+            mb = fmaxf(mb, s[u]);
+        }
+        const float mn = fmaxf(m, mb);
+        if (mn == -INFINITY) continue;
+        const float corr = exp2f(m - mn);
+        l *= corr;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[e] *= corr;
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            const float p = exp2f(s[u] - mn);
+            l += p;
+            float vf[8];
+            bf16x8_to_f32(vr[u], vf);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) acc[e] = fmaf(p, vf[e], acc[e]);
+        }
+        m = mn;
+    }
+
+    __shared__ float sm_m[NG], sm_l[NG];
+    __shared__ float sm_acc[NG][D];
+    const int grp = warp * GPW + grp_in_warp;
+    if (sub == 0) { sm_m[grp] = m; sm_l[grp] = l; }
+#pragma unroll
+    for (int e = 0; e < 8; ++e) sm_acc[grp][sub * 8 + e] = acc[e];
+    __syncthreads();
+    if (tid < D) {
+        float M = -INFINITY;
+#pragma unroll
+        for (int g = 0; g < NG; ++g) M = fmaxf(M, sm_m[g]);
+        float L = 0.f, A = 0.f;
+        if (M != -INFINITY) {
+#pragma unroll
+            for (int g = 0; g < NG; ++g) {
+                const float f = exp2f(sm_m[g] - M);
+                L = fmaf(sm_l[g], f, L);
+                A = fmaf(sm_acc[g][tid], f, A);
+            }
+        }
+        wo[tid] = A;
+        if (tid == 0) *ml = make_float2(M, L);
+    }
+}
+
+template <int D>
+__global__ void __launch_bounds__(D) decode_combine_kernel(
+        const float2* __restrict__ ws_ml, const float* __restrict__ ws_o, int32_t n_splits, int32_t H,
+        __nv_bfloat16* __restrict__ o, float* __restrict__ lse, int32_t* __restrict__ win_fill,
+        const int32_t* __restrict__ ring_len, const int32_t* __restrict__ win_idx, const int32_t* __restrict__ ks,
+        int32_t n_windows, int32_t W, int32_t C_ring, int32_t C_win) {
+    const int b = blockIdx.y, h = blockIdx.x, c = threadIdx.x;
+    const int64_t bh = (int64_t)b * H + h;
+    const float2* ml = ws_ml + bh * n_splits;
+    const float* wo = ws_o + bh * n_splits * D;
+    float M = -INFINITY;
+    for (int s = 0; s < n_splits; ++s) M = fmaxf(M, ml[s].x);
+    float L = 0.f, A = 0.f;
+    if (M != -INFINITY) {
+        for (int s = 0; s < n_splits; ++s) {
+            const float2 x = ml[s];
+            if (x.x == -INFINITY) continue;
+            const float f = exp2f(x.x - M);
+            L = fmaf(x.y, f, L);
+            A = fmaf(wo[(int64_t)s * D + c], f, A);
+        }
+    }
+    o[bh * D + c] = __float2bfloat16_rn(L > 0.f ? A / L : 0.f);
+    if (c == 0 && lse) lse[bh] = L > 0.f ? (M + log2f(L)) * 0.69314718055994531f : -INFINITY;
+    if (h == 0 && c == 0) {
+        int32_t Tw = 0;
+        if (decode_state_ok(ring_len[b], win_fill[b], win_idx[b], ks, n_windows, W, C_ring, C_win, &Tw))
+            win_fill[b] += 1;
+    }
+}
+
+template <int D>
+cudaError_t launch_decode_d(const focus_cache& c, const void* q, const void* k_new, const void* v_new,
+                            float scale, void* o, float* lse, void* workspace, int32_t* status,
+                            cudaStream_t stream) {
+    const int32_t ns = decode_num_splits(c);
+    float2* ws_ml = reinterpret_cast<float2*>(workspace);
+    float* ws_o = reinterpret_cast<float*>(ws_ml + (int64_t)c.B * c.H * ns);
+    dim3 grid(ns, c.H, c.B);
+    decode_split_kernel<D><<<grid, kDecodeThreads, 0, stream>>>(
+        (const uint4*)c.ring_k, (const uint4*)c.ring_v, (uint4*)c.win_k, (uint4*)c.win_v, c.ring_len,
+        c.win_fill, c.win_idx, c.k_per_window, c.n_windows, c.W, c.H, c.C_ring, c.C_win, (const uint4*)q,
+        (const uint4*)k_new, (const uint4*)v_new, scale * 1.4426950408889634f, ws_ml, ws_o, ns, status);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    decode_combine_kernel<D><<<dim3(c.H, c.B), D, 0, stream>>>(
+        ws_ml, ws_o, ns, c.H, (__nv_bfloat16*)o, lse, c.win_fill, c.ring_len, c.win_idx, c.k_per_window,
+        c.n_windows, c.W, c.C_ring, c.C_win);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+int32_t decode_num_splits(const focus_cache& c) {
+    return (int32_t)ceil_div64((int64_t)c.C_ring + c.C_win, kDecodeChunk);
+}
+
+cudaError_t launch_decode(const focus_cache& c, const void* q, const void* k_new, const void* v_new,
+                          float scale, void* o, float* lse, void* workspace, int32_t* status,
+                          cudaStream_t stream) {
+    if (c.d == 128) return launch_decode_d<128>(c, q, k_new, v_new, scale, o, lse, workspace, status, stream);
+    return launch_decode_d<64>(c, q, k_new, v_new, scale, o, lse, workspace, status, stream);
+}
+
+}  // namespace focus

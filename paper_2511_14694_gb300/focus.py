@@ -1,0 +1,276 @@
+"""Thin ctypes binding of libfocus.so (C ABI in include/focus.h).
+
+Argument marshalling only: torch tensors are passed as raw device pointers and
+the current torch stream as a cudaStream_t; every step of the compute path
+runs in the library's CUDA kernels. There is no CPU fallback: if the library
+cannot be loaded, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+
+import numpy as np
+import torch
+
+from . import _build
+
+FOCUS_OK = 0
+STATUS_NAMES = {0: "ok", 1: "invalid argument", 2: "unsupported", 3: "capacity", 4: "cuda", 5: "timeout",
+                6: "layout"}
+LAYOUT_CLOSE_TAIL = 1
+PREFILL_LEGACY_MMA = 1
+SUMMARY_TOKEN = 4
+
+
+class FocusError(RuntimeError):
+    def __init__(self, fn: str, code: int):
+        super().__init__(f"{fn} failed: {STATUS_NAMES.get(code, code)} ({code})")
+        self.code = code
+
+
+_P = ctypes.c_void_p
+_i32, _i64, _u32, _f32 = ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32, ctypes.c_float
+
+
+class LayoutOut(ctypes.Structure):
+    _fields_ = [("T", _i64), ("R", _i64), ("kind", _P), ("src", _P), ("pos", _P), ("win", _P), ("tok", _P),
+                ("win_off", _P), ("ring_off", _P), ("sum_idx", _P)]
+
+
+class CacheDesc(ctypes.Structure):
+    _fields_ = [("ring_k", _P), ("ring_v", _P), ("win_k", _P), ("win_v", _P), ("ring_len", _P),
+                ("win_fill", _P), ("win_idx", _P), ("k_per_window", _P), ("n_windows", _i32), ("W", _i32),
+                ("B", _i32), ("H", _i32), ("d", _i32), ("C_ring", _i32), ("C_win", _i32)]
+
+
+class PrefillArgs(ctypes.Structure):
+    _fields_ = [("q", _P), ("k", _P), ("v", _P), ("o", _P), ("lse", _P), ("T_span", _i64), ("d_win_off", _P),
+                ("d_ring_off", _P), ("n_windows", _i32), ("w_begin", _i32), ("w_end", _i32), ("max_rows", _i32),
+                ("scale", _f32),
+                ("flags", _u32)]
+
+
+class CompactArgs(ctypes.Structure):
+    _fields_ = [("src_k", _P), ("src_v", _P), ("src_T", _i64), ("src_row0", _i64), ("d_sum_idx", _P),
+                ("d_ring_off", _P), ("n_windows", _i32), ("w_begin", _i32), ("w_end", _i32)]
+
+
+_lib = None
+
+
+def lib_path() -> str:
+    return _build.LIB
+
+
+def load() -> ctypes.CDLL:
+    """Load libfocus.so (building it first if it is missing or stale)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if _build.is_stale():
+        _build.build()
+    lib = ctypes.CDLL(_build.LIB)
+    lib.focus_version.restype = _i32
+    lib.focus_status_string.restype = ctypes.c_char_p
+    lib.focus_status_string.argtypes = [ctypes.c_int]
+    lib.focus_get_device_status.restype = ctypes.c_int
+    lib.focus_get_device_status.argtypes = [_P, _i32, _P]
+    lib.focus_layout_size.restype = ctypes.c_int
+    lib.focus_layout_size.argtypes = [_i64, _i32, _i32, _P, _u32, _P, _P, _P]
+    lib.focus_layout.restype = ctypes.c_int
+    lib.focus_layout.argtypes = [_i64, _i32, _i32, _P, _u32, _i32, _P, ctypes.POINTER(LayoutOut), _P]
+    lib.focus_attn_prefill.restype = ctypes.c_int
+    lib.focus_attn_prefill.argtypes = [ctypes.POINTER(CacheDesc), ctypes.POINTER(PrefillArgs), _P]
+    lib.focus_decode_workspace_size.restype = ctypes.c_size_t
+    lib.focus_decode_workspace_size.argtypes = [ctypes.POINTER(CacheDesc)]
+    lib.focus_attn_decode.restype = ctypes.c_int
+    lib.focus_attn_decode.argtypes = [ctypes.POINTER(CacheDesc), _P, _P, _P, _f32, _P, _P, _P, ctypes.c_size_t, _P]
+    lib.focus_kv_compact.restype = ctypes.c_int
+    lib.focus_kv_compact.argtypes = [ctypes.POINTER(CacheDesc), ctypes.POINTER(CompactArgs), _P]
+    _lib = lib
+    return lib
+
+
+def _check(fn: str, code: int):
+    if code != FOCUS_OK:
+        raise FocusError(fn, code)
+
+
+def _ptr(t) -> int | None:
+    if t is None:
+        return None
+    if isinstance(t, np.ndarray):
+        return t.ctypes.data
+    return t.data_ptr()
+
+
+def _stream(stream=None) -> int:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+def _cuda(t: torch.Tensor, name: str, dtype=None):
+    if not (isinstance(t, torch.Tensor) and t.is_cuda and t.is_contiguous()):
+        raise ValueError(f"{name} must be a contiguous CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    return t
+
+
+# ----------------------------------------------------------------------------- layout
+
+def layout_size(N: int, W: int, k_sched, close_tail: bool = True):
+    """(T, R, M, max_rows) of the augmented layout (host arithmetic in the library)."""
+    lib = load()
+    M = -(-N // W)
+    k = np.ascontiguousarray(np.broadcast_to(np.asarray(k_sched, dtype=np.int32), (M,)))
+    T, R, mx = _i64(), _i64(), _i32()
+    _check("focus_layout_size", lib.focus_layout_size(N, W, M, k.ctypes.data, LAYOUT_CLOSE_TAIL if close_tail else 0,
+                                                      ctypes.byref(T), ctypes.byref(R), ctypes.byref(mx)))
+    return T.value, R.value, M, mx.value
+
+
+def layout_alloc(N: int, W: int, k_sched, B: int = 0, close_tail: bool = True, device="cuda") -> dict:
+    """Allocate the device outputs of focus_layout (sizes from focus_layout_size)."""
+    T, R, M, mx = layout_size(N, W, k_sched, close_tail)
+    k_host = np.ascontiguousarray(np.broadcast_to(np.asarray(k_sched, dtype=np.int32), (M,)))
+    out = dict(
+        kind=torch.empty(T, dtype=torch.uint8, device=device), src=torch.empty(T, dtype=torch.int32, device=device),
+        pos=torch.empty(T, dtype=torch.int32, device=device), win=torch.empty(T, dtype=torch.int32, device=device),
+        tok=torch.empty((B, T), dtype=torch.uint8, device=device) if B else None,
+        win_off=torch.empty(M + 1, dtype=torch.int32, device=device),
+        ring_off=torch.empty(M + 1, dtype=torch.int32, device=device),
+        sum_idx_buf=torch.empty(max(R, 1), dtype=torch.int32, device=device),
+        k=torch.from_numpy(k_host.copy()).to(device))
+    out["sum_idx"] = out["sum_idx_buf"][:R]
+    out.update(T=T, R=R, M=M, max_rows=mx, k_host=k_host, N=N, W=W, B=B, close_tail=close_tail)
+    return out
+
+
+def layout_run(L: dict, nt: torch.Tensor | None = None, stream=None) -> None:
+    """Launch focus_layout into buffers from layout_alloc (asynchronous)."""
+    lib = load()
+    if nt is not None:
+        _cuda(nt, "nt", torch.uint8)
+        if L["tok"] is None or tuple(nt.shape) != (L["B"], L["N"]):
+            raise ValueError("nt shape does not match the allocated layout")
+    desc = LayoutOut(L["T"], L["R"], _ptr(L["kind"]), _ptr(L["src"]), _ptr(L["pos"]), _ptr(L["win"]),
+                     _ptr(L["tok"]) if nt is not None else None, _ptr(L["win_off"]), _ptr(L["ring_off"]),
+                     _ptr(L["sum_idx_buf"]))
+    _check("focus_layout", lib.focus_layout(L["N"], L["W"], L["M"], _ptr(L["k"]),
+                                            LAYOUT_CLOSE_TAIL if L["close_tail"] else 0,
+                                            0 if nt is None else L["B"], _ptr(nt), ctypes.byref(desc),
+                                            _stream(stream)))
+
+
+def layout(N: int, W: int, k_sched, nt: torch.Tensor | None = None, close_tail: bool = True,
+           device="cuda", stream=None) -> dict:
+    """Build the augmented token layout on the device (focus_layout) and keep host
+    copies of the window/ring offsets for slicing per-window inputs (syncs)."""
+    L = layout_alloc(N, W, k_sched, 0 if nt is None else int(nt.shape[0]), close_tail, device)
+    layout_run(L, nt, stream)
+    L["win_off_host"] = L["win_off"].cpu().numpy()
+    L["ring_off_host"] = L["ring_off"].cpu().numpy()
+    return L
+
+
+# ----------------------------------------------------------------------------- cache
+
+class Cache:
+    """Caller-owned compressed KV cache (ring of retained FOCUS K/V + the
+    current window buffer) and its C descriptor."""
+
+    def __init__(self, B: int, H: int, d: int, C_ring: int, C_win: int = 0, W: int = 0, k_sched=None,
+                 device="cuda"):
+        self.B, self.H, self.d, self.C_ring, self.C_win, self.W = B, H, d, C_ring, C_win, W
+        bf = dict(dtype=torch.bfloat16, device=device)
+        self.ring_k = torch.zeros((B, H, max(C_ring, 1), d), **bf)
+        self.ring_v = torch.zeros((B, H, max(C_ring, 1), d), **bf)
+        self.win_k = torch.zeros((B, H, max(C_win, 1), d), **bf) if C_win else None
+        self.win_v = torch.zeros((B, H, max(C_win, 1), d), **bf) if C_win else None
+        self.ring_len = torch.zeros(B, dtype=torch.int32, device=device)
+        self.win_fill = torch.zeros(B, dtype=torch.int32, device=device)
+        self.win_idx = torch.zeros(B, dtype=torch.int32, device=device)
+        ks = np.zeros(1, np.int32) if k_sched is None else np.asarray(k_sched, dtype=np.int32).reshape(-1)
+        self.k_sched = torch.from_numpy(ks.copy()).to(device)
+        self.desc = CacheDesc(_ptr(self.ring_k), _ptr(self.ring_v), _ptr(self.win_k), _ptr(self.win_v),
+                              _ptr(self.ring_len), _ptr(self.win_fill), _ptr(self.win_idx), _ptr(self.k_sched),
+                              int(self.k_sched.numel()), W, B, H, d, C_ring, C_win)
+
+    def workspace_bytes(self) -> int:
+        return int(load().focus_decode_workspace_size(ctypes.byref(self.desc)))
+
+    def new_workspace(self) -> torch.Tensor:
+        n = self.workspace_bytes()
+        return torch.empty(max(n, 16) // 4 + 4, dtype=torch.float32, device=self.ring_k.device)
+
+
+# ----------------------------------------------------------------------------- verbs
+
+def attn_prefill(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | None = None, scale=None,
+                 o=None, lse=None, flags: int = 0, stream=None):
+    """focus_attn_prefill over windows [w_begin, w_end). q/k/v: bf16 [B, H, T_span, d]
+    holding the augmented rows of those windows. Returns (o, lse)."""
+    lib = load()
+    w_end = L["M"] if w_end is None else w_end
+    for name, t in (("q", q), ("k", k), ("v", v)):
+        _cuda(t, name, torch.bfloat16)
+    B, H, T_span, d = q.shape
+    if o is None:
+        o = torch.empty_like(q)
+    if lse is None:
+        lse = torch.empty((B, H, T_span), dtype=torch.float32, device=q.device)
+    scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
+    a = PrefillArgs(_ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse), T_span, _ptr(L["win_off"]), _ptr(L["ring_off"]),
+                    L["M"], w_begin, w_end, int(L["max_rows"]), scale, flags)
+    _check("focus_attn_prefill", lib.focus_attn_prefill(ctypes.byref(cache.desc), ctypes.byref(a), _stream(stream)))
+    return o, lse
+
+
+def kv_compact_bulk(cache: Cache, src_k, src_v, L: dict, w_begin: int = 0, w_end: int | None = None,
+                    src_row0: int = 0, stream=None):
+    """focus_kv_compact, bulk mode: gather the FOCUS rows of windows
+    [w_begin, w_end) of src into the ring."""
+    lib = load()
+    w_end = L["M"] if w_end is None else w_end
+    _cuda(src_k, "src_k", torch.bfloat16)
+    _cuda(src_v, "src_v", torch.bfloat16)
+    a = CompactArgs(_ptr(src_k), _ptr(src_v), int(src_k.shape[2]), int(src_row0), _ptr(L["sum_idx_buf"]),
+                    _ptr(L["ring_off"]), L["M"], w_begin, w_end)
+    _check("focus_kv_compact", lib.focus_kv_compact(ctypes.byref(cache.desc), ctypes.byref(a), _stream(stream)))
+
+
+def kv_compact_window(cache: Cache, stream=None):
+    """focus_kv_compact, window mode: retire every full window buffer."""
+    lib = load()
+    a = CompactArgs(None, None, 0, 0, None, None, 0, 0, 0)
+    _check("focus_kv_compact", lib.focus_kv_compact(ctypes.byref(cache.desc), ctypes.byref(a), _stream(stream)))
+
+
+def attn_decode(cache: Cache, q, k_new, v_new, scale=None, o=None, lse=None, workspace=None, stream=None):
+    """focus_attn_decode: one new token per sequence. q/k_new/v_new: bf16 [B, H, d]."""
+    lib = load()
+    for name, t in (("q", q), ("k_new", k_new), ("v_new", v_new)):
+        _cuda(t, name, torch.bfloat16)
+    if o is None:
+        o = torch.empty_like(q)
+    if lse is None:
+        lse = torch.empty(q.shape[:2], dtype=torch.float32, device=q.device)
+    if workspace is None:
+        workspace = cache.new_workspace()
+    scale = 1.0 / math.sqrt(q.shape[-1]) if scale is None else float(scale)
+    _check("focus_attn_decode",
+           lib.focus_attn_decode(ctypes.byref(cache.desc), _ptr(q), _ptr(k_new), _ptr(v_new), scale, _ptr(o),
+                                 _ptr(lse), _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                 _stream(stream)))
+    return o, lse
+
+
+def device_status(clear: bool = True, stream=None) -> int:
+    """Read (and by default clear) the sticky device status word; syncs the stream."""
+    lib = load()
+    v = _i32()
+    _check("focus_get_device_status", lib.focus_get_device_status(ctypes.byref(v), int(clear), _stream(stream)))
+    return v.value

@@ -1,0 +1,84 @@
+"""CPU checks of the C-ABI library: it builds, loads, exports every function
+include/focus.h declares, its struct layouts match the binding's, and its
+host-only logic (layout sizes, argument validation) is right. No kernel is
+launched here."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import focus_oracle as fo
+from paper_2511_14694_gb300 import focus, inputs
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "focus.h")
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?[A-Za-z_][A-Za-z0-9_]*\s*\*?\s*(focus_[a-z_0-9]+)\s*\(", src,
+                                 flags=re.M)))
+
+
+def test_library_exports_every_declared_function():
+    lib = focus.load()
+    names = declared_functions()
+    assert {"focus_layout", "focus_attn_prefill", "focus_attn_decode", "focus_kv_compact"} <= set(names)
+    for n in names:
+        assert hasattr(lib, n), f"{n} declared in focus.h but not exported"
+
+
+def test_struct_sizes_match_c_layout():
+    # 2 x int64 + 8 pointers; 8 pointers + 7 int32 (+pad); see focus.h
+    assert ctypes.sizeof(focus.LayoutOut) == 16 + 8 * 8
+    assert ctypes.sizeof(focus.CacheDesc) == 8 * 8 + 7 * 4 + 4
+    assert ctypes.sizeof(focus.PrefillArgs) == 5 * 8 + 8 + 2 * 8 + 6 * 4
+    assert ctypes.sizeof(focus.CompactArgs) == 2 * 8 + 2 * 8 + 2 * 8 + 3 * 4 + 4
+
+
+def test_version_and_status_strings():
+    lib = focus.load()
+    assert lib.focus_version() >= 100
+    for code in range(7):
+        assert lib.focus_status_string(code)
+
+
+@pytest.mark.parametrize("N,W,ks,close", [(4_000, 1_000, [100], True), (128_000, 1_000, [100], True),
+                                          (5_000, 1_024, [100], False), (10, 4, [3], True),
+                                          (256_000, 1_000, [10, 25, 50, 100, 200], True), (77, 100, [0], True)])
+def test_layout_size_matches_oracle(N, W, ks, close):
+    M = -(-N // W)
+    k = inputs.k_schedule(M, ks, seed=1)
+    T, R, M2, mx = focus.layout_size(N, W, k, close_tail=close)
+    To, Ro, Mo = fo.layout_size(N, W, k, close_tail=close)
+    assert (T, R, M2) == (To, Ro, Mo)
+    L = fo.layout(N, W, k, close_tail=close)
+    assert mx == int(np.diff(L["win_off"]).max())
+
+
+def test_host_validation_rejects_bad_arguments():
+    lib = focus.load()
+    T = ctypes.c_int64()
+    k = np.array([100], np.int32)
+    # wrong window count, negative N, missing schedule
+    assert lib.focus_layout_size(1000, 1000, 2, k.ctypes.data, 1, ctypes.byref(T), None, None) == 1
+    assert lib.focus_layout_size(-1, 1000, 0, k.ctypes.data, 1, ctypes.byref(T), None, None) == 1
+    assert lib.focus_layout_size(1000, 1000, 1, None, 1, ctypes.byref(T), None, None) == 1
+    assert lib.focus_layout_size(1000, 0, 1, k.ctypes.data, 1, ctypes.byref(T), None, None) == 1
+    neg = np.array([-3], np.int32)
+    assert lib.focus_layout_size(1000, 1000, 1, neg.ctypes.data, 1, ctypes.byref(T), None, None) == 1
+    # null descriptors
+    assert lib.focus_attn_prefill(None, None, None) == 1
+    assert lib.focus_kv_compact(None, None, None) == 1
+    assert lib.focus_attn_decode(None, None, None, None, 1.0, None, None, None, 0, None) == 1
+    # unsupported head dim is rejected before any CUDA call
+    c = focus.CacheDesc()
+    c.B, c.H, c.d, c.C_ring = 1, 1, 96, 0
+    a = focus.PrefillArgs()
+    assert lib.focus_attn_prefill(ctypes.byref(c), ctypes.byref(a), None) == 2
+    c.d = 128
+    # null q/k/v
+    assert lib.focus_attn_prefill(ctypes.byref(c), ctypes.byref(a), None) == 1
+    assert lib.focus_decode_workspace_size(None) == 0

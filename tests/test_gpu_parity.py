@@ -1,0 +1,313 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 oracle on the
+same seeded inputs.
+
+Bars: layout, position ids, gather indices and compaction are bit-exact.
+Attention output O: max-abs <= 2e-2 and mean-abs <= 2e-3, and (because the
+N(0,1)/sqrt(d) workloads give ~10x smaller outputs, where the absolute bars are
+loose) relative RMS error <= 1e-2. LSE: |error| <= 1e-3 * max(1, |LSE|).
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import focus_oracle as fo
+from paper_2511_14694_gb300 import focus, inputs, pipeline
+
+pytestmark = pytest.mark.gpu
+
+O_MAX_ABS, O_MEAN_ABS, O_REL_RMS, LSE_REL = 2e-2, 2e-3, 1e-2, 1e-3
+
+
+@pytest.fixture(autouse=True)
+def _clean_status():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    focus.device_status(clear=True)
+    yield
+    assert focus.device_status(clear=True) == 0, "a kernel reported an error"
+
+
+def assert_attn_close(o_gpu, lse_gpu, o_ref, lse_ref, what=""):
+    og = o_gpu.detach().float().cpu().double().numpy().reshape(o_ref.shape)
+    lg = lse_gpu.detach().cpu().double().numpy().reshape(lse_ref.shape)
+    assert np.isfinite(og).all() and np.isfinite(lg).all(), what
+    err = np.abs(og - o_ref)
+    rel_rms = math.sqrt(float((err ** 2).mean())) / max(math.sqrt(float((o_ref ** 2).mean())), 1e-30)
+    lerr = np.abs(lg - lse_ref) / np.maximum(1.0, np.abs(lse_ref))
+    msg = f"{what}: max {err.max():.3e} mean {err.mean():.3e} relrms {rel_rms:.3e} lse {lerr.max():.3e}"
+    assert err.max() <= O_MAX_ABS, msg
+    assert err.mean() <= O_MEAN_ABS, msg
+    assert rel_rms <= O_REL_RMS, msg
+    assert lerr.max() <= LSE_REL, msg
+
+
+def bits(t):
+    return t.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
+
+
+# ----------------------------------------------------------------------------- layout
+
+LAYOUT_CASES = [
+    (4_000, 1_000, [100], True), (128_000, 1_000, [100], True), (256_000, 1_000, [10, 25, 50, 100, 200], True),
+    (1_000_000, 1_000, [100], True), (10, 4, [3], True), (1, 1, [1], True), (500, 1_000, [0], True),
+    (77, 10, [20], True), (5_000, 1_024, [100], False), (5_000, 1_024, [100], True), (3_001, 3, [1, 2, 3, 4], False),
+    (2_048, 2_048, [1], True),
+]
+
+
+@pytest.mark.parametrize("N,W,ks,close", LAYOUT_CASES)
+def test_layout_bit_exact(N, W, ks, close):
+    M = -(-N // W)
+    k = inputs.k_schedule(M, ks, seed=N % 97)
+    nt = inputs.nucleotides(2, N, seed=5, device="cuda")
+    L = focus.layout(N, W, k, nt=nt, close_tail=close)
+    ref = fo.layout(N, W, k, nt=nt.cpu().numpy(), close_tail=close)
+    torch.cuda.synchronize()
+    assert (L["T"], L["R"], L["M"]) == (ref["T"], ref["R"], ref["M"])
+    for key in ("kind", "src", "pos", "win", "win_off", "ring_off", "sum_idx"):
+        assert np.array_equal(L[key].cpu().numpy(), ref[key]), key
+    assert np.array_equal(L["tok"].cpu().numpy(), ref["tok"])
+
+
+# ----------------------------------------------------------------------------- prefill, masked-parallel
+
+PREFILL_CASES = [
+    # N, W, k schedule, B, H, d, std
+    (4_000, 1_000, [100], 1, 4, 64, 1.0),            # 4 windows of 1 kb, k=100, the small parity workload
+    (1_000, 300, [7], 2, 2, 128, 1.0),
+    (777, 128, [1, 5, 50, 200], 1, 3, 64, 1.0),
+    (500, 1_000, [0], 1, 2, 128, 1.0),                # compression disabled: plain causal
+    (300, 64, [64], 1, 2, 64, 1.0),                   # T_w = 65: one row past a tile
+    (20_000, 200, [10], 1, 2, 128, 1.0 / math.sqrt(128)),   # ring of up to 990 rows
+    (3_333, 1_000, [3, 100, 1_000], 2, 1, 128, 1.0),  # ragged last window, k = W
+]
+
+
+def _masked_parallel(N, W, ks, B, H, d, std, seed=0, flags=0):
+    M = -(-N // W)
+    k = inputs.k_schedule(M, ks, seed=seed + 1)
+    L = focus.layout(N, W, k)
+    q, kk, v = inputs.qkv((B, H, L["T"], d), std=std, seed=seed + 2, device="cuda")
+    cache = focus.Cache(B, H, d, C_ring=max(L["R"], 1))
+    n = q.numel()
+    canary = torch.full((n + 4096,), 7.0, dtype=torch.bfloat16, device="cuda")
+    o = canary[:n].view(q.shape)
+    o, lse = pipeline.prefill_masked_parallel(cache, q, kk, v, L, o=o, flags=flags)
+    torch.cuda.synchronize()
+    assert bool((canary[n:] == 7.0).all()), "prefill wrote past its output"
+    return L, q, kk, v, cache, o, lse
+
+
+@pytest.mark.parametrize("N,W,ks,B,H,d,std", PREFILL_CASES)
+def test_prefill_masked_parallel_matches_oracle(N, W, ks, B, H, d, std):
+    L, q, k, v, cache, o, lse = _masked_parallel(N, W, ks, B, H, d, std, seed=N)
+    ref_L = fo.layout(N, W, L["k_host"])
+    T = L["T"]
+    heads = np.repeat(np.arange(B * H), T)
+    rows = np.tile(np.arange(T), B * H)
+    o_ref, lse_ref = fo.attn_rows(q.reshape(B * H, T, d).cpu(), k.reshape(B * H, T, d).cpu(),
+                                  v.reshape(B * H, T, d).cpu(), ref_L["kind"], ref_L["win"], 1.0 / math.sqrt(d),
+                                  heads, rows)
+    assert_attn_close(o, lse, o_ref.reshape(B, H, T, d), lse_ref.reshape(B, H, T), f"N={N} W={W} k={ks}")
+    # compaction: ring == the FOCUS rows, bit for bit
+    kb, vb = bits(k), bits(v)
+    assert np.array_equal(bits(cache.ring_k)[:, :, :L["R"]], kb[:, :, ref_L["sum_idx"]])
+    assert np.array_equal(bits(cache.ring_v)[:, :, :L["R"]], vb[:, :, ref_L["sum_idx"]])
+    assert (cache.ring_len.cpu().numpy() == L["R"]).all()
+
+
+def test_prefill_legacy_kernel_matches_oracle():
+    N, W, ks, B, H, d = 2_000, 500, [50], 1, 2, 128
+    L, q, k, v, cache, o, lse = _masked_parallel(N, W, ks, B, H, d, 1.0, seed=9, flags=focus.PREFILL_LEGACY_MMA)
+    ref_L = fo.layout(N, W, L["k_host"])
+    T = L["T"]
+    o_ref, lse_ref = fo.attn_rows(q.reshape(H, T, d).cpu(), k.reshape(H, T, d).cpu(), v.reshape(H, T, d).cpu(),
+                                  ref_L["kind"], ref_L["win"], 1.0 / math.sqrt(d), np.repeat(np.arange(H), T),
+                                  np.tile(np.arange(T), H))
+    assert_attn_close(o, lse, o_ref.reshape(B, H, T, d), lse_ref.reshape(B, H, T), "legacy")
+
+
+# ----------------------------------------------------------------------------- prefill, sequential / streaming
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_prefill_streaming_matches_sequential_oracle(d):
+    N, W, ks, B, H = 3_000, 500, [10, 50, 100, 7], 2, 2
+    M = -(-N // W)
+    k_s = inputs.k_schedule(M, ks, seed=4)
+    L = focus.layout(N, W, k_s)
+    q, k, v = inputs.qkv((B, H, L["T"], d), seed=21, device="cuda")
+    cache = focus.Cache(B, H, d, C_ring=L["R"])
+    o = torch.empty_like(q)
+    lse = torch.empty((B, H, L["T"]), dtype=torch.float32, device="cuda")
+    off = L["win_off_host"]
+    for w in range(M):
+        a, e = int(off[w]), int(off[w + 1])
+        sl = lambda t: t[:, :, a:e].contiguous()  # noqa: E731
+        ow, lw = pipeline.prefill_window(cache, sl(q), sl(k), sl(v), L, w)
+        o[:, :, a:e] = ow
+        lse[:, :, a:e] = lw
+    torch.cuda.synchronize()
+    ref_L = fo.layout(N, W, k_s)
+    for b in range(B):
+        for h in range(H):
+            o_ref, lse_ref, rk, rv = fo.prefill_sequential(q[b, h].cpu(), k[b, h].cpu(), v[b, h].cpu(),
+                                                           ref_L["win_off"], ref_L["kind"], 1.0 / math.sqrt(d))
+            assert_attn_close(o[b, h], lse[b, h], o_ref, lse_ref, f"stream b={b} h={h}")
+            assert np.array_equal(bits(cache.ring_k[b, h, :L["R"]]), rk)
+            assert np.array_equal(bits(cache.ring_v[b, h, :L["R"]]), rv)
+
+
+# ----------------------------------------------------------------------------- decode
+
+class DecodeModel:
+    """Host mirror of the decode cache evolved with the oracle's rules (App. A.2)."""
+
+    def __init__(self, ring_k, ring_v, R, win_k, win_v, fill, widx, W, k_sched):
+        self.rk, self.rv = bits(ring_k).copy(), bits(ring_v).copy()
+        self.wk, self.wv = bits(win_k).copy(), bits(win_v).copy()
+        self.R, self.fill, self.widx = R.copy(), fill.copy(), widx.copy()
+        self.W, self.k = W, np.asarray(k_sched)
+
+    def step(self, q, kn, vn, scale):
+        B, H, d = q.shape
+        qb, kb, vb = bits(q), bits(kn), bits(vn)
+        o = np.zeros((B, H, d))
+        lse = np.zeros((B, H))
+        for b in range(B):
+            oo, ll = fo.decode(qb[b], kb[b], vb[b], self.rk[b], self.rv[b], [self.R[b]] * H, self.wk[b], self.wv[b],
+                               [self.fill[b]] * H, scale)
+            o[b], lse[b] = oo, ll
+            f = self.fill[b]
+            self.wk[b, :, f], self.wv[b, :, f] = kb[b], vb[b]
+            self.fill[b] += 1
+            kw = int(self.k[self.widx[b]])
+            Tw = self.W + (-(-self.W // kw) if kw > 0 else 0)
+            if self.fill[b] == Tw:                       # window complete: retain its FOCUS rows
+                rows = fo.window_summary_rows(self.W, kw)
+                r = self.R[b]
+                self.rk[b, :, r:r + rows.size] = self.wk[b][:, rows]
+                self.rv[b, :, r:r + rows.size] = self.wv[b][:, rows]
+                self.R[b] += rows.size
+                self.fill[b] = 0
+                self.widx[b] += 1
+        return o, lse
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_decode_steps_match_oracle(d):
+    B, H, W = 3, 2, 50
+    k_sched = np.array([10, 7, 25, 50, 3, 10, 10, 10], np.int32)
+    C_ring, C_win = 512, 72
+    cache = focus.Cache(B, H, d, C_ring=C_ring, C_win=C_win, W=W, k_sched=k_sched)
+    g = torch.Generator(device="cuda").manual_seed(3)
+    for t in (cache.ring_k, cache.ring_v, cache.win_k, cache.win_v):
+        t.copy_(torch.randn(t.shape, generator=g, device="cuda").bfloat16())
+    R0 = np.array([0, 37, 300], np.int32)
+    widx0 = np.array([0, 1, 2], np.int32)
+    fill0 = np.array([0, 50, 20], np.int32)   # window 1 has T_w = 58
+    cache.ring_len.copy_(torch.from_numpy(R0))
+    cache.win_idx.copy_(torch.from_numpy(widx0))
+    cache.win_fill.copy_(torch.from_numpy(fill0))
+    model = DecodeModel(cache.ring_k, cache.ring_v, R0, cache.win_k, cache.win_v, fill0, widx0, W, k_sched)
+    ws = cache.new_workspace()
+    scale = 1.0 / math.sqrt(d)
+    for step in range(70):
+        q, kn, vn = inputs.qkv((B, H, d), seed=100 + step, device="cuda")
+        o, lse = focus.attn_decode(cache, q, kn, vn, workspace=ws)
+        focus.kv_compact_window(cache)
+        o_ref, lse_ref = model.step(q, kn, vn, scale)
+        assert_attn_close(o, lse, o_ref, lse_ref, f"decode step {step}")
+    torch.cuda.synchronize()
+    assert np.array_equal(cache.ring_len.cpu().numpy(), model.R)
+    assert np.array_equal(cache.win_fill.cpu().numpy(), model.fill)
+    assert np.array_equal(cache.win_idx.cpu().numpy(), model.widx)
+    for b in range(B):
+        assert np.array_equal(bits(cache.ring_k[b])[:, :model.R[b]], model.rk[b, :, :model.R[b]])
+        assert np.array_equal(bits(cache.ring_v[b])[:, :model.R[b]], model.rv[b, :, :model.R[b]])
+
+
+def test_decode_full_window_is_reported_not_trapped():
+    B, H, d, W = 1, 1, 64, 10
+    cache = focus.Cache(B, H, d, C_ring=16, C_win=11, W=W, k_sched=[10])
+    cache.win_fill.fill_(11)                      # T_w = 11: already full
+    q, kn, vn = inputs.qkv((B, H, d), seed=1, device="cuda")
+    focus.attn_decode(cache, q, kn, vn)
+    assert focus.device_status(clear=True) == 3   # FOCUS_ERR_CAPACITY
+    assert int(cache.win_fill[0]) == 11
+
+
+# ----------------------------------------------------------------------------- full-size workloads, sampled rows
+
+def _sample_rows(L, n_windows, rows_per_window, seed):
+    rng = np.random.default_rng(seed)
+    M = L["M"]
+    ws = sorted(set([0, M - 1] + list(rng.integers(0, M, size=n_windows - 2))))
+    off = L["win_off_host"]
+    rows = []
+    for w in ws:
+        a, e = int(off[w]), int(off[w + 1])
+        rows += [a, e - 1] + list(rng.integers(a, e, size=rows_per_window - 2))
+    return np.array(sorted(set(rows)), np.int64)
+
+
+@pytest.mark.parametrize("name", ["prefill_128kb_h32_d128", "prefill_256kb_ksweep_h32_d128"])
+def test_full_size_prefill_sampled(name):
+    from paper_2511_14694_gb300.workloads import WORKLOADS
+    cfg = WORKLOADS[name]
+    N, W, B, H, d = cfg["N"], cfg["W"], cfg["B"], cfg["H"], cfg["d"]
+    M = -(-N // W)
+    k_s = inputs.k_schedule(M, cfg["k"], seed=inputs.DEFAULT_SEED)
+    L = focus.layout(N, W, k_s)
+    q, k, v = inputs.qkv((B, H, L["T"], d), std=cfg["std"], seed=inputs.DEFAULT_SEED, device="cuda")
+    cache = focus.Cache(B, H, d, C_ring=L["R"])
+    o, lse = pipeline.prefill_masked_parallel(cache, q, k, v, L)
+    torch.cuda.synchronize()
+    rows = _sample_rows(L, 6, 4, seed=1)
+    heads = [0, 7, 31]
+    ref_L = fo.layout(N, W, k_s)
+    o_ref, lse_ref = fo.attn_rows(q[0, heads].cpu(), k[0, heads].cpu(), v[0, heads].cpu(), ref_L["kind"],
+                                  ref_L["win"], 1.0 / math.sqrt(d), np.repeat(np.arange(len(heads)), rows.size),
+                                  np.tile(rows, len(heads)))
+    og = o[0, heads][:, rows]
+    lg = lse[0, heads][:, rows]
+    assert_attn_close(og, lg, o_ref.reshape(len(heads), rows.size, d), lse_ref.reshape(len(heads), rows.size), name)
+    assert (cache.ring_len.cpu().numpy() == L["R"]).all()
+
+
+def test_full_size_decode_sampled():
+    """Batch 64, 32 heads, d=128, 10,000 retained summaries + partly filled windows
+    (fill ~ U{0..1009}); three steps, sequences at fill 1009 roll their window."""
+    from paper_2511_14694_gb300.workloads import WORKLOADS
+    cfg = WORKLOADS["decode_1mb_b64_h32_d128"]
+    B, H, d, W, R = cfg["B"], cfg["H"], cfg["d"], cfg["W"], cfg["R"]
+    k_sched = np.full(2_000, cfg["k"][0], np.int32)
+    T_w = W + W // cfg["k"][0]
+    cache = focus.Cache(B, H, d, C_ring=R + 256, C_win=1_024, W=W, k_sched=k_sched)
+    for i, t in enumerate((cache.ring_k, cache.ring_v, cache.win_k, cache.win_v)):
+        t.copy_(inputs.normal_bf16(t.shape, cfg["std"], seed=50 + i, device="cuda"))
+    fill0 = inputs.start_fill(B, T_w - 1, seed=inputs.DEFAULT_SEED)
+    fill0[:4] = T_w - 1
+    cache.ring_len.fill_(R)
+    cache.win_idx.fill_(R // (W // cfg["k"][0]))
+    cache.win_fill.copy_(torch.from_numpy(fill0))
+    rng = np.random.default_rng(0)
+    pairs = [(0, 0), (1, 5), (3, 31)] + [(int(b), int(h)) for b, h in zip(rng.integers(0, B, 9), rng.integers(0, H, 9))]
+    ws = cache.new_workspace()
+    for step in range(3):
+        R_now = cache.ring_len.cpu().numpy().copy()
+        fill_now = cache.win_fill.cpu().numpy().copy()
+        snap = {(b, h): (cache.ring_k[b, h].cpu(), cache.ring_v[b, h].cpu(), cache.win_k[b, h].cpu(),
+                         cache.win_v[b, h].cpu()) for b, h in pairs}
+        q, kn, vn = inputs.qkv((B, H, d), std=cfg["std"], seed=200 + step, device="cuda")
+        o, lse = focus.attn_decode(cache, q, kn, vn, workspace=ws)
+        focus.kv_compact_window(cache)
+        torch.cuda.synchronize()
+        for b, h in pairs:
+            rk, rv, wk, wv = snap[(b, h)]
+            o_ref, lse_ref = fo.decode(q[b, h][None].cpu(), kn[b, h][None].cpu(), vn[b, h][None].cpu(), rk[None],
+                                       rv[None], [R_now[b]], wk[None], wv[None], [fill_now[b]], 1.0 / math.sqrt(d))
+            assert_attn_close(o[b, h][None], lse[b, h][None], o_ref, lse_ref, f"decode b={b} h={h} step={step}")
+    assert (cache.ring_len.cpu().numpy()[:4] == R + W // cfg["k"][0]).all()
+    assert (cache.win_fill.cpu().numpy()[:4] == 2).all()
