@@ -1,0 +1,508 @@
+"""Benchmark of the FOCUS compressed-context attention path on GB300.
+
+Default workload: Evo-2-7B-shaped prefill, batch 1, N = 128,000 nt in 128
+windows of W = 1,000 with a summary every k = 100 nt (1,280 retained
+summaries), 32 heads, d = 128, bf16 Q/K/V ~ N(0,1)/sqrt(d). One step = the
+whole prefill path over that input: focus_layout -> focus_kv_compact (bulk,
+all windows) -> focus_attn_prefill (masked-parallel over all windows).
+The decode leg times focus_attn_decode + focus_kv_compact on batch 64 with
+10,000 retained summaries and partly filled windows per head (one leg = 256
+decode steps).
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl focus|reference]
+For N > 1 launch with torch.distributed.run; each rank runs the same workload
+on its own GPU (weak scaling, no collective on the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+NOMINAL_HBM_GBS = 7900.0
+METRIC = "compressed-context prefill tokens/s and decode tokens/s at 1 GB300; % of roofline"
+
+
+# ----------------------------------------------------------------------------- helpers
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return {k: float(d[k]) for k in ("hbm_gbs", "bf16_tflops", "bf16_tflops_sustained")}, "measured"
+    except Exception:
+        return dict(PEAKS_FALLBACK), "fallback"
+
+
+def visible_pairs(win_off, ring_off):
+    """Unmasked (query, key) pairs of the masked-parallel prefill: per window w,
+    T_w (T_w + 1) / 2 causal pairs plus T_w * R_w ring pairs."""
+    win_off = np.asarray(win_off, dtype=np.int64)
+    ring_off = np.asarray(ring_off, dtype=np.int64)
+    Tw = np.diff(win_off)
+    Rw = ring_off[:-1]
+    return int((Tw * (Tw + 1) // 2).sum() + (Tw * Rw).sum())
+
+
+def kernel_traffic(kernel_key: str, source: str):
+    """DRAM bytes per launch from a committed ncu summary, only while the kernel
+    source is unchanged since the counters were taken (else None)."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)[kernel_key]
+        with open(os.path.join(ROOT, source), "rb") as f:
+            sha = hashlib.sha256(f.read()).hexdigest()[:16]
+        return float(d["bytes_per_launch"]) if d.get("source_sha") == sha else None
+    except Exception:
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled every 200 ms while running."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index, self.proc, self.lines = index, None, []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200",
+                 "-i", str(self.index)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+            t0 = time.time()          # the timed region starts once sampling is live
+            while not self.lines and time.time() - t0 < 3.0 and self.proc.poll() is None:
+                time.sleep(0.02)
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.t.join(timeout=2)
+        return False
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[3:7]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- distributed
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ----------------------------------------------------------------------------- oracle (CPU baseline)
+
+def oracle_prefill_sample(cfg, L_host, q, k, v, budget_s=12.0, max_windows=None):
+    """Times the fp64 oracle's sequential prefill on a bounded sample of the
+    workload (a subset of heads and evenly spaced windows) and extrapolates to
+    the whole workload by visible pairs. Returns (seconds for the full workload,
+    description, cores)."""
+    from oracle import focus_oracle as fo
+    win_off, ring_off, kind = L_host["win_off"], L_host["ring_off"], L_host["kind"]
+    M = win_off.size - 1
+    d = cfg["d"]
+    total_pairs = visible_pairs(win_off, ring_off) * cfg["B"] * cfg["H"]
+    Tw = np.diff(win_off.astype(np.int64))
+    pairs_w = Tw * (Tw + 1) // 2 + Tw * ring_off[:-1].astype(np.int64)
+    # grow the sample until it takes about budget_s
+    n_w, spent, done_pairs, heads_done = 1, 0.0, 0, 0
+    h = 0
+    while spent < budget_s and heads_done < cfg["H"]:
+        step = max(1, M // n_w)
+        want = np.zeros(M, np.uint8)
+        want[::step] = 1
+        if max_windows:
+            want[np.nonzero(want)[0][max_windows:]] = 0
+        t0 = time.perf_counter()
+        fo.prefill_sequential(q[h], k[h], v[h], win_off, kind, 1.0 / math.sqrt(d), want=want)
+        spent += time.perf_counter() - t0
+        done_pairs += int(pairs_w[want.astype(bool)].sum())
+        heads_done += 1
+        h = (h + 1) % q.shape[0]
+        n_w = min(M, n_w * 2)
+    full_s = spent * total_pairs / max(done_pairs, 1)
+    desc = (f"fp64 oracle sequential prefill on {heads_done} head-passes over evenly spaced windows "
+            f"({done_pairs:,} of {total_pairs:,} visible pairs, {spent:.1f} s), extrapolated by visible pairs")
+    return full_s, desc, os.cpu_count()
+
+
+# ----------------------------------------------------------------------------- focus arm
+
+def run_prefill_leg(args, cfg, world, rank, local):
+    import torch
+    from paper_2511_14694_gb300 import focus, inputs, pipeline
+
+    B, N, W, H, d = cfg["B"], cfg["N"], cfg["W"], cfg["H"], cfg["d"]
+    M = -(-N // W)
+    k_s = inputs.k_schedule(M, cfg["k"], seed=inputs.DEFAULT_SEED)
+    dev = torch.device("cuda", local)
+    nt = inputs.nucleotides(B, N, seed=inputs.DEFAULT_SEED, device=dev)
+    L = focus.layout_alloc(N, W, k_s, B=B, device=dev)
+    q, k, v = inputs.qkv((B, H, L["T"], d), std=cfg["std"], seed=inputs.DEFAULT_SEED + rank, device=dev)
+    cache = focus.Cache(B, H, d, C_ring=max(L["R"], 1), device=dev)
+    o = torch.empty_like(q)
+    lse = torch.empty((B, H, L["T"]), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def front():
+        focus.layout_run(L, nt, stream=stream)
+        focus.kv_compact_bulk(cache, k, v, L, 0, L["M"], src_row0=0, stream=stream)
+
+    def attn():
+        focus.attn_prefill(cache, q, k, v, L, 0, L["M"], o=o, lse=lse, stream=stream, flags=args.prefill_flags)
+
+    for _ in range(args.warmup):
+        front()
+        attn()
+    torch.cuda.synchronize(dev)
+    assert focus.device_status(clear=True) == 0
+    win_off = L["win_off"].cpu().numpy()
+    ring_off = L["ring_off"].cpu().numpy()
+    pairs = visible_pairs(win_off, ring_off)
+    flops_per_step = 4.0 * d * H * B * pairs
+
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    with ClockSampler(local) as clk:
+        t_start.record(stream)
+        for i in range(args.steps):
+            front()
+            ev[i][0].record(stream)
+            attn()
+            ev[i][1].record(stream)
+        t_end.record(stream)
+        torch.cuda.synchronize(dev)
+        # if the timed region was shorter than three sampling periods, keep the same
+        # load running right after it until three samples exist
+        extra = 0
+        while len(clk.lines) < 3 and extra < 200 and not args.no_clock_wait:
+            front()
+            attn()
+            extra += 1
+            if extra % 20 == 0:
+                torch.cuda.synchronize(dev)
+        torch.cuda.synchronize(dev)
+    barrier(world)
+    assert focus.device_status(clear=True) == 0
+    step_ms = t_start.elapsed_time(t_end) / args.steps
+    step_ms = max_over_ranks(step_ms, world)
+    attn_ms = sum(a.elapsed_time(b) for a, b in ev) / args.steps
+    launches = 4 * args.steps   # layout scan + layout rows + bulk compaction + prefill
+
+    # end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        steps_e2e = max(1, min(args.steps, 5))
+        h_nt = nt.cpu().pin_memory()
+        h_q, h_k, h_v = (x.cpu().pin_memory() for x in (q, k, v))
+        h_o = torch.empty(o.shape, dtype=o.dtype).pin_memory()
+        h_lse = torch.empty(lse.shape, dtype=lse.dtype).pin_memory()
+
+        def e2e_step():
+            nt.copy_(h_nt, non_blocking=True)
+            q.copy_(h_q, non_blocking=True)
+            k.copy_(h_k, non_blocking=True)
+            v.copy_(h_v, non_blocking=True)
+            front()
+            attn()
+            h_o.copy_(o, non_blocking=True)
+            h_lse.copy_(lse, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize(dev)
+        barrier(world)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(steps_e2e):
+            e2e_step()
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        e2e_ms = max_over_ranks(e0.elapsed_time(e1) / steps_e2e, world)
+        h2d = sum(x.numel() * x.element_size() for x in (h_nt, h_q, h_k, h_v))
+        d2h = h_o.numel() * h_o.element_size() + h_lse.numel() * h_lse.element_size()
+        e2e = {"value": world * B * N / (e2e_ms / 1e3), "unit": "nt/s", "ms_per_step": e2e_ms,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps_e2e}
+        del h_q, h_k, h_v, h_o, h_lse
+
+    host_sample = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        host_sample = dict(win_off=win_off, ring_off=ring_off, kind=L["kind"].cpu().numpy(),
+                           q=q[0, :2].cpu(), k=k[0, :2].cpu(), v=v[0, :2].cpu())
+    res = dict(step_ms=step_ms, attn_ms=attn_ms, flops_per_step=flops_per_step, pairs=pairs, T=L["T"], R=L["R"],
+               clocks=clk.summary(), launches=launches, e2e=e2e, host_sample=host_sample, extra_steps=extra)
+    del q, k, v, o, lse, cache
+    torch.cuda.empty_cache()
+    return res
+
+
+def run_decode_leg(args, cfg, world, rank, local):
+    import torch
+    from paper_2511_14694_gb300 import focus, inputs
+
+    B, H, d, W, R = cfg["B"], cfg["H"], cfg["d"], cfg["W"], cfg["R"]
+    kk = cfg["k"][0]
+    Tw = W + -(-W // kk)
+    S = cfg["steps"]
+    dev = torch.device("cuda", local)
+    k_sched = np.full(R // (W // kk) + S // W + 16, kk, np.int32)
+    cache = focus.Cache(B, H, d, C_ring=R + 256, C_win=1_024, W=W, k_sched=k_sched, device=dev)
+    for i, t in enumerate((cache.ring_k, cache.ring_v, cache.win_k, cache.win_v)):
+        t.copy_(inputs.normal_bf16(t.shape, cfg["std"], seed=50 + i + 10 * rank, device=dev))
+    fill0 = inputs.start_fill(B, Tw - 1, seed=inputs.DEFAULT_SEED)
+    widx0 = R // (W // kk)
+    qs, ks_, vs = inputs.qkv((S, B, H, d), std=cfg["std"], seed=300 + rank, device=dev)
+    o = torch.empty((B, H, d), dtype=torch.bfloat16, device=dev)
+    lse = torch.empty((B, H), dtype=torch.float32, device=dev)
+    ws = cache.new_workspace()
+    stream = torch.cuda.current_stream(dev)
+
+    def reset():
+        cache.ring_len.fill_(R)
+        cache.win_idx.fill_(widx0)
+        cache.win_fill.copy_(torch.from_numpy(fill0).to(dev))
+
+    def leg(evs=None):
+        for s in range(S):
+            if evs is not None:
+                evs[s][0].record(stream)
+            focus.attn_decode(cache, qs[s], ks_[s], vs[s], o=o, lse=lse, workspace=ws, stream=stream)
+            if evs is not None:
+                evs[s][1].record(stream)
+            focus.kv_compact_window(cache, stream=stream)
+
+    reps = max(1, args.decode_reps)
+    reset()
+    leg()
+    torch.cuda.synchronize(dev)
+    assert focus.device_status(clear=True) == 0
+    # bytes the decode reads/writes per leg (host simulation of the fill/ring evolution)
+    fill = fill0.astype(np.int64).copy()
+    Rb = np.full(B, R, np.int64)
+    bytes_leg = 0
+    for _ in range(S):
+        bytes_leg += int(H * ((Rb + fill) * 2 * d * 2 + 6 * d * 2 + 4).sum())
+        fill += 1
+        full = fill == Tw
+        Rb[full] += Tw - W
+        fill[full] = 0
+    evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(S)]
+           for _ in range(reps)]
+    times = []
+    barrier(world)
+    with ClockSampler(local) as clk:
+        for r in range(reps):
+            reset()
+            torch.cuda.synchronize(dev)
+            t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            t0.record(stream)
+            leg(evs[r])
+            t1.record(stream)
+            torch.cuda.synchronize(dev)
+            times.append(t0.elapsed_time(t1))
+    barrier(world)
+    assert focus.device_status(clear=True) == 0
+    leg_ms = max_over_ranks(sum(times) / reps, world)
+    dec_ms = sum(a.elapsed_time(b) for rr in evs for a, b in rr) / reps
+    return dict(leg_ms=leg_ms, decode_kernels_ms=dec_ms, bytes_leg=bytes_leg, steps=S, B=B,
+                clocks=clk.summary(), launches=3 * S * reps)
+
+
+def run_focus(args, world, rank, local):
+    import torch
+    from paper_2511_14694_gb300.workloads import WORKLOADS
+    torch.cuda.set_device(local)
+    peaks, peaks_src = load_peaks()
+    cfg = WORKLOADS[args.workload]
+    pre = run_prefill_leg(args, cfg, world, rank, local)
+    dec = None
+    if not args.no_decode:
+        dec = run_decode_leg(args, WORKLOADS["decode_1mb_b64_h32_d128"], world, rank, local)
+    if rank != 0:
+        return
+    N_tot = world * cfg["B"] * cfg["N"]
+    value = N_tot / (pre["step_ms"] / 1e3)
+    achieved = pre["flops_per_step"] / (pre["attn_ms"] / 1e3) / 1e12
+    traffic = kernel_traffic("prefill_attention", "paper_2511_14694_gb300/csrc/prefill_mma.cu")
+    line = {
+        "metric": METRIC,
+        "value": value, "unit": "nt/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": pre["step_ms"], "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic (seeded N(0,1)/sqrt(d) bf16 Q/K/V, uniform A/C/G/T ids)",
+        "config": {"workload": args.workload, "B": cfg["B"], "N": cfg["N"], "W": cfg["W"], "k": list(cfg["k"]),
+                   "H": cfg["H"], "d": cfg["d"], "T_augmented": pre["T"], "R_retained": pre["R"],
+                   "step": "focus_layout + focus_kv_compact(bulk) + focus_attn_prefill(masked-parallel)",
+                   "l2": "inputs larger than L2 (Q/K/V %.2f GB per step)" % (3 * pre["T"] * cfg["H"] * cfg["d"] * 2 / 1e9),
+                   "prefill_kernel": "legacy mma.sync" if args.prefill_flags & 1 else "default"},
+        "augmented_tokens_per_s": world * cfg["B"] * pre["T"] / (pre["step_ms"] / 1e3),
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                     "frac": achieved / peaks["bf16_tflops"], "traffic": traffic,
+                     "peak_source": f"{peaks_src} bf16 dense burst",
+                     "frac_of_sustained": achieved / peaks["bf16_tflops_sustained"],
+                     "kernel": "prefill attention", "flop_per_launch": pre["flops_per_step"],
+                     "visible_pairs": pre["pairs"], "avg_launch_ms": pre["attn_ms"]},
+        "clocks": pre["clocks"],
+        "e2e": pre["e2e"],
+        "gpu_launches": pre["launches"],
+    }
+    if dec is not None:
+        gbs = dec["bytes_leg"] / (dec["decode_kernels_ms"] / 1e3) / 1e9
+        line["decode"] = {
+            "workload": "decode_1mb_b64_h32_d128", "value": world * dec["B"] * dec["steps"] / (dec["leg_ms"] / 1e3),
+            "unit": "tokens/s", "ms_per_step": dec["leg_ms"] / dec["steps"],
+            "step": "focus_attn_decode + focus_kv_compact(window)",
+            "roofline": {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                         "frac": gbs / peaks["hbm_gbs"], "frac_of_nominal": gbs / NOMINAL_HBM_GBS,
+                         "peak_source": f"{peaks_src} copy bandwidth", "bytes_per_step": dec["bytes_leg"] / dec["steps"],
+                         "avg_decode_call_ms": dec["decode_kernels_ms"] / dec["steps"],
+                         "traffic": kernel_traffic("decode_split", "paper_2511_14694_gb300/csrc/decode.cu")},
+            "clocks": dec["clocks"],
+        }
+        line["decode"]["gpu_launches"] = dec["launches"]
+    if pre["host_sample"] is not None:
+        hs = pre["host_sample"]
+        full_s, desc, cores = oracle_prefill_sample(cfg, hs, hs["q"], hs["k"], hs["v"], budget_s=args.cpu_budget)
+        line["cpu_baseline"] = {"value": cfg["B"] * cfg["N"] / full_s, "unit": "nt/s", "cores": cores,
+                                "kind": "oracle", "sample": desc}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------- reference arm (the oracle)
+
+def run_reference(args, world, rank, local):
+    """The fp64 CPU oracle timed on the host cores, on the same workload, metric
+    and unit; each step is a bounded sample extrapolated by visible pairs."""
+    if rank != 0:
+        return
+    import torch
+    from oracle import focus_oracle as fo
+    from paper_2511_14694_gb300 import inputs
+    from paper_2511_14694_gb300.workloads import WORKLOADS
+    cfg = WORKLOADS[args.workload]
+    B, N, W, H, d = cfg["B"], cfg["N"], cfg["W"], cfg["H"], cfg["d"]
+    M = -(-N // W)
+    k_s = inputs.k_schedule(M, cfg["k"], seed=inputs.DEFAULT_SEED)
+    L = fo.layout(N, W, k_s)
+    # two heads of inputs, drawn with the same generator recipe on the CPU
+    q, k, v = inputs.qkv((2, L["T"], d), std=cfg["std"], seed=inputs.DEFAULT_SEED, device="cpu")
+    hs = dict(win_off=L["win_off"], ring_off=L["ring_off"], kind=L["kind"])
+    budget = max(2.0, args.cpu_budget / max(1, args.steps + args.warmup))
+    for _ in range(args.warmup):
+        oracle_prefill_sample(cfg, hs, q, k, v, budget_s=budget, max_windows=4)
+    secs, desc = [], ""
+    for _ in range(args.steps):
+        full_s, desc, cores = oracle_prefill_sample(cfg, hs, q, k, v, budget_s=budget, max_windows=4)
+        secs.append(full_s)
+    full_s = statistics.median(secs)
+    value = B * N / full_s
+    line = {"metric": METRIC, "value": value, "unit": "nt/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": full_s * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": args.workload, "B": B, "N": N, "W": W, "k": list(cfg["k"]), "H": H, "d": d},
+            "cpu_baseline": {"value": value, "unit": "nt/s", "cores": os.cpu_count(), "kind": "oracle",
+                             "sample": desc},
+            "e2e": {"value": value, "unit": "nt/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="focus", choices=["focus", "reference"])
+    ap.add_argument("--workload", default="prefill_128kb_h32_d128")
+    ap.add_argument("--decode-reps", type=int, default=2)
+    ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--no-clock-wait", action="store_true",
+                    help="do not extend the load after a short timed region (profiling runs)")
+    ap.add_argument("--legacy", action="store_true", help="time the legacy mma.sync prefill kernel")
+    args = ap.parse_args()
+    args.warmup = max(3, args.warmup)
+    args.prefill_flags = 1 if args.legacy else 0
+    world, rank, local = dist_setup()
+    if args.impl == "reference":
+        run_reference(args, world, rank, local)
+    else:
+        run_focus(args, world, rank, local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

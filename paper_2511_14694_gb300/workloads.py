@@ -24,6 +24,9 @@ WORKLOADS = {
     # ultra-long streaming prefill with per-window compaction
     "stream_1mb_b4_h32_d128": dict(mode="stream", B=4, N=1_000_000, W=1_000, k=(100,), H=32, d=128,
                                    std=1.0 / math.sqrt(128), pool=8),
+    # a smaller prefill of the same shape (32 windows) for profiler captures: inputs still exceed L2
+    "prefill_32kb_h32_d128": dict(mode="prefill", B=1, N=32_000, W=1_000, k=(100,), H=32, d=128,
+                                  std=1.0 / math.sqrt(128)),
     # plain causal attention (no compression) at 128 kb, for the O(N^2) comparison
     "causal_128kb_h32_d128": dict(mode="prefill", B=1, N=128_000, W=128_000, k=(0,), H=32, d=128,
                                   std=1.0 / math.sqrt(128)),
