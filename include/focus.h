@@ -187,6 +187,34 @@ focus_status focus_attn_decode(const focus_cache* cache, const void* q, const vo
                                const void* v_new, float scale, void* o, float* lse,
                                void* workspace, size_t workspace_bytes, cudaStream_t stream);
 
+/* Allocation-free variant of focus_attn_decode. The paper has no counterpart:
+ * this entry point exists for callers that cannot hand the library scratch
+ * memory, e.g. a plugin inside a host runtime that owns all device memory and
+ * passes in only its input and output buffers, or a serving loop that must not
+ * call cudaMalloc/cudaFree (which can synchronise the device) between steps.
+ *
+ * Computes exactly what focus_attn_decode computes, with the same arguments
+ * minus the workspace. The split-K partials go to a fixed array of
+ * FOCUS_DECODE_NOALLOC_SCRATCH_BYTES inside the library, which every GPU that
+ * loads the library holds until the process exits. The call allocates nothing.
+ *   - If the cache needs more scratch than that (focus_decode_workspace_size(cache)
+ *     > FOCUS_DECODE_NOALLOC_SCRATCH_BYTES; batch 64 x 32 heads at d = 128 with
+ *     about 12k ring + window rows needs 12.8 MB) it returns FOCUS_ERR_CAPACITY
+ *     and launches nothing: use focus_attn_decode with a workspace instead.
+ *   - All calls on a device share the one array. Calls whose kernels overlap on
+ *     the GPU (different streams without ordering between them) race on it and
+ *     give wrong results; calls ordered on one stream are safe. The array keeps
+ *     the previous call's contents; this needs no clearing, because every split
+ *     writes its partial before the merge reads it.
+ *   - The first call on each device looks up the array's device address (with
+ *     that device current) and keeps it; make that first call before capturing
+ *     any stream. */
+#define FOCUS_DECODE_NOALLOC_SCRATCH_BYTES (16u << 20)
+
+focus_status focus_attn_decode_noalloc(const focus_cache* cache, const void* q, const void* k_new,
+                                       const void* v_new, float scale, void* o, float* lse,
+                                       cudaStream_t stream);
+
 /* ------------------------------------------------------------------------ */
 /* focus_kv_compact — KV retention after a window (App. A, "KV compression  */
 /* and budget"; Sec. 3.2 "KV retention and memory profile").               */

@@ -158,6 +158,19 @@ focus_status focus_attn_decode(const focus_cache* cache, const void* q, const vo
     return from_cuda(focus::launch_decode(*cache, q, k_new, v_new, scale, o, lse, workspace, st, stream));
 }
 
+focus_status focus_attn_decode_noalloc(const focus_cache* cache, const void* q, const void* k_new,
+                                       const void* v_new, float scale, void* o, float* lse, cudaStream_t stream) {
+    focus_status s = check_cache(cache, true);
+    if (s != FOCUS_OK) return s;
+    if (!q || !k_new || !v_new || !o || !isfinite(scale)) return FOCUS_ERR_INVALID_ARG;
+    if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(o)) return FOCUS_ERR_UNSUPPORTED;
+    if (focus_decode_workspace_size(cache) > (size_t)FOCUS_DECODE_NOALLOC_SCRATCH_BYTES) return FOCUS_ERR_CAPACITY;
+    int32_t* st = nullptr;
+    s = status_ptr(&st);
+    if (s != FOCUS_OK) return s;
+    return from_cuda(focus::launch_decode_noalloc(*cache, q, k_new, v_new, scale, o, lse, st, stream));
+}
+
 focus_status focus_kv_compact(const focus_cache* cache, const focus_compact_args* a, cudaStream_t stream) {
     if (!a) return FOCUS_ERR_INVALID_ARG;
     const bool bulk = a->src_k != nullptr;

@@ -47,6 +47,9 @@ cudaError_t launch_decode(const focus_cache& c, const void* q, const void* k_new
                           float scale, void* o, float* lse, void* workspace, int32_t* status,
                           cudaStream_t stream);
 
+cudaError_t launch_decode_noalloc(const focus_cache& c, const void* q, const void* k_new, const void* v_new,
+                                  float scale, void* o, float* lse, int32_t* status, cudaStream_t stream);
+
 cudaError_t launch_prefill_mma(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
                                cudaStream_t stream);
 

@@ -9,10 +9,22 @@
 // groups through shared memory and writes one partial (m, l, o) per split. A
 // second small kernel merges the splits with their log-sum-exp weights and
 // advances win_fill.
+#include <mutex>
+
 #include "common.cuh"
 
 namespace focus {
 namespace {
+
+// Fixed scratch for focus_attn_decode_noalloc. Callers that cannot allocate
+// device memory get their split-K partials here instead of in a workspace of
+// their own. Every device that loads the library keeps these bytes until the
+// process exits, and all calls share them.
+static __device__ __align__(256) unsigned char g_decode_scratch[FOCUS_DECODE_NOALLOC_SCRATCH_BYTES];
+
+constexpr int kMaxScratchDevices = 64;
+void* g_scratch_ptr[kMaxScratchDevices];
+std::mutex g_scratch_mu;
 
 constexpr int kDecodeChunk = 1024;   // keys per split
 constexpr int kDecodeThreads = 128;
@@ -235,6 +247,34 @@ cudaError_t launch_decode(const focus_cache& c, const void* q, const void* k_new
                           cudaStream_t stream) {
     if (c.d == 128) return launch_decode_d<128>(c, q, k_new, v_new, scale, o, lse, workspace, status, stream);
     return launch_decode_d<64>(c, q, k_new, v_new, scale, o, lse, workspace, status, stream);
+}
+
+// Device address of g_decode_scratch on the current device. Host code cannot
+// pass the array's name to a kernel (on the host it names a stand-in, not device
+// memory), so the first call on each device looks the address up, with that
+// device current, and keeps it.
+cudaError_t decode_noalloc_scratch(void** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxScratchDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(g_scratch_mu);
+    if (!g_scratch_ptr[dev]) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_decode_scratch);
+        if (e != cudaSuccess) return e;
+        g_scratch_ptr[dev] = p;
+    }
+    *out = g_scratch_ptr[dev];
+    return cudaSuccess;
+}
+
+cudaError_t launch_decode_noalloc(const focus_cache& c, const void* q, const void* k_new, const void* v_new,
+                                  float scale, void* o, float* lse, int32_t* status, cudaStream_t stream) {
+    void* scratch = nullptr;
+    cudaError_t e = decode_noalloc_scratch(&scratch);
+    if (e != cudaSuccess) return e;
+    return launch_decode(c, q, k_new, v_new, scale, o, lse, scratch, status, stream);
 }
 
 }  // namespace focus

@@ -87,6 +87,8 @@ def load() -> ctypes.CDLL:
     lib.focus_decode_workspace_size.argtypes = [ctypes.POINTER(CacheDesc)]
     lib.focus_attn_decode.restype = ctypes.c_int
     lib.focus_attn_decode.argtypes = [ctypes.POINTER(CacheDesc), _P, _P, _P, _f32, _P, _P, _P, ctypes.c_size_t, _P]
+    lib.focus_attn_decode_noalloc.restype = ctypes.c_int
+    lib.focus_attn_decode_noalloc.argtypes = [ctypes.POINTER(CacheDesc), _P, _P, _P, _f32, _P, _P, _P]
     lib.focus_kv_compact.restype = ctypes.c_int
     lib.focus_kv_compact.argtypes = [ctypes.POINTER(CacheDesc), ctypes.POINTER(CompactArgs), _P]
     _lib = lib
@@ -265,6 +267,24 @@ def attn_decode(cache: Cache, q, k_new, v_new, scale=None, o=None, lse=None, wor
            lib.focus_attn_decode(ctypes.byref(cache.desc), _ptr(q), _ptr(k_new), _ptr(v_new), scale, _ptr(o),
                                  _ptr(lse), _ptr(workspace), workspace.numel() * workspace.element_size(),
                                  _stream(stream)))
+    return o, lse
+
+
+def attn_decode_noalloc(cache: Cache, q, k_new, v_new, scale=None, o=None, lse=None, stream=None):
+    """focus_attn_decode_noalloc: same as attn_decode, but the library keeps the
+    split-K scratch in its own fixed device array, so the caller passes no
+    workspace (for callers that cannot allocate device memory)."""
+    lib = load()
+    for name, t in (("q", q), ("k_new", k_new), ("v_new", v_new)):
+        _cuda(t, name, torch.bfloat16)
+    if o is None:
+        o = torch.empty_like(q)
+    if lse is None:
+        lse = torch.empty(q.shape[:2], dtype=torch.float32, device=q.device)
+    scale = 1.0 / math.sqrt(q.shape[-1]) if scale is None else float(scale)
+    _check("focus_attn_decode_noalloc",
+           lib.focus_attn_decode_noalloc(ctypes.byref(cache.desc), _ptr(q), _ptr(k_new), _ptr(v_new), scale,
+                                         _ptr(o), _ptr(lse), _stream(stream)))
     return o, lse
 
 
