@@ -150,7 +150,7 @@ typedef struct focus_prefill_args {
     int32_t     n_windows;    /* M (the offsets arrays hold M+1 entries) */
     int32_t     w_begin, w_end;   /* 0 <= w_begin < w_end <= M */
     int32_t     max_rows;     /* >= every window's augmented row count in the span */
-    float       scale;        /* softmax scale, usually 1/sqrt(d) */
+    float       scale;        /* softmax scale > 0, usually 1/sqrt(d) */
     uint32_t    flags;        /* FOCUS_PREFILL_* */
 } focus_prefill_args;
 

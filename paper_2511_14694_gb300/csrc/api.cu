@@ -125,7 +125,7 @@ focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_ar
     if (!a || !a->q || !a->k || !a->v || !a->o || !a->d_win_off || !a->d_ring_off) return FOCUS_ERR_INVALID_ARG;
     if (a->w_begin < 0 || a->w_end <= a->w_begin || a->w_end > a->n_windows || a->T_span < 0 || a->max_rows <= 0)
         return FOCUS_ERR_INVALID_ARG;
-    if (!isfinite(a->scale)) return FOCUS_ERR_INVALID_ARG;
+    if (!isfinite(a->scale) || !(a->scale > 0.f)) return FOCUS_ERR_INVALID_ARG;
     if (!aligned16(a->q) || !aligned16(a->k) || !aligned16(a->v) || !aligned16(a->o)) return FOCUS_ERR_UNSUPPORTED;
     if (a->T_span == 0) return FOCUS_OK;
     const int64_t tiles = focus::ceil_div64(a->max_rows, 64) * (int64_t)(a->w_end - a->w_begin);
@@ -133,7 +133,8 @@ focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_ar
     int32_t* st = nullptr;
     s = status_ptr(&st);
     if (s != FOCUS_OK) return s;
-    return from_cuda(focus::launch_prefill_mma(*cache, *a, st, stream));
+    if (a->flags & FOCUS_PREFILL_LEGACY_MMA) return from_cuda(focus::launch_prefill_mma(*cache, *a, st, stream));
+    return from_cuda(focus::launch_prefill_tc(*cache, *a, st, stream));
 }
 
 size_t focus_decode_workspace_size(const focus_cache* cache) {

@@ -52,5 +52,7 @@ cudaError_t launch_decode_noalloc(const focus_cache& c, const void* q, const voi
 
 cudaError_t launch_prefill_mma(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
                                cudaStream_t stream);
+cudaError_t launch_prefill_tc(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
+                              cudaStream_t stream);
 
 }  // namespace focus

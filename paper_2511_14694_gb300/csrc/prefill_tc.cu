@@ -1,0 +1,429 @@
+// Windowed prefill attention over the compressed context on the 5th-generation
+// tensor cores (tcgen05.mma, accumulators in TMEM, operands staged by TMA).
+//
+// What it computes (Eq. focus-attn's visible set; App. A.1-A.2): row a of
+// window w attends to ring rows [0, ring_off[w]) (retained FOCUS K/V of all
+// earlier windows, fully visible) and to window rows [0, a] (causal). The mask
+// is analytic per 128-key tile: only the last partial ring tile (key >= R_w)
+// and the diagonal window tile (key > row) are masked.
+//
+// CTA = two 128-row Q tiles of one (sequence, head, window) that share every
+// K/V tile, 12 warps in three warpgroups:
+//   warp 0     TMA producer: Q tiles once, then K_j, V_j into a ring of slots
+//   warp 1     TMEM owner + MMA issuer (one thread):
+//                S_t = Q_t K_j^T            (SS, both operands K-major, SW128)
+//                O_t += P_t V_j             (TS, P_t in TMEM over S_t, V MN-major)
+//              in ping-pong order PV_0(j-1), QK_0(j), PV_1(j-1), QK_1(j)
+//   warps 2-3  idle (they keep the softmax warpgroups aligned to warpgroups)
+//   warps 4-7  softmax of tile 0, warps 8-11 softmax of tile 1: each thread owns
+//              one row (32x32b TMEM loads), online softmax in the log2 domain with
+//              lazy rescaling of O (only when the running max grows by > 8),
+//              writes P (bf16) back into TMEM, and at the end normalises O and
+//              stores O and the LSE.
+// TMEM: S_0 cols [0,128), S_1 [128,256), O_0 [256, 256+D), O_1 [256+D, 256+2D).
+// Every mbarrier wait is bounded; on timeout the kernel reports
+// FOCUS_ERR_TIMEOUT, drains its own copies/MMAs (bounded), frees TMEM, returns.
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
+#include "common.cuh"
+#include "sm100.cuh"
+
+namespace focus {
+namespace {
+
+using namespace sm100;
+
+constexpr int BM = 128;             // rows per Q tile
+constexpr int BN = 128;             // keys per K/V tile
+constexpr int kSlots = 4;           // K/V staging slots (each holds one K or one V tile)
+constexpr int kThreads = 384;       // 12 warps
+constexpr int kBoxBytes = 128 * 128;   // one TMA box: 128 rows x 64 bf16 (128 B, swizzled)
+constexpr uint64_t kWaitNs = 2000000000ull;   // 2 s bound on any wait
+constexpr float kRescaleThreshold = 8.0f;     // log2 units: rescale O only if the max grows by > 2^8
+
+template <int D>
+struct Cfg {
+    static constexpr int kBoxes = D / 64;                       // TMA boxes per 128-row tile
+    static constexpr int kTileBytes = kBoxes * kBoxBytes;       // one Q/K/V tile
+    static constexpr int kQOff = 0;
+    static constexpr int kSlotOff = 2 * kTileBytes;
+    static constexpr int kBarOff = kSlotOff + kSlots * kTileBytes;
+    static constexpr int kSmem = kBarOff + 256 + 1024;          // + barriers + alignment slack
+};
+
+struct Bars {
+    uint64_t q;
+    uint64_t kv_full[kSlots];
+    uint64_t kv_empty[kSlots];
+    uint64_t s_full[2];
+    uint64_t p_full[2];
+    uint64_t o_full[2];
+    uint64_t drain;
+    uint32_t tmem;
+    int32_t abort;
+};
+
+__device__ __forceinline__ void fail(Bars* bars, int32_t* status) {
+    report(status, FOCUS_ERR_TIMEOUT);
+    atomicExch(&bars->abort, 1);
+}
+__device__ __forceinline__ bool aborted(Bars* bars) { return *(volatile int32_t*)&bars->abort != 0; }
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
+        const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+        const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_rk,
+        const __grid_constant__ CUtensorMap tm_rv, __nv_bfloat16* __restrict__ o, float* __restrict__ lse,
+        int64_t T_span, const int32_t* __restrict__ win_off, const int32_t* __restrict__ ring_off, int32_t w_begin,
+        int32_t w_end, int32_t ctas_pw, int32_t H, int32_t C_ring, float scale_log2, int32_t* status) {
+    using C = Cfg<D>;
+    extern __shared__ unsigned char smem_raw[];
+    uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    Bars* bars = reinterpret_cast<Bars*>(smem + C::kBarOff);
+
+    // ---- work item (longest first: later windows have longer rings) --------
+    const int32_t wi = blockIdx.x / ctas_pw;
+    const int32_t cta = ctas_pw - 1 - (int32_t)(blockIdx.x % ctas_pw);
+    const int32_t w = w_end - 1 - wi;
+    const int h = blockIdx.y, b = blockIdx.z;
+    const int32_t bh = b * H + h;
+    const int32_t w0 = win_off[w_begin];
+    const int32_t Tw = win_off[w + 1] - win_off[w];
+    const int32_t a0 = cta * 2 * BM;
+    if (a0 >= Tw) return;                               // uniform: nothing allocated yet
+    // Once any CTA has given up on a wait, later CTAs skip their work so that a
+    // systematic stall costs one wave of bounded waits, not one per wave.
+    if (*(volatile int32_t*)status == FOCUS_ERR_TIMEOUT) return;
+    const int32_t Rw = ring_off[w];
+    if (Rw > C_ring || (int64_t)(win_off[w_end] - w0) > T_span) {
+        if (threadIdx.x == 0) report(status, FOCUS_ERR_CAPACITY);
+        return;
+    }
+    const int32_t row_base = win_off[w] - w0;           // first row of the window in the span tensors
+    const int n_ring = (Rw + BN - 1) / BN;
+    const bool valid1 = a0 + BM < Tw;
+    const int n_kv0 = n_ring + 2 * cta + 1;
+    const int n_kv1 = valid1 ? n_ring + 2 * cta + 2 : 0;
+    const int n_kv_max = valid1 ? n_kv1 : n_kv0;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    // ---- setup -------------------------------------------------------------
+    if (threadIdx.x == 0) {
+        mbar_init(smem_addr(&bars->q), 1);
+        for (int s = 0; s < kSlots; ++s) {
+            mbar_init(smem_addr(&bars->kv_full[s]), 1);
+            mbar_init(smem_addr(&bars->kv_empty[s]), 1);
+        }
+        for (int t = 0; t < 2; ++t) {
+            mbar_init(smem_addr(&bars->s_full[t]), 1);
+            mbar_init(smem_addr(&bars->p_full[t]), BM);
+            mbar_init(smem_addr(&bars->o_full[t]), 1);
+        }
+        mbar_init(smem_addr(&bars->drain), 1);
+        bars->abort = 0;
+        fence_barrier_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_addr(&bars->tmem), 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = bars->tmem;
+
+    if (warp == 0) {
+        // ================================================= TMA producer
+        if (lane == 0) {
+            prefetch_tmap(&tm_q);
+            prefetch_tmap(&tm_k);
+            prefetch_tmap(&tm_v);
+            prefetch_tmap(&tm_rk);
+            prefetch_tmap(&tm_rv);
+            const uint32_t bq = smem_addr(&bars->q);
+            mbar_expect_tx(bq, 2 * C::kTileBytes);
+            for (int t = 0; t < 2; ++t)
+                for (int x = 0; x < C::kBoxes; ++x)
+                    tma_load_3d(smem_addr(smem + C::kQOff + t * C::kTileBytes + x * kBoxBytes), &tm_q, x * 64,
+                                row_base + a0 + t * BM, bh, bq);
+            int issued = 0;
+            for (int j = 0; j < n_kv_max && !aborted(bars); ++j) {
+                const bool ring = j < n_ring;
+                const int32_t row = ring ? j * BN : row_base + (j - n_ring) * BN;
+                for (int part = 0; part < 2; ++part) {
+                    const int n = 2 * j + part, slot = n % kSlots, use = n / kSlots;
+                    if (use > 0 && !mbar_wait(smem_addr(&bars->kv_empty[slot]), (use - 1) & 1, kWaitNs)) {
+                        fail(bars, status);
+                        break;
+                    }
+                    const uint32_t bf = smem_addr(&bars->kv_full[slot]);
+                    mbar_expect_tx(bf, C::kTileBytes);
+                    const CUtensorMap* map = part == 0 ? (ring ? &tm_rk : &tm_k) : (ring ? &tm_rv : &tm_v);
+                    for (int x = 0; x < C::kBoxes; ++x)
+                        tma_load_3d(smem_addr(smem + C::kSlotOff + slot * C::kTileBytes + x * kBoxBytes), map,
+                                    x * 64, row, bh, bf);
+                    issued = n + 1;
+                }
+            }
+            // drain: every issued copy must land before the CTA can exit
+            mbar_wait(smem_addr(&bars->q), 0, kWaitNs);
+            for (int n = (issued > kSlots ? issued - kSlots : 0); n < issued; ++n)
+                mbar_wait(smem_addr(&bars->kv_full[n % kSlots]), (n / kSlots) & 1, kWaitNs);
+        }
+    } else if (warp == 1) {
+        // ================================================= MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, BN, false, false);
+            constexpr uint32_t idesc_pv = idesc_bf16_f32(BM, D, false, true);
+            const uint32_t sq = smem_addr(smem + C::kQOff);
+            const uint32_t sslot = smem_addr(smem + C::kSlotOff);
+            bool ok = mbar_wait(smem_addr(&bars->q), 0, kWaitNs);
+            if (!ok) fail(bars, status);
+            for (int j = 0; ok && j <= n_kv_max; ++j) {
+                int vslot = -1, kslot = -1;
+                if (j >= 1) {
+                    const int n = 2 * (j - 1) + 1;
+                    vslot = n % kSlots;
+                    if (!mbar_wait(smem_addr(&bars->kv_full[vslot]), (n / kSlots) & 1, kWaitNs)) { ok = false; break; }
+                }
+                if (j < n_kv_max) {
+                    const int n = 2 * j;
+                    kslot = n % kSlots;
+                    if (!mbar_wait(smem_addr(&bars->kv_full[kslot]), (n / kSlots) & 1, kWaitNs)) { ok = false; break; }
+                }
+                tc_fence_after();
+                for (int t = 0; t < 2; ++t) {
+                    const int nkt = t == 0 ? n_kv0 : n_kv1;
+                    if (j >= 1 && j - 1 < nkt) {              // O_t += P_t(j-1) V_{j-1}
+                        if (!mbar_wait(smem_addr(&bars->p_full[t]), (j - 1) & 1, kWaitNs)) { ok = false; break; }
+                        tc_fence_after();
+                        const uint32_t vbase = sslot + vslot * C::kTileBytes;
+#pragma unroll
+                        for (int kk = 0; kk < BN / 16; ++kk)
+                            mma_ts(tmem + 256 + t * D, tmem + t * 128 + kk * 8,
+                                   smem_desc_sw128(vbase + kk * 2048, kBoxBytes, 1024), idesc_pv,
+                                   (j - 1 > 0 || kk > 0) ? 1u : 0u);
+                        if (j - 1 == nkt - 1) mma_commit(smem_addr(&bars->o_full[t]));
+                    }
+                    if (j < nkt) {                           // S_t = Q_t K_j^T
+                        const uint32_t qbase = sq + t * C::kTileBytes;
+                        const uint32_t kbase = sslot + kslot * C::kTileBytes;
+#pragma unroll
+                        for (int kk = 0; kk < D / 16; ++kk) {
+                            const uint32_t off = (kk / 4) * kBoxBytes + (kk % 4) * 32;
+                            mma_ss(tmem + t * 128, smem_desc_sw128(qbase + off, 16, 1024),
+                                   smem_desc_sw128(kbase + off, 16, 1024), idesc_qk, kk > 0 ? 1u : 0u);
+                        }
+                        mma_commit(smem_addr(&bars->s_full[t]));
+                    }
+                }
+                if (!ok) break;
+                if (vslot >= 0) mma_commit(smem_addr(&bars->kv_empty[vslot]));
+                if (kslot >= 0) mma_commit(smem_addr(&bars->kv_empty[kslot]));
+            }
+            if (!ok) fail(bars, status);
+            // drain: all issued MMAs complete before TMEM is freed
+            mma_commit(smem_addr(&bars->drain));
+            mbar_wait(smem_addr(&bars->drain), 0, kWaitNs);
+        }
+    } else if (warp >= 4) {
+        // ================================================= softmax / epilogue
+        const int t = (warp - 4) >> 2;                    // 0: warps 4-7, 1: warps 8-11
+        const int quarter = warp & 3;                     // TMEM lanes this warp may access
+        const int r = quarter * 32 + lane;                // row within the Q tile
+        const int32_t aq = a0 + t * BM + r;               // in-window row
+        const int n_kv = t == 0 ? n_kv0 : n_kv1;
+        const int qt = 2 * cta + t;                       // q-tile index within the window
+        const uint32_t lane_addr = (uint32_t)(quarter * 32) << 16;
+        const uint32_t s_addr = tmem + lane_addr + t * 128;
+        const uint32_t o_addr = tmem + lane_addr + 256 + t * D;
+        float m_run = -INFINITY, l_run = 0.f;
+        bool ok = true;
+        for (int j = 0; j < n_kv; ++j) {
+            if (!mbar_wait(smem_addr(&bars->s_full[t]), j & 1, kWaitNs)) { ok = false; break; }
+            tc_fence_after();
+            uint32_t sr[128];
+            tmem_ld32(s_addr + 0, sr);
+            tmem_ld32(s_addr + 32, sr + 32);
+            tmem_ld32(s_addr + 64, sr + 64);
+            tmem_ld32(s_addr + 96, sr + 96);
+            tmem_wait_ld();
+            float* s = reinterpret_cast<float*>(sr);
+            // analytic mask
+            const bool ring = j < n_ring;
+            if (ring) {
+                const int lim = Rw - j * BN;              // keys [0, lim) of this tile are visible
+                if (lim < BN) {
+#pragma unroll
+                    for (int c = 0; c < BN; ++c)
+                        if (c >= lim) s[c] = -INFINITY;
+                }
+            } else if (j - n_ring == qt) {                // diagonal tile: key c visible iff c <= r
+#pragma unroll
+                for (int c = 0; c < BN; ++c)
+                    if (c > r) s[c] = -INFINITY;
+            }
+            float mt = -INFINITY;
+#pragma unroll
+            for (int c = 0; c < BN; ++c) mt = fmaxf(mt, s[c]);
+            const float m_new = fmaxf(m_run, mt * scale_log2);
+            const bool need = m_new > m_run + kRescaleThreshold;
+            const bool any_need = __any_sync(0xffffffffu, need);
+            const float factor = need ? ex2_approx(m_run - m_new) : 1.f;
+            if (need) m_run = m_new;
+            l_run *= factor;
+            const float neg_m = -m_run;
+            float lsum = 0.f;
+#pragma unroll
+            for (int h2 = 0; h2 < 2; ++h2) {
+                uint32_t pk[32];
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const float p0 = ex2_approx(fmaf(s[h2 * 64 + 2 * i], scale_log2, neg_m));
+                    const float p1 = ex2_approx(fmaf(s[h2 * 64 + 2 * i + 1], scale_log2, neg_m));
+                    lsum += p0 + p1;
+                    pk[i] = pack_bf16x2(p0, p1);
+                }
+                tmem_st32(s_addr + h2 * 32, pk);
+            }
+            l_run += lsum;
+            // Lazy rescale of O_t (written by PV_t(j-1), which completed before S_t(j)
+            // was signalled; PV_t(j) waits for this thread's arrival below).
+            if (any_need && j > 0) {
+#pragma unroll
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t orr[32];
+                    tmem_ld32(o_addr + c * 32, orr);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) orr[i] = __float_as_uint(__uint_as_float(orr[i]) * factor);
+                    tmem_st32(o_addr + c * 32, orr);
+                }
+            }
+            tmem_wait_st();
+            tc_fence_before();
+            mbar_arrive(smem_addr(&bars->p_full[t]));
+        }
+        // ---- epilogue: O / l -> bf16, staged in this tile's Q buffer ------------
+        if (ok && n_kv > 0) ok = mbar_wait(smem_addr(&bars->o_full[t]), 0, kWaitNs);
+        if (!ok && n_kv > 0) fail(bars, status);
+        __syncwarp();
+        if (ok && n_kv > 0) {
+            tc_fence_after();
+            const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
+            uint8_t* stage = smem + C::kQOff + t * C::kTileBytes;     // rows [r] of 2*D bytes, 16-B chunks swizzled
+            constexpr int CH = D / 8;
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t orr[32];
+                tmem_ld32(o_addr + c * 32, orr);
+                tmem_wait_ld();
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) {          // 4 chunks of 8 values
+                    uint4 v;
+                    v.x = pack_bf16x2(__uint_as_float(orr[q4 * 8 + 0]) * inv_l, __uint_as_float(orr[q4 * 8 + 1]) * inv_l);
+                    v.y = pack_bf16x2(__uint_as_float(orr[q4 * 8 + 2]) * inv_l, __uint_as_float(orr[q4 * 8 + 3]) * inv_l);
+                    v.z = pack_bf16x2(__uint_as_float(orr[q4 * 8 + 4]) * inv_l, __uint_as_float(orr[q4 * 8 + 5]) * inv_l);
+                    v.w = pack_bf16x2(__uint_as_float(orr[q4 * 8 + 6]) * inv_l, __uint_as_float(orr[q4 * 8 + 7]) * inv_l);
+                    const int chunk = c * 4 + q4;
+                    *reinterpret_cast<uint4*>(stage + r * (2 * D) + ((chunk ^ (r & 7)) << 4)) = v;
+                }
+            }
+            if (lse && aq < Tw)
+                lse[(int64_t)bh * T_span + row_base + aq] = (m_run + __log2f(l_run)) * 0.69314718055994531f;
+            __syncwarp();
+            // the warp stores the 32 rows it staged: 32/CH rows per instruction, coalesced
+            __nv_bfloat16* ob = o + ((int64_t)bh * T_span + row_base + a0 + t * BM) * D;
+            constexpr int RPI = 32 / CH;                  // rows per store instruction
+            for (int i = 0; i < 32; i += RPI) {
+                const int rr = quarter * 32 + i + lane / CH;
+                const int chunk = lane % CH;
+                if (a0 + t * BM + rr < Tw)
+                    *reinterpret_cast<uint4*>(ob + (int64_t)rr * D + chunk * 8) =
+                        *reinterpret_cast<const uint4*>(stage + rr * (2 * D) + ((chunk ^ (rr & 7)) << 4));
+            }
+        }
+    }
+
+    // ---- teardown ------------------------------------------------------------
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
+// ---------------------------------------------------------------- host side
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::mutex g_encode_mu;
+
+cudaError_t get_encode(PFN_cuTensorMapEncodeTiled_v12000* out) {
+    std::lock_guard<std::mutex> lock(g_encode_mu);
+    if (!g_encode) {
+        void* fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+        if (e != cudaSuccess) return e;
+        if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorNotSupported;
+        g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    *out = g_encode;
+    return cudaSuccess;
+}
+
+// 3-D map over a [BH][rows][d] bf16 tensor, box = 128 rows x 64 columns, 128-byte swizzle.
+cudaError_t make_map(CUtensorMap* m, const void* ptr, int d, int64_t rows, int64_t bh) {
+    PFN_cuTensorMapEncodeTiled_v12000 enc;
+    cudaError_t e = get_encode(&enc);
+    if (e != cudaSuccess) return e;
+    cuuint64_t dims[3] = {(cuuint64_t)d, (cuuint64_t)rows, (cuuint64_t)bh};
+    cuuint64_t strides[2] = {(cuuint64_t)d * 2, (cuuint64_t)d * 2 * (cuuint64_t)rows};
+    cuuint32_t box[3] = {64, 128, 1};
+    cuuint32_t es[3] = {1, 1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box, es,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+template <int D>
+cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t* status, cudaStream_t stream) {
+    const int64_t BH = (int64_t)c.B * c.H;
+    CUtensorMap tq, tk, tv, trk, trv;
+    cudaError_t e;
+    if ((e = make_map(&tq, a.q, D, a.T_span, BH)) != cudaSuccess) return e;
+    if ((e = make_map(&tk, a.k, D, a.T_span, BH)) != cudaSuccess) return e;
+    if ((e = make_map(&tv, a.v, D, a.T_span, BH)) != cudaSuccess) return e;
+    if (c.C_ring > 0) {
+        if ((e = make_map(&trk, c.ring_k, D, c.C_ring, BH)) != cudaSuccess) return e;
+        if ((e = make_map(&trv, c.ring_v, D, c.C_ring, BH)) != cudaSuccess) return e;
+    } else {                                   // no ring: the maps are never read
+        trk = tk;
+        trv = tv;
+    }
+    const int smem = Cfg<D>::kSmem;
+    e = cudaFuncSetAttribute(prefill_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    const int ctas_pw = (a.max_rows + 2 * BM - 1) / (2 * BM);
+    dim3 grid((unsigned)((a.w_end - a.w_begin) * ctas_pw), c.H, c.B);
+    prefill_tc_kernel<D><<<grid, kThreads, smem, stream>>>(tq, tk, tv, trk, trv, (__nv_bfloat16*)a.o, a.lse,
+                                                          a.T_span, a.d_win_off, a.d_ring_off, a.w_begin, a.w_end,
+                                                          ctas_pw, c.H, c.C_ring, a.scale * 1.4426950408889634f,
+                                                          status);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_prefill_tc(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
+                              cudaStream_t stream) {
+    if (c.d == 128) return launch_d<128>(c, a, status, stream);
+    return launch_d<64>(c, a, status, stream);
+}
+
+}  // namespace focus
