@@ -12,6 +12,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "sm100.cuh"
 
 namespace focus {
 namespace {
@@ -27,8 +28,18 @@ void* g_scratch_ptr[kMaxScratchDevices];
 std::mutex g_scratch_mu;
 
 constexpr int kDecodeChunk = 1024;   // keys per split
-constexpr int kDecodeThreads = 128;
-constexpr int kUnroll = 8;           // key rows in flight per lane group
+constexpr int kDecodeThreads = 128;  // consumer threads (plus one producer warp)
+constexpr int kStages = 4;           // shared-memory stages in flight per CTA
+template <int D>
+constexpr int kStageRows = 8192 / (2 * D);   // 8 KB of K and 8 KB of V per stage
+constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s bound on any wait
+template <int D>
+constexpr int decode_groups() { return (kDecodeThreads / 32) * (32 / (D / 8)); }   // lane groups per CTA
+template <int D>
+constexpr int decode_smem_bytes() {   // K/V stages + full/empty barriers + the group merge buffers
+    return 2 * kStages * kStageRows<D> * D * 2 + 2 * kStages * 8 + 2 * decode_groups<D>() * 4 +
+           decode_groups<D>() * D * 4;
+}
 
 __device__ __forceinline__ void bf16x8_to_f32(const uint4& u, float* f) {
     const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&u);
@@ -49,124 +60,190 @@ __device__ __forceinline__ bool decode_state_ok(int32_t R, int32_t fill, int32_t
     return fill >= 0 && fill < Tw && fill < C_win;
 }
 
+// Split kernel: 4 consumer warps + 1 producer warp. The producer streams the
+// split's key rows as contiguous bulk copies (ring part, window part, new row)
+// into a ring of shared-memory stages; consumers read each row with d/8 lanes
+// (16 B each, conflict-free), reduce the dot product with shuffles and keep a
+// per-lane-group online softmax (log2 domain) in registers.
 template <int D>
-__global__ void __launch_bounds__(kDecodeThreads) decode_split_kernel(
+__global__ void __launch_bounds__(kDecodeThreads + 32) decode_split_kernel(
         const uint4* __restrict__ ring_k, const uint4* __restrict__ ring_v, uint4* __restrict__ win_k,
         uint4* __restrict__ win_v, const int32_t* __restrict__ ring_len, const int32_t* __restrict__ win_fill,
         const int32_t* __restrict__ win_idx, const int32_t* __restrict__ ks, int32_t n_windows, int32_t W,
         int32_t H, int32_t C_ring, int32_t C_win, const uint4* __restrict__ q, const uint4* __restrict__ k_new,
         const uint4* __restrict__ v_new, float scale_log2, float2* __restrict__ ws_ml, float* __restrict__ ws_o,
         int32_t n_splits, int32_t* status) {
+    using namespace sm100;
     constexpr int CPR = D / 8;          // 16-byte chunks per row = lanes per key
     constexpr int GPW = 32 / CPR;       // key groups per warp
     constexpr int NG = (kDecodeThreads / 32) * GPW;
+    static_assert(NG == decode_groups<D>(), "group count");
+    constexpr int CH = kStageRows<D>;   // key rows per stage
+    constexpr int ROWB = D * 2;         // bytes per row
     const int b = blockIdx.z, h = blockIdx.y, split = blockIdx.x;
     const int64_t bh = (int64_t)b * H + h;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int sub = lane % CPR;
-    const int grp_in_warp = lane / CPR;
 
     const int32_t R = ring_len[b], fill = win_fill[b], widx = win_idx[b];
     int32_t Tw = 0;
     float2* ml = ws_ml + bh * n_splits + split;
     float* wo = ws_o + (bh * n_splits + split) * D;
-    if (!decode_state_ok(R, fill, widx, ks, n_windows, W, C_ring, C_win, &Tw)) {
-        if (split == 0 && h == 0 && tid == 0) report(status, FOCUS_ERR_CAPACITY);
+    const bool state_ok = decode_state_ok(R, fill, widx, ks, n_windows, W, C_ring, C_win, &Tw);
+    const int64_t total = (int64_t)R + fill + 1;
+    const int64_t s0 = (int64_t)split * kDecodeChunk;
+    const int64_t s1 = min(total, s0 + kDecodeChunk);
+    if (!state_ok || s0 >= s1) {
+        if (!state_ok && split == 0 && h == 0 && tid == 0) report(status, FOCUS_ERR_CAPACITY);
         for (int c = tid; c < D; c += blockDim.x) wo[c] = 0.f;
         if (tid == 0) *ml = make_float2(-INFINITY, 0.f);
         return;
     }
-    const int64_t total = (int64_t)R + fill + 1;
-    const int64_t s0 = (int64_t)split * kDecodeChunk;
-    const int64_t s1 = min(total, s0 + kDecodeChunk);
-
     if (split == 0 && tid < CPR) {      // append the new row to the window buffer
         win_k[(bh * C_win + fill) * CPR + tid] = k_new[bh * CPR + tid];
         win_v[(bh * C_win + fill) * CPR + tid] = v_new[bh * CPR + tid];
     }
 
+    extern __shared__ __align__(128) unsigned char smem[];
+    uint8_t* sK = smem;                                   // [kStages][CH][D] bf16
+    uint8_t* sV = smem + kStages * CH * ROWB;             // [kStages][CH][D] bf16
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + 2 * kStages * CH * ROWB);
+    uint64_t* empty = full + kStages;
+    float* sm_m = reinterpret_cast<float*>(empty + kStages);
+    float* sm_l = sm_m + NG;
+    float* sm_acc = sm_l + NG;                            // [NG][D]
+    __shared__ int32_t abort_flag;
+    const int n_chunks = (int)((s1 - s0 + CH - 1) / CH);
+
+    if (tid == 0) {
+        for (int i = 0; i < kStages; ++i) {
+            mbar_init(smem_addr(&full[i]), 1);
+            mbar_init(smem_addr(&empty[i]), kDecodeThreads / 32);
+        }
+        abort_flag = 0;
+        fence_barrier_init();
+    }
+    __syncthreads();
+
+    if (warp == kDecodeThreads / 32) {
+        // ------------------------------------------------ producer
+        if (lane == 0) {
+            const uint8_t* rk = reinterpret_cast<const uint8_t*>(ring_k) + bh * (int64_t)C_ring * ROWB;
+            const uint8_t* rv = reinterpret_cast<const uint8_t*>(ring_v) + bh * (int64_t)C_ring * ROWB;
+            const uint8_t* wk = reinterpret_cast<const uint8_t*>(win_k) + bh * (int64_t)C_win * ROWB;
+            const uint8_t* wv = reinterpret_cast<const uint8_t*>(win_v) + bh * (int64_t)C_win * ROWB;
+            const uint8_t* nk = reinterpret_cast<const uint8_t*>(k_new) + bh * ROWB;
+            const uint8_t* nv = reinterpret_cast<const uint8_t*>(v_new) + bh * ROWB;
+            int issued = 0;
+            for (int c = 0; c < n_chunks; ++c) {
+                const int st = c % kStages, use = c / kStages;
+                if (use > 0 && !mbar_wait(smem_addr(&empty[st]), (use - 1) & 1, kWaitNs)) {
+                    report(status, FOCUS_ERR_TIMEOUT);
+                    atomicExch(&abort_flag, 1);
+                    break;
+                }
+                const int64_t k0 = s0 + (int64_t)c * CH, k1 = min(s1, k0 + CH);
+                const uint32_t bar = smem_addr(&full[st]);
+                mbar_expect_tx(bar, (uint32_t)((k1 - k0) * ROWB * 2));
+                const uint32_t dk = smem_addr(sK + st * CH * ROWB), dv = smem_addr(sV + st * CH * ROWB);
+                int64_t a = k0, e = min(k1, (int64_t)R);               // ring rows
+                if (a < e) {
+                    bulk_load(dk, rk + a * ROWB, (uint32_t)((e - a) * ROWB), bar);
+                    bulk_load(dv, rv + a * ROWB, (uint32_t)((e - a) * ROWB), bar);
+                }
+                a = max(k0, (int64_t)R);
+                e = min(k1, (int64_t)R + fill);                        // current-window rows
+                if (a < e) {
+                    const uint32_t off = (uint32_t)((a - k0) * ROWB);
+                    bulk_load(dk + off, wk + (a - R) * ROWB, (uint32_t)((e - a) * ROWB), bar);
+                    bulk_load(dv + off, wv + (a - R) * ROWB, (uint32_t)((e - a) * ROWB), bar);
+                }
+                if (k1 == total) {                                      // the new row itself
+                    const uint32_t off = (uint32_t)((total - 1 - k0) * ROWB);
+                    bulk_load(dk + off, nk, ROWB, bar);
+                    bulk_load(dv + off, nv, ROWB, bar);
+                }
+                issued = c + 1;
+            }
+            for (int c = max(0, issued - kStages); c < issued; ++c)    // drain before exit
+                mbar_wait(smem_addr(&full[c % kStages]), (c / kStages) & 1, kWaitNs);
+        }
+        __syncthreads();
+        return;
+    }
+
+    // ---------------------------------------------------- consumers
+    const int sub = lane % CPR;
+    const int grp = warp * GPW + lane / CPR;
     float qf[8];
     bf16x8_to_f32(q[bh * CPR + sub], qf);
 #pragma unroll
     for (int e = 0; e < 8; ++e) qf[e] *= scale_log2;
-
     float m = -INFINITY, l = 0.f, acc[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) acc[e] = 0.f;
 
-    const uint4* rk = ring_k + bh * (int64_t)C_ring * CPR + sub;
-    const uint4* rv = ring_v + bh * (int64_t)C_ring * CPR + sub;
-    const uint4* wk = win_k + bh * (int64_t)C_win * CPR + sub;
-    const uint4* wv = win_v + bh * (int64_t)C_win * CPR + sub;
-    const uint4* nk = k_new + bh * CPR + sub;
-    const uint4* nv = v_new + bh * CPR + sub;
-
-    // Warp-uniform loop: every lane runs the same trip count so the shuffles
-    // below always have the full warp.
-    for (int64_t wbase = s0 + warp * GPW; wbase < s1; wbase += (int64_t)NG * kUnroll) {
-        uint4 kr[kUnroll], vr[kUnroll];
-        float s[kUnroll];
-#pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
-            const int64_t j = wbase + grp_in_warp + (int64_t)u * NG;
-            if (j < s1) {
-                const uint4 *kp, *vp;
-                if (j < R) { kp = rk + j * CPR; vp = rv + j * CPR; }
-                else if (j < (int64_t)R + fill) { kp = wk + (j - R) * CPR; vp = wv + (j - R) * CPR; }
-                else { kp = nk; vp = nv; }
-                kr[u] = __ldg(kp);
-                vr[u] = __ldg(vp);
-            } else {
-                kr[u] = make_uint4(0, 0, 0, 0);
-                vr[u] = make_uint4(0, 0, 0, 0);
-            }
+    for (int c = 0; c < n_chunks; ++c) {
+        const int st = c % kStages;
+        if (!mbar_wait(smem_addr(&full[st]), (c / kStages) & 1, kWaitNs) || abort_flag) {
+            report(status, FOCUS_ERR_TIMEOUT);
+            break;
         }
+        const int nrow = (int)min((int64_t)CH, s1 - (s0 + (int64_t)c * CH));
+        const uint8_t* kb = sK + st * CH * ROWB + sub * 16;
+        const uint8_t* vb = sV + st * CH * ROWB + sub * 16;
+        constexpr int U = CH / NG;
+        float s[U];
+        uint4 vr[U];
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
+        for (int u = 0; u < U; ++u) {
+            const int r = grp + u * NG;
+            const bool ok = r < nrow;
+            const uint4 kr = ok ? *reinterpret_cast<const uint4*>(kb + r * ROWB) : make_uint4(0, 0, 0, 0);
+            vr[u] = ok ? *reinterpret_cast<const uint4*>(vb + r * ROWB) : make_uint4(0, 0, 0, 0);
             float kf[8];
-            bf16x8_to_f32(kr[u], kf);
+            bf16x8_to_f32(kr, kf);
             float d0 = 0.f;
 #pragma unroll
             for (int e = 0; e < 8; ++e) d0 = fmaf(qf[e], kf[e], d0);
             s[u] = d0;
         }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_addr(&empty[st]));     // this warp is done with the stage
 #pragma unroll
         for (int off = CPR / 2; off >= 1; off >>= 1) {
 #pragma unroll
-            for (int u = 0; u < kUnroll; ++u) s[u] += __shfl_xor_sync(0xffffffffu, s[u], off);
+            for (int u = 0; u < U; ++u) s[u] += __shfl_xor_sync(0xffffffffu, s[u], off);
         }
         float mb = -INFINITY;
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
-            const int64_t j = wbase + grp_in_warp + (int64_t)u * NG;
-            if (j >= s1) s[u] = -INFINITY;
+        for (int u = 0; u < U; ++u) {
+            if (grp + u * NG >= nrow) s[u] = -INFINITY;
             mb = fmaxf(mb, s[u]);
         }
         const float mn = fmaxf(m, mb);
         if (mn == -INFINITY) continue;
-        const float corr = exp2f(m - mn);
-        l *= corr;
+        if (mn > m) {
+            const float corr = ex2_approx(m - mn);
+            l *= corr;
 #pragma unroll
-        for (int e = 0; e < 8; ++e) acc[e] *= corr;
+            for (int e = 0; e < 8; ++e) acc[e] *= corr;
+            m = mn;
+        }
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
-            const float p = exp2f(s[u] - mn);
+        for (int u = 0; u < U; ++u) {
+            const float p = ex2_approx(s[u] - m);
             l += p;
             float vf[8];
             bf16x8_to_f32(vr[u], vf);
 #pragma unroll
             for (int e = 0; e < 8; ++e) acc[e] = fmaf(p, vf[e], acc[e]);
         }
-        m = mn;
     }
 
-    __shared__ float sm_m[NG], sm_l[NG];
-    __shared__ float sm_acc[NG][D];
-    const int grp = warp * GPW + grp_in_warp;
     if (sub == 0) { sm_m[grp] = m; sm_l[grp] = l; }
 #pragma unroll
-    for (int e = 0; e < 8; ++e) sm_acc[grp][sub * 8 + e] = acc[e];
-    __syncthreads();
+    for (int e = 0; e < 8; ++e) sm_acc[grp * D + sub * 8 + e] = acc[e];
+    asm volatile("bar.sync 1, %0;" ::"n"(kDecodeThreads));       // consumers only
     if (tid < D) {
         float M = -INFINITY;
 #pragma unroll
@@ -175,14 +252,15 @@ __global__ void __launch_bounds__(kDecodeThreads) decode_split_kernel(
         if (M != -INFINITY) {
 #pragma unroll
             for (int g = 0; g < NG; ++g) {
-                const float f = exp2f(sm_m[g] - M);
+                const float f = ex2_approx(sm_m[g] - M);
                 L = fmaf(sm_l[g], f, L);
-                A = fmaf(sm_acc[g][tid], f, A);
+                A = fmaf(sm_acc[g * D + tid], f, A);
             }
         }
         wo[tid] = A;
         if (tid == 0) *ml = make_float2(M, L);
     }
+    __syncthreads();
 }
 
 template <int D>
@@ -224,7 +302,10 @@ cudaError_t launch_decode_d(const focus_cache& c, const void* q, const void* k_n
     float2* ws_ml = reinterpret_cast<float2*>(workspace);
     float* ws_o = reinterpret_cast<float*>(ws_ml + (int64_t)c.B * c.H * ns);
     dim3 grid(ns, c.H, c.B);
-    decode_split_kernel<D><<<grid, kDecodeThreads, 0, stream>>>(
+    constexpr int smem = decode_smem_bytes<D>();
+    cudaError_t e0 = cudaFuncSetAttribute(decode_split_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e0 != cudaSuccess) return e0;
+    decode_split_kernel<D><<<grid, kDecodeThreads + 32, smem, stream>>>(
         (const uint4*)c.ring_k, (const uint4*)c.ring_v, (uint4*)c.win_k, (uint4*)c.win_v, c.ring_len,
         c.win_fill, c.win_idx, c.k_per_window, c.n_windows, c.W, c.H, c.C_ring, c.C_win, (const uint4*)q,
         (const uint4*)k_new, (const uint4*)v_new, scale * 1.4426950408889634f, ws_ml, ws_o, ns, status);
