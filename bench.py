@@ -66,6 +66,8 @@ def kernel_traffic(kernel_key: str, source: str):
     try:
         with open(p) as f:
             d = json.load(f)[kernel_key]
+        if d.get("source") != source:
+            return None
         with open(os.path.join(ROOT, source), "rb") as f:
             sha = hashlib.sha256(f.read()).hexdigest()[:16]
         return float(d["bytes_per_launch"]) if d.get("source_sha") == sha else None
@@ -307,6 +309,63 @@ def run_prefill_leg(args, cfg, world, rank, local):
     return res
 
 
+def run_stream_leg(args, cfg, world, rank, local):
+    """Streaming prefill (App. A.2): for each window in order, focus_attn_prefill
+    over that window against the ring, then focus_kv_compact of that window.
+    Each window's Q/K/V is one of a pool of seeded windows (cycled)."""
+    import torch
+    from paper_2511_14694_gb300 import focus, inputs, pipeline
+
+    B, N, W, H, d, P = cfg["B"], cfg["N"], cfg["W"], cfg["H"], cfg["d"], cfg["pool"]
+    M = -(-N // W)
+    k_s = inputs.k_schedule(M, cfg["k"], seed=inputs.DEFAULT_SEED)
+    dev = torch.device("cuda", local)
+    L = focus.layout(N, W, k_s, device=dev)
+    off = L["win_off_host"]
+    Tw = int(np.diff(off).max())
+    if not (np.diff(off) == Tw).all():
+        raise ValueError("the streaming leg expects windows of equal augmented size")
+    pq, pk, pv = inputs.qkv((P, B, H, Tw, d), std=cfg["std"], seed=inputs.DEFAULT_SEED + rank, device=dev)
+    cache = focus.Cache(B, H, d, C_ring=max(L["R"], 1), device=dev)
+    outs = [torch.empty((B, H, Tw, d), dtype=torch.bfloat16, device=dev) for _ in range(2)]
+    lses = [torch.empty((B, H, Tw), dtype=torch.float32, device=dev) for _ in range(2)]
+    stream = torch.cuda.current_stream(dev)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(M)]
+
+    def step(timed=False):
+        for w in range(M):
+            if timed:
+                evs[w][0].record(stream)
+            focus.attn_prefill(cache, pq[w % P], pk[w % P], pv[w % P], L, w, w + 1, o=outs[w % 2], lse=lses[w % 2],
+                               stream=stream, flags=args.prefill_flags)
+            if timed:
+                evs[w][1].record(stream)
+            focus.kv_compact_bulk(cache, pk[w % P], pv[w % P], L, w, w + 1, src_row0=int(off[w]), stream=stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize(dev)
+    assert focus.device_status(clear=True) == 0
+    pairs = visible_pairs(off, L["ring_off_host"])
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    attn_ms = 0.0
+    barrier(world)
+    with ClockSampler(local) as clk:
+        t0.record(stream)
+        for _ in range(args.steps):
+            step(timed=True)
+            torch.cuda.synchronize(dev)
+            attn_ms += sum(a.elapsed_time(b) for a, b in evs)
+        t1.record(stream)
+        torch.cuda.synchronize(dev)
+    barrier(world)
+    assert focus.device_status(clear=True) == 0
+    step_ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, world)
+    return dict(step_ms=step_ms, attn_ms=attn_ms / args.steps, flops_per_step=4.0 * d * H * B * pairs, pairs=pairs,
+                T=L["T"], R=L["R"], clocks=clk.summary(), launches=2 * M * args.steps, e2e=None, host_sample=None,
+                per_launch_ms=attn_ms / args.steps / M)
+
+
 def run_decode_leg(args, cfg, world, rank, local):
     import torch
     from paper_2511_14694_gb300 import focus, inputs
@@ -385,16 +444,28 @@ def run_focus(args, world, rank, local):
     torch.cuda.set_device(local)
     peaks, peaks_src = load_peaks()
     cfg = WORKLOADS[args.workload]
-    pre = run_prefill_leg(args, cfg, world, rank, local)
+    if args.no_prefill:          # decode leg alone (profiling runs)
+        dec = run_decode_leg(args, WORKLOADS[args.decode_workload], world, rank, local)
+        if rank == 0:
+            print(json.dumps({"decode_workload": args.decode_workload, "leg_ms": dec["leg_ms"],
+                              "decode_call_ms": dec["decode_kernels_ms"] / dec["steps"],
+                              "GBps": dec["bytes_leg"] / (dec["decode_kernels_ms"] / 1e3) / 1e9}), flush=True)
+        return
+    if cfg["mode"] == "stream":
+        pre = run_stream_leg(args, cfg, world, rank, local)
+    else:
+        pre = run_prefill_leg(args, cfg, world, rank, local)
     dec = None
     if not args.no_decode:
-        dec = run_decode_leg(args, WORKLOADS["decode_1mb_b64_h32_d128"], world, rank, local)
+        dec = run_decode_leg(args, WORKLOADS[args.decode_workload], world, rank, local)
     if rank != 0:
         return
     N_tot = world * cfg["B"] * cfg["N"]
     value = N_tot / (pre["step_ms"] / 1e3)
     achieved = pre["flops_per_step"] / (pre["attn_ms"] / 1e3) / 1e12
-    traffic = kernel_traffic("prefill_attention", "paper_2511_14694_gb300/csrc/prefill_mma.cu")
+    traffic = None if args.legacy else kernel_traffic("prefill_attention", "paper_2511_14694_gb300/csrc/prefill_tc.cu")
+    if traffic is not None and cfg is not WORKLOADS["prefill_128kb_h32_d128"]:
+        traffic = None            # the committed counters are for the 128 kb workload only
     line = {
         "metric": METRIC,
         "value": value, "unit": "nt/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
@@ -402,16 +473,24 @@ def run_focus(args, world, rank, local):
         "dtype": "bf16", "data": "synthetic (seeded N(0,1)/sqrt(d) bf16 Q/K/V, uniform A/C/G/T ids)",
         "config": {"workload": args.workload, "B": cfg["B"], "N": cfg["N"], "W": cfg["W"], "k": list(cfg["k"]),
                    "H": cfg["H"], "d": cfg["d"], "T_augmented": pre["T"], "R_retained": pre["R"],
-                   "step": "focus_layout + focus_kv_compact(bulk) + focus_attn_prefill(masked-parallel)",
-                   "l2": "inputs larger than L2 (Q/K/V %.2f GB per step)" % (3 * pre["T"] * cfg["H"] * cfg["d"] * 2 / 1e9),
+                   "step": ("per window: focus_attn_prefill(window) + focus_kv_compact(window); all windows"
+                            if cfg["mode"] == "stream" else
+                            "focus_layout + focus_kv_compact(bulk) + focus_attn_prefill(masked-parallel)"),
+                   "l2": ("inputs larger than L2 (pool of %d windows' Q/K/V %.2f GB, ring %.2f GB)" % (
+                       cfg.get("pool", 0), 3 * cfg.get("pool", 0) * cfg["B"] * cfg["H"] * (pre["T"] // max(1, -(-cfg["N"] // cfg["W"]))) * cfg["d"] * 2 / 1e9,
+                       2 * cfg["B"] * cfg["H"] * pre["R"] * cfg["d"] * 2 / 1e9) if cfg["mode"] == "stream" else
+                          "inputs larger than L2 (Q/K/V %.2f GB per step)" % (3 * cfg["B"] * pre["T"] * cfg["H"] * cfg["d"] * 2 / 1e9)),
                    "prefill_kernel": "legacy mma.sync" if args.prefill_flags & 1 else "default"},
         "augmented_tokens_per_s": world * cfg["B"] * pre["T"] / (pre["step_ms"] / 1e3),
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
                      "frac": achieved / peaks["bf16_tflops"], "traffic": traffic,
                      "peak_source": f"{peaks_src} bf16 dense burst",
                      "frac_of_sustained": achieved / peaks["bf16_tflops_sustained"],
-                     "kernel": "prefill attention", "flop_per_launch": pre["flops_per_step"],
-                     "visible_pairs": pre["pairs"], "avg_launch_ms": pre["attn_ms"]},
+                     "kernel": "prefill attention",
+                     "flop_per_launch": pre["flops_per_step"] / (pre["launches"] // (2 * args.steps)
+                                                                 if cfg["mode"] == "stream" else 1),
+                     "visible_pairs": pre["pairs"], "avg_launch_ms": pre.get("per_launch_ms", pre["attn_ms"]),
+                     "launches_per_step": (pre["launches"] // (2 * args.steps)) if cfg["mode"] == "stream" else 1},
         "clocks": pre["clocks"],
         "e2e": pre["e2e"],
         "gpu_launches": pre["launches"],
@@ -419,14 +498,15 @@ def run_focus(args, world, rank, local):
     if dec is not None:
         gbs = dec["bytes_leg"] / (dec["decode_kernels_ms"] / 1e3) / 1e9
         line["decode"] = {
-            "workload": "decode_1mb_b64_h32_d128", "value": world * dec["B"] * dec["steps"] / (dec["leg_ms"] / 1e3),
+            "workload": args.decode_workload, "value": world * dec["B"] * dec["steps"] / (dec["leg_ms"] / 1e3),
             "unit": "tokens/s", "ms_per_step": dec["leg_ms"] / dec["steps"],
             "step": "focus_attn_decode + focus_kv_compact(window)",
             "roofline": {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                          "frac": gbs / peaks["hbm_gbs"], "frac_of_nominal": gbs / NOMINAL_HBM_GBS,
                          "peak_source": f"{peaks_src} copy bandwidth", "bytes_per_step": dec["bytes_leg"] / dec["steps"],
                          "avg_decode_call_ms": dec["decode_kernels_ms"] / dec["steps"],
-                         "traffic": kernel_traffic("decode_split", "paper_2511_14694_gb300/csrc/decode.cu")},
+                         "traffic": (kernel_traffic("decode_split", "paper_2511_14694_gb300/csrc/decode.cu")
+                                     if args.decode_workload == "decode_1mb_b64_h32_d128" else None)},
             "clocks": dec["clocks"],
         }
         line["decode"]["gpu_launches"] = dec["launches"]
@@ -485,6 +565,8 @@ def main():
     ap.add_argument("--workload", default="prefill_128kb_h32_d128")
     ap.add_argument("--decode-reps", type=int, default=2)
     ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-prefill", action="store_true", help="run only the decode leg (profiling)")
+    ap.add_argument("--decode-workload", default="decode_1mb_b64_h32_d128")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0)

@@ -17,6 +17,9 @@ WORKLOADS = {
     # plus up to 1,010 current-window rows per head, batch 64, 256 steps
     "decode_1mb_b64_h32_d128": dict(mode="decode", B=64, R=10_000, W=1_000, k=(100,), H=32, d=128,
                                     steps=256, std=1.0),
+    # the same cache shape at batch 8, for profiler captures (about 1.5 GB resident)
+    "decode_1mb_b8_h32_d128": dict(mode="decode", B=8, R=10_000, W=1_000, k=(100,), H=32, d=128,
+                                   steps=256, std=1.0),
     # randomized compression schedule: k per window from {10, 25, 50, 100, 200}
     "prefill_256kb_ksweep_h32_d128": dict(mode="prefill", B=1, N=256_000, W=1_000,
                                           k=(10, 25, 50, 100, 200), H=32, d=128,

@@ -311,3 +311,39 @@ def test_full_size_decode_sampled():
             assert_attn_close(o[b, h][None], lse[b, h][None], o_ref, lse_ref, f"decode b={b} h={h} step={step}")
     assert (cache.ring_len.cpu().numpy()[:4] == R + W // cfg["k"][0]).all()
     assert (cache.win_fill.cpu().numpy()[:4] == 2).all()
+
+
+def test_full_size_streaming_sampled():
+    """Batch 4, N = 1 Mb, W = 1,000, k = 100, 32 heads, d = 128: one prefill call and
+    one compaction per window (App. A.2). Sampled windows of two heads are checked
+    against the oracle's sequential form; the final ring (10,000 rows) bit-exactly."""
+    from paper_2511_14694_gb300.workloads import WORKLOADS
+    cfg = WORKLOADS["stream_1mb_b4_h32_d128"]
+    B, N, W, H, d, P = cfg["B"], cfg["N"], cfg["W"], cfg["H"], cfg["d"], cfg["pool"]
+    M = -(-N // W)
+    L = focus.layout(N, W, [cfg["k"][0]])
+    off = L["win_off_host"]
+    Tw = int(off[1] - off[0])
+    pq, pk, pv = inputs.qkv((P, B, H, Tw, d), std=cfg["std"], seed=inputs.DEFAULT_SEED, device="cuda")
+    cache = focus.Cache(B, H, d, C_ring=L["R"])
+    want = [0, 1, 437, 998, 999]
+    b, heads = 1, [0, 17]
+    got = {}
+    for w in range(M):
+        o, lse = pipeline.prefill_window(cache, pq[w % P], pk[w % P], pv[w % P], L, w)
+        if w in want:
+            got[w] = (o[b, heads].cpu(), lse[b, heads].cpu())
+    torch.cuda.synchronize()
+    assert (cache.ring_len.cpu().numpy() == L["R"]).all()
+    ref_L = fo.layout(N, W, [cfg["k"][0]])
+    want_mask = np.zeros(M, np.uint8)
+    want_mask[want] = 1
+    for i, h in enumerate(heads):
+        full = [torch.cat([t[w % P, b, h] for w in range(M)]).cpu() for t in (pq, pk, pv)]
+        o_ref, lse_ref, rk, rv = fo.prefill_sequential(*full, ref_L["win_off"], ref_L["kind"], 1.0 / math.sqrt(d),
+                                                       want=want_mask)
+        for w in want:
+            a, e = int(off[w]), int(off[w + 1])
+            assert_attn_close(got[w][0][i], got[w][1][i], o_ref[a:e], lse_ref[a:e], f"stream w={w} h={h}")
+        assert np.array_equal(bits(cache.ring_k[b, h]), rk)
+        assert np.array_equal(bits(cache.ring_v[b, h]), rv)
