@@ -266,28 +266,45 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
                 for (int c = 0; c < BN; ++c)
                     if (c > r) s[c] = -INFINITY;
             }
-            float mt = -INFINITY;
+            // row max: four independent chains of three-input max (depth 16, not 128)
+            float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-            for (int c = 0; c < BN; ++c) mt = fmaxf(mt, s[c]);
+            for (int c = 0; c < BN; c += 8) {
+                mx[0] = max3f(mx[0], s[c + 0], s[c + 1]);
+                mx[1] = max3f(mx[1], s[c + 2], s[c + 3]);
+                mx[2] = max3f(mx[2], s[c + 4], s[c + 5]);
+                mx[3] = max3f(mx[3], s[c + 6], s[c + 7]);
+            }
+            const float mt = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
             const float m_new = fmaxf(m_run, mt * scale_log2);
             const bool need = m_new > m_run + kRescaleThreshold;
             const bool any_need = __any_sync(0xffffffffu, need);
             const float factor = need ? ex2_approx(m_run - m_new) : 1.f;
             if (need) m_run = m_new;
             l_run *= factor;
-            const float neg_m = -m_run;
-            float lsum = 0.f;
+            // p = 2^(s * scale_log2 - m): packed FMA on pairs, ex2 per element, row sum in
+            // four packed partial sums (independent chains)
+            const uint64_t sc2 = f2_pack(scale_log2, scale_log2), nm2 = f2_pack(-m_run, -m_run);
+            uint64_t acc2[4] = {0, 0, 0, 0};
 #pragma unroll
             for (int h2 = 0; h2 < 2; ++h2) {
                 uint32_t pk[32];
 #pragma unroll
                 for (int i = 0; i < 32; ++i) {
-                    const float p0 = ex2_approx(fmaf(s[h2 * 64 + 2 * i], scale_log2, neg_m));
-                    const float p1 = ex2_approx(fmaf(s[h2 * 64 + 2 * i + 1], scale_log2, neg_m));
-                    lsum += p0 + p1;
+                    float x0, x1;
+                    f2_unpack(f2_fma(f2_pack(s[h2 * 64 + 2 * i], s[h2 * 64 + 2 * i + 1]), sc2, nm2), x0, x1);
+                    const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+                    acc2[i & 3] = f2_add(acc2[i & 3], f2_pack(p0, p1));
                     pk[i] = pack_bf16x2(p0, p1);
                 }
                 tmem_st32(s_addr + h2 * 32, pk);
+            }
+            float lsum = 0.f;
+#pragma unroll
+            for (int a = 0; a < 4; ++a) {
+                float lo, hi;
+                f2_unpack(acc2[a], lo, hi);
+                lsum += lo + hi;
             }
             l_run += lsum;
             // Lazy rescale of O_t (written by PV_t(j-1), which completed before S_t(j)
