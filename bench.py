@@ -137,12 +137,19 @@ class ClockSampler:
 # ----------------------------------------------------------------------------- distributed
 
 def dist_setup():
+    """One process per GPU (torch.distributed.run sets RANK / LOCAL_RANK /
+    WORLD_SIZE / MASTER_*). NCCL when CUDA is available, gloo otherwise; the
+    process group carries only the timing barrier and the max over ranks."""
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if world > 1:
+        import torch
         import torch.distributed as dist
-        dist.init_process_group("nccl")
+        backend = os.environ.get("FOCUS_DIST_BACKEND") or ("nccl" if torch.cuda.is_available() else "gloo")
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
     return world, rank, local
 
 
@@ -157,9 +164,16 @@ def max_over_ranks(x: float, world: int) -> float:
         return x
     import torch
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def weak_scaling_value(units_per_rank: float, world: int, max_seconds: float) -> float:
+    """Whole-job throughput: every rank processes its own units (no exchange), so
+    the job's units are world x units_per_rank, over the slowest rank's time."""
+    return world * units_per_rank / max_seconds
 
 
 # ----------------------------------------------------------------------------- oracle (CPU baseline)
@@ -460,8 +474,7 @@ def run_focus(args, world, rank, local):
         dec = run_decode_leg(args, WORKLOADS[args.decode_workload], world, rank, local)
     if rank != 0:
         return
-    N_tot = world * cfg["B"] * cfg["N"]
-    value = N_tot / (pre["step_ms"] / 1e3)
+    value = weak_scaling_value(cfg["B"] * cfg["N"], world, pre["step_ms"] / 1e3)
     achieved = pre["flops_per_step"] / (pre["attn_ms"] / 1e3) / 1e12
     traffic = None if args.legacy else kernel_traffic("prefill_attention", "paper_2511_14694_gb300/csrc/prefill_tc.cu")
     if traffic is not None and cfg is not WORKLOADS["prefill_128kb_h32_d128"]:

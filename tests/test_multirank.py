@@ -1,0 +1,69 @@
+"""The N > 1 path of bench.py on CPU: two ranks over gloo (127.0.0.1).
+
+The path shards over batch and heads with no data-path exchange (each rank runs
+its own replica of the workload on its own seeded inputs), so what crosses ranks
+is only the timing barrier and the max over ranks; the tests cover those and
+the reference arm's rank-0-only output."""
+import json
+import os
+import socket
+import subprocess
+import sys
+
+import pytest
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, q):
+    os.environ.update(RANK=str(rank), LOCAL_RANK=str(rank), WORLD_SIZE=str(world), MASTER_ADDR="127.0.0.1",
+                      MASTER_PORT=str(port), FOCUS_DIST_BACKEND="gloo")
+    import bench
+    w, r, _ = bench.dist_setup()
+    bench.barrier(w)
+    m = bench.max_over_ranks(10.0 + r, w)               # rank r "took" 10 + r ms
+    v = bench.weak_scaling_value(128_000, w, m / 1e3)
+    q.put((r, w, m, v))
+    import torch.distributed as dist
+    dist.destroy_process_group()
+
+
+def test_barrier_and_max_over_ranks_gloo():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_rank_main, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = sorted(q.get(timeout=120) for _ in range(2))
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    assert [r for r, *_ in res] == [0, 1]
+    for r, w, m, v in res:
+        assert w == 2 and m == 11.0                      # every rank sees the slowest rank's time
+        assert v == pytest.approx(2 * 128_000 / 0.011)   # whole-job units over the max time
+
+
+def test_reference_arm_two_ranks_prints_one_line():
+    port = _free_port()
+    env = dict(os.environ, FOCUS_DIST_BACKEND="gloo", OMP_NUM_THREADS="2")
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
+           "--master-addr", "127.0.0.1", "--master-port", str(port), "bench.py", "--impl", "reference",
+           "--gpus", "2", "--steps", "1", "--warmup", "0", "--cpu-budget", "1",
+           "--workload", "prefill_4kb_h4_d64"]
+    r = subprocess.run(cmd, cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1, r.stdout
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["value"] > 0
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["e2e"]["h2d_bytes_per_step"] == 0
