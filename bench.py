@@ -569,6 +569,71 @@ def run_reference(args, world, rank, local):
     print(json.dumps(line), flush=True)
 
 
+def run_memory_report(args, world, rank, local):
+    """Memory scaling with context length (the paper's Fig. "Scalability of memory
+    with context length", Sec. 4.5): peak device memory and time of a streaming
+    FOCUS prefill (one window's Q/K/V resident at a time, the retained ring
+    growing as N/k) against a full-cache causal prefill over the same N (Q/K/V
+    of all N rows resident), one attention layer, batch 1, 32 heads, d = 128."""
+    if rank != 0:
+        return
+    import torch
+    from paper_2511_14694_gb300 import focus, inputs
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    H, d, W, k = 32, 128, 1_000, 100
+    for N in [int(x) for x in args.memory_ns.split(",")]:
+        row = {"report": "memory_scaling", "N": N, "H": H, "d": d, "W": W, "k": k,
+               "kv_bytes_full": 2 * N * H * d * 2}
+        # FOCUS streaming: ring (retained summaries) + one window of Q/K/V/O at a time
+        torch.cuda.synchronize(dev)
+        torch.cuda.empty_cache()
+        torch.cuda.reset_peak_memory_stats(dev)
+        base = torch.cuda.memory_allocated(dev)
+        L = focus.layout(N, W, [k], device=dev)
+        off = L["win_off_host"]
+        Tw = int(np.diff(off).max())
+        row["kv_bytes_focus"] = 2 * (L["R"] + Tw) * H * d * 2
+        cache = focus.Cache(1, H, d, C_ring=max(L["R"], 1), device=dev)
+        q, kk, v = inputs.qkv((1, H, Tw, d), std=1 / math.sqrt(d), seed=1, device=dev)
+        o = torch.empty_like(q)
+        lse = torch.empty((1, H, Tw), dtype=torch.float32, device=dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for w in range(L["M"]):
+            a, e = int(off[w]), int(off[w + 1])
+            n = e - a
+            focus.attn_prefill(cache, q[:, :, :n].contiguous() if n != Tw else q, kk[:, :, :n].contiguous() if n != Tw else kk,
+                               v[:, :, :n].contiguous() if n != Tw else v, L, w, w + 1, o=o[:, :, :n].contiguous() if n != Tw else o,
+                               lse=lse[:, :, :n].contiguous() if n != Tw else lse)
+            focus.kv_compact_bulk(cache, kk[:, :, :n].contiguous() if n != Tw else kk,
+                                  v[:, :, :n].contiguous() if n != Tw else v, L, w, w + 1, src_row0=a)
+        e1.record()
+        torch.cuda.synchronize(dev)
+        assert focus.device_status(clear=True) == 0
+        row["focus_peak_bytes"] = torch.cuda.max_memory_allocated(dev) - base
+        row["focus_ms"] = e0.elapsed_time(e1)
+        del cache, q, kk, v, o, lse, L
+        # full cache: plain causal attention over all N rows (k = 0, one window)
+        if N <= args.memory_full_max:
+            torch.cuda.synchronize(dev)
+            torch.cuda.empty_cache()
+            torch.cuda.reset_peak_memory_stats(dev)
+            base = torch.cuda.memory_allocated(dev)
+            Lc = focus.layout(N, N, [0], device=dev)
+            cc = focus.Cache(1, H, d, C_ring=0, device=dev)
+            q, kk, v = inputs.qkv((1, H, N, d), std=1 / math.sqrt(d), seed=1, device=dev)
+            e0.record()
+            focus.attn_prefill(cc, q, kk, v, Lc)
+            e1.record()
+            torch.cuda.synchronize(dev)
+            assert focus.device_status(clear=True) == 0
+            row["full_peak_bytes"] = torch.cuda.max_memory_allocated(dev) - base
+            row["full_ms"] = e0.elapsed_time(e1)
+            del cc, q, kk, v, Lc
+        print(json.dumps(row), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -586,11 +651,17 @@ def main():
     ap.add_argument("--no-clock-wait", action="store_true",
                     help="do not extend the load after a short timed region (profiling runs)")
     ap.add_argument("--legacy", action="store_true", help="time the legacy mma.sync prefill kernel")
+    ap.add_argument("--memory-report", action="store_true",
+                    help="peak memory and time vs context length, FOCUS streaming vs full-cache causal")
+    ap.add_argument("--memory-ns", default="16000,32000,64000,128000,256000,512000,1000000")
+    ap.add_argument("--memory-full-max", type=int, default=256_000)
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     args.prefill_flags = 1 if args.legacy else 0
     world, rank, local = dist_setup()
-    if args.impl == "reference":
+    if args.memory_report:
+        run_memory_report(args, world, rank, local)
+    elif args.impl == "reference":
         run_reference(args, world, rank, local)
     else:
         run_focus(args, world, rank, local)
