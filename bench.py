@@ -184,7 +184,7 @@ def oracle_prefill_sample(cfg, L_host, q, k, v, budget_s=12.0, max_windows=None)
     the whole workload by visible pairs. Returns (seconds for the full workload,
     description, cores)."""
     from oracle import focus_oracle as fo
-    win_off, ring_off, kind = L_host["win_off"], L_host["ring_off"], L_host["kind"]
+    win_off, ring_off, keep = L_host["win_off"], L_host["ring_off"], L_host["keep"]
     M = win_off.size - 1
     d = cfg["d"]
     total_pairs = visible_pairs(win_off, ring_off) * cfg["B"] * cfg["H"]
@@ -200,7 +200,7 @@ def oracle_prefill_sample(cfg, L_host, q, k, v, budget_s=12.0, max_windows=None)
         if max_windows:
             want[np.nonzero(want)[0][max_windows:]] = 0
         t0 = time.perf_counter()
-        fo.prefill_sequential(q[h], k[h], v[h], win_off, kind, 1.0 / math.sqrt(d), want=want)
+        fo.prefill_sequential(q[h], k[h], v[h], win_off, keep, 1.0 / math.sqrt(d), want=want)
         spent += time.perf_counter() - t0
         done_pairs += int(pairs_w[want.astype(bool)].sum())
         heads_done += 1
@@ -549,7 +549,7 @@ def run_reference(args, world, rank, local):
     L = fo.layout(N, W, k_s)
     # two heads of inputs, drawn with the same generator recipe on the CPU
     q, k, v = inputs.qkv((2, L["T"], d), std=cfg["std"], seed=inputs.DEFAULT_SEED, device="cpu")
-    hs = dict(win_off=L["win_off"], ring_off=L["ring_off"], kind=L["kind"])
+    hs = dict(win_off=L["win_off"], ring_off=L["ring_off"], keep=L["keep"])
     budget = max(2.0, args.cpu_budget / max(1, args.steps + args.warmup))
     for _ in range(args.warmup):
         oracle_prefill_sample(cfg, hs, q, k, v, budget_s=budget, max_windows=4)

@@ -11,7 +11,10 @@
  *   (a) the retained FOCUS K/V of all earlier windows and (b) the rows of
  *   window w up to and including itself (Eq. focus-attn's visible set and the
  *   context C(t) of App. A.1). After window w only its FOCUS K/V is kept
- *   (App. A, "KV compression and budget"; App. A.2 streaming inference).
+ *   (App. A, "KV compression and budget"; App. A.2 streaming inference),
+ *   optionally with a boundary tail: the window's last `tail` ordinary rows
+ *   (App. A, "plus a small boundary tail if required"). Kept rows form the
+ *   ring that every later window attends to.
  *
  * Conventions for every entry point
  *   - Ownership: the caller allocates and owns every buffer. Pointers named
@@ -86,23 +89,25 @@ focus_status focus_get_device_status(int32_t* host_status, int32_t clear, cudaSt
  *   n_windows   M; must equal ceil(N/W)
  *   h_k         HOST array [M]: cadence k_w >= 0 per window (0 = no summaries)
  *   flags       FOCUS_LAYOUT_CLOSE_TAIL or 0
- * Outputs (any may be NULL): *T augmented length N + sum_w B_w, *R summaries,
- * *max_rows the largest per-window augmented row count. */
+ *   tail        boundary tail: ordinary rows kept at the end of each window (>= 0; 0 = none)
+ * Outputs (any may be NULL): *T augmented length N + sum_w B_w, *R kept rows
+ * (sum_w B_w + min(tail, n_w)), *max_rows the largest per-window augmented row count. */
 focus_status focus_layout_size(int64_t n_nt, int32_t W, int32_t n_windows, const int32_t* h_k,
-                               uint32_t flags, int64_t* T, int64_t* R, int32_t* max_rows);
+                               uint32_t flags, int32_t tail, int64_t* T, int64_t* R, int32_t* max_rows);
 
 /* Device arrays written by focus_layout. All are caller-allocated. */
 typedef struct focus_layout_out {
     int64_t  T;          /* capacity/expected augmented length (from focus_layout_size) */
-    int64_t  R;          /* expected number of summaries (from focus_layout_size) */
+    int64_t  R;          /* expected number of kept rows (from focus_layout_size) */
     uint8_t* kind;       /* [T] 0 = base, 1 = FOCUS summary */
     int32_t* src;        /* [T] nucleotide index; a summary names the last base of its k-mer */
     int32_t* pos;        /* [T] position id (0-based augmented index) */
     int32_t* win;        /* [T] window id */
     uint8_t* tok;        /* [B][T] token ids (nt id 0..3, summary FOCUS_SUMMARY_TOKEN); may be NULL */
+    uint8_t* keep;       /* [T] 1 if KV retention keeps the row (summary or boundary-tail base); may be NULL */
     int32_t* win_off;    /* [M+1] first augmented row of each window; win_off[M] = T */
-    int32_t* ring_off;   /* [M+1] summaries before each window; ring_off[M] = R */
-    int32_t* sum_idx;    /* [R] augmented index of each summary, in order (the compaction gather list) */
+    int32_t* ring_off;   /* [M+1] kept rows before each window; ring_off[M] = R */
+    int32_t* sum_idx;    /* [R] augmented index of each kept row, in order (the compaction gather list) */
 } focus_layout_out;
 
 /* Device layout builder. d_k: DEVICE array [M] of cadences (same values as the
@@ -110,7 +115,7 @@ typedef struct focus_layout_out {
  * (may be NULL, then tok is not written). If the device-computed T or R differs
  * from out->T / out->R the device status word is set to FOCUS_ERR_LAYOUT. */
 focus_status focus_layout(int64_t n_nt, int32_t W, int32_t n_windows, const int32_t* d_k,
-                          uint32_t flags, int32_t B, const uint8_t* d_nt,
+                          uint32_t flags, int32_t tail, int32_t B, const uint8_t* d_nt,
                           const focus_layout_out* out, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------ */
@@ -131,6 +136,7 @@ typedef struct focus_cache {
     int32_t  W;               /* window length in bases */
     int32_t  B, H, d;
     int32_t  C_ring, C_win;   /* capacities in rows */
+    int32_t  tail;            /* boundary tail kept by window-mode compaction (>= 0) */
 } focus_cache;
 
 /* ------------------------------------------------------------------------ */
@@ -232,9 +238,10 @@ typedef struct focus_compact_args {
     int32_t     n_windows;    /* M (the offsets arrays hold M+1 entries) */
     int32_t     w_begin, w_end;   /* 0 <= w_begin <= w_end <= M */
     /* Window mode (src_k == NULL): for each sequence b whose window buffer is full
-     * (win_fill[b] == W + ceil(W / k_{win_idx[b]})), append that window's FOCUS rows
-     * to the ring at ring_len[b], advance ring_len[b], reset win_fill[b] to 0 and
-     * increment win_idx[b]. Sequences with a partly filled window are untouched. */
+     * (win_fill[b] == W + ceil(W / k_{win_idx[b]})), append that window's kept rows
+     * (its FOCUS rows and its last cache->tail bases, in augmented order) to the ring
+     * at ring_len[b], advance ring_len[b], reset win_fill[b] to 0 and increment
+     * win_idx[b]. Sequences with a partly filled window are untouched. */
 } focus_compact_args;
 
 focus_status focus_kv_compact(const focus_cache* cache, const focus_compact_args* args,

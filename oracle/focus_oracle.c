@@ -17,6 +17,11 @@
  *   - Softmax scale is a caller argument; LSE is the natural log of the sum of
  *     exponentials of the scaled scores.
  *
+ * KV retention keeps each window's FOCUS rows and, optionally, a boundary
+ * tail: the last `tail` ordinary (base) rows of the window (App. A, "plus a
+ * small boundary tail if required"; App. A.2). tail = 0 is the paper's default.
+ * A kept row is visible to every later window.
+ *
  * Every loop below runs in the order the paper states the operation; nothing is
  * blocked, fused or reordered.
  */
@@ -50,11 +55,15 @@ static int summary_after(int64_t o, int64_t n, int32_t k, int close_partial) {
     return (o == n - 1) && close_partial;
 }
 
+/* Is the base at in-window offset o of an n-base window in its boundary tail? */
+static int in_tail(int64_t o, int64_t n, int32_t tail) { return tail > 0 && o >= n - tail; }
+
 /* Sizes of the augmented layout. Returns T (augmented length) and writes R
- * (retained summaries after the last window). Returns -1 on bad arguments. */
+ * (rows retained after the last window: summaries plus boundary tails).
+ * Returns -1 on bad arguments. */
 int64_t fo_layout_size(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
-                       int32_t close_tail, int64_t* R_out) {
-    if (N < 0 || W <= 0) return -1;
+                       int32_t close_tail, int32_t tail, int64_t* R_out) {
+    if (N < 0 || W <= 0 || tail < 0) return -1;
     int64_t M_expect = (N + W - 1) / W;
     if (M != M_expect) return -1;
     int64_t T = 0, R = 0;
@@ -64,6 +73,7 @@ int64_t fo_layout_size(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
         int close = (w < M - 1) || close_tail;
         for (int64_t o = 0; o < n; ++o) {
             T += 1;
+            if (in_tail(o, n, tail)) R += 1;
             if (summary_after(o, n, k_sched[w], close)) { T += 1; R += 1; }
         }
     }
@@ -78,17 +88,18 @@ int64_t fo_layout_size(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
  *   win[t]   window id w
  *   tok[b*T + t]  nucleotide id nt[b*N + src] for bases, 4 for summaries
  *                 (written only when nt and tok are both non-NULL)
+ *   keep[t]  1 if KV retention keeps the row (a summary, or a boundary-tail base)
  * plus win_off[M+1] (first augmented index of each window, win_off[M] = T),
- * ring_off[M+1] (summaries retained before each window, ring_off[M] = R) and
- * sum_idx[R] (augmented index of each summary, in order).
+ * ring_off[M+1] (rows retained before each window, ring_off[M] = R) and
+ * sum_idx[R] (augmented index of each retained row, in order).
  * Returns T, or -1 on bad arguments. */
 int64_t fo_layout(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
-                  int32_t close_tail, int32_t B, const uint8_t* nt,
+                  int32_t close_tail, int32_t tail, int32_t B, const uint8_t* nt,
                   uint8_t* kind, int32_t* src, int32_t* pos, int32_t* win,
-                  uint8_t* tok, int32_t* win_off, int32_t* ring_off,
+                  uint8_t* tok, uint8_t* keep, int32_t* win_off, int32_t* ring_off,
                   int32_t* sum_idx) {
     int64_t R_total = 0;
-    int64_t T_total = fo_layout_size(N, W, M, k_sched, close_tail, &R_total);
+    int64_t T_total = fo_layout_size(N, W, M, k_sched, close_tail, tail, &R_total);
     if (T_total < 0) return -1;
     int64_t t = 0, r = 0;
     for (int32_t w = 0; w < M; ++w) {
@@ -100,11 +111,14 @@ int64_t fo_layout(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
         for (int64_t o = 0; o < n; ++o) {
             int64_t base = start + o;
             kind[t] = 0; src[t] = (int32_t)base; pos[t] = (int32_t)t; win[t] = w;
+            keep[t] = (uint8_t)in_tail(o, n, tail);
+            if (keep[t]) { sum_idx[r] = (int32_t)t; r += 1; }
             if (nt && tok)
                 for (int32_t b = 0; b < B; ++b) tok[(int64_t)b * T_total + t] = nt[(int64_t)b * N + base];
             t += 1;
             if (summary_after(o, n, k_sched[w], close)) {
                 kind[t] = 1; src[t] = (int32_t)base; pos[t] = (int32_t)t; win[t] = w;
+                keep[t] = 1;
                 if (nt && tok)
                     for (int32_t b = 0; b < B; ++b) tok[(int64_t)b * T_total + t] = FO_SUMMARY_TOKEN;
                 sum_idx[r] = (int32_t)t;
@@ -152,13 +166,14 @@ static void softmax_row(int32_t d, const uint16_t* q, int64_t n_keys,
 /* ------------------------------------------------------------------------- */
 /* Masked-parallel form (App. A.1, "Cross-window consistency" (ii), with the  */
 /* visible set of Eq. focus-attn / C(t)): row i sees key j iff j <= i and     */
-/* (j is in the same window as i, or j is a FOCUS token).                     */
+/* (j is in the same window as i, or j is a retained row: a FOCUS token or a  */
+/* boundary-tail base; keep[] marks them).                                     */
 /*                                                                            */
 /* q, k, v: [n_heads][T][d] bf16 bits. Computes the requested rows only:     */
 /* row r is (head row_head[r], augmented index row_idx[r]). Outputs o[r][d],  */
 /* lse[r].                                                                    */
 /* ------------------------------------------------------------------------- */
-void fo_attn_rows(int64_t T, int32_t d, const uint8_t* kind, const int32_t* win,
+void fo_attn_rows(int64_t T, int32_t d, const uint8_t* keep, const int32_t* win,
                   const uint16_t* q, const uint16_t* k, const uint16_t* v,
                   double scale, int64_t n_rows, const int64_t* row_head,
                   const int64_t* row_idx, double* o, double* lse) {
@@ -171,7 +186,7 @@ void fo_attn_rows(int64_t T, int32_t d, const uint8_t* kind, const int32_t* win,
         const uint16_t** vr = (const uint16_t**)malloc(sizeof(void*) * (size_t)(i + 1));
         int64_t n = 0;
         for (int64_t j = 0; j <= i; ++j) {
-            int visible = (win[j] == win[i]) || (kind[j] == 1);
+            int visible = (win[j] == win[i]) || (keep[j] == 1);
             if (!visible) continue;
             kr[n] = kh + (size_t)j * d;
             vr[n] = vh + (size_t)j * d;
@@ -192,14 +207,14 @@ void fo_attn_rows(int64_t T, int32_t d, const uint8_t* kind, const int32_t* win,
 /* the retained set (App. A, "KV compression and budget").                    */
 /*                                                                            */
 /* One head: q, k, v are [T][d] bf16 bits; win_off[M+1] gives window rows;    */
-/* kind[T] marks FOCUS rows. want[M] (NULL = all) selects the windows whose    */
+/* keep[T] marks retained rows. want[M] (NULL = all) selects the windows whose */
 /* outputs are computed; retention runs for every window regardless. Writes   */
 /* o[T][d], lse[T] for computed windows (others untouched) and the retained   */
 /* KV (ring_k/ring_v, [ring_cap][d]) with its length in *R_out.               */
 /* Returns 0, or -1 if ring_cap is too small.                                 */
 /* ------------------------------------------------------------------------- */
 int32_t fo_prefill_sequential(int32_t d, int32_t M, const int32_t* win_off,
-                              const uint8_t* kind, const uint16_t* q,
+                              const uint8_t* keep, const uint16_t* q,
                               const uint16_t* k, const uint16_t* v, double scale,
                               const uint8_t* want, double* o, double* lse,
                               uint16_t* ring_k, uint16_t* ring_v, int64_t ring_cap,
@@ -229,9 +244,9 @@ int32_t fo_prefill_sequential(int32_t d, int32_t M, const int32_t* win_off,
                 free(vr);
             }
         }
-        /* window finished: keep FOCUS KV, drop ordinary KV */
+        /* window finished: keep FOCUS KV (and the boundary tail), drop the rest */
         for (int64_t j = a; j < e; ++j) {
-            if (kind[j] != 1) continue;
+            if (keep[j] != 1) continue;
             if (R >= ring_cap) return -1;
             memcpy(ring_k + (size_t)R * d, k + (size_t)j * d, sizeof(uint16_t) * (size_t)d);
             memcpy(ring_v + (size_t)R * d, v + (size_t)j * d, sizeof(uint16_t) * (size_t)d);
@@ -283,14 +298,19 @@ void fo_decode(int32_t d, int64_t n, const uint16_t* ring_k, const uint16_t* rin
     }
 }
 
-/* In-window offsets (augmented, 0-based) of the FOCUS rows of one window of n
- * bases with cadence k, i.e. which rows KV retention keeps (App. A, "KV
- * compression and budget"). Writes up to cap offsets; returns their count. */
-int32_t fo_window_summary_rows(int64_t n, int32_t k, int32_t close_partial,
-                               int32_t* out, int32_t cap) {
+/* In-window offsets (augmented, 0-based) of the rows KV retention keeps in one
+ * window of n bases with cadence k: its FOCUS rows and its last `tail` bases
+ * (App. A, "KV compression and budget"), in augmented order. Writes up to cap
+ * offsets; returns their count. */
+int32_t fo_window_retained_rows(int64_t n, int32_t k, int32_t close_partial, int32_t tail,
+                                int32_t* out, int32_t cap) {
     int64_t t = 0;
     int32_t c = 0;
     for (int64_t o = 0; o < n; ++o) {
+        if (in_tail(o, n, tail)) {
+            if (c < cap) out[c] = (int32_t)t;
+            c += 1;
+        }
         t += 1;
         if (summary_after(o, n, k, close_partial)) {
             if (c < cap) out[c] = (int32_t)t;

@@ -48,17 +48,17 @@ def _load(path: str | None = None):
     P = ctypes.c_void_p
     i64, i32, f64 = ctypes.c_int64, ctypes.c_int32, ctypes.c_double
     lib.fo_layout_size.restype = i64
-    lib.fo_layout_size.argtypes = [i64, i32, i32, P, i32, P]
+    lib.fo_layout_size.argtypes = [i64, i32, i32, P, i32, i32, P]
     lib.fo_layout.restype = i64
-    lib.fo_layout.argtypes = [i64, i32, i32, P, i32, i32, P, P, P, P, P, P, P, P, P]
+    lib.fo_layout.argtypes = [i64, i32, i32, P, i32, i32, i32, P, P, P, P, P, P, P, P, P, P]
     lib.fo_attn_rows.restype = None
     lib.fo_attn_rows.argtypes = [i64, i32, P, P, P, P, P, f64, i64, P, P, P, P]
     lib.fo_prefill_sequential.restype = i32
     lib.fo_prefill_sequential.argtypes = [i32, i32, P, P, P, P, P, f64, P, P, P, P, P, i64, P]
     lib.fo_decode.restype = None
     lib.fo_decode.argtypes = [i32, i64, P, P, i64, P, P, P, i64, P, P, P, P, f64, P, P]
-    lib.fo_window_summary_rows.restype = i32
-    lib.fo_window_summary_rows.argtypes = [i64, i32, i32, P, i32]
+    lib.fo_window_retained_rows.restype = i32
+    lib.fo_window_retained_rows.argtypes = [i64, i32, i32, i32, P, i32]
     _lib = lib
     return lib
 
@@ -106,23 +106,25 @@ def n_windows(N: int, W: int) -> int:
     return (N + W - 1) // W
 
 
-def layout_size(N: int, W: int, k_sched, close_tail: bool = True):
-    """(T, R, M): augmented length, retained summaries, windows (App. A)."""
+def layout_size(N: int, W: int, k_sched, close_tail: bool = True, tail: int = 0):
+    """(T, R, M): augmented length, retained rows (summaries + boundary tails),
+    windows (App. A)."""
     lib = _load()
     M = n_windows(N, W)
     k = _k_array(M, k_sched)
     R = np.zeros(1, np.int64)
-    T = lib.fo_layout_size(N, W, M, _ptr(k), int(close_tail), _ptr(R))
+    T = lib.fo_layout_size(N, W, M, _ptr(k), int(close_tail), int(tail), _ptr(R))
     if T < 0:
         raise ValueError("bad layout arguments")
     return int(T), int(R[0]), M
 
 
-def layout(N: int, W: int, k_sched, nt=None, close_tail: bool = True) -> dict:
+def layout(N: int, W: int, k_sched, nt=None, close_tail: bool = True, tail: int = 0) -> dict:
     """Token layout: summary insertion after every k bases per window (Sec. 3.2
-    "Setup and tokens"; App. A). ``nt``: uint8 [B, N] nucleotide ids or None."""
+    "Setup and tokens"; App. A). ``nt``: uint8 [B, N] nucleotide ids or None.
+    ``tail``: ordinary rows kept at the end of each window (boundary tail)."""
     lib = _load()
-    T, R, M = layout_size(N, W, k_sched, close_tail)
+    T, R, M = layout_size(N, W, k_sched, close_tail, tail)
     k = _k_array(M, k_sched)
     if nt is not None:
         nt = np.ascontiguousarray(np.asarray(nt, dtype=np.uint8).reshape(-1, N))
@@ -131,11 +133,11 @@ def layout(N: int, W: int, k_sched, nt=None, close_tail: bool = True) -> dict:
     else:
         B, tok = 0, None
     out = dict(
-        kind=np.zeros(T, np.uint8), src=np.zeros(T, np.int32), pos=np.zeros(T, np.int32),
+        kind=np.zeros(T, np.uint8), keep=np.zeros(T, np.uint8), src=np.zeros(T, np.int32), pos=np.zeros(T, np.int32),
         win=np.zeros(T, np.int32), win_off=np.zeros(M + 1, np.int32),
         ring_off=np.zeros(M + 1, np.int32), sum_idx=np.zeros(max(R, 1), np.int32))
-    t = lib.fo_layout(N, W, M, _ptr(k), int(close_tail), B, _ptr(nt), _ptr(out["kind"]),
-                      _ptr(out["src"]), _ptr(out["pos"]), _ptr(out["win"]), _ptr(tok),
+    t = lib.fo_layout(N, W, M, _ptr(k), int(close_tail), int(tail), B, _ptr(nt), _ptr(out["kind"]),
+                      _ptr(out["src"]), _ptr(out["pos"]), _ptr(out["win"]), _ptr(tok), _ptr(out["keep"]),
                       _ptr(out["win_off"]), _ptr(out["ring_off"]), _ptr(out["sum_idx"]))
     assert t == T
     out["sum_idx"] = out["sum_idx"][:R]
@@ -144,16 +146,18 @@ def layout(N: int, W: int, k_sched, nt=None, close_tail: bool = True) -> dict:
     return out
 
 
-def attn_rows(q, k, v, kind, win, scale: float, heads, rows):
+def attn_rows(q, k, v, keep, win, scale: float, heads, rows):
     """Masked-parallel attention at selected rows (App. A.1 (ii); Eq.
-    focus-attn's visible set). q/k/v: bf16 [n_heads, T, d]. ``heads``/``rows``:
-    equal-length integer sequences. Returns (o [n, d] fp64, lse [n] fp64)."""
+    focus-attn's visible set). q/k/v: bf16 [n_heads, T, d]; ``keep``: the layout's
+    retained-row flags (FOCUS rows, plus boundary-tail rows if any).
+    ``heads``/``rows``: equal-length integer sequences. Returns (o [n, d] fp64,
+    lse [n] fp64)."""
     lib = _load()
     qb, kb, vb = _bits(q), _bits(k), _bits(v)
     nh, T, d = qb.shape
-    kind = np.ascontiguousarray(kind, dtype=np.uint8)
+    keep = np.ascontiguousarray(keep, dtype=np.uint8)
     win = np.ascontiguousarray(win, dtype=np.int32)
-    assert kind.shape == (T,) and win.shape == (T,)
+    assert keep.shape == (T,) and win.shape == (T,)
     heads = np.ascontiguousarray(heads, dtype=np.int64)
     rows = np.ascontiguousarray(rows, dtype=np.int64)
     assert heads.shape == rows.shape
@@ -161,30 +165,30 @@ def attn_rows(q, k, v, kind, win, scale: float, heads, rows):
     n = rows.size
     o = np.zeros((n, d), np.float64)
     lse = np.zeros(n, np.float64)
-    lib.fo_attn_rows(T, d, _ptr(kind), _ptr(win), _ptr(qb), _ptr(kb), _ptr(vb), float(scale),
+    lib.fo_attn_rows(T, d, _ptr(keep), _ptr(win), _ptr(qb), _ptr(kb), _ptr(vb), float(scale),
                      n, _ptr(heads), _ptr(rows), _ptr(o), _ptr(lse))
     return o, lse
 
 
-def prefill_sequential(q, k, v, win_off, kind, scale: float, want=None, ring_cap=None):
+def prefill_sequential(q, k, v, win_off, keep, scale: float, want=None, ring_cap=None):
     """Sequential windowed form with KV retention (App. A.1 (i), App. A.2) for
-    ONE head: q/k/v bf16 [T, d]. Returns (o [T,d] fp64, lse [T] fp64,
-    ring_k uint16 [R,d], ring_v uint16 [R,d]). Rows of windows not in ``want``
-    are NaN."""
+    ONE head: q/k/v bf16 [T, d]; ``keep``: retained-row flags. Returns (o [T,d]
+    fp64, lse [T] fp64, ring_k uint16 [R,d], ring_v uint16 [R,d]). Rows of
+    windows not in ``want`` are NaN."""
     lib = _load()
     qb, kb, vb = _bits(q), _bits(k), _bits(v)
     T, d = qb.shape
     win_off = np.ascontiguousarray(win_off, dtype=np.int32)
     M = win_off.size - 1
-    kind = np.ascontiguousarray(kind, dtype=np.uint8)
-    cap = int(ring_cap if ring_cap is not None else max(int((kind == 1).sum()), 1))
+    keep = np.ascontiguousarray(keep, dtype=np.uint8)
+    cap = int(ring_cap if ring_cap is not None else max(int((keep == 1).sum()), 1))
     want_a = None if want is None else np.ascontiguousarray(want, dtype=np.uint8)
     o = np.full((T, d), np.nan)
     lse = np.full(T, np.nan)
     rk = np.zeros((cap, d), np.uint16)
     rv = np.zeros((cap, d), np.uint16)
     R = np.zeros(1, np.int64)
-    rc = lib.fo_prefill_sequential(d, M, _ptr(win_off), _ptr(kind), _ptr(qb), _ptr(kb), _ptr(vb),
+    rc = lib.fo_prefill_sequential(d, M, _ptr(win_off), _ptr(keep), _ptr(qb), _ptr(kb), _ptr(vb),
                                    float(scale), _ptr(want_a), _ptr(o), _ptr(lse), _ptr(rk), _ptr(rv),
                                    cap, _ptr(R))
     if rc != 0:
@@ -214,13 +218,13 @@ def decode(q, k_new, v_new, ring_k, ring_v, R, win_k, win_v, fill, scale: float)
     return o, lse
 
 
-def window_summary_rows(n: int, k: int, close_partial: bool = True) -> np.ndarray:
-    """In-window augmented offsets of the FOCUS rows that KV retention keeps
-    for a window of n bases with cadence k (App. A)."""
+def window_retained_rows(n: int, k: int, close_partial: bool = True, tail: int = 0) -> np.ndarray:
+    """In-window augmented offsets of the rows KV retention keeps for a window
+    of n bases with cadence k: its FOCUS rows and its last ``tail`` bases (App. A)."""
     lib = _load()
-    cap = n + 1
+    cap = 2 * n + 2
     out = np.zeros(cap, np.int32)
-    c = lib.fo_window_summary_rows(n, k, int(close_partial), _ptr(out), cap)
+    c = lib.fo_window_retained_rows(n, k, int(close_partial), int(tail), _ptr(out), cap)
     return out[:c]
 
 

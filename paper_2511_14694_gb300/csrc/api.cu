@@ -34,7 +34,7 @@ focus_status from_cuda(cudaError_t e) { return e == cudaSuccess ? FOCUS_OK : FOC
 
 focus_status check_cache(const focus_cache* c, bool need_window) {
     if (!c) return FOCUS_ERR_INVALID_ARG;
-    if (c->B <= 0 || c->H <= 0 || c->C_ring < 0 || c->C_win < 0) return FOCUS_ERR_INVALID_ARG;
+    if (c->B <= 0 || c->H <= 0 || c->C_ring < 0 || c->C_win < 0 || c->tail < 0) return FOCUS_ERR_INVALID_ARG;
     if (c->d != 64 && c->d != 128) return FOCUS_ERR_UNSUPPORTED;
     if ((int64_t)c->B > 65535 || (int64_t)c->H > 65535) return FOCUS_ERR_UNSUPPORTED;
     if (c->C_ring > 0 && (!c->ring_k || !c->ring_v)) return FOCUS_ERR_INVALID_ARG;
@@ -82,8 +82,8 @@ focus_status focus_get_device_status(int32_t* host_status, int32_t clear, cudaSt
 }
 
 focus_status focus_layout_size(int64_t n_nt, int32_t W, int32_t n_windows, const int32_t* h_k, uint32_t flags,
-                               int64_t* T, int64_t* R, int32_t* max_rows) {
-    if (n_nt < 0 || W <= 0 || (n_nt > 0 && !h_k)) return FOCUS_ERR_INVALID_ARG;
+                               int32_t tail, int64_t* T, int64_t* R, int32_t* max_rows) {
+    if (n_nt < 0 || W <= 0 || tail < 0 || (n_nt > 0 && !h_k)) return FOCUS_ERR_INVALID_ARG;
     if ((int64_t)n_windows != focus::ceil_div64(n_nt, W)) return FOCUS_ERR_INVALID_ARG;
     const bool close_tail = (flags & FOCUS_LAYOUT_CLOSE_TAIL) != 0;
     int64_t t = 0, r = 0, mx = 0;
@@ -93,7 +93,7 @@ focus_status focus_layout_size(int64_t n_nt, int32_t W, int32_t n_windows, const
         if (n > W) n = W;
         const int64_t rows = focus::window_rows(n, h_k[w], (w < n_windows - 1) || close_tail);
         t += rows;
-        r += rows - n;
+        r += rows - n + (n - focus::tail_start(n, tail));
         if (rows > mx) mx = rows;
     }
     if (t > INT32_MAX) return FOCUS_ERR_UNSUPPORTED;   // offsets are int32
@@ -104,8 +104,9 @@ focus_status focus_layout_size(int64_t n_nt, int32_t W, int32_t n_windows, const
 }
 
 focus_status focus_layout(int64_t n_nt, int32_t W, int32_t n_windows, const int32_t* d_k, uint32_t flags,
-                          int32_t B, const uint8_t* d_nt, const focus_layout_out* out, cudaStream_t stream) {
-    if (!out || n_nt < 0 || W <= 0 || B < 0) return FOCUS_ERR_INVALID_ARG;
+                          int32_t tail, int32_t B, const uint8_t* d_nt, const focus_layout_out* out,
+                          cudaStream_t stream) {
+    if (!out || n_nt < 0 || W <= 0 || B < 0 || tail < 0) return FOCUS_ERR_INVALID_ARG;
     if ((int64_t)n_windows != focus::ceil_div64(n_nt, W) || n_windows <= 0 || !d_k) return FOCUS_ERR_INVALID_ARG;
     if (out->T < 0 || out->R < 0 || out->T > INT32_MAX) return FOCUS_ERR_INVALID_ARG;
     if (!out->win_off || !out->ring_off) return FOCUS_ERR_INVALID_ARG;
@@ -115,8 +116,8 @@ focus_status focus_layout(int64_t n_nt, int32_t W, int32_t n_windows, const int3
     int32_t* st = nullptr;
     focus_status s = status_ptr(&st);
     if (s != FOCUS_OK) return s;
-    return from_cuda(focus::launch_layout(n_nt, W, n_windows, d_k, (flags & FOCUS_LAYOUT_CLOSE_TAIL) != 0, B, d_nt,
-                                          *out, st, stream));
+    return from_cuda(focus::launch_layout(n_nt, W, n_windows, d_k, (flags & FOCUS_LAYOUT_CLOSE_TAIL) != 0, tail, B,
+                                          d_nt, *out, st, stream));
 }
 
 focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_args* a, cudaStream_t stream) {

@@ -33,9 +33,15 @@ __host__ __device__ __forceinline__ int32_t window_summary_row(int32_t j, int32_
     return (int32_t)window_rows(W, k, true) - 1;
 }
 
+// First base of the boundary tail of an n-base window (bases at or after it are
+// kept with the FOCUS rows); tail = 0 means none.
+__host__ __device__ __forceinline__ int64_t tail_start(int64_t n, int32_t tail) {
+    return tail > 0 ? (n - tail > 0 ? n - tail : 0) : n;
+}
+
 // Kernel launchers (one translation unit each).
 cudaError_t launch_layout(int64_t N, int32_t W, int32_t M, const int32_t* d_k, bool close_tail,
-                          int32_t B, const uint8_t* d_nt, const focus_layout_out& out,
+                          int32_t tail, int32_t B, const uint8_t* d_nt, const focus_layout_out& out,
                           int32_t* status, cudaStream_t stream);
 
 cudaError_t launch_compact_bulk(const focus_cache& c, const focus_compact_args& a, int32_t* status,

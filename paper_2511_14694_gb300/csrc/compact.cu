@@ -1,7 +1,8 @@
 // KV retention / compaction (App. A, "KV compression and budget"; Sec. 3.2
 // "KV retention and memory profile"): after a window, only the FOCUS rows' K/V
-// are kept, appended to the per-(sequence, head) ring. Ordinary rows are simply
-// not copied. Pure data movement, bit-exact; 16-byte vector loads and stores.
+// (and, if asked for, the window's boundary tail of ordinary rows) are kept,
+// appended to the per-(sequence, head) ring. Other rows are simply not copied.
+// Pure data movement, bit-exact; 16-byte vector loads and stores.
 #include "common.cuh"
 
 namespace focus {
@@ -44,13 +45,15 @@ __global__ void __launch_bounds__(256) compact_bulk_kernel(
 }
 
 // Window mode: one CTA per sequence. If the current window buffer holds the
-// whole window (W bases + its summaries), append its FOCUS rows to the ring and
-// start the next window.
+// whole window (W bases + its summaries), append its kept rows (FOCUS rows and
+// the last `tail` bases) to the ring in augmented order and start the next
+// window. Kept row j is either summary j (j < B_w) or tail base j - B_w; each
+// one's buffer row and ring slot follow in closed form.
 __global__ void __launch_bounds__(256) compact_window_kernel(
         uint4* __restrict__ ring_k, uint4* __restrict__ ring_v, const uint4* __restrict__ win_k,
         const uint4* __restrict__ win_v, int32_t* __restrict__ ring_len, int32_t* __restrict__ win_fill,
         int32_t* __restrict__ win_idx, const int32_t* __restrict__ ks, int32_t n_windows, int32_t W,
-        int32_t H, int32_t chunks_per_row, int32_t C_ring, int32_t C_win, int32_t* status) {
+        int32_t H, int32_t chunks_per_row, int32_t C_ring, int32_t C_win, int32_t tail, int32_t* status) {
     const int32_t b = blockIdx.x;
     const int32_t fill = win_fill[b], widx = win_idx[b], R = ring_len[b];
     if (widx < 0 || widx >= n_windows) {
@@ -61,26 +64,38 @@ __global__ void __launch_bounds__(256) compact_window_kernel(
     const int32_t Tw = (int32_t)window_rows(W, k, true);
     if (fill != Tw) return;                  // window not complete yet
     const int32_t Bw = Tw - W;
-    if (R + Bw > C_ring || Tw > C_win) {
+    const int32_t ts = (int32_t)tail_start(W, tail);
+    const int32_t kept = Bw + (W - ts);
+    if (R + kept > C_ring || Tw > C_win) {
         if (threadIdx.x == 0) report(status, FOCUS_ERR_CAPACITY);
         return;
     }
-    const int64_t total = (int64_t)H * Bw * chunks_per_row;
+    const int64_t total = (int64_t)H * kept * chunks_per_row;
     for (int64_t i = threadIdx.x; i < total; i += blockDim.x) {
         const int32_t c = (int32_t)(i % chunks_per_row);
         const int64_t rest = i / chunks_per_row;
-        const int32_t j = (int32_t)(rest % Bw);
-        const int64_t h = rest / Bw;
+        const int32_t j = (int32_t)(rest % kept);
+        const int64_t h = rest / kept;
         const int64_t bh = (int64_t)b * H + h;
-        const int32_t row = window_summary_row(j, W, k);
+        int32_t row, slot;
+        if (j < Bw) {                       // summary j, after base min((j+1)k, W) - 1
+            row = window_summary_row(j, W, k);
+            const int32_t end = (int64_t)(j + 1) * k < W ? (j + 1) * k : W;
+            slot = j + (end > ts ? end - ts : 0);
+        } else {                            // tail base o
+            const int32_t o = ts + (j - Bw);
+            const int32_t before = k > 0 ? o / k : 0;   // summaries before base o
+            row = o + before;
+            slot = before + (j - Bw);
+        }
         const int64_t so = (bh * C_win + row) * chunks_per_row + c;
-        const int64_t d_o = (bh * C_ring + R + j) * chunks_per_row + c;
+        const int64_t d_o = (bh * C_ring + R + slot) * chunks_per_row + c;
         ring_k[d_o] = win_k[so];
         ring_v[d_o] = win_v[so];
     }
     __syncthreads();
     if (threadIdx.x == 0) {
-        ring_len[b] = R + Bw;
+        ring_len[b] = R + kept;
         win_fill[b] = 0;
         win_idx[b] = widx + 1;
     }
@@ -104,7 +119,7 @@ cudaError_t launch_compact_bulk(const focus_cache& c, const focus_compact_args& 
 cudaError_t launch_compact_window(const focus_cache& c, int32_t* status, cudaStream_t stream) {
     compact_window_kernel<<<c.B, 256, 0, stream>>>(
         (uint4*)c.ring_k, (uint4*)c.ring_v, (const uint4*)c.win_k, (const uint4*)c.win_v, c.ring_len,
-        c.win_fill, c.win_idx, c.k_per_window, c.n_windows, c.W, c.H, c.d / 8, c.C_ring, c.C_win, status);
+        c.win_fill, c.win_idx, c.k_per_window, c.n_windows, c.W, c.H, c.d / 8, c.C_ring, c.C_win, c.tail, status);
     return cudaGetLastError();
 }
 

@@ -36,13 +36,13 @@ _i32, _i64, _u32, _f32 = ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32, ctypes
 
 class LayoutOut(ctypes.Structure):
     _fields_ = [("T", _i64), ("R", _i64), ("kind", _P), ("src", _P), ("pos", _P), ("win", _P), ("tok", _P),
-                ("win_off", _P), ("ring_off", _P), ("sum_idx", _P)]
+                ("keep", _P), ("win_off", _P), ("ring_off", _P), ("sum_idx", _P)]
 
 
 class CacheDesc(ctypes.Structure):
     _fields_ = [("ring_k", _P), ("ring_v", _P), ("win_k", _P), ("win_v", _P), ("ring_len", _P),
                 ("win_fill", _P), ("win_idx", _P), ("k_per_window", _P), ("n_windows", _i32), ("W", _i32),
-                ("B", _i32), ("H", _i32), ("d", _i32), ("C_ring", _i32), ("C_win", _i32)]
+                ("B", _i32), ("H", _i32), ("d", _i32), ("C_ring", _i32), ("C_win", _i32), ("tail", _i32)]
 
 
 class PrefillArgs(ctypes.Structure):
@@ -78,9 +78,9 @@ def load() -> ctypes.CDLL:
     lib.focus_get_device_status.restype = ctypes.c_int
     lib.focus_get_device_status.argtypes = [_P, _i32, _P]
     lib.focus_layout_size.restype = ctypes.c_int
-    lib.focus_layout_size.argtypes = [_i64, _i32, _i32, _P, _u32, _P, _P, _P]
+    lib.focus_layout_size.argtypes = [_i64, _i32, _i32, _P, _u32, _i32, _P, _P, _P]
     lib.focus_layout.restype = ctypes.c_int
-    lib.focus_layout.argtypes = [_i64, _i32, _i32, _P, _u32, _i32, _P, ctypes.POINTER(LayoutOut), _P]
+    lib.focus_layout.argtypes = [_i64, _i32, _i32, _P, _u32, _i32, _i32, _P, ctypes.POINTER(LayoutOut), _P]
     lib.focus_attn_prefill.restype = ctypes.c_int
     lib.focus_attn_prefill.argtypes = [ctypes.POINTER(CacheDesc), ctypes.POINTER(PrefillArgs), _P]
     lib.focus_decode_workspace_size.restype = ctypes.c_size_t
@@ -123,23 +123,24 @@ def _cuda(t: torch.Tensor, name: str, dtype=None):
 
 # ----------------------------------------------------------------------------- layout
 
-def layout_size(N: int, W: int, k_sched, close_tail: bool = True):
+def layout_size(N: int, W: int, k_sched, close_tail: bool = True, tail: int = 0):
     """(T, R, M, max_rows) of the augmented layout (host arithmetic in the library)."""
     lib = load()
     M = -(-N // W)
     k = np.ascontiguousarray(np.broadcast_to(np.asarray(k_sched, dtype=np.int32), (M,)))
     T, R, mx = _i64(), _i64(), _i32()
     _check("focus_layout_size", lib.focus_layout_size(N, W, M, k.ctypes.data, LAYOUT_CLOSE_TAIL if close_tail else 0,
-                                                      ctypes.byref(T), ctypes.byref(R), ctypes.byref(mx)))
+                                                      int(tail), ctypes.byref(T), ctypes.byref(R), ctypes.byref(mx)))
     return T.value, R.value, M, mx.value
 
 
-def layout_alloc(N: int, W: int, k_sched, B: int = 0, close_tail: bool = True, device="cuda") -> dict:
+def layout_alloc(N: int, W: int, k_sched, B: int = 0, close_tail: bool = True, device="cuda", tail: int = 0) -> dict:
     """Allocate the device outputs of focus_layout (sizes from focus_layout_size)."""
-    T, R, M, mx = layout_size(N, W, k_sched, close_tail)
+    T, R, M, mx = layout_size(N, W, k_sched, close_tail, tail)
     k_host = np.ascontiguousarray(np.broadcast_to(np.asarray(k_sched, dtype=np.int32), (M,)))
     out = dict(
-        kind=torch.empty(T, dtype=torch.uint8, device=device), src=torch.empty(T, dtype=torch.int32, device=device),
+        kind=torch.empty(T, dtype=torch.uint8, device=device), keep=torch.empty(T, dtype=torch.uint8, device=device),
+        src=torch.empty(T, dtype=torch.int32, device=device),
         pos=torch.empty(T, dtype=torch.int32, device=device), win=torch.empty(T, dtype=torch.int32, device=device),
         tok=torch.empty((B, T), dtype=torch.uint8, device=device) if B else None,
         win_off=torch.empty(M + 1, dtype=torch.int32, device=device),
@@ -147,7 +148,7 @@ def layout_alloc(N: int, W: int, k_sched, B: int = 0, close_tail: bool = True, d
         sum_idx_buf=torch.empty(max(R, 1), dtype=torch.int32, device=device),
         k=torch.from_numpy(k_host.copy()).to(device))
     out["sum_idx"] = out["sum_idx_buf"][:R]
-    out.update(T=T, R=R, M=M, max_rows=mx, k_host=k_host, N=N, W=W, B=B, close_tail=close_tail)
+    out.update(T=T, R=R, M=M, max_rows=mx, k_host=k_host, N=N, W=W, B=B, close_tail=close_tail, tail=tail)
     return out
 
 
@@ -159,19 +160,19 @@ def layout_run(L: dict, nt: torch.Tensor | None = None, stream=None) -> None:
         if L["tok"] is None or tuple(nt.shape) != (L["B"], L["N"]):
             raise ValueError("nt shape does not match the allocated layout")
     desc = LayoutOut(L["T"], L["R"], _ptr(L["kind"]), _ptr(L["src"]), _ptr(L["pos"]), _ptr(L["win"]),
-                     _ptr(L["tok"]) if nt is not None else None, _ptr(L["win_off"]), _ptr(L["ring_off"]),
-                     _ptr(L["sum_idx_buf"]))
+                     _ptr(L["tok"]) if nt is not None else None, _ptr(L["keep"]), _ptr(L["win_off"]),
+                     _ptr(L["ring_off"]), _ptr(L["sum_idx_buf"]))
     _check("focus_layout", lib.focus_layout(L["N"], L["W"], L["M"], _ptr(L["k"]),
-                                            LAYOUT_CLOSE_TAIL if L["close_tail"] else 0,
+                                            LAYOUT_CLOSE_TAIL if L["close_tail"] else 0, int(L["tail"]),
                                             0 if nt is None else L["B"], _ptr(nt), ctypes.byref(desc),
                                             _stream(stream)))
 
 
 def layout(N: int, W: int, k_sched, nt: torch.Tensor | None = None, close_tail: bool = True,
-           device="cuda", stream=None) -> dict:
+           device="cuda", stream=None, tail: int = 0) -> dict:
     """Build the augmented token layout on the device (focus_layout) and keep host
     copies of the window/ring offsets for slicing per-window inputs (syncs)."""
-    L = layout_alloc(N, W, k_sched, 0 if nt is None else int(nt.shape[0]), close_tail, device)
+    L = layout_alloc(N, W, k_sched, 0 if nt is None else int(nt.shape[0]), close_tail, device, tail)
     layout_run(L, nt, stream)
     L["win_off_host"] = L["win_off"].cpu().numpy()
     L["ring_off_host"] = L["ring_off"].cpu().numpy()
@@ -185,8 +186,8 @@ class Cache:
     current window buffer) and its C descriptor."""
 
     def __init__(self, B: int, H: int, d: int, C_ring: int, C_win: int = 0, W: int = 0, k_sched=None,
-                 device="cuda"):
-        self.B, self.H, self.d, self.C_ring, self.C_win, self.W = B, H, d, C_ring, C_win, W
+                 device="cuda", tail: int = 0):
+        self.B, self.H, self.d, self.C_ring, self.C_win, self.W, self.tail = B, H, d, C_ring, C_win, W, tail
         bf = dict(dtype=torch.bfloat16, device=device)
         self.ring_k = torch.zeros((B, H, max(C_ring, 1), d), **bf)
         self.ring_v = torch.zeros((B, H, max(C_ring, 1), d), **bf)
@@ -199,7 +200,7 @@ class Cache:
         self.k_sched = torch.from_numpy(ks.copy()).to(device)
         self.desc = CacheDesc(_ptr(self.ring_k), _ptr(self.ring_v), _ptr(self.win_k), _ptr(self.win_v),
                               _ptr(self.ring_len), _ptr(self.win_fill), _ptr(self.win_idx), _ptr(self.k_sched),
-                              int(self.k_sched.numel()), W, B, H, d, C_ring, C_win)
+                              int(self.k_sched.numel()), W, B, H, d, C_ring, C_win, tail)
 
     def workspace_bytes(self) -> int:
         return int(load().focus_decode_workspace_size(ctypes.byref(self.desc)))

@@ -32,8 +32,8 @@ def test_library_exports_every_declared_function():
 
 def test_struct_sizes_match_c_layout():
     # 2 x int64 + 8 pointers; 8 pointers + 7 int32 (+pad); see focus.h
-    assert ctypes.sizeof(focus.LayoutOut) == 16 + 8 * 8
-    assert ctypes.sizeof(focus.CacheDesc) == 8 * 8 + 7 * 4 + 4
+    assert ctypes.sizeof(focus.LayoutOut) == 16 + 9 * 8
+    assert ctypes.sizeof(focus.CacheDesc) == 8 * 8 + 8 * 4
     assert ctypes.sizeof(focus.PrefillArgs) == 5 * 8 + 8 + 2 * 8 + 6 * 4
     assert ctypes.sizeof(focus.CompactArgs) == 2 * 8 + 2 * 8 + 2 * 8 + 3 * 4 + 4
 
@@ -45,16 +45,18 @@ def test_version_and_status_strings():
         assert lib.focus_status_string(code)
 
 
-@pytest.mark.parametrize("N,W,ks,close", [(4_000, 1_000, [100], True), (128_000, 1_000, [100], True),
-                                          (5_000, 1_024, [100], False), (10, 4, [3], True),
-                                          (256_000, 1_000, [10, 25, 50, 100, 200], True), (77, 100, [0], True)])
-def test_layout_size_matches_oracle(N, W, ks, close):
+@pytest.mark.parametrize("N,W,ks,close,tail", [(4_000, 1_000, [100], True, 0), (128_000, 1_000, [100], True, 0),
+                                               (5_000, 1_024, [100], False, 0), (10, 4, [3], True, 0),
+                                               (256_000, 1_000, [10, 25, 50, 100, 200], True, 0),
+                                               (77, 100, [0], True, 0), (4_000, 1_000, [100], True, 4),
+                                               (77, 10, [3], False, 20)])
+def test_layout_size_matches_oracle(N, W, ks, close, tail):
     M = -(-N // W)
     k = inputs.k_schedule(M, ks, seed=1)
-    T, R, M2, mx = focus.layout_size(N, W, k, close_tail=close)
-    To, Ro, Mo = fo.layout_size(N, W, k, close_tail=close)
+    T, R, M2, mx = focus.layout_size(N, W, k, close_tail=close, tail=tail)
+    To, Ro, Mo = fo.layout_size(N, W, k, close_tail=close, tail=tail)
     assert (T, R, M2) == (To, Ro, Mo)
-    L = fo.layout(N, W, k, close_tail=close)
+    L = fo.layout(N, W, k, close_tail=close, tail=tail)
     assert mx == int(np.diff(L["win_off"]).max())
 
 
@@ -63,12 +65,13 @@ def test_host_validation_rejects_bad_arguments():
     T = ctypes.c_int64()
     k = np.array([100], np.int32)
     # wrong window count, negative N, missing schedule
-    assert lib.focus_layout_size(1000, 1000, 2, k.ctypes.data, 1, ctypes.byref(T), None, None) == 1
-    assert lib.focus_layout_size(-1, 1000, 0, k.ctypes.data, 1, ctypes.byref(T), None, None) == 1
-    assert lib.focus_layout_size(1000, 1000, 1, None, 1, ctypes.byref(T), None, None) == 1
-    assert lib.focus_layout_size(1000, 0, 1, k.ctypes.data, 1, ctypes.byref(T), None, None) == 1
+    assert lib.focus_layout_size(1000, 1000, 2, k.ctypes.data, 1, 0, ctypes.byref(T), None, None) == 1
+    assert lib.focus_layout_size(-1, 1000, 0, k.ctypes.data, 1, 0, ctypes.byref(T), None, None) == 1
+    assert lib.focus_layout_size(1000, 1000, 1, None, 1, 0, ctypes.byref(T), None, None) == 1
+    assert lib.focus_layout_size(1000, 0, 1, k.ctypes.data, 1, 0, ctypes.byref(T), None, None) == 1
+    assert lib.focus_layout_size(1000, 1000, 1, k.ctypes.data, 1, -1, ctypes.byref(T), None, None) == 1
     neg = np.array([-3], np.int32)
-    assert lib.focus_layout_size(1000, 1000, 1, neg.ctypes.data, 1, ctypes.byref(T), None, None) == 1
+    assert lib.focus_layout_size(1000, 1000, 1, neg.ctypes.data, 1, 0, ctypes.byref(T), None, None) == 1
     # null descriptors
     assert lib.focus_attn_prefill(None, None, None) == 1
     assert lib.focus_kv_compact(None, None, None) == 1

@@ -55,18 +55,20 @@ LAYOUT_CASES = [
     (77, 10, [20], True), (5_000, 1_024, [100], False), (5_000, 1_024, [100], True), (3_001, 3, [1, 2, 3, 4], False),
     (2_048, 2_048, [1], True),
 ]
+TAIL_LAYOUT_CASES = [(4_000, 1_000, [100], True, 3), (3_001, 3, [1, 2, 3, 4], False, 1), (77, 10, [20], True, 10),
+                     (5_000, 1_024, [100], False, 50), (500, 1_000, [0], True, 7), (10, 4, [3], True, 100)]
 
 
-@pytest.mark.parametrize("N,W,ks,close", LAYOUT_CASES)
-def test_layout_bit_exact(N, W, ks, close):
+@pytest.mark.parametrize("N,W,ks,close,tail", [c + (0,) for c in LAYOUT_CASES] + TAIL_LAYOUT_CASES)
+def test_layout_bit_exact(N, W, ks, close, tail):
     M = -(-N // W)
     k = inputs.k_schedule(M, ks, seed=N % 97)
     nt = inputs.nucleotides(2, N, seed=5, device="cuda")
-    L = focus.layout(N, W, k, nt=nt, close_tail=close)
-    ref = fo.layout(N, W, k, nt=nt.cpu().numpy(), close_tail=close)
+    L = focus.layout(N, W, k, nt=nt, close_tail=close, tail=tail)
+    ref = fo.layout(N, W, k, nt=nt.cpu().numpy(), close_tail=close, tail=tail)
     torch.cuda.synchronize()
     assert (L["T"], L["R"], L["M"]) == (ref["T"], ref["R"], ref["M"])
-    for key in ("kind", "src", "pos", "win", "win_off", "ring_off", "sum_idx"):
+    for key in ("kind", "keep", "src", "pos", "win", "win_off", "ring_off", "sum_idx"):
         assert np.array_equal(L[key].cpu().numpy(), ref[key]), key
     assert np.array_equal(L["tok"].cpu().numpy(), ref["tok"])
 
@@ -83,12 +85,18 @@ PREFILL_CASES = [
     (20_000, 200, [10], 1, 2, 128, 1.0 / math.sqrt(128)),   # ring of up to 990 rows
     (3_333, 1_000, [3, 100, 1_000], 2, 1, 128, 1.0),  # ragged last window, k = W
 ]
+TAIL_PREFILL_CASES = [
+    # N, W, k schedule, B, H, d, std, tail
+    (3_000, 500, [10, 50], 1, 2, 128, 1.0, 3),
+    (1_000, 100, [7], 2, 1, 64, 1.0, 200),          # tail >= W: every row kept -> causal over all rows
+    (4_100, 1_000, [100], 1, 2, 128, 1.0 / math.sqrt(128), 30),
+]
 
 
-def _masked_parallel(N, W, ks, B, H, d, std, seed=0, flags=0):
+def _masked_parallel(N, W, ks, B, H, d, std, seed=0, flags=0, tail=0):
     M = -(-N // W)
     k = inputs.k_schedule(M, ks, seed=seed + 1)
-    L = focus.layout(N, W, k)
+    L = focus.layout(N, W, k, tail=tail)
     q, kk, v = inputs.qkv((B, H, L["T"], d), std=std, seed=seed + 2, device="cuda")
     cache = focus.Cache(B, H, d, C_ring=max(L["R"], 1))
     n = q.numel()
@@ -100,15 +108,15 @@ def _masked_parallel(N, W, ks, B, H, d, std, seed=0, flags=0):
     return L, q, kk, v, cache, o, lse
 
 
-@pytest.mark.parametrize("N,W,ks,B,H,d,std", PREFILL_CASES)
-def test_prefill_masked_parallel_matches_oracle(N, W, ks, B, H, d, std):
-    L, q, k, v, cache, o, lse = _masked_parallel(N, W, ks, B, H, d, std, seed=N)
-    ref_L = fo.layout(N, W, L["k_host"])
+@pytest.mark.parametrize("N,W,ks,B,H,d,std,tail", [c + (0,) for c in PREFILL_CASES] + TAIL_PREFILL_CASES)
+def test_prefill_masked_parallel_matches_oracle(N, W, ks, B, H, d, std, tail):
+    L, q, k, v, cache, o, lse = _masked_parallel(N, W, ks, B, H, d, std, seed=N, tail=tail)
+    ref_L = fo.layout(N, W, L["k_host"], tail=tail)
     T = L["T"]
     heads = np.repeat(np.arange(B * H), T)
     rows = np.tile(np.arange(T), B * H)
     o_ref, lse_ref = fo.attn_rows(q.reshape(B * H, T, d).cpu(), k.reshape(B * H, T, d).cpu(),
-                                  v.reshape(B * H, T, d).cpu(), ref_L["kind"], ref_L["win"], 1.0 / math.sqrt(d),
+                                  v.reshape(B * H, T, d).cpu(), ref_L["keep"], ref_L["win"], 1.0 / math.sqrt(d),
                                   heads, rows)
     assert_attn_close(o, lse, o_ref.reshape(B, H, T, d), lse_ref.reshape(B, H, T), f"N={N} W={W} k={ks}")
     # compaction: ring == the FOCUS rows, bit for bit
@@ -124,19 +132,19 @@ def test_prefill_legacy_kernel_matches_oracle():
     ref_L = fo.layout(N, W, L["k_host"])
     T = L["T"]
     o_ref, lse_ref = fo.attn_rows(q.reshape(H, T, d).cpu(), k.reshape(H, T, d).cpu(), v.reshape(H, T, d).cpu(),
-                                  ref_L["kind"], ref_L["win"], 1.0 / math.sqrt(d), np.repeat(np.arange(H), T),
+                                  ref_L["keep"], ref_L["win"], 1.0 / math.sqrt(d), np.repeat(np.arange(H), T),
                                   np.tile(np.arange(T), H))
     assert_attn_close(o, lse, o_ref.reshape(B, H, T, d), lse_ref.reshape(B, H, T), "legacy")
 
 
 # ----------------------------------------------------------------------------- prefill, sequential / streaming
 
-@pytest.mark.parametrize("d", [64, 128])
-def test_prefill_streaming_matches_sequential_oracle(d):
+@pytest.mark.parametrize("d,tail", [(64, 0), (128, 0), (128, 5)])
+def test_prefill_streaming_matches_sequential_oracle(d, tail):
     N, W, ks, B, H = 3_000, 500, [10, 50, 100, 7], 2, 2
     M = -(-N // W)
     k_s = inputs.k_schedule(M, ks, seed=4)
-    L = focus.layout(N, W, k_s)
+    L = focus.layout(N, W, k_s, tail=tail)
     q, k, v = inputs.qkv((B, H, L["T"], d), seed=21, device="cuda")
     cache = focus.Cache(B, H, d, C_ring=L["R"])
     o = torch.empty_like(q)
@@ -149,11 +157,11 @@ def test_prefill_streaming_matches_sequential_oracle(d):
         o[:, :, a:e] = ow
         lse[:, :, a:e] = lw
     torch.cuda.synchronize()
-    ref_L = fo.layout(N, W, k_s)
+    ref_L = fo.layout(N, W, k_s, tail=tail)
     for b in range(B):
         for h in range(H):
             o_ref, lse_ref, rk, rv = fo.prefill_sequential(q[b, h].cpu(), k[b, h].cpu(), v[b, h].cpu(),
-                                                           ref_L["win_off"], ref_L["kind"], 1.0 / math.sqrt(d))
+                                                           ref_L["win_off"], ref_L["keep"], 1.0 / math.sqrt(d))
             assert_attn_close(o[b, h], lse[b, h], o_ref, lse_ref, f"stream b={b} h={h}")
             assert np.array_equal(bits(cache.ring_k[b, h, :L["R"]]), rk)
             assert np.array_equal(bits(cache.ring_v[b, h, :L["R"]]), rv)
@@ -164,11 +172,11 @@ def test_prefill_streaming_matches_sequential_oracle(d):
 class DecodeModel:
     """Host mirror of the decode cache evolved with the oracle's rules (App. A.2)."""
 
-    def __init__(self, ring_k, ring_v, R, win_k, win_v, fill, widx, W, k_sched):
+    def __init__(self, ring_k, ring_v, R, win_k, win_v, fill, widx, W, k_sched, tail=0):
         self.rk, self.rv = bits(ring_k).copy(), bits(ring_v).copy()
         self.wk, self.wv = bits(win_k).copy(), bits(win_v).copy()
         self.R, self.fill, self.widx = R.copy(), fill.copy(), widx.copy()
-        self.W, self.k = W, np.asarray(k_sched)
+        self.W, self.k, self.tail = W, np.asarray(k_sched), tail
 
     def step(self, q, kn, vn, scale):
         B, H, d = q.shape
@@ -185,7 +193,7 @@ class DecodeModel:
             kw = int(self.k[self.widx[b]])
             Tw = self.W + (-(-self.W // kw) if kw > 0 else 0)
             if self.fill[b] == Tw:                       # window complete: retain its FOCUS rows
-                rows = fo.window_summary_rows(self.W, kw)
+                rows = fo.window_retained_rows(self.W, kw, True, self.tail)
                 r = self.R[b]
                 self.rk[b, :, r:r + rows.size] = self.wk[b][:, rows]
                 self.rv[b, :, r:r + rows.size] = self.wv[b][:, rows]
@@ -195,12 +203,12 @@ class DecodeModel:
         return o, lse
 
 
-@pytest.mark.parametrize("d", [64, 128])
-def test_decode_steps_match_oracle(d):
+@pytest.mark.parametrize("d,tail", [(64, 0), (128, 0), (128, 4)])
+def test_decode_steps_match_oracle(d, tail):
     B, H, W = 3, 2, 50
     k_sched = np.array([10, 7, 25, 50, 3, 10, 10, 10], np.int32)
     C_ring, C_win = 512, 72
-    cache = focus.Cache(B, H, d, C_ring=C_ring, C_win=C_win, W=W, k_sched=k_sched)
+    cache = focus.Cache(B, H, d, C_ring=C_ring, C_win=C_win, W=W, k_sched=k_sched, tail=tail)
     g = torch.Generator(device="cuda").manual_seed(3)
     for t in (cache.ring_k, cache.ring_v, cache.win_k, cache.win_v):
         t.copy_(torch.randn(t.shape, generator=g, device="cuda").bfloat16())
@@ -210,7 +218,7 @@ def test_decode_steps_match_oracle(d):
     cache.ring_len.copy_(torch.from_numpy(R0))
     cache.win_idx.copy_(torch.from_numpy(widx0))
     cache.win_fill.copy_(torch.from_numpy(fill0))
-    model = DecodeModel(cache.ring_k, cache.ring_v, R0, cache.win_k, cache.win_v, fill0, widx0, W, k_sched)
+    model = DecodeModel(cache.ring_k, cache.ring_v, R0, cache.win_k, cache.win_v, fill0, widx0, W, k_sched, tail)
     ws = cache.new_workspace()
     scale = 1.0 / math.sqrt(d)
     for step in range(70):
@@ -267,7 +275,7 @@ def test_full_size_prefill_sampled(name):
     rows = _sample_rows(L, 6, 4, seed=1)
     heads = [0, 7, 31]
     ref_L = fo.layout(N, W, k_s)
-    o_ref, lse_ref = fo.attn_rows(q[0, heads].cpu(), k[0, heads].cpu(), v[0, heads].cpu(), ref_L["kind"],
+    o_ref, lse_ref = fo.attn_rows(q[0, heads].cpu(), k[0, heads].cpu(), v[0, heads].cpu(), ref_L["keep"],
                                   ref_L["win"], 1.0 / math.sqrt(d), np.repeat(np.arange(len(heads)), rows.size),
                                   np.tile(rows, len(heads)))
     og = o[0, heads][:, rows]
@@ -340,7 +348,7 @@ def test_full_size_streaming_sampled():
     want_mask[want] = 1
     for i, h in enumerate(heads):
         full = [torch.cat([t[w % P, b, h] for w in range(M)]).cpu() for t in (pq, pk, pv)]
-        o_ref, lse_ref, rk, rv = fo.prefill_sequential(*full, ref_L["win_off"], ref_L["kind"], 1.0 / math.sqrt(d),
+        o_ref, lse_ref, rk, rv = fo.prefill_sequential(*full, ref_L["win_off"], ref_L["keep"], 1.0 / math.sqrt(d),
                                                        want=want_mask)
         for w in want:
             a, e = int(off[w]), int(off[w + 1])

@@ -13,11 +13,11 @@ SRC = os.path.join(os.path.dirname(fo.__file__), "focus_oracle.c")
 
 # (name, exact text in focus_oracle.c, replacement, pin functions that must fail)
 MUTANTS = [
-    ("ring_dropped", "int visible = (win[j] == win[i]) || (kind[j] == 1);",
+    ("ring_dropped", "int visible = (win[j] == win[i]) || (keep[j] == 1);",
      "int visible = (win[j] == win[i]);",
      [lambda: pins.test_lse_of_zero_scores_counts_visible_keys(),
-      lambda: pins.test_attn_matches_streaming_simulation(40, 7, [2], 2, 16)]),
-    ("all_past_visible", "int visible = (win[j] == win[i]) || (kind[j] == 1);",
+      lambda: pins.test_attn_matches_streaming_simulation(40, 7, [2], 2, 16, 0)]),
+    ("all_past_visible", "int visible = (win[j] == win[i]) || (keep[j] == 1);",
      "int visible = 1;",
      [lambda: pins.test_lse_of_zero_scores_counts_visible_keys()]),
     ("strict_causal", "for (int64_t j = 0; j <= i; ++j) {\n            int visible",
@@ -36,9 +36,14 @@ MUTANTS = [
     ("partial_kmer_open", "return (o == n - 1) && close_partial;", "return 0;",
      [lambda: pins.test_layout_fig1_golden(),
       lambda: pins.test_layout_sizes_closed_form(5_000, 1_024, [100])]),
-    ("retain_ordinary", "if (kind[j] != 1) continue;\n            if (R >= ring_cap)",
-     "if (kind[j] != 0) continue;\n            if (R >= ring_cap)",
-     [lambda: pins.test_sequential_equals_masked_parallel(700, 100, [10])]),
+    ("retain_ordinary", "if (keep[j] != 1) continue;\n            if (R >= ring_cap)",
+     "if (keep[j] != 0) continue;\n            if (R >= ring_cap)",
+     [lambda: pins.test_sequential_equals_masked_parallel(700, 100, [10], 0)]),
+    ("tail_off_by_one", "return tail > 0 && o >= n - tail;", "return tail > 0 && o > n - tail;",
+     [lambda: pins.test_layout_tail_counts_closed_form(4_000, 1_000, [100], 3)]),
+    ("tail_not_kept", "keep[t] = (uint8_t)in_tail(o, n, tail);", "keep[t] = 0;",
+     [lambda: pins.test_attn_matches_streaming_simulation(40, 7, [2], 2, 16, 2),
+      lambda: pins.test_tail_covering_every_base_is_causal_over_augmented()]),
     ("decode_skips_self", "        kr[c] = k_new + (size_t)s * d;\n        vr[c] = v_new + (size_t)s * d;\n        c += 1;\n",
      "", [lambda: pins.test_decode_equals_prefill_row()]),
 ]

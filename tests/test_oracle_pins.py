@@ -123,33 +123,55 @@ def test_layout_fig1_golden():
     assert list(L["ring_off"]) == [0, 2, 4, 5]
 
 
-def test_window_summary_rows_match_layout():
-    for n, k in [(1000, 100), (1024, 100), (4, 3), (7, 9), (5, 1)]:
-        L = fo.layout(n, n, [k])
-        assert np.array_equal(fo.window_summary_rows(n, k), np.nonzero(L["kind"] == 1)[0])
+def test_window_retained_rows_match_layout():
+    for n, k, t in [(1000, 100, 0), (1024, 100, 0), (4, 3, 0), (7, 9, 0), (5, 1, 0), (1000, 100, 3), (7, 3, 7),
+                    (10, 4, 1)]:
+        L = fo.layout(n, n, [k], tail=t)
+        assert np.array_equal(fo.window_retained_rows(n, k, True, t), np.nonzero(L["keep"] == 1)[0])
+
+
+@pytest.mark.parametrize("N,W,ks", LAYOUT_CASES)
+@pytest.mark.parametrize("tail", [1, 3, 2_000])
+def test_layout_tail_counts_closed_form(N, W, ks, tail):
+    """Boundary tail (App. A): each window keeps its B_w summaries plus its last
+    min(tail, n_w) bases; the kept bases are the window's last base rows."""
+    M = _ceil(N, W)
+    k = inputs.k_schedule(M, ks, seed=3)
+    L = fo.layout(N, W, k, tail=tail)
+    n_w = [min(W, N - w * W) for w in range(M)]
+    B_w = [(_ceil(n, int(kk)) if kk > 0 else 0) for n, kk in zip(n_w, k)]
+    assert L["R"] == sum(b + min(tail, n) for b, n in zip(B_w, n_w))
+    for w in range(M):
+        a, e = L["win_off"][w], L["win_off"][w + 1]
+        bases = [j for j in range(a, e) if L["kind"][j] == 0]
+        kept_bases = [j for j in range(a, e) if L["kind"][j] == 0 and L["keep"][j] == 1]
+        assert kept_bases == bases[len(bases) - min(tail, len(bases)):]
+    assert np.array_equal(L["keep"][L["kind"] == 1], np.ones(int((L["kind"] == 1).sum()), np.uint8))
 
 
 # ----------------------------------------------------------------------------- attention
 
 
-def _rand_case(N, W, ks, H, d, seed, std=1.0):
+def _rand_case(N, W, ks, H, d, seed, std=1.0, tail=0):
     M = _ceil(N, W)
     k = inputs.k_schedule(M, ks, seed=seed)
-    L = fo.layout(N, W, k)
+    L = fo.layout(N, W, k, tail=tail)
     q, kk, v = inputs.qkv((H, L["T"], d), std=std, seed=seed)
     return L, q, kk, v
 
 
-def _visible_sets_by_streaming(L):
+def _visible_sets_by_streaming(L, tail=0):
     """KV-retention simulation (App. A.2): process windows in order; a row sees
     the retained set plus the current window up to itself; after the window,
-    only FOCUS rows join the retained set."""
+    only its FOCUS rows (and its last `tail` base rows) join the retained set."""
     retained, vis = [], {}
     for w in range(L["M"]):
         a, e = L["win_off"][w], L["win_off"][w + 1]
         for i in range(a, e):
             vis[i] = list(retained) + list(range(a, i + 1))
-        retained += [j for j in range(a, e) if L["kind"][j] == 1]
+        bases = [j for j in range(a, e) if L["kind"][j] == 0]
+        tail_rows = set(bases[len(bases) - min(tail, len(bases)):]) if tail else set()
+        retained += [j for j in range(a, e) if L["kind"][j] == 1 or j in tail_rows]
     return vis
 
 
@@ -168,14 +190,15 @@ ATTN_CASES = [
 
 
 @pytest.mark.parametrize("N,W,ks,H,d", ATTN_CASES)
-def test_attn_matches_streaming_simulation(N, W, ks, H, d):
-    L, q, k, v = _rand_case(N, W, ks, H, d, seed=N + W)
+@pytest.mark.parametrize("tail", [0, 2])
+def test_attn_matches_streaming_simulation(N, W, ks, H, d, tail):
+    L, q, k, v = _rand_case(N, W, ks, H, d, seed=N + W, tail=tail)
     T = L["T"]
     scale = 1.0 / math.sqrt(d)
     heads = np.repeat(np.arange(H), T)
     rows = np.tile(np.arange(T), H)
-    o, lse = fo.attn_rows(q, k, v, L["kind"], L["win"], scale, heads, rows)
-    vis = _visible_sets_by_streaming(L)
+    o, lse = fo.attn_rows(q, k, v, L["keep"], L["win"], scale, heads, rows)
+    vis = _visible_sets_by_streaming(L, tail)
     qd, kd, vd = _f64(q), _f64(k), _f64(v)
     for r, (h, i) in enumerate(zip(heads, rows)):
         j = np.array(vis[i])
@@ -193,7 +216,7 @@ def test_no_compression_is_plain_causal():
     assert L["T"] == N and L["R"] == 0
     heads = np.repeat(np.arange(H), N)
     rows = np.tile(np.arange(N), H)
-    o, lse = fo.attn_rows(q, k, v, L["kind"], L["win"], 1.0 / math.sqrt(d), heads, rows)
+    o, lse = fo.attn_rows(q, k, v, L["keep"], L["win"], 1.0 / math.sqrt(d), heads, rows)
     qd, kd, vd = (x.to(torch.float64) for x in (q, k, v))
     ref = torch.nn.functional.scaled_dot_product_attention(qd, kd, vd, is_causal=True)
     np.testing.assert_allclose(o.reshape(H, N, d), ref.numpy(), rtol=0, atol=1e-12)
@@ -208,9 +231,23 @@ def test_single_window_with_summaries_is_causal_over_augmented():
     T = L["T"]
     heads = np.repeat(np.arange(H), T)
     rows = np.tile(np.arange(T), H)
-    o, _ = fo.attn_rows(q, k, v, L["kind"], L["win"], 0.3, heads, rows)
+    o, _ = fo.attn_rows(q, k, v, L["keep"], L["win"], 0.3, heads, rows)
     ref = torch.nn.functional.scaled_dot_product_attention(
         *(x.to(torch.float64) for x in (q, k, v)), is_causal=True, scale=0.3)
+    np.testing.assert_allclose(o.reshape(H, T, d), ref.numpy(), rtol=0, atol=1e-12)
+
+
+def test_tail_covering_every_base_is_causal_over_augmented():
+    """With a boundary tail at least as long as every window, every row is kept,
+    so every row sees all earlier rows: causal attention over the augmented
+    sequence (library SDPA, fp64)."""
+    N, W, H, d = 70, 16, 2, 16
+    L, q, k, v = _rand_case(N, W, [3], H, d, seed=9, tail=W)
+    T = L["T"]
+    assert L["R"] == T
+    o, lse = fo.attn_rows(q, k, v, L["keep"], L["win"], 0.4, np.repeat(np.arange(H), T), np.tile(np.arange(T), H))
+    ref = torch.nn.functional.scaled_dot_product_attention(
+        *(x.to(torch.float64) for x in (q, k, v)), is_causal=True, scale=0.4)
     np.testing.assert_allclose(o.reshape(H, T, d), ref.numpy(), rtol=0, atol=1e-12)
 
 
@@ -221,7 +258,7 @@ def test_softmax_rows_sum_to_one():
     T = L["T"]
     heads = np.repeat(np.arange(2), T)
     rows = np.tile(np.arange(T), 2)
-    o, _ = fo.attn_rows(q, k, v, L["kind"], L["win"], 1.0, heads, rows)
+    o, _ = fo.attn_rows(q, k, v, L["keep"], L["win"], 1.0, heads, rows)
     assert np.abs(o - 1.0).max() <= 1e-12
 
 
@@ -235,7 +272,7 @@ def test_lse_of_zero_scores_counts_visible_keys():
     T = L["T"]
     q = torch.zeros((1, T, 8), dtype=torch.bfloat16)
     _, k, v = inputs.qkv((1, T, 8), seed=9)
-    o, lse = fo.attn_rows(q, k, v, L["kind"], L["win"], 1.0, np.zeros(T, np.int64), np.arange(T))
+    o, lse = fo.attn_rows(q, k, v, L["keep"], L["win"], 1.0, np.zeros(T, np.int64), np.arange(T))
     w = L["win"]
     count = L["ring_off"][w] + (np.arange(T) - L["win_off"][w]) + 1
     np.testing.assert_allclose(lse, np.log(count), rtol=0, atol=1e-12)
@@ -243,7 +280,7 @@ def test_lse_of_zero_scores_counts_visible_keys():
 
 def test_first_row_sees_only_itself():
     L, q, k, v = _rand_case(30, 10, [3], 1, 8, seed=6)
-    o, lse = fo.attn_rows(q, k, v, L["kind"], L["win"], 0.5, [0], [0])
+    o, lse = fo.attn_rows(q, k, v, L["keep"], L["win"], 0.5, [0], [0])
     assert np.array_equal(o[0], _f64(v)[0, 0])
     assert lse[0] == pytest.approx(0.5 * float(_f64(q)[0, 0] @ _f64(k)[0, 0]), abs=1e-14)
 
@@ -251,16 +288,16 @@ def test_first_row_sees_only_itself():
 # ----------------------------------------------------------------------------- retention / sequential
 
 
-@pytest.mark.parametrize("N,W,ks", [(700, 100, [10]), (1024, 100, [7, 30, 100]), (333, 50, [1, 51]),
-                                    (90, 200, [4])])
-def test_sequential_equals_masked_parallel(N, W, ks):
+@pytest.mark.parametrize("N,W,ks,tail", [(700, 100, [10], 0), (1024, 100, [7, 30, 100], 0), (333, 50, [1, 51], 0),
+                                         (90, 200, [4], 0), (700, 100, [10], 3), (333, 50, [1, 51], 60)])
+def test_sequential_equals_masked_parallel(N, W, ks, tail):
     """App. A.1: sequential windows with KV dropping == masked-parallel."""
     H, d = 2, 16
-    L, q, k, v = _rand_case(N, W, ks, H, d, seed=N)
+    L, q, k, v = _rand_case(N, W, ks, H, d, seed=N, tail=tail)
     T = L["T"]
     for h in range(H):
-        o_s, lse_s, rk, rv = fo.prefill_sequential(q[h], k[h], v[h], L["win_off"], L["kind"], 0.25)
-        o_p, lse_p = fo.attn_rows(q, k, v, L["kind"], L["win"], 0.25, np.full(T, h), np.arange(T))
+        o_s, lse_s, rk, rv = fo.prefill_sequential(q[h], k[h], v[h], L["win_off"], L["keep"], 0.25)
+        o_p, lse_p = fo.attn_rows(q, k, v, L["keep"], L["win"], 0.25, np.full(T, h), np.arange(T))
         np.testing.assert_allclose(o_s, o_p, rtol=0, atol=1e-12)
         np.testing.assert_allclose(lse_s, lse_p, rtol=0, atol=1e-12)
         # retained KV == the FOCUS rows, bit for bit, count == sum_w B_w
@@ -275,7 +312,7 @@ def test_retained_count_after_n_windows():
     W, k, H, d = 200, 20, 1, 8
     for n in (1, 2, 5):
         L, q, kk, v = _rand_case(n * W, W, [k], H, d, seed=n)
-        _, _, rk, _ = fo.prefill_sequential(q[0], kk[0], v[0], L["win_off"], L["kind"], 1.0,
+        _, _, rk, _ = fo.prefill_sequential(q[0], kk[0], v[0], L["win_off"], L["keep"], 1.0,
                                             want=np.zeros(L["M"]))
         assert rk.shape[0] == n * W // k
 
@@ -291,7 +328,7 @@ def test_decode_equals_prefill_row():
     rng = np.random.default_rng(0)
     ts = rng.integers(0, L["T"], size=24)
     for h in range(H):
-        o_p, lse_p = fo.attn_rows(q, k, v, L["kind"], L["win"], 0.2, np.full(ts.size, h), ts)
+        o_p, lse_p = fo.attn_rows(q, k, v, L["keep"], L["win"], 0.2, np.full(ts.size, h), ts)
         for r, t in enumerate(ts):
             w = L["win"][t]
             ring_rows = L["sum_idx"][: L["ring_off"][w]]
