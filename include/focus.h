@@ -113,7 +113,8 @@ typedef struct focus_layout_out {
 /* Device layout builder. d_k: DEVICE array [M] of cadences (same values as the
  * host array given to focus_layout_size). d_nt: DEVICE uint8 [B][N] nucleotide ids
  * (may be NULL, then tok is not written). If the device-computed T or R differs
- * from out->T / out->R the device status word is set to FOCUS_ERR_LAYOUT. */
+ * from out->T / out->R the device status word is set to FOCUS_ERR_LAYOUT.
+ * N = 0 (M = 0) is valid: it only writes win_off[0] = ring_off[0] = 0. */
 focus_status focus_layout(int64_t n_nt, int32_t W, int32_t n_windows, const int32_t* d_k,
                           uint32_t flags, int32_t tail, int32_t B, const uint8_t* d_nt,
                           const focus_layout_out* out, cudaStream_t stream);

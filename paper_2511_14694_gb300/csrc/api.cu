@@ -107,7 +107,15 @@ focus_status focus_layout(int64_t n_nt, int32_t W, int32_t n_windows, const int3
                           int32_t tail, int32_t B, const uint8_t* d_nt, const focus_layout_out* out,
                           cudaStream_t stream) {
     if (!out || n_nt < 0 || W <= 0 || B < 0 || tail < 0) return FOCUS_ERR_INVALID_ARG;
-    if ((int64_t)n_windows != focus::ceil_div64(n_nt, W) || n_windows <= 0 || !d_k) return FOCUS_ERR_INVALID_ARG;
+    if ((int64_t)n_windows != focus::ceil_div64(n_nt, W)) return FOCUS_ERR_INVALID_ARG;
+    if (n_nt == 0) {                                   // empty sequence: nothing to lay out
+        if (out->T != 0 || out->R != 0) return FOCUS_ERR_INVALID_ARG;
+        if (!out->win_off || !out->ring_off) return FOCUS_ERR_INVALID_ARG;
+        cudaError_t e = cudaMemsetAsync(out->win_off, 0, sizeof(int32_t), stream);
+        if (e == cudaSuccess) e = cudaMemsetAsync(out->ring_off, 0, sizeof(int32_t), stream);
+        return from_cuda(e);
+    }
+    if (!d_k) return FOCUS_ERR_INVALID_ARG;
     if (out->T < 0 || out->R < 0 || out->T > INT32_MAX) return FOCUS_ERR_INVALID_ARG;
     if (!out->win_off || !out->ring_off) return FOCUS_ERR_INVALID_ARG;
     if (out->T > 0 && (!out->kind || !out->src || !out->pos || !out->win)) return FOCUS_ERR_INVALID_ARG;

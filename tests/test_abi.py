@@ -85,3 +85,20 @@ def test_host_validation_rejects_bad_arguments():
     # null q/k/v
     assert lib.focus_attn_prefill(ctypes.byref(c), ctypes.byref(a), None) == 1
     assert lib.focus_decode_workspace_size(None) == 0
+
+
+def test_layout_size_edge_cases():
+    lib = focus.load()
+    T, R, mx = ctypes.c_int64(-1), ctypes.c_int64(-1), ctypes.c_int32(-1)
+    # empty sequence: M = 0, nothing to lay out
+    assert lib.focus_layout_size(0, 1000, 0, None, 1, 0, ctypes.byref(T), ctypes.byref(R), ctypes.byref(mx)) == 0
+    assert (T.value, R.value, mx.value) == (0, 0, 0)
+    # single base, single window
+    k = np.array([1], np.int32)
+    assert lib.focus_layout_size(1, 1, 1, k.ctypes.data, 1, 0, ctypes.byref(T), ctypes.byref(R), None) == 0
+    assert (T.value, R.value) == (2, 1)
+    # an augmented length beyond int32 offsets is refused, not truncated
+    M = 2_000
+    kk = np.ones(M, np.int32)
+    assert lib.focus_layout_size(2_000_000_000, 1_000_000, M, kk.ctypes.data, 1, 0, ctypes.byref(T), None,
+                                 None) == 2

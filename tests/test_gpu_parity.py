@@ -246,6 +246,24 @@ def test_decode_full_window_is_reported_not_trapped():
     assert int(cache.win_fill[0]) == 11
 
 
+def test_layout_empty_sequence():
+    L = focus.layout(0, 1_000, [100])
+    assert (L["T"], L["R"], L["M"]) == (0, 0, 0)
+    assert L["win_off_host"].tolist() == [0] and L["ring_off_host"].tolist() == [0]
+
+
+def test_bulk_compaction_overflow_is_reported_not_trapped():
+    N, W, H, d = 4_000, 1_000, 2, 64
+    L = focus.layout(N, W, [100])
+    cache = focus.Cache(1, H, d, C_ring=L["R"] - 1)
+    k = inputs.normal_bf16((1, H, L["T"], d), 1.0, seed=3, device="cuda")
+    v = inputs.normal_bf16((1, H, L["T"], d), 1.0, seed=4, device="cuda")
+    focus.kv_compact_bulk(cache, k, v, L)
+    assert focus.device_status(clear=True) == 3   # FOCUS_ERR_CAPACITY
+    assert int(cache.ring_len[0]) == 0
+    assert not cache.ring_k.any()
+
+
 # ----------------------------------------------------------------------------- full-size workloads, sampled rows
 
 def _sample_rows(L, n_windows, rows_per_window, seed):
