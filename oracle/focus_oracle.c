@@ -320,3 +320,76 @@ int32_t fo_window_retained_rows(int64_t n, int32_t k, int32_t close_partial, int
     }
     return c;
 }
+
+/* ------------------------------------------------------------------------- */
+/* k-mer membership (Sec. 3.2 "Setup and tokens": a base belongs to exactly   */
+/* one k-mer; the FOCUS token S_i closes the k-mer B_i to its left). kmer[t] */
+/* is the 0-based index, within its window, of the k-mer row t belongs to: a  */
+/* base's own k-mer, or for a FOCUS token the k-mer it summarises. With k = 0 */
+/* (no summaries) the whole window is one segment, index 0. Returns T or -1.  */
+/* ------------------------------------------------------------------------- */
+int64_t fo_layout_kmer(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
+                       int32_t close_tail, int32_t* kmer) {
+    if (fo_layout_size(N, W, M, k_sched, close_tail, 0, NULL) < 0) return -1;
+    int64_t t = 0;
+    for (int32_t w = 0; w < M; ++w) {
+        int64_t start = (int64_t)w * W;
+        int64_t n = (N - start < W) ? (N - start) : W;
+        int close = (w < M - 1) || close_tail;
+        int32_t c = 0;
+        for (int64_t o = 0; o < n; ++o) {
+            kmer[t++] = c;
+            if (summary_after(o, n, k_sched[w], close)) {
+                kmer[t++] = c;
+                c += 1;
+            }
+        }
+    }
+    return t;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Main-text visibility (Sec. 3.2 "Visibility and summarization rule"), the  */
+/* k-mer-local mask. Row i of window w sees key j <= i iff                     */
+/*   - j is in window w and in the same k-mer as i (a base sees the earlier   */
+/*     bases of its own k-mer; a FOCUS token sees the k bases it summarises), */
+/*   - or j is a FOCUS token of window w (the preceding in-window summaries), */
+/*   - or j is the carried boundary of window w: the last FOCUS token of      */
+/*     window w-1 (S_{m,1} == S_{m-1,W}, "Windowing with a shared boundary"). */
+/* Nothing else of earlier windows is visible. kind/win/kmer: the layout's   */
+/* per-row arrays. Same row selection and outputs as fo_attn_rows.            */
+/* ------------------------------------------------------------------------- */
+void fo_attn_rows_kmer_local(int64_t T, int32_t d, const uint8_t* kind, const int32_t* win,
+                             const int32_t* kmer, const uint16_t* q, const uint16_t* k,
+                             const uint16_t* v, double scale, int64_t n_rows,
+                             const int64_t* row_head, const int64_t* row_idx, double* o,
+                             double* lse) {
+    int32_t M = T > 0 ? win[T - 1] + 1 : 0;
+    int64_t* last_focus = (int64_t*)malloc(sizeof(int64_t) * (size_t)(M > 0 ? M : 1));
+    for (int32_t w = 0; w < M; ++w) last_focus[w] = -1;
+    for (int64_t j = 0; j < T; ++j)
+        if (kind[j] == 1) last_focus[win[j]] = j;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t r = 0; r < n_rows; ++r) {
+        int64_t h = row_head[r], i = row_idx[r];
+        const uint16_t* kh = k + (size_t)h * (size_t)T * (size_t)d;
+        const uint16_t* vh = v + (size_t)h * (size_t)T * (size_t)d;
+        const uint16_t** kr = (const uint16_t**)malloc(sizeof(void*) * (size_t)(i + 1));
+        const uint16_t** vr = (const uint16_t**)malloc(sizeof(void*) * (size_t)(i + 1));
+        int64_t boundary = win[i] >= 1 ? last_focus[win[i] - 1] : -1;
+        int64_t n = 0;
+        for (int64_t j = 0; j <= i; ++j) {
+            int same_window = win[j] == win[i];
+            int visible = (same_window && kmer[j] == kmer[i]) || (same_window && kind[j] == 1) || j == boundary;
+            if (!visible) continue;
+            kr[n] = kh + (size_t)j * d;
+            vr[n] = vh + (size_t)j * d;
+            n += 1;
+        }
+        softmax_row(d, q + ((size_t)h * (size_t)T + (size_t)i) * d, n, kr, vr, scale,
+                    o + (size_t)r * d, lse + r);
+        free(kr);
+        free(vr);
+    }
+    free(last_focus);
+}

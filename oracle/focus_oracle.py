@@ -57,6 +57,10 @@ def _load(path: str | None = None):
     lib.fo_prefill_sequential.argtypes = [i32, i32, P, P, P, P, P, f64, P, P, P, P, P, i64, P]
     lib.fo_decode.restype = None
     lib.fo_decode.argtypes = [i32, i64, P, P, i64, P, P, P, i64, P, P, P, P, f64, P, P]
+    lib.fo_layout_kmer.restype = i64
+    lib.fo_layout_kmer.argtypes = [i64, i32, i32, P, i32, P]
+    lib.fo_attn_rows_kmer_local.restype = None
+    lib.fo_attn_rows_kmer_local.argtypes = [i64, i32, P, P, P, P, P, P, f64, i64, P, P, P, P]
     lib.fo_window_retained_rows.restype = i32
     lib.fo_window_retained_rows.argtypes = [i64, i32, i32, i32, P, i32]
     _lib = lib
@@ -167,6 +171,45 @@ def attn_rows(q, k, v, keep, win, scale: float, heads, rows):
     lse = np.zeros(n, np.float64)
     lib.fo_attn_rows(T, d, _ptr(keep), _ptr(win), _ptr(qb), _ptr(kb), _ptr(vb), float(scale),
                      n, _ptr(heads), _ptr(rows), _ptr(o), _ptr(lse))
+    return o, lse
+
+
+def layout_kmer(N: int, W: int, k_sched, close_tail: bool = True) -> np.ndarray:
+    """In-window k-mer index of every augmented row (Sec. 3.2 "Setup and
+    tokens"): a base's own k-mer, the summarised k-mer for a FOCUS row; 0 for
+    every row of a window with k = 0."""
+    lib = _load()
+    T, _, M = layout_size(N, W, k_sched, close_tail)
+    k = _k_array(M, k_sched)
+    out = np.zeros(max(T, 1), np.int32)
+    t = lib.fo_layout_kmer(N, W, M, _ptr(k), int(close_tail), _ptr(out))
+    if t < 0:
+        raise ValueError("bad layout arguments")
+    return out[:T]
+
+
+def attn_rows_kmer_local(q, k, v, kind, win, kmer, scale: float, heads, rows):
+    """Attention at selected rows under the main text's k-mer-local visibility
+    (Sec. 3.2 "Visibility and summarization rule"): own k-mer (causal), the
+    window's FOCUS rows, and the carried boundary (last FOCUS row of the previous
+    window). Arguments and outputs as in ``attn_rows``; ``kind``/``win``/``kmer``
+    are the layout's per-row arrays."""
+    lib = _load()
+    qb, kb, vb = _bits(q), _bits(k), _bits(v)
+    nh, T, d = qb.shape
+    kind = np.ascontiguousarray(kind, dtype=np.uint8)
+    win = np.ascontiguousarray(win, dtype=np.int32)
+    kmer = np.ascontiguousarray(kmer, dtype=np.int32)
+    assert kind.shape == (T,) and win.shape == (T,) and kmer.shape == (T,)
+    heads = np.ascontiguousarray(heads, dtype=np.int64)
+    rows = np.ascontiguousarray(rows, dtype=np.int64)
+    assert heads.shape == rows.shape
+    assert heads.size == 0 or (heads.min() >= 0 and heads.max() < nh and rows.min() >= 0 and rows.max() < T)
+    n = rows.size
+    o = np.zeros((n, d), np.float64)
+    lse = np.zeros(n, np.float64)
+    lib.fo_attn_rows_kmer_local(T, d, _ptr(kind), _ptr(win), _ptr(kmer), _ptr(qb), _ptr(kb), _ptr(vb),
+                                float(scale), n, _ptr(heads), _ptr(rows), _ptr(o), _ptr(lse))
     return o, lse
 
 

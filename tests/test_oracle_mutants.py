@@ -44,6 +44,24 @@ MUTANTS = [
     ("tail_not_kept", "keep[t] = (uint8_t)in_tail(o, n, tail);", "keep[t] = 0;",
      [lambda: pins.test_attn_matches_streaming_simulation(40, 7, [2], 2, 16, 2),
       lambda: pins.test_tail_covering_every_base_is_causal_over_augmented()]),
+    ("kmer_focus_in_next_kmer", "kmer[t++] = c;\n                c += 1;", "c += 1;\n                kmer[t++] = c;",
+     [lambda: pins.test_kmer_ids_closed_form(4_000, 1_000, [100]),
+      lambda: pins.test_kmer_local_lse_of_zero_scores_counts_visible_keys()]),
+    ("local_no_boundary", "|| (same_window && kind[j] == 1) || j == boundary;", "|| (same_window && kind[j] == 1);",
+     [lambda: pins.test_kmer_local_lse_of_zero_scores_counts_visible_keys(),
+      lambda: pins.test_kmer_local_equals_appendix_mask_for_two_single_kmer_windows()]),
+    ("local_all_focus_rows", "|| (same_window && kind[j] == 1) || j == boundary;", "|| kind[j] == 1;",
+     [lambda: pins.test_kmer_local_lse_of_zero_scores_counts_visible_keys(),
+      lambda: pins.test_kmer_local_invisible_rows_do_not_matter_and_visible_ones_do()]),
+    ("local_no_in_window_focus", "|| (same_window && kind[j] == 1) || j == boundary;", "|| j == boundary;",
+     [lambda: pins.test_kmer_local_lse_of_zero_scores_counts_visible_keys(),
+      lambda: pins.test_kmer_local_invisible_rows_do_not_matter_and_visible_ones_do()]),
+    ("local_whole_window", "int visible = (same_window && kmer[j] == kmer[i])", "int visible = (same_window)",
+     [lambda: pins.test_kmer_local_lse_of_zero_scores_counts_visible_keys(),
+      lambda: pins.test_kmer_local_invisible_rows_do_not_matter_and_visible_ones_do()]),
+    ("boundary_is_first_focus", "if (kind[j] == 1) last_focus[win[j]] = j;",
+     "if (kind[j] == 1 && last_focus[win[j]] < 0) last_focus[win[j]] = j;",
+     [lambda: pins.test_kmer_local_invisible_rows_do_not_matter_and_visible_ones_do()]),
     ("decode_skips_self", "        kr[c] = k_new + (size_t)s * d;\n        vr[c] = v_new + (size_t)s * d;\n        c += 1;\n",
      "", [lambda: pins.test_decode_equals_prefill_row()]),
 ]

@@ -354,3 +354,130 @@ def test_decode_ring_order_is_irrelevant():
     o2, l2 = fo.decode(q, kn, vn, ring_k[:, perm], ring_v[:, perm], [R] * n, win_k, win_v, [F] * n, 0.3)
     np.testing.assert_allclose(o1, o2, rtol=0, atol=1e-12)
     np.testing.assert_allclose(l1, l2, rtol=0, atol=1e-12)
+
+
+# ----------------------------------------------------------------------------- k-mer-local visibility (main text)
+
+def _local_case(N, W, ks, H, d, seed, std=1.0):
+    M = _ceil(N, W)
+    k = inputs.k_schedule(M, ks, seed=seed)
+    L = fo.layout(N, W, k)
+    L["k"] = k
+    L["kmer"] = fo.layout_kmer(N, W, k)
+    q, kk, v = inputs.qkv((H, L["T"], d), std=std, seed=seed)
+    return L, q, kk, v
+
+
+def _local(q, k, v, L, scale, heads, rows):
+    return fo.attn_rows_kmer_local(q, k, v, L["kind"], L["win"], L["kmer"], scale, heads, rows)
+
+
+@pytest.mark.parametrize("N,W,ks", LAYOUT_CASES)
+def test_kmer_ids_closed_form(N, W, ks):
+    """A window's rows come in blocks of k + 1 (k bases, then their FOCUS token),
+    the last block possibly shorter: row at in-window offset a belongs to k-mer
+    floor(a / (k + 1)); a window without summaries is one block."""
+    M = _ceil(N, W)
+    k = inputs.k_schedule(M, ks, seed=5)
+    L = fo.layout(N, W, k)
+    km = fo.layout_kmer(N, W, k)
+    w = L["win"]
+    a = np.arange(L["T"]) - L["win_off"][w]
+    kw = k[w].astype(np.int64)
+    expect = np.where(kw > 0, a // np.maximum(kw + 1, 1), 0)
+    assert np.array_equal(km, expect)
+
+
+def test_kmer_local_lse_of_zero_scores_counts_visible_keys():
+    """q = 0 => LSE_i = ln |visible(i)|. Under the main-text rule a row at offset
+    a of k-mer c (= a // (k+1)) of window w sees the a - c(k+1) + 1 rows of its
+    k-mer up to itself, the c FOCUS rows of the earlier k-mers of its window, and
+    the carried boundary when window w-1 has a FOCUS row (k_{w-1} > 0)."""
+    N, W, ks = 700, 60, [1, 7, 13, 0, 60, 100]
+    M = _ceil(N, W)
+    kk = inputs.k_schedule(M, ks, seed=8)
+    L = fo.layout(N, W, kk)
+    km = fo.layout_kmer(N, W, kk)
+    T = L["T"]
+    q = torch.zeros((1, T, 8), dtype=torch.bfloat16)
+    _, k, v = inputs.qkv((1, T, 8), seed=9)
+    _, lse = fo.attn_rows_kmer_local(q, k, v, L["kind"], L["win"], km, 1.0, np.zeros(T, np.int64), np.arange(T))
+    w = L["win"]
+    a = np.arange(T) - L["win_off"][w]
+    kw = kk[w].astype(np.int64)
+    c = np.where(kw > 0, a // np.maximum(kw + 1, 1), 0)
+    in_kmer = a - c * (kw + 1) + 1
+    boundary = (w >= 1) & (kk[np.maximum(w - 1, 0)] > 0)
+    count = in_kmer + c + boundary
+    np.testing.assert_allclose(lse, np.log(count), rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("k", [0, 64, 1_000])
+def test_kmer_local_single_kmer_window_is_causal(k):
+    """One window whose only k-mer spans it (k = 0, or k >= N): every row sees
+    every earlier row, i.e. causal attention over the augmented sequence
+    (library SDPA, fp64)."""
+    N, H, d = 57, 2, 16
+    L, q, kk, v = _local_case(N, 64, [k], H, d, seed=21)
+    T = L["T"]
+    o, lse = _local(q, kk, v, L, 0.35, np.repeat(np.arange(H), T), np.tile(np.arange(T), H))
+    ref = torch.nn.functional.scaled_dot_product_attention(
+        *(x.to(torch.float64) for x in (q, kk, v)), is_causal=True, scale=0.35)
+    np.testing.assert_allclose(o.reshape(H, T, d), ref.numpy(), rtol=0, atol=1e-12)
+
+
+def test_kmer_local_equals_appendix_mask_for_two_single_kmer_windows():
+    """With k >= W every window is one k-mer closed by one FOCUS row; with two
+    windows the only retained row before window 1 is window 0's FOCUS row, which
+    is also the carried boundary, so both visibility rules give the same sets
+    (the appendix form is pinned independently above)."""
+    N, W, H, d = 90, 50, 2, 16
+    L, q, kk, v = _local_case(N, W, [50], H, d, seed=22)
+    assert L["M"] == 2 and L["R"] == 2
+    T = L["T"]
+    heads, rows = np.repeat(np.arange(H), T), np.tile(np.arange(T), H)
+    o1, l1 = _local(q, kk, v, L, 0.25, heads, rows)
+    o2, l2 = fo.attn_rows(q, kk, v, L["keep"], L["win"], 0.25, heads, rows)
+    np.testing.assert_allclose(o1, o2, rtol=0, atol=1e-13)
+    np.testing.assert_allclose(l1, l2, rtol=0, atol=1e-13)
+
+
+def _perturb_rows(x, rows, seed):
+    y = x.clone()
+    g = torch.Generator().manual_seed(seed)
+    y[:, rows] = torch.randn(y[:, rows].shape, generator=g).to(y.dtype) * 3
+    return y
+
+
+def test_kmer_local_invisible_rows_do_not_matter_and_visible_ones_do():
+    """Main text: earlier windows' rows are reachable only through the carried
+    boundary, and a row does not see the bases of other k-mers. Rewriting the
+    K/V of every other earlier row leaves window w's outputs bit-identical;
+    rewriting the boundary, or an earlier in-window FOCUS row, changes them."""
+    N, W, H, d = 300, 60, 1, 16
+    L, q, kk, v = _local_case(N, W, [10], H, d, seed=23)
+    w = 3
+    a, e = int(L["win_off"][w]), int(L["win_off"][w + 1])
+    rows = np.arange(a, e)
+    heads = np.zeros(rows.size, np.int64)
+    o0, l0 = _local(q, kk, v, L, 0.25, heads, rows)
+    prev = np.arange(int(L["win_off"][w - 1]), a)
+    boundary = int(prev[L["kind"][prev] == 1][-1])
+    assert boundary == a - 1
+    hidden = [j for j in range(a) if j != boundary]
+    # bases of the window's first k-mer are hidden from the rows of its later k-mers
+    later = rows[L["kmer"][rows] >= 1]
+    first_bases = [j for j in range(a, e) if L["kmer"][j] == 0 and L["kind"][j] == 0]
+    o1, l1 = _local(_perturb_rows(q, [], 1), _perturb_rows(kk, hidden, 2), _perturb_rows(v, hidden, 3), L, 0.25,
+                    heads, rows)
+    assert np.array_equal(o0, o1) and np.array_equal(l0, l1)
+    ol0, _ = _local(q, kk, v, L, 0.25, np.zeros(later.size, np.int64), later)
+    ol1, _ = _local(q, _perturb_rows(kk, first_bases, 4), _perturb_rows(v, first_bases, 5), L, 0.25,
+                    np.zeros(later.size, np.int64), later)
+    assert np.array_equal(ol0, ol1)
+    ob, _ = _local(q, _perturb_rows(kk, [boundary], 6), _perturb_rows(v, [boundary], 7), L, 0.25, heads, rows)
+    assert np.abs(ob - o0).max(axis=1).min() > 0          # every row of window w sees the boundary
+    first_focus = [j for j in range(a, e) if L["kmer"][j] == 0 and L["kind"][j] == 1]
+    of, _ = _local(q, _perturb_rows(kk, first_focus, 8), _perturb_rows(v, first_focus, 9), L, 0.25,
+                   np.zeros(later.size, np.int64), later)
+    assert np.abs(of - ol0).max(axis=1).min() > 0         # every later k-mer sees the first FOCUS row
