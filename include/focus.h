@@ -165,12 +165,30 @@ typedef struct focus_prefill_args {
  * comparison baseline; same results within rounding). */
 #define FOCUS_PREFILL_LEGACY_MMA 1u
 
+/* Main-text k-mer-local visibility (Sec. 3.2 "Visibility and summarization rule")
+ * instead of the appendix mask. Row a of window w, in k-mer c = a / (k_w + 1)
+ * (the whole window is one k-mer when k_w = 0), sees
+ *   - window rows [c (k_w + 1), a]: the earlier rows of its own k-mer and itself,
+ *   - the FOCUS rows of k-mers 0..c-1 of window w, read from the ring at rows
+ *     [ring_off[w], ring_off[w] + c),
+ *   - the carried boundary, ring row ring_off[w] - 1, when window w-1 has FOCUS
+ *     rows (its last FOCUS row, S_{m,1} = S_{m-1,W}),
+ * and nothing else. Requires cache->k_per_window (device [n_windows], the
+ * layout's k schedule, n_windows >= w_end), cache->tail == 0 and a layout built
+ * with tail 0 (FOCUS_ERR_UNSUPPORTED otherwise), and the FOCUS rows of windows
+ * w_begin-1 .. w_end-1 already in the ring: compact before this call, also when
+ * streaming. Not combinable with FOCUS_PREFILL_LEGACY_MMA (FOCUS_ERR_UNSUPPORTED). */
+#define FOCUS_PREFILL_KMER_LOCAL 2u
+
 /* Row a of window w (a = in-window augmented offset) gets
  *   o = softmax_j(scale * q·k_j) v_j over j ∈ ring[0, ring_off[w]) ∪ window rows [0, a]
  * and lse = ln Σ_j exp(scale * q·k_j). The ring rows are cache->ring_k/ring_v of the
  * same (b, h); ring_off[w] <= C_ring is required for every window of the span.
  * Masked-parallel use: bulk-compact all summaries first, then one call over all
- * windows. Streaming use: one call per window, then compact that window. */
+ * windows. Streaming use: one call per window, then compact that window.
+ * Keys are read in 128-row tiles and masked keys get weight 0, so every row of
+ * ring_k/ring_v [0, C_ring) and of k/v [0, T_span) must hold finite values (a
+ * zero-initialised cache does). Unknown flag bits: FOCUS_ERR_INVALID_ARG. */
 focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_args* args,
                                 cudaStream_t stream);
 

@@ -7,6 +7,15 @@
 // is analytic per 128-key tile: only the last partial ring tile (key >= R_w)
 // and the diagonal window tile (key > row) are masked.
 //
+// k-mer-local mode (LOCAL; Sec. 3.2 "Visibility and summarization rule"): row a
+// of k-mer c = a / (k_w + 1) sees the rows [c (k_w + 1), a] of its own k-mer, the
+// FOCUS rows of k-mers 0..c-1 of its window and the carried boundary (the last
+// FOCUS row of window w-1). The ring already holds window w's own FOCUS rows
+// right after the boundary, so the CTA reads ring rows
+// [ring_off[w] - boundary, ring_off[w] + c_last) and window rows from the first
+// row of its first k-mer to its last row; each row's visible keys are one
+// interval per tile.
+//
 // CTA = two 128-row Q tiles of one (sequence, head, window) that share every
 // K/V tile, 12 warps in three warpgroups:
 //   warp 0     TMA producer: Q tiles once, then K_j, V_j into a ring of slots
@@ -71,13 +80,14 @@ __device__ __forceinline__ void fail(Bars* bars, int32_t* status) {
 }
 __device__ __forceinline__ bool aborted(Bars* bars) { return *(volatile int32_t*)&bars->abort != 0; }
 
-template <int D>
+template <int D, bool LOCAL>
 __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
         const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
         const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_rk,
         const __grid_constant__ CUtensorMap tm_rv, __nv_bfloat16* __restrict__ o, float* __restrict__ lse,
         int64_t T_span, const int32_t* __restrict__ win_off, const int32_t* __restrict__ ring_off, int32_t w_begin,
-        int32_t w_end, int32_t ctas_pw, int32_t H, int32_t C_ring, float scale_log2, int32_t* status) {
+        int32_t w_end, int32_t ctas_pw, int32_t H, int32_t C_ring, float scale_log2, int32_t* status,
+        const int32_t* __restrict__ k_per_window) {
     using C = Cfg<D>;
     extern __shared__ unsigned char smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -97,15 +107,31 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
     // systematic stall costs one wave of bounded waits, not one per wave.
     if (*(volatile int32_t*)status == FOCUS_ERR_TIMEOUT) return;
     const int32_t Rw = ring_off[w];
-    if (Rw > C_ring || (int64_t)(win_off[w_end] - w0) > T_span) {
+    // LOCAL: k-mer length + 1 (a window without summaries, or with k >= T_w, is one
+    // k-mer), boundary present?, key ranges [ring_lo, ...) and [win_lo, ...)
+    int32_t kdiv = 1, bnd = 0, ring_lo = 0, win_lo = 0, ring_hi = Rw;
+    int n_ring, n_win = 0;
+    if (LOCAL) {
+        const int32_t kw = k_per_window[w];
+        kdiv = (kw > 0 && kw < Tw ? kw : Tw) + 1;
+        bnd = (w >= 1 && ring_off[w - 1] < Rw) ? 1 : 0;
+        const int32_t a_last = (a0 + 2 * BM < Tw ? a0 + 2 * BM : Tw) - 1;
+        ring_lo = Rw - bnd;
+        ring_hi = Rw + a_last / kdiv;
+        win_lo = (a0 / kdiv) * kdiv;
+        n_ring = (ring_hi - ring_lo + BN - 1) / BN;
+        n_win = (a_last + 1 - win_lo + BN - 1) / BN;
+    } else {
+        n_ring = (Rw + BN - 1) / BN;
+    }
+    if (ring_hi > C_ring || (int64_t)(win_off[w_end] - w0) > T_span) {
         if (threadIdx.x == 0) report(status, FOCUS_ERR_CAPACITY);
         return;
     }
     const int32_t row_base = win_off[w] - w0;           // first row of the window in the span tensors
-    const int n_ring = (Rw + BN - 1) / BN;
     const bool valid1 = a0 + BM < Tw;
-    const int n_kv0 = n_ring + 2 * cta + 1;
-    const int n_kv1 = valid1 ? n_ring + 2 * cta + 2 : 0;
+    const int n_kv0 = LOCAL ? n_ring + n_win : n_ring + 2 * cta + 1;
+    const int n_kv1 = valid1 ? (LOCAL ? n_ring + n_win : n_ring + 2 * cta + 2) : 0;
     const int n_kv_max = valid1 ? n_kv1 : n_kv0;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -152,7 +178,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
             int issued = 0;
             for (int j = 0; j < n_kv_max && !aborted(bars); ++j) {
                 const bool ring = j < n_ring;
-                const int32_t row = ring ? j * BN : row_base + (j - n_ring) * BN;
+                const int32_t row = ring ? ring_lo + j * BN : row_base + win_lo + (j - n_ring) * BN;
                 for (int part = 0; part < 2; ++part) {
                     const int n = 2 * j + part, slot = n % kSlots, use = n / kSlots;
                     if (use > 0 && !mbar_wait(smem_addr(&bars->kv_empty[slot]), (use - 1) & 1, kWaitNs)) {
@@ -240,6 +266,11 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
         const uint32_t lane_addr = (uint32_t)(quarter * 32) << 16;
         const uint32_t s_addr = tmem + lane_addr + t * 128;
         const uint32_t o_addr = tmem + lane_addr + 256 + t * D;
+        // LOCAL: the row's k-mer starts at in-window row lo_row; it sees ring keys
+        // [ring_lo, ring_lo + ring_lim) (boundary + earlier in-window FOCUS rows)
+        const int32_t c_row = LOCAL ? aq / kdiv : 0;
+        const int32_t lo_row = c_row * kdiv;
+        const int32_t ring_lim = c_row + bnd;
         float m_run = -INFINITY, l_run = 0.f;
         bool ok = true;
         for (int j = 0; j < n_kv; ++j) {
@@ -254,7 +285,22 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
             float* s = reinterpret_cast<float*>(sr);
             // analytic mask
             const bool ring = j < n_ring;
-            if (ring) {
+            if (LOCAL) {                                  // visible keys of this tile: columns [lo, hi]
+                int32_t lo, hi;
+                if (ring) {
+                    lo = 0;
+                    hi = ring_lim - j * BN - 1;
+                } else {
+                    const int32_t base = win_lo + (j - n_ring) * BN;
+                    lo = lo_row - base;
+                    hi = aq - base;
+                }
+                if (lo > 0 || hi < BN - 1) {
+#pragma unroll
+                    for (int c = 0; c < BN; ++c)
+                        if (c < lo || c > hi) s[c] = -INFINITY;
+                }
+            } else if (ring) {
                 const int lim = Rw - j * BN;              // keys [0, lim) of this tile are visible
                 if (lim < BN) {
 #pragma unroll
@@ -284,7 +330,10 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
             l_run *= factor;
             // p = 2^(s * scale_log2 - m): packed FMA on pairs, ex2 per element, row sum in
             // four packed partial sums (independent chains)
-            const uint64_t sc2 = f2_pack(scale_log2, scale_log2), nm2 = f2_pack(-m_run, -m_run);
+            // LOCAL rows can meet tiles with no visible key before their first one:
+            // subtract 0 instead of -inf there (every p is then exactly 0)
+            const float m_sub = (LOCAL && m_run == -INFINITY) ? 0.f : m_run;
+            const uint64_t sc2 = f2_pack(scale_log2, scale_log2), nm2 = f2_pack(-m_sub, -m_sub);
             uint64_t acc2[4] = {0, 0, 0, 0};
 #pragma unroll
             for (int h2 = 0; h2 < 2; ++h2) {
@@ -408,7 +457,7 @@ cudaError_t make_map(CUtensorMap* m, const void* ptr, int d, int64_t rows, int64
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-template <int D>
+template <int D, bool LOCAL>
 cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t* status, cudaStream_t stream) {
     const int64_t BH = (int64_t)c.B * c.H;
     CUtensorMap tq, tk, tv, trk, trv;
@@ -424,14 +473,13 @@ cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t*
         trv = tv;
     }
     const int smem = Cfg<D>::kSmem;
-    e = cudaFuncSetAttribute(prefill_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    e = cudaFuncSetAttribute(prefill_tc_kernel<D, LOCAL>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     const int ctas_pw = (a.max_rows + 2 * BM - 1) / (2 * BM);
     dim3 grid((unsigned)((a.w_end - a.w_begin) * ctas_pw), c.H, c.B);
-    prefill_tc_kernel<D><<<grid, kThreads, smem, stream>>>(tq, tk, tv, trk, trv, (__nv_bfloat16*)a.o, a.lse,
-                                                          a.T_span, a.d_win_off, a.d_ring_off, a.w_begin, a.w_end,
-                                                          ctas_pw, c.H, c.C_ring, a.scale * 1.4426950408889634f,
-                                                          status);
+    prefill_tc_kernel<D, LOCAL><<<grid, kThreads, smem, stream>>>(
+        tq, tk, tv, trk, trv, (__nv_bfloat16*)a.o, a.lse, a.T_span, a.d_win_off, a.d_ring_off,
+        a.w_begin, a.w_end, ctas_pw, c.H, c.C_ring, a.scale * 1.4426950408889634f, status, c.k_per_window);
     return cudaGetLastError();
 }
 
@@ -439,8 +487,9 @@ cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t*
 
 cudaError_t launch_prefill_tc(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
                               cudaStream_t stream) {
-    if (c.d == 128) return launch_d<128>(c, a, status, stream);
-    return launch_d<64>(c, a, status, stream);
+    const bool local = (a.flags & FOCUS_PREFILL_KMER_LOCAL) != 0;
+    if (c.d == 128) return local ? launch_d<128, true>(c, a, status, stream) : launch_d<128, false>(c, a, status, stream);
+    return local ? launch_d<64, true>(c, a, status, stream) : launch_d<64, false>(c, a, status, stream);
 }
 
 }  // namespace focus

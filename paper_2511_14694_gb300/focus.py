@@ -21,6 +21,7 @@ STATUS_NAMES = {0: "ok", 1: "invalid argument", 2: "unsupported", 3: "capacity",
                 6: "layout"}
 LAYOUT_CLOSE_TAIL = 1
 PREFILL_LEGACY_MMA = 1
+PREFILL_KMER_LOCAL = 2
 SUMMARY_TOKEN = 4
 
 

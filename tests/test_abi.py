@@ -102,3 +102,27 @@ def test_layout_size_edge_cases():
     kk = np.ones(M, np.int32)
     assert lib.focus_layout_size(2_000_000_000, 1_000_000, M, kk.ctypes.data, 1, 0, ctypes.byref(T), None,
                                  None) == 2
+
+
+def test_prefill_flag_checks_need_no_gpu():
+    """Flag validation happens on the host before any CUDA call (T_span = 0 makes
+    a valid call a no-op)."""
+    lib = focus.load()
+    c = focus.CacheDesc()
+    c.B, c.H, c.d, c.C_ring = 1, 1, 64, 0
+    a = focus.PrefillArgs()
+    a.q = a.k = a.v = a.o = 4096
+    a.d_win_off = a.d_ring_off = 4096
+    a.n_windows, a.w_begin, a.w_end, a.max_rows, a.scale, a.T_span = 2, 0, 2, 10, 0.125, 0
+    call = lambda flags: (setattr(a, "flags", flags), lib.focus_attn_prefill(ctypes.byref(c), ctypes.byref(a), None))[1]  # noqa: E731
+    assert call(0) == 0
+    assert call(focus.PREFILL_LEGACY_MMA) == 0
+    assert call(8) == 1                                                   # unknown flag bit
+    assert call(focus.PREFILL_KMER_LOCAL) == 1                            # no k schedule
+    c.k_per_window, c.n_windows = 4096, 1
+    assert call(focus.PREFILL_KMER_LOCAL) == 1                            # schedule shorter than w_end
+    c.n_windows = 2
+    assert call(focus.PREFILL_KMER_LOCAL) == 0
+    assert call(focus.PREFILL_KMER_LOCAL | focus.PREFILL_LEGACY_MMA) == 2
+    c.tail = 1
+    assert call(focus.PREFILL_KMER_LOCAL) == 2                            # boundary tails not supported

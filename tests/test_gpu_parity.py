@@ -137,6 +137,92 @@ def test_prefill_legacy_kernel_matches_oracle():
     assert_attn_close(o, lse, o_ref.reshape(B, H, T, d), lse_ref.reshape(B, H, T), "legacy")
 
 
+# ----------------------------------------------------------------------------- prefill, k-mer-local mask (Sec. 3.2)
+
+LOCAL_PREFILL_CASES = [
+    # N, W, k schedule (cycled over the windows), B, H, d, std
+    (4_000, 1_000, [100], 1, 2, 64, 1.0),
+    (5_000, 1_024, [100], 1, 2, 128, 1.0),                   # partial k-mer closes every window
+    (3_001, 300, [1, 7, 50, 0, 300, 1_000], 2, 1, 128, 1.0),  # k = 1 (300 FOCUS rows: 3 ring tiles), k = 0
+                                                             # (no boundary for the next window), k >= W, ragged end
+    (2_000, 2_000, [0], 1, 1, 64, 1.0),                      # one window, one k-mer: causal
+    (20_000, 200, [10], 1, 2, 128, 1.0 / math.sqrt(128)),
+    (300, 64, [64], 1, 2, 64, 1.0),                          # T_w = 65: one row past a tile
+    (1_500, 700, [3, 128, 255], 1, 1, 64, 1.0),              # k-mers that straddle 128-row tiles
+]
+
+
+def _local_case(N, W, ks, B, H, d, std, seed):
+    M = -(-N // W)
+    k = np.resize(np.asarray(ks, np.int32), M)
+    L = focus.layout(N, W, k)
+    q, kk, v = inputs.qkv((B, H, L["T"], d), std=std, seed=seed, device="cuda")
+    cache = focus.Cache(B, H, d, C_ring=max(L["R"], 1), k_sched=k)
+    return L, k, q, kk, v, cache
+
+
+def _local_ref(N, W, k, q, kk, v, heads, rows):
+    B, H, T, d = q.shape
+    ref_L = fo.layout(N, W, k)
+    km = fo.layout_kmer(N, W, k)
+    return fo.attn_rows_kmer_local(q.reshape(B * H, T, d).cpu(), kk.reshape(B * H, T, d).cpu(),
+                                   v.reshape(B * H, T, d).cpu(), ref_L["kind"], ref_L["win"], km, 1.0 / math.sqrt(d),
+                                   heads, rows)
+
+
+@pytest.mark.parametrize("N,W,ks,B,H,d,std", LOCAL_PREFILL_CASES)
+def test_prefill_kmer_local_matches_oracle(N, W, ks, B, H, d, std):
+    L, k, q, kk, v, cache = _local_case(N, W, ks, B, H, d, std, seed=N + 7)
+    n = q.numel()
+    canary = torch.full((n + 4096,), 7.0, dtype=torch.bfloat16, device="cuda")
+    o = canary[:n].view(q.shape)
+    o, lse = pipeline.prefill_masked_parallel(cache, q, kk, v, L, o=o, flags=focus.PREFILL_KMER_LOCAL)
+    torch.cuda.synchronize()
+    assert bool((canary[n:] == 7.0).all()), "prefill wrote past its output"
+    T = L["T"]
+    heads = np.repeat(np.arange(B * H), T)
+    rows = np.tile(np.arange(T), B * H)
+    o_ref, lse_ref = _local_ref(N, W, k, q, kk, v, heads, rows)
+    assert_attn_close(o, lse, o_ref.reshape(B, H, T, d), lse_ref.reshape(B, H, T), f"local N={N} W={W} k={ks}")
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_prefill_kmer_local_streaming_matches_oracle(d):
+    """Window by window: compact window w into the ring, then prefill it."""
+    N, W, ks, B, H = 3_000, 500, [10, 50, 0, 7, 100, 500], 2, 2
+    L, k, q, kk, v, cache = _local_case(N, W, ks, B, H, d, 1.0, seed=31)
+    o = torch.empty_like(q)
+    lse = torch.empty((B, H, L["T"]), dtype=torch.float32, device="cuda")
+    off = L["win_off_host"]
+    for w in range(L["M"]):
+        a, e = int(off[w]), int(off[w + 1])
+        sl = lambda t: t[:, :, a:e].contiguous()  # noqa: E731
+        ow, lw = pipeline.prefill_window(cache, sl(q), sl(kk), sl(v), L, w, flags=focus.PREFILL_KMER_LOCAL)
+        o[:, :, a:e] = ow
+        lse[:, :, a:e] = lw
+    torch.cuda.synchronize()
+    T = L["T"]
+    heads = np.repeat(np.arange(B * H), T)
+    rows = np.tile(np.arange(T), B * H)
+    o_ref, lse_ref = _local_ref(N, W, k, q, kk, v, heads, rows)
+    assert_attn_close(o, lse, o_ref.reshape(B, H, T, d), lse_ref.reshape(B, H, T), "local streaming")
+
+
+def test_prefill_kmer_local_argument_checks():
+    N, W = 1_000, 500
+    L, k, q, kk, v, cache = _local_case(N, W, [10], 1, 1, 64, 1.0, seed=1)
+    bad_tail = focus.Cache(1, 1, 64, C_ring=L["R"], k_sched=k, tail=2)
+    with pytest.raises(RuntimeError, match="unsupported"):
+        focus.attn_prefill(bad_tail, q, kk, v, L, flags=focus.PREFILL_KMER_LOCAL)
+    no_k = focus.Cache(1, 1, 64, C_ring=L["R"])          # k schedule of one window, two needed
+    with pytest.raises(RuntimeError, match="invalid"):
+        focus.attn_prefill(no_k, q, kk, v, L, flags=focus.PREFILL_KMER_LOCAL)
+    with pytest.raises(RuntimeError, match="unsupported"):
+        focus.attn_prefill(cache, q, kk, v, L, flags=focus.PREFILL_KMER_LOCAL | focus.PREFILL_LEGACY_MMA)
+    with pytest.raises(RuntimeError, match="invalid"):
+        focus.attn_prefill(cache, q, kk, v, L, flags=8)
+
+
 # ----------------------------------------------------------------------------- prefill, sequential / streaming
 
 @pytest.mark.parametrize("d,tail", [(64, 0), (128, 0), (128, 5)])
