@@ -59,6 +59,25 @@ def visible_pairs(win_off, ring_off):
     return int((Tw * (Tw + 1) // 2).sum() + (Tw * Rw).sum())
 
 
+def kmer_local_row_counts(win_off, ring_off, k_sched):
+    """Keys each row sees under the k-mer-local mask (Sec. 3.2): a row at
+    in-window offset a of k-mer c = a // (k+1) sees a - c(k+1) + 1 rows of its
+    k-mer, c earlier in-window FOCUS rows and the carried boundary when the
+    previous window kept rows (a window with k = 0, or k >= T_w, is one k-mer)."""
+    win_off = np.asarray(win_off, dtype=np.int64)
+    ring_off = np.asarray(ring_off, dtype=np.int64)
+    k_sched = np.asarray(k_sched, dtype=np.int64)
+    rows = np.arange(win_off[-1])
+    w = np.searchsorted(win_off, rows, side="right") - 1
+    a = rows - win_off[w]
+    Tw = np.diff(win_off)[w]
+    kw = k_sched[w]
+    kdiv = np.where((kw > 0) & (kw < Tw), kw, Tw) + 1
+    c = a // kdiv
+    bnd = ((w >= 1) & (ring_off[np.maximum(w - 1, 0)] < ring_off[w])).astype(np.int64)
+    return a - c * kdiv + 1 + c + bnd
+
+
 def kernel_traffic(kernel_key: str, source: str):
     """DRAM bytes per launch from a committed ncu summary, only while the kernel
     source is unchanged since the counters were taken (else None)."""
@@ -212,6 +231,36 @@ def oracle_prefill_sample(cfg, L_host, q, k, v, budget_s=12.0, max_windows=None)
     return full_s, desc, os.cpu_count()
 
 
+def oracle_local_sample(cfg, L_host, k_sched, q, k, v, budget_s=12.0, max_windows=None):
+    """As oracle_prefill_sample, for the k-mer-local mask: the oracle's
+    attn_rows_kmer_local over all rows of evenly spaced windows, one head per
+    pass, extrapolated by visible pairs."""
+    from oracle import focus_oracle as fo
+    win_off, ring_off = L_host["win_off"], L_host["ring_off"]
+    M = win_off.size - 1
+    d = cfg["d"]
+    counts = kmer_local_row_counts(win_off, ring_off, k_sched)
+    total_pairs = int(counts.sum()) * cfg["B"] * cfg["H"]
+    n_w, spent, done_pairs, heads_done, h = 1, 0.0, 0, 0, 0
+    while spent < budget_s and heads_done < cfg["H"]:
+        ws = np.arange(0, M, max(1, M // n_w))
+        if max_windows:
+            ws = ws[:max_windows]
+        rows = np.concatenate([np.arange(win_off[w], win_off[w + 1]) for w in ws]).astype(np.int64)
+        t0 = time.perf_counter()
+        fo.attn_rows_kmer_local(q[h:h + 1], k[h:h + 1], v[h:h + 1], L_host["kind"], L_host["win"], L_host["kmer"],
+                                1.0 / math.sqrt(d), np.zeros(rows.size, np.int64), rows)
+        spent += time.perf_counter() - t0
+        done_pairs += int(counts[rows].sum())
+        heads_done += 1
+        h = (h + 1) % q.shape[0]
+        n_w = min(M, n_w * 2)
+    full_s = spent * total_pairs / max(done_pairs, 1)
+    desc = (f"fp64 oracle k-mer-local attention on {heads_done} head-passes over evenly spaced windows "
+            f"({done_pairs:,} of {total_pairs:,} visible pairs, {spent:.1f} s), extrapolated by visible pairs")
+    return full_s, desc, os.cpu_count()
+
+
 # ----------------------------------------------------------------------------- focus arm
 
 def run_prefill_leg(args, cfg, world, rank, local):
@@ -225,7 +274,7 @@ def run_prefill_leg(args, cfg, world, rank, local):
     nt = inputs.nucleotides(B, N, seed=inputs.DEFAULT_SEED, device=dev)
     L = focus.layout_alloc(N, W, k_s, B=B, device=dev)
     q, k, v = inputs.qkv((B, H, L["T"], d), std=cfg["std"], seed=inputs.DEFAULT_SEED + rank, device=dev)
-    cache = focus.Cache(B, H, d, C_ring=max(L["R"], 1), device=dev)
+    cache = focus.Cache(B, H, d, C_ring=max(L["R"], 1), device=dev, k_sched=k_s)
     o = torch.empty_like(q)
     lse = torch.empty((B, H, L["T"]), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
@@ -244,8 +293,12 @@ def run_prefill_leg(args, cfg, world, rank, local):
     assert focus.device_status(clear=True) == 0
     win_off = L["win_off"].cpu().numpy()
     ring_off = L["ring_off"].cpu().numpy()
-    pairs = visible_pairs(win_off, ring_off)
+    local_mask = bool(args.prefill_flags & focus.PREFILL_KMER_LOCAL)
+    pairs = (int(kmer_local_row_counts(win_off, ring_off, k_s).sum()) if local_mask
+             else visible_pairs(win_off, ring_off))
     flops_per_step = 4.0 * d * H * B * pairs
+    # algorithmic bytes of one prefill launch: read Q, K, V and write O once (bf16), write LSE (fp32)
+    bytes_per_step = float(B * H * L["T"] * (8 * d + 4))
 
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -315,8 +368,10 @@ def run_prefill_leg(args, cfg, world, rank, local):
     host_sample = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         host_sample = dict(win_off=win_off, ring_off=ring_off, kind=L["kind"].cpu().numpy(),
+                           win=L["win"].cpu().numpy(), keep=L["keep"].cpu().numpy(), k_sched=k_s,
                            q=q[0, :2].cpu(), k=k[0, :2].cpu(), v=v[0, :2].cpu())
     res = dict(step_ms=step_ms, attn_ms=attn_ms, flops_per_step=flops_per_step, pairs=pairs, T=L["T"], R=L["R"],
+               bytes_per_step=bytes_per_step, local_mask=local_mask,
                clocks=clk.summary(), launches=launches, e2e=e2e, host_sample=host_sample, extra_steps=extra)
     del q, k, v, o, lse, cache
     torch.cuda.empty_cache()
@@ -340,7 +395,8 @@ def run_stream_leg(args, cfg, world, rank, local):
     if not (np.diff(off) == Tw).all():
         raise ValueError("the streaming leg expects windows of equal augmented size")
     pq, pk, pv = inputs.qkv((P, B, H, Tw, d), std=cfg["std"], seed=inputs.DEFAULT_SEED + rank, device=dev)
-    cache = focus.Cache(B, H, d, C_ring=max(L["R"], 1), device=dev)
+    cache = focus.Cache(B, H, d, C_ring=max(L["R"], 1), device=dev, k_sched=k_s)
+    local_mask = bool(args.prefill_flags & focus.PREFILL_KMER_LOCAL)
     outs = [torch.empty((B, H, Tw, d), dtype=torch.bfloat16, device=dev) for _ in range(2)]
     lses = [torch.empty((B, H, Tw), dtype=torch.float32, device=dev) for _ in range(2)]
     stream = torch.cuda.current_stream(dev)
@@ -348,19 +404,23 @@ def run_stream_leg(args, cfg, world, rank, local):
 
     def step(timed=False):
         for w in range(M):
+            if local_mask:        # the k-mer-local mask reads the window's own FOCUS rows from the ring
+                focus.kv_compact_bulk(cache, pk[w % P], pv[w % P], L, w, w + 1, src_row0=int(off[w]), stream=stream)
             if timed:
                 evs[w][0].record(stream)
             focus.attn_prefill(cache, pq[w % P], pk[w % P], pv[w % P], L, w, w + 1, o=outs[w % 2], lse=lses[w % 2],
                                stream=stream, flags=args.prefill_flags)
             if timed:
                 evs[w][1].record(stream)
-            focus.kv_compact_bulk(cache, pk[w % P], pv[w % P], L, w, w + 1, src_row0=int(off[w]), stream=stream)
+            if not local_mask:
+                focus.kv_compact_bulk(cache, pk[w % P], pv[w % P], L, w, w + 1, src_row0=int(off[w]), stream=stream)
 
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize(dev)
     assert focus.device_status(clear=True) == 0
-    pairs = visible_pairs(off, L["ring_off_host"])
+    pairs = (int(kmer_local_row_counts(off, L["ring_off_host"], k_s).sum()) if local_mask
+             else visible_pairs(off, L["ring_off_host"]))
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     attn_ms = 0.0
     barrier(world)
@@ -377,7 +437,8 @@ def run_stream_leg(args, cfg, world, rank, local):
     step_ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, world)
     return dict(step_ms=step_ms, attn_ms=attn_ms / args.steps, flops_per_step=4.0 * d * H * B * pairs, pairs=pairs,
                 T=L["T"], R=L["R"], clocks=clk.summary(), launches=2 * M * args.steps, e2e=None, host_sample=None,
-                per_launch_ms=attn_ms / args.steps / M)
+                per_launch_ms=attn_ms / args.steps / M, local_mask=local_mask,
+                bytes_per_step=float(B * H * L["T"] * (8 * d + 4)))
 
 
 def run_decode_leg(args, cfg, world, rank, local):
@@ -476,7 +537,10 @@ def run_focus(args, world, rank, local):
         return
     value = weak_scaling_value(cfg["B"] * cfg["N"], world, pre["step_ms"] / 1e3)
     achieved = pre["flops_per_step"] / (pre["attn_ms"] / 1e3) / 1e12
-    traffic = None if args.legacy else kernel_traffic("prefill_attention", "paper_2511_14694_gb300/csrc/prefill_tc.cu")
+    local_mask = pre.get("local_mask", False)
+    traffic = None if args.legacy else kernel_traffic(
+        "prefill_attention_kmer_local" if local_mask else "prefill_attention",
+        "paper_2511_14694_gb300/csrc/prefill_tc.cu")
     if traffic is not None and cfg is not WORKLOADS["prefill_128kb_h32_d128"]:
         traffic = None            # the committed counters are for the 128 kb workload only
     line = {
@@ -493,7 +557,8 @@ def run_focus(args, world, rank, local):
                        cfg.get("pool", 0), 3 * cfg.get("pool", 0) * cfg["B"] * cfg["H"] * (pre["T"] // max(1, -(-cfg["N"] // cfg["W"]))) * cfg["d"] * 2 / 1e9,
                        2 * cfg["B"] * cfg["H"] * pre["R"] * cfg["d"] * 2 / 1e9) if cfg["mode"] == "stream" else
                           "inputs larger than L2 (Q/K/V %.2f GB per step)" % (3 * cfg["B"] * pre["T"] * cfg["H"] * cfg["d"] * 2 / 1e9)),
-                   "prefill_kernel": "legacy mma.sync" if args.prefill_flags & 1 else "default"},
+                   "prefill_kernel": "legacy mma.sync" if args.prefill_flags & 1 else "default",
+                   "mask": "k-mer-local (Sec. 3.2)" if local_mask else "appendix (App. A, Eq. focus-attn)"},
         "augmented_tokens_per_s": world * cfg["B"] * pre["T"] / (pre["step_ms"] / 1e3),
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
                      "frac": achieved / peaks["bf16_tflops"], "traffic": traffic,
@@ -508,6 +573,17 @@ def run_focus(args, world, rank, local):
         "e2e": pre["e2e"],
         "gpu_launches": pre["launches"],
     }
+    if local_mask:
+        # a few visible keys per row: the launch moves far more bytes than it does FLOPs
+        gbs = pre["bytes_per_step"] / (pre["attn_ms"] / 1e3) / 1e9
+        line["roofline"] = {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                            "frac": gbs / peaks["hbm_gbs"], "traffic": traffic,
+                            "peak_source": f"{peaks_src} copy bandwidth", "kernel": "prefill attention (k-mer-local)",
+                            "tflops": achieved, "visible_pairs": pre["pairs"]}
+        n_launch = (pre["launches"] // (2 * args.steps)) if cfg["mode"] == "stream" else 1
+        line["roofline"].update(bytes_per_launch=pre["bytes_per_step"] / n_launch,
+                                flop_per_launch=pre["flops_per_step"] / n_launch,
+                                avg_launch_ms=pre.get("per_launch_ms", pre["attn_ms"]), launches_per_step=n_launch)
     if dec is not None:
         gbs = dec["bytes_leg"] / (dec["decode_kernels_ms"] / 1e3) / 1e9
         line["decode"] = {
@@ -525,7 +601,13 @@ def run_focus(args, world, rank, local):
         line["decode"]["gpu_launches"] = dec["launches"]
     if pre["host_sample"] is not None:
         hs = pre["host_sample"]
-        full_s, desc, cores = oracle_prefill_sample(cfg, hs, hs["q"], hs["k"], hs["v"], budget_s=args.cpu_budget)
+        if local_mask:
+            from oracle import focus_oracle as fo
+            hs["kmer"] = fo.layout_kmer(cfg["N"], cfg["W"], hs["k_sched"])
+            full_s, desc, cores = oracle_local_sample(cfg, hs, hs["k_sched"], hs["q"], hs["k"], hs["v"],
+                                                      budget_s=args.cpu_budget)
+        else:
+            full_s, desc, cores = oracle_prefill_sample(cfg, hs, hs["q"], hs["k"], hs["v"], budget_s=args.cpu_budget)
         line["cpu_baseline"] = {"value": cfg["B"] * cfg["N"] / full_s, "unit": "nt/s", "cores": cores,
                                 "kind": "oracle", "sample": desc}
     print(json.dumps(line), flush=True)
@@ -549,20 +631,26 @@ def run_reference(args, world, rank, local):
     L = fo.layout(N, W, k_s)
     # two heads of inputs, drawn with the same generator recipe on the CPU
     q, k, v = inputs.qkv((2, L["T"], d), std=cfg["std"], seed=inputs.DEFAULT_SEED, device="cpu")
-    hs = dict(win_off=L["win_off"], ring_off=L["ring_off"], keep=L["keep"])
+    hs = dict(win_off=L["win_off"], ring_off=L["ring_off"], keep=L["keep"], kind=L["kind"], win=L["win"])
     budget = max(2.0, args.cpu_budget / max(1, args.steps + args.warmup))
+    if args.mask == "kmer_local":
+        hs["kmer"] = fo.layout_kmer(N, W, k_s)
+        sample = lambda: oracle_local_sample(cfg, hs, k_s, q, k, v, budget_s=budget, max_windows=4)  # noqa: E731
+    else:
+        sample = lambda: oracle_prefill_sample(cfg, hs, q, k, v, budget_s=budget, max_windows=4)  # noqa: E731
     for _ in range(args.warmup):
-        oracle_prefill_sample(cfg, hs, q, k, v, budget_s=budget, max_windows=4)
+        sample()
     secs, desc = [], ""
     for _ in range(args.steps):
-        full_s, desc, cores = oracle_prefill_sample(cfg, hs, q, k, v, budget_s=budget, max_windows=4)
+        full_s, desc, cores = sample()
         secs.append(full_s)
     full_s = statistics.median(secs)
     value = B * N / full_s
     line = {"metric": METRIC, "value": value, "unit": "nt/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": full_s * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
-            "config": {"workload": args.workload, "B": B, "N": N, "W": W, "k": list(cfg["k"]), "H": H, "d": d},
+            "config": {"workload": args.workload, "B": B, "N": N, "W": W, "k": list(cfg["k"]), "H": H, "d": d,
+                       "mask": args.mask},
             "cpu_baseline": {"value": value, "unit": "nt/s", "cores": os.cpu_count(), "kind": "oracle",
                              "sample": desc},
             "e2e": {"value": value, "unit": "nt/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -651,13 +739,15 @@ def main():
     ap.add_argument("--no-clock-wait", action="store_true",
                     help="do not extend the load after a short timed region (profiling runs)")
     ap.add_argument("--legacy", action="store_true", help="time the legacy mma.sync prefill kernel")
+    ap.add_argument("--mask", default="appendix", choices=["appendix", "kmer_local"],
+                    help="prefill visibility: App. A (default) or the k-mer-local rule of Sec. 3.2")
     ap.add_argument("--memory-report", action="store_true",
                     help="peak memory and time vs context length, FOCUS streaming vs full-cache causal")
     ap.add_argument("--memory-ns", default="16000,32000,64000,128000,256000,512000,1000000")
     ap.add_argument("--memory-full-max", type=int, default=256_000)
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
-    args.prefill_flags = 1 if args.legacy else 0
+    args.prefill_flags = (1 if args.legacy else 0) | (2 if args.mask == "kmer_local" else 0)
     world, rank, local = dist_setup()
     if args.memory_report:
         run_memory_report(args, world, rank, local)

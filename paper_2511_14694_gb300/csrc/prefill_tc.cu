@@ -110,7 +110,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
     // LOCAL: k-mer length + 1 (a window without summaries, or with k >= T_w, is one
     // k-mer), boundary present?, key ranges [ring_lo, ...) and [win_lo, ...)
     int32_t kdiv = 1, bnd = 0, ring_lo = 0, win_lo = 0, ring_hi = Rw;
-    int n_ring, n_win = 0;
+    int n_ring, n_win = 0, n_win0 = 0;
     if (LOCAL) {
         const int32_t kw = k_per_window[w];
         kdiv = (kw > 0 && kw < Tw ? kw : Tw) + 1;
@@ -121,6 +121,8 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
         win_lo = (a0 / kdiv) * kdiv;
         n_ring = (ring_hi - ring_lo + BN - 1) / BN;
         n_win = (a_last + 1 - win_lo + BN - 1) / BN;
+        // Q tile 0 ends at row a0 + BM - 1: its window keys are a prefix of the CTA's
+        n_win0 = ((a0 + BM < Tw ? a0 + BM : Tw) - win_lo + BN - 1) / BN;
     } else {
         n_ring = (Rw + BN - 1) / BN;
     }
@@ -130,7 +132,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
     }
     const int32_t row_base = win_off[w] - w0;           // first row of the window in the span tensors
     const bool valid1 = a0 + BM < Tw;
-    const int n_kv0 = LOCAL ? n_ring + n_win : n_ring + 2 * cta + 1;
+    const int n_kv0 = LOCAL ? n_ring + n_win0 : n_ring + 2 * cta + 1;
     const int n_kv1 = valid1 ? (LOCAL ? n_ring + n_win : n_ring + 2 * cta + 2) : 0;
     const int n_kv_max = valid1 ? n_kv1 : n_kv0;
 
