@@ -393,3 +393,112 @@ void fo_attn_rows_kmer_local(int64_t T, int32_t d, const uint8_t* kind, const in
     }
     free(last_focus);
 }
+
+/* ------------------------------------------------------------------------- */
+/* Rotary position embedding at the layout's position ids (RoFormer, Su et    */
+/* al. 2021; the position id of a row is its augmented index, Sec. 3.2 "each  */
+/* FOCUS token occupies a real sequence position"). Rotate-half pairing: for  */
+/* i < d/2, the pair (x_i, x_{i+d/2}) is turned by the angle p * theta_i,     */
+/* theta_i = base^(-2i/d):                                                    */
+/*   y_i       = x_i cos(p theta_i) - x_{i+d/2} sin(p theta_i)                */
+/*   y_{i+d/2} = x_{i+d/2} cos(p theta_i) + x_i sin(p theta_i)               */
+/* x: [n][d] bf16 bits, pos[n]; y: [n][d] fp64.                               */
+/* ------------------------------------------------------------------------- */
+void fo_rope(int64_t n, int32_t d, const int64_t* pos, double base, const uint16_t* x, double* y) {
+    int32_t h = d / 2;
+    for (int64_t r = 0; r < n; ++r) {
+        const uint16_t* xr = x + (size_t)r * d;
+        double* yr = y + (size_t)r * d;
+        for (int32_t i = 0; i < h; ++i) {
+            double theta = pow(base, -2.0 * (double)i / (double)d);
+            double a = (double)pos[r] * theta;
+            double c = cos(a), s = sin(a);
+            double lo = bf16_to_f64(xr[i]), hi = bf16_to_f64(xr[i + h]);
+            yr[i] = lo * c - hi * s;
+            yr[i + h] = hi * c + lo * s;
+        }
+    }
+}
+
+/* Softmax attention of one fp64 query over fp64 key rows (same arithmetic as */
+/* softmax_row; used where Q and K carry the rotary embedding).              */
+static void softmax_row_f64(int32_t d, const double* q, int64_t n_keys, const double* const* krows,
+                            const uint16_t* const* vrows, double scale, double* o, double* lse) {
+    double* s = (double*)malloc(sizeof(double) * (size_t)(n_keys > 0 ? n_keys : 1));
+    double m = -INFINITY;
+    for (int64_t j = 0; j < n_keys; ++j) {
+        double dot = 0.0;
+        for (int32_t c = 0; c < d; ++c) dot += q[c] * krows[j][c];
+        s[j] = scale * dot;
+        if (s[j] > m) m = s[j];
+    }
+    double l = 0.0;
+    for (int32_t c = 0; c < d; ++c) o[c] = 0.0;
+    for (int64_t j = 0; j < n_keys; ++j) {
+        double p = exp(s[j] - m);
+        l += p;
+        for (int32_t c = 0; c < d; ++c) o[c] += p * bf16_to_f64(vrows[j][c]);
+    }
+    for (int32_t c = 0; c < d; ++c) o[c] /= l;
+    *lse = m + log(l);
+    free(s);
+}
+
+/* fo_attn_rows with fp64 queries and keys (e.g. after fo_rope): the same     */
+/* visible set (App. A: same window, or a retained row), qf/kf [n_heads][T][d] */
+/* fp64, v bf16 bits.                                                         */
+void fo_attn_rows_f64(int64_t T, int32_t d, const uint8_t* keep, const int32_t* win, const double* qf,
+                      const double* kf, const uint16_t* v, double scale, int64_t n_rows,
+                      const int64_t* row_head, const int64_t* row_idx, double* o, double* lse) {
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t r = 0; r < n_rows; ++r) {
+        int64_t h = row_head[r], i = row_idx[r];
+        const double* kh = kf + (size_t)h * (size_t)T * (size_t)d;
+        const uint16_t* vh = v + (size_t)h * (size_t)T * (size_t)d;
+        const double** kr = (const double**)malloc(sizeof(void*) * (size_t)(i + 1));
+        const uint16_t** vr = (const uint16_t**)malloc(sizeof(void*) * (size_t)(i + 1));
+        int64_t n = 0;
+        for (int64_t j = 0; j <= i; ++j) {
+            if (!((win[j] == win[i]) || (keep[j] == 1))) continue;
+            kr[n] = kh + (size_t)j * d;
+            vr[n] = vh + (size_t)j * d;
+            n += 1;
+        }
+        softmax_row_f64(d, qf + ((size_t)h * (size_t)T + (size_t)i) * d, n, kr, vr, scale,
+                        o + (size_t)r * d, lse + r);
+        free(kr);
+        free(vr);
+    }
+}
+
+/* fo_decode with fp64 queries and keys: ring_k/win_k/k_new/q fp64 (already   */
+/* rotated by the caller), values bf16 bits; otherwise identical.            */
+void fo_decode_f64(int32_t d, int64_t n, const double* ring_k, const uint16_t* ring_v,
+                   int64_t ring_stride, const int64_t* R, const double* win_k,
+                   const uint16_t* win_v, int64_t win_stride, const int64_t* fill,
+                   const double* q, const double* k_new, const uint16_t* v_new,
+                   double scale, double* o, double* lse) {
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t s = 0; s < n; ++s) {
+        int64_t nk = R[s] + fill[s] + 1;
+        const double** kr = (const double**)malloc(sizeof(void*) * (size_t)nk);
+        const uint16_t** vr = (const uint16_t**)malloc(sizeof(void*) * (size_t)nk);
+        int64_t c = 0;
+        for (int64_t j = 0; j < R[s]; ++j) {
+            kr[c] = ring_k + ((size_t)s * ring_stride + (size_t)j) * d;
+            vr[c] = ring_v + ((size_t)s * ring_stride + (size_t)j) * d;
+            c += 1;
+        }
+        for (int64_t j = 0; j < fill[s]; ++j) {
+            kr[c] = win_k + ((size_t)s * win_stride + (size_t)j) * d;
+            vr[c] = win_v + ((size_t)s * win_stride + (size_t)j) * d;
+            c += 1;
+        }
+        kr[c] = k_new + (size_t)s * d;
+        vr[c] = v_new + (size_t)s * d;
+        c += 1;
+        softmax_row_f64(d, q + (size_t)s * d, c, kr, vr, scale, o + (size_t)s * d, lse + s);
+        free(kr);
+        free(vr);
+    }
+}

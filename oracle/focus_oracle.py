@@ -61,6 +61,12 @@ def _load(path: str | None = None):
     lib.fo_layout_kmer.argtypes = [i64, i32, i32, P, i32, P]
     lib.fo_attn_rows_kmer_local.restype = None
     lib.fo_attn_rows_kmer_local.argtypes = [i64, i32, P, P, P, P, P, P, f64, i64, P, P, P, P]
+    lib.fo_rope.restype = None
+    lib.fo_rope.argtypes = [i64, i32, P, f64, P, P]
+    lib.fo_attn_rows_f64.restype = None
+    lib.fo_attn_rows_f64.argtypes = [i64, i32, P, P, P, P, P, f64, i64, P, P, P, P]
+    lib.fo_decode_f64.restype = None
+    lib.fo_decode_f64.argtypes = [i32, i64, P, P, i64, P, P, P, i64, P, P, P, P, f64, P, P]
     lib.fo_window_retained_rows.restype = i32
     lib.fo_window_retained_rows.argtypes = [i64, i32, i32, i32, P, i32]
     _lib = lib
@@ -258,6 +264,64 @@ def decode(q, k_new, v_new, ring_k, ring_v, R, win_k, win_v, fill, scale: float)
     lib.fo_decode(d, n, _ptr(rkb), _ptr(rvb), rkb.shape[1], _ptr(R), _ptr(wkb), _ptr(wvb),
                   wkb.shape[1], _ptr(fill), _ptr(qb), _ptr(knb), _ptr(vnb), float(scale),
                   _ptr(o), _ptr(lse))
+    return o, lse
+
+
+def rope(x, pos, base: float) -> np.ndarray:
+    """Rotary position embedding (RoFormer, rotate-half pairing) of bf16 rows
+    ``x`` [..., d] at positions ``pos`` (broadcast to x's leading shape; the
+    layout's position ids). Returns fp64 [..., d]."""
+    lib = _load()
+    xb = _bits(x)
+    d = xb.shape[-1]
+    lead = xb.shape[:-1]
+    p = np.ascontiguousarray(np.broadcast_to(np.asarray(pos, dtype=np.int64), lead)).reshape(-1)
+    n = p.size
+    y = np.zeros((n, d), np.float64)
+    lib.fo_rope(n, d, _ptr(p), float(base), _ptr(np.ascontiguousarray(xb.reshape(n, d))), _ptr(y))
+    return y.reshape(xb.shape)
+
+
+def attn_rows_f64(qf, kf, v, keep, win, scale: float, heads, rows):
+    """``attn_rows`` with fp64 queries and keys (e.g. after ``rope``):
+    qf/kf fp64 [n_heads, T, d], v bf16 [n_heads, T, d]."""
+    lib = _load()
+    qf = np.ascontiguousarray(qf, dtype=np.float64)
+    kf = np.ascontiguousarray(kf, dtype=np.float64)
+    vb = _bits(v)
+    nh, T, d = qf.shape
+    assert kf.shape == qf.shape and vb.shape == qf.shape
+    keep = np.ascontiguousarray(keep, dtype=np.uint8)
+    win = np.ascontiguousarray(win, dtype=np.int32)
+    heads = np.ascontiguousarray(heads, dtype=np.int64)
+    rows = np.ascontiguousarray(rows, dtype=np.int64)
+    assert heads.shape == rows.shape
+    n = rows.size
+    o = np.zeros((n, d), np.float64)
+    lse = np.zeros(n, np.float64)
+    lib.fo_attn_rows_f64(T, d, _ptr(keep), _ptr(win), _ptr(qf), _ptr(kf), _ptr(vb), float(scale), n,
+                         _ptr(heads), _ptr(rows), _ptr(o), _ptr(lse))
+    return o, lse
+
+
+def decode_f64(qf, knf, v_new, ring_kf, ring_v, R, win_kf, win_v, fill, scale: float):
+    """``decode`` with fp64 queries and keys (rotated by the caller): qf/knf
+    fp64 [n, d]; ring_kf fp64 [n, C_ring, d]; win_kf fp64 [n, C_win, d]; values
+    bf16."""
+    lib = _load()
+    qf = np.ascontiguousarray(qf, dtype=np.float64)
+    knf = np.ascontiguousarray(knf, dtype=np.float64)
+    rkf = np.ascontiguousarray(ring_kf, dtype=np.float64)
+    wkf = np.ascontiguousarray(win_kf, dtype=np.float64)
+    vnb, rvb, wvb = _bits(v_new), _bits(ring_v), _bits(win_v)
+    n, d = qf.shape
+    R = np.ascontiguousarray(R, dtype=np.int64)
+    fill = np.ascontiguousarray(fill, dtype=np.int64)
+    assert (R <= rkf.shape[1]).all() and (fill < wkf.shape[1] + 1).all()
+    o = np.zeros((n, d), np.float64)
+    lse = np.zeros(n, np.float64)
+    lib.fo_decode_f64(d, n, _ptr(rkf), _ptr(rvb), rkf.shape[1], _ptr(R), _ptr(wkf), _ptr(wvb), wkf.shape[1],
+                      _ptr(fill), _ptr(qf), _ptr(knf), _ptr(vnb), float(scale), _ptr(o), _ptr(lse))
     return o, lse
 
 

@@ -62,6 +62,20 @@ MUTANTS = [
     ("boundary_is_first_focus", "if (kind[j] == 1) last_focus[win[j]] = j;",
      "if (kind[j] == 1 && last_focus[win[j]] < 0) last_focus[win[j]] = j;",
      [lambda: pins.test_kmer_local_invisible_rows_do_not_matter_and_visible_ones_do()]),
+    ("rope_sin_sign", "yr[i + h] = hi * c + lo * s;", "yr[i + h] = hi * c - lo * s;",
+     [lambda: pins.test_rope_one_hot_closed_form(64),
+      lambda: pins.test_rope_position_zero_is_identity_and_pairs_keep_their_norm()]),
+    ("rope_interleaved_pairs", "double lo = bf16_to_f64(xr[i]), hi = bf16_to_f64(xr[i + h]);",
+     "double lo = bf16_to_f64(xr[(2 * i) % d]), hi = bf16_to_f64(xr[(2 * i + 1) % d]);",
+     [lambda: pins.test_rope_one_hot_closed_form(64)]),
+    ("rope_frequency", "double theta = pow(base, -2.0 * (double)i / (double)d);",
+     "double theta = pow(base, -1.0 * (double)i / (double)d);",
+     [lambda: pins.test_rope_one_hot_closed_form(128)]),
+    ("rope_position_off_by_one", "double a = (double)pos[r] * theta;", "double a = (double)(pos[r] + 1) * theta;",
+     [lambda: pins.test_rope_position_zero_is_identity_and_pairs_keep_their_norm()]),
+    ("f64_attention_drops_ring", "if (!((win[j] == win[i]) || (keep[j] == 1))) continue;",
+     "if (!(win[j] == win[i])) continue;",
+     [lambda: pins.test_fp64_attention_variants_equal_the_pinned_bf16_ones()]),
     ("decode_skips_self", "        kr[c] = k_new + (size_t)s * d;\n        vr[c] = v_new + (size_t)s * d;\n        c += 1;\n",
      "", [lambda: pins.test_decode_equals_prefill_row()]),
 ]

@@ -481,3 +481,76 @@ def test_kmer_local_invisible_rows_do_not_matter_and_visible_ones_do():
     of, _ = _local(q, _perturb_rows(kk, first_focus, 8), _perturb_rows(v, first_focus, 9), L, 0.25,
                    np.zeros(later.size, np.int64), later)
     assert np.abs(of - ol0).max(axis=1).min() > 0         # every later k-mer sees the first FOCUS row
+
+
+# ----------------------------------------------------------------------------- rotary position embedding
+
+def _one_hot_bf16(d, idx):
+    x = torch.zeros(d, dtype=torch.bfloat16)
+    x[idx] = 1.0
+    return x
+
+
+@pytest.mark.parametrize("d", [8, 64, 128])
+def test_rope_one_hot_closed_form(d):
+    """RoFormer rotation, rotate-half pairing: e_i at position p goes to
+    cos(p t_i) e_i + sin(p t_i) e_{i+d/2} and e_{i+d/2} to
+    -sin(p t_i) e_i + cos(p t_i) e_{i+d/2}, t_i = base^(-2i/d): t_0 = 1 and
+    t_{d/4} = base^(-1/2)."""
+    base, h = 10_000.0, d // 2
+    for i, theta in ((0, 1.0), (d // 4, base ** -0.5), (h - 1, base ** (-2.0 * (h - 1) / d))):
+        for p in (0, 1, 7, 123_457, 1_010_000):
+            y = fo.rope(_one_hot_bf16(d, i), p, base)
+            e = np.zeros(d)
+            e[i], e[i + h] = math.cos(p * theta), math.sin(p * theta)
+            np.testing.assert_allclose(y, e, rtol=0, atol=1e-12)
+            y = fo.rope(_one_hot_bf16(d, i + h), p, base)
+            e = np.zeros(d)
+            e[i], e[i + h] = -math.sin(p * theta), math.cos(p * theta)
+            np.testing.assert_allclose(y, e, rtol=0, atol=1e-12)
+
+
+def test_rope_position_zero_is_identity_and_pairs_keep_their_norm():
+    x = inputs.normal_bf16((50, 64), 1.0, seed=3)
+    pos = np.arange(50) * 20_011
+    np.testing.assert_array_equal(fo.rope(x, 0, 500_000.0), _f64(x))
+    y = fo.rope(x, pos, 500_000.0)
+    xf = _f64(x)
+    np.testing.assert_allclose(y[:, :32] ** 2 + y[:, 32:] ** 2, xf[:, :32] ** 2 + xf[:, 32:] ** 2, rtol=1e-13, atol=0)
+
+
+def test_rope_attention_depends_only_on_relative_positions():
+    """<R(p) q, R(p') k> depends on p - p' only, so adding one offset to every
+    position leaves the attention outputs unchanged."""
+    L, q, k, v = _rand_case(300, 60, [7], 2, 32, seed=12)
+    T = L["T"]
+    heads, rows = np.repeat(np.arange(2), T), np.tile(np.arange(T), 2)
+    outs = []
+    for shift in (0, 987_654):
+        pos = np.arange(T) + shift
+        qf = fo.rope(q, pos, 10_000.0)
+        kf = fo.rope(k, pos, 10_000.0)
+        outs.append(fo.attn_rows_f64(qf, kf, v, L["keep"], L["win"], 0.2, heads, rows))
+    np.testing.assert_allclose(outs[0][0], outs[1][0], rtol=0, atol=1e-9)
+    np.testing.assert_allclose(outs[0][1], outs[1][1], rtol=0, atol=1e-9)
+
+
+def test_fp64_attention_variants_equal_the_pinned_bf16_ones():
+    """attn_rows_f64 / decode_f64 on the exactly widened bf16 inputs equal
+    attn_rows / decode (pinned above) to the last bit of fp64 arithmetic."""
+    L, q, k, v = _rand_case(400, 50, [1, 10, 60], 2, 16, seed=13)
+    T = L["T"]
+    heads, rows = np.repeat(np.arange(2), T), np.tile(np.arange(T), 2)
+    o1, l1 = fo.attn_rows(q, k, v, L["keep"], L["win"], 0.3, heads, rows)
+    o2, l2 = fo.attn_rows_f64(_f64(q), _f64(k), v, L["keep"], L["win"], 0.3, heads, rows)
+    np.testing.assert_allclose(o1, o2, rtol=0, atol=1e-15)
+    np.testing.assert_allclose(l1, l2, rtol=0, atol=1e-14)
+    n, d, C = 3, 16, 20
+    qn, kn, vn = inputs.qkv((n, d), seed=14)
+    rk, rv, wk = inputs.qkv((n, C, d), seed=15)
+    wv = inputs.normal_bf16((n, C, d), 1.0, seed=16)
+    R, fill = np.array([0, 5, 20]), np.array([3, 0, 19])
+    a = fo.decode(qn, kn, vn, rk, rv, R, wk, wv, fill, 0.25)
+    b = fo.decode_f64(_f64(qn), _f64(kn), vn, _f64(rk), rv, R, _f64(wk), wv, fill, 0.25)
+    np.testing.assert_allclose(a[0], b[0], rtol=0, atol=1e-15)
+    np.testing.assert_allclose(a[1], b[1], rtol=0, atol=1e-14)
