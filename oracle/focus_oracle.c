@@ -137,17 +137,13 @@ int64_t fo_layout(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
 /* rows: s_j = scale * <q, k_j>, m = max s, l = sum exp(s_j - m),             */
 /* o = sum exp(s_j - m) v_j / l, LSE = m + ln l.                              */
 /* ------------------------------------------------------------------------- */
-static void softmax_row(int32_t d, const uint16_t* q, int64_t n_keys,
-                        const uint16_t* const* krows, const uint16_t* const* vrows,
-                        double scale, double* o, double* lse) {
-    double* qd = (double*)malloc(sizeof(double) * (size_t)d);
-    double* s = (double*)malloc(sizeof(double) * (size_t)(n_keys > 0 ? n_keys : 1));
-    for (int32_t c = 0; c < d; ++c) qd[c] = bf16_to_f64(q[c]);
+
+/* The part after the dot products: s[j] holds <q, k_j> on entry. */
+static void softmax_of_dots(int32_t d, int64_t n_keys, double* s, const uint16_t* const* vrows,
+                            double scale, double* o, double* lse) {
     double m = -INFINITY;
     for (int64_t j = 0; j < n_keys; ++j) {
-        double dot = 0.0;
-        for (int32_t c = 0; c < d; ++c) dot += qd[c] * bf16_to_f64(krows[j][c]);
-        s[j] = scale * dot;
+        s[j] = scale * s[j];
         if (s[j] > m) m = s[j];
     }
     double l = 0.0;
@@ -159,6 +155,20 @@ static void softmax_row(int32_t d, const uint16_t* q, int64_t n_keys,
     }
     for (int32_t c = 0; c < d; ++c) o[c] /= l;
     *lse = m + log(l);
+}
+
+static void softmax_row(int32_t d, const uint16_t* q, int64_t n_keys,
+                        const uint16_t* const* krows, const uint16_t* const* vrows,
+                        double scale, double* o, double* lse) {
+    double* qd = (double*)malloc(sizeof(double) * (size_t)d);
+    double* s = (double*)malloc(sizeof(double) * (size_t)(n_keys > 0 ? n_keys : 1));
+    for (int32_t c = 0; c < d; ++c) qd[c] = bf16_to_f64(q[c]);
+    for (int64_t j = 0; j < n_keys; ++j) {
+        double dot = 0.0;
+        for (int32_t c = 0; c < d; ++c) dot += qd[c] * bf16_to_f64(krows[j][c]);
+        s[j] = dot;
+    }
+    softmax_of_dots(d, n_keys, s, vrows, scale, o, lse);
     free(s);
     free(qd);
 }
@@ -420,27 +430,17 @@ void fo_rope(int64_t n, int32_t d, const int64_t* pos, double base, const uint16
     }
 }
 
-/* Softmax attention of one fp64 query over fp64 key rows (same arithmetic as */
-/* softmax_row; used where Q and K carry the rotary embedding).              */
+/* Softmax attention of one fp64 query over fp64 key rows (used where Q and K */
+/* carry the rotary embedding).                                              */
 static void softmax_row_f64(int32_t d, const double* q, int64_t n_keys, const double* const* krows,
                             const uint16_t* const* vrows, double scale, double* o, double* lse) {
     double* s = (double*)malloc(sizeof(double) * (size_t)(n_keys > 0 ? n_keys : 1));
-    double m = -INFINITY;
     for (int64_t j = 0; j < n_keys; ++j) {
         double dot = 0.0;
         for (int32_t c = 0; c < d; ++c) dot += q[c] * krows[j][c];
-        s[j] = scale * dot;
-        if (s[j] > m) m = s[j];
+        s[j] = dot;
     }
-    double l = 0.0;
-    for (int32_t c = 0; c < d; ++c) o[c] = 0.0;
-    for (int64_t j = 0; j < n_keys; ++j) {
-        double p = exp(s[j] - m);
-        l += p;
-        for (int32_t c = 0; c < d; ++c) o[c] += p * bf16_to_f64(vrows[j][c]);
-    }
-    for (int32_t c = 0; c < d; ++c) o[c] /= l;
-    *lse = m + log(l);
+    softmax_of_dots(d, n_keys, s, vrows, scale, o, lse);
     free(s);
 }
 

@@ -27,7 +27,7 @@ MUTANTS = [
      [lambda: pins.test_no_compression_is_plain_causal()]),
     ("k_for_v", "dot += qd[c] * bf16_to_f64(krows[j][c]);", "dot += qd[c] * bf16_to_f64(vrows[j][c]);",
      [lambda: pins.test_no_compression_is_plain_causal()]),
-    ("scale_dropped", "s[j] = scale * dot;", "s[j] = dot;",
+    ("scale_dropped", "s[j] = scale * s[j];", "s[j] = s[j];",
      [lambda: pins.test_no_compression_is_plain_causal()]),
     ("lse_no_max", "*lse = m + log(l);", "*lse = log(l);",
      [lambda: pins.test_first_row_sees_only_itself()]),
@@ -76,8 +76,8 @@ MUTANTS = [
     ("f64_attention_drops_ring", "if (!((win[j] == win[i]) || (keep[j] == 1))) continue;",
      "if (!(win[j] == win[i])) continue;",
      [lambda: pins.test_fp64_attention_variants_equal_the_pinned_bf16_ones()]),
-    ("decode_skips_self", "        kr[c] = k_new + (size_t)s * d;\n        vr[c] = v_new + (size_t)s * d;\n        c += 1;\n",
-     "", [lambda: pins.test_decode_equals_prefill_row()]),
+    ("decode_skips_self", "        kr[c] = k_new + (size_t)s * d;\n        vr[c] = v_new + (size_t)s * d;\n        c += 1;\n"
+     "        softmax_row(d,", "        softmax_row(d,", [lambda: pins.test_decode_equals_prefill_row()]),
 ]
 
 
