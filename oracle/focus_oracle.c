@@ -414,7 +414,20 @@ void fo_attn_rows_kmer_local(int64_t T, int32_t d, const uint8_t* kind, const in
 /*   y_{i+d/2} = x_{i+d/2} cos(p theta_i) + x_i sin(p theta_i)               */
 /* x: [n][d] bf16 bits, pos[n]; y: [n][d] fp64.                               */
 /* ------------------------------------------------------------------------- */
-void fo_rope(int64_t n, int32_t d, const int64_t* pos, double base, const uint16_t* x, double* y) {
+/* Round x to the nearest bf16 value (8 significant bits), ties to even, in one
+ * step from fp64 (bf16 keeps fp32's exponent range; these values are normal). */
+double fo_round_bf16(double x) {
+    if (x == 0.0 || !isfinite(x)) return x;
+    int e;
+    double m = frexp(x, &e);                 /* x = m 2^e, 0.5 <= |m| < 1 */
+    double r = nearbyint(ldexp(m, 8));       /* default rounding mode: to nearest, ties to even */
+    return ldexp(r, e - 8);
+}
+
+/* round_bf16 != 0: each output is rounded once to bf16, the element type of the
+ * rotated rows in a bf16 attention path. */
+void fo_rope(int64_t n, int32_t d, const int64_t* pos, double base, int32_t round_bf16, const uint16_t* x,
+             double* y) {
     int32_t h = d / 2;
     for (int64_t r = 0; r < n; ++r) {
         const uint16_t* xr = x + (size_t)r * d;
@@ -426,6 +439,10 @@ void fo_rope(int64_t n, int32_t d, const int64_t* pos, double base, const uint16
             double lo = bf16_to_f64(xr[i]), hi = bf16_to_f64(xr[i + h]);
             yr[i] = lo * c - hi * s;
             yr[i + h] = hi * c + lo * s;
+            if (round_bf16) {
+                yr[i] = fo_round_bf16(yr[i]);
+                yr[i + h] = fo_round_bf16(yr[i + h]);
+            }
         }
     }
 }

@@ -62,7 +62,9 @@ def _load(path: str | None = None):
     lib.fo_attn_rows_kmer_local.restype = None
     lib.fo_attn_rows_kmer_local.argtypes = [i64, i32, P, P, P, P, P, P, f64, i64, P, P, P, P]
     lib.fo_rope.restype = None
-    lib.fo_rope.argtypes = [i64, i32, P, f64, P, P]
+    lib.fo_rope.argtypes = [i64, i32, P, f64, i32, P, P]
+    lib.fo_round_bf16.restype = f64
+    lib.fo_round_bf16.argtypes = [f64]
     lib.fo_attn_rows_f64.restype = None
     lib.fo_attn_rows_f64.argtypes = [i64, i32, P, P, P, P, P, f64, i64, P, P, P, P]
     lib.fo_decode_f64.restype = None
@@ -267,10 +269,16 @@ def decode(q, k_new, v_new, ring_k, ring_v, R, win_k, win_v, fill, scale: float)
     return o, lse
 
 
-def rope(x, pos, base: float) -> np.ndarray:
+def round_bf16(x: float) -> float:
+    """Nearest bf16 value of x (ties to even), rounded once from fp64."""
+    return float(_load().fo_round_bf16(float(x)))
+
+
+def rope(x, pos, base: float, round_bf16: bool = False) -> np.ndarray:
     """Rotary position embedding (RoFormer, rotate-half pairing) of bf16 rows
     ``x`` [..., d] at positions ``pos`` (broadcast to x's leading shape; the
-    layout's position ids). Returns fp64 [..., d]."""
+    layout's position ids). Returns fp64 [..., d]; with ``round_bf16`` each value
+    is rounded once to bf16, the element type of rotated rows in a bf16 path."""
     lib = _load()
     xb = _bits(x)
     d = xb.shape[-1]
@@ -278,7 +286,7 @@ def rope(x, pos, base: float) -> np.ndarray:
     p = np.ascontiguousarray(np.broadcast_to(np.asarray(pos, dtype=np.int64), lead)).reshape(-1)
     n = p.size
     y = np.zeros((n, d), np.float64)
-    lib.fo_rope(n, d, _ptr(p), float(base), _ptr(np.ascontiguousarray(xb.reshape(n, d))), _ptr(y))
+    lib.fo_rope(n, d, _ptr(p), float(base), int(round_bf16), _ptr(np.ascontiguousarray(xb.reshape(n, d))), _ptr(y))
     return y.reshape(xb.shape)
 
 

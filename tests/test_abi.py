@@ -33,7 +33,7 @@ def test_library_exports_every_declared_function():
 def test_struct_sizes_match_c_layout():
     # 2 x int64 + 8 pointers; 8 pointers + 7 int32 (+pad); see focus.h
     assert ctypes.sizeof(focus.LayoutOut) == 16 + 9 * 8
-    assert ctypes.sizeof(focus.CacheDesc) == 8 * 8 + 8 * 4
+    assert ctypes.sizeof(focus.CacheDesc) == 8 * 8 + 8 * 4 + 8 + 8
     assert ctypes.sizeof(focus.PrefillArgs) == 5 * 8 + 8 + 2 * 8 + 6 * 4
     assert ctypes.sizeof(focus.CompactArgs) == 2 * 8 + 2 * 8 + 2 * 8 + 3 * 4 + 4
 
@@ -126,3 +126,26 @@ def test_prefill_flag_checks_need_no_gpu():
     assert call(focus.PREFILL_KMER_LOCAL | focus.PREFILL_LEGACY_MMA) == 2
     c.tail = 1
     assert call(focus.PREFILL_KMER_LOCAL) == 2                            # boundary tails not supported
+
+
+def test_rope_argument_checks_need_no_gpu():
+    """A negative or non-finite rotary base is refused on the host; decode with
+    the rotary embedding needs pos_base."""
+    lib = focus.load()
+    c = focus.CacheDesc()
+    c.B, c.H, c.d, c.C_ring = 1, 1, 64, 0
+    a = focus.PrefillArgs()
+    a.q = a.k = a.v = a.o = 4096
+    a.d_win_off = a.d_ring_off = 4096
+    a.n_windows, a.w_begin, a.w_end, a.max_rows, a.scale, a.T_span = 1, 0, 1, 10, 0.125, 0
+    for bad in (-1.0, float("nan"), float("inf")):
+        c.rope_theta = bad
+        assert lib.focus_attn_prefill(ctypes.byref(c), ctypes.byref(a), None) == 1
+    c.rope_theta = 10_000.0
+    assert lib.focus_attn_prefill(ctypes.byref(c), ctypes.byref(a), None) == 0
+    c.win_k = c.win_v = c.ring_len = c.win_fill = c.win_idx = c.k_per_window = 4096
+    c.W, c.n_windows, c.C_win = 10, 1, 16
+    assert lib.focus_attn_decode(ctypes.byref(c), 4096, 4096, 4096, ctypes.c_float(0.125), 4096, None, 4096,
+                                 1 << 20, None) == 1
+    assert lib.focus_attn_decode_noalloc(ctypes.byref(c), 4096, 4096, 4096, ctypes.c_float(0.125), 4096, None,
+                                         None) == 1

@@ -1,0 +1,224 @@
+"""GPU parity of the rotary position embedding (RoFormer rotation at the
+layout's position ids) against the fp64 oracle: masked-parallel and streaming
+prefill, the rotated ring written by bulk compaction, decode with window
+roll-over, and a 1 Mb stream whose positions reach ~10^6.
+
+The rotated rows of a bf16 path are bf16: the oracle rotates in fp64 and rounds
+once to bf16 (nearest, ties to even); the kernels rotate in fp32 and round once,
+so the two can differ by one bf16 step where the exact value lies near a
+rounding boundary. Attention uses the bars of test_gpu_parity; stored rotated
+keys are compared within half a bf16 step (2^-8 relative) of the exact rotation,
+or within one step (2^-7) of the oracle's rounded rows.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import focus_oracle as fo
+from paper_2511_14694_gb300 import focus, inputs, pipeline
+from test_gpu_parity import assert_attn_close, bits
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(autouse=True)
+def _clean_status():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    focus.device_status(clear=True)
+    yield
+    assert focus.device_status(clear=True) == 0, "a kernel reported an error"
+
+
+def assert_keys_close(gpu_bf16, ref_f64, what="", rel=2.0 ** -8):
+    """rel = 2^-8: one rounding of the exact value; 2^-7: against a reference that
+    was itself rounded (the two may pick neighbouring bf16 values)."""
+    g = gpu_bf16.detach().float().cpu().double().numpy()
+    err = np.abs(g - ref_f64)
+    bound = rel * np.abs(ref_f64) + 1e-5
+    assert (err <= bound).all(), f"{what}: worst excess {(err - bound).max():.3e}"
+
+
+def _case(N, W, ks, B, H, d, theta, seed, std=1.0):
+    M = -(-N // W)
+    k = np.resize(np.asarray(ks, np.int32), M)
+    L = focus.layout(N, W, k)
+    q, kk, v = inputs.qkv((B, H, L["T"], d), std=std, seed=seed, device="cuda")
+    cache = focus.Cache(B, H, d, C_ring=max(L["R"], 1), k_sched=k, rope_theta=theta)
+    return L, k, q, kk, v, cache
+
+
+def _ref_all_rows(N, W, k, q, kk, v, theta):
+    B, H, T, d = q.shape
+    ref_L = fo.layout(N, W, k)
+    pos = np.arange(T)
+    qf = fo.rope(q.reshape(B * H, T, d).cpu(), pos, theta, round_bf16=True)
+    kf = fo.rope(kk.reshape(B * H, T, d).cpu(), pos, theta, round_bf16=True)
+    heads, rows = np.repeat(np.arange(B * H), T), np.tile(np.arange(T), B * H)
+    o, lse = fo.attn_rows_f64(qf, kf, v.reshape(B * H, T, d).cpu(), ref_L["keep"], ref_L["win"],
+                              1.0 / math.sqrt(d), heads, rows)
+    return o.reshape(B, H, T, d), lse.reshape(B, H, T), kf.reshape(B, H, T, d), ref_L
+
+
+ROPE_CASES = [
+    # N, W, k schedule (cycled), B, H, d, rope base
+    (4_000, 1_000, [100], 1, 2, 64, 10_000.0),
+    (5_000, 1_024, [100], 1, 2, 128, 500_000.0),
+    (3_001, 300, [1, 7, 50, 0, 300, 1_000], 2, 1, 128, 10_000.0),
+    (300, 64, [64], 1, 2, 64, 1_000.0),
+]
+
+
+@pytest.mark.parametrize("N,W,ks,B,H,d,theta", ROPE_CASES)
+def test_prefill_rope_masked_parallel_matches_oracle(N, W, ks, B, H, d, theta):
+    L, k, q, kk, v, cache = _case(N, W, ks, B, H, d, theta, seed=N + 3)
+    o, lse = pipeline.prefill_masked_parallel(cache, q, kk, v, L)
+    torch.cuda.synchronize()
+    o_ref, lse_ref, kf, ref_L = _ref_all_rows(N, W, k, q, kk, v, theta)
+    assert_attn_close(o, lse, o_ref, lse_ref, f"rope N={N} W={W} k={ks}")
+    # the ring holds the FOCUS rows' keys rotated at their position ids, values as they were
+    R = L["R"]
+    assert_keys_close(cache.ring_k[:, :, :R], kf[:, :, ref_L["sum_idx"]], "ring K", rel=2.0 ** -7)
+    assert np.array_equal(bits(cache.ring_v)[:, :, :R], bits(v)[:, :, ref_L["sum_idx"]])
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_prefill_rope_streaming_matches_oracle(d):
+    N, W, ks, B, H, theta = 3_000, 500, [10, 50, 0, 7, 100, 500], 2, 2, 10_000.0
+    L, k, q, kk, v, cache = _case(N, W, ks, B, H, d, theta, seed=41)
+    o = torch.empty_like(q)
+    lse = torch.empty((B, H, L["T"]), dtype=torch.float32, device="cuda")
+    off = L["win_off_host"]
+    for w in range(L["M"]):
+        a, e = int(off[w]), int(off[w + 1])
+        sl = lambda t: t[:, :, a:e].contiguous()  # noqa: E731
+        ow, lw = pipeline.prefill_window(cache, sl(q), sl(kk), sl(v), L, w)
+        o[:, :, a:e] = ow
+        lse[:, :, a:e] = lw
+    torch.cuda.synchronize()
+    o_ref, lse_ref, kf, ref_L = _ref_all_rows(N, W, k, q, kk, v, theta)
+    assert_attn_close(o, lse, o_ref, lse_ref, "rope streaming")
+    assert_keys_close(cache.ring_k[:, :, :L["R"]], kf[:, :, ref_L["sum_idx"]], "ring K", rel=2.0 ** -7)
+
+
+class RopeDecodeModel:
+    """Host mirror of the decode cache with fp64 (rotated) keys, evolved with the
+    oracle's rules (App. A.2): each step rotates q and k_new at the new row's
+    position id pos_base + fill, appends, and retires full windows."""
+
+    def __init__(self, cache, W, k_sched, theta):
+        B, H = cache.B, cache.H
+        self.rk = cache.ring_k.float().cpu().double().numpy().copy()
+        self.rv = bits(cache.ring_v).copy()
+        self.wk = cache.win_k.float().cpu().double().numpy().copy()
+        self.wv = bits(cache.win_v).copy()
+        self.R = cache.ring_len.cpu().numpy().copy()
+        self.fill = cache.win_fill.cpu().numpy().copy()
+        self.widx = cache.win_idx.cpu().numpy().copy()
+        self.pos = cache.pos_base.cpu().numpy().astype(np.int64).copy()
+        self.W, self.k, self.theta, self.H = W, np.asarray(k_sched), theta, H
+
+    def step(self, q, kn, vn, scale):
+        B, H, d = q.shape
+        o, lse = np.zeros((B, H, d)), np.zeros((B, H))
+        for b in range(B):
+            p = self.pos[b] + self.fill[b]
+            qf = fo.rope(q[b].cpu(), p, self.theta, round_bf16=True)
+            kf = fo.rope(kn[b].cpu(), p, self.theta, round_bf16=True)
+            o[b], lse[b] = fo.decode_f64(qf, kf, vn[b].cpu(), self.rk[b], self.rv[b], [self.R[b]] * H, self.wk[b],
+                                         self.wv[b], [self.fill[b]] * H, scale)
+            f = self.fill[b]
+            self.wk[b, :, f], self.wv[b, :, f] = kf, bits(vn[b])
+            self.fill[b] += 1
+            kw = int(self.k[self.widx[b]])
+            Tw = self.W + (-(-self.W // kw) if kw > 0 else 0)
+            if self.fill[b] == Tw:
+                rows = fo.window_retained_rows(self.W, kw, True, 0)
+                r = self.R[b]
+                self.rk[b, :, r:r + rows.size] = self.wk[b][:, rows]
+                self.rv[b, :, r:r + rows.size] = self.wv[b][:, rows]
+                self.R[b] += rows.size
+                self.fill[b] = 0
+                self.widx[b] += 1
+                self.pos[b] += Tw
+        return o, lse
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_decode_rope_steps_match_oracle(d):
+    B, H, W, theta = 3, 2, 50, 10_000.0
+    k_sched = np.array([10, 7, 25, 50, 3, 10, 10, 10], np.int32)
+    cache = focus.Cache(B, H, d, C_ring=512, C_win=72, W=W, k_sched=k_sched, rope_theta=theta)
+    g = torch.Generator(device="cuda").manual_seed(5)
+    for t in (cache.ring_k, cache.ring_v, cache.win_k, cache.win_v):
+        t.copy_(torch.randn(t.shape, generator=g, device="cuda").bfloat16())
+    cache.ring_len.copy_(torch.tensor([0, 37, 300], dtype=torch.int32))
+    cache.win_idx.copy_(torch.tensor([0, 1, 2], dtype=torch.int32))
+    cache.win_fill.copy_(torch.tensor([0, 50, 20], dtype=torch.int32))   # window 1 has T_w = 58
+    cache.pos_base.copy_(torch.tensor([0, 1_234, 987_000], dtype=torch.int32))
+    model = RopeDecodeModel(cache, W, k_sched, theta)
+    ws = cache.new_workspace()
+    scale = 1.0 / math.sqrt(d)
+    for step in range(70):
+        q, kn, vn = inputs.qkv((B, H, d), seed=300 + step, device="cuda")
+        o, lse = focus.attn_decode(cache, q, kn, vn, workspace=ws)
+        focus.kv_compact_window(cache)
+        o_ref, lse_ref = model.step(q, kn, vn, scale)
+        assert_attn_close(o, lse, o_ref, lse_ref, f"rope decode step {step}")
+    torch.cuda.synchronize()
+    assert np.array_equal(cache.ring_len.cpu().numpy(), model.R)
+    assert np.array_equal(cache.win_fill.cpu().numpy(), model.fill)
+    assert np.array_equal(cache.pos_base.cpu().numpy(), model.pos)
+    for b in range(B):
+        R, f = int(model.R[b]), int(model.fill[b])
+        assert_keys_close(cache.ring_k[b, :, :R], model.rk[b, :, :R], f"ring K b={b}", rel=2.0 ** -7)
+        assert_keys_close(cache.win_k[b, :, :f], model.wk[b, :, :f], f"window K b={b}", rel=2.0 ** -7)
+
+
+def test_full_size_streaming_rope_sampled():
+    """Batch 4, N = 1 Mb, W = 1,000, k = 100, 32 heads, d = 128, base 500,000: one
+    prefill and one compaction per window; positions reach 1,009,999. Sampled
+    windows of two heads against the oracle, which sees each row's visible set
+    (the ring rows before its window, then its window up to itself) rotated at
+    the rows' true position ids."""
+    from paper_2511_14694_gb300.workloads import WORKLOADS
+    cfg = WORKLOADS["stream_1mb_b4_h32_d128"]
+    B, N, W, H, d, P = cfg["B"], cfg["N"], cfg["W"], cfg["H"], cfg["d"], cfg["pool"]
+    theta = 500_000.0
+    M = -(-N // W)
+    L = focus.layout(N, W, [cfg["k"][0]])
+    off, roff = L["win_off_host"], L["ring_off_host"]
+    Tw = int(off[1] - off[0])
+    pq, pk, pv = inputs.qkv((P, B, H, Tw, d), std=cfg["std"], seed=inputs.DEFAULT_SEED, device="cuda")
+    cache = focus.Cache(B, H, d, C_ring=L["R"], rope_theta=theta)
+    want = [0, 1, 998, 999]
+    b, heads = 1, [0, 17]
+    got = {}
+    for w in range(M):
+        o, lse = pipeline.prefill_window(cache, pq[w % P], pk[w % P], pv[w % P], L, w)
+        if w in want:
+            got[w] = (o[b, heads].cpu(), lse[b, heads].cpu())
+    torch.cuda.synchronize()
+    ref_L = fo.layout(N, W, [cfg["k"][0]])
+    sum_idx = ref_L["sum_idx"]
+    for i, h in enumerate(heads):
+        pq_h, pk_h, pv_h = (t[:, b, h].cpu() for t in (pq, pk, pv))     # [P, T_w, d]
+        for w in want:
+            a, e = int(off[w]), int(off[w + 1])
+            R_w = int(roff[w])
+            ring_rows = sum_idx[:R_w]                         # augmented indices of the retained rows
+            src_w = torch.from_numpy(ring_rows // Tw)         # every window has T_w rows here
+            in_w = torch.from_numpy(ring_rows % Tw)
+            ring_k, ring_v = pk_h[src_w % P, in_w], pv_h[src_w % P, in_w]
+            kf = np.concatenate([fo.rope(ring_k, ring_rows, theta, round_bf16=True).reshape(R_w, d),
+                                 fo.rope(pk_h[w % P], np.arange(a, e), theta, round_bf16=True)])
+            qf = np.concatenate([np.zeros((R_w, d)), fo.rope(pq_h[w % P], np.arange(a, e), theta, round_bf16=True)])
+            vv = torch.cat([ring_v, pv_h[w % P]])
+            keep = np.concatenate([np.ones(R_w, np.uint8), np.zeros(e - a, np.uint8)])
+            win = np.concatenate([np.zeros(R_w, np.int32), np.ones(e - a, np.int32)])
+            rows = np.arange(R_w, R_w + e - a)
+            o_ref, lse_ref = fo.attn_rows_f64(qf[None], kf[None], vv[None], keep, win, 1.0 / math.sqrt(d),
+                                              np.zeros(rows.size, np.int64), rows)
+            assert_attn_close(got[w][0][i], got[w][1][i], o_ref, lse_ref, f"rope stream w={w} h={h}")

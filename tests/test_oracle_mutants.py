@@ -76,6 +76,8 @@ MUTANTS = [
     ("f64_attention_drops_ring", "if (!((win[j] == win[i]) || (keep[j] == 1))) continue;",
      "if (!(win[j] == win[i])) continue;",
      [lambda: pins.test_fp64_attention_variants_equal_the_pinned_bf16_ones()]),
+    ("round_bf16_ties_away", "double r = nearbyint(ldexp(m, 8));", "double r = round(ldexp(m, 8));",
+     [lambda: pins.test_round_bf16_is_nearest_even_and_matches_torch()]),
     ("decode_skips_self", "        kr[c] = k_new + (size_t)s * d;\n        vr[c] = v_new + (size_t)s * d;\n        c += 1;\n"
      "        softmax_row(d,", "        softmax_row(d,", [lambda: pins.test_decode_equals_prefill_row()]),
 ]

@@ -554,3 +554,26 @@ def test_fp64_attention_variants_equal_the_pinned_bf16_ones():
     b = fo.decode_f64(_f64(qn), _f64(kn), vn, _f64(rk), rv, R, _f64(wk), wv, fill, 0.25)
     np.testing.assert_allclose(a[0], b[0], rtol=0, atol=1e-15)
     np.testing.assert_allclose(a[1], b[1], rtol=0, atol=1e-14)
+
+
+def test_round_bf16_is_nearest_even_and_matches_torch():
+    """Ties go to the even significand (1 + 2^-8 lies halfway between 1 and
+    1 + 2^-7); otherwise the nearest bf16 value, as torch's fp32 -> bf16
+    conversion gives for values that fp32 holds exactly."""
+    assert fo.round_bf16(1.0 + 2.0 ** -8) == 1.0
+    assert fo.round_bf16(1.0 + 3 * 2.0 ** -8) == 1.0 + 2.0 ** -6
+    assert fo.round_bf16(-(1.0 + 3 * 2.0 ** -8)) == -(1.0 + 2.0 ** -6)
+    assert fo.round_bf16(1.0 + 2.0 ** -8 + 2.0 ** -30) == 1.0 + 2.0 ** -7
+    x = inputs.normal_bf16((2000,), 3.0, seed=9).float() * (1 + 1e-3)
+    ref = x.to(torch.bfloat16).double().numpy()
+    got = np.array([fo.round_bf16(float(v)) for v in x.double().numpy()])
+    np.testing.assert_array_equal(got, ref)
+
+
+def test_rope_rounded_is_the_rounded_exact_rotation():
+    x = inputs.normal_bf16((40, 64), 1.0, seed=10)
+    pos = np.arange(40) * 9_973
+    y = fo.rope(x, pos, 10_000.0)
+    yr = fo.rope(x, pos, 10_000.0, round_bf16=True)
+    np.testing.assert_array_equal(yr, np.vectorize(fo.round_bf16)(y))
+    assert (np.abs(yr - y) <= 2.0 ** -8 * np.abs(y)).all()     # half a step of 8 significant bits
