@@ -138,7 +138,24 @@ typedef struct focus_cache {
     int32_t  B, H, d;
     int32_t  C_ring, C_win;   /* capacities in rows */
     int32_t  tail;            /* boundary tail kept by window-mode compaction (>= 0) */
+    int32_t* pos_base;        /* device [B] position id of the current window's first row, or NULL;
+                                 window-mode compaction adds the retired window's T_w to it */
+    float    rope_theta;      /* rotary-embedding base; 0 = none (see below) */
 } focus_cache;
+
+/* Rotary position embedding at the layout's position ids (RoFormer; the paper
+ * gives each FOCUS token a real sequence position, Sec. 3.2, and names no base).
+ * With rope_theta > 0 every query and key the library receives is rotated before
+ * use: for i < d/2 the pair (x_i, x_{i+d/2}) turns by the angle p * theta_i,
+ * theta_i = rope_theta^(-2i/d), p = the row's position id (its global augmented
+ * index). Keys enter the cache rotated: focus_kv_compact in bulk mode rotates the
+ * rows it copies (p = sum_idx entry), focus_attn_decode appends the rotated new
+ * key (p = pos_base[b] + win_fill[b], so pos_base is required), and window-mode
+ * compaction copies already rotated rows. focus_attn_prefill rotates q and the
+ * current windows' k (p = win_off[w] + in-window row) and reads the ring as
+ * stored. Angles are reduced modulo 2 pi in fp64 before the fp32 sine and cosine;
+ * rotated values are rounded to bf16 before they are used. rope_theta must be
+ * finite and >= 0 (FOCUS_ERR_INVALID_ARG otherwise). */
 
 /* ------------------------------------------------------------------------ */
 /* focus_attn_prefill — windowed attention over the compressed context      */

@@ -34,6 +34,7 @@ focus_status from_cuda(cudaError_t e) { return e == cudaSuccess ? FOCUS_OK : FOC
 
 focus_status check_cache(const focus_cache* c, bool need_window) {
     if (!c) return FOCUS_ERR_INVALID_ARG;
+    if (!isfinite(c->rope_theta) || c->rope_theta < 0.f) return FOCUS_ERR_INVALID_ARG;
     if (c->B <= 0 || c->H <= 0 || c->C_ring < 0 || c->C_win < 0 || c->tail < 0) return FOCUS_ERR_INVALID_ARG;
     if (c->d != 64 && c->d != 128) return FOCUS_ERR_UNSUPPORTED;
     if ((int64_t)c->B > 65535 || (int64_t)c->H > 65535) return FOCUS_ERR_UNSUPPORTED;
@@ -49,6 +50,20 @@ focus_status check_cache(const focus_cache* c, bool need_window) {
 }
 
 }  // namespace
+
+namespace focus {
+
+void rope_table_fill(RopeTable* t, int d, float base) {
+    const int h = d / 2, G = 1024 / d;
+    for (int i = 0; i < kRopeMaxPairs; ++i) {
+        const double theta = i < h ? pow((double)base, -2.0 * i / d) : 0.0;
+        t->theta[i] = theta;
+        for (int g = 0; g < kRopeOffRows; ++g)
+            t->off[g][i] = g <= G ? make_float2((float)cos(g * theta), (float)sin(g * theta)) : make_float2(1.f, 0.f);
+    }
+}
+
+}  // namespace focus
 
 extern "C" {
 
@@ -154,8 +169,7 @@ focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_ar
 
 size_t focus_decode_workspace_size(const focus_cache* cache) {
     if (check_cache(cache, false) != FOCUS_OK) return 0;
-    const int64_t ns = focus::decode_num_splits(*cache);
-    return (size_t)((int64_t)cache->B * cache->H * ns * (2 + cache->d)) * sizeof(float);
+    return focus::decode_workspace_bytes(*cache);
 }
 
 focus_status focus_attn_decode(const focus_cache* cache, const void* q, const void* k_new, const void* v_new,
@@ -164,6 +178,7 @@ focus_status focus_attn_decode(const focus_cache* cache, const void* q, const vo
     focus_status s = check_cache(cache, true);
     if (s != FOCUS_OK) return s;
     if (!q || !k_new || !v_new || !o || !workspace || !isfinite(scale)) return FOCUS_ERR_INVALID_ARG;
+    if (cache->rope_theta > 0.f && !cache->pos_base) return FOCUS_ERR_INVALID_ARG;
     if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(o) || !aligned16(workspace))
         return FOCUS_ERR_UNSUPPORTED;
     if (workspace_bytes < focus_decode_workspace_size(cache)) return FOCUS_ERR_CAPACITY;
@@ -179,6 +194,7 @@ focus_status focus_attn_decode_noalloc(const focus_cache* cache, const void* q, 
     focus_status s = check_cache(cache, true);
     if (s != FOCUS_OK) return s;
     if (!q || !k_new || !v_new || !o || !isfinite(scale)) return FOCUS_ERR_INVALID_ARG;
+    if (cache->rope_theta > 0.f && !cache->pos_base) return FOCUS_ERR_INVALID_ARG;
     if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(o)) return FOCUS_ERR_UNSUPPORTED;
     if (focus_decode_workspace_size(cache) > (size_t)FOCUS_DECODE_NOALLOC_SCRATCH_BYTES) return FOCUS_ERR_CAPACITY;
     int32_t* st = nullptr;
@@ -202,6 +218,7 @@ focus_status focus_kv_compact(const focus_cache* cache, const focus_compact_args
             return FOCUS_ERR_INVALID_ARG;
         if (!aligned16(a->src_k) || !aligned16(a->src_v)) return FOCUS_ERR_UNSUPPORTED;
         if (a->w_end == a->w_begin) return FOCUS_OK;
+        if (cache->rope_theta > 0.f) return from_cuda(focus::launch_compact_bulk_rope(*cache, *a, st, stream));
         return from_cuda(focus::launch_compact_bulk(*cache, *a, st, stream));
     }
     return from_cuda(focus::launch_compact_window(*cache, st, stream));

@@ -39,6 +39,52 @@ __host__ __device__ __forceinline__ int64_t tail_start(int64_t n, int32_t tail) 
     return tail > 0 ? (n - tail > 0 ? n - tail : 0) : n;
 }
 
+// ---------------------------------------------------------------- rotary embedding
+// RoFormer rotation with rotate-half pairing at the layout's position ids: the
+// pair (x_i, x_{i+d/2}), i < d/2, turns by p * theta_i, theta_i = base^(-2i/d).
+// Positions reach ~10^6, where an fp32 angle p * theta_i is off by up to ~0.1 rad,
+// so every angle a kernel starts from is formed and reduced modulo 2 pi in fp64
+// and only the reduced angle goes to the fp32 sin/cos. Along a tile, rows step by
+// a fixed offset whose cos/sin come from a host table (fp64 there), so a kernel
+// needs one fp64 angle per pair and tile start, not per element.
+constexpr int kRopeMaxPairs = 64;         // d/2 for d <= 128
+constexpr int kRopeOffRows = 17;          // offsets g = 0..G, G = 1024 / d <= 16
+
+struct RopeTable {
+    double theta[kRopeMaxPairs];          // theta_i
+    float2 off[kRopeOffRows][kRopeMaxPairs];   // (cos, sin)(g * theta_i)
+};
+
+// Host: fill the table for head dimension d (even, <= 128) and base > 0.
+void rope_table_fill(RopeTable* t, int d, float base);
+
+// (cos, sin) of the fp64 angle a, reduced to [-pi, pi] in fp64 first.
+__device__ __forceinline__ float2 rope_cs(double a) {
+    const double two_pi = 6.283185307179586476925286766559;
+    const double r = a - two_pi * rint(a * (1.0 / two_pi));
+    float s, c;
+    __sincosf((float)r, &s, &c);
+    return make_float2(c, s);
+}
+
+// (c1 + i s1)(c2 + i s2): the rotation by the sum of two angles.
+__device__ __forceinline__ float2 rope_mul(float2 a, float2 b) {
+    return make_float2(a.x * b.x - a.y * b.y, a.y * b.x + a.x * b.y);
+}
+
+// Rotate eight pairs held as two 16-byte chunks of bf16 (lo: x_i.., hi: x_{i+d/2}..).
+__device__ __forceinline__ void rope_rotate8(uint4& lo, uint4& hi, const float2* cs) {
+    __nv_bfloat162* l = reinterpret_cast<__nv_bfloat162*>(&lo);
+    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&hi);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const float2 a = __bfloat1622float2(l[e]), b = __bfloat1622float2(h[e]);
+        const float2 c0 = cs[2 * e], c1 = cs[2 * e + 1];
+        l[e] = __floats2bfloat162_rn(a.x * c0.x - b.x * c0.y, a.y * c1.x - b.y * c1.y);
+        h[e] = __floats2bfloat162_rn(b.x * c0.x + a.x * c0.y, b.y * c1.x + a.y * c1.y);
+    }
+}
+
 // Kernel launchers (one translation unit each).
 cudaError_t launch_layout(int64_t N, int32_t W, int32_t M, const int32_t* d_k, bool close_tail,
                           int32_t tail, int32_t B, const uint8_t* d_nt, const focus_layout_out& out,
@@ -46,9 +92,12 @@ cudaError_t launch_layout(int64_t N, int32_t W, int32_t M, const int32_t* d_k, b
 
 cudaError_t launch_compact_bulk(const focus_cache& c, const focus_compact_args& a, int32_t* status,
                                 cudaStream_t stream);
+cudaError_t launch_compact_bulk_rope(const focus_cache& c, const focus_compact_args& a, int32_t* status,
+                                     cudaStream_t stream);
 cudaError_t launch_compact_window(const focus_cache& c, int32_t* status, cudaStream_t stream);
 
 int32_t decode_num_splits(const focus_cache& c);
+size_t decode_workspace_bytes(const focus_cache& c);
 cudaError_t launch_decode(const focus_cache& c, const void* q, const void* k_new, const void* v_new,
                           float scale, void* o, float* lse, void* workspace, int32_t* status,
                           cudaStream_t stream);

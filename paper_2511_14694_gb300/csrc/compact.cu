@@ -44,6 +44,50 @@ __global__ void __launch_bounds__(256) compact_bulk_kernel(
         for (int32_t b = threadIdx.x; b < B; b += blockDim.x) ring_len[b] = r1;
 }
 
+// Bulk mode with the rotary embedding: ring K rows are stored rotated at their
+// position id p = sum_idx[r]. One thread owns one ring row and one pair of
+// 16-byte chunks (columns 8j.. and 8j + d/2..), forms the eight angles p theta_i
+// once (fp64) and applies them to every (sequence, head); V is copied as is.
+template <int D>
+__global__ void __launch_bounds__(256) compact_bulk_rope_kernel(
+        uint4* __restrict__ ring_k, uint4* __restrict__ ring_v, const uint4* __restrict__ src_k,
+        const uint4* __restrict__ src_v, int32_t BH, int32_t B, int32_t C_ring, int64_t src_T, int64_t src_row0,
+        const int32_t* __restrict__ sum_idx, const int32_t* __restrict__ ring_off, int32_t w_begin, int32_t w_end,
+        int32_t* __restrict__ ring_len, const __grid_constant__ RopeTable rope, int32_t* status) {
+    constexpr int CPR = D / 8, HALF = D / 16;   // chunks per row, chunk pairs per row
+    const int32_t r0 = ring_off[w_begin], r1 = ring_off[w_end];
+    const int64_t rows = r1 - r0;
+    if (r1 > C_ring) {
+        if (blockIdx.x == 0 && threadIdx.x == 0) report(status, FOCUS_ERR_CAPACITY);
+        return;
+    }
+    for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < rows * HALF;
+         u += (int64_t)gridDim.x * blockDim.x) {
+        const int j = (int)(u % HALF);
+        const int64_t r = r0 + u / HALF;
+        const int64_t p = sum_idx[r];
+        const int64_t srow = p - src_row0;
+        if (srow < 0 || srow >= src_T) {
+            report(status, FOCUS_ERR_INVALID_ARG);
+            continue;
+        }
+        float2 cs[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) cs[e] = rope_cs((double)p * rope.theta[8 * j + e]);
+        for (int64_t bh = 0; bh < BH; ++bh) {
+            const int64_t so = (bh * src_T + srow) * CPR, d_o = (bh * C_ring + r) * CPR;
+            uint4 lo = src_k[so + j], hi = src_k[so + j + HALF];
+            rope_rotate8(lo, hi, cs);
+            ring_k[d_o + j] = lo;
+            ring_k[d_o + j + HALF] = hi;
+            ring_v[d_o + j] = src_v[so + j];
+            ring_v[d_o + j + HALF] = src_v[so + j + HALF];
+        }
+    }
+    if (blockIdx.x == 0)
+        for (int32_t b = threadIdx.x; b < B; b += blockDim.x) ring_len[b] = r1;
+}
+
 // Window mode: one CTA per sequence. If the current window buffer holds the
 // whole window (W bases + its summaries), append its kept rows (FOCUS rows and
 // the last `tail` bases) to the ring in augmented order and start the next
@@ -53,7 +97,8 @@ __global__ void __launch_bounds__(256) compact_window_kernel(
         uint4* __restrict__ ring_k, uint4* __restrict__ ring_v, const uint4* __restrict__ win_k,
         const uint4* __restrict__ win_v, int32_t* __restrict__ ring_len, int32_t* __restrict__ win_fill,
         int32_t* __restrict__ win_idx, const int32_t* __restrict__ ks, int32_t n_windows, int32_t W,
-        int32_t H, int32_t chunks_per_row, int32_t C_ring, int32_t C_win, int32_t tail, int32_t* status) {
+        int32_t H, int32_t chunks_per_row, int32_t C_ring, int32_t C_win, int32_t tail,
+        int32_t* __restrict__ pos_base, int32_t* status) {
     const int32_t b = blockIdx.x;
     const int32_t fill = win_fill[b], widx = win_idx[b], R = ring_len[b];
     if (widx < 0 || widx >= n_windows) {
@@ -98,6 +143,7 @@ __global__ void __launch_bounds__(256) compact_window_kernel(
         ring_len[b] = R + kept;
         win_fill[b] = 0;
         win_idx[b] = widx + 1;
+        if (pos_base) pos_base[b] += Tw;
     }
 }
 
@@ -119,7 +165,26 @@ cudaError_t launch_compact_bulk(const focus_cache& c, const focus_compact_args& 
 cudaError_t launch_compact_window(const focus_cache& c, int32_t* status, cudaStream_t stream) {
     compact_window_kernel<<<c.B, 256, 0, stream>>>(
         (uint4*)c.ring_k, (uint4*)c.ring_v, (const uint4*)c.win_k, (const uint4*)c.win_v, c.ring_len,
-        c.win_fill, c.win_idx, c.k_per_window, c.n_windows, c.W, c.H, c.d / 8, c.C_ring, c.C_win, c.tail, status);
+        c.win_fill, c.win_idx, c.k_per_window, c.n_windows, c.W, c.H, c.d / 8, c.C_ring, c.C_win, c.tail,
+        c.pos_base, status);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_compact_bulk_rope(const focus_cache& c, const focus_compact_args& a, int32_t* status,
+                                     cudaStream_t stream) {
+    int dev = 0, sms = 152;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    RopeTable rope;
+    rope_table_fill(&rope, c.d, c.rope_theta);
+    if (c.d == 128)
+        compact_bulk_rope_kernel<128><<<sms * 2, 256, 0, stream>>>(
+            (uint4*)c.ring_k, (uint4*)c.ring_v, (const uint4*)a.src_k, (const uint4*)a.src_v, c.B * c.H, c.B,
+            c.C_ring, a.src_T, a.src_row0, a.d_sum_idx, a.d_ring_off, a.w_begin, a.w_end, c.ring_len, rope, status);
+    else
+        compact_bulk_rope_kernel<64><<<sms * 2, 256, 0, stream>>>(
+            (uint4*)c.ring_k, (uint4*)c.ring_v, (const uint4*)a.src_k, (const uint4*)a.src_v, c.B * c.H, c.B,
+            c.C_ring, a.src_T, a.src_row0, a.d_sum_idx, a.d_ring_off, a.w_begin, a.w_end, c.ring_len, rope, status);
     return cudaGetLastError();
 }
 

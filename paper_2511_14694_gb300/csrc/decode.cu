@@ -294,6 +294,34 @@ __global__ void __launch_bounds__(D) decode_combine_kernel(
     }
 }
 
+// Rotary embedding of the new row: q and k_new turn by p theta_i with
+// p = pos_base[b] + win_fill[b], the new row's position id. One block per
+// (head, sequence), one thread per pair; the rotated rows go to the workspace and
+// the split kernel reads them in place of q and k_new.
+template <int D>
+__global__ void __launch_bounds__(D / 2) decode_rope_kernel(
+        const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k_new,
+        __nv_bfloat16* __restrict__ q_rot, __nv_bfloat16* __restrict__ k_rot, const int32_t* __restrict__ pos_base,
+        const int32_t* __restrict__ win_fill, int32_t H, const __grid_constant__ RopeTable rope) {
+    const int b = blockIdx.y, h = blockIdx.x, i = threadIdx.x;
+    const int64_t row = ((int64_t)b * H + h) * D;
+    const int64_t p = (int64_t)pos_base[b] + win_fill[b];
+    const float2 cs = rope_cs((double)p * rope.theta[i]);
+    const float ql = __bfloat162float(q[row + i]), qh = __bfloat162float(q[row + i + D / 2]);
+    const float kl = __bfloat162float(k_new[row + i]), kh = __bfloat162float(k_new[row + i + D / 2]);
+    q_rot[row + i] = __float2bfloat16_rn(ql * cs.x - qh * cs.y);
+    q_rot[row + i + D / 2] = __float2bfloat16_rn(qh * cs.x + ql * cs.y);
+    k_rot[row + i] = __float2bfloat16_rn(kl * cs.x - kh * cs.y);
+    k_rot[row + i + D / 2] = __float2bfloat16_rn(kh * cs.x + kl * cs.y);
+}
+
+// Workspace: split partials (m, l) and o, then, with the rotary embedding, the
+// rotated q and k_new (16-byte aligned).
+size_t partials_bytes(const focus_cache& c) {
+    return (size_t)((int64_t)c.B * c.H * decode_num_splits(c) * (2 + c.d)) * sizeof(float);
+}
+size_t rope_rows_offset(const focus_cache& c) { return (partials_bytes(c) + 255) & ~(size_t)255; }
+
 template <int D>
 cudaError_t launch_decode_d(const focus_cache& c, const void* q, const void* k_new, const void* v_new,
                             float scale, void* o, float* lse, void* workspace, int32_t* status,
@@ -302,6 +330,18 @@ cudaError_t launch_decode_d(const focus_cache& c, const void* q, const void* k_n
     float2* ws_ml = reinterpret_cast<float2*>(workspace);
     float* ws_o = reinterpret_cast<float*>(ws_ml + (int64_t)c.B * c.H * ns);
     dim3 grid(ns, c.H, c.B);
+    if (c.rope_theta > 0.f) {
+        __nv_bfloat16* q_rot = reinterpret_cast<__nv_bfloat16*>((char*)workspace + rope_rows_offset(c));
+        __nv_bfloat16* k_rot = q_rot + (int64_t)c.B * c.H * D;
+        RopeTable rope;
+        rope_table_fill(&rope, D, c.rope_theta);
+        decode_rope_kernel<D><<<dim3(c.H, c.B), D / 2, 0, stream>>>(
+            (const __nv_bfloat16*)q, (const __nv_bfloat16*)k_new, q_rot, k_rot, c.pos_base, c.win_fill, c.H, rope);
+        cudaError_t er = cudaGetLastError();
+        if (er != cudaSuccess) return er;
+        q = q_rot;
+        k_new = k_rot;
+    }
     constexpr int smem = decode_smem_bytes<D>();
     cudaError_t e0 = cudaFuncSetAttribute(decode_split_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e0 != cudaSuccess) return e0;
@@ -321,6 +361,11 @@ cudaError_t launch_decode_d(const focus_cache& c, const void* q, const void* k_n
 
 int32_t decode_num_splits(const focus_cache& c) {
     return (int32_t)ceil_div64((int64_t)c.C_ring + c.C_win, kDecodeChunk);
+}
+
+size_t decode_workspace_bytes(const focus_cache& c) {
+    if (c.rope_theta > 0.f) return rope_rows_offset(c) + 2 * (size_t)c.B * c.H * c.d * sizeof(__nv_bfloat16);
+    return partials_bytes(c);
 }
 
 cudaError_t launch_decode(const focus_cache& c, const void* q, const void* k_new, const void* v_new,

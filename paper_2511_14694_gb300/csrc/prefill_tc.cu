@@ -30,6 +30,13 @@
 //              writes P (bf16) back into TMEM, and at the end normalises O and
 //              stores O and the LSE.
 // TMEM: S_0 cols [0,128), S_1 [128,256), O_0 [256, 256+D), O_1 [256+D, 256+2D).
+//
+// Rotary embedding (ROPE): the softmax warps rotate the two Q tiles in shared
+// memory before the first S = Q K^T (q_rot barrier), and warps 2-3 rotate each
+// window K tile between its TMA arrival and its MMA (k_rot barriers); ring tiles
+// arrive rotated. Each rotating thread owns eight column pairs (i, i + d/2) of a
+// set of rows spaced G apart: one fp64 angle per pair and tile (or 64-row
+// segment) start, then the fixed per-row offsets of a host table.
 // Every mbarrier wait is bounded; on timeout the kernel reports
 // FOCUS_ERR_TIMEOUT, drains its own copies/MMAs (bounded), frees TMEM, returns.
 #include <cudaTypedefs.h>
@@ -59,7 +66,18 @@ struct Cfg {
     static constexpr int kQOff = 0;
     static constexpr int kSlotOff = 2 * kTileBytes;
     static constexpr int kBarOff = kSlotOff + kSlots * kTileBytes;
-    static constexpr int kSmem = kBarOff + 256 + 1024;          // + barriers + alignment slack
+    static constexpr int kRopeOff = kBarOff + 256;              // float2 [4][64] Q bases + [64] K bases
+    static constexpr int kSmem = kRopeOff + 5 * 64 * 8 + 1024;  // + alignment slack
+};
+
+// Kernel argument: the rotary table only for the ROPE variants.
+template <bool ROPE>
+struct RopeArg {
+    RopeTable t;
+};
+template <>
+struct RopeArg<false> {
+    int unused;
 };
 
 struct Bars {
@@ -70,6 +88,8 @@ struct Bars {
     uint64_t p_full[2];
     uint64_t o_full[2];
     uint64_t drain;
+    uint64_t q_rot;       // ROPE: the Q tiles are rotated
+    uint64_t k_rot[2];    // ROPE: the K tile in slot 0 / 2 is rotated (K tiles use the even slots)
     uint32_t tmem;
     int32_t abort;
 };
@@ -80,14 +100,15 @@ __device__ __forceinline__ void fail(Bars* bars, int32_t* status) {
 }
 __device__ __forceinline__ bool aborted(Bars* bars) { return *(volatile int32_t*)&bars->abort != 0; }
 
-template <int D, bool LOCAL>
+template <int D, bool LOCAL, bool ROPE>
 __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
         const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
         const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_rk,
         const __grid_constant__ CUtensorMap tm_rv, __nv_bfloat16* __restrict__ o, float* __restrict__ lse,
         int64_t T_span, const int32_t* __restrict__ win_off, const int32_t* __restrict__ ring_off, int32_t w_begin,
         int32_t w_end, int32_t ctas_pw, int32_t H, int32_t C_ring, float scale_log2, int32_t* status,
-        const int32_t* __restrict__ k_per_window) {
+        const int32_t* __restrict__ k_per_window, const __grid_constant__ RopeArg<ROPE> rope) {
+    static_assert(!ROPE || kSlots == 4, "K tiles must use the even slots");
     using C = Cfg<D>;
     extern __shared__ unsigned char smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -151,6 +172,9 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
             mbar_init(smem_addr(&bars->o_full[t]), 1);
         }
         mbar_init(smem_addr(&bars->drain), 1);
+        mbar_init(smem_addr(&bars->q_rot), 256);
+        mbar_init(smem_addr(&bars->k_rot[0]), 1);
+        mbar_init(smem_addr(&bars->k_rot[1]), 1);
         bars->abort = 0;
         fence_barrier_init();
     }
@@ -208,7 +232,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
             constexpr uint32_t idesc_pv = idesc_bf16_f32(BM, D, false, true);
             const uint32_t sq = smem_addr(smem + C::kQOff);
             const uint32_t sslot = smem_addr(smem + C::kSlotOff);
-            bool ok = mbar_wait(smem_addr(&bars->q), 0, kWaitNs);
+            bool ok = mbar_wait(smem_addr(ROPE ? &bars->q_rot : &bars->q), 0, kWaitNs);
             if (!ok) fail(bars, status);
             for (int j = 0; ok && j <= n_kv_max; ++j) {
                 int vslot = -1, kslot = -1;
@@ -220,7 +244,8 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
                 if (j < n_kv_max) {
                     const int n = 2 * j;
                     kslot = n % kSlots;
-                    if (!mbar_wait(smem_addr(&bars->kv_full[kslot]), (n / kSlots) & 1, kWaitNs)) { ok = false; break; }
+                    const uint32_t kbar = ROPE ? smem_addr(&bars->k_rot[kslot >> 1]) : smem_addr(&bars->kv_full[kslot]);
+                    if (!mbar_wait(kbar, (n / kSlots) & 1, kWaitNs)) { ok = false; break; }
                 }
                 tc_fence_after();
                 for (int t = 0; t < 2; ++t) {
@@ -257,6 +282,51 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
             mma_commit(smem_addr(&bars->drain));
             mbar_wait(smem_addr(&bars->drain), 0, kWaitNs);
         }
+    } else if (ROPE && warp < 4) {
+        // ================================================= K rotation (warps 2-3)
+        if constexpr (ROPE) {
+            constexpr int HALF = D / 16, G = 64 / HALF;
+            const int tau = threadIdx.x - 64;
+            float2* kb = reinterpret_cast<float2*>(smem + C::kRopeOff) + 4 * 64;
+            const int jj = tau % HALF, g = tau / HALF;
+            for (int j = 0; j < n_kv_max; ++j) {
+                const int n = 2 * j, slot = n % kSlots;
+                if (!mbar_wait(smem_addr(&bars->kv_full[slot]), (n / kSlots) & 1, kWaitNs)) {
+                    fail(bars, status);
+                    break;
+                }
+                if (j >= n_ring) {
+                    const int64_t pos0 = (int64_t)win_off[w] + win_lo + (int64_t)(j - n_ring) * BN;
+                    if (tau < D / 2) kb[tau] = rope_cs((double)pos0 * rope.t.theta[tau]);
+                    named_bar_sync(3, 64);
+                    float2 cs[8], st[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        cs[e] = rope_mul(kb[8 * jj + e], rope.t.off[g][8 * jj + e]);
+                        st[e] = rope.t.off[G][8 * jj + e];
+                    }
+                    uint8_t* tile = smem + C::kSlotOff + slot * C::kTileBytes;
+                    const int clo = 8 * jj, chi = 8 * jj + D / 2;
+#pragma unroll 2
+                    for (int m = 0; m < BN / G; ++m) {
+                        const int r = g + G * m;
+                        uint4* plo = reinterpret_cast<uint4*>(tile + (clo / 64) * kBoxBytes + r * 128 +
+                                                              ((((clo % 64) / 8) ^ (r & 7)) << 4));
+                        uint4* phi = reinterpret_cast<uint4*>(tile + (chi / 64) * kBoxBytes + r * 128 +
+                                                              ((((chi % 64) / 8) ^ (r & 7)) << 4));
+                        uint4 lo = *plo, hi = *phi;
+                        rope_rotate8(lo, hi, cs);
+                        *plo = lo;
+                        *phi = hi;
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) cs[e] = rope_mul(cs[e], st[e]);
+                    }
+                    fence_proxy_async_smem();
+                    named_bar_sync(3, 64);
+                }
+                if (tau == 0) mbar_arrive(smem_addr(&bars->k_rot[slot >> 1]));
+            }
+        }
     } else if (warp >= 4) {
         // ================================================= softmax / epilogue
         const int t = (warp - 4) >> 2;                    // 0: warps 4-7, 1: warps 8-11
@@ -275,6 +345,45 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
         const int32_t ring_lim = c_row + bnd;
         float m_run = -INFINITY, l_run = 0.f;
         bool ok = true;
+        if constexpr (ROPE) {
+            // rotate both Q tiles: thread tau owns pair chunk jj of rows 64 seg + g + G m
+            constexpr int HALF = D / 16, G = 64 / HALF;
+            const int tau = threadIdx.x - 128, seg = tau >> 6;
+            float2* qb = reinterpret_cast<float2*>(smem + C::kRopeOff);    // [4][64]
+            const int64_t pos0 = (int64_t)win_off[w] + a0 + 64 * seg;
+            if ((tau & 63) < D / 2) qb[seg * 64 + (tau & 63)] = rope_cs((double)pos0 * rope.t.theta[tau & 63]);
+            named_bar_sync(2, 256);
+            const int jj = tau % HALF, g = (tau / HALF) % G;
+            float2 cs[8], st[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                cs[e] = rope_mul(qb[seg * 64 + 8 * jj + e], rope.t.off[g][8 * jj + e]);
+                st[e] = rope.t.off[G][8 * jj + e];
+            }
+            ok = mbar_wait(smem_addr(&bars->q), 0, kWaitNs);
+            if (ok) {
+                const int clo = 8 * jj, chi = 8 * jj + D / 2;
+#pragma unroll 2
+                for (int m = 0; m < 64 / G; ++m) {
+                    const int rho = 64 * seg + g + G * m, tq = rho >> 7, rr = rho & 127;
+                    uint8_t* tile = smem + C::kQOff + tq * C::kTileBytes;
+                    uint4* plo = reinterpret_cast<uint4*>(tile + (clo / 64) * kBoxBytes + rr * 128 +
+                                                          ((((clo % 64) / 8) ^ (rr & 7)) << 4));
+                    uint4* phi = reinterpret_cast<uint4*>(tile + (chi / 64) * kBoxBytes + rr * 128 +
+                                                          ((((chi % 64) / 8) ^ (rr & 7)) << 4));
+                    uint4 lo = *plo, hi = *phi;
+                    rope_rotate8(lo, hi, cs);
+                    *plo = lo;
+                    *phi = hi;
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) cs[e] = rope_mul(cs[e], st[e]);
+                }
+                fence_proxy_async_smem();
+            } else {
+                fail(bars, status);
+            }
+            mbar_arrive(smem_addr(&bars->q_rot));
+        }
         for (int j = 0; j < n_kv; ++j) {
             if (!mbar_wait(smem_addr(&bars->s_full[t]), j & 1, kWaitNs)) { ok = false; break; }
             tc_fence_after();
@@ -459,7 +568,7 @@ cudaError_t make_map(CUtensorMap* m, const void* ptr, int d, int64_t rows, int64
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-template <int D, bool LOCAL>
+template <int D, bool LOCAL, bool ROPE>
 cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t* status, cudaStream_t stream) {
     const int64_t BH = (int64_t)c.B * c.H;
     CUtensorMap tq, tk, tv, trk, trv;
@@ -475,13 +584,16 @@ cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t*
         trv = tv;
     }
     const int smem = Cfg<D>::kSmem;
-    e = cudaFuncSetAttribute(prefill_tc_kernel<D, LOCAL>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    e = cudaFuncSetAttribute(prefill_tc_kernel<D, LOCAL, ROPE>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     const int ctas_pw = (a.max_rows + 2 * BM - 1) / (2 * BM);
     dim3 grid((unsigned)((a.w_end - a.w_begin) * ctas_pw), c.H, c.B);
-    prefill_tc_kernel<D, LOCAL><<<grid, kThreads, smem, stream>>>(
+    RopeArg<ROPE> rope;
+    if constexpr (ROPE) rope_table_fill(&rope.t, D, c.rope_theta);
+    else rope.unused = 0;
+    prefill_tc_kernel<D, LOCAL, ROPE><<<grid, kThreads, smem, stream>>>(
         tq, tk, tv, trk, trv, (__nv_bfloat16*)a.o, a.lse, a.T_span, a.d_win_off, a.d_ring_off,
-        a.w_begin, a.w_end, ctas_pw, c.H, c.C_ring, a.scale * 1.4426950408889634f, status, c.k_per_window);
+        a.w_begin, a.w_end, ctas_pw, c.H, c.C_ring, a.scale * 1.4426950408889634f, status, c.k_per_window, rope);
     return cudaGetLastError();
 }
 
@@ -489,9 +601,13 @@ cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t*
 
 cudaError_t launch_prefill_tc(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
                               cudaStream_t stream) {
-    const bool local = (a.flags & FOCUS_PREFILL_KMER_LOCAL) != 0;
-    if (c.d == 128) return local ? launch_d<128, true>(c, a, status, stream) : launch_d<128, false>(c, a, status, stream);
-    return local ? launch_d<64, true>(c, a, status, stream) : launch_d<64, false>(c, a, status, stream);
+    const bool local = (a.flags & FOCUS_PREFILL_KMER_LOCAL) != 0, rope = c.rope_theta > 0.f;
+    if (c.d == 128) {
+        if (rope) return local ? launch_d<128, true, true>(c, a, status, stream) : launch_d<128, false, true>(c, a, status, stream);
+        return local ? launch_d<128, true, false>(c, a, status, stream) : launch_d<128, false, false>(c, a, status, stream);
+    }
+    if (rope) return local ? launch_d<64, true, true>(c, a, status, stream) : launch_d<64, false, true>(c, a, status, stream);
+    return local ? launch_d<64, true, false>(c, a, status, stream) : launch_d<64, false, false>(c, a, status, stream);
 }
 
 }  // namespace focus

@@ -43,7 +43,8 @@ class LayoutOut(ctypes.Structure):
 class CacheDesc(ctypes.Structure):
     _fields_ = [("ring_k", _P), ("ring_v", _P), ("win_k", _P), ("win_v", _P), ("ring_len", _P),
                 ("win_fill", _P), ("win_idx", _P), ("k_per_window", _P), ("n_windows", _i32), ("W", _i32),
-                ("B", _i32), ("H", _i32), ("d", _i32), ("C_ring", _i32), ("C_win", _i32), ("tail", _i32)]
+                ("B", _i32), ("H", _i32), ("d", _i32), ("C_ring", _i32), ("C_win", _i32), ("tail", _i32),
+                ("pos_base", _P), ("rope_theta", _f32)]
 
 
 class PrefillArgs(ctypes.Structure):
@@ -187,8 +188,12 @@ class Cache:
     current window buffer) and its C descriptor."""
 
     def __init__(self, B: int, H: int, d: int, C_ring: int, C_win: int = 0, W: int = 0, k_sched=None,
-                 device="cuda", tail: int = 0):
+                 device="cuda", tail: int = 0, rope_theta: float = 0.0):
+        """``rope_theta`` > 0 turns on the rotary embedding of queries and keys at
+        their position ids; ``pos_base`` [B] (zeros here) holds the position id of
+        each sequence's current decode window's first row."""
         self.B, self.H, self.d, self.C_ring, self.C_win, self.W, self.tail = B, H, d, C_ring, C_win, W, tail
+        self.rope_theta = float(rope_theta)
         bf = dict(dtype=torch.bfloat16, device=device)
         self.ring_k = torch.zeros((B, H, max(C_ring, 1), d), **bf)
         self.ring_v = torch.zeros((B, H, max(C_ring, 1), d), **bf)
@@ -197,11 +202,13 @@ class Cache:
         self.ring_len = torch.zeros(B, dtype=torch.int32, device=device)
         self.win_fill = torch.zeros(B, dtype=torch.int32, device=device)
         self.win_idx = torch.zeros(B, dtype=torch.int32, device=device)
+        self.pos_base = torch.zeros(B, dtype=torch.int32, device=device)
         ks = np.zeros(1, np.int32) if k_sched is None else np.asarray(k_sched, dtype=np.int32).reshape(-1)
         self.k_sched = torch.from_numpy(ks.copy()).to(device)
         self.desc = CacheDesc(_ptr(self.ring_k), _ptr(self.ring_v), _ptr(self.win_k), _ptr(self.win_v),
                               _ptr(self.ring_len), _ptr(self.win_fill), _ptr(self.win_idx), _ptr(self.k_sched),
-                              int(self.k_sched.numel()), W, B, H, d, C_ring, C_win, tail)
+                              int(self.k_sched.numel()), W, B, H, d, C_ring, C_win, tail, _ptr(self.pos_base),
+                              self.rope_theta)
 
     def workspace_bytes(self) -> int:
         return int(load().focus_decode_workspace_size(ctypes.byref(self.desc)))
