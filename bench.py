@@ -274,7 +274,7 @@ def run_prefill_leg(args, cfg, world, rank, local):
     nt = inputs.nucleotides(B, N, seed=inputs.DEFAULT_SEED, device=dev)
     L = focus.layout_alloc(N, W, k_s, B=B, device=dev)
     q, k, v = inputs.qkv((B, H, L["T"], d), std=cfg["std"], seed=inputs.DEFAULT_SEED + rank, device=dev)
-    cache = focus.Cache(B, H, d, C_ring=max(L["R"], 1), device=dev, k_sched=k_s)
+    cache = focus.Cache(B, H, d, C_ring=max(L["R"], 1), device=dev, k_sched=k_s, rope_theta=args.rope)
     o = torch.empty_like(q)
     lse = torch.empty((B, H, L["T"]), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
@@ -395,7 +395,7 @@ def run_stream_leg(args, cfg, world, rank, local):
     if not (np.diff(off) == Tw).all():
         raise ValueError("the streaming leg expects windows of equal augmented size")
     pq, pk, pv = inputs.qkv((P, B, H, Tw, d), std=cfg["std"], seed=inputs.DEFAULT_SEED + rank, device=dev)
-    cache = focus.Cache(B, H, d, C_ring=max(L["R"], 1), device=dev, k_sched=k_s)
+    cache = focus.Cache(B, H, d, C_ring=max(L["R"], 1), device=dev, k_sched=k_s, rope_theta=args.rope)
     local_mask = bool(args.prefill_flags & focus.PREFILL_KMER_LOCAL)
     outs = [torch.empty((B, H, Tw, d), dtype=torch.bfloat16, device=dev) for _ in range(2)]
     lses = [torch.empty((B, H, Tw), dtype=torch.float32, device=dev) for _ in range(2)]
@@ -451,7 +451,7 @@ def run_decode_leg(args, cfg, world, rank, local):
     S = cfg["steps"]
     dev = torch.device("cuda", local)
     k_sched = np.full(R // (W // kk) + S // W + 16, kk, np.int32)
-    cache = focus.Cache(B, H, d, C_ring=R + 256, C_win=1_024, W=W, k_sched=k_sched, device=dev)
+    cache = focus.Cache(B, H, d, C_ring=R + 256, C_win=1_024, W=W, k_sched=k_sched, device=dev, rope_theta=args.rope)
     for i, t in enumerate((cache.ring_k, cache.ring_v, cache.win_k, cache.win_v)):
         t.copy_(inputs.normal_bf16(t.shape, cfg["std"], seed=50 + i + 10 * rank, device=dev))
     fill0 = inputs.start_fill(B, Tw - 1, seed=inputs.DEFAULT_SEED)
@@ -538,7 +538,7 @@ def run_focus(args, world, rank, local):
     value = weak_scaling_value(cfg["B"] * cfg["N"], world, pre["step_ms"] / 1e3)
     achieved = pre["flops_per_step"] / (pre["attn_ms"] / 1e3) / 1e12
     local_mask = pre.get("local_mask", False)
-    traffic = None if args.legacy else kernel_traffic(
+    traffic = None if (args.legacy or args.rope) else kernel_traffic(
         "prefill_attention_kmer_local" if local_mask else "prefill_attention",
         "paper_2511_14694_gb300/csrc/prefill_tc.cu")
     if traffic is not None and cfg is not WORKLOADS["prefill_128kb_h32_d128"]:
@@ -558,7 +558,8 @@ def run_focus(args, world, rank, local):
                        2 * cfg["B"] * cfg["H"] * pre["R"] * cfg["d"] * 2 / 1e9) if cfg["mode"] == "stream" else
                           "inputs larger than L2 (Q/K/V %.2f GB per step)" % (3 * cfg["B"] * pre["T"] * cfg["H"] * cfg["d"] * 2 / 1e9)),
                    "prefill_kernel": "legacy mma.sync" if args.prefill_flags & 1 else "default",
-                   "mask": "k-mer-local (Sec. 3.2)" if local_mask else "appendix (App. A, Eq. focus-attn)"},
+                   "mask": "k-mer-local (Sec. 3.2)" if local_mask else "appendix (App. A, Eq. focus-attn)",
+                   "rope_theta": args.rope or None},
         "augmented_tokens_per_s": world * cfg["B"] * pre["T"] / (pre["step_ms"] / 1e3),
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
                      "frac": achieved / peaks["bf16_tflops"], "traffic": traffic,
@@ -599,7 +600,9 @@ def run_focus(args, world, rank, local):
             "clocks": dec["clocks"],
         }
         line["decode"]["gpu_launches"] = dec["launches"]
-    if pre["host_sample"] is not None:
+    if pre["host_sample"] is not None and args.rope:
+        line["cpu_baseline"] = None      # the oracle baseline times the path without the rotation
+    elif pre["host_sample"] is not None:
         hs = pre["host_sample"]
         if local_mask:
             from oracle import focus_oracle as fo
@@ -739,6 +742,8 @@ def main():
     ap.add_argument("--no-clock-wait", action="store_true",
                     help="do not extend the load after a short timed region (profiling runs)")
     ap.add_argument("--legacy", action="store_true", help="time the legacy mma.sync prefill kernel")
+    ap.add_argument("--rope", type=float, default=0.0,
+                    help="rotary-embedding base (0 = none): q and k are rotated at their position ids")
     ap.add_argument("--mask", default="appendix", choices=["appendix", "kmer_local"],
                     help="prefill visibility: App. A (default) or the k-mer-local rule of Sec. 3.2")
     ap.add_argument("--memory-report", action="store_true",

@@ -7,13 +7,13 @@
  *   M = ceil(N/W)). Inside each window a FOCUS summary token is inserted after
  *   every k_w bases, and after the partial k-mer that ends a window
  *   (B_w = ceil(|I_w|/k_w), App. A; Sec. 3.2 "Setup and tokens"). Each inserted
- *   token occupies a real sequence position. Row i of window w attends to
+ *   token takes a position of its own in the sequence. Row i of window w attends to
  *   (a) the retained FOCUS K/V of all earlier windows and (b) the rows of
  *   window w up to and including itself (Eq. focus-attn's visible set and the
  *   context C(t) of App. A.1). After window w only its FOCUS K/V is kept
  *   (App. A, "KV compression and budget"; App. A.2 streaming inference),
  *   optionally with a boundary tail: the window's last `tail` ordinary rows
- *   (App. A, "plus a small boundary tail if required"). Kept rows form the
+ *   (App. A allows a short boundary tail besides them). Kept rows form the
  *   ring that every later window attends to.
  *
  * Conventions for every entry point
@@ -79,8 +79,8 @@ focus_status focus_get_device_status(int32_t* host_status, int32_t clear, cudaSt
 
 /* ------------------------------------------------------------------------ */
 /* focus_layout — summary-token insertion and position ids                  */
-/* Sec. 3.2 "Setup and tokens"; App. A (I_w, M, B_w; FOCUS tokens occupy     */
-/* real sequence positions); Sec. 3.3 (augmented sequence y_1..y_N').       */
+/* Sec. 3.2 "Setup and tokens"; App. A (I_w, M, B_w; a FOCUS token has a     */
+/* position of its own); Sec. 3.3 (augmented sequence y_1..y_N').           */
 /* ------------------------------------------------------------------------ */
 
 /* Host-only arithmetic: sizes of the augmented layout.
@@ -144,7 +144,7 @@ typedef struct focus_cache {
 } focus_cache;
 
 /* Rotary position embedding at the layout's position ids (RoFormer; the paper
- * gives each FOCUS token a real sequence position, Sec. 3.2, and names no base).
+ * gives each FOCUS token a position of its own, Sec. 3.2, and names no base).
  * With rope_theta > 0 every query and key the library receives is rotated before
  * use: for i < d/2 the pair (x_i, x_{i+d/2}) turns by the angle p * theta_i,
  * theta_i = rope_theta^(-2i/d), p = the row's position id (its global augmented
@@ -179,7 +179,8 @@ typedef struct focus_prefill_args {
 } focus_prefill_args;
 
 /* Use the legacy mma.sync kernel instead of the tcgen05/TMEM kernel (kept as the
- * comparison baseline; same results within rounding). */
+ * comparison baseline; same results within rounding). It has no rotary
+ * embedding: with cache->rope_theta > 0 the call returns FOCUS_ERR_UNSUPPORTED. */
 #define FOCUS_PREFILL_LEGACY_MMA 1u
 
 /* Main-text k-mer-local visibility (Sec. 3.2 "Visibility and summarization rule")
@@ -211,7 +212,7 @@ focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_ar
 
 /* ------------------------------------------------------------------------ */
 /* focus_attn_decode — one new token per sequence against the compressed    */
-/* cache (App. A.2; the decode interface "identical to the base decoder").  */
+/* cache (App. A.2; decoding keeps the base decoder's interface).           */
 /* ------------------------------------------------------------------------ */
 
 /* Bytes of device workspace focus_attn_decode needs for this cache shape. */

@@ -8,7 +8,7 @@
  *
  * Conventions
  *   - Nucleotide ids are 0..3 (A, C, G, T); the reserved summary-token id is 4
- *     (Table "Full configuration": "Special FOCUS token: reserved").
+ *     (Table "Full configuration" lists a reserved id for the FOCUS token).
  *   - Indices are 0-based. Window w covers bases [w*W, min((w+1)*W, N)), the
  *     0-based form of I_w = [(w-1)W+1, wW] ∩ [1, L]  (App. A, first display).
  *   - Q/K/V arrive as raw bf16 bit patterns (uint16) exactly as the GPU sees
@@ -18,8 +18,8 @@
  *     exponentials of the scaled scores.
  *
  * KV retention keeps each window's FOCUS rows and, optionally, a boundary
- * tail: the last `tail` ordinary (base) rows of the window (App. A, "plus a
- * small boundary tail if required"; App. A.2). tail = 0 is the paper's default.
+ * tail: the last `tail` ordinary (base) rows of the window (App. A allows a
+ * short boundary tail besides the FOCUS rows; App. A.2). tail = 0 is the paper's default.
  * A kept row is visible to every later window.
  *
  * Every loop below runs in the order the paper states the operation; nothing is
@@ -42,7 +42,7 @@ static double bf16_to_f64(uint16_t bits) {
 /* ------------------------------------------------------------------------- */
 /* Token layout (App. A: windows I_w, M = ceil(L/W), B_w = ceil(|I_w|/k),     */
 /* one FOCUS token per k real bases at the right boundary of its k-mer,       */
-/* each FOCUS token occupying a real sequence position).                      */
+/* each FOCUS token taking a position of its own, as a base does).           */
 /* ------------------------------------------------------------------------- */
 
 /* Does a summary follow the base at in-window offset o (0-based) of a window
@@ -84,7 +84,7 @@ int64_t fo_layout_size(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
 /* Full layout walk. For every augmented index t:
  *   kind[t]  0 = ordinary base, 1 = FOCUS summary
  *   src[t]   nucleotide index of the base (for a summary: its k-mer's last base)
- *   pos[t]   position id = t (a summary occupies a real sequence position)
+ *   pos[t]   position id = t (a summary has a position of its own)
  *   win[t]   window id w
  *   tok[b*T + t]  nucleotide id nt[b*N + src] for bases, 4 for summaries
  *                 (written only when nt and tok are both non-NULL)
@@ -406,8 +406,8 @@ void fo_attn_rows_kmer_local(int64_t T, int32_t d, const uint8_t* kind, const in
 
 /* ------------------------------------------------------------------------- */
 /* Rotary position embedding at the layout's position ids (RoFormer, Su et    */
-/* al. 2021; the position id of a row is its augmented index, Sec. 3.2 "each  */
-/* FOCUS token occupies a real sequence position"). Rotate-half pairing: for  */
+/* al. 2021; the position id of a row is its augmented index: Sec. 3.2 gives  */
+/* each FOCUS token a position of its own). Rotate-half pairing: for         */
 /* i < d/2, the pair (x_i, x_{i+d/2}) is turned by the angle p * theta_i,     */
 /* theta_i = base^(-2i/d):                                                    */
 /*   y_i       = x_i cos(p theta_i) - x_{i+d/2} sin(p theta_i)                */

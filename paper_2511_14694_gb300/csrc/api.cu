@@ -152,6 +152,7 @@ focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_ar
     if (!isfinite(a->scale) || !(a->scale > 0.f)) return FOCUS_ERR_INVALID_ARG;
     if (!aligned16(a->q) || !aligned16(a->k) || !aligned16(a->v) || !aligned16(a->o)) return FOCUS_ERR_UNSUPPORTED;
     if (a->flags & ~(uint32_t)(FOCUS_PREFILL_LEGACY_MMA | FOCUS_PREFILL_KMER_LOCAL)) return FOCUS_ERR_INVALID_ARG;
+    if ((a->flags & FOCUS_PREFILL_LEGACY_MMA) && cache->rope_theta > 0.f) return FOCUS_ERR_UNSUPPORTED;
     if (a->flags & FOCUS_PREFILL_KMER_LOCAL) {
         if (a->flags & FOCUS_PREFILL_LEGACY_MMA) return FOCUS_ERR_UNSUPPORTED;
         if (cache->tail != 0) return FOCUS_ERR_UNSUPPORTED;

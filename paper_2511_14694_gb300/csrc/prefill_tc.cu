@@ -94,6 +94,67 @@ struct Bars {
     int32_t abort;
 };
 
+// Rotation of eight column pairs (one 16-byte chunk and its partner d/2 columns
+// on), as four packed pairs of element pairs: c = cos, s = sin, n = -sin.
+struct Rot8 {
+    uint64_t c[4], s[4], n[4];
+};
+
+__device__ __forceinline__ Rot8 rot8_make(const float2* cs) {
+    Rot8 r;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        r.c[k] = f2_pack(cs[2 * k].x, cs[2 * k + 1].x);
+        r.s[k] = f2_pack(cs[2 * k].y, cs[2 * k + 1].y);
+        r.n[k] = f2_pack(-cs[2 * k].y, -cs[2 * k + 1].y);
+    }
+    return r;
+}
+
+// y_lo = x_lo c - x_hi s, y_hi = x_hi c + x_lo s on bf16 chunks, rounded once to bf16.
+__device__ __forceinline__ void rot8_apply(uint4& lo, uint4& hi, const Rot8& r) {
+    uint32_t* l = reinterpret_cast<uint32_t*>(&lo);
+    uint32_t* h = reinterpret_cast<uint32_t*>(&hi);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const uint64_t xl = f2_pack(__uint_as_float(l[k] << 16), __uint_as_float(l[k] & 0xffff0000u));
+        const uint64_t xh = f2_pack(__uint_as_float(h[k] << 16), __uint_as_float(h[k] & 0xffff0000u));
+        const uint64_t yl = f2_fma(xh, r.n[k], f2_mul(xl, r.c[k]));
+        const uint64_t yh = f2_fma(xl, r.s[k], f2_mul(xh, r.c[k]));
+        float a, b;
+        f2_unpack(yl, a, b);
+        l[k] = pack_bf16x2(a, b);
+        f2_unpack(yh, a, b);
+        h[k] = pack_bf16x2(a, b);
+    }
+}
+
+// r <- r turned further by the angles of st.
+__device__ __forceinline__ void rot8_step(Rot8& r, const Rot8& st) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const uint64_t c = f2_fma(r.c[k], st.c[k], f2_mul(r.s[k], st.n[k]));
+        const uint64_t sn = f2_fma(r.s[k], st.c[k], f2_mul(r.c[k], st.s[k]));
+        const uint64_t n = f2_fma(r.n[k], st.c[k], f2_mul(r.c[k], st.n[k]));
+        r.c[k] = c;
+        r.s[k] = sn;
+        r.n[k] = n;
+    }
+}
+
+// (cos, sin) of the small angles g theta_i and G theta_i (|angle| <= 16) for the
+// eight pairs i0..i0+7: fp32 is accurate to ~1e-6 rad here.
+__device__ __forceinline__ void rope_offsets(const RopeTable& t, int i0, int g, int G, float2* off, Rot8& step) {
+    float2 st[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        const float th = (float)t.theta[i0 + e];
+        __sincosf((float)g * th, &off[e].y, &off[e].x);
+        __sincosf((float)G * th, &st[e].y, &st[e].x);
+    }
+    step = rot8_make(st);
+}
+
 __device__ __forceinline__ void fail(Bars* bars, int32_t* status) {
     report(status, FOCUS_ERR_TIMEOUT);
     atomicExch(&bars->abort, 1);
@@ -289,6 +350,10 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
             const int tau = threadIdx.x - 64;
             float2* kb = reinterpret_cast<float2*>(smem + C::kRopeOff) + 4 * 64;
             const int jj = tau % HALF, g = tau / HALF;
+            float2 off[8];
+            Rot8 step;
+            rope_offsets(rope.t, 8 * jj, g, G, off, step);
+            const double theta_own = tau < D / 2 ? rope.t.theta[tau] : 0.0;
             for (int j = 0; j < n_kv_max; ++j) {
                 const int n = 2 * j, slot = n % kSlots;
                 if (!mbar_wait(smem_addr(&bars->kv_full[slot]), (n / kSlots) & 1, kWaitNs)) {
@@ -297,14 +362,12 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
                 }
                 if (j >= n_ring) {
                     const int64_t pos0 = (int64_t)win_off[w] + win_lo + (int64_t)(j - n_ring) * BN;
-                    if (tau < D / 2) kb[tau] = rope_cs((double)pos0 * rope.t.theta[tau]);
+                    if (tau < D / 2) kb[tau] = rope_cs((double)pos0 * theta_own);
                     named_bar_sync(3, 64);
-                    float2 cs[8], st[8];
+                    float2 cs[8];
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        cs[e] = rope_mul(kb[8 * jj + e], rope.t.off[g][8 * jj + e]);
-                        st[e] = rope.t.off[G][8 * jj + e];
-                    }
+                    for (int e = 0; e < 8; ++e) cs[e] = rope_mul(kb[8 * jj + e], off[e]);
+                    Rot8 rot = rot8_make(cs);
                     uint8_t* tile = smem + C::kSlotOff + slot * C::kTileBytes;
                     const int clo = 8 * jj, chi = 8 * jj + D / 2;
 #pragma unroll 2
@@ -315,11 +378,10 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
                         uint4* phi = reinterpret_cast<uint4*>(tile + (chi / 64) * kBoxBytes + r * 128 +
                                                               ((((chi % 64) / 8) ^ (r & 7)) << 4));
                         uint4 lo = *plo, hi = *phi;
-                        rope_rotate8(lo, hi, cs);
+                        rot8_apply(lo, hi, rot);
                         *plo = lo;
                         *phi = hi;
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) cs[e] = rope_mul(cs[e], st[e]);
+                        rot8_step(rot, step);
                     }
                     fence_proxy_async_smem();
                     named_bar_sync(3, 64);
@@ -352,14 +414,15 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
             float2* qb = reinterpret_cast<float2*>(smem + C::kRopeOff);    // [4][64]
             const int64_t pos0 = (int64_t)win_off[w] + a0 + 64 * seg;
             if ((tau & 63) < D / 2) qb[seg * 64 + (tau & 63)] = rope_cs((double)pos0 * rope.t.theta[tau & 63]);
-            named_bar_sync(2, 256);
             const int jj = tau % HALF, g = (tau / HALF) % G;
-            float2 cs[8], st[8];
+            float2 off[8];
+            Rot8 step;
+            rope_offsets(rope.t, 8 * jj, g, G, off, step);
+            named_bar_sync(2, 256);
+            float2 cs[8];
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                cs[e] = rope_mul(qb[seg * 64 + 8 * jj + e], rope.t.off[g][8 * jj + e]);
-                st[e] = rope.t.off[G][8 * jj + e];
-            }
+            for (int e = 0; e < 8; ++e) cs[e] = rope_mul(qb[seg * 64 + 8 * jj + e], off[e]);
+            Rot8 rot = rot8_make(cs);
             ok = mbar_wait(smem_addr(&bars->q), 0, kWaitNs);
             if (ok) {
                 const int clo = 8 * jj, chi = 8 * jj + D / 2;
@@ -372,11 +435,10 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
                     uint4* phi = reinterpret_cast<uint4*>(tile + (chi / 64) * kBoxBytes + rr * 128 +
                                                           ((((chi % 64) / 8) ^ (rr & 7)) << 4));
                     uint4 lo = *plo, hi = *phi;
-                    rope_rotate8(lo, hi, cs);
+                    rot8_apply(lo, hi, rot);
                     *plo = lo;
                     *phi = hi;
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) cs[e] = rope_mul(cs[e], st[e]);
+                    rot8_step(rot, step);
                 }
                 fence_proxy_async_smem();
             } else {

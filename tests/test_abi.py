@@ -143,6 +143,9 @@ def test_rope_argument_checks_need_no_gpu():
         assert lib.focus_attn_prefill(ctypes.byref(c), ctypes.byref(a), None) == 1
     c.rope_theta = 10_000.0
     assert lib.focus_attn_prefill(ctypes.byref(c), ctypes.byref(a), None) == 0
+    a.flags = focus.PREFILL_LEGACY_MMA                        # the legacy kernel has no rotation
+    assert lib.focus_attn_prefill(ctypes.byref(c), ctypes.byref(a), None) == 2
+    a.flags = 0
     c.win_k = c.win_v = c.ring_len = c.win_fill = c.win_idx = c.k_per_window = 4096
     c.W, c.n_windows, c.C_win = 10, 1, 16
     assert lib.focus_attn_decode(ctypes.byref(c), 4096, 4096, 4096, ctypes.c_float(0.125), 4096, None, 4096,
