@@ -58,24 +58,39 @@ static int summary_after(int64_t o, int64_t n, int32_t k, int close_partial) {
 /* Is the base at in-window offset o of an n-base window in its boundary tail? */
 static int in_tail(int64_t o, int64_t n, int32_t tail) { return tail > 0 && o >= n - tail; }
 
+/* Window w covers the W_sched[w] bases after the previous windows' (the last
+ * one may hold fewer): windows of one length W are W_sched[w] = W, and adaptive
+ * windowing (choosing W, like k, per region; Sec. 5) gives each its own.
+ * Returns 0 if the schedule of M windows covers exactly N bases with every
+ * window non-empty, else -1. */
+static int32_t check_windows(int64_t N, int32_t M, const int32_t* W_sched) {
+    if (N < 0 || M < 0 || (M > 0 && !W_sched)) return -1;
+    int64_t start = 0;
+    for (int32_t w = 0; w < M; ++w) {
+        if (W_sched[w] <= 0 || start >= N) return -1;
+        start += W_sched[w];
+    }
+    return start >= N ? 0 : -1;
+}
+
+static int64_t window_bases(int64_t N, int64_t start, int32_t W) { return (N - start < W) ? (N - start) : W; }
+
 /* Sizes of the augmented layout. Returns T (augmented length) and writes R
  * (rows retained after the last window: summaries plus boundary tails).
  * Returns -1 on bad arguments. */
-int64_t fo_layout_size(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
-                       int32_t close_tail, int32_t tail, int64_t* R_out) {
-    if (N < 0 || W <= 0 || tail < 0) return -1;
-    int64_t M_expect = (N + W - 1) / W;
-    if (M != M_expect) return -1;
-    int64_t T = 0, R = 0;
+int64_t fo_layout_size_sched(int64_t N, int32_t M, const int32_t* W_sched, const int32_t* k_sched,
+                             int32_t close_tail, int32_t tail, int64_t* R_out) {
+    if (tail < 0 || check_windows(N, M, W_sched) != 0) return -1;
+    int64_t T = 0, R = 0, start = 0;
     for (int32_t w = 0; w < M; ++w) {
-        int64_t start = (int64_t)w * W;
-        int64_t n = (N - start < W) ? (N - start) : W;
+        int64_t n = window_bases(N, start, W_sched[w]);
         int close = (w < M - 1) || close_tail;
         for (int64_t o = 0; o < n; ++o) {
             T += 1;
             if (in_tail(o, n, tail)) R += 1;
             if (summary_after(o, n, k_sched[w], close)) { T += 1; R += 1; }
         }
+        start += W_sched[w];
     }
     if (R_out) *R_out = R;
     return T;
@@ -90,24 +105,25 @@ int64_t fo_layout_size(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
  *                 (written only when nt and tok are both non-NULL)
  *   keep[t]  1 if KV retention keeps the row (a summary, or a boundary-tail base)
  * plus win_off[M+1] (first augmented index of each window, win_off[M] = T),
- * ring_off[M+1] (rows retained before each window, ring_off[M] = R) and
- * sum_idx[R] (augmented index of each retained row, in order).
+ * ring_off[M+1] (rows retained before each window, ring_off[M] = R),
+ * sum_idx[R] (augmented index of each retained row, in order) and, if not NULL,
+ * base_off[M+1] (first base of each window, base_off[M] = N).
  * Returns T, or -1 on bad arguments. */
-int64_t fo_layout(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
-                  int32_t close_tail, int32_t tail, int32_t B, const uint8_t* nt,
-                  uint8_t* kind, int32_t* src, int32_t* pos, int32_t* win,
-                  uint8_t* tok, uint8_t* keep, int32_t* win_off, int32_t* ring_off,
-                  int32_t* sum_idx) {
+int64_t fo_layout_sched(int64_t N, int32_t M, const int32_t* W_sched, const int32_t* k_sched,
+                        int32_t close_tail, int32_t tail, int32_t B, const uint8_t* nt,
+                        uint8_t* kind, int32_t* src, int32_t* pos, int32_t* win,
+                        uint8_t* tok, uint8_t* keep, int32_t* win_off, int32_t* ring_off,
+                        int32_t* sum_idx, int32_t* base_off) {
     int64_t R_total = 0;
-    int64_t T_total = fo_layout_size(N, W, M, k_sched, close_tail, tail, &R_total);
+    int64_t T_total = fo_layout_size_sched(N, M, W_sched, k_sched, close_tail, tail, &R_total);
     if (T_total < 0) return -1;
-    int64_t t = 0, r = 0;
+    int64_t t = 0, r = 0, start = 0;
     for (int32_t w = 0; w < M; ++w) {
-        int64_t start = (int64_t)w * W;
-        int64_t n = (N - start < W) ? (N - start) : W;
+        int64_t n = window_bases(N, start, W_sched[w]);
         int close = (w < M - 1) || close_tail;
         win_off[w] = (int32_t)t;
         ring_off[w] = (int32_t)r;
+        if (base_off) base_off[w] = (int32_t)start;
         for (int64_t o = 0; o < n; ++o) {
             int64_t base = start + o;
             kind[t] = 0; src[t] = (int32_t)base; pos[t] = (int32_t)t; win[t] = w;
@@ -126,10 +142,42 @@ int64_t fo_layout(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
                 t += 1;
             }
         }
+        start += W_sched[w];
     }
     win_off[M] = (int32_t)t;
     ring_off[M] = (int32_t)r;
+    if (base_off) base_off[M] = (int32_t)N;
     return t;
+}
+
+/* Windows of one length W: M = ceil(N/W) windows of W bases (App. A, I_w). */
+static int32_t* fixed_windows(int64_t N, int32_t W, int32_t M) {
+    if (W <= 0 || M < 0 || (int64_t)M != (N + W - 1) / W) return NULL;
+    int32_t* s = (int32_t*)malloc(sizeof(int32_t) * (size_t)(M > 0 ? M : 1));
+    for (int32_t w = 0; w < M; ++w) s[w] = W;
+    return s;
+}
+
+int64_t fo_layout_size(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
+                       int32_t close_tail, int32_t tail, int64_t* R_out) {
+    int32_t* Ws = fixed_windows(N, W, M);
+    if (!Ws) return -1;
+    int64_t T = fo_layout_size_sched(N, M, Ws, k_sched, close_tail, tail, R_out);
+    free(Ws);
+    return T;
+}
+
+int64_t fo_layout(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
+                  int32_t close_tail, int32_t tail, int32_t B, const uint8_t* nt,
+                  uint8_t* kind, int32_t* src, int32_t* pos, int32_t* win,
+                  uint8_t* tok, uint8_t* keep, int32_t* win_off, int32_t* ring_off,
+                  int32_t* sum_idx) {
+    int32_t* Ws = fixed_windows(N, W, M);
+    if (!Ws) return -1;
+    int64_t T = fo_layout_sched(N, M, Ws, k_sched, close_tail, tail, B, nt, kind, src, pos, win, tok, keep,
+                                win_off, ring_off, sum_idx, NULL);
+    free(Ws);
+    return T;
 }
 
 /* ------------------------------------------------------------------------- */
@@ -338,13 +386,12 @@ int32_t fo_window_retained_rows(int64_t n, int32_t k, int32_t close_partial, int
 /* base's own k-mer, or for a FOCUS token the k-mer it summarises. With k = 0 */
 /* (no summaries) the whole window is one segment, index 0. Returns T or -1.  */
 /* ------------------------------------------------------------------------- */
-int64_t fo_layout_kmer(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
-                       int32_t close_tail, int32_t* kmer) {
-    if (fo_layout_size(N, W, M, k_sched, close_tail, 0, NULL) < 0) return -1;
-    int64_t t = 0;
+int64_t fo_layout_kmer_sched(int64_t N, int32_t M, const int32_t* W_sched, const int32_t* k_sched,
+                             int32_t close_tail, int32_t* kmer) {
+    if (fo_layout_size_sched(N, M, W_sched, k_sched, close_tail, 0, NULL) < 0) return -1;
+    int64_t t = 0, start = 0;
     for (int32_t w = 0; w < M; ++w) {
-        int64_t start = (int64_t)w * W;
-        int64_t n = (N - start < W) ? (N - start) : W;
+        int64_t n = window_bases(N, start, W_sched[w]);
         int close = (w < M - 1) || close_tail;
         int32_t c = 0;
         for (int64_t o = 0; o < n; ++o) {
@@ -354,8 +401,18 @@ int64_t fo_layout_kmer(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
                 c += 1;
             }
         }
+        start += W_sched[w];
     }
     return t;
+}
+
+int64_t fo_layout_kmer(int64_t N, int32_t W, int32_t M, const int32_t* k_sched,
+                       int32_t close_tail, int32_t* kmer) {
+    int32_t* Ws = fixed_windows(N, W, M);
+    if (!Ws) return -1;
+    int64_t T = fo_layout_kmer_sched(N, M, Ws, k_sched, close_tail, kmer);
+    free(Ws);
+    return T;
 }
 
 /* ------------------------------------------------------------------------- */

@@ -57,6 +57,12 @@ def _load(path: str | None = None):
     lib.fo_prefill_sequential.argtypes = [i32, i32, P, P, P, P, P, f64, P, P, P, P, P, i64, P]
     lib.fo_decode.restype = None
     lib.fo_decode.argtypes = [i32, i64, P, P, i64, P, P, P, i64, P, P, P, P, f64, P, P]
+    lib.fo_layout_size_sched.restype = i64
+    lib.fo_layout_size_sched.argtypes = [i64, i32, P, P, i32, i32, P]
+    lib.fo_layout_sched.restype = i64
+    lib.fo_layout_sched.argtypes = [i64, i32, P, P, i32, i32, i32, P, P, P, P, P, P, P, P, P, P, P]
+    lib.fo_layout_kmer_sched.restype = i64
+    lib.fo_layout_kmer_sched.argtypes = [i64, i32, P, P, i32, P]
     lib.fo_layout_kmer.restype = i64
     lib.fo_layout_kmer.argtypes = [i64, i32, i32, P, i32, P]
     lib.fo_attn_rows_kmer_local.restype = None
@@ -118,25 +124,44 @@ def n_windows(N: int, W: int) -> int:
     return (N + W - 1) // W
 
 
-def layout_size(N: int, W: int, k_sched, close_tail: bool = True, tail: int = 0):
+def window_schedule(N: int, W) -> np.ndarray:
+    """Base lengths of the windows that cover N bases: M = ceil(N/W) copies of
+    an integer W, or the shortest prefix of a per-window sequence W (adaptive
+    windowing) whose sum reaches N."""
+    if np.ndim(W) == 0:
+        return np.full(n_windows(N, int(W)), int(W), np.int32)
+    Ws = np.asarray(W, dtype=np.int64).reshape(-1)
+    if N == 0:
+        return np.zeros(0, np.int32)
+    cover = np.cumsum(Ws)
+    if cover.size == 0 or cover[-1] < N:
+        raise ValueError("window schedule does not cover the sequence")
+    M = int(np.searchsorted(cover, N) + 1)
+    return np.ascontiguousarray(Ws[:M].astype(np.int32))
+
+
+def layout_size(N: int, W, k_sched, close_tail: bool = True, tail: int = 0):
     """(T, R, M): augmented length, retained rows (summaries + boundary tails),
-    windows (App. A)."""
+    windows (App. A). W: one window length, or a per-window schedule."""
     lib = _load()
-    M = n_windows(N, W)
+    Ws = window_schedule(N, W)
+    M = Ws.size
     k = _k_array(M, k_sched)
     R = np.zeros(1, np.int64)
-    T = lib.fo_layout_size(N, W, M, _ptr(k), int(close_tail), int(tail), _ptr(R))
+    T = lib.fo_layout_size_sched(N, M, _ptr(Ws), _ptr(k), int(close_tail), int(tail), _ptr(R))
     if T < 0:
         raise ValueError("bad layout arguments")
     return int(T), int(R[0]), M
 
 
-def layout(N: int, W: int, k_sched, nt=None, close_tail: bool = True, tail: int = 0) -> dict:
+def layout(N: int, W, k_sched, nt=None, close_tail: bool = True, tail: int = 0) -> dict:
     """Token layout: summary insertion after every k bases per window (Sec. 3.2
-    "Setup and tokens"; App. A). ``nt``: uint8 [B, N] nucleotide ids or None.
-    ``tail``: ordinary rows kept at the end of each window (boundary tail)."""
+    "Setup and tokens"; App. A). W: one window length or a per-window schedule.
+    ``nt``: uint8 [B, N] nucleotide ids or None. ``tail``: ordinary rows kept at
+    the end of each window (boundary tail)."""
     lib = _load()
     T, R, M = layout_size(N, W, k_sched, close_tail, tail)
+    Ws = window_schedule(N, W)
     k = _k_array(M, k_sched)
     if nt is not None:
         nt = np.ascontiguousarray(np.asarray(nt, dtype=np.uint8).reshape(-1, N))
@@ -147,14 +172,15 @@ def layout(N: int, W: int, k_sched, nt=None, close_tail: bool = True, tail: int 
     out = dict(
         kind=np.zeros(T, np.uint8), keep=np.zeros(T, np.uint8), src=np.zeros(T, np.int32), pos=np.zeros(T, np.int32),
         win=np.zeros(T, np.int32), win_off=np.zeros(M + 1, np.int32),
-        ring_off=np.zeros(M + 1, np.int32), sum_idx=np.zeros(max(R, 1), np.int32))
-    t = lib.fo_layout(N, W, M, _ptr(k), int(close_tail), int(tail), B, _ptr(nt), _ptr(out["kind"]),
-                      _ptr(out["src"]), _ptr(out["pos"]), _ptr(out["win"]), _ptr(tok), _ptr(out["keep"]),
-                      _ptr(out["win_off"]), _ptr(out["ring_off"]), _ptr(out["sum_idx"]))
+        ring_off=np.zeros(M + 1, np.int32), sum_idx=np.zeros(max(R, 1), np.int32),
+        base_off=np.zeros(M + 1, np.int32))
+    t = lib.fo_layout_sched(N, M, _ptr(Ws), _ptr(k), int(close_tail), int(tail), B, _ptr(nt), _ptr(out["kind"]),
+                            _ptr(out["src"]), _ptr(out["pos"]), _ptr(out["win"]), _ptr(tok), _ptr(out["keep"]),
+                            _ptr(out["win_off"]), _ptr(out["ring_off"]), _ptr(out["sum_idx"]), _ptr(out["base_off"]))
     assert t == T
     out["sum_idx"] = out["sum_idx"][:R]
     out["tok"] = tok
-    out.update(T=T, R=R, M=M)
+    out.update(T=T, R=R, M=M, W_sched=Ws)
     return out
 
 
@@ -182,15 +208,16 @@ def attn_rows(q, k, v, keep, win, scale: float, heads, rows):
     return o, lse
 
 
-def layout_kmer(N: int, W: int, k_sched, close_tail: bool = True) -> np.ndarray:
+def layout_kmer(N: int, W, k_sched, close_tail: bool = True) -> np.ndarray:
     """In-window k-mer index of every augmented row (Sec. 3.2 "Setup and
     tokens"): a base's own k-mer, the summarised k-mer for a FOCUS row; 0 for
     every row of a window with k = 0."""
     lib = _load()
     T, _, M = layout_size(N, W, k_sched, close_tail)
+    Ws = window_schedule(N, W)
     k = _k_array(M, k_sched)
     out = np.zeros(max(T, 1), np.int32)
-    t = lib.fo_layout_kmer(N, W, M, _ptr(k), int(close_tail), _ptr(out))
+    t = lib.fo_layout_kmer_sched(N, M, _ptr(Ws), _ptr(k), int(close_tail), _ptr(out))
     if t < 0:
         raise ValueError("bad layout arguments")
     return out[:T]

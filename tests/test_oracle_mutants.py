@@ -78,6 +78,10 @@ MUTANTS = [
      [lambda: pins.test_fp64_attention_variants_equal_the_pinned_bf16_ones()]),
     ("round_bf16_ties_away", "double r = nearbyint(ldexp(m, 8));", "double r = round(ldexp(m, 8));",
      [lambda: pins.test_round_bf16_is_nearest_even_and_matches_torch()]),
+    ("last_window_full", "static int64_t window_bases(int64_t N, int64_t start, int32_t W) { return (N - start < W) ? (N - start) : W; }",
+     "static int64_t window_bases(int64_t N, int64_t start, int32_t W) { (void)N; (void)start; return W; }",
+     [lambda: pins.test_layout_sizes_closed_form(5_000, 1_024, [100]),
+      lambda: pins.test_adaptive_windows_sizes_and_offsets_closed_form(1_037, [64, 1_000, 1_000], [8, 100, 3])]),
     ("decode_skips_self", "        kr[c] = k_new + (size_t)s * d;\n        vr[c] = v_new + (size_t)s * d;\n        c += 1;\n"
      "        softmax_row(d,", "        softmax_row(d,", [lambda: pins.test_decode_equals_prefill_row()]),
 ]

@@ -70,14 +70,28 @@ def test_layout_positions_closed_form(k):
     assert np.array_equal(L["win_off"], np.arange(n + 1) * (W + W // k))
 
 
+def _cuts(N, W):
+    """Window boundaries: multiples of an integer W, or the running sums of a
+    per-window schedule, up to N."""
+    if np.ndim(W) == 0:
+        return list(range(0, N, W)) + [N]
+    cuts = [0]
+    for x in W:
+        if cuts[-1] >= N:
+            break
+        cuts.append(min(N, cuts[-1] + int(x)))
+    return cuts
+
+
 def _string_layout(seq, W, ks, close_tail=True):
     """Independent construction: cut the base string into windows, each window
     into k-chunks, and write 'S' after every chunk (the last chunk of the final
     window only if close_tail)."""
     out = []
-    M = _ceil(len(seq), W)
+    cuts = _cuts(len(seq), W)
+    M = len(cuts) - 1
     for w in range(M):
-        chunk = seq[w * W:(w + 1) * W]
+        chunk = seq[cuts[w]:cuts[w + 1]]
         k = int(ks[w])
         if k == 0:
             out.append(chunk)
@@ -577,3 +591,69 @@ def test_rope_rounded_is_the_rounded_exact_rotation():
     yr = fo.rope(x, pos, 10_000.0, round_bf16=True)
     np.testing.assert_array_equal(yr, np.vectorize(fo.round_bf16)(y))
     assert (np.abs(yr - y) <= 2.0 ** -8 * np.abs(y)).all()     # half a step of 8 significant bits
+
+
+# ----------------------------------------------------------------------------- adaptive windows (W per window)
+
+SCHED_CASES = [
+    (2_500, [400, 1_000, 100, 1_000], [10, 25, 7, 200]),
+    (1_037, [64, 1_000, 1_000], [8, 100, 3]),          # the last window is partial; the third is never reached
+    (37, [1, 2, 3, 50], [1, 1, 2, 9]),
+    (300, [128, 64, 32, 16, 8, 52], [0, 5, 32, 1, 9, 13]),
+]
+
+
+@pytest.mark.parametrize("N,Ws,ks", SCHED_CASES)
+def test_adaptive_windows_sizes_and_offsets_closed_form(N, Ws, ks):
+    """Adaptive windowing (Sec. 5: W and k chosen per region): window w holds
+    the next W_w bases (the last one what is left); T = N + sum ceil(n_w/k_w),
+    R = sum B_w, and base_off is the running sum of the window lengths."""
+    cuts = _cuts(N, Ws)
+    M = len(cuts) - 1
+    k = np.asarray(ks[:M], np.int32)
+    T, R, M2 = fo.layout_size(N, Ws, k)
+    assert M2 == M
+    n_w = np.diff(cuts)
+    B_w = [(_ceil(int(n), int(kk)) if kk > 0 else 0) for n, kk in zip(n_w, k)]
+    assert (R, T) == (sum(B_w), N + sum(B_w))
+    L = fo.layout(N, Ws, k)
+    assert np.array_equal(L["base_off"], cuts)
+    assert np.array_equal(np.diff(L["win_off"]), n_w + np.array(B_w))
+
+
+@pytest.mark.parametrize("N,Ws,ks", SCHED_CASES)
+@pytest.mark.parametrize("close_tail", [True, False])
+def test_adaptive_windows_match_string_construction(N, Ws, ks, close_tail):
+    M = len(_cuts(N, Ws)) - 1
+    k = np.asarray(ks[:M], np.int32)
+    nt = inputs.nucleotides(1, N, seed=12).numpy()
+    L = fo.layout(N, Ws, k, nt=nt, close_tail=close_tail)
+    seq = "".join("ACGT"[x] for x in nt[0])
+    assert "".join("ACGTS"[x] for x in L["tok"][0]) == _string_layout(seq, Ws, k, close_tail)
+    km = fo.layout_kmer(N, Ws, k, close_tail=close_tail)
+    w = L["win"]
+    a = np.arange(L["T"]) - L["win_off"][w]
+    kw = k[w].astype(np.int64)
+    assert np.array_equal(km, np.where(kw > 0, a // np.maximum(kw + 1, 1), 0))
+
+
+@pytest.mark.parametrize("tail", [0, 3])
+def test_adaptive_windows_attention_matches_streaming_simulation(tail):
+    N, Ws, ks, H, d = 300, [128, 64, 32, 16, 8, 52], [0, 5, 32, 1, 9, 13], 2, 16
+    L = fo.layout(N, Ws, ks, tail=tail)
+    q, k, v = inputs.qkv((H, L["T"], d), seed=77)
+    T = L["T"]
+    heads, rows = np.repeat(np.arange(H), T), np.tile(np.arange(T), H)
+    o, lse = fo.attn_rows(q, k, v, L["keep"], L["win"], 0.25, heads, rows)
+    vis = _visible_sets_by_streaming(L, tail)
+    qd, kd, vd = _f64(q), _f64(k), _f64(v)
+    for r, (h, i) in enumerate(zip(heads, rows)):
+        j = np.array(vis[i])
+        sc = 0.25 * (kd[h, j] @ qd[h, i])
+        np.testing.assert_allclose(o[r], scipy.special.softmax(sc) @ vd[h, j], rtol=0, atol=1e-12)
+        assert abs(lse[r] - scipy.special.logsumexp(sc)) <= 1e-12 * max(1.0, abs(lse[r]))
+
+
+def test_window_schedule_must_cover_the_sequence():
+    with pytest.raises(ValueError):
+        fo.layout_size(100, [30, 30], [5])
