@@ -108,6 +108,8 @@ typedef struct focus_layout_out {
     int32_t* win_off;    /* [M+1] first augmented row of each window; win_off[M] = T */
     int32_t* ring_off;   /* [M+1] kept rows before each window; ring_off[M] = R */
     int32_t* sum_idx;    /* [R] augmented index of each kept row, in order (the compaction gather list) */
+    int32_t* base_off;   /* [M+1] first base of each window; base_off[M] = N. May be NULL for
+                            focus_layout; required by focus_layout_sched */
 } focus_layout_out;
 
 /* Device layout builder. d_k: DEVICE array [M] of cadences (same values as the
@@ -118,6 +120,19 @@ typedef struct focus_layout_out {
 focus_status focus_layout(int64_t n_nt, int32_t W, int32_t n_windows, const int32_t* d_k,
                           uint32_t flags, int32_t tail, int32_t B, const uint8_t* d_nt,
                           const focus_layout_out* out, cudaStream_t stream);
+
+/* Adaptive windowing (Sec. 5: W and k chosen per region): window w covers the
+ * next W_sched[w] bases, the last window whatever is left. The n_windows
+ * lengths must all be > 0 and cover exactly n_nt bases (the last window
+ * non-empty); otherwise FOCUS_ERR_INVALID_ARG (host) or FOCUS_ERR_INVALID_ARG in
+ * the device status word. h_W is a HOST array, d_W the DEVICE copy of the same
+ * values; everything else is as in focus_layout_size / focus_layout, which are
+ * the case W_sched[w] = W. */
+focus_status focus_layout_size_sched(int64_t n_nt, int32_t n_windows, const int32_t* h_W, const int32_t* h_k,
+                                     uint32_t flags, int32_t tail, int64_t* T, int64_t* R, int32_t* max_rows);
+focus_status focus_layout_sched(int64_t n_nt, int32_t n_windows, const int32_t* d_W, const int32_t* d_k,
+                                uint32_t flags, int32_t tail, int32_t B, const uint8_t* d_nt,
+                                const focus_layout_out* out, cudaStream_t stream);
 
 /* ------------------------------------------------------------------------ */
 /* Compressed KV cache (caller-owned). App. A.2 "Streaming with controlled   */
@@ -141,6 +156,7 @@ typedef struct focus_cache {
     int32_t* pos_base;        /* device [B] position id of the current window's first row, or NULL;
                                  window-mode compaction adds the retired window's T_w to it */
     float    rope_theta;      /* rotary-embedding base; 0 = none (see below) */
+    const int32_t* W_per_window; /* device [n_windows] window lengths (adaptive windowing), or NULL: W */
 } focus_cache;
 
 /* Rotary position embedding at the layout's position ids (RoFormer; the paper

@@ -43,7 +43,7 @@ focus_status check_cache(const focus_cache* c, bool need_window) {
     if (need_window) {
         if (!c->win_k || !c->win_v || !c->ring_len || !c->win_fill || !c->win_idx || !c->k_per_window)
             return FOCUS_ERR_INVALID_ARG;
-        if (c->W <= 0 || c->n_windows <= 0 || c->C_win <= 0) return FOCUS_ERR_INVALID_ARG;
+        if ((c->W <= 0 && !c->W_per_window) || c->n_windows <= 0 || c->C_win <= 0) return FOCUS_ERR_INVALID_ARG;
         if (!aligned16(c->win_k) || !aligned16(c->win_v)) return FOCUS_ERR_UNSUPPORTED;
     }
     return FOCUS_OK;
@@ -96,21 +96,31 @@ focus_status focus_get_device_status(int32_t* host_status, int32_t clear, cudaSt
     return FOCUS_OK;
 }
 
-focus_status focus_layout_size(int64_t n_nt, int32_t W, int32_t n_windows, const int32_t* h_k, uint32_t flags,
-                               int32_t tail, int64_t* T, int64_t* R, int32_t* max_rows) {
-    if (n_nt < 0 || W <= 0 || tail < 0 || (n_nt > 0 && !h_k)) return FOCUS_ERR_INVALID_ARG;
-    if ((int64_t)n_windows != focus::ceil_div64(n_nt, W)) return FOCUS_ERR_INVALID_ARG;
+}  // extern "C"
+
+namespace {
+
+// Host sizes of a layout; sched = false means windows of W bases (h_W unused).
+focus_status layout_size_impl(int64_t n_nt, int32_t W, bool sched, const int32_t* h_W, int32_t n_windows,
+                              const int32_t* h_k, uint32_t flags, int32_t tail, int64_t* T, int64_t* R,
+                              int32_t* max_rows) {
+    if (n_nt < 0 || tail < 0 || n_windows < 0 || (n_nt > 0 && !h_k)) return FOCUS_ERR_INVALID_ARG;
+    if (!sched && (W <= 0 || (int64_t)n_windows != focus::ceil_div64(n_nt, W))) return FOCUS_ERR_INVALID_ARG;
+    if (sched && n_windows > 0 && !h_W) return FOCUS_ERR_INVALID_ARG;
     const bool close_tail = (flags & FOCUS_LAYOUT_CLOSE_TAIL) != 0;
-    int64_t t = 0, r = 0, mx = 0;
+    int64_t t = 0, r = 0, mx = 0, start = 0;
     for (int32_t w = 0; w < n_windows; ++w) {
-        if (h_k[w] < 0) return FOCUS_ERR_INVALID_ARG;
-        int64_t n = n_nt - (int64_t)w * W;
-        if (n > W) n = W;
+        const int64_t len = sched ? h_W[w] : W;
+        if (h_k[w] < 0 || len <= 0 || start >= n_nt) return FOCUS_ERR_INVALID_ARG;
+        int64_t n = n_nt - start;
+        if (n > len) n = len;
         const int64_t rows = focus::window_rows(n, h_k[w], (w < n_windows - 1) || close_tail);
         t += rows;
         r += rows - n + (n - focus::tail_start(n, tail));
         if (rows > mx) mx = rows;
+        start += len;
     }
+    if (start < n_nt) return FOCUS_ERR_INVALID_ARG;   // the windows do not cover the sequence
     if (t > INT32_MAX) return FOCUS_ERR_UNSUPPORTED;   // offsets are int32
     if (T) *T = t;
     if (R) *R = r;
@@ -118,29 +128,58 @@ focus_status focus_layout_size(int64_t n_nt, int32_t W, int32_t n_windows, const
     return FOCUS_OK;
 }
 
-focus_status focus_layout(int64_t n_nt, int32_t W, int32_t n_windows, const int32_t* d_k, uint32_t flags,
-                          int32_t tail, int32_t B, const uint8_t* d_nt, const focus_layout_out* out,
-                          cudaStream_t stream) {
-    if (!out || n_nt < 0 || W <= 0 || B < 0 || tail < 0) return FOCUS_ERR_INVALID_ARG;
-    if ((int64_t)n_windows != focus::ceil_div64(n_nt, W)) return FOCUS_ERR_INVALID_ARG;
+focus_status layout_impl(int64_t n_nt, int32_t W, bool sched, const int32_t* d_W, int32_t n_windows,
+                         const int32_t* d_k, uint32_t flags, int32_t tail, int32_t B, const uint8_t* d_nt,
+                         const focus_layout_out* out, cudaStream_t stream) {
+    if (!out || n_nt < 0 || B < 0 || tail < 0 || n_windows < 0) return FOCUS_ERR_INVALID_ARG;
+    if (!sched && (W <= 0 || (int64_t)n_windows != focus::ceil_div64(n_nt, W))) return FOCUS_ERR_INVALID_ARG;
+    if (sched && n_windows > 0 && !d_W) return FOCUS_ERR_INVALID_ARG;
     if (n_nt == 0) {                                   // empty sequence: nothing to lay out
-        if (out->T != 0 || out->R != 0) return FOCUS_ERR_INVALID_ARG;
+        if (n_windows != 0 || out->T != 0 || out->R != 0) return FOCUS_ERR_INVALID_ARG;
         if (!out->win_off || !out->ring_off) return FOCUS_ERR_INVALID_ARG;
         cudaError_t e = cudaMemsetAsync(out->win_off, 0, sizeof(int32_t), stream);
         if (e == cudaSuccess) e = cudaMemsetAsync(out->ring_off, 0, sizeof(int32_t), stream);
+        if (e == cudaSuccess && out->base_off) e = cudaMemsetAsync(out->base_off, 0, sizeof(int32_t), stream);
         return from_cuda(e);
     }
-    if (!d_k) return FOCUS_ERR_INVALID_ARG;
+    if (!d_k || n_windows == 0) return FOCUS_ERR_INVALID_ARG;
     if (out->T < 0 || out->R < 0 || out->T > INT32_MAX) return FOCUS_ERR_INVALID_ARG;
     if (!out->win_off || !out->ring_off) return FOCUS_ERR_INVALID_ARG;
+    if (sched && !out->base_off) return FOCUS_ERR_INVALID_ARG;
     if (out->T > 0 && (!out->kind || !out->src || !out->pos || !out->win)) return FOCUS_ERR_INVALID_ARG;
     if (out->R > 0 && !out->sum_idx) return FOCUS_ERR_INVALID_ARG;
     if (out->tok && (!d_nt || B <= 0)) return FOCUS_ERR_INVALID_ARG;
     int32_t* st = nullptr;
     focus_status s = status_ptr(&st);
     if (s != FOCUS_OK) return s;
-    return from_cuda(focus::launch_layout(n_nt, W, n_windows, d_k, (flags & FOCUS_LAYOUT_CLOSE_TAIL) != 0, tail, B,
-                                          d_nt, *out, st, stream));
+    return from_cuda(focus::launch_layout(n_nt, W, sched ? d_W : nullptr, n_windows, d_k, (flags & FOCUS_LAYOUT_CLOSE_TAIL) != 0, tail,
+                                          B, d_nt, *out, st, stream));
+}
+
+}  // namespace
+
+extern "C" {
+
+focus_status focus_layout_size(int64_t n_nt, int32_t W, int32_t n_windows, const int32_t* h_k, uint32_t flags,
+                               int32_t tail, int64_t* T, int64_t* R, int32_t* max_rows) {
+    return layout_size_impl(n_nt, W, false, nullptr, n_windows, h_k, flags, tail, T, R, max_rows);
+}
+
+focus_status focus_layout_size_sched(int64_t n_nt, int32_t n_windows, const int32_t* h_W, const int32_t* h_k,
+                                     uint32_t flags, int32_t tail, int64_t* T, int64_t* R, int32_t* max_rows) {
+    return layout_size_impl(n_nt, 0, true, h_W, n_windows, h_k, flags, tail, T, R, max_rows);
+}
+
+focus_status focus_layout(int64_t n_nt, int32_t W, int32_t n_windows, const int32_t* d_k, uint32_t flags,
+                          int32_t tail, int32_t B, const uint8_t* d_nt, const focus_layout_out* out,
+                          cudaStream_t stream) {
+    return layout_impl(n_nt, W, false, nullptr, n_windows, d_k, flags, tail, B, d_nt, out, stream);
+}
+
+focus_status focus_layout_sched(int64_t n_nt, int32_t n_windows, const int32_t* d_W, const int32_t* d_k,
+                                uint32_t flags, int32_t tail, int32_t B, const uint8_t* d_nt,
+                                const focus_layout_out* out, cudaStream_t stream) {
+    return layout_impl(n_nt, 0, true, d_W, n_windows, d_k, flags, tail, B, d_nt, out, stream);
 }
 
 focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_args* a, cudaStream_t stream) {

@@ -86,9 +86,15 @@ __device__ __forceinline__ void rope_rotate8(uint4& lo, uint4& hi, const float2*
 }
 
 // Kernel launchers (one translation unit each).
-cudaError_t launch_layout(int64_t N, int32_t W, int32_t M, const int32_t* d_k, bool close_tail,
+// d_W: per-window lengths (device) or NULL for windows of W bases.
+cudaError_t launch_layout(int64_t N, int32_t W, const int32_t* d_W, int32_t M, const int32_t* d_k, bool close_tail,
                           int32_t tail, int32_t B, const uint8_t* d_nt, const focus_layout_out& out,
                           int32_t* status, cudaStream_t stream);
+
+// Length of window w of a cache: the schedule's entry, or the fixed W.
+__device__ __forceinline__ int32_t cache_window_len(const int32_t* W_per_window, int32_t W, int32_t w) {
+    return W_per_window ? W_per_window[w] : W;
+}
 
 cudaError_t launch_compact_bulk(const focus_cache& c, const focus_compact_args& a, int32_t* status,
                                 cudaStream_t stream);

@@ -96,9 +96,9 @@ __global__ void __launch_bounds__(256) compact_bulk_rope_kernel(
 __global__ void __launch_bounds__(256) compact_window_kernel(
         uint4* __restrict__ ring_k, uint4* __restrict__ ring_v, const uint4* __restrict__ win_k,
         const uint4* __restrict__ win_v, int32_t* __restrict__ ring_len, int32_t* __restrict__ win_fill,
-        int32_t* __restrict__ win_idx, const int32_t* __restrict__ ks, int32_t n_windows, int32_t W,
+        int32_t* __restrict__ win_idx, const int32_t* __restrict__ ks, int32_t n_windows, int32_t W_fixed,
         int32_t H, int32_t chunks_per_row, int32_t C_ring, int32_t C_win, int32_t tail,
-        int32_t* __restrict__ pos_base, int32_t* status) {
+        int32_t* __restrict__ pos_base, int32_t* status, const int32_t* __restrict__ W_per_window) {
     const int32_t b = blockIdx.x;
     const int32_t fill = win_fill[b], widx = win_idx[b], R = ring_len[b];
     if (widx < 0 || widx >= n_windows) {
@@ -106,6 +106,7 @@ __global__ void __launch_bounds__(256) compact_window_kernel(
         return;
     }
     const int32_t k = ks[widx];
+    const int32_t W = cache_window_len(W_per_window, W_fixed, widx);
     const int32_t Tw = (int32_t)window_rows(W, k, true);
     if (fill != Tw) return;                  // window not complete yet
     const int32_t Bw = Tw - W;
@@ -166,7 +167,7 @@ cudaError_t launch_compact_window(const focus_cache& c, int32_t* status, cudaStr
     compact_window_kernel<<<c.B, 256, 0, stream>>>(
         (uint4*)c.ring_k, (uint4*)c.ring_v, (const uint4*)c.win_k, (const uint4*)c.win_v, c.ring_len,
         c.win_fill, c.win_idx, c.k_per_window, c.n_windows, c.W, c.H, c.d / 8, c.C_ring, c.C_win, c.tail,
-        c.pos_base, status);
+        c.pos_base, status, c.W_per_window);
     return cudaGetLastError();
 }
 

@@ -53,9 +53,9 @@ __device__ __forceinline__ void bf16x8_to_f32(const uint4& u, float* f) {
 
 __device__ __forceinline__ bool decode_state_ok(int32_t R, int32_t fill, int32_t widx, const int32_t* ks,
                                                 int32_t n_windows, int32_t W, int32_t C_ring, int32_t C_win,
-                                                int32_t* Tw_out) {
+                                                int32_t* Tw_out, const int32_t* W_per_window) {
     if (widx < 0 || widx >= n_windows || R < 0 || R > C_ring) return false;
-    const int32_t Tw = (int32_t)window_rows(W, ks[widx], true);
+    const int32_t Tw = (int32_t)window_rows(cache_window_len(W_per_window, W, widx), ks[widx], true);
     *Tw_out = Tw;
     return fill >= 0 && fill < Tw && fill < C_win;
 }
@@ -72,7 +72,7 @@ __global__ void __launch_bounds__(kDecodeThreads + 32) decode_split_kernel(
         const int32_t* __restrict__ win_idx, const int32_t* __restrict__ ks, int32_t n_windows, int32_t W,
         int32_t H, int32_t C_ring, int32_t C_win, const uint4* __restrict__ q, const uint4* __restrict__ k_new,
         const uint4* __restrict__ v_new, float scale_log2, float2* __restrict__ ws_ml, float* __restrict__ ws_o,
-        int32_t n_splits, int32_t* status) {
+        int32_t n_splits, int32_t* status, const int32_t* __restrict__ W_per_window) {
     using namespace sm100;
     constexpr int CPR = D / 8;          // 16-byte chunks per row = lanes per key
     constexpr int GPW = 32 / CPR;       // key groups per warp
@@ -88,7 +88,7 @@ __global__ void __launch_bounds__(kDecodeThreads + 32) decode_split_kernel(
     int32_t Tw = 0;
     float2* ml = ws_ml + bh * n_splits + split;
     float* wo = ws_o + (bh * n_splits + split) * D;
-    const bool state_ok = decode_state_ok(R, fill, widx, ks, n_windows, W, C_ring, C_win, &Tw);
+    const bool state_ok = decode_state_ok(R, fill, widx, ks, n_windows, W, C_ring, C_win, &Tw, W_per_window);
     const int64_t total = (int64_t)R + fill + 1;
     const int64_t s0 = (int64_t)split * kDecodeChunk;
     const int64_t s1 = min(total, s0 + kDecodeChunk);
@@ -268,7 +268,7 @@ __global__ void __launch_bounds__(D) decode_combine_kernel(
         const float2* __restrict__ ws_ml, const float* __restrict__ ws_o, int32_t n_splits, int32_t H,
         __nv_bfloat16* __restrict__ o, float* __restrict__ lse, int32_t* __restrict__ win_fill,
         const int32_t* __restrict__ ring_len, const int32_t* __restrict__ win_idx, const int32_t* __restrict__ ks,
-        int32_t n_windows, int32_t W, int32_t C_ring, int32_t C_win) {
+        int32_t n_windows, int32_t W, int32_t C_ring, int32_t C_win, const int32_t* __restrict__ W_per_window) {
     const int b = blockIdx.y, h = blockIdx.x, c = threadIdx.x;
     const int64_t bh = (int64_t)b * H + h;
     const float2* ml = ws_ml + bh * n_splits;
@@ -289,7 +289,8 @@ __global__ void __launch_bounds__(D) decode_combine_kernel(
     if (c == 0 && lse) lse[bh] = L > 0.f ? (M + log2f(L)) * 0.69314718055994531f : -INFINITY;
     if (h == 0 && c == 0) {
         int32_t Tw = 0;
-        if (decode_state_ok(ring_len[b], win_fill[b], win_idx[b], ks, n_windows, W, C_ring, C_win, &Tw))
+        if (decode_state_ok(ring_len[b], win_fill[b], win_idx[b], ks, n_windows, W, C_ring, C_win, &Tw,
+                            W_per_window))
             win_fill[b] += 1;
     }
 }
@@ -348,12 +349,13 @@ cudaError_t launch_decode_d(const focus_cache& c, const void* q, const void* k_n
     decode_split_kernel<D><<<grid, kDecodeThreads + 32, smem, stream>>>(
         (const uint4*)c.ring_k, (const uint4*)c.ring_v, (uint4*)c.win_k, (uint4*)c.win_v, c.ring_len,
         c.win_fill, c.win_idx, c.k_per_window, c.n_windows, c.W, c.H, c.C_ring, c.C_win, (const uint4*)q,
-        (const uint4*)k_new, (const uint4*)v_new, scale * 1.4426950408889634f, ws_ml, ws_o, ns, status);
+        (const uint4*)k_new, (const uint4*)v_new, scale * 1.4426950408889634f, ws_ml, ws_o, ns, status,
+        c.W_per_window);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     decode_combine_kernel<D><<<dim3(c.H, c.B), D, 0, stream>>>(
         ws_ml, ws_o, ns, c.H, (__nv_bfloat16*)o, lse, c.win_fill, c.ring_len, c.win_idx, c.k_per_window,
-        c.n_windows, c.W, c.C_ring, c.C_win);
+        c.n_windows, c.W, c.C_ring, c.C_win, c.W_per_window);
     return cudaGetLastError();
 }
 

@@ -37,14 +37,14 @@ _i32, _i64, _u32, _f32 = ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32, ctypes
 
 class LayoutOut(ctypes.Structure):
     _fields_ = [("T", _i64), ("R", _i64), ("kind", _P), ("src", _P), ("pos", _P), ("win", _P), ("tok", _P),
-                ("keep", _P), ("win_off", _P), ("ring_off", _P), ("sum_idx", _P)]
+                ("keep", _P), ("win_off", _P), ("ring_off", _P), ("sum_idx", _P), ("base_off", _P)]
 
 
 class CacheDesc(ctypes.Structure):
     _fields_ = [("ring_k", _P), ("ring_v", _P), ("win_k", _P), ("win_v", _P), ("ring_len", _P),
                 ("win_fill", _P), ("win_idx", _P), ("k_per_window", _P), ("n_windows", _i32), ("W", _i32),
                 ("B", _i32), ("H", _i32), ("d", _i32), ("C_ring", _i32), ("C_win", _i32), ("tail", _i32),
-                ("pos_base", _P), ("rope_theta", _f32)]
+                ("pos_base", _P), ("rope_theta", _f32), ("W_per_window", _P)]
 
 
 class PrefillArgs(ctypes.Structure):
@@ -83,6 +83,10 @@ def load() -> ctypes.CDLL:
     lib.focus_layout_size.argtypes = [_i64, _i32, _i32, _P, _u32, _i32, _P, _P, _P]
     lib.focus_layout.restype = ctypes.c_int
     lib.focus_layout.argtypes = [_i64, _i32, _i32, _P, _u32, _i32, _i32, _P, ctypes.POINTER(LayoutOut), _P]
+    lib.focus_layout_size_sched.restype = ctypes.c_int
+    lib.focus_layout_size_sched.argtypes = [_i64, _i32, _P, _P, _u32, _i32, _P, _P, _P]
+    lib.focus_layout_sched.restype = ctypes.c_int
+    lib.focus_layout_sched.argtypes = [_i64, _i32, _P, _P, _u32, _i32, _i32, _P, ctypes.POINTER(LayoutOut), _P]
     lib.focus_attn_prefill.restype = ctypes.c_int
     lib.focus_attn_prefill.argtypes = [ctypes.POINTER(CacheDesc), ctypes.POINTER(PrefillArgs), _P]
     lib.focus_decode_workspace_size.restype = ctypes.c_size_t
@@ -125,20 +129,44 @@ def _cuda(t: torch.Tensor, name: str, dtype=None):
 
 # ----------------------------------------------------------------------------- layout
 
-def layout_size(N: int, W: int, k_sched, close_tail: bool = True, tail: int = 0):
-    """(T, R, M, max_rows) of the augmented layout (host arithmetic in the library)."""
+def window_lengths(N: int, W):
+    """None for windows of one integer length W; for a per-window sequence W
+    (adaptive windowing) the int32 lengths of the windows that cover N bases: the
+    shortest prefix whose sum reaches N."""
+    if np.ndim(W) == 0:
+        return None
+    Ws = np.asarray(W, dtype=np.int64).reshape(-1)
+    if N == 0:
+        return np.zeros(0, np.int32)
+    cover = np.cumsum(Ws)
+    if cover.size == 0 or cover[-1] < N:
+        raise ValueError("window lengths do not cover the sequence")
+    return np.ascontiguousarray(Ws[:int(np.searchsorted(cover, N)) + 1].astype(np.int32))
+
+
+def layout_size(N: int, W, k_sched, close_tail: bool = True, tail: int = 0):
+    """(T, R, M, max_rows) of the augmented layout (host arithmetic in the
+    library). W: one window length, or a per-window sequence."""
     lib = load()
-    M = -(-N // W)
+    Ws = window_lengths(N, W)
+    M = -(-N // int(W)) if Ws is None else int(Ws.size)
     k = np.ascontiguousarray(np.broadcast_to(np.asarray(k_sched, dtype=np.int32), (M,)))
     T, R, mx = _i64(), _i64(), _i32()
-    _check("focus_layout_size", lib.focus_layout_size(N, W, M, k.ctypes.data, LAYOUT_CLOSE_TAIL if close_tail else 0,
-                                                      int(tail), ctypes.byref(T), ctypes.byref(R), ctypes.byref(mx)))
+    flags = LAYOUT_CLOSE_TAIL if close_tail else 0
+    if Ws is None:
+        _check("focus_layout_size", lib.focus_layout_size(N, int(W), M, k.ctypes.data, flags, int(tail),
+                                                          ctypes.byref(T), ctypes.byref(R), ctypes.byref(mx)))
+    else:
+        _check("focus_layout_size_sched", lib.focus_layout_size_sched(N, M, Ws.ctypes.data, k.ctypes.data, flags,
+                                                                      int(tail), ctypes.byref(T), ctypes.byref(R),
+                                                                      ctypes.byref(mx)))
     return T.value, R.value, M, mx.value
 
 
-def layout_alloc(N: int, W: int, k_sched, B: int = 0, close_tail: bool = True, device="cuda", tail: int = 0) -> dict:
+def layout_alloc(N: int, W, k_sched, B: int = 0, close_tail: bool = True, device="cuda", tail: int = 0) -> dict:
     """Allocate the device outputs of focus_layout (sizes from focus_layout_size)."""
     T, R, M, mx = layout_size(N, W, k_sched, close_tail, tail)
+    Ws = window_lengths(N, W)
     k_host = np.ascontiguousarray(np.broadcast_to(np.asarray(k_sched, dtype=np.int32), (M,)))
     out = dict(
         kind=torch.empty(T, dtype=torch.uint8, device=device), keep=torch.empty(T, dtype=torch.uint8, device=device),
@@ -147,10 +175,12 @@ def layout_alloc(N: int, W: int, k_sched, B: int = 0, close_tail: bool = True, d
         tok=torch.empty((B, T), dtype=torch.uint8, device=device) if B else None,
         win_off=torch.empty(M + 1, dtype=torch.int32, device=device),
         ring_off=torch.empty(M + 1, dtype=torch.int32, device=device),
+        base_off=torch.empty(M + 1, dtype=torch.int32, device=device),
+        W_dev=None if Ws is None else torch.from_numpy(Ws.copy()).to(device),
         sum_idx_buf=torch.empty(max(R, 1), dtype=torch.int32, device=device),
         k=torch.from_numpy(k_host.copy()).to(device))
     out["sum_idx"] = out["sum_idx_buf"][:R]
-    out.update(T=T, R=R, M=M, max_rows=mx, k_host=k_host, N=N, W=W, B=B, close_tail=close_tail, tail=tail)
+    out.update(T=T, R=R, M=M, max_rows=mx, k_host=k_host, N=N, W=W, W_host=Ws, B=B, close_tail=close_tail, tail=tail)
     return out
 
 
@@ -163,11 +193,16 @@ def layout_run(L: dict, nt: torch.Tensor | None = None, stream=None) -> None:
             raise ValueError("nt shape does not match the allocated layout")
     desc = LayoutOut(L["T"], L["R"], _ptr(L["kind"]), _ptr(L["src"]), _ptr(L["pos"]), _ptr(L["win"]),
                      _ptr(L["tok"]) if nt is not None else None, _ptr(L["keep"]), _ptr(L["win_off"]),
-                     _ptr(L["ring_off"]), _ptr(L["sum_idx_buf"]))
-    _check("focus_layout", lib.focus_layout(L["N"], L["W"], L["M"], _ptr(L["k"]),
-                                            LAYOUT_CLOSE_TAIL if L["close_tail"] else 0, int(L["tail"]),
-                                            0 if nt is None else L["B"], _ptr(nt), ctypes.byref(desc),
-                                            _stream(stream)))
+                     _ptr(L["ring_off"]), _ptr(L["sum_idx_buf"]), _ptr(L["base_off"]))
+    flags = LAYOUT_CLOSE_TAIL if L["close_tail"] else 0
+    B = 0 if nt is None else L["B"]
+    if L["W_dev"] is None:
+        _check("focus_layout", lib.focus_layout(L["N"], int(L["W"]), L["M"], _ptr(L["k"]), flags, int(L["tail"]), B,
+                                                _ptr(nt), ctypes.byref(desc), _stream(stream)))
+    else:
+        _check("focus_layout_sched", lib.focus_layout_sched(L["N"], L["M"], _ptr(L["W_dev"]), _ptr(L["k"]), flags,
+                                                            int(L["tail"]), B, _ptr(nt), ctypes.byref(desc),
+                                                            _stream(stream)))
 
 
 def layout(N: int, W: int, k_sched, nt: torch.Tensor | None = None, close_tail: bool = True,
@@ -178,6 +213,7 @@ def layout(N: int, W: int, k_sched, nt: torch.Tensor | None = None, close_tail: 
     layout_run(L, nt, stream)
     L["win_off_host"] = L["win_off"].cpu().numpy()
     L["ring_off_host"] = L["ring_off"].cpu().numpy()
+    L["base_off_host"] = L["base_off"].cpu().numpy()
     return L
 
 
@@ -188,10 +224,12 @@ class Cache:
     current window buffer) and its C descriptor."""
 
     def __init__(self, B: int, H: int, d: int, C_ring: int, C_win: int = 0, W: int = 0, k_sched=None,
-                 device="cuda", tail: int = 0, rope_theta: float = 0.0):
+                 device="cuda", tail: int = 0, rope_theta: float = 0.0, W_sched=None):
         """``rope_theta`` > 0 turns on the rotary embedding of queries and keys at
         their position ids; ``pos_base`` [B] (zeros here) holds the position id of
-        each sequence's current decode window's first row."""
+        each sequence's current decode window's first row. ``W_sched`` (one length
+        per window, adaptive windowing) replaces the fixed W for decode and
+        window-mode compaction."""
         self.B, self.H, self.d, self.C_ring, self.C_win, self.W, self.tail = B, H, d, C_ring, C_win, W, tail
         self.rope_theta = float(rope_theta)
         bf = dict(dtype=torch.bfloat16, device=device)
@@ -203,12 +241,14 @@ class Cache:
         self.win_fill = torch.zeros(B, dtype=torch.int32, device=device)
         self.win_idx = torch.zeros(B, dtype=torch.int32, device=device)
         self.pos_base = torch.zeros(B, dtype=torch.int32, device=device)
+        self.W_sched = (None if W_sched is None else
+                        torch.from_numpy(np.asarray(W_sched, dtype=np.int32).reshape(-1).copy()).to(device))
         ks = np.zeros(1, np.int32) if k_sched is None else np.asarray(k_sched, dtype=np.int32).reshape(-1)
         self.k_sched = torch.from_numpy(ks.copy()).to(device)
         self.desc = CacheDesc(_ptr(self.ring_k), _ptr(self.ring_v), _ptr(self.win_k), _ptr(self.win_v),
                               _ptr(self.ring_len), _ptr(self.win_fill), _ptr(self.win_idx), _ptr(self.k_sched),
                               int(self.k_sched.numel()), W, B, H, d, C_ring, C_win, tail, _ptr(self.pos_base),
-                              self.rope_theta)
+                              self.rope_theta, _ptr(self.W_sched))
 
     def workspace_bytes(self) -> int:
         return int(load().focus_decode_workspace_size(ctypes.byref(self.desc)))

@@ -32,8 +32,8 @@ def test_library_exports_every_declared_function():
 
 def test_struct_sizes_match_c_layout():
     # 2 x int64 + 8 pointers; 8 pointers + 7 int32 (+pad); see focus.h
-    assert ctypes.sizeof(focus.LayoutOut) == 16 + 9 * 8
-    assert ctypes.sizeof(focus.CacheDesc) == 8 * 8 + 8 * 4 + 8 + 8
+    assert ctypes.sizeof(focus.LayoutOut) == 16 + 10 * 8
+    assert ctypes.sizeof(focus.CacheDesc) == 8 * 8 + 8 * 4 + 8 + 8 + 8
     assert ctypes.sizeof(focus.PrefillArgs) == 5 * 8 + 8 + 2 * 8 + 6 * 4
     assert ctypes.sizeof(focus.CompactArgs) == 2 * 8 + 2 * 8 + 2 * 8 + 3 * 4 + 4
 
@@ -152,3 +152,26 @@ def test_rope_argument_checks_need_no_gpu():
                                  1 << 20, None) == 1
     assert lib.focus_attn_decode_noalloc(ctypes.byref(c), 4096, 4096, 4096, ctypes.c_float(0.125), 4096, None,
                                          None) == 1
+
+
+@pytest.mark.parametrize("N,Ws,ks,tail", [(2_500, [400, 1_000, 100, 1_000], [10, 25, 7, 200], 0),
+                                          (1_037, [64, 1_000, 1_000], [8, 100, 3], 5),
+                                          (300, [128, 64, 32, 16, 8, 52], [0, 5, 32, 1, 9, 13], 2)])
+def test_layout_size_sched_matches_oracle(N, Ws, ks, tail):
+    T, R, M, mx = focus.layout_size(N, Ws, ks[:len(fo.window_schedule(N, Ws))], tail=tail)
+    L = fo.layout(N, Ws, ks[:M], tail=tail)
+    assert (T, R, M) == (L["T"], L["R"], L["M"])
+    assert mx == int(np.diff(L["win_off"]).max())
+
+
+def test_layout_size_sched_rejects_bad_schedules():
+    lib = focus.load()
+    T = ctypes.c_int64()
+    k = np.array([5, 5, 5], np.int32)
+    for Ws, M in (([30, 30], 2), ([30, 0, 80], 3), ([60, 50, 10], 3), ([40, 50], 2)):
+        w = np.array(Ws, np.int32)
+        assert lib.focus_layout_size_sched(100, M, w.ctypes.data, k.ctypes.data, 1, 0, ctypes.byref(T), None,
+                                           None) == 1, Ws
+    w = np.array([30, 30, 40], np.int32)
+    assert lib.focus_layout_size_sched(100, 3, w.ctypes.data, k.ctypes.data, 1, 0, ctypes.byref(T), None, None) == 0
+    assert lib.focus_layout_size_sched(100, 3, None, k.ctypes.data, 1, 0, ctypes.byref(T), None, None) == 1
