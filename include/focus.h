@@ -157,7 +157,15 @@ typedef struct focus_cache {
                                  window-mode compaction adds the retired window's T_w to it */
     float    rope_theta;      /* rotary-embedding base; 0 = none (see below) */
     const int32_t* W_per_window; /* device [n_windows] window lengths (adaptive windowing), or NULL: W */
+    int32_t  q_per_kv;        /* query heads per K/V head (grouped-query heads); 0 or 1 = one each */
 } focus_cache;
+
+/* Grouped-query heads (q_per_kv = g > 1; not in the paper): H counts K/V heads.
+ * Keys, values, the ring and the window buffer have H heads; queries, outputs
+ * and LSE have H * g heads, and query head hq uses K/V head hq / g. The cache
+ * and its K/V traffic shrink by g. Decode serves up to four query heads of a
+ * group per K/V pass. The legacy prefill kernel refuses g > 1
+ * (FOCUS_ERR_UNSUPPORTED); g must be <= 64 (FOCUS_ERR_INVALID_ARG). */
 
 /* Rotary position embedding at the layout's position ids (RoFormer; the paper
  * gives each FOCUS token a position of its own, Sec. 3.2, and names no base).

@@ -35,6 +35,7 @@ focus_status from_cuda(cudaError_t e) { return e == cudaSuccess ? FOCUS_OK : FOC
 focus_status check_cache(const focus_cache* c, bool need_window) {
     if (!c) return FOCUS_ERR_INVALID_ARG;
     if (!isfinite(c->rope_theta) || c->rope_theta < 0.f) return FOCUS_ERR_INVALID_ARG;
+    if (c->q_per_kv < 0 || c->q_per_kv > 64) return FOCUS_ERR_INVALID_ARG;
     if (c->B <= 0 || c->H <= 0 || c->C_ring < 0 || c->C_win < 0 || c->tail < 0) return FOCUS_ERR_INVALID_ARG;
     if (c->d != 64 && c->d != 128) return FOCUS_ERR_UNSUPPORTED;
     if ((int64_t)c->B > 65535 || (int64_t)c->H > 65535) return FOCUS_ERR_UNSUPPORTED;
@@ -191,7 +192,8 @@ focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_ar
     if (!isfinite(a->scale) || !(a->scale > 0.f)) return FOCUS_ERR_INVALID_ARG;
     if (!aligned16(a->q) || !aligned16(a->k) || !aligned16(a->v) || !aligned16(a->o)) return FOCUS_ERR_UNSUPPORTED;
     if (a->flags & ~(uint32_t)(FOCUS_PREFILL_LEGACY_MMA | FOCUS_PREFILL_KMER_LOCAL)) return FOCUS_ERR_INVALID_ARG;
-    if ((a->flags & FOCUS_PREFILL_LEGACY_MMA) && cache->rope_theta > 0.f) return FOCUS_ERR_UNSUPPORTED;
+    if ((a->flags & FOCUS_PREFILL_LEGACY_MMA) && (cache->rope_theta > 0.f || cache->q_per_kv > 1))
+        return FOCUS_ERR_UNSUPPORTED;
     if (a->flags & FOCUS_PREFILL_KMER_LOCAL) {
         if (a->flags & FOCUS_PREFILL_LEGACY_MMA) return FOCUS_ERR_UNSUPPORTED;
         if (cache->tail != 0) return FOCUS_ERR_UNSUPPORTED;

@@ -35,10 +35,10 @@ constexpr int kStageRows = 8192 / (2 * D);   // 8 KB of K and 8 KB of V per stag
 constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s bound on any wait
 template <int D>
 constexpr int decode_groups() { return (kDecodeThreads / 32) * (32 / (D / 8)); }   // lane groups per CTA
-template <int D>
-constexpr int decode_smem_bytes() {   // K/V stages + full/empty barriers + the group merge buffers
-    return 2 * kStages * kStageRows<D> * D * 2 + 2 * kStages * 8 + 2 * decode_groups<D>() * 4 +
-           decode_groups<D>() * D * 4;
+template <int D, int QG>
+constexpr int decode_smem_bytes() {   // K/V stages + full/empty barriers + the group merge buffers (per query)
+    return 2 * kStages * kStageRows<D> * D * 2 + 2 * kStages * 8 + QG * (2 * decode_groups<D>() * 4 +
+           decode_groups<D>() * D * 4);
 }
 
 __device__ __forceinline__ void bf16x8_to_f32(const uint4& u, float* f) {
@@ -65,14 +65,18 @@ __device__ __forceinline__ bool decode_state_ok(int32_t R, int32_t fill, int32_t
 // into a ring of shared-memory stages; consumers read each row with d/8 lanes
 // (16 B each, conflict-free), reduce the dot product with shuffles and keep a
 // per-lane-group online softmax (log2 domain) in registers.
-template <int D>
+//
+// Grouped-query heads (q_per_kv = g > 1): one CTA serves QG of the g query
+// heads that share its K/V head, so each K/V row it streams is used QG times
+// (blockIdx.y = kv head * (g / QG) + which QG-slice of the group).
+template <int D, int QG>
 __global__ void __launch_bounds__(kDecodeThreads + 32) decode_split_kernel(
         const uint4* __restrict__ ring_k, const uint4* __restrict__ ring_v, uint4* __restrict__ win_k,
         uint4* __restrict__ win_v, const int32_t* __restrict__ ring_len, const int32_t* __restrict__ win_fill,
         const int32_t* __restrict__ win_idx, const int32_t* __restrict__ ks, int32_t n_windows, int32_t W,
         int32_t H, int32_t C_ring, int32_t C_win, const uint4* __restrict__ q, const uint4* __restrict__ k_new,
         const uint4* __restrict__ v_new, float scale_log2, float2* __restrict__ ws_ml, float* __restrict__ ws_o,
-        int32_t n_splits, int32_t* status, const int32_t* __restrict__ W_per_window) {
+        int32_t n_splits, int32_t* status, const int32_t* __restrict__ W_per_window, int32_t q_per_kv) {
     using namespace sm100;
     constexpr int CPR = D / 8;          // 16-byte chunks per row = lanes per key
     constexpr int GPW = 32 / CPR;       // key groups per warp
@@ -80,25 +84,28 @@ __global__ void __launch_bounds__(kDecodeThreads + 32) decode_split_kernel(
     static_assert(NG == decode_groups<D>(), "group count");
     constexpr int CH = kStageRows<D>;   // key rows per stage
     constexpr int ROWB = D * 2;         // bytes per row
-    const int b = blockIdx.z, h = blockIdx.y, split = blockIdx.x;
-    const int64_t bh = (int64_t)b * H + h;
+    const int slices = q_per_kv / QG;
+    const int b = blockIdx.z, h = blockIdx.y / slices, slice = blockIdx.y % slices, split = blockIdx.x;
+    const int64_t bh = (int64_t)b * H + h;                         // K/V head
+    const int64_t bhq0 = bh * q_per_kv + (int64_t)slice * QG;      // first of this CTA's query heads
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 
     const int32_t R = ring_len[b], fill = win_fill[b], widx = win_idx[b];
     int32_t Tw = 0;
-    float2* ml = ws_ml + bh * n_splits + split;
-    float* wo = ws_o + (bh * n_splits + split) * D;
     const bool state_ok = decode_state_ok(R, fill, widx, ks, n_windows, W, C_ring, C_win, &Tw, W_per_window);
     const int64_t total = (int64_t)R + fill + 1;
     const int64_t s0 = (int64_t)split * kDecodeChunk;
     const int64_t s1 = min(total, s0 + kDecodeChunk);
     if (!state_ok || s0 >= s1) {
-        if (!state_ok && split == 0 && h == 0 && tid == 0) report(status, FOCUS_ERR_CAPACITY);
-        for (int c = tid; c < D; c += blockDim.x) wo[c] = 0.f;
-        if (tid == 0) *ml = make_float2(-INFINITY, 0.f);
+        if (!state_ok && split == 0 && blockIdx.y == 0 && tid == 0) report(status, FOCUS_ERR_CAPACITY);
+        for (int j = 0; j < QG; ++j) {
+            float* wo = ws_o + ((bhq0 + j) * n_splits + split) * D;
+            for (int c = tid; c < D; c += blockDim.x) wo[c] = 0.f;
+            if (tid == 0) ws_ml[(bhq0 + j) * n_splits + split] = make_float2(-INFINITY, 0.f);
+        }
         return;
     }
-    if (split == 0 && tid < CPR) {      // append the new row to the window buffer
+    if (split == 0 && slice == 0 && tid < CPR) {      // append the new row to the window buffer
         win_k[(bh * C_win + fill) * CPR + tid] = k_new[bh * CPR + tid];
         win_v[(bh * C_win + fill) * CPR + tid] = v_new[bh * CPR + tid];
     }
@@ -108,9 +115,9 @@ __global__ void __launch_bounds__(kDecodeThreads + 32) decode_split_kernel(
     uint8_t* sV = smem + kStages * CH * ROWB;             // [kStages][CH][D] bf16
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + 2 * kStages * CH * ROWB);
     uint64_t* empty = full + kStages;
-    float* sm_m = reinterpret_cast<float*>(empty + kStages);
-    float* sm_l = sm_m + NG;
-    float* sm_acc = sm_l + NG;                            // [NG][D]
+    float* sm_m = reinterpret_cast<float*>(empty + kStages);   // [QG][NG]
+    float* sm_l = sm_m + QG * NG;                               // [QG][NG]
+    float* sm_acc = sm_l + QG * NG;                             // [QG][NG][D]
     __shared__ int32_t abort_flag;
     const int n_chunks = (int)((s1 - s0 + CH - 1) / CH);
 
@@ -174,13 +181,21 @@ __global__ void __launch_bounds__(kDecodeThreads + 32) decode_split_kernel(
     // ---------------------------------------------------- consumers
     const int sub = lane % CPR;
     const int grp = warp * GPW + lane / CPR;
-    float qf[8];
-    bf16x8_to_f32(q[bh * CPR + sub], qf);
+    float qf[QG][8];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) qf[e] *= scale_log2;
-    float m = -INFINITY, l = 0.f, acc[8];
+    for (int j = 0; j < QG; ++j) {
+        bf16x8_to_f32(q[(bhq0 + j) * CPR + sub], qf[j]);
 #pragma unroll
-    for (int e = 0; e < 8; ++e) acc[e] = 0.f;
+        for (int e = 0; e < 8; ++e) qf[j][e] *= scale_log2;
+    }
+    float m[QG], l[QG], acc[QG][8];
+#pragma unroll
+    for (int j = 0; j < QG; ++j) {
+        m[j] = -INFINITY;
+        l[j] = 0.f;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[j][e] = 0.f;
+    }
 
     for (int c = 0; c < n_chunks; ++c) {
         const int st = c % kStages;
@@ -192,7 +207,7 @@ __global__ void __launch_bounds__(kDecodeThreads + 32) decode_split_kernel(
         const uint8_t* kb = sK + st * CH * ROWB + sub * 16;
         const uint8_t* vb = sV + st * CH * ROWB + sub * 16;
         constexpr int U = CH / NG;
-        float s[U];
+        float s[QG][U];
         uint4 vr[U];
 #pragma unroll
         for (int u = 0; u < U; ++u) {
@@ -202,63 +217,79 @@ __global__ void __launch_bounds__(kDecodeThreads + 32) decode_split_kernel(
             vr[u] = ok ? *reinterpret_cast<const uint4*>(vb + r * ROWB) : make_uint4(0, 0, 0, 0);
             float kf[8];
             bf16x8_to_f32(kr, kf);
-            float d0 = 0.f;
 #pragma unroll
-            for (int e = 0; e < 8; ++e) d0 = fmaf(qf[e], kf[e], d0);
-            s[u] = d0;
+            for (int j = 0; j < QG; ++j) {
+                float d0 = 0.f;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) d0 = fmaf(qf[j][e], kf[e], d0);
+                s[j][u] = d0;
+            }
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_addr(&empty[st]));     // this warp is done with the stage
 #pragma unroll
         for (int off = CPR / 2; off >= 1; off >>= 1) {
 #pragma unroll
-            for (int u = 0; u < U; ++u) s[u] += __shfl_xor_sync(0xffffffffu, s[u], off);
+            for (int j = 0; j < QG; ++j)
+#pragma unroll
+                for (int u = 0; u < U; ++u) s[j][u] += __shfl_xor_sync(0xffffffffu, s[j][u], off);
         }
-        float mb = -INFINITY;
+#pragma unroll
+        for (int j = 0; j < QG; ++j) {
+            float mb = -INFINITY;
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                if (grp + u * NG >= nrow) s[j][u] = -INFINITY;
+                mb = fmaxf(mb, s[j][u]);
+            }
+            const float mn = fmaxf(m[j], mb);
+            if (mn == -INFINITY) continue;
+            if (mn > m[j]) {
+                const float corr = ex2_approx(m[j] - mn);
+                l[j] *= corr;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc[j][e] *= corr;
+                m[j] = mn;
+            }
+        }
 #pragma unroll
         for (int u = 0; u < U; ++u) {
-            if (grp + u * NG >= nrow) s[u] = -INFINITY;
-            mb = fmaxf(mb, s[u]);
-        }
-        const float mn = fmaxf(m, mb);
-        if (mn == -INFINITY) continue;
-        if (mn > m) {
-            const float corr = ex2_approx(m - mn);
-            l *= corr;
-#pragma unroll
-            for (int e = 0; e < 8; ++e) acc[e] *= corr;
-            m = mn;
-        }
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const float p = ex2_approx(s[u] - m);
-            l += p;
             float vf[8];
             bf16x8_to_f32(vr[u], vf);
 #pragma unroll
-            for (int e = 0; e < 8; ++e) acc[e] = fmaf(p, vf[e], acc[e]);
+            for (int j = 0; j < QG; ++j) {
+                if (m[j] == -INFINITY) continue;
+                const float p = ex2_approx(s[j][u] - m[j]);
+                l[j] += p;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc[j][e] = fmaf(p, vf[e], acc[j][e]);
+            }
         }
     }
 
-    if (sub == 0) { sm_m[grp] = m; sm_l[grp] = l; }
 #pragma unroll
-    for (int e = 0; e < 8; ++e) sm_acc[grp * D + sub * 8 + e] = acc[e];
+    for (int j = 0; j < QG; ++j) {
+        if (sub == 0) { sm_m[j * NG + grp] = m[j]; sm_l[j * NG + grp] = l[j]; }
+#pragma unroll
+        for (int e = 0; e < 8; ++e) sm_acc[(j * NG + grp) * D + sub * 8 + e] = acc[j][e];
+    }
     asm volatile("bar.sync 1, %0;" ::"n"(kDecodeThreads));       // consumers only
-    if (tid < D) {
+    for (int col = tid; col < QG * D; col += kDecodeThreads) {
+        const int j = col / D, cc = col % D;
         float M = -INFINITY;
 #pragma unroll
-        for (int g = 0; g < NG; ++g) M = fmaxf(M, sm_m[g]);
+        for (int g = 0; g < NG; ++g) M = fmaxf(M, sm_m[j * NG + g]);
         float L = 0.f, A = 0.f;
         if (M != -INFINITY) {
 #pragma unroll
             for (int g = 0; g < NG; ++g) {
-                const float f = ex2_approx(sm_m[g] - M);
-                L = fmaf(sm_l[g], f, L);
-                A = fmaf(sm_acc[g * D + tid], f, A);
+                const float f = ex2_approx(sm_m[j * NG + g] - M);
+                L = fmaf(sm_l[j * NG + g], f, L);
+                A = fmaf(sm_acc[(j * NG + g) * D + cc], f, A);
             }
         }
-        wo[tid] = A;
-        if (tid == 0) *ml = make_float2(M, L);
+        ws_o[((bhq0 + j) * n_splits + split) * D + cc] = A;
+        if (cc == 0) ws_ml[(bhq0 + j) * n_splits + split] = make_float2(M, L);
     }
     __syncthreads();
 }
@@ -269,7 +300,7 @@ __global__ void __launch_bounds__(D) decode_combine_kernel(
         __nv_bfloat16* __restrict__ o, float* __restrict__ lse, int32_t* __restrict__ win_fill,
         const int32_t* __restrict__ ring_len, const int32_t* __restrict__ win_idx, const int32_t* __restrict__ ks,
         int32_t n_windows, int32_t W, int32_t C_ring, int32_t C_win, const int32_t* __restrict__ W_per_window) {
-    const int b = blockIdx.y, h = blockIdx.x, c = threadIdx.x;
+    const int b = blockIdx.y, h = blockIdx.x, c = threadIdx.x;   // h: query head, H: query heads
     const int64_t bh = (int64_t)b * H + h;
     const float2* ml = ws_ml + bh * n_splits;
     const float* wo = ws_o + bh * n_splits * D;
@@ -303,58 +334,76 @@ template <int D>
 __global__ void __launch_bounds__(D / 2) decode_rope_kernel(
         const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ k_new,
         __nv_bfloat16* __restrict__ q_rot, __nv_bfloat16* __restrict__ k_rot, const int32_t* __restrict__ pos_base,
-        const int32_t* __restrict__ win_fill, int32_t H, const __grid_constant__ RopeTable rope) {
-    const int b = blockIdx.y, h = blockIdx.x, i = threadIdx.x;
-    const int64_t row = ((int64_t)b * H + h) * D;
+        const int32_t* __restrict__ win_fill, int32_t H, int32_t q_per_kv, const __grid_constant__ RopeTable rope) {
+    const int b = blockIdx.y, hq = blockIdx.x, i = threadIdx.x;    // grid: query heads x sequences
+    const int64_t qrow = ((int64_t)b * H * q_per_kv + hq) * D;
     const int64_t p = (int64_t)pos_base[b] + win_fill[b];
     const float2 cs = rope_cs((double)p * rope.theta[i]);
-    const float ql = __bfloat162float(q[row + i]), qh = __bfloat162float(q[row + i + D / 2]);
-    const float kl = __bfloat162float(k_new[row + i]), kh = __bfloat162float(k_new[row + i + D / 2]);
-    q_rot[row + i] = __float2bfloat16_rn(ql * cs.x - qh * cs.y);
-    q_rot[row + i + D / 2] = __float2bfloat16_rn(qh * cs.x + ql * cs.y);
-    k_rot[row + i] = __float2bfloat16_rn(kl * cs.x - kh * cs.y);
-    k_rot[row + i + D / 2] = __float2bfloat16_rn(kh * cs.x + kl * cs.y);
+    const float ql = __bfloat162float(q[qrow + i]), qh = __bfloat162float(q[qrow + i + D / 2]);
+    q_rot[qrow + i] = __float2bfloat16_rn(ql * cs.x - qh * cs.y);
+    q_rot[qrow + i + D / 2] = __float2bfloat16_rn(qh * cs.x + ql * cs.y);
+    if (hq % q_per_kv == 0) {                                      // the K/V head's new key, once
+        const int64_t krow = ((int64_t)b * H + hq / q_per_kv) * D;
+        const float kl = __bfloat162float(k_new[krow + i]), kh = __bfloat162float(k_new[krow + i + D / 2]);
+        k_rot[krow + i] = __float2bfloat16_rn(kl * cs.x - kh * cs.y);
+        k_rot[krow + i + D / 2] = __float2bfloat16_rn(kh * cs.x + kl * cs.y);
+    }
 }
 
 // Workspace: split partials (m, l) and o, then, with the rotary embedding, the
 // rotated q and k_new (16-byte aligned).
+int32_t q_heads_per_kv(const focus_cache& c) { return c.q_per_kv > 1 ? c.q_per_kv : 1; }
+
 size_t partials_bytes(const focus_cache& c) {
-    return (size_t)((int64_t)c.B * c.H * decode_num_splits(c) * (2 + c.d)) * sizeof(float);
+    return (size_t)((int64_t)c.B * c.H * q_heads_per_kv(c) * decode_num_splits(c) * (2 + c.d)) * sizeof(float);
 }
 size_t rope_rows_offset(const focus_cache& c) { return (partials_bytes(c) + 255) & ~(size_t)255; }
+
+template <int D, int QG>
+cudaError_t launch_decode_split(const focus_cache& c, int32_t ns, const void* q, const void* k_new,
+                                const void* v_new, float scale, float2* ws_ml, float* ws_o, int32_t* status,
+                                cudaStream_t stream) {
+    const int32_t g = q_heads_per_kv(c);
+    constexpr int smem = decode_smem_bytes<D, QG>();
+    cudaError_t e0 = cudaFuncSetAttribute(decode_split_kernel<D, QG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          smem);
+    if (e0 != cudaSuccess) return e0;
+    decode_split_kernel<D, QG><<<dim3(ns, c.H * (g / QG), c.B), kDecodeThreads + 32, smem, stream>>>(
+        (const uint4*)c.ring_k, (const uint4*)c.ring_v, (uint4*)c.win_k, (uint4*)c.win_v, c.ring_len,
+        c.win_fill, c.win_idx, c.k_per_window, c.n_windows, c.W, c.H, c.C_ring, c.C_win, (const uint4*)q,
+        (const uint4*)k_new, (const uint4*)v_new, scale * 1.4426950408889634f, ws_ml, ws_o, ns, status,
+        c.W_per_window, g);
+    return cudaGetLastError();
+}
 
 template <int D>
 cudaError_t launch_decode_d(const focus_cache& c, const void* q, const void* k_new, const void* v_new,
                             float scale, void* o, float* lse, void* workspace, int32_t* status,
                             cudaStream_t stream) {
     const int32_t ns = decode_num_splits(c);
+    const int32_t g = q_heads_per_kv(c);
+    const int64_t Hq = (int64_t)c.H * g;
     float2* ws_ml = reinterpret_cast<float2*>(workspace);
-    float* ws_o = reinterpret_cast<float*>(ws_ml + (int64_t)c.B * c.H * ns);
-    dim3 grid(ns, c.H, c.B);
+    float* ws_o = reinterpret_cast<float*>(ws_ml + (int64_t)c.B * Hq * ns);
     if (c.rope_theta > 0.f) {
         __nv_bfloat16* q_rot = reinterpret_cast<__nv_bfloat16*>((char*)workspace + rope_rows_offset(c));
-        __nv_bfloat16* k_rot = q_rot + (int64_t)c.B * c.H * D;
+        __nv_bfloat16* k_rot = q_rot + (int64_t)c.B * Hq * D;
         RopeTable rope;
         rope_table_fill(&rope, D, c.rope_theta);
-        decode_rope_kernel<D><<<dim3(c.H, c.B), D / 2, 0, stream>>>(
-            (const __nv_bfloat16*)q, (const __nv_bfloat16*)k_new, q_rot, k_rot, c.pos_base, c.win_fill, c.H, rope);
+        decode_rope_kernel<D><<<dim3((unsigned)Hq, c.B), D / 2, 0, stream>>>(
+            (const __nv_bfloat16*)q, (const __nv_bfloat16*)k_new, q_rot, k_rot, c.pos_base, c.win_fill, c.H, g,
+            rope);
         cudaError_t er = cudaGetLastError();
         if (er != cudaSuccess) return er;
         q = q_rot;
         k_new = k_rot;
     }
-    constexpr int smem = decode_smem_bytes<D>();
-    cudaError_t e0 = cudaFuncSetAttribute(decode_split_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e0 != cudaSuccess) return e0;
-    decode_split_kernel<D><<<grid, kDecodeThreads + 32, smem, stream>>>(
-        (const uint4*)c.ring_k, (const uint4*)c.ring_v, (uint4*)c.win_k, (uint4*)c.win_v, c.ring_len,
-        c.win_fill, c.win_idx, c.k_per_window, c.n_windows, c.W, c.H, c.C_ring, c.C_win, (const uint4*)q,
-        (const uint4*)k_new, (const uint4*)v_new, scale * 1.4426950408889634f, ws_ml, ws_o, ns, status,
-        c.W_per_window);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = (g % 4 == 0)   ? launch_decode_split<D, 4>(c, ns, q, k_new, v_new, scale, ws_ml, ws_o, status, stream)
+                    : (g % 2 == 0) ? launch_decode_split<D, 2>(c, ns, q, k_new, v_new, scale, ws_ml, ws_o, status, stream)
+                                   : launch_decode_split<D, 1>(c, ns, q, k_new, v_new, scale, ws_ml, ws_o, status, stream);
     if (e != cudaSuccess) return e;
-    decode_combine_kernel<D><<<dim3(c.H, c.B), D, 0, stream>>>(
-        ws_ml, ws_o, ns, c.H, (__nv_bfloat16*)o, lse, c.win_fill, c.ring_len, c.win_idx, c.k_per_window,
+    decode_combine_kernel<D><<<dim3((unsigned)Hq, c.B), D, 0, stream>>>(
+        ws_ml, ws_o, ns, (int32_t)Hq, (__nv_bfloat16*)o, lse, c.win_fill, c.ring_len, c.win_idx, c.k_per_window,
         c.n_windows, c.W, c.C_ring, c.C_win, c.W_per_window);
     return cudaGetLastError();
 }
@@ -366,7 +415,8 @@ int32_t decode_num_splits(const focus_cache& c) {
 }
 
 size_t decode_workspace_bytes(const focus_cache& c) {
-    if (c.rope_theta > 0.f) return rope_rows_offset(c) + 2 * (size_t)c.B * c.H * c.d * sizeof(__nv_bfloat16);
+    if (c.rope_theta > 0.f)
+        return rope_rows_offset(c) + (size_t)c.B * c.H * (q_heads_per_kv(c) + 1) * c.d * sizeof(__nv_bfloat16);
     return partials_bytes(c);
 }
 

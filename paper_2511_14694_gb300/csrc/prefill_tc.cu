@@ -161,14 +161,24 @@ __device__ __forceinline__ void fail(Bars* bars, int32_t* status) {
 }
 __device__ __forceinline__ bool aborted(Bars* bars) { return *(volatile int32_t*)&bars->abort != 0; }
 
-template <int D, bool LOCAL, bool ROPE>
+// Q/O/LSE row of this CTA's query head, read afresh from the block index where
+// it is used (keeping it in a register across the softmax loop costs spills).
+__device__ __forceinline__ int32_t query_head_row(int32_t H, int32_t q_per_kv) {
+    uint32_t x, y, z;
+    asm volatile("mov.u32 %0, %%ctaid.x;" : "=r"(x));
+    asm volatile("mov.u32 %0, %%ctaid.y;" : "=r"(y));
+    asm volatile("mov.u32 %0, %%ctaid.z;" : "=r"(z));
+    return ((int32_t)z * H + (int32_t)y) * q_per_kv + (int32_t)(x % (uint32_t)q_per_kv);
+}
+
+template <int D, bool LOCAL, bool ROPE, bool GQA>
 __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
         const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
         const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_rk,
         const __grid_constant__ CUtensorMap tm_rv, __nv_bfloat16* __restrict__ o, float* __restrict__ lse,
         int64_t T_span, const int32_t* __restrict__ win_off, const int32_t* __restrict__ ring_off, int32_t w_begin,
         int32_t w_end, int32_t ctas_pw, int32_t H, int32_t C_ring, float scale_log2, int32_t* status,
-        const int32_t* __restrict__ k_per_window, const __grid_constant__ RopeArg<ROPE> rope) {
+        const int32_t* __restrict__ k_per_window, const __grid_constant__ RopeArg<ROPE> rope, int32_t q_per_kv) {
     static_assert(!ROPE || kSlots == 4, "K tiles must use the even slots");
     using C = Cfg<D>;
     extern __shared__ unsigned char smem_raw[];
@@ -176,11 +186,15 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
     Bars* bars = reinterpret_cast<Bars*>(smem + C::kBarOff);
 
     // ---- work item (longest first: later windows have longer rings) --------
-    const int32_t wi = blockIdx.x / ctas_pw;
-    const int32_t cta = ctas_pw - 1 - (int32_t)(blockIdx.x % ctas_pw);
+    // GQA: the q_per_kv query heads that share a K/V head are adjacent in launch
+    // order (a separate instantiation: the division costs registers elsewhere)
+    const uint32_t item = GQA ? blockIdx.x / (uint32_t)q_per_kv : blockIdx.x;
+    const int32_t member = GQA ? (int32_t)(blockIdx.x % (uint32_t)q_per_kv) : 0;
+    const int32_t wi = item / ctas_pw;
+    const int32_t cta = ctas_pw - 1 - (int32_t)(item % ctas_pw);
     const int32_t w = w_end - 1 - wi;
-    const int h = blockIdx.y, b = blockIdx.z;
-    const int32_t bh = b * H + h;
+    const int h = blockIdx.y, b = blockIdx.z;     // h: K/V head
+    const int32_t bh = b * H + h;                   // K/V and ring rows
     const int32_t w0 = win_off[w_begin];
     const int32_t Tw = win_off[w + 1] - win_off[w];
     const int32_t a0 = cta * 2 * BM;
@@ -261,7 +275,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
             for (int t = 0; t < 2; ++t)
                 for (int x = 0; x < C::kBoxes; ++x)
                     tma_load_3d(smem_addr(smem + C::kQOff + t * C::kTileBytes + x * kBoxBytes), &tm_q, x * 64,
-                                row_base + a0 + t * BM, bh, bq);
+                                row_base + a0 + t * BM, GQA ? bh * q_per_kv + member : bh, bq);
             int issued = 0;
             for (int j = 0; j < n_kv_max && !aborted(bars); ++j) {
                 const bool ring = j < n_ring;
@@ -571,11 +585,12 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
                     *reinterpret_cast<uint4*>(stage + r * (2 * D) + ((chunk ^ (r & 7)) << 4)) = v;
                 }
             }
+            const int32_t bhq = GQA ? query_head_row(H, q_per_kv) : bh;   // Q, O and LSE rows
             if (lse && aq < Tw)
-                lse[(int64_t)bh * T_span + row_base + aq] = (m_run + __log2f(l_run)) * 0.69314718055994531f;
+                lse[(int64_t)bhq * T_span + row_base + aq] = (m_run + __log2f(l_run)) * 0.69314718055994531f;
             __syncwarp();
             // the warp stores the 32 rows it staged: 32/CH rows per instruction, coalesced
-            __nv_bfloat16* ob = o + ((int64_t)bh * T_span + row_base + a0 + t * BM) * D;
+            __nv_bfloat16* ob = o + ((int64_t)bhq * T_span + row_base + a0 + t * BM) * D;
             constexpr int RPI = 32 / CH;                  // rows per store instruction
             for (int i = 0; i < 32; i += RPI) {
                 const int rr = quarter * 32 + i + lane / CH;
@@ -630,12 +645,13 @@ cudaError_t make_map(CUtensorMap* m, const void* ptr, int d, int64_t rows, int64
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-template <int D, bool LOCAL, bool ROPE>
+template <int D, bool LOCAL, bool ROPE, bool GQA>
 cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t* status, cudaStream_t stream) {
     const int64_t BH = (int64_t)c.B * c.H;
+    const int32_t g = c.q_per_kv > 1 ? c.q_per_kv : 1;
     CUtensorMap tq, tk, tv, trk, trv;
     cudaError_t e;
-    if ((e = make_map(&tq, a.q, D, a.T_span, BH)) != cudaSuccess) return e;
+    if ((e = make_map(&tq, a.q, D, a.T_span, BH * g)) != cudaSuccess) return e;
     if ((e = make_map(&tk, a.k, D, a.T_span, BH)) != cudaSuccess) return e;
     if ((e = make_map(&tv, a.v, D, a.T_span, BH)) != cudaSuccess) return e;
     if (c.C_ring > 0) {
@@ -646,30 +662,42 @@ cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t*
         trv = tv;
     }
     const int smem = Cfg<D>::kSmem;
-    e = cudaFuncSetAttribute(prefill_tc_kernel<D, LOCAL, ROPE>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    e = cudaFuncSetAttribute(prefill_tc_kernel<D, LOCAL, ROPE, GQA>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             smem);
     if (e != cudaSuccess) return e;
     const int ctas_pw = (a.max_rows + 2 * BM - 1) / (2 * BM);
-    dim3 grid((unsigned)((a.w_end - a.w_begin) * ctas_pw), c.H, c.B);
+    dim3 grid((unsigned)((a.w_end - a.w_begin) * ctas_pw * g), c.H, c.B);
     RopeArg<ROPE> rope;
     if constexpr (ROPE) rope_table_fill(&rope.t, D, c.rope_theta);
     else rope.unused = 0;
-    prefill_tc_kernel<D, LOCAL, ROPE><<<grid, kThreads, smem, stream>>>(
+    prefill_tc_kernel<D, LOCAL, ROPE, GQA><<<grid, kThreads, smem, stream>>>(
         tq, tk, tv, trk, trv, (__nv_bfloat16*)a.o, a.lse, a.T_span, a.d_win_off, a.d_ring_off,
-        a.w_begin, a.w_end, ctas_pw, c.H, c.C_ring, a.scale * 1.4426950408889634f, status, c.k_per_window, rope);
+        a.w_begin, a.w_end, ctas_pw, c.H, c.C_ring, a.scale * 1.4426950408889634f, status, c.k_per_window, rope, g);
     return cudaGetLastError();
 }
 
 }  // namespace
 
+template <bool GQA>
+cudaError_t dispatch(const focus_cache& c, const focus_prefill_args& a, int32_t* status, cudaStream_t stream,
+                     bool local, bool rope) {
+    if (c.d == 128) {
+        if (rope) return local ? launch_d<128, true, true, GQA>(c, a, status, stream)
+                               : launch_d<128, false, true, GQA>(c, a, status, stream);
+        return local ? launch_d<128, true, false, GQA>(c, a, status, stream)
+                     : launch_d<128, false, false, GQA>(c, a, status, stream);
+    }
+    if (rope) return local ? launch_d<64, true, true, GQA>(c, a, status, stream)
+                           : launch_d<64, false, true, GQA>(c, a, status, stream);
+    return local ? launch_d<64, true, false, GQA>(c, a, status, stream)
+                 : launch_d<64, false, false, GQA>(c, a, status, stream);
+}
+
 cudaError_t launch_prefill_tc(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
                               cudaStream_t stream) {
     const bool local = (a.flags & FOCUS_PREFILL_KMER_LOCAL) != 0, rope = c.rope_theta > 0.f;
-    if (c.d == 128) {
-        if (rope) return local ? launch_d<128, true, true>(c, a, status, stream) : launch_d<128, false, true>(c, a, status, stream);
-        return local ? launch_d<128, true, false>(c, a, status, stream) : launch_d<128, false, false>(c, a, status, stream);
-    }
-    if (rope) return local ? launch_d<64, true, true>(c, a, status, stream) : launch_d<64, false, true>(c, a, status, stream);
-    return local ? launch_d<64, true, false>(c, a, status, stream) : launch_d<64, false, false>(c, a, status, stream);
+    if (c.q_per_kv > 1) return dispatch<true>(c, a, status, stream, local, rope);
+    return dispatch<false>(c, a, status, stream, local, rope);
 }
 
 }  // namespace focus

@@ -44,7 +44,7 @@ class CacheDesc(ctypes.Structure):
     _fields_ = [("ring_k", _P), ("ring_v", _P), ("win_k", _P), ("win_v", _P), ("ring_len", _P),
                 ("win_fill", _P), ("win_idx", _P), ("k_per_window", _P), ("n_windows", _i32), ("W", _i32),
                 ("B", _i32), ("H", _i32), ("d", _i32), ("C_ring", _i32), ("C_win", _i32), ("tail", _i32),
-                ("pos_base", _P), ("rope_theta", _f32), ("W_per_window", _P)]
+                ("pos_base", _P), ("rope_theta", _f32), ("W_per_window", _P), ("q_per_kv", _i32)]
 
 
 class PrefillArgs(ctypes.Structure):
@@ -224,12 +224,14 @@ class Cache:
     current window buffer) and its C descriptor."""
 
     def __init__(self, B: int, H: int, d: int, C_ring: int, C_win: int = 0, W: int = 0, k_sched=None,
-                 device="cuda", tail: int = 0, rope_theta: float = 0.0, W_sched=None):
+                 device="cuda", tail: int = 0, rope_theta: float = 0.0, W_sched=None, q_per_kv: int = 1):
         """``rope_theta`` > 0 turns on the rotary embedding of queries and keys at
         their position ids; ``pos_base`` [B] (zeros here) holds the position id of
         each sequence's current decode window's first row. ``W_sched`` (one length
         per window, adaptive windowing) replaces the fixed W for decode and
-        window-mode compaction."""
+        window-mode compaction. ``q_per_kv`` query heads share each of the H K/V
+        heads (grouped-query heads): queries and outputs have H * q_per_kv heads."""
+        self.q_per_kv = int(q_per_kv)
         self.B, self.H, self.d, self.C_ring, self.C_win, self.W, self.tail = B, H, d, C_ring, C_win, W, tail
         self.rope_theta = float(rope_theta)
         bf = dict(dtype=torch.bfloat16, device=device)
@@ -248,7 +250,7 @@ class Cache:
         self.desc = CacheDesc(_ptr(self.ring_k), _ptr(self.ring_v), _ptr(self.win_k), _ptr(self.win_v),
                               _ptr(self.ring_len), _ptr(self.win_fill), _ptr(self.win_idx), _ptr(self.k_sched),
                               int(self.k_sched.numel()), W, B, H, d, C_ring, C_win, tail, _ptr(self.pos_base),
-                              self.rope_theta, _ptr(self.W_sched))
+                              self.rope_theta, _ptr(self.W_sched), self.q_per_kv)
 
     def workspace_bytes(self) -> int:
         return int(load().focus_decode_workspace_size(ctypes.byref(self.desc)))
@@ -260,6 +262,13 @@ class Cache:
 
 # ----------------------------------------------------------------------------- verbs
 
+def _check_heads(cache: Cache, q, k, v):
+    g = max(cache.q_per_kv, 1)
+    if q.shape[1] != cache.H * g or k.shape[1] != cache.H or v.shape[1] != cache.H:
+        raise ValueError(f"heads: q {q.shape[1]} (want {cache.H * g}), k {k.shape[1]}, v {v.shape[1]} "
+                         f"(want {cache.H})")
+
+
 def attn_prefill(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | None = None, scale=None,
                  o=None, lse=None, flags: int = 0, stream=None):
     """focus_attn_prefill over windows [w_begin, w_end). q/k/v: bf16 [B, H, T_span, d]
@@ -268,6 +277,7 @@ def attn_prefill(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | 
     w_end = L["M"] if w_end is None else w_end
     for name, t in (("q", q), ("k", k), ("v", v)):
         _cuda(t, name, torch.bfloat16)
+    _check_heads(cache, q, k, v)
     B, H, T_span, d = q.shape
     if o is None:
         o = torch.empty_like(q)
@@ -305,6 +315,7 @@ def attn_decode(cache: Cache, q, k_new, v_new, scale=None, o=None, lse=None, wor
     lib = load()
     for name, t in (("q", q), ("k_new", k_new), ("v_new", v_new)):
         _cuda(t, name, torch.bfloat16)
+    _check_heads(cache, q, k_new, v_new)
     if o is None:
         o = torch.empty_like(q)
     if lse is None:

@@ -33,7 +33,7 @@ def test_library_exports_every_declared_function():
 def test_struct_sizes_match_c_layout():
     # 2 x int64 + 8 pointers; 8 pointers + 7 int32 (+pad); see focus.h
     assert ctypes.sizeof(focus.LayoutOut) == 16 + 10 * 8
-    assert ctypes.sizeof(focus.CacheDesc) == 8 * 8 + 8 * 4 + 8 + 8 + 8
+    assert ctypes.sizeof(focus.CacheDesc) == 8 * 8 + 8 * 4 + 8 + 8 + 8 + 8
     assert ctypes.sizeof(focus.PrefillArgs) == 5 * 8 + 8 + 2 * 8 + 6 * 4
     assert ctypes.sizeof(focus.CompactArgs) == 2 * 8 + 2 * 8 + 2 * 8 + 3 * 4 + 4
 
