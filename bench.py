@@ -273,8 +273,10 @@ def run_prefill_leg(args, cfg, world, rank, local):
     dev = torch.device("cuda", local)
     nt = inputs.nucleotides(B, N, seed=inputs.DEFAULT_SEED, device=dev)
     L = focus.layout_alloc(N, W, k_s, B=B, device=dev)
-    q, k, v = inputs.qkv((B, H, L["T"], d), std=cfg["std"], seed=inputs.DEFAULT_SEED + rank, device=dev)
-    cache = focus.Cache(B, H, d, C_ring=max(L["R"], 1), device=dev, k_sched=k_s, rope_theta=args.rope)
+    g = args.q_per_kv
+    q, k, v = inputs.qkv((B, H, L["T"], d), std=cfg["std"], seed=inputs.DEFAULT_SEED + rank, device=dev, q_per_kv=g)
+    cache = focus.Cache(B, H // g, d, C_ring=max(L["R"], 1), device=dev, k_sched=k_s, rope_theta=args.rope,
+                        q_per_kv=g)
     o = torch.empty_like(q)
     lse = torch.empty((B, H, L["T"]), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
@@ -298,7 +300,7 @@ def run_prefill_leg(args, cfg, world, rank, local):
              else visible_pairs(win_off, ring_off))
     flops_per_step = 4.0 * d * H * B * pairs
     # algorithmic bytes of one prefill launch: read Q, K, V and write O once (bf16), write LSE (fp32)
-    bytes_per_step = float(B * H * L["T"] * (8 * d + 4))
+    bytes_per_step = float(B * L["T"] * (H * (4 * d + 4) + (H // g) * 4 * d))
 
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -394,8 +396,15 @@ def run_stream_leg(args, cfg, world, rank, local):
     Tw = int(np.diff(off).max())
     if not (np.diff(off) == Tw).all():
         raise ValueError("the streaming leg expects windows of equal augmented size")
-    pq, pk, pv = inputs.qkv((P, B, H, Tw, d), std=cfg["std"], seed=inputs.DEFAULT_SEED + rank, device=dev)
-    cache = focus.Cache(B, H, d, C_ring=max(L["R"], 1), device=dev, k_sched=k_s, rope_theta=args.rope)
+    g = args.q_per_kv
+    if g == 1:
+        pq, pk, pv = inputs.qkv((P, B, H, Tw, d), std=cfg["std"], seed=inputs.DEFAULT_SEED + rank, device=dev)
+    else:                            # grouped-query heads: K/V with H / g heads
+        pq = inputs.normal_bf16((P, B, H, Tw, d), cfg["std"], seed=3 * (inputs.DEFAULT_SEED + rank) + 1, device=dev)
+        pk, pv = (inputs.normal_bf16((P, B, H // g, Tw, d), cfg["std"], seed=3 * (inputs.DEFAULT_SEED + rank) + i,
+                                     device=dev) for i in (2, 3))
+    cache = focus.Cache(B, H // g, d, C_ring=max(L["R"], 1), device=dev, k_sched=k_s, rope_theta=args.rope,
+                        q_per_kv=g)
     local_mask = bool(args.prefill_flags & focus.PREFILL_KMER_LOCAL)
     outs = [torch.empty((B, H, Tw, d), dtype=torch.bfloat16, device=dev) for _ in range(2)]
     lses = [torch.empty((B, H, Tw), dtype=torch.float32, device=dev) for _ in range(2)]
@@ -438,7 +447,7 @@ def run_stream_leg(args, cfg, world, rank, local):
     return dict(step_ms=step_ms, attn_ms=attn_ms / args.steps, flops_per_step=4.0 * d * H * B * pairs, pairs=pairs,
                 T=L["T"], R=L["R"], clocks=clk.summary(), launches=2 * M * args.steps, e2e=None, host_sample=None,
                 per_launch_ms=attn_ms / args.steps / M, local_mask=local_mask,
-                bytes_per_step=float(B * H * L["T"] * (8 * d + 4)))
+                bytes_per_step=float(B * L["T"] * (H * (4 * d + 4) + (H // g) * 4 * d)))
 
 
 def run_decode_leg(args, cfg, world, rank, local):
@@ -446,17 +455,21 @@ def run_decode_leg(args, cfg, world, rank, local):
     from paper_2511_14694_gb300 import focus, inputs
 
     B, H, d, W, R = cfg["B"], cfg["H"], cfg["d"], cfg["W"], cfg["R"]
+    g = args.q_per_kv
+    Hk = H // g                      # K/V heads; H query heads
     kk = cfg["k"][0]
     Tw = W + -(-W // kk)
     S = cfg["steps"]
     dev = torch.device("cuda", local)
     k_sched = np.full(R // (W // kk) + S // W + 16, kk, np.int32)
-    cache = focus.Cache(B, H, d, C_ring=R + 256, C_win=1_024, W=W, k_sched=k_sched, device=dev, rope_theta=args.rope)
+    cache = focus.Cache(B, Hk, d, C_ring=R + 256, C_win=1_024, W=W, k_sched=k_sched, device=dev, rope_theta=args.rope,
+                        q_per_kv=g)
     for i, t in enumerate((cache.ring_k, cache.ring_v, cache.win_k, cache.win_v)):
         t.copy_(inputs.normal_bf16(t.shape, cfg["std"], seed=50 + i + 10 * rank, device=dev))
     fill0 = inputs.start_fill(B, Tw - 1, seed=inputs.DEFAULT_SEED)
     widx0 = R // (W // kk)
-    qs, ks_, vs = inputs.qkv((S, B, H, d), std=cfg["std"], seed=300 + rank, device=dev)
+    qs = inputs.normal_bf16((S, B, H, d), cfg["std"], seed=300 + rank, device=dev)
+    ks_, vs = (inputs.normal_bf16((S, B, Hk, d), cfg["std"], seed=400 + 2 * rank + i, device=dev) for i in (0, 1))
     o = torch.empty((B, H, d), dtype=torch.bfloat16, device=dev)
     lse = torch.empty((B, H), dtype=torch.float32, device=dev)
     ws = cache.new_workspace()
@@ -486,7 +499,9 @@ def run_decode_leg(args, cfg, world, rank, local):
     Rb = np.full(B, R, np.int64)
     bytes_leg = 0
     for _ in range(S):
-        bytes_leg += int(H * ((Rb + fill) * 2 * d * 2 + 6 * d * 2 + 4).sum())
+        # K/V rows of ring + window once per K/V head; q read, o written (and lse) per query
+        # head; k_new, v_new read and appended per K/V head
+        bytes_leg += int((Hk * ((Rb + fill) * 2 * d * 2 + 4 * d * 2) + H * (2 * d * 2 + 4)).sum())
         fill += 1
         full = fill == Tw
         Rb[full] += Tw - W
@@ -559,7 +574,8 @@ def run_focus(args, world, rank, local):
                           "inputs larger than L2 (Q/K/V %.2f GB per step)" % (3 * cfg["B"] * pre["T"] * cfg["H"] * cfg["d"] * 2 / 1e9)),
                    "prefill_kernel": "legacy mma.sync" if args.prefill_flags & 1 else "default",
                    "mask": "k-mer-local (Sec. 3.2)" if local_mask else "appendix (App. A, Eq. focus-attn)",
-                   "rope_theta": args.rope or None},
+                   "rope_theta": args.rope or None,
+                   "q_per_kv": args.q_per_kv},
         "augmented_tokens_per_s": world * cfg["B"] * pre["T"] / (pre["step_ms"] / 1e3),
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
                      "frac": achieved / peaks["bf16_tflops"], "traffic": traffic,
@@ -600,8 +616,8 @@ def run_focus(args, world, rank, local):
             "clocks": dec["clocks"],
         }
         line["decode"]["gpu_launches"] = dec["launches"]
-    if pre["host_sample"] is not None and args.rope:
-        line["cpu_baseline"] = None      # the oracle baseline times the path without the rotation
+    if pre["host_sample"] is not None and (args.rope or args.q_per_kv > 1):
+        line["cpu_baseline"] = None      # the oracle baseline times the default path only
     elif pre["host_sample"] is not None:
         hs = pre["host_sample"]
         if local_mask:
@@ -744,6 +760,8 @@ def main():
     ap.add_argument("--legacy", action="store_true", help="time the legacy mma.sync prefill kernel")
     ap.add_argument("--rope", type=float, default=0.0,
                     help="rotary-embedding base (0 = none): q and k are rotated at their position ids")
+    ap.add_argument("--q-per-kv", type=int, default=1,
+                    help="grouped-query heads: the workload's H query heads share H / G K/V heads")
     ap.add_argument("--mask", default="appendix", choices=["appendix", "kmer_local"],
                     help="prefill visibility: App. A (default) or the k-mer-local rule of Sec. 3.2")
     ap.add_argument("--memory-report", action="store_true",
@@ -753,6 +771,8 @@ def main():
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     args.prefill_flags = (1 if args.legacy else 0) | (2 if args.mask == "kmer_local" else 0)
+    if args.q_per_kv < 1:
+        ap.error("--q-per-kv must be >= 1")
     world, rank, local = dist_setup()
     if args.memory_report:
         run_memory_report(args, world, rank, local)

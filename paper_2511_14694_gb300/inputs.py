@@ -50,9 +50,11 @@ def normal_bf16(shape, std: float, seed: int, device="cpu") -> torch.Tensor:
     return x.to(torch.bfloat16)
 
 
-def qkv(shape, std: float = 1.0, seed: int = DEFAULT_SEED, device="cpu"):
-    """Three independent bf16 tensors of the given shape (Q, K, V)."""
-    return tuple(normal_bf16(shape, std, seed * 3 + i + 1, device) for i in range(3))
+def qkv(shape, std: float = 1.0, seed: int = DEFAULT_SEED, device="cpu", q_per_kv: int = 1):
+    """Three independent bf16 tensors (Q, K, V) of the given shape [B, H, ...];
+    with q_per_kv = g > 1 (grouped-query heads) K and V have H / g heads."""
+    kv_shape = tuple(shape) if q_per_kv <= 1 else (shape[0], shape[1] // q_per_kv) + tuple(shape[2:])
+    return tuple(normal_bf16(shape if i == 0 else kv_shape, std, seed * 3 + i + 1, device) for i in range(3))
 
 
 def start_fill(B: int, hi: int, seed: int = DEFAULT_SEED) -> np.ndarray:
