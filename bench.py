@@ -281,9 +281,13 @@ def run_prefill_leg(args, cfg, world, rank, local):
     lse = torch.empty((B, H, L["T"]), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
 
-    def front():
+    def front(evc=None):
         focus.layout_run(L, nt, stream=stream)
+        if evc is not None:
+            evc[0].record(stream)
         focus.kv_compact_bulk(cache, k, v, L, 0, L["M"], src_row0=0, stream=stream)
+        if evc is not None:
+            evc[1].record(stream)
 
     def attn():
         focus.attn_prefill(cache, q, k, v, L, 0, L["M"], o=o, lse=lse, stream=stream, flags=args.prefill_flags)
@@ -303,13 +307,14 @@ def run_prefill_leg(args, cfg, world, rank, local):
     bytes_per_step = float(B * L["T"] * (H * (4 * d + 4) + (H // g) * 4 * d))
 
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    evc = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier(world)
     torch.cuda.synchronize(dev)
     with ClockSampler(local) as clk:
         t_start.record(stream)
         for i in range(args.steps):
-            front()
+            front(evc[i])
             ev[i][0].record(stream)
             attn()
             ev[i][1].record(stream)
@@ -327,9 +332,25 @@ def run_prefill_leg(args, cfg, world, rank, local):
         torch.cuda.synchronize(dev)
     barrier(world)
     assert focus.device_status(clear=True) == 0
+    # the compaction alone (outside the timed step), each launch after an L2 flush
+    # (its 42 MB would otherwise stay in the 129 MB L2 between launches)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    n_c = 20
+    cev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_c)]
+    for i in range(n_c):
+        flush.fill_(i & 0xff)
+        cev[i][0].record(stream)
+        focus.kv_compact_bulk(cache, k, v, L, 0, L["M"], src_row0=0, stream=stream)
+        cev[i][1].record(stream)
+    torch.cuda.synchronize(dev)
+    compact_alone_ms = sum(a.elapsed_time(b) for a, b in cev) / n_c
+    del flush
     step_ms = t_start.elapsed_time(t_end) / args.steps
     step_ms = max_over_ranks(step_ms, world)
     attn_ms = sum(a.elapsed_time(b) for a, b in ev) / args.steps
+    compact_ms = sum(a.elapsed_time(b) for a, b in evc) / args.steps
+    # compaction moves R rows of K and V per K/V head: read once, written once
+    compact_bytes = float(L["R"] * B * (H // g) * 2 * (2 * d) * 2)
     launches = 4 * args.steps   # layout scan + layout rows + bulk compaction + prefill
 
     # end to end through the public API with host buffers
@@ -373,7 +394,9 @@ def run_prefill_leg(args, cfg, world, rank, local):
                            win=L["win"].cpu().numpy(), keep=L["keep"].cpu().numpy(), k_sched=k_s,
                            q=q[0, :2].cpu(), k=k[0, :2].cpu(), v=v[0, :2].cpu())
     res = dict(step_ms=step_ms, attn_ms=attn_ms, flops_per_step=flops_per_step, pairs=pairs, T=L["T"], R=L["R"],
-               bytes_per_step=bytes_per_step, local_mask=local_mask,
+               bytes_per_step=bytes_per_step, local_mask=local_mask, compact_ms=compact_alone_ms,
+               compact_in_step_ms=compact_ms,
+               compact_bytes=compact_bytes,
                clocks=clk.summary(), launches=launches, e2e=e2e, host_sample=host_sample, extra_steps=extra)
     del q, k, v, o, lse, cache
     torch.cuda.empty_cache()
@@ -601,6 +624,15 @@ def run_focus(args, world, rank, local):
         line["roofline"].update(bytes_per_launch=pre["bytes_per_step"] / n_launch,
                                 flop_per_launch=pre["flops_per_step"] / n_launch,
                                 avg_launch_ms=pre.get("per_launch_ms", pre["attn_ms"]), launches_per_step=n_launch)
+    if "compact_ms" in pre:
+        cgbs = pre["compact_bytes"] / (pre["compact_ms"] / 1e3) / 1e9
+        line["compaction"] = {"kernel": "focus_kv_compact (bulk)", "avg_launch_ms": pre["compact_ms"],
+                              "timing": "20 launches after the timed region, each after an L2 flush; in-step event time "
+                                        f"{pre['compact_in_step_ms']:.4f} ms",
+                              "bytes_per_launch": pre["compact_bytes"],
+                              "roofline": {"bound": "hbm", "achieved": cgbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                                           "frac": cgbs / peaks["hbm_gbs"],
+                                           "peak_source": f"{peaks_src} copy bandwidth"}}
     if dec is not None:
         gbs = dec["bytes_leg"] / (dec["decode_kernels_ms"] / 1e3) / 1e9
         line["decode"] = {

@@ -9,38 +9,56 @@ namespace focus {
 namespace {
 
 // Bulk mode: ring[b,h, r] <- src[b,h, sum_idx[r] - src_row0] for r in
-// [ring_off[w_begin], ring_off[w_end]). One thread moves one 16-byte chunk of
-// K and the same chunk of V; grid-stride over all chunks.
+// [ring_off[w_begin], ring_off[w_end]). Grid: (x, heads), x striding over
+// blocks of kBulkRows rows; CPR threads move one row (16 bytes each of K and
+// V), and every thread issues the loads of its kBulkRows / (256 / CPR) rows
+// before any store, so each SM keeps several KB in flight. No 64-bit division
+// in the index arithmetic.
+constexpr int kBulkRows = 64;
+
+template <int CPR>
 __global__ void __launch_bounds__(256) compact_bulk_kernel(
         uint4* __restrict__ ring_k, uint4* __restrict__ ring_v, const uint4* __restrict__ src_k,
-        const uint4* __restrict__ src_v, int32_t BH, int32_t B, int32_t chunks_per_row, int32_t C_ring,
-        int64_t src_T, int64_t src_row0, const int32_t* __restrict__ sum_idx,
-        const int32_t* __restrict__ ring_off, int32_t w_begin, int32_t w_end,
+        const uint4* __restrict__ src_v, int32_t BH, int32_t B, int32_t C_ring, int64_t src_T, int64_t src_row0,
+        const int32_t* __restrict__ sum_idx, const int32_t* __restrict__ ring_off, int32_t w_begin, int32_t w_end,
         int32_t* __restrict__ ring_len, int32_t* status) {
+    constexpr int RPP = 256 / CPR;                 // rows per pass of the CTA
+    constexpr int PASSES = kBulkRows / RPP;
     const int32_t r0 = ring_off[w_begin], r1 = ring_off[w_end];
-    const int64_t rows = r1 - r0;
     if (r1 > C_ring) {
-        if (blockIdx.x == 0 && threadIdx.x == 0) report(status, FOCUS_ERR_CAPACITY);
+        if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) report(status, FOCUS_ERR_CAPACITY);
         return;
     }
-    const int64_t total = (int64_t)BH * rows * chunks_per_row;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
-         i += (int64_t)gridDim.x * blockDim.x) {
-        const int32_t c = (int32_t)(i % chunks_per_row);
-        const int64_t rest = i / chunks_per_row;
-        const int64_t r = r0 + rest % rows;
-        const int64_t bh = rest / rows;
-        const int64_t srow = (int64_t)sum_idx[r] - src_row0;
-        if (srow < 0 || srow >= src_T) {
-            report(status, FOCUS_ERR_INVALID_ARG);
-            continue;
+    const int c = threadIdx.x % CPR, sub = threadIdx.x / CPR;
+    for (int32_t rb = r0 + (int32_t)blockIdx.x * kBulkRows; rb < r1; rb += (int32_t)gridDim.x * kBulkRows)
+    for (int64_t bh = blockIdx.y; bh < BH; bh += gridDim.y) {
+        uint4 kx[PASSES], vx[PASSES];
+        int32_t rr[PASSES];
+#pragma unroll
+        for (int p = 0; p < PASSES; ++p) {
+            const int32_t r = rb + p * RPP + sub;
+            rr[p] = -1;
+            if (r < r1) {
+                const int64_t srow = (int64_t)sum_idx[r] - src_row0;
+                if (srow < 0 || srow >= src_T) {
+                    report(status, FOCUS_ERR_INVALID_ARG);
+                    continue;
+                }
+                const int64_t so = (bh * src_T + srow) * CPR + c;
+                kx[p] = src_k[so];
+                vx[p] = src_v[so];
+                rr[p] = r;
+            }
         }
-        const int64_t so = (bh * src_T + srow) * chunks_per_row + c;
-        const int64_t d_o = (bh * C_ring + r) * chunks_per_row + c;
-        ring_k[d_o] = src_k[so];
-        ring_v[d_o] = src_v[so];
+#pragma unroll
+        for (int p = 0; p < PASSES; ++p) {
+            if (rr[p] < 0) continue;
+            const int64_t d_o = (bh * C_ring + rr[p]) * CPR + c;
+            ring_k[d_o] = kx[p];
+            ring_v[d_o] = vx[p];
+        }
     }
-    if (blockIdx.x == 0)
+    if (blockIdx.x == 0 && blockIdx.y == 0)
         for (int32_t b = threadIdx.x; b < B; b += blockDim.x) ring_len[b] = r1;
 }
 
@@ -152,14 +170,24 @@ __global__ void __launch_bounds__(256) compact_window_kernel(
 
 cudaError_t launch_compact_bulk(const focus_cache& c, const focus_compact_args& a, int32_t* status,
                                 cudaStream_t stream) {
+    // the span's row count lives on the device (ring_off): a grid that fills the
+    // GPU strides over its row blocks
     int dev = 0, sms = 152;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const int32_t cpr = c.d / 8;
-    compact_bulk_kernel<<<sms * 4, 256, 0, stream>>>(
-        (uint4*)c.ring_k, (uint4*)c.ring_v, (const uint4*)a.src_k, (const uint4*)a.src_v, c.B * c.H, c.B,
-        cpr, c.C_ring, a.src_T, a.src_row0, a.d_sum_idx, a.d_ring_off, a.w_begin, a.w_end, c.ring_len,
-        status);
+    const int64_t BH = (int64_t)c.B * c.H;
+    const unsigned by = (unsigned)(BH < 65535 ? BH : 65535);
+    const int64_t span_cap = ceil_div64(c.C_ring > 0 ? c.C_ring : 1, kBulkRows);
+    int64_t bx = ceil_div64(8 * (int64_t)sms, by);
+    if (bx > span_cap) bx = span_cap;
+    if (c.d == 128)
+        compact_bulk_kernel<16><<<dim3((unsigned)bx, by), 256, 0, stream>>>(
+            (uint4*)c.ring_k, (uint4*)c.ring_v, (const uint4*)a.src_k, (const uint4*)a.src_v, (int32_t)BH, c.B,
+            c.C_ring, a.src_T, a.src_row0, a.d_sum_idx, a.d_ring_off, a.w_begin, a.w_end, c.ring_len, status);
+    else
+        compact_bulk_kernel<8><<<dim3((unsigned)bx, by), 256, 0, stream>>>(
+            (uint4*)c.ring_k, (uint4*)c.ring_v, (const uint4*)a.src_k, (const uint4*)a.src_v, (int32_t)BH, c.B,
+            c.C_ring, a.src_T, a.src_row0, a.d_sum_idx, a.d_ring_off, a.w_begin, a.w_end, c.ring_len, status);
     return cudaGetLastError();
 }
 
