@@ -459,3 +459,87 @@ def test_full_size_streaming_sampled():
             assert_attn_close(got[w][0][i], got[w][1][i], o_ref[a:e], lse_ref[a:e], f"stream w={w} h={h}")
         assert np.array_equal(bits(cache.ring_k[b, h]), rk)
         assert np.array_equal(bits(cache.ring_v[b, h]), rv)
+
+
+# ----------------------------------------------------------------------------- full-size: the extra modes, sampled rows
+
+def test_full_size_kmer_local_prefill_sampled():
+    """128 kb, 32 heads, d = 128, k-mer-local mask (Sec. 3.2), in the launch
+    configuration the bench times; sampled rows of three heads."""
+    from paper_2511_14694_gb300.workloads import WORKLOADS
+    cfg = WORKLOADS["prefill_128kb_h32_d128"]
+    N, W, B, H, d = cfg["N"], cfg["W"], cfg["B"], cfg["H"], cfg["d"]
+    M = -(-N // W)
+    k_s = inputs.k_schedule(M, cfg["k"], seed=inputs.DEFAULT_SEED)
+    L = focus.layout(N, W, k_s)
+    q, k, v = inputs.qkv((B, H, L["T"], d), std=cfg["std"], seed=inputs.DEFAULT_SEED, device="cuda")
+    cache = focus.Cache(B, H, d, C_ring=L["R"], k_sched=k_s)
+    o, lse = pipeline.prefill_masked_parallel(cache, q, k, v, L, flags=focus.PREFILL_KMER_LOCAL)
+    torch.cuda.synchronize()
+    rows = _sample_rows(L, 6, 4, seed=2)
+    heads = [0, 13, 31]
+    ref_L = fo.layout(N, W, k_s)
+    km = fo.layout_kmer(N, W, k_s)
+    o_ref, lse_ref = fo.attn_rows_kmer_local(q[0, heads].cpu(), k[0, heads].cpu(), v[0, heads].cpu(), ref_L["kind"],
+                                             ref_L["win"], km, 1.0 / math.sqrt(d),
+                                             np.repeat(np.arange(len(heads)), rows.size), np.tile(rows, len(heads)))
+    assert_attn_close(o[0, heads][:, rows], lse[0, heads][:, rows], o_ref.reshape(len(heads), rows.size, d),
+                      lse_ref.reshape(len(heads), rows.size), "full-size k-mer-local")
+
+
+def test_full_size_rope_prefill_sampled():
+    """128 kb, 32 heads, d = 128, rotary base 500,000 (positions up to 129,279):
+    sampled rows of two heads against the oracle's fp64 rotation rounded to bf16."""
+    from paper_2511_14694_gb300.workloads import WORKLOADS
+    cfg = WORKLOADS["prefill_128kb_h32_d128"]
+    N, W, B, H, d, theta = cfg["N"], cfg["W"], cfg["B"], cfg["H"], cfg["d"], 500_000.0
+    L = focus.layout(N, W, cfg["k"])
+    q, k, v = inputs.qkv((B, H, L["T"], d), std=cfg["std"], seed=inputs.DEFAULT_SEED, device="cuda")
+    cache = focus.Cache(B, H, d, C_ring=L["R"], rope_theta=theta)
+    o, lse = pipeline.prefill_masked_parallel(cache, q, k, v, L)
+    torch.cuda.synchronize()
+    rows = _sample_rows(L, 5, 4, seed=3)
+    heads = [0, 21]
+    ref_L = fo.layout(N, W, cfg["k"])
+    pos = np.arange(L["T"])
+    qf = fo.rope(q[0, heads].cpu(), pos, theta, round_bf16=True)
+    kf = fo.rope(k[0, heads].cpu(), pos, theta, round_bf16=True)
+    o_ref, lse_ref = fo.attn_rows_f64(qf, kf, v[0, heads].cpu(), ref_L["keep"], ref_L["win"], 1.0 / math.sqrt(d),
+                                      np.repeat(np.arange(len(heads)), rows.size), np.tile(rows, len(heads)))
+    assert_attn_close(o[0, heads][:, rows], lse[0, heads][:, rows], o_ref.reshape(len(heads), rows.size, d),
+                      lse_ref.reshape(len(heads), rows.size), "full-size rope")
+
+
+def test_full_size_gqa_decode_sampled():
+    """Batch 64, 32 query heads over 8 K/V heads (q_per_kv = 4), d = 128, 10,000
+    retained rows + partly filled windows: two steps, sampled query heads."""
+    from paper_2511_14694_gb300.workloads import WORKLOADS
+    cfg = WORKLOADS["decode_1mb_b64_h32_d128"]
+    B, Hq, d, W, R, g = cfg["B"], cfg["H"], cfg["d"], cfg["W"], cfg["R"], 4
+    H = Hq // g
+    kk = cfg["k"][0]
+    Tw = W + W // kk
+    cache = focus.Cache(B, H, d, C_ring=R + 256, C_win=1_024, W=W, k_sched=np.full(2_000, kk, np.int32), q_per_kv=g)
+    for i, t in enumerate((cache.ring_k, cache.ring_v, cache.win_k, cache.win_v)):
+        t.copy_(inputs.normal_bf16(t.shape, cfg["std"], seed=60 + i, device="cuda"))
+    fill0 = inputs.start_fill(B, Tw - 1, seed=inputs.DEFAULT_SEED)
+    cache.ring_len.fill_(R)
+    cache.win_idx.fill_(R // (W // kk))
+    cache.win_fill.copy_(torch.from_numpy(fill0))
+    ws = cache.new_workspace()
+    pairs = [(0, 0), (5, 3), (17, 31), (63, 12)]
+    for step in range(2):
+        R_now, fill_now = cache.ring_len.cpu().numpy().copy(), cache.win_fill.cpu().numpy().copy()
+        snap = {(b, hq): tuple(x[b, hq // g].cpu() for x in (cache.ring_k, cache.ring_v, cache.win_k, cache.win_v))
+                for b, hq in pairs}
+        q = inputs.normal_bf16((B, Hq, d), cfg["std"], seed=210 + step, device="cuda")
+        kn, vn = (inputs.normal_bf16((B, H, d), cfg["std"], seed=220 + 2 * step + i, device="cuda") for i in (0, 1))
+        o, lse = focus.attn_decode(cache, q, kn, vn, workspace=ws)
+        focus.kv_compact_window(cache)
+        torch.cuda.synchronize()
+        for b, hq in pairs:
+            rk, rv, wk, wv = snap[(b, hq)]
+            o_ref, lse_ref = fo.decode(q[b, hq][None].cpu(), kn[b, hq // g][None].cpu(), vn[b, hq // g][None].cpu(),
+                                       rk[None], rv[None], [R_now[b]], wk[None], wv[None], [fill_now[b]],
+                                       1.0 / math.sqrt(d))
+            assert_attn_close(o[b, hq][None], lse[b, hq][None], o_ref, lse_ref, f"gqa decode b={b} hq={hq}")
