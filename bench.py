@@ -332,19 +332,6 @@ def run_prefill_leg(args, cfg, world, rank, local):
         torch.cuda.synchronize(dev)
     barrier(world)
     assert focus.device_status(clear=True) == 0
-    # the compaction alone (outside the timed step), each launch after an L2 flush
-    # (its 42 MB would otherwise stay in the 129 MB L2 between launches)
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
-    n_c = 20
-    cev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_c)]
-    for i in range(n_c):
-        flush.fill_(i & 0xff)
-        cev[i][0].record(stream)
-        focus.kv_compact_bulk(cache, k, v, L, 0, L["M"], src_row0=0, stream=stream)
-        cev[i][1].record(stream)
-    torch.cuda.synchronize(dev)
-    compact_alone_ms = sum(a.elapsed_time(b) for a, b in cev) / n_c
-    del flush
     step_ms = t_start.elapsed_time(t_end) / args.steps
     step_ms = max_over_ranks(step_ms, world)
     attn_ms = sum(a.elapsed_time(b) for a, b in ev) / args.steps
@@ -394,8 +381,7 @@ def run_prefill_leg(args, cfg, world, rank, local):
                            win=L["win"].cpu().numpy(), keep=L["keep"].cpu().numpy(), k_sched=k_s,
                            q=q[0, :2].cpu(), k=k[0, :2].cpu(), v=v[0, :2].cpu())
     res = dict(step_ms=step_ms, attn_ms=attn_ms, flops_per_step=flops_per_step, pairs=pairs, T=L["T"], R=L["R"],
-               bytes_per_step=bytes_per_step, local_mask=local_mask, compact_ms=compact_alone_ms,
-               compact_in_step_ms=compact_ms,
+               bytes_per_step=bytes_per_step, local_mask=local_mask, compact_ms=compact_ms,
                compact_bytes=compact_bytes,
                clocks=clk.summary(), launches=launches, e2e=e2e, host_sample=host_sample, extra_steps=extra)
     del q, k, v, o, lse, cache
@@ -627,8 +613,8 @@ def run_focus(args, world, rank, local):
     if "compact_ms" in pre:
         cgbs = pre["compact_bytes"] / (pre["compact_ms"] / 1e3) / 1e9
         line["compaction"] = {"kernel": "focus_kv_compact (bulk)", "avg_launch_ms": pre["compact_ms"],
-                              "timing": "20 launches after the timed region, each after an L2 flush; in-step event time "
-                                        f"{pre['compact_in_step_ms']:.4f} ms",
+                              "timing": "CUDA events around the compaction inside each timed step (after the "
+                                        "previous step's prefill); a ~10 us launch, so the launch gap counts",
                               "bytes_per_launch": pre["compact_bytes"],
                               "roofline": {"bound": "hbm", "achieved": cgbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                                            "frac": cgbs / peaks["hbm_gbs"],

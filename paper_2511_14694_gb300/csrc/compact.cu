@@ -4,62 +4,89 @@
 // appended to the per-(sequence, head) ring. Other rows are simply not copied.
 // Pure data movement, bit-exact; 16-byte vector loads and stores.
 #include "common.cuh"
+#include "sm100.cuh"
 
 namespace focus {
 namespace {
 
 // Bulk mode: ring[b,h, r] <- src[b,h, sum_idx[r] - src_row0] for r in
-// [ring_off[w_begin], ring_off[w_end]). Grid: (x, heads), x striding over
-// blocks of kBulkRows rows; CPR threads move one row (16 bytes each of K and
-// V), and every thread issues the loads of its kBulkRows / (256 / CPR) rows
-// before any store, so each SM keeps several KB in flight. No 64-bit division
-// in the index arithmetic.
+// [ring_off[w_begin], ring_off[w_end]). One warp per unit of 64 ring rows of one
+// (sequence, head): its lanes gather the rows' K and V into shared memory with
+// one cp.async.bulk per row (the copy engine keeps far more bytes in flight than
+// per-thread loads, whose outstanding misses per SM are capped), and since the
+// unit's ring rows are contiguous, two bulk stores write it out.
 constexpr int kBulkRows = 64;
 
-template <int CPR>
-__global__ void __launch_bounds__(256) compact_bulk_kernel(
-        uint4* __restrict__ ring_k, uint4* __restrict__ ring_v, const uint4* __restrict__ src_k,
-        const uint4* __restrict__ src_v, int32_t BH, int32_t B, int32_t C_ring, int64_t src_T, int64_t src_row0,
+template <int D>
+__global__ void __launch_bounds__(32) compact_bulk_kernel(
+        uint8_t* __restrict__ ring_k, uint8_t* __restrict__ ring_v, const uint8_t* __restrict__ src_k,
+        const uint8_t* __restrict__ src_v, int32_t BH, int32_t B, int32_t C_ring, int64_t src_T, int64_t src_row0,
         const int32_t* __restrict__ sum_idx, const int32_t* __restrict__ ring_off, int32_t w_begin, int32_t w_end,
         int32_t* __restrict__ ring_len, int32_t* status) {
-    constexpr int RPP = 256 / CPR;                 // rows per pass of the CTA
-    constexpr int PASSES = kBulkRows / RPP;
+    using namespace sm100;
+    constexpr int ROWB = 2 * D;
+    __shared__ __align__(128) uint8_t sk[kBulkRows * ROWB];
+    __shared__ __align__(128) uint8_t sv[kBulkRows * ROWB];
+    __shared__ uint64_t bar;
+    const int lane = threadIdx.x;
     const int32_t r0 = ring_off[w_begin], r1 = ring_off[w_end];
     if (r1 > C_ring) {
-        if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) report(status, FOCUS_ERR_CAPACITY);
+        if (blockIdx.x == 0 && lane == 0) report(status, FOCUS_ERR_CAPACITY);
         return;
     }
-    const int c = threadIdx.x % CPR, sub = threadIdx.x / CPR;
-    for (int32_t rb = r0 + (int32_t)blockIdx.x * kBulkRows; rb < r1; rb += (int32_t)gridDim.x * kBulkRows)
-    for (int64_t bh = blockIdx.y; bh < BH; bh += gridDim.y) {
-        uint4 kx[PASSES], vx[PASSES];
-        int32_t rr[PASSES];
+    if (lane == 0) {
+        mbar_init(smem_addr(&bar), 1);
+        fence_barrier_init();
+    }
+    __syncwarp();
+    const int32_t nrb = (r1 - r0 + kBulkRows - 1) / kBulkRows;
+    const int64_t units = (int64_t)nrb * BH;
+    uint32_t phase = 0;
+    for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
+        const int32_t rs = r0 + (int32_t)(u % nrb) * kBulkRows;
+        const int64_t bh = u / nrb;
+        const int32_t rows = r1 - rs < kBulkRows ? r1 - rs : kBulkRows;
+        // each lane owns rows lane and lane + 32 of the unit
+        int64_t srow[2];
+        bool bad = false;
 #pragma unroll
-        for (int p = 0; p < PASSES; ++p) {
-            const int32_t r = rb + p * RPP + sub;
-            rr[p] = -1;
-            if (r < r1) {
-                const int64_t srow = (int64_t)sum_idx[r] - src_row0;
-                if (srow < 0 || srow >= src_T) {
-                    report(status, FOCUS_ERR_INVALID_ARG);
-                    continue;
-                }
-                const int64_t so = (bh * src_T + srow) * CPR + c;
-                kx[p] = src_k[so];
-                vx[p] = src_v[so];
-                rr[p] = r;
+        for (int q = 0; q < 2; ++q) {
+            const int i = lane + 32 * q;
+            srow[q] = i < rows ? (int64_t)sum_idx[rs + i] - src_row0 : 0;
+            if (i < rows && (srow[q] < 0 || srow[q] >= src_T)) bad = true;
+        }
+        if (__any_sync(0xffffffffu, bad)) {
+            if (lane == 0) report(status, FOCUS_ERR_INVALID_ARG);
+            continue;
+        }
+        if (lane == 0) mbar_expect_tx(smem_addr(&bar), (uint32_t)(rows * 2 * ROWB));
+        __syncwarp();
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            const int i = lane + 32 * q;
+            if (i < rows) {
+                const int64_t so = (bh * src_T + srow[q]) * ROWB;
+                bulk_load(smem_addr(sk + i * ROWB), src_k + so, ROWB, smem_addr(&bar));
+                bulk_load(smem_addr(sv + i * ROWB), src_v + so, ROWB, smem_addr(&bar));
             }
         }
-#pragma unroll
-        for (int p = 0; p < PASSES; ++p) {
-            if (rr[p] < 0) continue;
-            const int64_t d_o = (bh * C_ring + rr[p]) * CPR + c;
-            ring_k[d_o] = kx[p];
-            ring_v[d_o] = vx[p];
+        if (!mbar_wait(smem_addr(&bar), phase, 2000000000ull)) {
+            if (lane == 0) report(status, FOCUS_ERR_TIMEOUT);
+            break;
         }
+        phase ^= 1u;
+        if (lane == 0) {
+            const int64_t d_o = (bh * C_ring + rs) * ROWB;
+            bulk_store(ring_k + d_o, smem_addr(sk), (uint32_t)(rows * ROWB));
+            bulk_store(ring_v + d_o, smem_addr(sv), (uint32_t)(rows * ROWB));
+            bulk_commit();
+            bulk_wait_read_all();              // the buffers are reused by the next unit
+        }
+        __syncwarp();
     }
-    if (blockIdx.x == 0 && blockIdx.y == 0)
-        for (int32_t b = threadIdx.x; b < B; b += blockDim.x) ring_len[b] = r1;
+    if (lane == 0) bulk_wait_all();            // the ring rows are written before the CTA exits
+    if (blockIdx.x == 0)
+        for (int32_t b = lane; b < B; b += 32) ring_len[b] = r1;
 }
 
 // Bulk mode with the rotary embedding: ring K rows are stored rotated at their
@@ -170,24 +197,22 @@ __global__ void __launch_bounds__(256) compact_window_kernel(
 
 cudaError_t launch_compact_bulk(const focus_cache& c, const focus_compact_args& a, int32_t* status,
                                 cudaStream_t stream) {
-    // the span's row count lives on the device (ring_off): a grid that fills the
-    // GPU strides over its row blocks
+    // the span's row count lives on the device (ring_off): at most one warp per
+    // possible unit, at most eight per SM; each strides over the units
     int dev = 0, sms = 152;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int64_t BH = (int64_t)c.B * c.H;
-    const unsigned by = (unsigned)(BH < 65535 ? BH : 65535);
-    const int64_t span_cap = ceil_div64(c.C_ring > 0 ? c.C_ring : 1, kBulkRows);
-    int64_t bx = ceil_div64(8 * (int64_t)sms, by);
-    if (bx > span_cap) bx = span_cap;
+    int64_t grid = ceil_div64(c.C_ring > 0 ? c.C_ring : 1, kBulkRows) * BH;
+    if (grid > 8 * (int64_t)sms) grid = 8 * (int64_t)sms;
     if (c.d == 128)
-        compact_bulk_kernel<16><<<dim3((unsigned)bx, by), 256, 0, stream>>>(
-            (uint4*)c.ring_k, (uint4*)c.ring_v, (const uint4*)a.src_k, (const uint4*)a.src_v, (int32_t)BH, c.B,
-            c.C_ring, a.src_T, a.src_row0, a.d_sum_idx, a.d_ring_off, a.w_begin, a.w_end, c.ring_len, status);
+        compact_bulk_kernel<128><<<(unsigned)grid, 32, 0, stream>>>(
+            (uint8_t*)c.ring_k, (uint8_t*)c.ring_v, (const uint8_t*)a.src_k, (const uint8_t*)a.src_v, (int32_t)BH,
+            c.B, c.C_ring, a.src_T, a.src_row0, a.d_sum_idx, a.d_ring_off, a.w_begin, a.w_end, c.ring_len, status);
     else
-        compact_bulk_kernel<8><<<dim3((unsigned)bx, by), 256, 0, stream>>>(
-            (uint4*)c.ring_k, (uint4*)c.ring_v, (const uint4*)a.src_k, (const uint4*)a.src_v, (int32_t)BH, c.B,
-            c.C_ring, a.src_T, a.src_row0, a.d_sum_idx, a.d_ring_off, a.w_begin, a.w_end, c.ring_len, status);
+        compact_bulk_kernel<64><<<(unsigned)grid, 32, 0, stream>>>(
+            (uint8_t*)c.ring_k, (uint8_t*)c.ring_v, (const uint8_t*)a.src_k, (const uint8_t*)a.src_v, (int32_t)BH,
+            c.B, c.C_ring, a.src_T, a.src_row0, a.d_sum_idx, a.d_ring_off, a.w_begin, a.w_end, c.ring_len, status);
     return cudaGetLastError();
 }
 
