@@ -294,6 +294,277 @@ __global__ void __launch_bounds__(kDecodeThreads + 32) decode_split_kernel(
     __syncthreads();
 }
 
+// ---------------------------------------------------------------------------
+// Grouped-query decode on the tensor cores (q_per_kv = g >= 2): a CTA serves
+// QG <= 8 query heads of one K/V head. The QG queries are the rows of the A
+// operand of mma.sync m16n8k16 (rows QG..15 are zero), so every K/V row streamed
+// from HBM feeds all QG queries through the MMA instead of QG dot products and
+// shuffle reductions on the CUDA cores. The producer warp's lanes copy each key
+// row (ring, window or the new row) into a shared-memory stage whose rows are
+// padded by 16 bytes, which keeps the ldmatrix reads conflict-free; each
+// consumer warp takes 16 keys of a 64-row stage: S = Q K^T (K through ldmatrix),
+// online softmax on the S fragments, O += P V (P reused from the S registers as
+// the A operand, V through ldmatrix.trans). Partials (m, l, o) per query head go
+// to the same workspace as the CUDA-core kernel and the same combine kernel.
+// ---------------------------------------------------------------------------
+constexpr int kMmaStageRows = 64;            // 16 keys per consumer warp
+constexpr int kMmaStages = 3;
+
+template <int D>
+constexpr int mma_row_stride() { return D * 2; }
+template <int D, int QG>
+constexpr int decode_mma_smem_bytes() {
+    return 2 * kMmaStages * kMmaStageRows * mma_row_stride<D>() + 2 * kMmaStages * 8 +
+           QG * (kDecodeThreads / 32) * (2 + D) * 4;
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
+}
+__device__ __forceinline__ void mma_16816(float* c, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
+                                          uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};\n"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+template <int D, int QG>
+__global__ void __launch_bounds__(kDecodeThreads + 32) decode_split_mma_kernel(
+        const uint8_t* __restrict__ ring_k, const uint8_t* __restrict__ ring_v, uint4* __restrict__ win_k,
+        uint4* __restrict__ win_v, const int32_t* __restrict__ ring_len, const int32_t* __restrict__ win_fill,
+        const int32_t* __restrict__ win_idx, const int32_t* __restrict__ ks, int32_t n_windows, int32_t W,
+        int32_t H, int32_t C_ring, int32_t C_win, const uint32_t* __restrict__ q, const uint4* __restrict__ k_new,
+        const uint4* __restrict__ v_new, float scale_log2, float2* __restrict__ ws_ml, float* __restrict__ ws_o,
+        int32_t n_splits, int32_t* status, const int32_t* __restrict__ W_per_window, int32_t q_per_kv) {
+    using namespace sm100;
+    static_assert(QG >= 2 && QG <= 8, "one query per A row, rows 0..7");
+    constexpr int CPR = D / 8, ROWB = D * 2, RS = mma_row_stride<D>(), CH = kMmaStageRows;
+    constexpr int NW = kDecodeThreads / 32;
+    const int slices = q_per_kv / QG;
+    const int b = blockIdx.z, h = blockIdx.y / slices, slice = blockIdx.y % slices, split = blockIdx.x;
+    const int64_t bh = (int64_t)b * H + h;
+    const int64_t bhq0 = bh * q_per_kv + (int64_t)slice * QG;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+
+    const int32_t R = ring_len[b], fill = win_fill[b], widx = win_idx[b];
+    int32_t Tw = 0;
+    const bool state_ok = decode_state_ok(R, fill, widx, ks, n_windows, W, C_ring, C_win, &Tw, W_per_window);
+    const int64_t total = (int64_t)R + fill + 1;
+    const int64_t s0 = (int64_t)split * kDecodeChunk;
+    const int64_t s1 = min(total, s0 + kDecodeChunk);
+    if (!state_ok || s0 >= s1) {
+        if (!state_ok && split == 0 && blockIdx.y == 0 && tid == 0) report(status, FOCUS_ERR_CAPACITY);
+        for (int j = 0; j < QG; ++j) {
+            float* wo = ws_o + ((bhq0 + j) * n_splits + split) * D;
+            for (int c = tid; c < D; c += blockDim.x) wo[c] = 0.f;
+            if (tid == 0) ws_ml[(bhq0 + j) * n_splits + split] = make_float2(-INFINITY, 0.f);
+        }
+        return;
+    }
+    if (split == 0 && slice == 0 && tid < CPR) {      // append the new row to the window buffer
+        win_k[(bh * C_win + fill) * CPR + tid] = k_new[bh * CPR + tid];
+        win_v[(bh * C_win + fill) * CPR + tid] = v_new[bh * CPR + tid];
+    }
+
+    extern __shared__ __align__(128) unsigned char smem[];
+    uint8_t* sK = smem;                                         // [stages][CH][RS]
+    uint8_t* sV = smem + kMmaStages * CH * RS;
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + 2 * kMmaStages * CH * RS);
+    uint64_t* empty = full + kMmaStages;
+    float* sm_m = reinterpret_cast<float*>(empty + kMmaStages);   // [NW][QG]
+    float* sm_l = sm_m + NW * QG;                                  // [NW][QG]
+    float* sm_o = sm_l + NW * QG;                                  // [NW][QG][D]
+    __shared__ int32_t abort_flag;
+    const int n_chunks = (int)((s1 - s0 + CH - 1) / CH);
+
+    if (tid == 0) {
+        for (int i = 0; i < kMmaStages; ++i) {
+            mbar_init(smem_addr(&full[i]), 1);
+            mbar_init(smem_addr(&empty[i]), NW);
+        }
+        abort_flag = 0;
+        fence_barrier_init();
+    }
+    __syncthreads();
+
+    if (warp == NW) {
+        // ------------------------------------------------ producer: one bulk copy per row
+        const uint8_t* rk = ring_k + bh * (int64_t)C_ring * ROWB;
+        const uint8_t* rv = ring_v + bh * (int64_t)C_ring * ROWB;
+        const uint8_t* wk = reinterpret_cast<const uint8_t*>(win_k) + bh * (int64_t)C_win * ROWB;
+        const uint8_t* wv = reinterpret_cast<const uint8_t*>(win_v) + bh * (int64_t)C_win * ROWB;
+        const uint8_t* nk = reinterpret_cast<const uint8_t*>(k_new) + bh * ROWB;
+        const uint8_t* nv = reinterpret_cast<const uint8_t*>(v_new) + bh * ROWB;
+        int issued = 0;
+        for (int c = 0; c < n_chunks; ++c) {
+            const int st = c % kMmaStages, use = c / kMmaStages;
+            bool ok = true;
+            if (lane == 0 && use > 0 && !mbar_wait(smem_addr(&empty[st]), (use - 1) & 1, kWaitNs)) ok = false;
+            if (!__all_sync(0xffffffffu, ok)) {
+                if (lane == 0) {
+                    report(status, FOCUS_ERR_TIMEOUT);
+                    atomicExch(&abort_flag, 1);
+                }
+                break;
+            }
+            const int64_t k0 = s0 + (int64_t)c * CH, k1 = min(s1, k0 + CH);
+            const uint32_t bar = smem_addr(&full[st]);
+            if (lane == 0) {                                 // at most three contiguous copies per tensor
+                mbar_expect_tx(bar, (uint32_t)((k1 - k0) * ROWB * 2));
+                const uint32_t dk = smem_addr(sK + st * CH * RS), dv = smem_addr(sV + st * CH * RS);
+                int64_t a = k0, e = min(k1, (int64_t)R);                 // ring rows
+                if (a < e) {
+                    bulk_load(dk, rk + a * ROWB, (uint32_t)((e - a) * ROWB), bar);
+                    bulk_load(dv, rv + a * ROWB, (uint32_t)((e - a) * ROWB), bar);
+                }
+                a = max(k0, (int64_t)R);
+                e = min(k1, (int64_t)R + fill);                          // current-window rows
+                if (a < e) {
+                    const uint32_t off = (uint32_t)((a - k0) * ROWB);
+                    bulk_load(dk + off, wk + (a - R) * ROWB, (uint32_t)((e - a) * ROWB), bar);
+                    bulk_load(dv + off, wv + (a - R) * ROWB, (uint32_t)((e - a) * ROWB), bar);
+                }
+                if (k1 == total) {                                        // the new row itself
+                    const uint32_t off = (uint32_t)((total - 1 - k0) * ROWB);
+                    bulk_load(dk + off, nk, ROWB, bar);
+                    bulk_load(dv + off, nv, ROWB, bar);
+                }
+            }
+            __syncwarp();
+            issued = c + 1;
+        }
+        if (lane == 0)                                               // drain before exit
+            for (int c = max(0, issued - kMmaStages); c < issued; ++c)
+                mbar_wait(smem_addr(&full[c % kMmaStages]), (c / kMmaStages) & 1, kWaitNs);
+        __syncthreads();
+        return;
+    }
+
+    // ---------------------------------------------------- consumers
+    const int g = lane >> 2, t4 = lane & 3;                 // fragment row (query) and column pair
+    // Q as A fragments: rows g < QG hold the CTA's query heads, rows 8..15 are zero
+    uint32_t qa[D / 16][2];
+#pragma unroll
+    for (int kk = 0; kk < D / 16; ++kk) {
+        const bool row = g < QG;
+        const int64_t qw = (bhq0 + (row ? g : 0)) * (D / 2) + kk * 8 + t4;   // 32-bit words of q
+        qa[kk][0] = row ? q[qw] : 0u;
+        qa[kk][1] = row ? q[qw + 4] : 0u;
+    }
+    float m = -INFINITY, l = 0.f;
+    float oacc[D / 8][4];
+#pragma unroll
+    for (int i = 0; i < D / 8; ++i) oacc[i][0] = oacc[i][1] = oacc[i][2] = oacc[i][3] = 0.f;
+
+    for (int c = 0; c < n_chunks; ++c) {
+        const int st = c % kMmaStages;
+        if (!mbar_wait(smem_addr(&full[st]), (c / kMmaStages) & 1, kWaitNs) || abort_flag) {
+            report(status, FOCUS_ERR_TIMEOUT);
+            break;
+        }
+        const int nrow = (int)min((int64_t)CH, s1 - (s0 + (int64_t)c * CH));
+        const int key0 = warp * 16;                          // this warp's 16 keys of the stage
+        if (key0 < nrow) {
+            const uint8_t* cK = sK + st * CH * RS;
+            uint8_t* cV = sV + st * CH * RS;
+            if (key0 + 16 > nrow) {
+                // the split's last, partial stage: rows past the keys were never
+                // written; their P is 0, but 0 x NaN is not, so zero this warp's
+                // unused V rows (the stage is not refilled after the last chunk)
+                const int nz = key0 + 16 - nrow;
+                for (int i = lane; i < nz * CPR; i += 32)
+                    *reinterpret_cast<uint4*>(cV + (nrow + i / CPR) * RS + (i % CPR) * 16) = make_uint4(0, 0, 0, 0);
+                __syncwarp();
+            }
+            float sacc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+            const int mi = lane >> 3;
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+                const int key = key0 + (mi >> 1) * 8 + (lane & 7);
+                const int chunk = kk * 2 + (mi & 1);
+                uint32_t r0, r1, r2, r3;
+                ldsm_x4(smem_addr(cK + key * RS + chunk * 16), r0, r1, r2, r3);
+                mma_16816(sacc[0], qa[kk][0], 0u, qa[kk][1], 0u, r0, r1);
+                mma_16816(sacc[1], qa[kk][0], 0u, qa[kk][1], 0u, r2, r3);
+            }
+            // online softmax on row g (columns 2 t4, 2 t4 + 1 of each 8-key block)
+            float sv[4];
+#pragma unroll
+            for (int n = 0; n < 2; ++n)
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const int key = key0 + n * 8 + 2 * t4 + e;
+                    sv[n * 2 + e] = key < nrow ? sacc[n][e] * scale_log2 : -INFINITY;
+                }
+            float mx = fmaxf(fmaxf(sv[0], sv[1]), fmaxf(sv[2], sv[3]));
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+            const float mn = fmaxf(m, mx);
+            const float corr = ex2_approx(m - mn);               // 0 when m was -inf
+            l *= corr;
+#pragma unroll
+            for (int i = 0; i < D / 8; ++i) { oacc[i][0] *= corr; oacc[i][1] *= corr; }
+            m = mn;
+            float p[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                p[e] = ex2_approx(sv[e] - m);
+                l += p[e];
+            }
+            const uint32_t pa0 = pack_bf16x2(p[0], p[1]), pa2 = pack_bf16x2(p[2], p[3]);
+#pragma unroll
+            for (int dp = 0; dp < D / 16; ++dp) {
+                const int key = key0 + (mi & 1) * 8 + (lane & 7);
+                const int chunk = 2 * dp + (mi >> 1);
+                uint32_t r0, r1, r2, r3;
+                ldsm_x4_t(smem_addr(cV + key * RS + chunk * 16), r0, r1, r2, r3);
+                mma_16816(oacc[2 * dp], pa0, 0u, pa2, 0u, r0, r1);
+                mma_16816(oacc[2 * dp + 1], pa0, 0u, pa2, 0u, r2, r3);
+            }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_addr(&empty[st]));
+    }
+
+    // ---- merge the four warps' partials per query head -----------------------
+    l += __shfl_xor_sync(0xffffffffu, l, 1);
+    l += __shfl_xor_sync(0xffffffffu, l, 2);
+    if (g < QG) {
+        if (t4 == 0) { sm_m[warp * QG + g] = m; sm_l[warp * QG + g] = l; }
+#pragma unroll
+        for (int i = 0; i < D / 8; ++i) {
+            sm_o[(warp * QG + g) * D + i * 8 + 2 * t4] = oacc[i][0];
+            sm_o[(warp * QG + g) * D + i * 8 + 2 * t4 + 1] = oacc[i][1];
+        }
+    }
+    asm volatile("bar.sync 1, %0;" ::"n"(kDecodeThreads));       // consumers only
+    for (int col = tid; col < QG * D; col += kDecodeThreads) {
+        const int j = col / D, cc = col % D;
+        float M = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < NW; ++w) M = fmaxf(M, sm_m[w * QG + j]);
+        float L = 0.f, A = 0.f;
+        if (M != -INFINITY) {
+#pragma unroll
+            for (int w = 0; w < NW; ++w) {
+                const float f = ex2_approx(sm_m[w * QG + j] - M);
+                L = fmaf(sm_l[w * QG + j], f, L);
+                A = fmaf(sm_o[(w * QG + j) * D + cc], f, A);
+            }
+        }
+        ws_o[((bhq0 + j) * n_splits + split) * D + cc] = A;
+        if (cc == 0) ws_ml[(bhq0 + j) * n_splits + split] = make_float2(M, L);
+    }
+    __syncthreads();
+}
+
 template <int D>
 __global__ void __launch_bounds__(D) decode_combine_kernel(
         const float2* __restrict__ ws_ml, const float* __restrict__ ws_o, int32_t n_splits, int32_t H,
@@ -376,6 +647,23 @@ cudaError_t launch_decode_split(const focus_cache& c, int32_t ns, const void* q,
     return cudaGetLastError();
 }
 
+template <int D, int QG>
+cudaError_t launch_decode_split_mma(const focus_cache& c, int32_t ns, const void* q, const void* k_new,
+                                    const void* v_new, float scale, float2* ws_ml, float* ws_o, int32_t* status,
+                                    cudaStream_t stream) {
+    const int32_t g = q_heads_per_kv(c);
+    constexpr int smem = decode_mma_smem_bytes<D, QG>();
+    cudaError_t e0 = cudaFuncSetAttribute(decode_split_mma_kernel<D, QG>,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e0 != cudaSuccess) return e0;
+    decode_split_mma_kernel<D, QG><<<dim3(ns, c.H * (g / QG), c.B), kDecodeThreads + 32, smem, stream>>>(
+        (const uint8_t*)c.ring_k, (const uint8_t*)c.ring_v, (uint4*)c.win_k, (uint4*)c.win_v, c.ring_len,
+        c.win_fill, c.win_idx, c.k_per_window, c.n_windows, c.W, c.H, c.C_ring, c.C_win, (const uint32_t*)q,
+        (const uint4*)k_new, (const uint4*)v_new, scale * 1.4426950408889634f, ws_ml, ws_o, ns, status,
+        c.W_per_window, g);
+    return cudaGetLastError();
+}
+
 template <int D>
 cudaError_t launch_decode_d(const focus_cache& c, const void* q, const void* k_new, const void* v_new,
                             float scale, void* o, float* lse, void* workspace, int32_t* status,
@@ -398,9 +686,13 @@ cudaError_t launch_decode_d(const focus_cache& c, const void* q, const void* k_n
         q = q_rot;
         k_new = k_rot;
     }
-    cudaError_t e = (g % 4 == 0)   ? launch_decode_split<D, 4>(c, ns, q, k_new, v_new, scale, ws_ml, ws_o, status, stream)
-                    : (g % 2 == 0) ? launch_decode_split<D, 2>(c, ns, q, k_new, v_new, scale, ws_ml, ws_o, status, stream)
-                                   : launch_decode_split<D, 1>(c, ns, q, k_new, v_new, scale, ws_ml, ws_o, status, stream);
+    // grouped heads go to the tensor-core kernel (up to eight query heads per K/V
+    // pass); one query head per K/V head, or an odd group, to the CUDA-core one
+    cudaError_t e =
+        (g % 8 == 0)   ? launch_decode_split_mma<D, 8>(c, ns, q, k_new, v_new, scale, ws_ml, ws_o, status, stream)
+        : (g % 4 == 0) ? launch_decode_split_mma<D, 4>(c, ns, q, k_new, v_new, scale, ws_ml, ws_o, status, stream)
+        : (g % 2 == 0) ? launch_decode_split_mma<D, 2>(c, ns, q, k_new, v_new, scale, ws_ml, ws_o, status, stream)
+                       : launch_decode_split<D, 1>(c, ns, q, k_new, v_new, scale, ws_ml, ws_o, status, stream);
     if (e != cudaSuccess) return e;
     decode_combine_kernel<D><<<dim3((unsigned)Hq, c.B), D, 0, stream>>>(
         ws_ml, ws_o, ns, (int32_t)Hq, (__nv_bfloat16*)o, lse, c.win_fill, c.ring_len, c.win_idx, c.k_per_window,
