@@ -2,7 +2,8 @@
 // inference: the retained FOCUS K/V of earlier windows are the history, the
 // current window's rows are attended causally; the new row sees itself).
 //
-// HBM-bound: every K/V row of the ring and of the window buffer is read once.
+// HBM-bound: every K/V row of the ring and of the window buffer is read once
+// per K/V head (grouped query heads share the pass, see the tensor-core kernel).
 // Split-K over keys: grid (split, head, sequence); each CTA streams a chunk of
 // keys with 16-byte loads (d/8 lanes per key row, several rows in flight per
 // thread), keeps a per-lane-group online softmax in registers, merges the
@@ -68,7 +69,8 @@ __device__ __forceinline__ bool decode_state_ok(int32_t R, int32_t fill, int32_t
 //
 // Grouped-query heads (q_per_kv = g > 1): one CTA serves QG of the g query
 // heads that share its K/V head, so each K/V row it streams is used QG times
-// (blockIdx.y = kv head * (g / QG) + which QG-slice of the group).
+// (blockIdx.y = kv head * (g / QG) + which QG-slice of the group). Even groups
+// go to the tensor-core kernel below; this one serves g = 1 and odd g (QG = 1).
 template <int D, int QG>
 __global__ void __launch_bounds__(kDecodeThreads + 32) decode_split_kernel(
         const uint4* __restrict__ ring_k, const uint4* __restrict__ ring_v, uint4* __restrict__ win_k,
@@ -296,26 +298,32 @@ __global__ void __launch_bounds__(kDecodeThreads + 32) decode_split_kernel(
 
 // ---------------------------------------------------------------------------
 // Grouped-query decode on the tensor cores (q_per_kv = g >= 2): a CTA serves
-// QG <= 8 query heads of one K/V head. The QG queries are the rows of the A
+// QG <= 16 query heads of one K/V head. The QG queries are the rows of the A
 // operand of mma.sync m16n8k16 (rows QG..15 are zero), so every K/V row streamed
 // from HBM feeds all QG queries through the MMA instead of QG dot products and
-// shuffle reductions on the CUDA cores. The producer warp's lanes copy each key
-// row (ring, window or the new row) into a shared-memory stage whose rows are
-// padded by 16 bytes, which keeps the ldmatrix reads conflict-free; each
-// consumer warp takes 16 keys of a 64-row stage: S = Q K^T (K through ldmatrix),
-// online softmax on the S fragments, O += P V (P reused from the S registers as
-// the A operand, V through ldmatrix.trans). Partials (m, l, o) per query head go
-// to the same workspace as the CUDA-core kernel and the same combine kernel.
+// shuffle reductions on the CUDA cores.
+//
+// Each of the four warps streams its own blocks of 16 keys (block j of the split
+// goes to warp j mod 4) through a three-slot cp.async ring: a lane copies 16-byte
+// chunks of K and V rows (ring, window or the new row, chosen per row) and
+// stores chunk c of row r at chunk c ^ (r mod 8), so the eight rows an ldmatrix
+// phase reads sit in eight different bank groups. Rows past the split's last key
+// are zero-filled by the copy (source size 0), which keeps 0 x NaN out of P V.
+// Per block: S = Q K^T (K through ldmatrix), online softmax on the S fragments,
+// O += P V (P reused from the S registers as the A operand, V through
+// ldmatrix.trans). The warps' partials are merged per query head and written to
+// the same workspace, for the same combine kernel, as the CUDA-core kernel's.
 // ---------------------------------------------------------------------------
-constexpr int kMmaStageRows = 64;            // 16 keys per consumer warp
-constexpr int kMmaStages = 3;
+constexpr int kMmaBlockKeys = 16;            // keys per warp block (the MMA's N = 2 x 8)
+constexpr int kMmaSlots = 3;                 // cp.async slots per warp
 
 template <int D>
-constexpr int mma_row_stride() { return D * 2; }
+constexpr int mma_slot_bytes() { return 2 * kMmaBlockKeys * D * 2; }    // K and V rows of one block
 template <int D, int QG>
 constexpr int decode_mma_smem_bytes() {
-    return 2 * kMmaStages * kMmaStageRows * mma_row_stride<D>() + 2 * kMmaStages * 8 +
-           QG * (kDecodeThreads / 32) * (2 + D) * 4;
+    constexpr int stages = (kDecodeThreads / 32) * kMmaSlots * mma_slot_bytes<D>();
+    constexpr int merge = QG * (kDecodeThreads / 32) * (2 + D) * 4;     // reuses the stage bytes
+    return stages > merge ? stages : merge;
 }
 
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
@@ -334,9 +342,23 @@ __device__ __forceinline__ void mma_16816(float* c, uint32_t a0, uint32_t a1, ui
         : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
+// 16-byte global -> shared copy; src_bytes = 0 stores zeros and reads nothing
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+
+// byte offset of 16-byte chunk `chunk` of row `row` in a swizzled block
+template <int D>
+__device__ __forceinline__ uint32_t swz(int row, int chunk) {
+    return (uint32_t)(row * (D * 2) + ((chunk ^ (row & 7)) << 4));
+}
 
 template <int D, int QG>
-__global__ void __launch_bounds__(kDecodeThreads + 32) decode_split_mma_kernel(
+__global__ void __launch_bounds__(kDecodeThreads) decode_split_mma_kernel(
         const uint8_t* __restrict__ ring_k, const uint8_t* __restrict__ ring_v, uint4* __restrict__ win_k,
         uint4* __restrict__ win_v, const int32_t* __restrict__ ring_len, const int32_t* __restrict__ win_fill,
         const int32_t* __restrict__ win_idx, const int32_t* __restrict__ ks, int32_t n_windows, int32_t W,
@@ -344,9 +366,11 @@ __global__ void __launch_bounds__(kDecodeThreads + 32) decode_split_mma_kernel(
         const uint4* __restrict__ v_new, float scale_log2, float2* __restrict__ ws_ml, float* __restrict__ ws_o,
         int32_t n_splits, int32_t* status, const int32_t* __restrict__ W_per_window, int32_t q_per_kv) {
     using namespace sm100;
-    static_assert(QG >= 2 && QG <= 8, "one query per A row, rows 0..7");
-    constexpr int CPR = D / 8, ROWB = D * 2, RS = mma_row_stride<D>(), CH = kMmaStageRows;
-    constexpr int NW = kDecodeThreads / 32;
+    static_assert(QG >= 2 && QG <= 16, "one query per A row");
+    constexpr bool HI = QG > 8;                                      // rows 8..15 hold queries too
+    constexpr int CPR = D / 8, ROWB = D * 2, NW = kDecodeThreads / 32, BK = kMmaBlockKeys;
+    constexpr int SLOT = mma_slot_bytes<D>(), HALF = SLOT / 2;       // K rows, then V rows
+    constexpr int PER_LANE = BK * CPR / 32;                          // chunks per lane per tensor
     const int slices = q_per_kv / QG;
     const int b = blockIdx.z, h = blockIdx.y / slices, slice = blockIdx.y % slices, split = blockIdx.x;
     const int64_t bh = (int64_t)b * H + h;
@@ -374,177 +398,140 @@ __global__ void __launch_bounds__(kDecodeThreads + 32) decode_split_mma_kernel(
     }
 
     extern __shared__ __align__(128) unsigned char smem[];
-    uint8_t* sK = smem;                                         // [stages][CH][RS]
-    uint8_t* sV = smem + kMmaStages * CH * RS;
-    uint64_t* full = reinterpret_cast<uint64_t*>(smem + 2 * kMmaStages * CH * RS);
-    uint64_t* empty = full + kMmaStages;
-    float* sm_m = reinterpret_cast<float*>(empty + kMmaStages);   // [NW][QG]
-    float* sm_l = sm_m + NW * QG;                                  // [NW][QG]
-    float* sm_o = sm_l + NW * QG;                                  // [NW][QG][D]
-    __shared__ int32_t abort_flag;
-    const int n_chunks = (int)((s1 - s0 + CH - 1) / CH);
+    const uint32_t my_slots = smem_addr(smem) + (uint32_t)(warp * kMmaSlots * SLOT);
+    const uint8_t* rk = ring_k + bh * (int64_t)C_ring * ROWB;
+    const uint8_t* rv = ring_v + bh * (int64_t)C_ring * ROWB;
+    const uint8_t* wk = reinterpret_cast<const uint8_t*>(win_k) + bh * (int64_t)C_win * ROWB;
+    const uint8_t* wv = reinterpret_cast<const uint8_t*>(win_v) + bh * (int64_t)C_win * ROWB;
+    const uint8_t* nk = reinterpret_cast<const uint8_t*>(k_new) + bh * ROWB;
+    const uint8_t* nv = reinterpret_cast<const uint8_t*>(v_new) + bh * ROWB;
 
-    if (tid == 0) {
-        for (int i = 0; i < kMmaStages; ++i) {
-            mbar_init(smem_addr(&full[i]), 1);
-            mbar_init(smem_addr(&empty[i]), NW);
-        }
-        abort_flag = 0;
-        fence_barrier_init();
-    }
-    __syncthreads();
-
-    if (warp == NW) {
-        // ------------------------------------------------ producer: one bulk copy per row
-        const uint8_t* rk = ring_k + bh * (int64_t)C_ring * ROWB;
-        const uint8_t* rv = ring_v + bh * (int64_t)C_ring * ROWB;
-        const uint8_t* wk = reinterpret_cast<const uint8_t*>(win_k) + bh * (int64_t)C_win * ROWB;
-        const uint8_t* wv = reinterpret_cast<const uint8_t*>(win_v) + bh * (int64_t)C_win * ROWB;
-        const uint8_t* nk = reinterpret_cast<const uint8_t*>(k_new) + bh * ROWB;
-        const uint8_t* nv = reinterpret_cast<const uint8_t*>(v_new) + bh * ROWB;
-        int issued = 0;
-        for (int c = 0; c < n_chunks; ++c) {
-            const int st = c % kMmaStages, use = c / kMmaStages;
-            bool ok = true;
-            if (lane == 0 && use > 0 && !mbar_wait(smem_addr(&empty[st]), (use - 1) & 1, kWaitNs)) ok = false;
-            if (!__all_sync(0xffffffffu, ok)) {
-                if (lane == 0) {
-                    report(status, FOCUS_ERR_TIMEOUT);
-                    atomicExch(&abort_flag, 1);
-                }
-                break;
+    const int nb = (int)((s1 - s0 + BK - 1) / BK);                    // key blocks in the split
+    const int my_nb = nb > warp ? (nb - warp + NW - 1) / NW : 0;      // this warp's: warp, warp + NW, ...
+    auto load_block = [&](int i) {                                    // the warp's i-th block into slot i % 3
+        const int64_t kb = s0 + (int64_t)(warp + i * NW) * BK;
+        const uint32_t dst = my_slots + (uint32_t)((i % kMmaSlots) * SLOT);
+#pragma unroll
+        for (int u = 0; u < PER_LANE; ++u) {
+            const int idx = u * 32 + lane, r = idx / CPR, ch = idx % CPR;
+            const int64_t key = kb + r;
+            const uint8_t *sk = nk, *sv = nv;                         // the new row (or a zero-filled one)
+            if (key < R) {
+                sk = rk + key * ROWB;
+                sv = rv + key * ROWB;
+            } else if (key < (int64_t)R + fill) {
+                sk = wk + (key - R) * ROWB;
+                sv = wv + (key - R) * ROWB;
             }
-            const int64_t k0 = s0 + (int64_t)c * CH, k1 = min(s1, k0 + CH);
-            const uint32_t bar = smem_addr(&full[st]);
-            if (lane == 0) {                                 // at most three contiguous copies per tensor
-                mbar_expect_tx(bar, (uint32_t)((k1 - k0) * ROWB * 2));
-                const uint32_t dk = smem_addr(sK + st * CH * RS), dv = smem_addr(sV + st * CH * RS);
-                int64_t a = k0, e = min(k1, (int64_t)R);                 // ring rows
-                if (a < e) {
-                    bulk_load(dk, rk + a * ROWB, (uint32_t)((e - a) * ROWB), bar);
-                    bulk_load(dv, rv + a * ROWB, (uint32_t)((e - a) * ROWB), bar);
-                }
-                a = max(k0, (int64_t)R);
-                e = min(k1, (int64_t)R + fill);                          // current-window rows
-                if (a < e) {
-                    const uint32_t off = (uint32_t)((a - k0) * ROWB);
-                    bulk_load(dk + off, wk + (a - R) * ROWB, (uint32_t)((e - a) * ROWB), bar);
-                    bulk_load(dv + off, wv + (a - R) * ROWB, (uint32_t)((e - a) * ROWB), bar);
-                }
-                if (k1 == total) {                                        // the new row itself
-                    const uint32_t off = (uint32_t)((total - 1 - k0) * ROWB);
-                    bulk_load(dk + off, nk, ROWB, bar);
-                    bulk_load(dv + off, nv, ROWB, bar);
-                }
-            }
-            __syncwarp();
-            issued = c + 1;
+            const uint32_t n = key < s1 ? 16u : 0u;
+            cp_async16(dst + swz<D>(r, ch), sk + ch * 16, n);
+            cp_async16(dst + HALF + swz<D>(r, ch), sv + ch * 16, n);
         }
-        if (lane == 0)                                               // drain before exit
-            for (int c = max(0, issued - kMmaStages); c < issued; ++c)
-                mbar_wait(smem_addr(&full[c % kMmaStages]), (c / kMmaStages) & 1, kWaitNs);
-        __syncthreads();
-        return;
+    };
+#pragma unroll
+    for (int i = 0; i < kMmaSlots - 1; ++i) {
+        if (i < my_nb) load_block(i);
+        cp_async_commit();
     }
 
-    // ---------------------------------------------------- consumers
-    const int g = lane >> 2, t4 = lane & 3;                 // fragment row (query) and column pair
-    // Q as A fragments: rows g < QG hold the CTA's query heads, rows 8..15 are zero
-    uint32_t qa[D / 16][2];
+    const int g = lane >> 2, t4 = lane & 3;                 // fragment rows g, g + 8 and column pair
+    // Q as A fragments: rows below QG hold the CTA's query heads, the rest are zero
+    uint32_t qa[D / 16][4];
 #pragma unroll
     for (int kk = 0; kk < D / 16; ++kk) {
-        const bool row = g < QG;
-        const int64_t qw = (bhq0 + (row ? g : 0)) * (D / 2) + kk * 8 + t4;   // 32-bit words of q
-        qa[kk][0] = row ? q[qw] : 0u;
-        qa[kk][1] = row ? q[qw + 4] : 0u;
+#pragma unroll
+        for (int hr = 0; hr < 2; ++hr) {
+            const int row = g + 8 * hr;
+            const bool live = row < QG;
+            const int64_t qw = (bhq0 + (live ? row : 0)) * (D / 2) + kk * 8 + t4;   // 32-bit words of q
+            qa[kk][hr] = live ? q[qw] : 0u;
+            qa[kk][2 + hr] = live ? q[qw + 4] : 0u;
+        }
     }
-    float m = -INFINITY, l = 0.f;
+    float m[2] = {-INFINITY, -INFINITY}, l[2] = {0.f, 0.f};   // rows g and g + 8
     float oacc[D / 8][4];
 #pragma unroll
     for (int i = 0; i < D / 8; ++i) oacc[i][0] = oacc[i][1] = oacc[i][2] = oacc[i][3] = 0.f;
+    const int mi = lane >> 3;
 
-    for (int c = 0; c < n_chunks; ++c) {
-        const int st = c % kMmaStages;
-        if (!mbar_wait(smem_addr(&full[st]), (c / kMmaStages) & 1, kWaitNs) || abort_flag) {
-            report(status, FOCUS_ERR_TIMEOUT);
-            break;
-        }
-        const int nrow = (int)min((int64_t)CH, s1 - (s0 + (int64_t)c * CH));
-        const int key0 = warp * 16;                          // this warp's 16 keys of the stage
-        if (key0 < nrow) {
-            const uint8_t* cK = sK + st * CH * RS;
-            uint8_t* cV = sV + st * CH * RS;
-            if (key0 + 16 > nrow) {
-                // the split's last, partial stage: rows past the keys were never
-                // written; their P is 0, but 0 x NaN is not, so zero this warp's
-                // unused V rows (the stage is not refilled after the last chunk)
-                const int nz = key0 + 16 - nrow;
-                for (int i = lane; i < nz * CPR; i += 32)
-                    *reinterpret_cast<uint4*>(cV + (nrow + i / CPR) * RS + (i % CPR) * 16) = make_uint4(0, 0, 0, 0);
-                __syncwarp();
-            }
-            float sacc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-            const int mi = lane >> 3;
+    for (int i = 0; i < my_nb; ++i) {
+        if (i + kMmaSlots - 1 < my_nb) load_block(i + kMmaSlots - 1);   // into the slot read at i - 1
+        cp_async_commit();
+        cp_async_wait<kMmaSlots - 1>();                                  // block i has landed
+        __syncwarp();
+        const uint32_t cK = my_slots + (uint32_t)((i % kMmaSlots) * SLOT), cV = cK + HALF;
+        const int nrow = (int)min((int64_t)BK, s1 - (s0 + (int64_t)(warp + i * NW) * BK));
+        float sacc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
 #pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-                const int key = key0 + (mi >> 1) * 8 + (lane & 7);
-                const int chunk = kk * 2 + (mi & 1);
-                uint32_t r0, r1, r2, r3;
-                ldsm_x4(smem_addr(cK + key * RS + chunk * 16), r0, r1, r2, r3);
-                mma_16816(sacc[0], qa[kk][0], 0u, qa[kk][1], 0u, r0, r1);
-                mma_16816(sacc[1], qa[kk][0], 0u, qa[kk][1], 0u, r2, r3);
-            }
-            // online softmax on row g (columns 2 t4, 2 t4 + 1 of each 8-key block)
+        for (int kk = 0; kk < D / 16; ++kk) {
+            const int key = (mi >> 1) * 8 + (lane & 7);
+            uint32_t r0, r1, r2, r3;
+            ldsm_x4(cK + swz<D>(key, kk * 2 + (mi & 1)), r0, r1, r2, r3);
+            mma_16816(sacc[0], qa[kk][0], qa[kk][1], qa[kk][2], qa[kk][3], r0, r1);
+            mma_16816(sacc[1], qa[kk][0], qa[kk][1], qa[kk][2], qa[kk][3], r2, r3);
+        }
+        // online softmax on rows g (accumulators 0, 1) and g + 8 (2, 3), columns
+        // 2 t4 and 2 t4 + 1 of each 8-key half
+        uint32_t pa[4] = {0u, 0u, 0u, 0u};                   // P as the A operand of P V
+#pragma unroll
+        for (int hr = 0; hr < (HI ? 2 : 1); ++hr) {
             float sv[4];
 #pragma unroll
             for (int n = 0; n < 2; ++n)
 #pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    const int key = key0 + n * 8 + 2 * t4 + e;
-                    sv[n * 2 + e] = key < nrow ? sacc[n][e] * scale_log2 : -INFINITY;
-                }
+                for (int e = 0; e < 2; ++e)
+                    sv[n * 2 + e] = n * 8 + 2 * t4 + e < nrow ? sacc[n][2 * hr + e] * scale_log2 : -INFINITY;
             float mx = fmaxf(fmaxf(sv[0], sv[1]), fmaxf(sv[2], sv[3]));
             mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
             mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-            const float mn = fmaxf(m, mx);
-            const float corr = ex2_approx(m - mn);               // 0 when m was -inf
-            l *= corr;
+            const float mn = fmaxf(m[hr], mx);
+            const float corr = ex2_approx(m[hr] - mn);       // 0 when m was -inf
+            l[hr] *= corr;
 #pragma unroll
-            for (int i = 0; i < D / 8; ++i) { oacc[i][0] *= corr; oacc[i][1] *= corr; }
-            m = mn;
+            for (int d8 = 0; d8 < D / 8; ++d8) { oacc[d8][2 * hr] *= corr; oacc[d8][2 * hr + 1] *= corr; }
+            m[hr] = mn;
             float p[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
-                p[e] = ex2_approx(sv[e] - m);
-                l += p[e];
+                p[e] = ex2_approx(sv[e] - mn);
+                l[hr] += p[e];
             }
-            const uint32_t pa0 = pack_bf16x2(p[0], p[1]), pa2 = pack_bf16x2(p[2], p[3]);
-#pragma unroll
-            for (int dp = 0; dp < D / 16; ++dp) {
-                const int key = key0 + (mi & 1) * 8 + (lane & 7);
-                const int chunk = 2 * dp + (mi >> 1);
-                uint32_t r0, r1, r2, r3;
-                ldsm_x4_t(smem_addr(cV + key * RS + chunk * 16), r0, r1, r2, r3);
-                mma_16816(oacc[2 * dp], pa0, 0u, pa2, 0u, r0, r1);
-                mma_16816(oacc[2 * dp + 1], pa0, 0u, pa2, 0u, r2, r3);
-            }
+            pa[hr] = pack_bf16x2(p[0], p[1]);
+            pa[2 + hr] = pack_bf16x2(p[2], p[3]);
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(smem_addr(&empty[st]));
+#pragma unroll
+        for (int dp = 0; dp < D / 16; ++dp) {
+            const int key = (mi & 1) * 8 + (lane & 7);
+            uint32_t r0, r1, r2, r3;
+            ldsm_x4_t(cV + swz<D>(key, 2 * dp + (mi >> 1)), r0, r1, r2, r3);
+            mma_16816(oacc[2 * dp], pa[0], pa[1], pa[2], pa[3], r0, r1);
+            mma_16816(oacc[2 * dp + 1], pa[0], pa[1], pa[2], pa[3], r2, r3);
+        }
+        __syncwarp();                                        // slot i % 3 is refilled at i + 1
     }
+    cp_async_wait<0>();
 
-    // ---- merge the four warps' partials per query head -----------------------
-    l += __shfl_xor_sync(0xffffffffu, l, 1);
-    l += __shfl_xor_sync(0xffffffffu, l, 2);
-    if (g < QG) {
-        if (t4 == 0) { sm_m[warp * QG + g] = m; sm_l[warp * QG + g] = l; }
+    // ---- merge the four warps' partials per query head (in the stage bytes) --
+    __syncthreads();
+    float* sm_m = reinterpret_cast<float*>(smem);          // [NW][QG]
+    float* sm_l = sm_m + NW * QG;                           // [NW][QG]
+    float* sm_o = sm_l + NW * QG;                           // [NW][QG][D]
 #pragma unroll
-        for (int i = 0; i < D / 8; ++i) {
-            sm_o[(warp * QG + g) * D + i * 8 + 2 * t4] = oacc[i][0];
-            sm_o[(warp * QG + g) * D + i * 8 + 2 * t4 + 1] = oacc[i][1];
+    for (int hr = 0; hr < 2; ++hr) {
+        const int row = g + 8 * hr;
+        float lr = l[hr];
+        lr += __shfl_xor_sync(0xffffffffu, lr, 1);
+        lr += __shfl_xor_sync(0xffffffffu, lr, 2);
+        if (row < QG) {
+            if (t4 == 0) { sm_m[warp * QG + row] = m[hr]; sm_l[warp * QG + row] = lr; }
+#pragma unroll
+            for (int d8 = 0; d8 < D / 8; ++d8) {
+                sm_o[(warp * QG + row) * D + d8 * 8 + 2 * t4] = oacc[d8][2 * hr];
+                sm_o[(warp * QG + row) * D + d8 * 8 + 2 * t4 + 1] = oacc[d8][2 * hr + 1];
+            }
         }
     }
-    asm volatile("bar.sync 1, %0;" ::"n"(kDecodeThreads));       // consumers only
+    __syncthreads();
     for (int col = tid; col < QG * D; col += kDecodeThreads) {
         const int j = col / D, cc = col % D;
         float M = -INFINITY;
@@ -562,7 +549,6 @@ __global__ void __launch_bounds__(kDecodeThreads + 32) decode_split_mma_kernel(
         ws_o[((bhq0 + j) * n_splits + split) * D + cc] = A;
         if (cc == 0) ws_ml[(bhq0 + j) * n_splits + split] = make_float2(M, L);
     }
-    __syncthreads();
 }
 
 template <int D>
@@ -656,7 +642,7 @@ cudaError_t launch_decode_split_mma(const focus_cache& c, int32_t ns, const void
     cudaError_t e0 = cudaFuncSetAttribute(decode_split_mma_kernel<D, QG>,
                                           cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e0 != cudaSuccess) return e0;
-    decode_split_mma_kernel<D, QG><<<dim3(ns, c.H * (g / QG), c.B), kDecodeThreads + 32, smem, stream>>>(
+    decode_split_mma_kernel<D, QG><<<dim3(ns, c.H * (g / QG), c.B), kDecodeThreads, smem, stream>>>(
         (const uint8_t*)c.ring_k, (const uint8_t*)c.ring_v, (uint4*)c.win_k, (uint4*)c.win_v, c.ring_len,
         c.win_fill, c.win_idx, c.k_per_window, c.n_windows, c.W, c.H, c.C_ring, c.C_win, (const uint32_t*)q,
         (const uint4*)k_new, (const uint4*)v_new, scale * 1.4426950408889634f, ws_ml, ws_o, ns, status,
@@ -686,10 +672,11 @@ cudaError_t launch_decode_d(const focus_cache& c, const void* q, const void* k_n
         q = q_rot;
         k_new = k_rot;
     }
-    // grouped heads go to the tensor-core kernel (up to eight query heads per K/V
-    // pass); one query head per K/V head, or an odd group, to the CUDA-core one
+    // grouped heads go to the tensor-core kernel (up to sixteen query heads per
+    // K/V pass); one query head per K/V head, or an odd group, to the CUDA-core one
     cudaError_t e =
-        (g % 8 == 0)   ? launch_decode_split_mma<D, 8>(c, ns, q, k_new, v_new, scale, ws_ml, ws_o, status, stream)
+        (g % 16 == 0)  ? launch_decode_split_mma<D, 16>(c, ns, q, k_new, v_new, scale, ws_ml, ws_o, status, stream)
+        : (g % 8 == 0) ? launch_decode_split_mma<D, 8>(c, ns, q, k_new, v_new, scale, ws_ml, ws_o, status, stream)
         : (g % 4 == 0) ? launch_decode_split_mma<D, 4>(c, ns, q, k_new, v_new, scale, ws_ml, ws_o, status, stream)
         : (g % 2 == 0) ? launch_decode_split_mma<D, 2>(c, ns, q, k_new, v_new, scale, ws_ml, ws_o, status, stream)
                        : launch_decode_split<D, 1>(c, ns, q, k_new, v_new, scale, ws_ml, ws_o, status, stream);

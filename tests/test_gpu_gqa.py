@@ -141,3 +141,32 @@ def test_gqa_rejects_mismatched_heads():
     q = torch.zeros((1, 2, L["T"], 64), dtype=torch.bfloat16, device="cuda")   # needs 8 query heads
     with pytest.raises(ValueError):
         focus.attn_prefill(cache, q, q, q, L)
+
+
+@pytest.mark.parametrize("g,d", [(2, 64), (8, 128), (16, 64), (16, 128)])
+def test_gqa_decode_multi_split_matches_oracle(g, d):
+    """Several 1,024-key splits per head with ragged tails: ring lengths 2,900 and
+    1,025 (one key into the second split), window fills 3 and 0. Each query head
+    group is served per K/V pass (g = 16 as two slices of eight)."""
+    B, H, W, kw = 2, 2, 50, 10
+    cache = focus.Cache(B, H, d, C_ring=3_000, C_win=64, W=W, k_sched=np.full(400, kw, np.int32), q_per_kv=g)
+    gen = torch.Generator(device="cuda").manual_seed(23)
+    for t in (cache.ring_k, cache.ring_v, cache.win_k, cache.win_v):
+        t.copy_(torch.randn(t.shape, generator=gen, device="cuda").bfloat16())
+    R, fill = np.array([2_900, 1_025], np.int32), np.array([3, 0], np.int32)
+    cache.ring_len.copy_(torch.from_numpy(R))
+    cache.win_idx.copy_(torch.tensor([7, 3], dtype=torch.int32))
+    cache.win_fill.copy_(torch.from_numpy(fill))
+    rk, rv, wk, wv = (bits(t).copy() for t in (cache.ring_k, cache.ring_v, cache.win_k, cache.win_v))
+    Hq = H * g
+    q = inputs.normal_bf16((B, Hq, d), 1.0, seed=41, device="cuda")
+    kn, vn = (inputs.normal_bf16((B, H, d), 1.0, seed=s, device="cuda") for s in (42, 43))
+    o, lse = focus.attn_decode(cache, q, kn, vn)
+    qb, kb, vb = bits(q), bits(kn), bits(vn)
+    o_ref, lse_ref = np.zeros((B, Hq, d)), np.zeros((B, Hq))
+    e = np.arange(Hq) // g
+    for b in range(B):
+        o_ref[b], lse_ref[b] = fo.decode(qb[b], kb[b][e], vb[b][e], rk[b][e], rv[b][e], [R[b]] * Hq,
+                                         wk[b][e], wv[b][e], [fill[b]] * Hq, 1 / math.sqrt(d))
+    assert_attn_close(o, lse, o_ref, lse_ref, f"gqa decode multi-split g={g} d={d}")
+    assert np.array_equal(cache.win_fill.cpu().numpy(), fill + 1)
