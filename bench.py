@@ -78,6 +78,16 @@ def kmer_local_row_counts(win_off, ring_off, k_sched):
     return a - c * kdiv + 1 + c + bnd
 
 
+def decode_traffic(args):
+    """Committed DRAM bytes per decode call for the batch-64 decode workload: the
+    CUDA-core kernel at one query head per K/V head, the tensor-core kernel at
+    eight (the two configurations with counters); None otherwise."""
+    if args.decode_workload != "decode_1mb_b64_h32_d128" or args.rope:
+        return None
+    key = {1: "decode_split", 8: "decode_split_mma_g8"}.get(args.q_per_kv)
+    return kernel_traffic(key, "paper_2511_14694_gb300/csrc/decode.cu") if key else None
+
+
 def kernel_traffic(kernel_key: str, source: str):
     """DRAM bytes per launch from a committed ncu summary, only while the kernel
     source is unchanged since the counters were taken (else None)."""
@@ -629,8 +639,7 @@ def run_focus(args, world, rank, local):
                          "frac": gbs / peaks["hbm_gbs"], "frac_of_nominal": gbs / NOMINAL_HBM_GBS,
                          "peak_source": f"{peaks_src} copy bandwidth", "bytes_per_step": dec["bytes_leg"] / dec["steps"],
                          "avg_decode_call_ms": dec["decode_kernels_ms"] / dec["steps"],
-                         "traffic": (kernel_traffic("decode_split", "paper_2511_14694_gb300/csrc/decode.cu")
-                                     if args.decode_workload == "decode_1mb_b64_h32_d128" else None)},
+                         "traffic": decode_traffic(args)},
             "clocks": dec["clocks"],
         }
         line["decode"]["gpu_launches"] = dec["launches"]
