@@ -90,16 +90,20 @@ def decode_traffic(args):
 
 def kernel_traffic(kernel_key: str, source: str):
     """DRAM bytes per launch from a committed ncu summary, only while the kernel
-    source is unchanged since the counters were taken (else None)."""
+    source (and the prefill kernels' shared header) is unchanged since the
+    counters were taken (else None)."""
     p = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(p) as f:
             d = json.load(f)[kernel_key]
         if d.get("source") != source:
             return None
-        with open(os.path.join(ROOT, source), "rb") as f:
-            sha = hashlib.sha256(f.read()).hexdigest()[:16]
-        return float(d["bytes_per_launch"]) if d.get("source_sha") == sha else None
+        # the kernel's own source and the headers it shares with no other kernel
+        for path, want in [(source, d.get("source_sha"))] + sorted(d.get("deps", {}).items()):
+            with open(os.path.join(ROOT, path), "rb") as f:
+                if hashlib.sha256(f.read()).hexdigest()[:16] != want:
+                    return None
+        return float(d["bytes_per_launch"])
     except Exception:
         return None
 
@@ -290,6 +294,7 @@ def run_prefill_leg(args, cfg, world, rank, local):
     o = torch.empty_like(q)
     lse = torch.empty((B, H, L["T"]), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
+    kernel_name = focus.prefill_kernel(cache, q, k, v, L, flags=args.prefill_flags, o=o)
 
     def front(evc=None):
         focus.layout_run(L, nt, stream=stream)
@@ -390,7 +395,8 @@ def run_prefill_leg(args, cfg, world, rank, local):
         host_sample = dict(win_off=win_off, ring_off=ring_off, kind=L["kind"].cpu().numpy(),
                            win=L["win"].cpu().numpy(), keep=L["keep"].cpu().numpy(), k_sched=k_s,
                            q=q[0, :2].cpu(), k=k[0, :2].cpu(), v=v[0, :2].cpu())
-    res = dict(step_ms=step_ms, attn_ms=attn_ms, flops_per_step=flops_per_step, pairs=pairs, T=L["T"], R=L["R"],
+    res = dict(kernel=kernel_name,
+               step_ms=step_ms, attn_ms=attn_ms, flops_per_step=flops_per_step, pairs=pairs, T=L["T"], R=L["R"],
                bytes_per_step=bytes_per_step, local_mask=local_mask, compact_ms=compact_ms,
                compact_bytes=compact_bytes,
                clocks=clk.summary(), launches=launches, e2e=e2e, host_sample=host_sample, extra_steps=extra)
@@ -429,6 +435,7 @@ def run_stream_leg(args, cfg, world, rank, local):
     lses = [torch.empty((B, H, Tw), dtype=torch.float32, device=dev) for _ in range(2)]
     stream = torch.cuda.current_stream(dev)
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(M)]
+    kernel_name = focus.prefill_kernel(cache, pq[0], pk[0], pv[0], L, M - 1, M, flags=args.prefill_flags, o=outs[0])
 
     def step(timed=False):
         for w in range(M):
@@ -463,7 +470,8 @@ def run_stream_leg(args, cfg, world, rank, local):
     barrier(world)
     assert focus.device_status(clear=True) == 0
     step_ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, world)
-    return dict(step_ms=step_ms, attn_ms=attn_ms / args.steps, flops_per_step=4.0 * d * H * B * pairs, pairs=pairs,
+    return dict(kernel=kernel_name,
+                step_ms=step_ms, attn_ms=attn_ms / args.steps, flops_per_step=4.0 * d * H * B * pairs, pairs=pairs,
                 T=L["T"], R=L["R"], clocks=clk.summary(), launches=2 * M * args.steps, e2e=None, host_sample=None,
                 per_launch_ms=attn_ms / args.steps / M, local_mask=local_mask,
                 bytes_per_step=float(B * L["T"] * (H * (4 * d + 4) + (H // g) * 4 * d)))
@@ -572,11 +580,15 @@ def run_focus(args, world, rank, local):
     value = weak_scaling_value(cfg["B"] * cfg["N"], world, pre["step_ms"] / 1e3)
     achieved = pre["flops_per_step"] / (pre["attn_ms"] / 1e3) / 1e12
     local_mask = pre.get("local_mask", False)
-    traffic = None if (args.legacy or args.rope) else kernel_traffic(
-        "prefill_attention_kmer_local" if local_mask else "prefill_attention",
-        "paper_2511_14694_gb300/csrc/prefill_tc.cu")
-    if traffic is not None and cfg is not WORKLOADS["prefill_128kb_h32_d128"]:
-        traffic = None            # the committed counters are for the 128 kb workload only
+    # committed DRAM counters exist for the 128 kb workload's appendix-mask kernel
+    # (persistent) and k-mer-local kernel (one CTA per item), default heads
+    traffic_key = {("tcgen05 persistent", False): ("prefill_attention", "prefill_tc_persistent.cu"),
+                   ("tcgen05, one CTA per work item", True): ("prefill_attention_kmer_local", "prefill_tc.cu")
+                   }.get((pre["kernel"], local_mask))
+    traffic = None
+    if (traffic_key and not args.rope and args.q_per_kv == 1
+            and cfg is WORKLOADS["prefill_128kb_h32_d128"]):
+        traffic = kernel_traffic(traffic_key[0], "paper_2511_14694_gb300/csrc/" + traffic_key[1])
     line = {
         "metric": METRIC,
         "value": value, "unit": "nt/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
@@ -591,7 +603,7 @@ def run_focus(args, world, rank, local):
                        cfg.get("pool", 0), 3 * cfg.get("pool", 0) * cfg["B"] * cfg["H"] * (pre["T"] // max(1, -(-cfg["N"] // cfg["W"]))) * cfg["d"] * 2 / 1e9,
                        2 * cfg["B"] * cfg["H"] * pre["R"] * cfg["d"] * 2 / 1e9) if cfg["mode"] == "stream" else
                           "inputs larger than L2 (Q/K/V %.2f GB per step)" % (3 * cfg["B"] * pre["T"] * cfg["H"] * cfg["d"] * 2 / 1e9)),
-                   "prefill_kernel": "legacy mma.sync" if args.prefill_flags & 1 else "default",
+                   "prefill_kernel": pre["kernel"],
                    "mask": "k-mer-local (Sec. 3.2)" if local_mask else "appendix (App. A, Eq. focus-attn)",
                    "rope_theta": args.rope or None,
                    "q_per_kv": args.q_per_kv},

@@ -234,6 +234,23 @@ typedef struct focus_prefill_args {
 focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_args* args,
                                 cudaStream_t stream);
 
+/* Which kernel focus_attn_prefill launches for these arguments. Host only: no
+ * device work, no CUDA call; the arguments are checked as focus_attn_prefill
+ * checks them (same return codes). *kernel receives
+ *   FOCUS_PREFILL_KERNEL_LEGACY      the mma.sync kernel (FOCUS_PREFILL_LEGACY_MMA),
+ *   FOCUS_PREFILL_KERNEL_PERSISTENT  the tcgen05 kernel with one CTA per SM walking
+ *                                    the work items (two 128-row Q tiles of a window
+ *                                    each): appendix mask, no rotary embedding, and
+ *                                    cache->C_ring + args->max_rows <= 4096 (short
+ *                                    items, whose start-up and epilogue it overlaps),
+ *   FOCUS_PREFILL_KERNEL_PER_ITEM    the tcgen05 kernel with one CTA per work item
+ *                                    (every other case).
+ * Both tcgen05 kernels compute the same rows (within rounding order). */
+#define FOCUS_PREFILL_KERNEL_LEGACY 0
+#define FOCUS_PREFILL_KERNEL_PER_ITEM 1
+#define FOCUS_PREFILL_KERNEL_PERSISTENT 2
+focus_status focus_prefill_kernel(const focus_cache* cache, const focus_prefill_args* args, int32_t* kernel);
+
 /* ------------------------------------------------------------------------ */
 /* focus_attn_decode — one new token per sequence against the compressed    */
 /* cache (App. A.2; decoding keeps the base decoder's interface).           */

@@ -183,7 +183,7 @@ focus_status focus_layout_sched(int64_t n_nt, int32_t n_windows, const int32_t* 
     return layout_impl(n_nt, 0, true, d_W, n_windows, d_k, flags, tail, B, d_nt, out, stream);
 }
 
-focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_args* a, cudaStream_t stream) {
+static focus_status check_prefill(const focus_cache* cache, const focus_prefill_args* a) {
     focus_status s = check_cache(cache, false);
     if (s != FOCUS_OK) return s;
     if (!a || !a->q || !a->k || !a->v || !a->o || !a->d_win_off || !a->d_ring_off) return FOCUS_ERR_INVALID_ARG;
@@ -199,6 +199,20 @@ focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_ar
         if (cache->tail != 0) return FOCUS_ERR_UNSUPPORTED;
         if (!cache->k_per_window || cache->n_windows < a->w_end) return FOCUS_ERR_INVALID_ARG;
     }
+    return FOCUS_OK;
+}
+
+focus_status focus_prefill_kernel(const focus_cache* cache, const focus_prefill_args* a, int32_t* kernel) {
+    if (!kernel) return FOCUS_ERR_INVALID_ARG;
+    focus_status s = check_prefill(cache, a);
+    if (s != FOCUS_OK) return s;
+    *kernel = focus::prefill_kernel_choice(*cache, *a);
+    return FOCUS_OK;
+}
+
+focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_args* a, cudaStream_t stream) {
+    focus_status s = check_prefill(cache, a);
+    if (s != FOCUS_OK) return s;
     if (a->T_span == 0) return FOCUS_OK;
     const int64_t tiles = focus::ceil_div64(a->max_rows, 64) * (int64_t)(a->w_end - a->w_begin);
     if (tiles > INT32_MAX) return FOCUS_ERR_UNSUPPORTED;

@@ -113,6 +113,8 @@ cudaError_t launch_decode_noalloc(const focus_cache& c, const void* q, const voi
 
 cudaError_t launch_prefill_mma(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
                                cudaStream_t stream);
+// FOCUS_PREFILL_KERNEL_* that launch_prefill_tc (or the legacy flag) selects.
+int32_t prefill_kernel_choice(const focus_cache& c, const focus_prefill_args& a);
 cudaError_t launch_prefill_tc(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
                               cudaStream_t stream);
 

@@ -39,36 +39,64 @@
 // segment) start, then the fixed per-row offsets of a host table.
 // Every mbarrier wait is bounded; on timeout the kernel reports
 // FOCUS_ERR_TIMEOUT, drains its own copies/MMAs (bounded), frees TMEM, returns.
-#include <cudaTypedefs.h>
-
 #include <mutex>
 
-#include "common.cuh"
-#include "sm100.cuh"
+#include "prefill_tc_common.cuh"
 
 namespace focus {
+namespace prefill {
+
+// ---------------------------------------------------------------- tensor maps
+
 namespace {
 
-using namespace sm100;
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::mutex g_encode_mu;
 
-constexpr int BM = 128;             // rows per Q tile
-constexpr int BN = 128;             // keys per K/V tile
-constexpr int kSlots = 4;           // K/V staging slots (each holds one K or one V tile)
-constexpr int kThreads = 384;       // 12 warps
-constexpr int kBoxBytes = 128 * 128;   // one TMA box: 128 rows x 64 bf16 (128 B, swizzled)
-constexpr uint64_t kWaitNs = 2000000000ull;   // 2 s bound on any wait
-constexpr float kRescaleThreshold = 8.0f;     // log2 units: rescale O only if the max grows by > 2^8
+cudaError_t get_encode(PFN_cuTensorMapEncodeTiled_v12000* out) {
+    std::lock_guard<std::mutex> lock(g_encode_mu);
+    if (!g_encode) {
+        void* fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+        if (e != cudaSuccess) return e;
+        if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorNotSupported;
+        g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    *out = g_encode;
+    return cudaSuccess;
+}
 
-template <int D>
-struct Cfg {
-    static constexpr int kBoxes = D / 64;                       // TMA boxes per 128-row tile
-    static constexpr int kTileBytes = kBoxes * kBoxBytes;       // one Q/K/V tile
-    static constexpr int kQOff = 0;
-    static constexpr int kSlotOff = 2 * kTileBytes;
-    static constexpr int kBarOff = kSlotOff + kSlots * kTileBytes;
-    static constexpr int kRopeOff = kBarOff + 256;              // float2 [4][64] Q bases + [64] K bases
-    static constexpr int kSmem = kRopeOff + 5 * 64 * 8 + 1024;  // + alignment slack
-};
+}  // namespace
+
+// 3-D map over a [BH][rows][d] bf16 tensor, box = 128 rows x 64 columns, 128-byte swizzle.
+cudaError_t make_map(CUtensorMap* m, const void* ptr, int d, int64_t rows, int64_t bh) {
+    PFN_cuTensorMapEncodeTiled_v12000 enc;
+    cudaError_t e = get_encode(&enc);
+    if (e != cudaSuccess) return e;
+    cuuint64_t dims[3] = {(cuuint64_t)d, (cuuint64_t)rows, (cuuint64_t)bh};
+    cuuint64_t strides[2] = {(cuuint64_t)d * 2, (cuuint64_t)d * 2 * (cuuint64_t)rows};
+    cuuint32_t box[3] = {64, 128, 1};
+    cuuint32_t es[3] = {1, 1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box, es,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+}  // namespace prefill
+
+namespace {
+
+using namespace prefill;
+
+// Register split (variants without the rotary embedding): warpgroup 0 (TMA, MMA
+// and two idle warps) gives registers back, the two softmax warpgroups take
+// them: 128 x 56 + 256 x 224 = 384 x 168. With the rotary embedding warps 2-3
+// rotate K tiles and need their registers (every split tried spilled more than
+// none), so those variants keep 168 each.
+constexpr int kRegsIssue = 56, kRegsSoftmax = 224;
+static_assert(128 * kRegsIssue + 256 * kRegsSoftmax <= kThreads * kLaunchRegs, "register split over budget");
 
 // Kernel argument: the rotary table only for the ROPE variants.
 template <bool ROPE>
@@ -78,20 +106,6 @@ struct RopeArg {
 template <>
 struct RopeArg<false> {
     int unused;
-};
-
-struct Bars {
-    uint64_t q;
-    uint64_t kv_full[kSlots];
-    uint64_t kv_empty[kSlots];
-    uint64_t s_full[2];
-    uint64_t p_full[2];
-    uint64_t o_full[2];
-    uint64_t drain;
-    uint64_t q_rot;       // ROPE: the Q tiles are rotated
-    uint64_t k_rot[2];    // ROPE: the K tile in slot 0 / 2 is rotated (K tiles use the even slots)
-    uint32_t tmem;
-    int32_t abort;
 };
 
 // Rotation of eight column pairs (one 16-byte chunk and its partner d/2 columns
@@ -154,12 +168,6 @@ __device__ __forceinline__ void rope_offsets(const RopeTable& t, int i0, int g, 
     }
     step = rot8_make(st);
 }
-
-__device__ __forceinline__ void fail(Bars* bars, int32_t* status) {
-    report(status, FOCUS_ERR_TIMEOUT);
-    atomicExch(&bars->abort, 1);
-}
-__device__ __forceinline__ bool aborted(Bars* bars) { return *(volatile int32_t*)&bars->abort != 0; }
 
 // Q/O/LSE row of this CTA's query head, read afresh from the block index where
 // it is used (keeping it in a register across the softmax loop costs spills).
@@ -262,6 +270,8 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
     tc_fence_after();
     const uint32_t tmem = bars->tmem;
 
+    if (warp < 4) {
+    if constexpr (!ROPE) setmaxnreg_dec<kRegsIssue>();
     if (warp == 0) {
         // ================================================= TMA producer
         if (lane == 0) {
@@ -357,7 +367,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
             mma_commit(smem_addr(&bars->drain));
             mbar_wait(smem_addr(&bars->drain), 0, kWaitNs);
         }
-    } else if (ROPE && warp < 4) {
+    } else if (ROPE) {
         // ================================================= K rotation (warps 2-3)
         if constexpr (ROPE) {
             constexpr int HALF = D / 16, G = 64 / HALF;
@@ -403,8 +413,10 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
                 if (tau == 0) mbar_arrive(smem_addr(&bars->k_rot[slot >> 1]));
             }
         }
-    } else if (warp >= 4) {
+    }
+    } else {
         // ================================================= softmax / epilogue
+        if constexpr (!ROPE) setmaxnreg_inc<kRegsSoftmax>();
         const int t = (warp - 4) >> 2;                    // 0: warps 4-7, 1: warps 8-11
         const int quarter = warp & 3;                     // TMEM lanes this warp may access
         const int r = quarter * 32 + lane;                // row within the Q tile
@@ -499,63 +511,8 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
                 for (int c = 0; c < BN; ++c)
                     if (c > r) s[c] = -INFINITY;
             }
-            // row max: four independent chains of three-input max (depth 16, not 128)
-            float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-#pragma unroll
-            for (int c = 0; c < BN; c += 8) {
-                mx[0] = max3f(mx[0], s[c + 0], s[c + 1]);
-                mx[1] = max3f(mx[1], s[c + 2], s[c + 3]);
-                mx[2] = max3f(mx[2], s[c + 4], s[c + 5]);
-                mx[3] = max3f(mx[3], s[c + 6], s[c + 7]);
-            }
-            const float mt = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
-            const float m_new = fmaxf(m_run, mt * scale_log2);
-            const bool need = m_new > m_run + kRescaleThreshold;
-            const bool any_need = __any_sync(0xffffffffu, need);
-            const float factor = need ? ex2_approx(m_run - m_new) : 1.f;
-            if (need) m_run = m_new;
-            l_run *= factor;
-            // p = 2^(s * scale_log2 - m): packed FMA on pairs, ex2 per element, row sum in
-            // four packed partial sums (independent chains)
-            // LOCAL rows can meet tiles with no visible key before their first one:
-            // subtract 0 instead of -inf there (every p is then exactly 0)
-            const float m_sub = (LOCAL && m_run == -INFINITY) ? 0.f : m_run;
-            const uint64_t sc2 = f2_pack(scale_log2, scale_log2), nm2 = f2_pack(-m_sub, -m_sub);
-            uint64_t acc2[4] = {0, 0, 0, 0};
-#pragma unroll
-            for (int h2 = 0; h2 < 2; ++h2) {
-                uint32_t pk[32];
-#pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    float x0, x1;
-                    f2_unpack(f2_fma(f2_pack(s[h2 * 64 + 2 * i], s[h2 * 64 + 2 * i + 1]), sc2, nm2), x0, x1);
-                    const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
-                    acc2[i & 3] = f2_add(acc2[i & 3], f2_pack(p0, p1));
-                    pk[i] = pack_bf16x2(p0, p1);
-                }
-                tmem_st32(s_addr + h2 * 32, pk);
-            }
-            float lsum = 0.f;
-#pragma unroll
-            for (int a = 0; a < 4; ++a) {
-                float lo, hi;
-                f2_unpack(acc2[a], lo, hi);
-                lsum += lo + hi;
-            }
-            l_run += lsum;
-            // Lazy rescale of O_t (written by PV_t(j-1), which completed before S_t(j)
-            // was signalled; PV_t(j) waits for this thread's arrival below).
-            if (any_need && j > 0) {
-#pragma unroll
-                for (int c = 0; c < D / 32; ++c) {
-                    uint32_t orr[32];
-                    tmem_ld32(o_addr + c * 32, orr);
-                    tmem_wait_ld();
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) orr[i] = __float_as_uint(__uint_as_float(orr[i]) * factor);
-                    tmem_st32(o_addr + c * 32, orr);
-                }
-            }
+            // LOCAL rows can meet tiles with no visible key before their first one
+            softmax_tile<D, LOCAL>(s, s_addr, o_addr, scale_log2, m_run, l_run, j > 0);
             tmem_wait_st();
             tc_fence_before();
             mbar_arrive(smem_addr(&bars->p_full[t]));
@@ -611,40 +568,6 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
     }
 }
 
-// ---------------------------------------------------------------- host side
-
-PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
-std::mutex g_encode_mu;
-
-cudaError_t get_encode(PFN_cuTensorMapEncodeTiled_v12000* out) {
-    std::lock_guard<std::mutex> lock(g_encode_mu);
-    if (!g_encode) {
-        void* fn = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
-        if (e != cudaSuccess) return e;
-        if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorNotSupported;
-        g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
-    }
-    *out = g_encode;
-    return cudaSuccess;
-}
-
-// 3-D map over a [BH][rows][d] bf16 tensor, box = 128 rows x 64 columns, 128-byte swizzle.
-cudaError_t make_map(CUtensorMap* m, const void* ptr, int d, int64_t rows, int64_t bh) {
-    PFN_cuTensorMapEncodeTiled_v12000 enc;
-    cudaError_t e = get_encode(&enc);
-    if (e != cudaSuccess) return e;
-    cuuint64_t dims[3] = {(cuuint64_t)d, (cuuint64_t)rows, (cuuint64_t)bh};
-    cuuint64_t strides[2] = {(cuuint64_t)d * 2, (cuuint64_t)d * 2 * (cuuint64_t)rows};
-    cuuint32_t box[3] = {64, 128, 1};
-    cuuint32_t es[3] = {1, 1, 1};
-    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box, es,
-                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
-}
-
 template <int D, bool LOCAL, bool ROPE, bool GQA>
 cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t* status, cudaStream_t stream) {
     const int64_t BH = (int64_t)c.B * c.H;
@@ -665,6 +588,13 @@ cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t*
     e = cudaFuncSetAttribute(prefill_tc_kernel<D, LOCAL, ROPE, GQA>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              smem);
     if (e != cudaSuccess) return e;
+    if constexpr (!ROPE) {
+        // the register split needs the launch registers it was sized for: with
+        // fewer, the softmax warpgroups' setmaxnreg.inc could never be served
+        cudaFuncAttributes fa;
+        if ((e = cudaFuncGetAttributes(&fa, prefill_tc_kernel<D, LOCAL, ROPE, GQA>)) != cudaSuccess) return e;
+        if (fa.numRegs < kLaunchRegs) return cudaErrorInvalidConfiguration;
+    }
     const int ctas_pw = (a.max_rows + 2 * BM - 1) / (2 * BM);
     dim3 grid((unsigned)((a.w_end - a.w_begin) * ctas_pw * g), c.H, c.B);
     RopeArg<ROPE> rope;
@@ -693,9 +623,25 @@ cudaError_t dispatch(const focus_cache& c, const focus_prefill_args& a, int32_t*
                  : launch_d<64, false, false, GQA>(c, a, status, stream);
 }
 
+// Work items of at most kPersistentMaxRows / 128 K/V tiles (ring capacity plus the
+// longest window) spend a large share of their time in per-CTA start-up and the O
+// epilogue; the persistent kernel overlaps those with the neighbouring items.
+// Longer items keep one CTA per item: the hardware's block scheduling balances
+// them better, and that kernel's per-tile loop is ~4% faster.
+constexpr int64_t kPersistentMaxRows = 4096;
+
+int32_t prefill_kernel_choice(const focus_cache& c, const focus_prefill_args& a) {
+    if (a.flags & FOCUS_PREFILL_LEGACY_MMA) return FOCUS_PREFILL_KERNEL_LEGACY;
+    const bool local = (a.flags & FOCUS_PREFILL_KMER_LOCAL) != 0, rope = c.rope_theta > 0.f;
+    if (!local && !rope && (int64_t)c.C_ring + a.max_rows <= kPersistentMaxRows) return FOCUS_PREFILL_KERNEL_PERSISTENT;
+    return FOCUS_PREFILL_KERNEL_PER_ITEM;
+}
+
 cudaError_t launch_prefill_tc(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
                               cudaStream_t stream) {
     const bool local = (a.flags & FOCUS_PREFILL_KMER_LOCAL) != 0, rope = c.rope_theta > 0.f;
+    if (prefill_kernel_choice(c, a) == FOCUS_PREFILL_KERNEL_PERSISTENT)
+        return prefill::launch_prefill_tc_persistent(c, a, status, stream);
     if (c.q_per_kv > 1) return dispatch<true>(c, a, status, stream, local, rope);
     return dispatch<false>(c, a, status, stream, local, rope);
 }

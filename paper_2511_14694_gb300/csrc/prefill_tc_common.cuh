@@ -1,0 +1,139 @@
+// Shared by the two tcgen05 prefill kernels: prefill_tc.cu (one CTA per work
+// item of two 128-row Q tiles; every mask and the rotary embedding) and
+// prefill_tc_persistent.cu (one CTA per SM walking the work items; appendix
+// mask only). Tile geometry, shared-memory layout, barriers, the online softmax
+// of one S tile, and the TMA tensor maps.
+#pragma once
+
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+#include "sm100.cuh"
+
+namespace focus {
+namespace prefill {
+
+using namespace sm100;
+
+constexpr int BM = 128;             // rows per Q tile
+constexpr int BN = 128;             // keys per K/V tile
+constexpr int kSlots = 4;           // K/V staging slots (each holds one K or one V tile)
+constexpr int kThreads = 384;       // 12 warps
+constexpr int kLaunchRegs = 168;    // registers per thread at launch: 65,536 / 384 rounded down to 8
+constexpr int kBoxBytes = 128 * 128;   // one TMA box: 128 rows x 64 bf16 (128 B, swizzled)
+constexpr uint64_t kWaitNs = 2000000000ull;   // 2 s bound on any wait
+constexpr float kRescaleThreshold = 8.0f;     // log2 units: rescale O only if the max grows by > 2^8
+
+template <int D>
+struct Cfg {
+    static constexpr int kBoxes = D / 64;                       // TMA boxes per 128-row tile
+    static constexpr int kTileBytes = kBoxes * kBoxBytes;       // one Q/K/V tile
+    static constexpr int kQOff = 0;
+    static constexpr int kSlotOff = 2 * kTileBytes;
+    static constexpr int kBarOff = kSlotOff + kSlots * kTileBytes;
+    static constexpr int kRopeOff = kBarOff + 256;              // float2 [4][64] Q bases + [64] K bases
+    static constexpr int kSmem = kRopeOff + 5 * 64 * 8 + 1024;  // + alignment slack
+    // persistent kernel: no rotary bases; O staging of 8 warps x 32 rows x 64 B
+    static constexpr int kStageOff = kBarOff + 256;
+    static constexpr int kSmemPersistent = kStageOff + 8 * 2048 + 1024;
+};
+
+struct Bars {
+    uint64_t q;
+    uint64_t kv_full[kSlots];
+    uint64_t kv_empty[kSlots];
+    uint64_t s_full[2];
+    uint64_t p_full[2];
+    uint64_t o_full[2];
+    uint64_t drain;
+    uint64_t q_rot;       // rotary embedding: the Q tiles are rotated
+    uint64_t k_rot[2];    // rotary embedding: the K tile in slot 0 / 2 is rotated (K tiles use the even slots)
+    uint64_t o_free[2];   // persistent: the epilogue has read O_t
+    uint64_t q_free;      // persistent: every QK of the current item has completed, Q may be reloaded
+    uint32_t tmem;
+    int32_t abort;
+};
+static_assert(sizeof(Bars) <= 256, "barriers must fit their 256-byte slot");
+
+__device__ __forceinline__ void fail(Bars* bars, int32_t* status) {
+    report(status, FOCUS_ERR_TIMEOUT);
+    atomicExch(&bars->abort, 1);
+}
+__device__ __forceinline__ bool aborted(Bars* bars) { return *(volatile int32_t*)&bars->abort != 0; }
+
+// Online softmax of one S tile in the log2 domain for the row this thread owns:
+// s holds the row's BN masked scores, (m_run, l_run) the running max and sum.
+// P = 2^(s scale - m) goes back to TMEM over S as bf16 pairs (two 32-column
+// stores); when the max grows by more than 2^kRescaleThreshold for any row of the
+// warp, l and, once a PV has written it (has_o), O_t in TMEM are rescaled.
+// ZERO_FLOOR: a row whose scores have all been -inf so far subtracts 0 instead of
+// -inf, so that every p is exactly 0 (masks that can hide a whole tile of a row).
+template <int D, bool ZERO_FLOOR>
+__device__ __forceinline__ void softmax_tile(const float* s, uint32_t s_addr, uint32_t o_addr, float scale_log2,
+                                             float& m_run, float& l_run, bool has_o) {
+    // row max: four independent chains of three-input max (depth 16, not 128)
+    float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+    for (int c = 0; c < BN; c += 8) {
+        mx[0] = max3f(mx[0], s[c + 0], s[c + 1]);
+        mx[1] = max3f(mx[1], s[c + 2], s[c + 3]);
+        mx[2] = max3f(mx[2], s[c + 4], s[c + 5]);
+        mx[3] = max3f(mx[3], s[c + 6], s[c + 7]);
+    }
+    const float mt = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+    const float m_new = fmaxf(m_run, mt * scale_log2);
+    const bool need = m_new > m_run + kRescaleThreshold;
+    const bool any_need = __any_sync(0xffffffffu, need);
+    const float factor = need ? ex2_approx(m_run - m_new) : 1.f;
+    if (need) m_run = m_new;
+    l_run *= factor;
+    // p = 2^(s * scale_log2 - m): packed FMA on pairs, ex2 per element, row sum in
+    // four packed partial sums (independent chains)
+    const float m_sub = (ZERO_FLOOR && m_run == -INFINITY) ? 0.f : m_run;
+    const uint64_t sc2 = f2_pack(scale_log2, scale_log2), nm2 = f2_pack(-m_sub, -m_sub);
+    uint64_t acc2[4] = {0, 0, 0, 0};
+#pragma unroll
+    for (int h2 = 0; h2 < 2; ++h2) {
+        uint32_t pk[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+            float x0, x1;
+            f2_unpack(f2_fma(f2_pack(s[h2 * 64 + 2 * i], s[h2 * 64 + 2 * i + 1]), sc2, nm2), x0, x1);
+            const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+            acc2[i & 3] = f2_add(acc2[i & 3], f2_pack(p0, p1));
+            pk[i] = pack_bf16x2(p0, p1);
+        }
+        tmem_st32(s_addr + h2 * 32, pk);
+    }
+    float lsum = 0.f;
+#pragma unroll
+    for (int a = 0; a < 4; ++a) {
+        float lo, hi;
+        f2_unpack(acc2[a], lo, hi);
+        lsum += lo + hi;
+    }
+    l_run += lsum;
+    // Lazy rescale of O_t (written by the previous PV, which completed before this
+    // S tile was signalled; the next PV waits for this thread's arrival).
+    if (any_need && has_o) {
+#pragma unroll
+        for (int c = 0; c < D / 32; ++c) {
+            uint32_t orr[32];
+            tmem_ld32(o_addr + c * 32, orr);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) orr[i] = __float_as_uint(__uint_as_float(orr[i]) * factor);
+            tmem_st32(o_addr + c * 32, orr);
+        }
+    }
+}
+
+// 3-D map over a [BH][rows][d] bf16 tensor, box = 128 rows x 64 columns, 128-byte swizzle.
+cudaError_t make_map(CUtensorMap* m, const void* ptr, int d, int64_t rows, int64_t bh);
+
+// The persistent kernel (appendix mask, no rotary embedding).
+cudaError_t launch_prefill_tc_persistent(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
+                                         cudaStream_t stream);
+
+}  // namespace prefill
+}  // namespace focus

@@ -1,0 +1,442 @@
+// Persistent variant of the tcgen05 prefill kernel for short work items
+// (appendix mask, no rotary embedding): one CTA per SM walks the work items in
+// rounds, so that the start-up of item i+1 (its Q and first K/V loads, its first
+// QK) and the epilogue of item i overlap the other item's tiles.
+//
+// Same computation as prefill_tc.cu (Eq. focus-attn's visible set; App.
+// A.1-A.2): row a of window w attends to ring rows [0, ring_off[w]) and to window
+// rows [0, a]. Same warp roles and TMEM columns; what changes is that every
+// barrier phase runs on across items:
+//   warp 0     TMA producer: per item, Q tiles (once the previous item's last QK
+//              has completed: q_free), then K_j, V_j into the slot ring, whose
+//              slot and phase count on across items
+//   warp 1     MMA issuer: per item as in prefill_tc.cu; an item's first PV into
+//              O_t waits until the previous item's epilogue has read O_t (o_free)
+//   warps 2-3  idle
+//   warps 4-11 softmax per tile (the shared softmax_tile), then the epilogue:
+//              O_t / l to bf16 through a per-warp staging buffer (the Q buffers may
+//              already hold the next item's Q), arrive on o_free once O_t is read
+// Register split: warpgroup 0 keeps 104 registers (the item loops carry more state
+// than the one-item kernel's 56 allow without spills), the softmax warpgroups take
+// 200: 128 x 104 + 256 x 200 = 384 x 168.
+// Every mbarrier wait is bounded; on timeout the kernel reports
+// FOCUS_ERR_TIMEOUT, drains its own copies/MMAs (bounded), frees TMEM, returns.
+#include "prefill_tc_common.cuh"
+
+namespace focus {
+namespace prefill {
+namespace {
+
+constexpr int kRegsIssue = 104, kRegsSoftmax = 200;
+static_assert(128 * kRegsIssue + 256 * kRegsSoftmax <= kThreads * kLaunchRegs, "register split over budget");
+
+// Geometry of one work item: two 128-row Q tiles of one (sequence, head,
+// window). Items are numbered head by head (sequences, then K/V heads, outermost;
+// within a head the windows longest first, each window's Q-tile pairs longest
+// first, and with GQA the query heads of a group innermost): the CTAs working
+// at the same time then share one head's K/V tiles in L2.
+struct ItemGeom {
+    int32_t w, cta, member, bh, Tw, a0, Rw, row_base;
+    int32_t n_ring, n_kv0, n_kv1, n_kv_max;
+    bool valid, cap_err;
+};
+
+template <bool GQA>
+__device__ __forceinline__ ItemGeom item_geom(int64_t idx, int32_t per_head, int32_t ctas_pw, int32_t q_per_kv,
+                                              int32_t H, const int32_t* __restrict__ win_off,
+                                              const int32_t* __restrict__ ring_off, int32_t w_begin,
+                                              int32_t w_end, int32_t C_ring, int64_t T_span) {
+    ItemGeom I;
+    // per_head: items of one K/V head = windows x pairs (x query heads per group)
+    const uint32_t x = (uint32_t)(idx % per_head);
+    const int64_t rest = idx / per_head;
+    const int32_t h = (int32_t)(rest % H), b = (int32_t)(rest / H);
+    const uint32_t item = GQA ? x / (uint32_t)q_per_kv : x;
+    I.member = GQA ? (int32_t)(x % (uint32_t)q_per_kv) : 0;
+    const int32_t wi = item / ctas_pw;
+    I.cta = ctas_pw - 1 - (int32_t)(item % ctas_pw);
+    I.w = w_end - 1 - wi;
+    I.bh = b * H + h;
+    const int32_t w0 = win_off[w_begin];
+    const int32_t w_first = win_off[I.w];
+    I.Tw = win_off[I.w + 1] - w_first;
+    I.a0 = I.cta * 2 * BM;
+    I.valid = I.a0 < I.Tw;
+    I.cap_err = false;
+    I.Rw = ring_off[I.w];
+    I.n_ring = (I.Rw + BN - 1) / BN;
+    if (I.valid && (I.Rw > C_ring || (int64_t)(win_off[w_end] - w0) > T_span)) {
+        I.cap_err = true;
+        I.valid = false;
+    }
+    I.row_base = w_first - w0;                          // first row of the window in the span tensors
+    const bool valid1 = I.a0 + BM < I.Tw;
+    I.n_kv0 = I.n_ring + 2 * I.cta + 1;
+    I.n_kv1 = valid1 ? I.n_ring + 2 * I.cta + 2 : 0;
+    I.n_kv_max = valid1 ? I.n_kv1 : I.n_kv0;
+    return I;
+}
+
+template <int D, bool GQA>
+__global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
+        const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+        const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_rk,
+        const __grid_constant__ CUtensorMap tm_rv, __nv_bfloat16* __restrict__ o, float* __restrict__ lse,
+        int64_t T_span, const int32_t* __restrict__ win_off, const int32_t* __restrict__ ring_off, int32_t w_begin,
+        int32_t w_end, int32_t ctas_pw, int32_t H, int32_t C_ring, float scale_log2, int32_t* status,
+        int32_t q_per_kv, int64_t n_items) {
+    using C = Cfg<D>;
+    extern __shared__ unsigned char smem_raw[];
+    uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    Bars* bars = reinterpret_cast<Bars*>(smem + C::kBarOff);
+    // Once any CTA has given up on a wait, CTAs that start later skip their work so
+    // that a systematic stall costs one round of bounded waits.
+    if (*(volatile int32_t*)status == FOCUS_ERR_TIMEOUT) return;
+    const int32_t per_head = (w_end - w_begin) * ctas_pw * (GQA ? q_per_kv : 1);
+    auto geom = [&](int64_t idx) {
+        return item_geom<GQA>(idx, per_head, ctas_pw, q_per_kv, H, win_off, ring_off, w_begin, w_end, C_ring, T_span);
+    };
+    // round k of a CTA: positions k G .. k G + G - 1 of the longest-first order, in
+    // snake order (forward on even rounds, backward on odd) to balance the CTAs
+    auto snake_item = [&](int64_t k) {
+        return k * (int64_t)gridDim.x + ((k & 1) ? (int64_t)(gridDim.x - 1 - blockIdx.x) : (int64_t)blockIdx.x);
+    };
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    // ---- setup (once per CTA) -------------------------------------------------
+    if (threadIdx.x == 0) {
+        mbar_init(smem_addr(&bars->q), 1);
+        mbar_init(smem_addr(&bars->q_free), 1);
+        for (int s = 0; s < kSlots; ++s) {
+            mbar_init(smem_addr(&bars->kv_full[s]), 1);
+            mbar_init(smem_addr(&bars->kv_empty[s]), 1);
+        }
+        for (int t = 0; t < 2; ++t) {
+            mbar_init(smem_addr(&bars->s_full[t]), 1);
+            mbar_init(smem_addr(&bars->p_full[t]), BM);
+            mbar_init(smem_addr(&bars->o_full[t]), 1);
+            mbar_init(smem_addr(&bars->o_free[t]), BM);
+        }
+        mbar_init(smem_addr(&bars->drain), 1);
+        bars->abort = 0;
+        fence_barrier_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_addr(&bars->tmem), 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = bars->tmem;
+
+    if (warp < 4) {
+        setmaxnreg_dec<kRegsIssue>();
+        if (warp == 0 && lane == 0) {
+            // ============================================= TMA producer
+            prefetch_tmap(&tm_q);
+            prefetch_tmap(&tm_k);
+            prefetch_tmap(&tm_v);
+            prefetch_tmap(&tm_rk);
+            prefetch_tmap(&tm_rv);
+            const uint32_t bq = smem_addr(&bars->q);
+            int64_t n_issued = 0;                        // K/V loads issued (two per tile), across items
+            int it = 0;                                  // valid items started
+            bool ok = true;
+            for (int64_t k = 0; ok && k * (int64_t)gridDim.x < n_items && !aborted(bars); ++k) {
+                const int64_t idx = snake_item(k);
+                if (idx >= n_items) continue;
+                const ItemGeom I = geom(idx);
+                if (I.cap_err) report(status, FOCUS_ERR_CAPACITY);
+                if (!I.valid) continue;
+                // the Q buffers are free once every QK MMA of the previous item has completed
+                if (it > 0 && !mbar_wait(smem_addr(&bars->q_free), (it - 1) & 1, kWaitNs)) {
+                    fail(bars, status);
+                    break;
+                }
+                mbar_expect_tx(bq, 2 * C::kTileBytes);
+                const int32_t qrow = GQA ? I.bh * q_per_kv + I.member : I.bh;
+                for (int t = 0; t < 2; ++t)
+                    for (int x = 0; x < C::kBoxes; ++x)
+                        tma_load_3d(smem_addr(smem + C::kQOff + t * C::kTileBytes + x * kBoxBytes), &tm_q, x * 64,
+                                    I.row_base + I.a0 + t * BM, qrow, bq);
+                for (int j = 0; j < I.n_kv_max; ++j) {
+                    const bool ring = j < I.n_ring;
+                    const int32_t row = ring ? j * BN : I.row_base + (j - I.n_ring) * BN;
+                    for (int part = 0; part < 2; ++part) {
+                        const int64_t n = n_issued;
+                        const int slot = (int)(n % kSlots);
+                        const int64_t use = n / kSlots;
+                        if (use > 0 && !mbar_wait(smem_addr(&bars->kv_empty[slot]), (uint32_t)((use - 1) & 1),
+                                                  kWaitNs)) {
+                            fail(bars, status);
+                            ok = false;
+                            break;
+                        }
+                        const uint32_t bf = smem_addr(&bars->kv_full[slot]);
+                        mbar_expect_tx(bf, C::kTileBytes);
+                        const CUtensorMap* map = part == 0 ? (ring ? &tm_rk : &tm_k) : (ring ? &tm_rv : &tm_v);
+                        for (int x = 0; x < C::kBoxes; ++x)
+                            tma_load_3d(smem_addr(smem + C::kSlotOff + slot * C::kTileBytes + x * kBoxBytes), map,
+                                        x * 64, row, I.bh, bf);
+                        n_issued = n + 1;
+                    }
+                    if (!ok) break;
+                }
+                ++it;
+            }
+            // drain: every issued copy must land before the CTA can exit
+            if (it > 0) mbar_wait(bq, (it - 1) & 1, kWaitNs);
+            for (int64_t n = (n_issued > kSlots ? n_issued - kSlots : 0); n < n_issued; ++n)
+                mbar_wait(smem_addr(&bars->kv_full[n % kSlots]), (uint32_t)((n / kSlots) & 1), kWaitNs);
+        } else if (warp == 1 && lane == 0) {
+            // ============================================= MMA issuer
+            constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, BN, false, false);
+            constexpr uint32_t idesc_pv = idesc_bf16_f32(BM, D, false, true);
+            const uint32_t sq = smem_addr(smem + C::kQOff);
+            const uint32_t sslot = smem_addr(smem + C::kSlotOff);
+            int64_t nt0 = 0;                 // K/V tiles consumed before this item
+            int it = 0;                      // valid items
+            int pc[2] = {0, 0};              // P tiles consumed per Q tile (p_full phases)
+            int oc[2] = {0, 0};              // items with an epilogue per Q tile (o_free phases)
+            bool ok = true;
+            for (int64_t k = 0; ok && k * (int64_t)gridDim.x < n_items && !aborted(bars); ++k) {
+                const int64_t idx = snake_item(k);
+                if (idx >= n_items) continue;
+                const ItemGeom I = geom(idx);
+                if (!I.valid) continue;
+                if (!mbar_wait(smem_addr(&bars->q), it & 1, kWaitNs)) { ok = false; break; }
+                for (int j = 0; ok && j <= I.n_kv_max; ++j) {
+                    int vslot = -1, kslot = -1;
+                    if (j >= 1) {
+                        const int64_t n = 2 * (nt0 + j - 1) + 1;
+                        vslot = (int)(n % kSlots);
+                        if (!mbar_wait(smem_addr(&bars->kv_full[vslot]), (uint32_t)((n / kSlots) & 1), kWaitNs)) {
+                            ok = false;
+                            break;
+                        }
+                    }
+                    if (j < I.n_kv_max) {
+                        const int64_t n = 2 * (nt0 + j);
+                        kslot = (int)(n % kSlots);
+                        if (!mbar_wait(smem_addr(&bars->kv_full[kslot]), (uint32_t)((n / kSlots) & 1), kWaitNs)) {
+                            ok = false;
+                            break;
+                        }
+                    }
+                    tc_fence_after();
+                    for (int t = 0; t < 2; ++t) {
+                        const int nkt = t == 0 ? I.n_kv0 : I.n_kv1;
+                        if (j >= 1 && j - 1 < nkt) {              // O_t += P_t(j-1) V_{j-1}
+                            // the first PV of an item overwrites O_t: the previous item's
+                            // epilogue must have read it
+                            if (j == 1 && oc[t] > 0 &&
+                                !mbar_wait(smem_addr(&bars->o_free[t]), (oc[t] - 1) & 1, kWaitNs)) {
+                                ok = false;
+                                break;
+                            }
+                            if (!mbar_wait(smem_addr(&bars->p_full[t]), pc[t] & 1, kWaitNs)) { ok = false; break; }
+                            ++pc[t];
+                            tc_fence_after();
+                            const uint32_t vbase = sslot + vslot * C::kTileBytes;
+#pragma unroll
+                            for (int kk = 0; kk < BN / 16; ++kk)
+                                mma_ts(tmem + 256 + t * D, tmem + t * 128 + kk * 8,
+                                       smem_desc_sw128(vbase + kk * 2048, kBoxBytes, 1024), idesc_pv,
+                                       (j - 1 > 0 || kk > 0) ? 1u : 0u);
+                            if (j - 1 == nkt - 1) {
+                                mma_commit(smem_addr(&bars->o_full[t]));
+                                ++oc[t];
+                            }
+                        }
+                        if (j < nkt) {                           // S_t = Q_t K_j^T
+                            const uint32_t qbase = sq + t * C::kTileBytes;
+                            const uint32_t kbase = sslot + kslot * C::kTileBytes;
+#pragma unroll
+                            for (int kk = 0; kk < D / 16; ++kk) {
+                                const uint32_t off = (kk / 4) * kBoxBytes + (kk % 4) * 32;
+                                mma_ss(tmem + t * 128, smem_desc_sw128(qbase + off, 16, 1024),
+                                       smem_desc_sw128(kbase + off, 16, 1024), idesc_qk, kk > 0 ? 1u : 0u);
+                            }
+                            mma_commit(smem_addr(&bars->s_full[t]));
+                        }
+                    }
+                    if (!ok) break;
+                    if (j == I.n_kv_max - 1) mma_commit(smem_addr(&bars->q_free));   // last QK of the item issued
+                    if (vslot >= 0) mma_commit(smem_addr(&bars->kv_empty[vslot]));
+                    if (kslot >= 0) mma_commit(smem_addr(&bars->kv_empty[kslot]));
+                }
+                nt0 += I.n_kv_max;
+                ++it;
+            }
+            if (!ok) fail(bars, status);
+            // drain: all issued MMAs complete before TMEM is freed
+            mma_commit(smem_addr(&bars->drain));
+            mbar_wait(smem_addr(&bars->drain), 0, kWaitNs);
+        }
+    } else {
+        // ================================================= softmax / epilogue
+        setmaxnreg_inc<kRegsSoftmax>();
+        const int t = (warp - 4) >> 2;                    // 0: warps 4-7, 1: warps 8-11
+        const int quarter = warp & 3;                     // TMEM lanes this warp may access
+        const int r = quarter * 32 + lane;                // row within the Q tile
+        const uint32_t lane_addr = (uint32_t)(quarter * 32) << 16;
+        const uint32_t s_addr = tmem + lane_addr + t * 128;
+        const uint32_t o_addr = tmem + lane_addr + 256 + t * D;
+        int sc = 0, oc = 0;                               // s_full / o_full phases
+        bool ok = true;
+        for (int64_t k = 0; ok && k * (int64_t)gridDim.x < n_items && !aborted(bars); ++k) {
+            const int64_t idx = snake_item(k);
+            if (idx >= n_items) continue;
+            const ItemGeom I = geom(idx);
+            if (!I.valid) continue;
+            const int n_kv = t == 0 ? I.n_kv0 : I.n_kv1;
+            if (n_kv == 0) continue;
+            const int qt = 2 * I.cta + t;                 // q-tile index within the window
+            float m_run = -INFINITY, l_run = 0.f;
+            for (int j = 0; j < n_kv; ++j) {
+                if (!mbar_wait(smem_addr(&bars->s_full[t]), sc & 1, kWaitNs)) { ok = false; break; }
+                ++sc;
+                tc_fence_after();
+                uint32_t sr[128];
+                tmem_ld32(s_addr + 0, sr);
+                tmem_ld32(s_addr + 32, sr + 32);
+                tmem_ld32(s_addr + 64, sr + 64);
+                tmem_ld32(s_addr + 96, sr + 96);
+                tmem_wait_ld();
+                float* s = reinterpret_cast<float*>(sr);
+                // analytic mask: the ring's last partial tile and the diagonal window tile
+                if (j < I.n_ring) {
+                    const int lim = I.Rw - j * BN;        // keys [0, lim) of this tile are visible
+                    if (lim < BN) {
+#pragma unroll
+                        for (int c = 0; c < BN; ++c)
+                            if (c >= lim) s[c] = -INFINITY;
+                    }
+                } else if (j - I.n_ring == qt) {          // key c visible iff c <= r
+#pragma unroll
+                    for (int c = 0; c < BN; ++c)
+                        if (c > r) s[c] = -INFINITY;
+                }
+                softmax_tile<D, false>(s, s_addr, o_addr, scale_log2, m_run, l_run, j > 0);
+                tmem_wait_st();
+                tc_fence_before();
+                mbar_arrive(smem_addr(&bars->p_full[t]));
+            }
+            if (!ok) {
+                fail(bars, status);
+                break;
+            }
+            // ---- epilogue: O / l -> bf16 through a per-warp staging buffer (the Q
+            // buffer may already hold the next item's Q), LSE; O_t is then free for
+            // the next item's first PV. The item geometry is recomputed here from an
+            // opaque copy of its index, so none of it stays live across the loop.
+            int64_t idx_e = idx;
+            asm volatile("mov.b64 %0, %0;" : "+l"(idx_e));
+            const ItemGeom E = geom(idx_e);
+            const int32_t aq = E.a0 + t * BM + r;         // in-window row
+            ok = mbar_wait(smem_addr(&bars->o_full[t]), oc & 1, kWaitNs);
+            ++oc;
+            if (!ok) {
+                fail(bars, status);
+                break;
+            }
+            tc_fence_after();
+            const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
+            const int32_t bhq = GQA ? E.bh * q_per_kv + E.member : E.bh;   // Q, O and LSE rows
+            // each warp stages a 32-column chunk of its 32 rows (64 B per row, 16-byte
+            // pieces swizzled by row so both the row writes and the coalesced reads
+            // are conflict-free), then stores 8 rows x 64 B per instruction
+            uint8_t* stage = smem + C::kStageOff + (warp - 4) * 2048;
+            __nv_bfloat16* otile = o + ((int64_t)bhq * T_span + E.row_base + E.a0 + t * BM + quarter * 32) * D;
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t orr[32];
+                tmem_ld32(o_addr + c * 32, orr);
+                tmem_wait_ld();
+                if (c == D / 32 - 1) {                    // all of O_t read: release it
+                    tc_fence_before();
+                    mbar_arrive(smem_addr(&bars->o_free[t]));
+                }
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    uint4 v;
+                    v.x = pack_bf16x2(__uint_as_float(orr[q4 * 8 + 0]) * inv_l, __uint_as_float(orr[q4 * 8 + 1]) * inv_l);
+                    v.y = pack_bf16x2(__uint_as_float(orr[q4 * 8 + 2]) * inv_l, __uint_as_float(orr[q4 * 8 + 3]) * inv_l);
+                    v.z = pack_bf16x2(__uint_as_float(orr[q4 * 8 + 4]) * inv_l, __uint_as_float(orr[q4 * 8 + 5]) * inv_l);
+                    v.w = pack_bf16x2(__uint_as_float(orr[q4 * 8 + 6]) * inv_l, __uint_as_float(orr[q4 * 8 + 7]) * inv_l);
+                    *reinterpret_cast<uint4*>(stage + lane * 64 + ((q4 ^ ((lane >> 1) & 3)) << 4)) = v;
+                }
+                __syncwarp();
+#pragma unroll
+                for (int i = 0; i < 32; i += 8) {
+                    const int rr = i + (lane >> 2), q4 = lane & 3;
+                    if (E.a0 + t * BM + quarter * 32 + rr < E.Tw)
+                        *reinterpret_cast<uint4*>(otile + (int64_t)rr * D + c * 32 + q4 * 8) =
+                            *reinterpret_cast<const uint4*>(stage + rr * 64 + ((q4 ^ ((rr >> 1) & 3)) << 4));
+                }
+                __syncwarp();
+            }
+            if (lse && aq < E.Tw)
+                lse[(int64_t)bhq * T_span + E.row_base + aq] = (m_run + __log2f(l_run)) * 0.69314718055994531f;
+        }
+    }
+
+    // ---- teardown ------------------------------------------------------------
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
+template <int D, bool GQA>
+cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t* status, cudaStream_t stream) {
+    const int64_t BH = (int64_t)c.B * c.H;
+    const int32_t g = c.q_per_kv > 1 ? c.q_per_kv : 1;
+    CUtensorMap tq, tk, tv, trk, trv;
+    cudaError_t e;
+    if ((e = make_map(&tq, a.q, D, a.T_span, BH * g)) != cudaSuccess) return e;
+    if ((e = make_map(&tk, a.k, D, a.T_span, BH)) != cudaSuccess) return e;
+    if ((e = make_map(&tv, a.v, D, a.T_span, BH)) != cudaSuccess) return e;
+    if (c.C_ring > 0) {
+        if ((e = make_map(&trk, c.ring_k, D, c.C_ring, BH)) != cudaSuccess) return e;
+        if ((e = make_map(&trv, c.ring_v, D, c.C_ring, BH)) != cudaSuccess) return e;
+    } else {                                   // no ring: the maps are never read
+        trk = tk;
+        trv = tv;
+    }
+    const int smem = Cfg<D>::kSmemPersistent;
+    auto* kernel = prefill_tc_persistent_kernel<D, GQA>;
+    if ((e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
+        return e;
+    // the register split needs the launch registers it was sized for: with fewer,
+    // the softmax warpgroups' setmaxnreg.inc could never be served
+    cudaFuncAttributes fa;
+    if ((e = cudaFuncGetAttributes(&fa, kernel)) != cudaSuccess) return e;
+    if (fa.numRegs < kLaunchRegs) return cudaErrorInvalidConfiguration;
+    int dev = 0, sms = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+    const int ctas_pw = (a.max_rows + 2 * BM - 1) / (2 * BM);
+    // one CTA per SM, each walking every gridDim.x-th work item
+    const int64_t n_items = (int64_t)(a.w_end - a.w_begin) * ctas_pw * g * c.H * c.B;
+    const dim3 grid((unsigned)(n_items < sms ? n_items : sms));
+    kernel<<<grid, kThreads, smem, stream>>>(tq, tk, tv, trk, trv, (__nv_bfloat16*)a.o, a.lse, a.T_span,
+                                             a.d_win_off, a.d_ring_off, a.w_begin, a.w_end, ctas_pw, c.H, c.C_ring,
+                                             a.scale * 1.4426950408889634f, status, g, n_items);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_prefill_tc_persistent(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
+                                         cudaStream_t stream) {
+    const bool gqa = c.q_per_kv > 1;
+    if (c.d == 128) return gqa ? launch_d<128, true>(c, a, status, stream) : launch_d<128, false>(c, a, status, stream);
+    return gqa ? launch_d<64, true>(c, a, status, stream) : launch_d<64, false>(c, a, status, stream);
+}
+
+}  // namespace prefill
+}  // namespace focus

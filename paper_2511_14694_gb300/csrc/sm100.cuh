@@ -192,7 +192,10 @@ __device__ __forceinline__ void mma_commit(uint32_t bar) {
                  : "memory");
 }
 
-// Register rebalancing between warpgroups (all 4 warps of a warpgroup execute it).
+// Register rebalancing between warpgroups: all four warps of a warpgroup execute
+// the same call. inc blocks until the CTA's pool (its launch registers minus what
+// the other warpgroups hold) can supply the new count, so the counts of all
+// warpgroups must sum to at most the block's launch registers.
 template <int N>
 __device__ __forceinline__ void setmaxnreg_inc() {
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));

@@ -89,6 +89,8 @@ def load() -> ctypes.CDLL:
     lib.focus_layout_sched.argtypes = [_i64, _i32, _P, _P, _u32, _i32, _i32, _P, ctypes.POINTER(LayoutOut), _P]
     lib.focus_attn_prefill.restype = ctypes.c_int
     lib.focus_attn_prefill.argtypes = [ctypes.POINTER(CacheDesc), ctypes.POINTER(PrefillArgs), _P]
+    lib.focus_prefill_kernel.restype = ctypes.c_int
+    lib.focus_prefill_kernel.argtypes = [ctypes.POINTER(CacheDesc), ctypes.POINTER(PrefillArgs), _P]
     lib.focus_decode_workspace_size.restype = ctypes.c_size_t
     lib.focus_decode_workspace_size.argtypes = [ctypes.POINTER(CacheDesc)]
     lib.focus_attn_decode.restype = ctypes.c_int
@@ -288,6 +290,25 @@ def attn_prefill(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | 
                     L["M"], w_begin, w_end, int(L["max_rows"]), scale, flags)
     _check("focus_attn_prefill", lib.focus_attn_prefill(ctypes.byref(cache.desc), ctypes.byref(a), _stream(stream)))
     return o, lse
+
+
+PREFILL_KERNELS = {0: "legacy mma.sync", 1: "tcgen05, one CTA per work item", 2: "tcgen05 persistent"}
+
+
+def prefill_kernel(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | None = None, flags: int = 0,
+                   o=None) -> str:
+    """Name of the kernel focus_attn_prefill would launch for these arguments
+    (focus_prefill_kernel: host only, nothing runs on the device)."""
+    lib = load()
+    w_end = L["M"] if w_end is None else w_end
+    T_span = q.shape[2]
+    a = PrefillArgs(_ptr(q), _ptr(k), _ptr(v), _ptr(q if o is None else o), 0, T_span, _ptr(L["win_off"]),
+                    _ptr(L["ring_off"]), L["M"], w_begin, w_end, int(L["max_rows"]), 1.0 / math.sqrt(q.shape[3]),
+                    flags)
+    out = ctypes.c_int32()
+    _check("focus_prefill_kernel", lib.focus_prefill_kernel(ctypes.byref(cache.desc), ctypes.byref(a),
+                                                           ctypes.byref(out)))
+    return PREFILL_KERNELS[out.value]
 
 
 def kv_compact_bulk(cache: Cache, src_k, src_v, L: dict, w_begin: int = 0, w_end: int | None = None,

@@ -30,6 +30,9 @@ WORKLOADS = {
     # a smaller prefill of the same shape (32 windows) for profiler captures: inputs still exceed L2
     "prefill_32kb_h32_d128": dict(mode="prefill", B=1, N=32_000, W=1_000, k=(100,), H=32, d=128,
                                   std=1.0 / math.sqrt(128)),
+    # plain causal attention at 16 kb (long work items, inputs above L2) for profiler captures
+    "causal_16kb_h32_d128": dict(mode="prefill", B=1, N=16_000, W=16_000, k=(0,), H=32, d=128,
+                                 std=1.0 / math.sqrt(128)),
     # plain causal attention (no compression) at 128 kb, for the O(N^2) comparison
     "causal_128kb_h32_d128": dict(mode="prefill", B=1, N=128_000, W=128_000, k=(0,), H=32, d=128,
                                   std=1.0 / math.sqrt(128)),

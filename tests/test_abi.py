@@ -128,6 +128,42 @@ def test_prefill_flag_checks_need_no_gpu():
     assert call(focus.PREFILL_KMER_LOCAL) == 2                            # boundary tails not supported
 
 
+def test_prefill_kernel_choice_needs_no_gpu():
+    """focus_prefill_kernel names the kernel focus_attn_prefill would launch: the
+    persistent tcgen05 kernel for the appendix mask without the rotary embedding
+    while C_ring + max_rows <= 4,096, the one-CTA-per-item kernel otherwise, the
+    legacy kernel on request; arguments are checked as for the launch."""
+    lib = focus.load()
+    c = focus.CacheDesc()
+    c.B, c.H, c.d = 1, 2, 128
+    c.ring_k = c.ring_v = 4096                        # never dereferenced: the query touches no memory
+    a = focus.PrefillArgs()
+    a.q = a.k = a.v = a.o = 4096
+    a.d_win_off = a.d_ring_off = 4096
+    a.n_windows, a.w_begin, a.w_end, a.scale, a.T_span = 128, 0, 128, 0.125, 129_280
+
+    def choice(C_ring, max_rows, flags=0):
+        c.C_ring, a.max_rows, a.flags = C_ring, max_rows, flags
+        out = ctypes.c_int32(-1)
+        rc = lib.focus_prefill_kernel(ctypes.byref(c), ctypes.byref(a), ctypes.byref(out))
+        return rc, out.value
+
+    assert choice(1_280, 1_010) == (0, 2)            # 128 windows of 1 kb, k = 100: short items
+    assert choice(3_086, 1_010) == (0, 2)            # exactly 4,096 rows
+    assert choice(3_087, 1_010) == (0, 1)
+    assert choice(10_000, 1_010) == (0, 1)           # a long ring
+    assert choice(1, 128_000) == (0, 1)              # one long window
+    assert choice(1_280, 1_010, focus.PREFILL_LEGACY_MMA) == (0, 0)
+    c.k_per_window, c.n_windows = 4096, 128
+    assert choice(1_280, 1_010, focus.PREFILL_KMER_LOCAL) == (0, 1)
+    c.rope_theta = 10_000.0
+    assert choice(1_280, 1_010) == (0, 1)
+    assert choice(1_280, 1_010, focus.PREFILL_LEGACY_MMA)[0] == 2      # legacy has no rotary embedding
+    c.rope_theta = 0.0
+    assert choice(1_280, 1_010, 8)[0] == 1                              # unknown flag bit
+    assert lib.focus_prefill_kernel(ctypes.byref(c), ctypes.byref(a), None) == 1
+
+
 def test_rope_argument_checks_need_no_gpu():
     """A negative or non-finite rotary base is refused on the host; decode with
     the rotary embedding needs pos_base."""

@@ -11,7 +11,7 @@ import torch
 
 from oracle import focus_oracle as fo
 from paper_2511_14694_gb300 import focus, inputs, pipeline
-from test_gpu_parity import assert_attn_close, bits
+from test_gpu_parity import PER_ITEM_C_RING, assert_attn_close, bits
 
 pytestmark = pytest.mark.gpu
 
@@ -30,17 +30,25 @@ def _expand(x, g):
     return x.repeat_interleave(g, dim=1)
 
 
-@pytest.mark.parametrize("g,d,flags,rope", [(2, 128, 0, 0.0), (4, 64, 0, 0.0), (8, 128, 0, 0.0), (3, 64, 0, 0.0),
-                                            (4, 128, "local", 0.0), (2, 128, 0, 10_000.0)])
-def test_gqa_prefill_masked_parallel_matches_oracle(g, d, flags, rope):
+@pytest.mark.parametrize("g,d,flags,rope,c_ring", [(2, 128, 0, 0.0, None), (4, 64, 0, 0.0, None),
+                                                   (8, 128, 0, 0.0, None), (3, 64, 0, 0.0, None),
+                                                   (4, 128, 0, 0.0, PER_ITEM_C_RING), (3, 64, 0, 0.0, PER_ITEM_C_RING),
+                                                   (4, 128, "local", 0.0, None), (2, 128, 0, 10_000.0, None)])
+def test_gqa_prefill_masked_parallel_matches_oracle(g, d, flags, rope, c_ring):
+    """A ring sized to the retained rows selects the persistent kernel for the
+    appendix mask; PER_ITEM_C_RING the one-CTA-per-item kernel (which also serves
+    the k-mer-local mask and the rotary embedding)."""
     N, W, ks, B, H = 5_000, 1_000, [100, 10, 50, 100, 7], 1, 2
     k = np.resize(np.asarray(ks, np.int32), 5)
     L = focus.layout(N, W, k)
     T = L["T"]
     q = inputs.normal_bf16((B, H * g, T, d), 1.0, seed=1, device="cuda")
     kk, v = (inputs.normal_bf16((B, H, T, d), 1.0, seed=s, device="cuda") for s in (2, 3))
-    cache = focus.Cache(B, H, d, C_ring=L["R"], k_sched=k, q_per_kv=g, rope_theta=rope)
+    cache = focus.Cache(B, H, d, C_ring=c_ring or L["R"], k_sched=k, q_per_kv=g, rope_theta=rope)
     fl = focus.PREFILL_KMER_LOCAL if flags == "local" else 0
+    persistent = c_ring is None and not fl and not rope
+    assert focus.prefill_kernel(cache, q, kk, v, L, flags=fl) == ("tcgen05 persistent" if persistent
+                                                                  else "tcgen05, one CTA per work item")
     o, lse = pipeline.prefill_masked_parallel(cache, q, kk, v, L, flags=fl)
     torch.cuda.synchronize()
     assert o.shape == q.shape and lse.shape == (B, H * g, T)

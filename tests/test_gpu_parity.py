@@ -93,12 +93,17 @@ TAIL_PREFILL_CASES = [
 ]
 
 
-def _masked_parallel(N, W, ks, B, H, d, std, seed=0, flags=0, tail=0):
+# Ring capacity that sends the appendix-mask prefill to the one-CTA-per-item
+# kernel: the persistent kernel serves only C_ring + max_rows <= 4,096 rows.
+PER_ITEM_C_RING = 8_192
+
+
+def _masked_parallel(N, W, ks, B, H, d, std, seed=0, flags=0, tail=0, c_ring=None):
     M = -(-N // W)
     k = inputs.k_schedule(M, ks, seed=seed + 1)
     L = focus.layout(N, W, k, tail=tail)
     q, kk, v = inputs.qkv((B, H, L["T"], d), std=std, seed=seed + 2, device="cuda")
-    cache = focus.Cache(B, H, d, C_ring=max(L["R"], 1))
+    cache = focus.Cache(B, H, d, C_ring=c_ring or max(L["R"], 1))
     n = q.numel()
     canary = torch.full((n + 4096,), 7.0, dtype=torch.bfloat16, device="cuda")
     o = canary[:n].view(q.shape)
@@ -108,9 +113,15 @@ def _masked_parallel(N, W, ks, B, H, d, std, seed=0, flags=0, tail=0):
     return L, q, kk, v, cache, o, lse
 
 
+@pytest.mark.parametrize("c_ring", [None, PER_ITEM_C_RING], ids=["persistent", "per_item"])
 @pytest.mark.parametrize("N,W,ks,B,H,d,std,tail", [c + (0,) for c in PREFILL_CASES] + TAIL_PREFILL_CASES)
-def test_prefill_masked_parallel_matches_oracle(N, W, ks, B, H, d, std, tail):
-    L, q, k, v, cache, o, lse = _masked_parallel(N, W, ks, B, H, d, std, seed=N, tail=tail)
+def test_prefill_masked_parallel_matches_oracle(N, W, ks, B, H, d, std, tail, c_ring):
+    """Both tcgen05 kernels on the same inputs: a ring sized to the retained rows
+    selects the persistent kernel for these short work items, a large ring the
+    one-CTA-per-item kernel."""
+    L, q, k, v, cache, o, lse = _masked_parallel(N, W, ks, B, H, d, std, seed=N, tail=tail, c_ring=c_ring)
+    assert focus.prefill_kernel(cache, q, k, v, L) == ("tcgen05 persistent" if c_ring is None
+                                                       else "tcgen05, one CTA per work item")
     ref_L = fo.layout(N, W, L["k_host"], tail=tail)
     T = L["T"]
     heads = np.repeat(np.arange(B * H), T)
