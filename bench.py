@@ -355,24 +355,20 @@ def run_prefill_leg(args, cfg, world, rank, local):
     compact_bytes = float(L["R"] * B * (H // g) * 2 * (2 * d) * 2)
     launches = 4 * args.steps   # layout scan + layout rows + bulk compaction + prefill
 
-    # end to end through the public API with host buffers
+    # end to end through the public API with host buffers: the pipelined host-buffer
+    # prefill (copies of one head group overlap the kernels of the others)
     e2e = None
     if not args.no_e2e:
         steps_e2e = max(1, min(args.steps, 5))
-        h_nt = nt.cpu().pin_memory()
-        h_q, h_k, h_v = (x.cpu().pin_memory() for x in (q, k, v))
-        h_o = torch.empty(o.shape, dtype=o.dtype).pin_memory()
-        h_lse = torch.empty(lse.shape, dtype=lse.dtype).pin_memory()
+        host = dict(nt=nt.cpu().pin_memory(), q=q.cpu().pin_memory(), k=k.cpu().pin_memory(),
+                    v=v.cpu().pin_memory(), o=torch.empty(o.shape, dtype=o.dtype).pin_memory(),
+                    lse=torch.empty(lse.shape, dtype=lse.dtype).pin_memory())
+        devb = dict(nt=nt, q=q, k=k, v=v, o=o, lse=lse)
+        h_nt, h_q, h_k, h_v, h_o, h_lse = (host[n] for n in ("nt", "q", "k", "v", "o", "lse"))
 
         def e2e_step():
-            nt.copy_(h_nt, non_blocking=True)
-            q.copy_(h_q, non_blocking=True)
-            k.copy_(h_k, non_blocking=True)
-            v.copy_(h_v, non_blocking=True)
-            front()
-            attn()
-            h_o.copy_(o, non_blocking=True)
-            h_lse.copy_(lse, non_blocking=True)
+            pipeline.prefill_masked_parallel_host(cache, L, host, devb, groups=args.e2e_groups,
+                                                  flags=args.prefill_flags, stream=stream)
 
         e2e_step()
         torch.cuda.synchronize(dev)
@@ -387,8 +383,10 @@ def run_prefill_leg(args, cfg, world, rank, local):
         h2d = sum(x.numel() * x.element_size() for x in (h_nt, h_q, h_k, h_v))
         d2h = h_o.numel() * h_o.element_size() + h_lse.numel() * h_lse.element_size()
         e2e = {"value": world * B * N / (e2e_ms / 1e3), "unit": "nt/s", "ms_per_step": e2e_ms,
-               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps_e2e}
-        del h_q, h_k, h_v, h_o, h_lse
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps_e2e,
+               "api": "pipeline.prefill_masked_parallel_host (%d head groups; copies overlap kernels)"
+                      % args.e2e_groups}
+        del h_q, h_k, h_v, h_o, h_lse, host
 
     host_sample = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -792,6 +790,8 @@ def main():
     ap.add_argument("--no-prefill", action="store_true", help="run only the decode leg (profiling)")
     ap.add_argument("--decode-workload", default="decode_1mb_b64_h32_d128")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--e2e-groups", type=int, default=16,
+                    help="head (or sequence) groups of the pipelined host-buffer prefill timed as e2e")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--no-clock-wait", action="store_true",

@@ -254,6 +254,30 @@ class Cache:
                               int(self.k_sched.numel()), W, B, H, d, C_ring, C_win, tail, _ptr(self.pos_base),
                               self.rope_theta, _ptr(self.W_sched), self.q_per_kv)
 
+    def part(self, b0: int = 0, b1: int | None = None, h0: int = 0, h1: int | None = None) -> "Cache":
+        """A view of sequences [b0, b1) and K/V heads [h0, h1) sharing this cache's
+        memory, for calls that process the cache in groups. The part must be
+        contiguous in the [B, H, rows, d] buffers: all heads, or one sequence."""
+        b1 = self.B if b1 is None else b1
+        h1 = self.H if h1 is None else h1
+        if not (0 <= b0 < b1 <= self.B and 0 <= h0 < h1 <= self.H):
+            raise ValueError(f"cache part [{b0}, {b1}) x [{h0}, {h1}) outside B={self.B}, H={self.H}")
+        if (h0, h1) != (0, self.H) and b1 - b0 != 1:
+            raise ValueError("a head range needs a single sequence (the part must be contiguous)")
+        v = object.__new__(Cache)
+        v.__dict__.update(self.__dict__)
+        v.B, v.H = b1 - b0, h1 - h0
+        for name in ("ring_k", "ring_v", "win_k", "win_v"):
+            t = getattr(self, name)
+            setattr(v, name, None if t is None else t[b0:b1, h0:h1])
+        for name in ("ring_len", "win_fill", "win_idx", "pos_base"):
+            setattr(v, name, getattr(self, name)[b0:b1])
+        v.desc = CacheDesc(_ptr(v.ring_k), _ptr(v.ring_v), _ptr(v.win_k), _ptr(v.win_v), _ptr(v.ring_len),
+                           _ptr(v.win_fill), _ptr(v.win_idx), _ptr(self.k_sched), int(self.k_sched.numel()), self.W,
+                           v.B, v.H, self.d, self.C_ring, self.C_win, self.tail, _ptr(v.pos_base), self.rope_theta,
+                           _ptr(self.W_sched), self.q_per_kv)
+        return v
+
     def workspace_bytes(self) -> int:
         return int(load().focus_decode_workspace_size(ctypes.byref(self.desc)))
 

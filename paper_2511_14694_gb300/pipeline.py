@@ -4,7 +4,10 @@ sequences of C-ABI calls. No arithmetic happens here; each step is a kernel.
 - masked-parallel: bulk-compact every window's FOCUS K/V into the ring, then one
   prefill call over all windows (window w reads ring prefix ring_off[w]);
 - sequential (streaming, App. A.2): for each window, prefill it against the ring,
-  then compact its FOCUS K/V into the ring.
+  then compact its FOCUS K/V into the ring;
+- masked-parallel from and to pinned host memory: the same calls per group of
+  heads (or sequences), with the host-device copies of one group on side
+  streams overlapping the kernels of the others.
 
 Under the k-mer-local mask (``focus.PREFILL_KMER_LOCAL``, Sec. 3.2) a row also
 reads its own window's FOCUS rows from the ring, so the streaming step compacts
@@ -13,6 +16,8 @@ step, so the order changes no value).
 """
 from __future__ import annotations
 
+import torch
+
 from . import focus
 
 
@@ -20,6 +25,62 @@ def prefill_masked_parallel(cache: focus.Cache, q, k, v, L: dict, scale=None, o=
                             stream=None):
     focus.kv_compact_bulk(cache, k, v, L, 0, L["M"], src_row0=0, stream=stream)
     return focus.attn_prefill(cache, q, k, v, L, 0, L["M"], scale=scale, o=o, lse=lse, flags=flags, stream=stream)
+
+
+_side_streams: dict = {}
+
+
+def prefill_masked_parallel_host(cache: focus.Cache, L: dict, host: dict, dev: dict, groups: int = 8, scale=None,
+                                 flags=0, stream=None):
+    """Masked-parallel prefill of a layer whose inputs and outputs live in pinned
+    host memory: host["nt"] (uint8 [B, N]), host["q"/"k"/"v"] (bf16 [B, H, T, d])
+    in, host["o"] (bf16) and host["lse"] (fp32 [B, H, T]) out; ``dev`` holds
+    device tensors of the same shapes, reused across calls.
+
+    The layout runs once; then the K/V heads (one sequence) or the sequences go
+    in ``groups`` parts, and part i's Q/K/V copy in on one side stream, its
+    compaction and attention run on ``stream``, and its O/LSE copy out on a second
+    side stream, so that the copies of one part overlap the compute and copies
+    of the others. Work is only enqueued: when ``stream`` is done, so is
+    everything, outputs in host memory included."""
+    cur = stream if stream is not None else torch.cuda.current_stream()
+    key = cur.device
+    if key not in _side_streams:
+        _side_streams[key] = (torch.cuda.Stream(device=key), torch.cuda.Stream(device=key))
+    s_in, s_out = _side_streams[key]
+    B, H, g = cache.B, cache.H, max(cache.q_per_kv, 1)
+    by_head = B == 1
+    n = H if by_head else B
+    groups = max(1, min(groups, n))
+    bounds = [n * i // groups for i in range(groups + 1)]
+    # the previous call's compute and copy-out are done with the device buffers
+    s_in.wait_stream(cur)
+    s_in.wait_stream(s_out)
+    with torch.cuda.stream(s_in):
+        dev["nt"].copy_(host["nt"], non_blocking=True)
+    cur.wait_stream(s_in)
+    focus.layout_run(L, dev["nt"], stream=cur)
+    for lo, hi in zip(bounds[:-1], bounds[1:]):
+        if by_head:
+            part = cache.part(h0=lo, h1=hi)
+            kv, qo = (slice(None), slice(lo, hi)), (slice(None), slice(lo * g, hi * g))
+        else:
+            part = cache.part(b0=lo, b1=hi)
+            kv = qo = (slice(lo, hi),)
+        with torch.cuda.stream(s_in):
+            dev["q"][qo].copy_(host["q"][qo], non_blocking=True)
+            dev["k"][kv].copy_(host["k"][kv], non_blocking=True)
+            dev["v"][kv].copy_(host["v"][kv], non_blocking=True)
+        cur.wait_stream(s_in)
+        focus.kv_compact_bulk(part, dev["k"][kv], dev["v"][kv], L, 0, L["M"], src_row0=0, stream=cur)
+        focus.attn_prefill(part, dev["q"][qo], dev["k"][kv], dev["v"][kv], L, 0, L["M"], scale=scale,
+                           o=dev["o"][qo], lse=dev["lse"][qo], flags=flags, stream=cur)
+        s_out.wait_stream(cur)
+        with torch.cuda.stream(s_out):
+            host["o"][qo].copy_(dev["o"][qo], non_blocking=True)
+            host["lse"][qo].copy_(dev["lse"][qo], non_blocking=True)
+    cur.wait_stream(s_out)
+    return host["o"], host["lse"]
 
 
 def prefill_window(cache: focus.Cache, q_w, k_w, v_w, L: dict, w: int, scale=None, o=None, lse=None, flags=0,

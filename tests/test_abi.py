@@ -211,3 +211,18 @@ def test_layout_size_sched_rejects_bad_schedules():
     w = np.array([30, 30, 40], np.int32)
     assert lib.focus_layout_size_sched(100, 3, w.ctypes.data, k.ctypes.data, 1, 0, ctypes.byref(T), None, None) == 0
     assert lib.focus_layout_size_sched(100, 3, None, k.ctypes.data, 1, 0, ctypes.byref(T), None, None) == 1
+
+
+def test_cache_part_checks_contiguity():
+    """Cache.part views a contiguous part of the cache: all heads of a range of
+    sequences, or a head range of one sequence (no device needed)."""
+    c = focus.Cache(2, 4, 64, C_ring=16, device="cpu")
+    p = c.part(h0=1, h1=3, b0=1, b1=2)
+    assert (p.desc.B, p.desc.H) == (1, 2)
+    assert p.desc.ring_k == c.ring_k.data_ptr() + (1 * 4 + 1) * 16 * 64 * 2
+    assert p.desc.ring_len == c.ring_len.data_ptr() + 4
+    assert c.part(b0=1).desc.B == 1
+    with pytest.raises(ValueError):
+        c.part(h0=1, h1=3)                        # two sequences x a head range: not contiguous
+    with pytest.raises(ValueError):
+        c.part(b0=2)
