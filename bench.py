@@ -475,6 +475,41 @@ def run_stream_leg(args, cfg, world, rank, local):
                 bytes_per_step=float(B * L["T"] * (H * (4 * d + 4) + (H // g) * 4 * d)))
 
 
+def run_embed_leg(args, world, rank, local):
+    """focus_embed_tokens on the 128 kb layout's token stream (129,280 rows) at an
+    Evo-2-7B-like width D: T x D bf16 written once, T token bytes read. CUDA events
+    around each launch; the output (1.06 GB at D = 4,096) exceeds L2."""
+    import torch
+    from paper_2511_14694_gb300 import focus, inputs
+    from paper_2511_14694_gb300.workloads import WORKLOADS
+    cfg = WORKLOADS["prefill_128kb_h32_d128"]
+    N, W, D = cfg["N"], cfg["W"], args.embed_d
+    M = -(-N // W)
+    k_s = inputs.k_schedule(M, cfg["k"], seed=inputs.DEFAULT_SEED)
+    dev = torch.device("cuda", local)
+    nt = inputs.nucleotides(1, N, seed=inputs.DEFAULT_SEED + rank, device=dev)
+    L = focus.layout_alloc(N, W, k_s, B=1, device=dev)
+    focus.layout_run(L, nt)
+    table = inputs.normal_bf16((5, D), 1.0, seed=inputs.DEFAULT_SEED, device=dev)
+    out = torch.empty((1, L["T"], D), dtype=torch.bfloat16, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    for _ in range(3):
+        focus.embed_tokens(L["tok"], table, out=out, stream=stream)
+    reps = 10
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+    torch.cuda.synchronize(dev)
+    for a, b in ev:
+        a.record(stream)
+        focus.embed_tokens(L["tok"], table, out=out, stream=stream)
+        b.record(stream)
+    torch.cuda.synchronize(dev)
+    assert focus.device_status(clear=True) == 0
+    ms = sorted(a.elapsed_time(b) for a, b in ev)[reps // 2]
+    nbytes = float(L["T"] * D * 2 + L["T"] + 5 * D * 2)
+    del out
+    return dict(ms=ms, bytes=nbytes, T=L["T"], D=D)
+
+
 def run_decode_leg(args, cfg, world, rank, local):
     import torch
     from paper_2511_14694_gb300 import focus, inputs
@@ -573,6 +608,7 @@ def run_focus(args, world, rank, local):
     dec = None
     if not args.no_decode:
         dec = run_decode_leg(args, WORKLOADS[args.decode_workload], world, rank, local)
+    emb = None if args.embed_d <= 0 else run_embed_leg(args, world, rank, local)
     if rank != 0:
         return
     value = weak_scaling_value(cfg["B"] * cfg["N"], world, pre["step_ms"] / 1e3)
@@ -639,6 +675,14 @@ def run_focus(args, world, rank, local):
                               "roofline": {"bound": "hbm", "achieved": cgbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                                            "frac": cgbs / peaks["hbm_gbs"],
                                            "peak_source": f"{peaks_src} copy bandwidth"}}
+    if emb is not None:
+        egbs = emb["bytes"] / (emb["ms"] / 1e3) / 1e9
+        line["embedding"] = {"kernel": "focus_embed_tokens", "rows": emb["T"], "D": emb["D"],
+                             "avg_launch_ms": emb["ms"], "bytes_per_launch": emb["bytes"],
+                             "timing": "CUDA events around each of 10 launches (median); output larger than L2",
+                             "roofline": {"bound": "hbm", "achieved": egbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                                          "frac": egbs / peaks["hbm_gbs"],
+                                          "peak_source": f"{peaks_src} copy bandwidth"}}
     if dec is not None:
         gbs = dec["bytes_leg"] / (dec["decode_kernels_ms"] / 1e3) / 1e9
         line["decode"] = {
@@ -790,6 +834,8 @@ def main():
     ap.add_argument("--no-prefill", action="store_true", help="run only the decode leg (profiling)")
     ap.add_argument("--decode-workload", default="decode_1mb_b64_h32_d128")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--embed-d", type=int, default=4096,
+                    help="width of the token-embedding gather timed beside the step (0 = skip)")
     ap.add_argument("--e2e-groups", type=int, default=16,
                     help="head (or sequence) groups of the pipelined host-buffer prefill timed as e2e")
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -325,6 +325,23 @@ typedef struct focus_compact_args {
 focus_status focus_kv_compact(const focus_cache* cache, const focus_compact_args* args,
                               cudaStream_t stream);
 
+/* ------------------------------------------------------------------------ */
+/* focus_embed_tokens — input rows of the augmented sequence (Sec. 3.2      */
+/* "Setup and tokens": the FOCUS summary is a learned token inserted after  */
+/* every k-mer; App. A: the inserted tokens take positions of their own).   */
+/* ------------------------------------------------------------------------ */
+/* out[i][:] = table[tok[i]][:] for i < n_rows: the token stream focus_layout
+ * writes (nucleotide ids 0..3, FOCUS_SUMMARY_TOKEN for a summary) looked up in an
+ * embedding table whose row FOCUS_SUMMARY_TOKEN is the summary token's vector.
+ * Device pointers, caller-owned: d_tok uint8 [n_rows] (e.g. layout tok, B x T
+ * rows), d_table bf16 [n_tokens][D], d_out bf16 [n_rows][D]; D a positive
+ * multiple of 8 and both bf16 pointers 16-byte aligned (else
+ * FOCUS_ERR_UNSUPPORTED), 1 <= n_tokens <= 256. A token >= n_tokens writes a zero
+ * row and sets the device status word to FOCUS_ERR_INVALID_ARG. n_rows = 0 is a
+ * no-op. Asynchronous on `stream`. */
+focus_status focus_embed_tokens(const uint8_t* d_tok, int64_t n_rows, const void* d_table, int32_t n_tokens,
+                                int32_t D, void* d_out, cudaStream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -360,6 +360,22 @@ def decode_f64(qf, knf, v_new, ring_kf, ring_v, R, win_kf, win_v, fill, scale: f
     return o, lse
 
 
+def embed_tokens(tok, table_bits) -> np.ndarray:
+    """Input rows of the augmented sequence (Sec. 3.2 "Setup and tokens": the
+    FOCUS summary is a learned token inserted after each k-mer; App. A: each
+    inserted token takes a position of its own): row i is the embedding-table row
+    of token tok[i]. ``table_bits``: uint16 bf16 patterns [n_tokens, D]; returns
+    the uint16 patterns [*tok.shape, D] (a lookup moves bits, nothing rounds).
+    A token outside the table gives a zero row."""
+    tok = np.asarray(tok)
+    table = np.asarray(table_bits, dtype=np.uint16)
+    out = np.zeros((*tok.shape, table.shape[1]), np.uint16)
+    for idx in np.ndindex(*tok.shape):
+        if int(tok[idx]) < table.shape[0]:
+            out[idx] = table[int(tok[idx])]
+    return out
+
+
 def window_retained_rows(n: int, k: int, close_partial: bool = True, tail: int = 0) -> np.ndarray:
     """In-window augmented offsets of the rows KV retention keeps for a window
     of n bases with cadence k: its FOCUS rows and its last ``tail`` bases (App. A)."""

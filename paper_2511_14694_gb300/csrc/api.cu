@@ -280,4 +280,18 @@ focus_status focus_kv_compact(const focus_cache* cache, const focus_compact_args
     return from_cuda(focus::launch_compact_window(*cache, st, stream));
 }
 
+focus_status focus_embed_tokens(const uint8_t* d_tok, int64_t n_rows, const void* d_table, int32_t n_tokens,
+                                int32_t D, void* d_out, cudaStream_t stream) {
+    if (n_rows < 0 || n_tokens < 1 || n_tokens > 256 || D <= 0) return FOCUS_ERR_INVALID_ARG;
+    if (D % 8 != 0) return FOCUS_ERR_UNSUPPORTED;
+    if (n_rows == 0) return FOCUS_OK;
+    if (!d_tok || !d_table || !d_out) return FOCUS_ERR_INVALID_ARG;
+    if (!aligned16(d_table) || !aligned16(d_out)) return FOCUS_ERR_UNSUPPORTED;
+    if (n_rows > INT64_MAX / D) return FOCUS_ERR_UNSUPPORTED;
+    int32_t* st = nullptr;
+    focus_status s = status_ptr(&st);
+    if (s != FOCUS_OK) return s;
+    return from_cuda(focus::launch_embed_tokens(d_tok, n_rows, d_table, n_tokens, D, d_out, st, stream));
+}
+
 }  // extern "C"

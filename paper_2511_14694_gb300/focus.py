@@ -99,6 +99,8 @@ def load() -> ctypes.CDLL:
     lib.focus_attn_decode_noalloc.argtypes = [ctypes.POINTER(CacheDesc), _P, _P, _P, _f32, _P, _P, _P]
     lib.focus_kv_compact.restype = ctypes.c_int
     lib.focus_kv_compact.argtypes = [ctypes.POINTER(CacheDesc), ctypes.POINTER(CompactArgs), _P]
+    lib.focus_embed_tokens.restype = ctypes.c_int
+    lib.focus_embed_tokens.argtypes = [_P, _i64, _P, _i32, _i32, _P, _P]
     _lib = lib
     return lib
 
@@ -333,6 +335,24 @@ def prefill_kernel(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int 
     _check("focus_prefill_kernel", lib.focus_prefill_kernel(ctypes.byref(cache.desc), ctypes.byref(a),
                                                            ctypes.byref(out)))
     return PREFILL_KERNELS[out.value]
+
+
+def embed_tokens(tok, table, out=None, stream=None):
+    """focus_embed_tokens: out[..., :] = table[tok[...]] for the layout's token
+    stream (uint8, any shape, e.g. L["tok"] [B, T]) and a bf16 table
+    [n_tokens, D]; returns out (bf16 [*tok.shape, D])."""
+    lib = load()
+    _cuda(tok, "tok", torch.uint8)
+    _cuda(table, "table", torch.bfloat16)
+    n_tokens, D = table.shape
+    if out is None:
+        out = torch.empty((*tok.shape, D), dtype=torch.bfloat16, device=tok.device)
+    _cuda(out, "out", torch.bfloat16)
+    if tuple(out.shape) != (*tok.shape, D):
+        raise ValueError(f"out shape {tuple(out.shape)}, want {(*tok.shape, D)}")
+    _check("focus_embed_tokens", lib.focus_embed_tokens(_ptr(tok), tok.numel(), _ptr(table), n_tokens, D, _ptr(out),
+                                                        _stream(stream)))
+    return out
 
 
 def kv_compact_bulk(cache: Cache, src_k, src_v, L: dict, w_begin: int = 0, w_end: int | None = None,

@@ -226,3 +226,19 @@ def test_cache_part_checks_contiguity():
         c.part(h0=1, h1=3)                        # two sequences x a head range: not contiguous
     with pytest.raises(ValueError):
         c.part(b0=2)
+
+
+def test_embed_tokens_argument_checks_need_no_gpu():
+    """focus_embed_tokens refuses bad widths and tables on the host; no rows is a
+    no-op that touches no pointer."""
+    lib = focus.load()
+    call = lambda n_rows, tab, n_tok, D, out: lib.focus_embed_tokens(4096, n_rows, tab, n_tok, D, out, None)  # noqa: E731
+    assert call(0, None, 5, 64, None) == 0                   # nothing to do
+    assert call(10, 4096, 0, 64, 4096) == 1                  # empty table
+    assert call(10, 4096, 257, 64, 4096) == 1                # token ids are bytes
+    assert call(10, 4096, 5, 0, 4096) == 1
+    assert call(10, 4096, 5, 12, 4096) == 2                  # D not a multiple of 8
+    assert call(10, 4104, 5, 64, 4096) == 2                  # table not 16-byte aligned
+    assert call(10, 4096, 5, 64, 4100) == 2                  # out not 16-byte aligned
+    assert call(-1, 4096, 5, 64, 4096) == 1
+    assert lib.focus_embed_tokens(None, 10, 4096, 5, 64, 4096, None) == 1

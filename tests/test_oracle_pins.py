@@ -657,3 +657,50 @@ def test_adaptive_windows_attention_matches_streaming_simulation(tail):
 def test_window_schedule_must_cover_the_sequence():
     with pytest.raises(ValueError):
         fo.layout_size(100, [30, 30], [5])
+
+
+# ----------------------------------------------------------------------------- token embedding (Sec. 3.2)
+
+def test_embed_tokens_one_hot_table_spells_the_string_layout():
+    """With a table whose row j is the one-hot vector of j (bf16 1.0 = 0x3F80),
+    each output row names its token, so the rows spell the independent string
+    construction of the layout (a summary 'S' after every k bases)."""
+    N, W, ks = 777, 100, [7, 30, 100]
+    M = _ceil(N, W)
+    k = inputs.k_schedule(M, ks, seed=5)
+    nt = inputs.nucleotides(2, N, seed=13).numpy()
+    L = fo.layout(N, W, k, nt=nt)
+    n_tok, D = 5, 8
+    table = np.zeros((n_tok, D), np.uint16)
+    table[np.arange(n_tok), np.arange(n_tok)] = 0x3F80
+    out = fo.embed_tokens(L["tok"], table)
+    assert out.shape == (2, L["T"], D)
+    for b in range(2):
+        got = "".join("ACGTS"[int(np.argmax(r))] for r in out[b])
+        assert got == _string_layout("".join("ACGT"[x] for x in nt[b]), W, k, True)
+        assert (out[b][:, n_tok:] == 0).all() and (out[b] != 0).sum() == L["T"]
+
+
+def test_embed_tokens_summary_rows_sit_at_summary_positions():
+    """The summary token's vector appears exactly on the layout's summary rows,
+    T - N of them (T = N + sum_w ceil(n_w / k_w), App. A), and nucleotide rows
+    carry their base's vector."""
+    N, W, ks = 4_000, 1_000, [100]
+    M = _ceil(N, W)
+    k = inputs.k_schedule(M, ks, seed=1)
+    nt = inputs.nucleotides(1, N, seed=3).numpy()
+    L = fo.layout(N, W, k, nt=nt)
+    rng = np.random.default_rng(0)
+    table = rng.integers(0, 1 << 16, size=(5, 64), dtype=np.uint16)
+    out = fo.embed_tokens(L["tok"], table)[0]
+    is_summary = (out == table[fo.SUMMARY_TOKEN]).all(axis=1)
+    assert is_summary.sum() == L["T"] - N == M * _ceil(W, 100)
+    assert np.array_equal(is_summary, L["kind"] == 1)
+    base_rows = np.flatnonzero(L["kind"] == 0)
+    assert np.array_equal(out[base_rows], table[nt[0][L["src"][base_rows]]])
+
+
+def test_embed_tokens_out_of_table_token_is_a_zero_row():
+    table = np.full((5, 8), 0x3F80, np.uint16)
+    out = fo.embed_tokens(np.array([0, 9, 4], np.uint8), table)
+    assert (out[1] == 0).all() and (out[0] == 0x3F80).all() and (out[2] == 0x3F80).all()
