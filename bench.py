@@ -761,15 +761,29 @@ def run_memory_report(args, world, rank, local):
     """Memory scaling with context length (the paper's Fig. "Scalability of memory
     with context length", Sec. 4.5): peak device memory and time of a streaming
     FOCUS prefill (one window's Q/K/V resident at a time, the retained ring
-    growing as N/k) against a full-cache causal prefill over the same N (Q/K/V
-    of all N rows resident), one attention layer, batch 1, 32 heads, d = 128."""
+    growing as N/k), of the masked-parallel FOCUS prefill (all rows resident, one
+    launch) and of a full-cache causal prefill over the same N (Q/K/V of all N
+    rows resident), one attention layer, batch 1, 32 heads, d = 128. Each time is
+    the second of two passes."""
     if rank != 0:
         return
     import torch
-    from paper_2511_14694_gb300 import focus, inputs
+    from paper_2511_14694_gb300 import focus, inputs, pipeline
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     H, d, W, k = 32, 128, 1_000, 100
+
+    def timed(fn):
+        fn()                                               # warm-up pass, not timed
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize(dev)
+        e0.record()
+        fn()
+        e1.record()
+        torch.cuda.synchronize(dev)
+        assert focus.device_status(clear=True) == 0
+        return e0.elapsed_time(e1)
+
     for N in [int(x) for x in args.memory_ns.split(",")]:
         row = {"report": "memory_scaling", "N": N, "H": H, "d": d, "W": W, "k": k,
                "kv_bytes_full": 2 * N * H * d * 2}
@@ -786,21 +800,29 @@ def run_memory_report(args, world, rank, local):
         q, kk, v = inputs.qkv((1, H, Tw, d), std=1 / math.sqrt(d), seed=1, device=dev)
         o = torch.empty_like(q)
         lse = torch.empty((1, H, Tw), dtype=torch.float32, device=dev)
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record()
-        for w in range(L["M"]):
-            a, e = int(off[w]), int(off[w + 1])
-            n = e - a
-            focus.attn_prefill(cache, q[:, :, :n].contiguous() if n != Tw else q, kk[:, :, :n].contiguous() if n != Tw else kk,
-                               v[:, :, :n].contiguous() if n != Tw else v, L, w, w + 1, o=o[:, :, :n].contiguous() if n != Tw else o,
-                               lse=lse[:, :, :n].contiguous() if n != Tw else lse)
-            focus.kv_compact_bulk(cache, kk[:, :, :n].contiguous() if n != Tw else kk,
-                                  v[:, :, :n].contiguous() if n != Tw else v, L, w, w + 1, src_row0=a)
-        e1.record()
-        torch.cuda.synchronize(dev)
-        assert focus.device_status(clear=True) == 0
+        def stream():
+            for w in range(L["M"]):
+                a, e = int(off[w]), int(off[w + 1])
+                n = e - a
+                cut = (lambda t: t[:, :, :n].contiguous()) if n != Tw else (lambda t: t)
+                focus.attn_prefill(cache, cut(q), cut(kk), cut(v), L, w, w + 1, o=cut(o), lse=cut(lse))
+                focus.kv_compact_bulk(cache, cut(kk), cut(v), L, w, w + 1, src_row0=a)
+
+        row["focus_ms"] = timed(stream)
         row["focus_peak_bytes"] = torch.cuda.max_memory_allocated(dev) - base
-        row["focus_ms"] = e0.elapsed_time(e1)
+        del cache, q, kk, v, o, lse
+        # FOCUS masked-parallel: Q/K/V of all rows resident, bulk compaction + one launch
+        torch.cuda.synchronize(dev)
+        torch.cuda.empty_cache()
+        torch.cuda.reset_peak_memory_stats(dev)
+        base = torch.cuda.memory_allocated(dev)
+        cache = focus.Cache(1, H, d, C_ring=max(L["R"], 1), device=dev)
+        q, kk, v = inputs.qkv((1, H, L["T"], d), std=1 / math.sqrt(d), seed=1, device=dev)
+        o = torch.empty_like(q)
+        lse = torch.empty((1, H, L["T"]), dtype=torch.float32, device=dev)
+        row["focus_parallel_ms"] = timed(lambda: pipeline.prefill_masked_parallel(cache, q, kk, v, L, o=o, lse=lse))
+        row["focus_parallel_peak_bytes"] = torch.cuda.max_memory_allocated(dev) - base
+        row["focus_parallel_kernel"] = focus.prefill_kernel(cache, q, kk, v, L)
         del cache, q, kk, v, o, lse, L
         # full cache: plain causal attention over all N rows (k = 0, one window)
         if N <= args.memory_full_max:
@@ -811,14 +833,11 @@ def run_memory_report(args, world, rank, local):
             Lc = focus.layout(N, N, [0], device=dev)
             cc = focus.Cache(1, H, d, C_ring=0, device=dev)
             q, kk, v = inputs.qkv((1, H, N, d), std=1 / math.sqrt(d), seed=1, device=dev)
-            e0.record()
-            focus.attn_prefill(cc, q, kk, v, Lc)
-            e1.record()
-            torch.cuda.synchronize(dev)
-            assert focus.device_status(clear=True) == 0
+            o = torch.empty_like(q)
+            lse = torch.empty((1, H, N), dtype=torch.float32, device=dev)
+            row["full_ms"] = timed(lambda: focus.attn_prefill(cc, q, kk, v, Lc, o=o, lse=lse))
             row["full_peak_bytes"] = torch.cuda.max_memory_allocated(dev) - base
-            row["full_ms"] = e0.elapsed_time(e1)
-            del cc, q, kk, v, Lc
+            del cc, q, kk, v, o, lse, Lc
         print(json.dumps(row), flush=True)
 
 
