@@ -404,8 +404,9 @@ def run_prefill_leg(args, cfg, world, rank, local):
 
 
 def run_stream_leg(args, cfg, world, rank, local):
-    """Streaming prefill (App. A.2): for each window in order, focus_attn_prefill
-    over that window against the ring, then focus_kv_compact of that window.
+    """Streaming prefill (App. A.2): for each window in order, focus_kv_compact of
+    that window, then focus_attn_prefill over it against the ring, consecutive
+    windows' attention overlapping on two streams (pipeline.prefill_streaming).
     Each window's Q/K/V is one of a pool of seeded windows (cycled)."""
     import torch
     from paper_2511_14694_gb300 import focus, inputs, pipeline
@@ -436,17 +437,10 @@ def run_stream_leg(args, cfg, world, rank, local):
     kernel_name = focus.prefill_kernel(cache, pq[0], pk[0], pv[0], L, M - 1, M, flags=args.prefill_flags, o=outs[0])
 
     def step(timed=False):
-        for w in range(M):
-            if local_mask:        # the k-mer-local mask reads the window's own FOCUS rows from the ring
-                focus.kv_compact_bulk(cache, pk[w % P], pv[w % P], L, w, w + 1, src_row0=int(off[w]), stream=stream)
-            if timed:
-                evs[w][0].record(stream)
-            focus.attn_prefill(cache, pq[w % P], pk[w % P], pv[w % P], L, w, w + 1, o=outs[w % 2], lse=lses[w % 2],
-                               stream=stream, flags=args.prefill_flags)
-            if timed:
-                evs[w][1].record(stream)
-            if not local_mask:
-                focus.kv_compact_bulk(cache, pk[w % P], pv[w % P], L, w, w + 1, src_row0=int(off[w]), stream=stream)
+        # each window's compaction, then its attention on one of two side streams:
+        # consecutive windows' launches overlap (pipeline.prefill_streaming)
+        pipeline.prefill_streaming(cache, L, lambda w: (pq[w % P], pk[w % P], pv[w % P]), outs, lses,
+                                   flags=args.prefill_flags, stream=stream, events=evs if timed else None)
 
     for _ in range(args.warmup):
         step()
@@ -468,8 +462,10 @@ def run_stream_leg(args, cfg, world, rank, local):
     barrier(world)
     assert focus.device_status(clear=True) == 0
     step_ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, world)
+    # the attention launches overlap, so the rate is taken over the whole step
+    # (compactions and gaps included); per_launch_ms is each launch on its stream
     return dict(kernel=kernel_name,
-                step_ms=step_ms, attn_ms=attn_ms / args.steps, flops_per_step=4.0 * d * H * B * pairs, pairs=pairs,
+                step_ms=step_ms, attn_ms=step_ms, flops_per_step=4.0 * d * H * B * pairs, pairs=pairs,
                 T=L["T"], R=L["R"], clocks=clk.summary(), launches=2 * M * args.steps, e2e=None, host_sample=None,
                 per_launch_ms=attn_ms / args.steps / M, local_mask=local_mask,
                 bytes_per_step=float(B * L["T"] * (H * (4 * d + 4) + (H // g) * 4 * d)))
@@ -630,7 +626,8 @@ def run_focus(args, world, rank, local):
         "dtype": "bf16", "data": "synthetic (seeded N(0,1)/sqrt(d) bf16 Q/K/V, uniform A/C/G/T ids)",
         "config": {"workload": args.workload, "B": cfg["B"], "N": cfg["N"], "W": cfg["W"], "k": list(cfg["k"]),
                    "H": cfg["H"], "d": cfg["d"], "T_augmented": pre["T"], "R_retained": pre["R"],
-                   "step": ("per window: focus_attn_prefill(window) + focus_kv_compact(window); all windows"
+                   "step": ("per window: focus_kv_compact(window) + focus_attn_prefill(window), consecutive "
+                            "windows' attention overlapping on two streams; all windows; rate over the whole step"
                             if cfg["mode"] == "stream" else
                             "focus_layout + focus_kv_compact(bulk) + focus_attn_prefill(masked-parallel)"),
                    "l2": ("inputs larger than L2 (pool of %d windows' Q/K/V %.2f GB, ring %.2f GB)" % (

@@ -7,7 +7,9 @@ sequences of C-ABI calls. No arithmetic happens here; each step is a kernel.
   then compact its FOCUS K/V into the ring;
 - masked-parallel from and to pinned host memory: the same calls per group of
   heads (or sequences), with the host-device copies of one group on side
-  streams overlapping the kernels of the others.
+  streams overlapping the kernels of the others;
+- streaming with overlapping windows: each window's compaction first, then its
+  attention on one of two side streams, so consecutive windows' launches overlap.
 
 Under the k-mer-local mask (``focus.PREFILL_KMER_LOCAL``, Sec. 3.2) a row also
 reads its own window's FOCUS rows from the ring, so the streaming step compacts
@@ -81,6 +83,50 @@ def prefill_masked_parallel_host(cache: focus.Cache, L: dict, host: dict, dev: d
             host["lse"][qo].copy_(dev["lse"][qo], non_blocking=True)
     cur.wait_stream(s_out)
     return host["o"], host["lse"]
+
+
+def prefill_streaming(cache: focus.Cache, L: dict, window_qkv, outs, lses, w_begin: int = 0, w_end: int | None = None,
+                      scale=None, flags=0, stream=None, events=None):
+    """Streaming prefill (App. A.2) of windows [w_begin, w_end) with the
+    attention of consecutive windows overlapping. window_qkv(w) gives window w's
+    (q, k, v) ([B, H, T_w, d] each); window w writes outs[i] and lses[i],
+    i = w % len(outs) (two buffers suffice; one per window keeps every output).
+
+    Window w's FOCUS rows are compacted into the ring before its attention (a
+    copy of input rows: window w reads ring rows [0, ring_off[w]) only, so the
+    order changes no value), all compactions in order on ``stream``. The
+    attention of window w then needs only the compaction of window w - 1, not the
+    attention of window w - 1: it runs on side stream i % 2 after that
+    compaction, so the tail of one launch overlaps the start of the next (windows
+    that share a buffer share a stream, so a buffer is never written by two
+    launches at once).
+    ``events``: optional list of (start, end) CUDA events per window, recorded
+    around each attention launch on its stream. Work is only enqueued; when
+    ``stream`` is done, so is everything."""
+    cur = stream if stream is not None else torch.cuda.current_stream()
+    key = cur.device
+    if key not in _side_streams:
+        _side_streams[key] = (torch.cuda.Stream(device=key), torch.cuda.Stream(device=key))
+    side = _side_streams[key]
+    w_end = L["M"] if w_end is None else w_end
+    off = L["win_off_host"]
+    for s_ in side:
+        s_.wait_stream(cur)                    # inputs and buffers written before the call
+    for w in range(w_begin, w_end):
+        q, k, v = window_qkv(w)
+        focus.kv_compact_bulk(cache, k, v, L, w, w + 1, src_row0=int(off[w]), stream=cur)
+        i = w % len(outs)
+        s_ = side[i % 2]
+        s_.wait_stream(cur)                    # ring rows of windows <= w are in place
+        if events is not None:
+            events[w - w_begin][0].record(s_)
+        focus.attn_prefill(cache, q, k, v, L, w, w + 1, scale=scale, o=outs[i], lse=lses[i], flags=flags,
+                           stream=s_)
+        if events is not None:
+            events[w - w_begin][1].record(s_)
+    for s_ in side:
+        cur.wait_stream(s_)
+    return outs, lses
 
 
 def prefill_window(cache: focus.Cache, q_w, k_w, v_w, L: dict, w: int, scale=None, o=None, lse=None, flags=0,

@@ -264,6 +264,33 @@ def test_prefill_streaming_matches_sequential_oracle(d, tail):
             assert np.array_equal(bits(cache.ring_v[b, h, :L["R"]]), rv)
 
 
+@pytest.mark.parametrize("d,tail,flags", [(128, 0, 0), (64, 3, 0), (128, 0, focus.PREFILL_KMER_LOCAL)])
+def test_prefill_streaming_overlapped_equals_sequential(d, tail, flags):
+    """pipeline.prefill_streaming (compaction first, consecutive windows' attention
+    overlapping on two streams) gives, bit for bit, the outputs and ring of the
+    one-window-at-a-time loop (which the test above pins to the oracle)."""
+    N, W, ks, B, H = 3_000, 500, [10, 50, 100, 7], 2, 2
+    M = -(-N // W)
+    k_s = inputs.k_schedule(M, ks, seed=4)
+    L = focus.layout(N, W, k_s, tail=tail)
+    q, k, v = inputs.qkv((B, H, L["T"], d), seed=23, device="cuda")
+    off = L["win_off_host"]
+    win = lambda t, w: t[:, :, int(off[w]):int(off[w + 1])].contiguous()  # noqa: E731
+    c_seq = focus.Cache(B, H, d, C_ring=L["R"], k_sched=k_s, tail=tail)
+    seq = [pipeline.prefill_window(c_seq, win(q, w), win(k, w), win(v, w), L, w, flags=flags) for w in range(M)]
+    c_ovl = focus.Cache(B, H, d, C_ring=L["R"], k_sched=k_s, tail=tail)
+    qkv_w = [(win(q, w), win(k, w), win(v, w)) for w in range(M)]
+    outs = [torch.empty_like(x[0]) for x in qkv_w]
+    lses = [torch.empty(x[0].shape[:3], dtype=torch.float32, device="cuda") for x in qkv_w]
+    pipeline.prefill_streaming(c_ovl, L, lambda w: qkv_w[w], outs, lses, flags=flags)
+    torch.cuda.synchronize()
+    for w in range(M):
+        assert np.array_equal(bits(outs[w]), bits(seq[w][0])), f"window {w}"
+        assert torch.equal(lses[w], seq[w][1]), f"window {w}"
+    assert np.array_equal(bits(c_ovl.ring_k), bits(c_seq.ring_k))
+    assert np.array_equal(bits(c_ovl.ring_v), bits(c_seq.ring_v))
+
+
 # ----------------------------------------------------------------------------- decode
 
 class DecodeModel:
