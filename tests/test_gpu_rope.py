@@ -110,6 +110,7 @@ class RopeDecodeModel:
 
     def __init__(self, cache, W, k_sched, theta):
         B, H = cache.B, cache.H
+        self.g = max(cache.q_per_kv, 1)          # query heads per K/V head
         self.rk = cache.ring_k.float().cpu().double().numpy().copy()
         self.rv = bits(cache.ring_v).copy()
         self.wk = cache.win_k.float().cpu().double().numpy().copy()
@@ -121,14 +122,15 @@ class RopeDecodeModel:
         self.W, self.k, self.theta, self.H = W, np.asarray(k_sched), theta, H
 
     def step(self, q, kn, vn, scale):
-        B, H, d = q.shape
-        o, lse = np.zeros((B, H, d)), np.zeros((B, H))
+        B, Hq, d = q.shape
+        e = np.arange(Hq) // self.g              # K/V head of each query head
+        o, lse = np.zeros((B, Hq, d)), np.zeros((B, Hq))
         for b in range(B):
             p = self.pos[b] + self.fill[b]
             qf = fo.rope(q[b].cpu(), p, self.theta, round_bf16=True)
             kf = fo.rope(kn[b].cpu(), p, self.theta, round_bf16=True)
-            o[b], lse[b] = fo.decode_f64(qf, kf, vn[b].cpu(), self.rk[b], self.rv[b], [self.R[b]] * H, self.wk[b],
-                                         self.wv[b], [self.fill[b]] * H, scale)
+            o[b], lse[b] = fo.decode_f64(qf, kf[e], bits(vn[b])[e], self.rk[b][e], self.rv[b][e], [self.R[b]] * Hq,
+                                         self.wk[b][e], self.wv[b][e], [self.fill[b]] * Hq, scale)
             f = self.fill[b]
             self.wk[b, :, f], self.wv[b, :, f] = kf, bits(vn[b])
             self.fill[b] += 1
@@ -175,6 +177,36 @@ def test_decode_rope_steps_match_oracle(d):
         R, f = int(model.R[b]), int(model.fill[b])
         assert_keys_close(cache.ring_k[b, :, :R], model.rk[b, :, :R], f"ring K b={b}", rel=2.0 ** -7)
         assert_keys_close(cache.win_k[b, :, :f], model.wk[b, :, :f], f"window K b={b}", rel=2.0 ** -7)
+
+
+@pytest.mark.parametrize("g,d", [(4, 128), (3, 64), (8, 64)])
+def test_decode_rope_grouped_heads_match_oracle(g, d):
+    """The rotary embedding with grouped-query heads: q rotated per query head,
+    k_new per K/V head, on the tensor-core kernel (even g) and the CUDA-core one
+    (odd g), across window retirements."""
+    B, H, W, theta = 2, 2, 50, 10_000.0
+    k_sched = np.array([10, 25, 7, 50, 10, 10], np.int32)
+    cache = focus.Cache(B, H, d, C_ring=256, C_win=64, W=W, k_sched=k_sched, rope_theta=theta, q_per_kv=g)
+    gen = torch.Generator(device="cuda").manual_seed(17)
+    for t in (cache.ring_k, cache.ring_v, cache.win_k, cache.win_v):
+        t.copy_(torch.randn(t.shape, generator=gen, device="cuda").bfloat16())
+    cache.ring_len.copy_(torch.tensor([20, 130], dtype=torch.int32))
+    cache.win_idx.copy_(torch.tensor([1, 2], dtype=torch.int32))
+    cache.win_fill.copy_(torch.tensor([40, 3], dtype=torch.int32))
+    cache.pos_base.copy_(torch.tensor([5_000, 77_777], dtype=torch.int32))
+    model = RopeDecodeModel(cache, W, k_sched, theta)
+    ws = cache.new_workspace()
+    scale = 1.0 / math.sqrt(d)
+    for step in range(30):
+        q = inputs.normal_bf16((B, H * g, d), 1.0, seed=500 + step, device="cuda")
+        kn, vn = (inputs.normal_bf16((B, H, d), 1.0, seed=800 + 2 * step + i, device="cuda") for i in (0, 1))
+        o, lse = focus.attn_decode(cache, q, kn, vn, workspace=ws)
+        focus.kv_compact_window(cache)
+        o_ref, lse_ref = model.step(q, kn, vn, scale)
+        assert_attn_close(o, lse, o_ref, lse_ref, f"rope gqa g={g} decode step {step}")
+    torch.cuda.synchronize()
+    assert np.array_equal(cache.ring_len.cpu().numpy(), model.R)
+    assert np.array_equal(cache.pos_base.cpu().numpy(), model.pos)
 
 
 def test_full_size_streaming_rope_sampled():
