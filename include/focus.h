@@ -325,6 +325,16 @@ typedef struct focus_compact_args {
 focus_status focus_kv_compact(const focus_cache* cache, const focus_compact_args* args,
                               cudaStream_t stream);
 
+/* Self-test of the failure path (no fault, no hang): one CTA waits, with the
+ * bounded mbarrier wait every kernel of this library uses, on a barrier nothing
+ * arrives on; after limit_ns it gives up and sets the device status word to
+ * FOCUS_ERR_TIMEOUT, as a kernel whose copies or MMAs never completed would. The
+ * context stays usable. Kernels that find FOCUS_ERR_TIMEOUT already set skip their
+ * work (so that a systematic stall costs one round of waits), so clear the word
+ * (focus_get_device_status with clear != 0) before further calls.
+ * 0 < limit_ns <= 10 s, else FOCUS_ERR_INVALID_ARG. Asynchronous on `stream`. */
+focus_status focus_selftest_timeout(uint64_t limit_ns, cudaStream_t stream);
+
 /* ------------------------------------------------------------------------ */
 /* focus_embed_tokens — input rows of the augmented sequence (Sec. 3.2      */
 /* "Setup and tokens": the FOCUS summary is a learned token inserted after  */

@@ -280,6 +280,14 @@ focus_status focus_kv_compact(const focus_cache* cache, const focus_compact_args
     return from_cuda(focus::launch_compact_window(*cache, st, stream));
 }
 
+focus_status focus_selftest_timeout(uint64_t limit_ns, cudaStream_t stream) {
+    if (limit_ns == 0 || limit_ns > 10000000000ull) return FOCUS_ERR_INVALID_ARG;
+    int32_t* st = nullptr;
+    focus_status s = status_ptr(&st);
+    if (s != FOCUS_OK) return s;
+    return from_cuda(focus::launch_selftest_timeout(limit_ns, st, stream));
+}
+
 focus_status focus_embed_tokens(const uint8_t* d_tok, int64_t n_rows, const void* d_table, int32_t n_tokens,
                                 int32_t D, void* d_out, cudaStream_t stream) {
     if (n_rows < 0 || n_tokens < 1 || n_tokens > 256 || D <= 0) return FOCUS_ERR_INVALID_ARG;

@@ -101,6 +101,7 @@ cudaError_t launch_compact_bulk(const focus_cache& c, const focus_compact_args& 
 cudaError_t launch_compact_bulk_rope(const focus_cache& c, const focus_compact_args& a, int32_t* status,
                                      cudaStream_t stream);
 cudaError_t launch_compact_window(const focus_cache& c, int32_t* status, cudaStream_t stream);
+cudaError_t launch_selftest_timeout(uint64_t limit_ns, int32_t* status, cudaStream_t stream);
 cudaError_t launch_embed_tokens(const uint8_t* tok, int64_t n_rows, const void* table, int32_t n_tokens, int32_t D,
                                 void* out, int32_t* status, cudaStream_t stream);
 

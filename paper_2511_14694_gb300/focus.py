@@ -99,6 +99,8 @@ def load() -> ctypes.CDLL:
     lib.focus_attn_decode_noalloc.argtypes = [ctypes.POINTER(CacheDesc), _P, _P, _P, _f32, _P, _P, _P]
     lib.focus_kv_compact.restype = ctypes.c_int
     lib.focus_kv_compact.argtypes = [ctypes.POINTER(CacheDesc), ctypes.POINTER(CompactArgs), _P]
+    lib.focus_selftest_timeout.restype = ctypes.c_int
+    lib.focus_selftest_timeout.argtypes = [ctypes.c_uint64, _P]
     lib.focus_embed_tokens.restype = ctypes.c_int
     lib.focus_embed_tokens.argtypes = [_P, _i64, _P, _i32, _i32, _P, _P]
     _lib = lib
@@ -256,6 +258,19 @@ class Cache:
                               int(self.k_sched.numel()), W, B, H, d, C_ring, C_win, tail, _ptr(self.pos_base),
                               self.rope_theta, _ptr(self.W_sched), self.q_per_kv)
 
+    _STATE = ("ring_k", "ring_v", "win_k", "win_v", "ring_len", "win_fill", "win_idx", "pos_base")
+
+    def snapshot(self) -> dict:
+        """Copies of the cache state (ring and window K/V, ring_len, win_fill,
+        win_idx, pos_base) on the same device: a checkpoint of a decode stream."""
+        return {n: getattr(self, n).clone() for n in self._STATE if getattr(self, n) is not None}
+
+    def restore(self, state: dict) -> None:
+        """Copy a snapshot back in place (same shapes); decoding then continues
+        exactly as from the moment the snapshot was taken."""
+        for n, t in state.items():
+            getattr(self, n).copy_(t)
+
     def part(self, b0: int = 0, b1: int | None = None, h0: int = 0, h1: int | None = None) -> "Cache":
         """A view of sequences [b0, b1) and K/V heads [h0, h1) sharing this cache's
         memory, for calls that process the cache in groups. The part must be
@@ -411,6 +426,12 @@ def attn_decode_noalloc(cache: Cache, q, k_new, v_new, scale=None, o=None, lse=N
            lib.focus_attn_decode_noalloc(ctypes.byref(cache.desc), _ptr(q), _ptr(k_new), _ptr(v_new), scale,
                                          _ptr(o), _ptr(lse), _stream(stream)))
     return o, lse
+
+
+def selftest_timeout(limit_ns: int = 20_000_000, stream=None) -> None:
+    """focus_selftest_timeout: a bounded device wait that nothing completes gives up
+    after limit_ns and sets FOCUS_ERR_TIMEOUT in the device status word."""
+    _check("focus_selftest_timeout", load().focus_selftest_timeout(int(limit_ns), _stream(stream)))
 
 
 def device_status(clear: bool = True, stream=None) -> int:

@@ -242,3 +242,23 @@ def test_embed_tokens_argument_checks_need_no_gpu():
     assert call(10, 4096, 5, 64, 4100) == 2                  # out not 16-byte aligned
     assert call(-1, 4096, 5, 64, 4096) == 1
     assert lib.focus_embed_tokens(None, 10, 4096, 5, 64, 4096, None) == 1
+
+
+def test_selftest_timeout_argument_checks_need_no_gpu():
+    """The failure-path self-test refuses a zero or over-long wait on the host."""
+    lib = focus.load()
+    assert lib.focus_selftest_timeout(0, None) == 1
+    assert lib.focus_selftest_timeout(10_000_000_001, None) == 1
+
+
+def test_cache_snapshot_restore_round_trip():
+    """A snapshot holds copies of the whole cache state and restores it in place."""
+    c = focus.Cache(2, 1, 64, C_ring=8, C_win=4, W=3, k_sched=[2], device="cpu")
+    c.ring_k.fill_(1.0)
+    c.win_fill.fill_(2)
+    snap = c.snapshot()
+    assert set(snap) == {"ring_k", "ring_v", "win_k", "win_v", "ring_len", "win_fill", "win_idx", "pos_base"}
+    c.ring_k.fill_(3.0)
+    c.win_fill.fill_(0)
+    c.restore(snap)
+    assert bool((c.ring_k == 1.0).all()) and bool((c.win_fill == 2).all())
