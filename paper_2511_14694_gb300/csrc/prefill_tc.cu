@@ -283,9 +283,8 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
             const uint32_t bq = smem_addr(&bars->q);
             mbar_expect_tx(bq, 2 * C::kTileBytes);
             for (int t = 0; t < 2; ++t)
-                for (int x = 0; x < C::kBoxes; ++x)
-                    tma_load_3d(smem_addr(smem + C::kQOff + t * C::kTileBytes + x * kBoxBytes), &tm_q, x * 64,
-                                row_base + a0 + t * BM, GQA ? bh * q_per_kv + member : bh, bq);
+                load_tile<D>(smem_addr(smem + C::kQOff + t * C::kTileBytes), &tm_q, row_base + a0 + t * BM,
+                             GQA ? bh * q_per_kv + member : bh, bq);
             int issued = 0;
             for (int j = 0; j < n_kv_max && !aborted(bars); ++j) {
                 const bool ring = j < n_ring;
@@ -299,9 +298,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
                     const uint32_t bf = smem_addr(&bars->kv_full[slot]);
                     mbar_expect_tx(bf, C::kTileBytes);
                     const CUtensorMap* map = part == 0 ? (ring ? &tm_rk : &tm_k) : (ring ? &tm_rv : &tm_v);
-                    for (int x = 0; x < C::kBoxes; ++x)
-                        tma_load_3d(smem_addr(smem + C::kSlotOff + slot * C::kTileBytes + x * kBoxBytes), map,
-                                    x * 64, row, bh, bf);
+                    load_tile<D>(smem_addr(smem + C::kSlotOff + slot * C::kTileBytes), map, row, bh, bf);
                     issued = n + 1;
                 }
             }
@@ -313,8 +310,6 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
     } else if (warp == 1) {
         // ================================================= MMA issuer
         if (lane == 0) {
-            constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, BN, false, false);
-            constexpr uint32_t idesc_pv = idesc_bf16_f32(BM, D, false, true);
             const uint32_t sq = smem_addr(smem + C::kQOff);
             const uint32_t sslot = smem_addr(smem + C::kSlotOff);
             bool ok = mbar_wait(smem_addr(ROPE ? &bars->q_rot : &bars->q), 0, kWaitNs);
@@ -338,23 +333,11 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
                     if (j >= 1 && j - 1 < nkt) {              // O_t += P_t(j-1) V_{j-1}
                         if (!mbar_wait(smem_addr(&bars->p_full[t]), (j - 1) & 1, kWaitNs)) { ok = false; break; }
                         tc_fence_after();
-                        const uint32_t vbase = sslot + vslot * C::kTileBytes;
-#pragma unroll
-                        for (int kk = 0; kk < BN / 16; ++kk)
-                            mma_ts(tmem + 256 + t * D, tmem + t * 128 + kk * 8,
-                                   smem_desc_sw128(vbase + kk * 2048, kBoxBytes, 1024), idesc_pv,
-                                   (j - 1 > 0 || kk > 0) ? 1u : 0u);
+                        issue_pv<D>(tmem + 256 + t * D, tmem + t * 128, sslot + vslot * C::kTileBytes, j - 1 > 0);
                         if (j - 1 == nkt - 1) mma_commit(smem_addr(&bars->o_full[t]));
                     }
                     if (j < nkt) {                           // S_t = Q_t K_j^T
-                        const uint32_t qbase = sq + t * C::kTileBytes;
-                        const uint32_t kbase = sslot + kslot * C::kTileBytes;
-#pragma unroll
-                        for (int kk = 0; kk < D / 16; ++kk) {
-                            const uint32_t off = (kk / 4) * kBoxBytes + (kk % 4) * 32;
-                            mma_ss(tmem + t * 128, smem_desc_sw128(qbase + off, 16, 1024),
-                                   smem_desc_sw128(kbase + off, 16, 1024), idesc_qk, kk > 0 ? 1u : 0u);
-                        }
+                        issue_qk<D>(tmem + t * 128, sq + t * C::kTileBytes, sslot + kslot * C::kTileBytes);
                         mma_commit(smem_addr(&bars->s_full[t]));
                     }
                 }

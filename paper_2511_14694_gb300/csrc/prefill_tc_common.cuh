@@ -61,6 +61,39 @@ __device__ __forceinline__ void fail(Bars* bars, int32_t* status) {
 }
 __device__ __forceinline__ bool aborted(Bars* bars) { return *(volatile int32_t*)&bars->abort != 0; }
 
+// One 128-row tile of a [BH][rows][D] bf16 tensor into shared memory as D/64 TMA
+// boxes of 128 rows x 64 columns (128-byte swizzle), completing on `bar`.
+template <int D>
+__device__ __forceinline__ void load_tile(uint32_t dst, const CUtensorMap* map, int32_t row, int32_t bh, uint32_t bar) {
+#pragma unroll
+    for (int x = 0; x < D / 64; ++x) tma_load_3d(dst + x * kBoxBytes, map, x * 64, row, bh, bar);
+}
+
+// S (TMEM, 128 fp32 columns) = Q K^T for one 128-row Q tile and one 128-key K
+// tile, both K-major in shared memory: D/16 MMAs of 128x128x16.
+template <int D>
+__device__ __forceinline__ void issue_qk(uint32_t s_tmem, uint32_t qbase, uint32_t kbase) {
+    constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, false, false);
+#pragma unroll
+    for (int kk = 0; kk < D / 16; ++kk) {
+        const uint32_t off = (kk / 4) * kBoxBytes + (kk % 4) * 32;
+        mma_ss(s_tmem, smem_desc_sw128(qbase + off, 16, 1024), smem_desc_sw128(kbase + off, 16, 1024), idesc,
+               kk > 0 ? 1u : 0u);
+    }
+}
+
+// O (TMEM, D fp32 columns) (+)= P V for one Q tile: P bf16 in TMEM over S, V an
+// MN-major 128-key tile in shared memory; BN/16 MMAs of 128xDx16. `accumulate` is
+// false for the first tile of an item, whose PV overwrites O.
+template <int D>
+__device__ __forceinline__ void issue_pv(uint32_t o_tmem, uint32_t p_tmem, uint32_t vbase, bool accumulate) {
+    constexpr uint32_t idesc = idesc_bf16_f32(BM, D, false, true);
+#pragma unroll
+    for (int kk = 0; kk < BN / 16; ++kk)
+        mma_ts(o_tmem, p_tmem + kk * 8, smem_desc_sw128(vbase + kk * 2048, kBoxBytes, 1024), idesc,
+               (accumulate || kk > 0) ? 1u : 0u);
+}
+
 // Online softmax of one S tile in the log2 domain for the row this thread owns:
 // s holds the row's BN masked scores, (m_run, l_run) the running max and sum.
 // P = 2^(s scale - m) goes back to TMEM over S as bf16 pairs (two 32-column

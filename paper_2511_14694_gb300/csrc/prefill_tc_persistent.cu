@@ -157,9 +157,8 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
                 mbar_expect_tx(bq, 2 * C::kTileBytes);
                 const int32_t qrow = GQA ? I.bh * q_per_kv + I.member : I.bh;
                 for (int t = 0; t < 2; ++t)
-                    for (int x = 0; x < C::kBoxes; ++x)
-                        tma_load_3d(smem_addr(smem + C::kQOff + t * C::kTileBytes + x * kBoxBytes), &tm_q, x * 64,
-                                    I.row_base + I.a0 + t * BM, qrow, bq);
+                    load_tile<D>(smem_addr(smem + C::kQOff + t * C::kTileBytes), &tm_q, I.row_base + I.a0 + t * BM,
+                                 qrow, bq);
                 for (int j = 0; j < I.n_kv_max; ++j) {
                     const bool ring = j < I.n_ring;
                     const int32_t row = ring ? j * BN : I.row_base + (j - I.n_ring) * BN;
@@ -176,9 +175,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
                         const uint32_t bf = smem_addr(&bars->kv_full[slot]);
                         mbar_expect_tx(bf, C::kTileBytes);
                         const CUtensorMap* map = part == 0 ? (ring ? &tm_rk : &tm_k) : (ring ? &tm_rv : &tm_v);
-                        for (int x = 0; x < C::kBoxes; ++x)
-                            tma_load_3d(smem_addr(smem + C::kSlotOff + slot * C::kTileBytes + x * kBoxBytes), map,
-                                        x * 64, row, I.bh, bf);
+                        load_tile<D>(smem_addr(smem + C::kSlotOff + slot * C::kTileBytes), map, row, I.bh, bf);
                         n_issued = n + 1;
                     }
                     if (!ok) break;
@@ -191,8 +188,6 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
                 mbar_wait(smem_addr(&bars->kv_full[n % kSlots]), (uint32_t)((n / kSlots) & 1), kWaitNs);
         } else if (warp == 1 && lane == 0) {
             // ============================================= MMA issuer
-            constexpr uint32_t idesc_qk = idesc_bf16_f32(BM, BN, false, false);
-            constexpr uint32_t idesc_pv = idesc_bf16_f32(BM, D, false, true);
             const uint32_t sq = smem_addr(smem + C::kQOff);
             const uint32_t sslot = smem_addr(smem + C::kSlotOff);
             int64_t nt0 = 0;                 // K/V tiles consumed before this item
@@ -238,26 +233,14 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
                             if (!mbar_wait(smem_addr(&bars->p_full[t]), pc[t] & 1, kWaitNs)) { ok = false; break; }
                             ++pc[t];
                             tc_fence_after();
-                            const uint32_t vbase = sslot + vslot * C::kTileBytes;
-#pragma unroll
-                            for (int kk = 0; kk < BN / 16; ++kk)
-                                mma_ts(tmem + 256 + t * D, tmem + t * 128 + kk * 8,
-                                       smem_desc_sw128(vbase + kk * 2048, kBoxBytes, 1024), idesc_pv,
-                                       (j - 1 > 0 || kk > 0) ? 1u : 0u);
+                            issue_pv<D>(tmem + 256 + t * D, tmem + t * 128, sslot + vslot * C::kTileBytes, j - 1 > 0);
                             if (j - 1 == nkt - 1) {
                                 mma_commit(smem_addr(&bars->o_full[t]));
                                 ++oc[t];
                             }
                         }
                         if (j < nkt) {                           // S_t = Q_t K_j^T
-                            const uint32_t qbase = sq + t * C::kTileBytes;
-                            const uint32_t kbase = sslot + kslot * C::kTileBytes;
-#pragma unroll
-                            for (int kk = 0; kk < D / 16; ++kk) {
-                                const uint32_t off = (kk / 4) * kBoxBytes + (kk % 4) * 32;
-                                mma_ss(tmem + t * 128, smem_desc_sw128(qbase + off, 16, 1024),
-                                       smem_desc_sw128(kbase + off, 16, 1024), idesc_qk, kk > 0 ? 1u : 0u);
-                            }
+                            issue_qk<D>(tmem + t * 128, sq + t * C::kTileBytes, sslot + kslot * C::kTileBytes);
                             mma_commit(smem_addr(&bars->s_full[t]));
                         }
                     }
