@@ -2,6 +2,8 @@
 the pins in test_oracle_pins.py fail for each one: a pin that no mistake can
 trip pins nothing."""
 import os
+
+import numpy as np
 import subprocess
 
 import pytest
@@ -100,3 +102,28 @@ def test_pins_catch_planted_mistake(tmp_path, name, old, new, checks):
         for check in checks:
             with pytest.raises((AssertionError, ValueError, IndexError)):
                 check()
+
+
+# The token-embedding lookup is Python in the oracle: plant its mistakes by
+# replacing the function for the duration of the pins.
+_embed = fo.embed_tokens
+EMBED_MUTANTS = [
+    ("embed_token_off_by_one", lambda tok, table: _embed((np.asarray(tok).astype(np.int64) + 1) % 5, table)),
+    ("embed_summary_as_base", lambda tok, table: _embed(np.where(np.asarray(tok) == fo.SUMMARY_TOKEN, 0, tok),
+                                                         table)),
+    ("embed_transposed_table", lambda tok, table: _embed(tok, np.ascontiguousarray(
+        np.asarray(table)[:, ::-1]))),
+]
+
+
+@pytest.mark.parametrize("name,mutant", EMBED_MUTANTS, ids=[m[0] for m in EMBED_MUTANTS])
+def test_embed_mutant_trips_a_pin(name, mutant, monkeypatch):
+    monkeypatch.setattr(fo, "embed_tokens", mutant)
+    tripped = False
+    for pin in (pins.test_embed_tokens_one_hot_table_spells_the_string_layout,
+                pins.test_embed_tokens_summary_rows_sit_at_summary_positions):
+        try:
+            pin()
+        except (AssertionError, IndexError):      # a wrong row can name a token that does not exist
+            tripped = True
+    assert tripped, f"no embedding pin caught the mutant {name}"
