@@ -92,11 +92,16 @@ using namespace prefill;
 
 // Register split (variants without the rotary embedding): warpgroup 0 (TMA, MMA
 // and two idle warps) gives registers back, the two softmax warpgroups take
-// them: 128 x 56 + 256 x 224 = 384 x 168. With the rotary embedding warps 2-3
-// rotate K tiles and need their registers (every split tried spilled more than
-// none), so those variants keep 168 each.
-constexpr int kRegsIssue = 56, kRegsSoftmax = 224;
-static_assert(128 * kRegsIssue + 256 * kRegsSoftmax <= kThreads * kLaunchRegs, "register split over budget");
+// them: 128 x 72 + 256 x 216 = 128 x 56 + 256 x 224 = 384 x 168 (d = 128 issues
+// twice the MMAs per tile and keeps its base descriptors live). With the rotary
+// embedding warps 2-3 rotate K tiles and need their registers (every split tried
+// spilled more than none), so those variants keep 168 each.
+template <int D>
+constexpr int kRegsIssue = D == 128 ? 72 : 56;
+template <int D>
+constexpr int kRegsSoftmax = D == 128 ? 216 : 224;
+static_assert(128 * kRegsIssue<128> + 256 * kRegsSoftmax<128> <= kThreads * kLaunchRegs, "register split over budget");
+static_assert(128 * kRegsIssue<64> + 256 * kRegsSoftmax<64> <= kThreads * kLaunchRegs, "register split over budget");
 
 // Kernel argument: the rotary table only for the ROPE variants.
 template <bool ROPE>
@@ -271,7 +276,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
     const uint32_t tmem = bars->tmem;
 
     if (warp < 4) {
-    if constexpr (!ROPE) setmaxnreg_dec<kRegsIssue>();
+    if constexpr (!ROPE) setmaxnreg_dec<kRegsIssue<D>>();
     if (warp == 0) {
         // ================================================= TMA producer
         if (lane == 0) {
@@ -285,27 +290,34 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
             for (int t = 0; t < 2; ++t)
                 load_tile<D>(smem_addr(smem + C::kQOff + t * C::kTileBytes), &tm_q, row_base + a0 + t * BM,
                              GQA ? bh * q_per_kv + member : bh, bq);
+            // group g = {V_{g-1}, K_g}: everything MMA iteration g reads, in stage g % 2
             int issued = 0;
-            for (int j = 0; j < n_kv_max && !aborted(bars); ++j) {
-                const bool ring = j < n_ring;
-                const int32_t row = ring ? ring_lo + j * BN : row_base + win_lo + (j - n_ring) * BN;
-                for (int part = 0; part < 2; ++part) {
-                    const int n = 2 * j + part, slot = n % kSlots, use = n / kSlots;
-                    if (use > 0 && !mbar_wait(smem_addr(&bars->kv_empty[slot]), (use - 1) & 1, kWaitNs)) {
-                        fail(bars, status);
-                        break;
-                    }
-                    const uint32_t bf = smem_addr(&bars->kv_full[slot]);
-                    mbar_expect_tx(bf, C::kTileBytes);
-                    const CUtensorMap* map = part == 0 ? (ring ? &tm_rk : &tm_k) : (ring ? &tm_rv : &tm_v);
-                    load_tile<D>(smem_addr(smem + C::kSlotOff + slot * C::kTileBytes), map, row, bh, bf);
-                    issued = n + 1;
+            for (int g = 0; g <= n_kv_max && !aborted(bars); ++g) {
+                const int st = g & 1, use = g >> 1;
+                if (use > 0 && !mbar_wait(smem_addr(&bars->kv_empty[st]), (use - 1) & 1, kWaitNs)) {
+                    fail(bars, status);
+                    break;
                 }
+                const uint32_t bf = smem_addr(&bars->kv_full[st]);
+                mbar_expect_tx(bf, (uint32_t)(((g >= 1) + (g < n_kv_max)) * C::kTileBytes));
+                const uint32_t sbase = smem_addr(smem + C::kSlotOff + 2 * st * C::kTileBytes);
+                if (g >= 1) {
+                    const int jv = g - 1;
+                    const bool ring = jv < n_ring;
+                    const int32_t row = ring ? ring_lo + jv * BN : row_base + win_lo + (jv - n_ring) * BN;
+                    load_tile<D>(sbase, ring ? &tm_rv : &tm_v, row, bh, bf);
+                }
+                if (g < n_kv_max) {
+                    const bool ring = g < n_ring;
+                    const int32_t row = ring ? ring_lo + g * BN : row_base + win_lo + (g - n_ring) * BN;
+                    load_tile<D>(sbase + C::kTileBytes, ring ? &tm_rk : &tm_k, row, bh, bf);
+                }
+                issued = g + 1;
             }
             // drain: every issued copy must land before the CTA can exit
             mbar_wait(smem_addr(&bars->q), 0, kWaitNs);
-            for (int n = (issued > kSlots ? issued - kSlots : 0); n < issued; ++n)
-                mbar_wait(smem_addr(&bars->kv_full[n % kSlots]), (n / kSlots) & 1, kWaitNs);
+            for (int g = (issued > 2 ? issued - 2 : 0); g < issued; ++g)
+                mbar_wait(smem_addr(&bars->kv_full[g & 1]), (g >> 1) & 1, kWaitNs);
         }
     } else if (warp == 1) {
         // ================================================= MMA issuer
@@ -315,35 +327,30 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
             bool ok = mbar_wait(smem_addr(ROPE ? &bars->q_rot : &bars->q), 0, kWaitNs);
             if (!ok) fail(bars, status);
             for (int j = 0; ok && j <= n_kv_max; ++j) {
-                int vslot = -1, kslot = -1;
-                if (j >= 1) {
-                    const int n = 2 * (j - 1) + 1;
-                    vslot = n % kSlots;
-                    if (!mbar_wait(smem_addr(&bars->kv_full[vslot]), (n / kSlots) & 1, kWaitNs)) { ok = false; break; }
-                }
-                if (j < n_kv_max) {
-                    const int n = 2 * j;
-                    kslot = n % kSlots;
-                    const uint32_t kbar = ROPE ? smem_addr(&bars->k_rot[kslot >> 1]) : smem_addr(&bars->kv_full[kslot]);
-                    if (!mbar_wait(kbar, (n / kSlots) & 1, kWaitNs)) { ok = false; break; }
-                }
+                const int st = j & 1;
+                // K_j of a rotary variant is ready once warps 2-3 have rotated it
+                // (they waited for the stage); V alone (the last group) on the stage
+                const uint32_t bar = (ROPE && j < n_kv_max) ? smem_addr(&bars->k_rot[st]) : smem_addr(&bars->kv_full[st]);
+                if (!mbar_wait(bar, (j >> 1) & 1, kWaitNs)) { ok = false; break; }
+                if (ROPE && j < n_kv_max && j >= 1 &&
+                    !mbar_wait(smem_addr(&bars->kv_full[st]), (j >> 1) & 1, kWaitNs)) { ok = false; break; }
+                const uint32_t vbase = sslot + 2 * st * C::kTileBytes, kbase = vbase + C::kTileBytes;
                 tc_fence_after();
                 for (int t = 0; t < 2; ++t) {
                     const int nkt = t == 0 ? n_kv0 : n_kv1;
                     if (j >= 1 && j - 1 < nkt) {              // O_t += P_t(j-1) V_{j-1}
                         if (!mbar_wait(smem_addr(&bars->p_full[t]), (j - 1) & 1, kWaitNs)) { ok = false; break; }
                         tc_fence_after();
-                        issue_pv<D>(tmem + 256 + t * D, tmem + t * 128, sslot + vslot * C::kTileBytes, j - 1 > 0);
+                        issue_pv<D>(tmem + 256 + t * D, tmem + t * 128, vbase, j - 1 > 0);
                         if (j - 1 == nkt - 1) mma_commit(smem_addr(&bars->o_full[t]));
                     }
                     if (j < nkt) {                           // S_t = Q_t K_j^T
-                        issue_qk<D>(tmem + t * 128, sq + t * C::kTileBytes, sslot + kslot * C::kTileBytes);
+                        issue_qk<D>(tmem + t * 128, sq + t * C::kTileBytes, kbase);
                         mma_commit(smem_addr(&bars->s_full[t]));
                     }
                 }
                 if (!ok) break;
-                if (vslot >= 0) mma_commit(smem_addr(&bars->kv_empty[vslot]));
-                if (kslot >= 0) mma_commit(smem_addr(&bars->kv_empty[kslot]));
+                mma_commit(smem_addr(&bars->kv_empty[st]));
             }
             if (!ok) fail(bars, status);
             // drain: all issued MMAs complete before TMEM is freed
@@ -362,8 +369,8 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
             rope_offsets(rope.t, 8 * jj, g, G, off, step);
             const double theta_own = tau < D / 2 ? rope.t.theta[tau] : 0.0;
             for (int j = 0; j < n_kv_max; ++j) {
-                const int n = 2 * j, slot = n % kSlots;
-                if (!mbar_wait(smem_addr(&bars->kv_full[slot]), (n / kSlots) & 1, kWaitNs)) {
+                const int st = j & 1, slot = 2 * st + 1;        // K_j: stage j % 2, second slot
+                if (!mbar_wait(smem_addr(&bars->kv_full[st]), (j >> 1) & 1, kWaitNs)) {
                     fail(bars, status);
                     break;
                 }
@@ -393,13 +400,13 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
                     fence_proxy_async_smem();
                     named_bar_sync(3, 64);
                 }
-                if (tau == 0) mbar_arrive(smem_addr(&bars->k_rot[slot >> 1]));
+                if (tau == 0) mbar_arrive(smem_addr(&bars->k_rot[st]));
             }
         }
     }
     } else {
         // ================================================= softmax / epilogue
-        if constexpr (!ROPE) setmaxnreg_inc<kRegsSoftmax>();
+        if constexpr (!ROPE) setmaxnreg_inc<kRegsSoftmax<D>>();
         const int t = (warp - 4) >> 2;                    // 0: warps 4-7, 1: warps 8-11
         const int quarter = warp & 3;                     // TMEM lanes this warp may access
         const int r = quarter * 32 + lane;                // row within the Q tile

@@ -74,11 +74,13 @@ __device__ __forceinline__ void load_tile(uint32_t dst, const CUtensorMap* map, 
 template <int D>
 __device__ __forceinline__ void issue_qk(uint32_t s_tmem, uint32_t qbase, uint32_t kbase) {
     constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, false, false);
+    // the start address is the descriptor's low field (address >> 4, shared
+    // addresses < 256 KB), so an offset is added to a base descriptor
+    const uint64_t dq = smem_desc_sw128(qbase, 16, 1024), dk = smem_desc_sw128(kbase, 16, 1024);
 #pragma unroll
     for (int kk = 0; kk < D / 16; ++kk) {
-        const uint32_t off = (kk / 4) * kBoxBytes + (kk % 4) * 32;
-        mma_ss(s_tmem, smem_desc_sw128(qbase + off, 16, 1024), smem_desc_sw128(kbase + off, 16, 1024), idesc,
-               kk > 0 ? 1u : 0u);
+        const uint32_t off = ((kk / 4) * kBoxBytes + (kk % 4) * 32) >> 4;
+        mma_ss(s_tmem, dq + off, dk + off, idesc, kk > 0 ? 1u : 0u);
     }
 }
 
@@ -88,10 +90,10 @@ __device__ __forceinline__ void issue_qk(uint32_t s_tmem, uint32_t qbase, uint32
 template <int D>
 __device__ __forceinline__ void issue_pv(uint32_t o_tmem, uint32_t p_tmem, uint32_t vbase, bool accumulate) {
     constexpr uint32_t idesc = idesc_bf16_f32(BM, D, false, true);
+    const uint64_t dv = smem_desc_sw128(vbase, kBoxBytes, 1024);
 #pragma unroll
     for (int kk = 0; kk < BN / 16; ++kk)
-        mma_ts(o_tmem, p_tmem + kk * 8, smem_desc_sw128(vbase + kk * 2048, kBoxBytes, 1024), idesc,
-               (accumulate || kk > 0) ? 1u : 0u);
+        mma_ts(o_tmem, p_tmem + kk * 8, dv + (uint64_t)(kk * 2048 >> 4), idesc, (accumulate || kk > 0) ? 1u : 0u);
 }
 
 // Online softmax of one S tile in the log2 domain for the row this thread owns:

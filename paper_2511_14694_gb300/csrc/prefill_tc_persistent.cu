@@ -8,10 +8,12 @@
 // rows [0, a]. Same warp roles and TMEM columns; what changes is that every
 // barrier phase runs on across items:
 //   warp 0     TMA producer: per item, Q tiles (once the previous item's last QK
-//              has completed: q_free), then K_j, V_j into the slot ring, whose
-//              slot and phase count on across items
-//   warp 1     MMA issuer: per item as in prefill_tc.cu; an item's first PV into
-//              O_t waits until the previous item's epilogue has read O_t (o_free)
+//              has completed: q_free), then one group per MMA iteration j, {V_{j-1},
+//              K_j}, into one of two stages of two slots each; one mbarrier per
+//              stage, whose phase counts on across items
+//   warp 1     MMA issuer: per item as in prefill_tc.cu, but with one stage wait
+//              and one stage release per iteration; an item's first PV into O_t
+//              waits until the previous item's epilogue has read O_t (o_free)
 //   warps 2-3  idle
 //   warps 4-11 softmax per tile (the shared softmax_tile), then the epilogue:
 //              O_t / l to bf16 through a per-warp staging buffer (the Q buffers may
@@ -19,6 +21,11 @@
 // Register split: warpgroup 0 keeps 104 registers (the item loops carry more state
 // than the one-item kernel's 56 allow without spills), the softmax warpgroups take
 // 200: 128 x 104 + 256 x 200 = 384 x 168.
+// The tensor core queues about one MMA ahead of its issuing thread, so every
+// instruction the issuer runs between MMA blocks (a satisfied mbarrier wait
+// costs ~100 cycles) leaves the pipe idle: hence the grouped stages (one wait
+// instead of two per iteration) and descriptors formed once per tile (issue_qk,
+// issue_pv).
 // Every mbarrier wait is bounded; on timeout the kernel reports
 // FOCUS_ERR_TIMEOUT, drains its own copies/MMAs (bounded), frees TMEM, returns.
 #include "prefill_tc_common.cuh"
@@ -140,7 +147,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
             prefetch_tmap(&tm_rk);
             prefetch_tmap(&tm_rv);
             const uint32_t bq = smem_addr(&bars->q);
-            int64_t n_issued = 0;                        // K/V loads issued (two per tile), across items
+            int64_t n_issued = 0;                        // K/V groups issued (one per MMA iteration), across items
             int it = 0;                                  // valid items started
             bool ok = true;
             for (int64_t k = 0; ok && k * (int64_t)gridDim.x < n_items && !aborted(bars); ++k) {
@@ -159,38 +166,43 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
                 for (int t = 0; t < 2; ++t)
                     load_tile<D>(smem_addr(smem + C::kQOff + t * C::kTileBytes), &tm_q, I.row_base + I.a0 + t * BM,
                                  qrow, bq);
-                for (int j = 0; j < I.n_kv_max; ++j) {
-                    const bool ring = j < I.n_ring;
-                    const int32_t row = ring ? j * BN : I.row_base + (j - I.n_ring) * BN;
-                    for (int part = 0; part < 2; ++part) {
-                        const int64_t n = n_issued;
-                        const int slot = (int)(n % kSlots);
-                        const int64_t use = n / kSlots;
-                        if (use > 0 && !mbar_wait(smem_addr(&bars->kv_empty[slot]), (uint32_t)((use - 1) & 1),
-                                                  kWaitNs)) {
-                            fail(bars, status);
-                            ok = false;
-                            break;
-                        }
-                        const uint32_t bf = smem_addr(&bars->kv_full[slot]);
-                        mbar_expect_tx(bf, C::kTileBytes);
-                        const CUtensorMap* map = part == 0 ? (ring ? &tm_rk : &tm_k) : (ring ? &tm_rv : &tm_v);
-                        load_tile<D>(smem_addr(smem + C::kSlotOff + slot * C::kTileBytes), map, row, I.bh, bf);
-                        n_issued = n + 1;
+                // group g = {V_{g-1}, K_g}: everything MMA iteration g reads, in one stage
+                for (int g = 0; g <= I.n_kv_max; ++g) {
+                    const int64_t n = n_issued;
+                    const int st = (int)(n & 1);
+                    const int64_t use = n >> 1;
+                    if (use > 0 && !mbar_wait(smem_addr(&bars->kv_empty[st]), (uint32_t)((use - 1) & 1), kWaitNs)) {
+                        fail(bars, status);
+                        ok = false;
+                        break;
                     }
-                    if (!ok) break;
+                    const uint32_t bf = smem_addr(&bars->kv_full[st]);
+                    mbar_expect_tx(bf, (uint32_t)(((g >= 1) + (g < I.n_kv_max)) * C::kTileBytes));
+                    const uint32_t sbase = smem_addr(smem + C::kSlotOff + 2 * st * C::kTileBytes);
+                    if (g >= 1) {
+                        const int jv = g - 1;
+                        const bool ring = jv < I.n_ring;
+                        const int32_t row = ring ? jv * BN : I.row_base + (jv - I.n_ring) * BN;
+                        load_tile<D>(sbase, ring ? &tm_rv : &tm_v, row, I.bh, bf);
+                    }
+                    if (g < I.n_kv_max) {
+                        const bool ring = g < I.n_ring;
+                        const int32_t row = ring ? g * BN : I.row_base + (g - I.n_ring) * BN;
+                        load_tile<D>(sbase + C::kTileBytes, ring ? &tm_rk : &tm_k, row, I.bh, bf);
+                    }
+                    n_issued = n + 1;
                 }
                 ++it;
             }
             // drain: every issued copy must land before the CTA can exit
             if (it > 0) mbar_wait(bq, (it - 1) & 1, kWaitNs);
-            for (int64_t n = (n_issued > kSlots ? n_issued - kSlots : 0); n < n_issued; ++n)
-                mbar_wait(smem_addr(&bars->kv_full[n % kSlots]), (uint32_t)((n / kSlots) & 1), kWaitNs);
+            for (int64_t n = (n_issued > 2 ? n_issued - 2 : 0); n < n_issued; ++n)
+                mbar_wait(smem_addr(&bars->kv_full[n & 1]), (uint32_t)((n >> 1) & 1), kWaitNs);
         } else if (warp == 1 && lane == 0) {
             // ============================================= MMA issuer
             const uint32_t sq = smem_addr(smem + C::kQOff);
             const uint32_t sslot = smem_addr(smem + C::kSlotOff);
-            int64_t nt0 = 0;                 // K/V tiles consumed before this item
+            int64_t nt0 = 0;                 // K/V groups consumed before this item
             int it = 0;                      // valid items
             int pc[2] = {0, 0};              // P tiles consumed per Q tile (p_full phases)
             int oc[2] = {0, 0};              // items with an epilogue per Q tile (o_free phases)
@@ -202,23 +214,13 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
                 if (!I.valid) continue;
                 if (!mbar_wait(smem_addr(&bars->q), it & 1, kWaitNs)) { ok = false; break; }
                 for (int j = 0; ok && j <= I.n_kv_max; ++j) {
-                    int vslot = -1, kslot = -1;
-                    if (j >= 1) {
-                        const int64_t n = 2 * (nt0 + j - 1) + 1;
-                        vslot = (int)(n % kSlots);
-                        if (!mbar_wait(smem_addr(&bars->kv_full[vslot]), (uint32_t)((n / kSlots) & 1), kWaitNs)) {
-                            ok = false;
-                            break;
-                        }
+                    const int64_t n = nt0 + j;                 // this iteration's group
+                    const int st = (int)(n & 1);
+                    if (!mbar_wait(smem_addr(&bars->kv_full[st]), (uint32_t)((n >> 1) & 1), kWaitNs)) {
+                        ok = false;
+                        break;
                     }
-                    if (j < I.n_kv_max) {
-                        const int64_t n = 2 * (nt0 + j);
-                        kslot = (int)(n % kSlots);
-                        if (!mbar_wait(smem_addr(&bars->kv_full[kslot]), (uint32_t)((n / kSlots) & 1), kWaitNs)) {
-                            ok = false;
-                            break;
-                        }
-                    }
+                    const uint32_t vbase = sslot + 2 * st * C::kTileBytes, kbase = vbase + C::kTileBytes;
                     tc_fence_after();
                     for (int t = 0; t < 2; ++t) {
                         const int nkt = t == 0 ? I.n_kv0 : I.n_kv1;
@@ -233,23 +235,22 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
                             if (!mbar_wait(smem_addr(&bars->p_full[t]), pc[t] & 1, kWaitNs)) { ok = false; break; }
                             ++pc[t];
                             tc_fence_after();
-                            issue_pv<D>(tmem + 256 + t * D, tmem + t * 128, sslot + vslot * C::kTileBytes, j - 1 > 0);
+                            issue_pv<D>(tmem + 256 + t * D, tmem + t * 128, vbase, j - 1 > 0);
                             if (j - 1 == nkt - 1) {
                                 mma_commit(smem_addr(&bars->o_full[t]));
                                 ++oc[t];
                             }
                         }
                         if (j < nkt) {                           // S_t = Q_t K_j^T
-                            issue_qk<D>(tmem + t * 128, sq + t * C::kTileBytes, sslot + kslot * C::kTileBytes);
+                            issue_qk<D>(tmem + t * 128, sq + t * C::kTileBytes, kbase);
                             mma_commit(smem_addr(&bars->s_full[t]));
                         }
                     }
                     if (!ok) break;
                     if (j == I.n_kv_max - 1) mma_commit(smem_addr(&bars->q_free));   // last QK of the item issued
-                    if (vslot >= 0) mma_commit(smem_addr(&bars->kv_empty[vslot]));
-                    if (kslot >= 0) mma_commit(smem_addr(&bars->kv_empty[kslot]));
+                    mma_commit(smem_addr(&bars->kv_empty[st]));
                 }
-                nt0 += I.n_kv_max;
+                nt0 += I.n_kv_max + 1;
                 ++it;
             }
             if (!ok) fail(bars, status);
