@@ -18,7 +18,9 @@
 //
 // CTA = two 128-row Q tiles of one (sequence, head, window) that share every
 // K/V tile, 12 warps in three warpgroups:
-//   warp 0     TMA producer: Q tiles once, then K_j, V_j into a ring of slots
+//   warp 0     TMA producer: Q tiles once, then per MMA iteration j the group
+//              {V_{j-1}, K_j} into one of two stages (one full/empty mbarrier pair
+//              per stage, so the issuer waits once per iteration)
 //   warp 1     TMEM owner + MMA issuer (one thread):
 //                S_t = Q_t K_j^T            (SS, both operands K-major, SW128)
 //                O_t += P_t V_j             (TS, P_t in TMEM over S_t, V MN-major)
@@ -33,7 +35,7 @@
 //
 // Rotary embedding (ROPE): the softmax warps rotate the two Q tiles in shared
 // memory before the first S = Q K^T (q_rot barrier), and warps 2-3 rotate each
-// window K tile between its TMA arrival and its MMA (k_rot barriers); ring tiles
+// window K tile between its stage's arrival and its MMA (k_rot, one per stage); ring tiles
 // arrive rotated. Each rotating thread owns eight column pairs (i, i + d/2) of a
 // set of rows spaced G apart: one fp64 angle per pair and tile (or 64-row
 // segment) start, then the fixed per-row offsets of a host table.
@@ -192,7 +194,6 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
         int64_t T_span, const int32_t* __restrict__ win_off, const int32_t* __restrict__ ring_off, int32_t w_begin,
         int32_t w_end, int32_t ctas_pw, int32_t H, int32_t C_ring, float scale_log2, int32_t* status,
         const int32_t* __restrict__ k_per_window, const __grid_constant__ RopeArg<ROPE> rope, int32_t q_per_kv) {
-    static_assert(!ROPE || kSlots == 4, "K tiles must use the even slots");
     using C = Cfg<D>;
     extern __shared__ unsigned char smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -250,7 +251,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
     // ---- setup -------------------------------------------------------------
     if (threadIdx.x == 0) {
         mbar_init(smem_addr(&bars->q), 1);
-        for (int s = 0; s < kSlots; ++s) {
+        for (int s = 0; s < kStages; ++s) {
             mbar_init(smem_addr(&bars->kv_full[s]), 1);
             mbar_init(smem_addr(&bars->kv_empty[s]), 1);
         }

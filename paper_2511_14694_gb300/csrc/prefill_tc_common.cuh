@@ -17,7 +17,8 @@ using namespace sm100;
 
 constexpr int BM = 128;             // rows per Q tile
 constexpr int BN = 128;             // keys per K/V tile
-constexpr int kSlots = 4;           // K/V staging slots (each holds one K or one V tile)
+constexpr int kStages = 2;          // K/V stages, each one MMA iteration's {V_{j-1}, K_j}
+constexpr int kSlots = 2 * kStages; // K/V tiles in shared memory (stage s: slots 2s (V) and 2s + 1 (K))
 constexpr int kThreads = 384;       // 12 warps
 constexpr int kLaunchRegs = 168;    // registers per thread at launch: 65,536 / 384 rounded down to 8
 constexpr int kBoxBytes = 128 * 128;   // one TMA box: 128 rows x 64 bf16 (128 B, swizzled)
@@ -40,14 +41,14 @@ struct Cfg {
 
 struct Bars {
     uint64_t q;
-    uint64_t kv_full[kSlots];
-    uint64_t kv_empty[kSlots];
+    uint64_t kv_full[kStages];   // stage landed (TMA complete_tx)
+    uint64_t kv_empty[kStages];  // the stage's MMAs have completed
     uint64_t s_full[2];
     uint64_t p_full[2];
     uint64_t o_full[2];
     uint64_t drain;
     uint64_t q_rot;       // rotary embedding: the Q tiles are rotated
-    uint64_t k_rot[2];    // rotary embedding: the K tile in slot 0 / 2 is rotated (K tiles use the even slots)
+    uint64_t k_rot[kStages];  // rotary embedding: the K tile of the stage is rotated
     uint64_t o_free[2];   // persistent: the epilogue has read O_t
     uint64_t q_free;      // persistent: every QK of the current item has completed, Q may be reloaded
     uint32_t tmem;

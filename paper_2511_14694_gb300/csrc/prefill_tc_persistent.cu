@@ -114,7 +114,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
     if (threadIdx.x == 0) {
         mbar_init(smem_addr(&bars->q), 1);
         mbar_init(smem_addr(&bars->q_free), 1);
-        for (int s = 0; s < kSlots; ++s) {
+        for (int s = 0; s < kStages; ++s) {
             mbar_init(smem_addr(&bars->kv_full[s]), 1);
             mbar_init(smem_addr(&bars->kv_empty[s]), 1);
         }
