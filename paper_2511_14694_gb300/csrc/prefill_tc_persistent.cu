@@ -10,7 +10,9 @@
 //   warp 0     TMA producer: per item, Q tiles (once the previous item's last QK
 //              has completed: q_free), then one group per MMA iteration j, {V_{j-1},
 //              K_j}, into one of two stages of two slots each; one mbarrier per
-//              stage, whose phase counts on across items
+//              stage, whose phase counts on across items. After an item's first
+//              group it forms the next item's geometry and prefetches that item's
+//              Q tiles into L2, so the Q load after q_free does not wait on DRAM
 //   warp 1     MMA issuer: per item as in prefill_tc.cu, but with one stage wait
 //              and one stage release per iteration; an item's first PV into O_t
 //              waits until the previous item's epilogue has read O_t (o_free)
@@ -108,6 +110,20 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
     auto snake_item = [&](int64_t k) {
         return k * (int64_t)gridDim.x + ((k & 1) ? (int64_t)(gridDim.x - 1 - blockIdx.x) : (int64_t)blockIdx.x);
     };
+    // the first valid item of round k or later (k is left at its round); .valid is
+    // false when none is left. cap_report: report items beyond the capacities.
+    auto next_valid = [&](int64_t& k, bool cap_report) {
+        ItemGeom I;
+        I.valid = false;
+        for (; k * (int64_t)gridDim.x < n_items; ++k) {
+            const int64_t idx = snake_item(k);
+            if (idx >= n_items) continue;
+            I = geom(idx);
+            if (cap_report && I.cap_err) report(status, FOCUS_ERR_CAPACITY);
+            if (I.valid) break;
+        }
+        return I;
+    };
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     // ---- setup (once per CTA) -------------------------------------------------
@@ -150,12 +166,12 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
             int64_t n_issued = 0;                        // K/V groups issued (one per MMA iteration), across items
             int it = 0;                                  // valid items started
             bool ok = true;
-            for (int64_t k = 0; ok && k * (int64_t)gridDim.x < n_items && !aborted(bars); ++k) {
-                const int64_t idx = snake_item(k);
-                if (idx >= n_items) continue;
-                const ItemGeom I = geom(idx);
-                if (I.cap_err) report(status, FOCUS_ERR_CAPACITY);
-                if (!I.valid) continue;
+            int64_t k = 0;
+            ItemGeom I = next_valid(k, true);
+            while (ok && I.valid && !aborted(bars)) {
+                int64_t kn = k + 1;
+                ItemGeom N;
+                N.valid = false;
                 // the Q buffers are free once every QK MMA of the previous item has completed
                 if (it > 0 && !mbar_wait(smem_addr(&bars->q_free), (it - 1) & 1, kWaitNs)) {
                     fail(bars, status);
@@ -191,8 +207,21 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
                         load_tile<D>(sbase + C::kTileBytes, ring ? &tm_rk : &tm_k, row, I.bh, bf);
                     }
                     n_issued = n + 1;
+                    if (g == 0) {
+                        // the next item, and its Q tiles into L2 while this item runs
+                        N = next_valid(kn, true);
+                        if (N.valid) {
+                            const int32_t nq = GQA ? N.bh * q_per_kv + N.member : N.bh;
+                            for (int t = 0; t < 2; ++t)
+#pragma unroll
+                                for (int x = 0; x < D / 64; ++x)
+                                    tma_prefetch_3d(&tm_q, x * 64, N.row_base + N.a0 + t * BM, nq);
+                        }
+                    }
                 }
                 ++it;
+                I = N;
+                k = kn;
             }
             // drain: every issued copy must land before the CTA can exit
             if (it > 0) mbar_wait(bq, (it - 1) & 1, kWaitNs);
