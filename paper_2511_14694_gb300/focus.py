@@ -417,6 +417,7 @@ def attn_decode_noalloc(cache: Cache, q, k_new, v_new, scale=None, o=None, lse=N
     lib = load()
     for name, t in (("q", q), ("k_new", k_new), ("v_new", v_new)):
         _cuda(t, name, torch.bfloat16)
+    _check_heads(cache, q, k_new, v_new)
     if o is None:
         o = torch.empty_like(q)
     if lse is None:

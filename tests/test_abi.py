@@ -262,3 +262,25 @@ def test_cache_snapshot_restore_round_trip():
     c.win_fill.fill_(0)
     c.restore(snap)
     assert bool((c.ring_k == 1.0).all()) and bool((c.win_fill == 2).all())
+
+
+def test_decode_bindings_check_head_counts_before_any_call(monkeypatch):
+    # q must have H * q_per_kv heads and k_new/v_new H: a mismatch is a ValueError
+    # raised on the host, before the library is called (a short q or o would be
+    # read or written past its end by the kernels)
+    import torch
+
+    class NoLib:
+        def __getattr__(self, name):
+            raise AssertionError(f"{name} called despite mismatched heads")
+
+    monkeypatch.setattr(focus, "load", lambda: NoLib())
+    monkeypatch.setattr(focus, "_cuda", lambda t, name, dtype=None: t)
+    cache = type("C", (), {"H": 4, "q_per_kv": 4})()
+    q = torch.zeros((2, 4, 128), dtype=torch.bfloat16)         # should be 16 query heads
+    kv = torch.zeros((2, 4, 128), dtype=torch.bfloat16)
+    for fn in (focus.attn_decode_noalloc, focus.attn_decode):
+        with pytest.raises(ValueError, match="heads"):
+            fn(cache, q, kv, kv)
+    with pytest.raises(ValueError, match="heads"):
+        focus.attn_decode_noalloc(cache, torch.zeros((2, 16, 128)), kv[:, :2], kv)

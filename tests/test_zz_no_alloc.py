@@ -20,30 +20,37 @@ from paper_2511_14694_gb300 import focus, inputs
 pytestmark = pytest.mark.gpu
 
 
-def _cache_pair(B, H, d, R, fill, C_ring, C_win, W, k):
+def _cache_pair(B, H, d, R, fill, C_ring, C_win, W, k, g, rope):
     caches = []
     for _ in range(2):
-        c = focus.Cache(B, H, d, C_ring=C_ring, C_win=C_win, W=W, k_sched=[k] * 64)
+        c = focus.Cache(B, H, d, C_ring=C_ring, C_win=C_win, W=W, k_sched=[k] * 64, q_per_kv=g, rope_theta=rope)
         for i, t in enumerate((c.ring_k, c.ring_v, c.win_k, c.win_v)):
             t.copy_(inputs.normal_bf16(t.shape, 1.0, seed=70 + i, device="cuda"))
         c.ring_len.fill_(R)
         c.win_idx.fill_(3)
         c.win_fill.copy_(torch.from_numpy(np.asarray(fill, np.int32)))
+        c.pos_base.fill_(3 * (W + -(-W // k)))
         caches.append(c)
     return caches
 
 
-def test_noalloc_decode_matches_workspace_decode_on_consecutive_calls():
+# (query heads per K/V head, rotary base): the CUDA-core split kernel without
+# rotation, and the grouped-query tensor-core kernel with the rotated q/k rows
+# that the library also keeps in its fixed array
+@pytest.mark.parametrize("g,rope", [(1, 0.0), (4, 1e4)])
+def test_noalloc_decode_matches_workspace_decode_on_consecutive_calls(g, rope):
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
     focus.device_status(clear=True)
     B, H, d, W, k = 8, 4, 128, 1_000, 100
     fill = [0, 5, 1_008, 1_009, 300, 999, 17, 640]        # two sequences finish their window
-    ref, noalloc = _cache_pair(B, H, d, 2_000, fill, C_ring=2_100, C_win=1_024, W=W, k=k)
+    ref, noalloc = _cache_pair(B, H, d, 2_000, fill, C_ring=2_100, C_win=1_024, W=W, k=k, g=g, rope=rope)
     assert ref.workspace_bytes() <= (16 << 20)
     ws = ref.new_workspace()
     for step in range(2):
-        q, kn, vn = inputs.qkv((B, H, d), seed=500 + step, device="cuda")
+        q = inputs.normal_bf16((B, H * g, d), 1.0, seed=500 + step, device="cuda")
+        kn = inputs.normal_bf16((B, H, d), 1.0, seed=600 + step, device="cuda")
+        vn = inputs.normal_bf16((B, H, d), 1.0, seed=700 + step, device="cuda")
         o_ref, lse_ref = focus.attn_decode(ref, q, kn, vn, workspace=ws)
         focus.kv_compact_window(ref)
         o_na, lse_na = focus.attn_decode_noalloc(noalloc, q, kn, vn)
@@ -53,9 +60,10 @@ def test_noalloc_decode_matches_workspace_decode_on_consecutive_calls():
         lerr = ((lse_na - lse_ref).abs() / lse_ref.abs().clamp(min=1.0)).max().item()
         assert err <= 2e-2 and lerr <= 1e-3, (step, err, lerr)
         for a, b in ((ref.ring_len, noalloc.ring_len), (ref.win_fill, noalloc.win_fill),
-                     (ref.win_idx, noalloc.win_idx)):
+                     (ref.win_idx, noalloc.win_idx), (ref.pos_base, noalloc.pos_base)):
             assert torch.equal(a, b)
-    assert torch.equal(ref.ring_k, noalloc.ring_k) and torch.equal(ref.win_v, noalloc.win_v)
+    assert torch.equal(ref.ring_k, noalloc.ring_k) and torch.equal(ref.win_k, noalloc.win_k)
+    assert torch.equal(ref.win_v, noalloc.win_v)
     assert focus.device_status(clear=True) == 0
 
 
