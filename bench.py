@@ -211,68 +211,61 @@ def weak_scaling_value(units_per_rank: float, world: int, max_seconds: float) ->
 
 # ----------------------------------------------------------------------------- oracle (CPU baseline)
 
-def oracle_prefill_sample(cfg, L_host, q, k, v, budget_s=12.0, max_windows=None):
-    """Times the fp64 oracle's sequential prefill on a bounded sample of the
-    workload (a subset of heads and evenly spaced windows) and extrapolates to
-    the whole workload by visible pairs. Returns (seconds for the full workload,
-    description, cores)."""
+def oracle_head_times(cfg, L_host, k_sched, q, k, v, n_heads, mask="appendix"):
+    """Times the fp64 oracle on whole heads of the workload: every window and
+    every row of one (sequence, head) per pass, the sequential form of App. A.1
+    for the appendix mask or every row under the k-mer-local mask of Sec. 3.2.
+    Each (sequence, head) has the same visible pairs, so the whole workload takes
+    B x H x the seconds of one pass. q/k/v hold a few heads' inputs, cycled (the
+    timing does not depend on the values). Returns the per-pass seconds."""
     from oracle import focus_oracle as fo
-    win_off, ring_off, keep = L_host["win_off"], L_host["ring_off"], L_host["keep"]
-    M = win_off.size - 1
-    d = cfg["d"]
-    total_pairs = visible_pairs(win_off, ring_off) * cfg["B"] * cfg["H"]
-    Tw = np.diff(win_off.astype(np.int64))
-    pairs_w = Tw * (Tw + 1) // 2 + Tw * ring_off[:-1].astype(np.int64)
-    # grow the sample until it takes about budget_s
-    n_w, spent, done_pairs, heads_done = 1, 0.0, 0, 0
-    h = 0
-    while spent < budget_s and heads_done < cfg["H"]:
-        step = max(1, M // n_w)
-        want = np.zeros(M, np.uint8)
-        want[::step] = 1
-        if max_windows:
-            want[np.nonzero(want)[0][max_windows:]] = 0
+    win_off = L_host["win_off"]
+    scale = 1.0 / math.sqrt(cfg["d"])
+    rows = None
+    if mask == "kmer_local":
+        rows = np.arange(int(win_off[-1]), dtype=np.int64)
+    secs = []
+    for i in range(n_heads):
+        h = i % q.shape[0]
         t0 = time.perf_counter()
-        fo.prefill_sequential(q[h], k[h], v[h], win_off, keep, 1.0 / math.sqrt(d), want=want)
-        spent += time.perf_counter() - t0
-        done_pairs += int(pairs_w[want.astype(bool)].sum())
-        heads_done += 1
-        h = (h + 1) % q.shape[0]
-        n_w = min(M, n_w * 2)
-    full_s = spent * total_pairs / max(done_pairs, 1)
-    desc = (f"fp64 oracle sequential prefill on {heads_done} head-passes over evenly spaced windows "
-            f"({done_pairs:,} of {total_pairs:,} visible pairs, {spent:.1f} s), extrapolated by visible pairs")
-    return full_s, desc, os.cpu_count()
+        if mask == "kmer_local":
+            fo.attn_rows_kmer_local(q[h:h + 1], k[h:h + 1], v[h:h + 1], L_host["kind"], L_host["win"],
+                                    L_host["kmer"], scale, np.zeros(rows.size, np.int64), rows)
+        else:
+            fo.prefill_sequential(q[h], k[h], v[h], win_off, L_host["keep"], scale)
+        secs.append(time.perf_counter() - t0)
+    return secs
 
 
-def oracle_local_sample(cfg, L_host, k_sched, q, k, v, budget_s=12.0, max_windows=None):
-    """As oracle_prefill_sample, for the k-mer-local mask: the oracle's
-    attn_rows_kmer_local over all rows of evenly spaced windows, one head per
-    pass, extrapolated by visible pairs."""
-    from oracle import focus_oracle as fo
-    win_off, ring_off = L_host["win_off"], L_host["ring_off"]
-    M = win_off.size - 1
-    d = cfg["d"]
-    counts = kmer_local_row_counts(win_off, ring_off, k_sched)
-    total_pairs = int(counts.sum()) * cfg["B"] * cfg["H"]
-    n_w, spent, done_pairs, heads_done, h = 1, 0.0, 0, 0, 0
-    while spent < budget_s and heads_done < cfg["H"]:
-        ws = np.arange(0, M, max(1, M // n_w))
-        if max_windows:
-            ws = ws[:max_windows]
-        rows = np.concatenate([np.arange(win_off[w], win_off[w + 1]) for w in ws]).astype(np.int64)
-        t0 = time.perf_counter()
-        fo.attn_rows_kmer_local(q[h:h + 1], k[h:h + 1], v[h:h + 1], L_host["kind"], L_host["win"], L_host["kmer"],
-                                1.0 / math.sqrt(d), np.zeros(rows.size, np.int64), rows)
-        spent += time.perf_counter() - t0
-        done_pairs += int(counts[rows].sum())
-        heads_done += 1
-        h = (h + 1) % q.shape[0]
-        n_w = min(M, n_w * 2)
-    full_s = spent * total_pairs / max(done_pairs, 1)
-    desc = (f"fp64 oracle k-mer-local attention on {heads_done} head-passes over evenly spaced windows "
-            f"({done_pairs:,} of {total_pairs:,} visible pairs, {spent:.1f} s), extrapolated by visible pairs")
-    return full_s, desc, os.cpu_count()
+def oracle_baseline(cfg, secs, mask):
+    """(nt/s of the whole workload, description) from per-head oracle passes."""
+    per_head = statistics.median(secs)
+    full_s = per_head * cfg["B"] * cfg["H"]
+    desc = ("fp64 oracle (%s), %d whole (sequence, head) passes of %d, every window and row; %.3f s per pass "
+            "(median); the workload's %d passes do the same visible pairs each, so its time is %d x that "
+            "(extrapolated by passes)" % ("k-mer-local rows" if mask == "kmer_local" else "sequential prefill",
+                                          len(secs), cfg["B"] * cfg["H"], per_head, cfg["B"] * cfg["H"],
+                                          cfg["B"] * cfg["H"]))
+    return cfg["B"] * cfg["N"] / full_s, desc, full_s
+
+
+def workload_config(args, cfg, T, R, name=None, mask=None, rope=None, q_per_kv=None):
+    """The config object of a bench line: the workload's shape, identical for the
+    library arm and the reference (oracle) arm."""
+    mask = args.mask if mask is None else mask
+    rope = args.rope if rope is None else rope
+    g = args.q_per_kv if q_per_kv is None else q_per_kv
+    if cfg["mode"] == "stream":
+        tw = T // max(1, -(-cfg["N"] // cfg["W"]))
+        l2 = "inputs larger than L2 (pool of %d windows' Q/K/V %.2f GB, ring %.2f GB)" % (
+            cfg["pool"], 3 * cfg["pool"] * cfg["B"] * cfg["H"] * tw * cfg["d"] * 2 / 1e9,
+            2 * cfg["B"] * cfg["H"] * R * cfg["d"] * 2 / 1e9)
+    else:
+        l2 = "inputs larger than L2 (Q/K/V %.2f GB per step)" % (3 * cfg["B"] * T * cfg["H"] * cfg["d"] * 2 / 1e9)
+    return {"workload": name or args.workload, "B": cfg["B"], "N": cfg["N"], "W": cfg["W"], "k": list(cfg["k"]),
+            "H": cfg["H"], "d": cfg["d"], "T_augmented": int(T), "R_retained": int(R),
+            "mask": "k-mer-local (Sec. 3.2)" if mask == "kmer_local" else "appendix (App. A, Eq. focus-attn)",
+            "rope_theta": rope or None, "q_per_kv": g, "l2": l2}
 
 
 # ----------------------------------------------------------------------------- focus arm
@@ -393,7 +386,8 @@ def run_prefill_leg(args, cfg, world, rank, local):
         host_sample = dict(win_off=win_off, ring_off=ring_off, kind=L["kind"].cpu().numpy(),
                            win=L["win"].cpu().numpy(), keep=L["keep"].cpu().numpy(), k_sched=k_s,
                            q=q[0, :2].cpu(), k=k[0, :2].cpu(), v=v[0, :2].cpu())
-    res = dict(kernel=kernel_name,
+    res = dict(kernel=kernel_name, attn_launches_per_step=1,
+               step_desc="focus_layout + focus_kv_compact(bulk) + focus_attn_prefill(masked-parallel)",
                step_ms=step_ms, attn_ms=attn_ms, flops_per_step=flops_per_step, pairs=pairs, T=L["T"], R=L["R"],
                bytes_per_step=bytes_per_step, local_mask=local_mask, compact_ms=compact_ms,
                compact_bytes=compact_bytes,
@@ -436,11 +430,14 @@ def run_stream_leg(args, cfg, world, rank, local):
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(M)]
     kernel_name = focus.prefill_kernel(cache, pq[0], pk[0], pv[0], L, M - 1, M, flags=args.prefill_flags, o=outs[0])
 
+    cevs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(M)]
+
     def step(timed=False):
         # each window's compaction, then its attention on one of two side streams:
         # consecutive windows' launches overlap (pipeline.prefill_streaming)
         pipeline.prefill_streaming(cache, L, lambda w: (pq[w % P], pk[w % P], pv[w % P]), outs, lses,
-                                   flags=args.prefill_flags, stream=stream, events=evs if timed else None)
+                                   flags=args.prefill_flags, stream=stream, events=evs if timed else None,
+                                   compact_events=cevs if timed else None)
 
     for _ in range(args.warmup):
         step()
@@ -449,7 +446,7 @@ def run_stream_leg(args, cfg, world, rank, local):
     pairs = (int(kmer_local_row_counts(off, L["ring_off_host"], k_s).sum()) if local_mask
              else visible_pairs(off, L["ring_off_host"]))
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    attn_ms = 0.0
+    attn_ms = compact_ms = 0.0
     barrier(world)
     with ClockSampler(local) as clk:
         t0.record(stream)
@@ -457,14 +454,37 @@ def run_stream_leg(args, cfg, world, rank, local):
             step(timed=True)
             torch.cuda.synchronize(dev)
             attn_ms += sum(a.elapsed_time(b) for a, b in evs)
+            compact_ms += sum(a.elapsed_time(b) for a, b in cevs)
         t1.record(stream)
         torch.cuda.synchronize(dev)
     barrier(world)
+    # the window compaction alone (nothing else running): re-copies windows' kept
+    # rows to the ring slots they already hold
+    n_alone = min(M, 100)
+    aev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_alone)]
+    for w, (a, b) in enumerate(aev):
+        a.record(stream)
+        focus.kv_compact_bulk(cache, pk[w % P], pv[w % P], L, w, w + 1, src_row0=int(off[w]), stream=stream)
+        b.record(stream)
+    torch.cuda.synchronize(dev)
+    alone_ms = statistics.median(a.elapsed_time(b) for a, b in aev)
     assert focus.device_status(clear=True) == 0
     step_ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, world)
     # the attention launches overlap, so the rate is taken over the whole step
     # (compactions and gaps included); per_launch_ms is each launch on its stream
-    return dict(kernel=kernel_name,
+    # per-window compaction: the window's kept rows of every (sequence, K/V head), read and written
+    wc_ms = compact_ms / args.steps / M
+    wc_bytes = float((L["R"] / M) * B * (H // g) * 2 * (2 * d) * 2)
+    return dict(kernel=kernel_name, attn_launches_per_step=M,
+                step_desc=("per window: focus_kv_compact(window) + focus_attn_prefill(window), consecutive "
+                           "windows' attention overlapping on two streams; all windows; rate over the whole step"),
+                window_compaction={"kernel": "focus_kv_compact (one window)", "bytes_per_launch": wc_bytes,
+                                   "in_step_ms": wc_ms,
+                                   "in_step_note": "CUDA events on the main stream inside the step: includes "
+                                                   "waiting for SMs held by the overlapping attention launches",
+                                   "alone_ms": alone_ms, "alone_GBps": wc_bytes / (alone_ms / 1e3) / 1e9,
+                                   "alone_note": "median of %d launches with nothing else running: a ~1 MB "
+                                                 "launch, launch-latency bound" % n_alone},
                 step_ms=step_ms, attn_ms=step_ms, flops_per_step=4.0 * d * H * B * pairs, pairs=pairs,
                 T=L["T"], R=L["R"], clocks=clk.summary(), launches=2 * M * args.steps, e2e=None, host_sample=None,
                 per_launch_ms=attn_ms / args.steps / M, local_mask=local_mask,
@@ -584,6 +604,100 @@ def run_decode_leg(args, cfg, world, rank, local):
                 clocks=clk.summary(), launches=3 * S * reps)
 
 
+def prefill_roofline(pre, peaks, peaks_src, traffic=None):
+    """Roofline object of a prefill leg's attention kernel: visible-pair FLOPs
+    (appendix mask) or bytes (k-mer-local mask, a few keys per row) per launch
+    over the average launch time."""
+    n_launch = pre["attn_launches_per_step"]
+    achieved = pre["flops_per_step"] / (pre["attn_ms"] / 1e3) / 1e12
+    common = {"traffic": traffic, "visible_pairs": pre["pairs"], "avg_launch_ms": pre.get("per_launch_ms",
+                                                                                         pre["attn_ms"]),
+              "launches_per_step": n_launch, "flop_per_launch": pre["flops_per_step"] / n_launch,
+              "prefill_kernel": pre["kernel"]}
+    if pre["local_mask"]:
+        gbs = pre["bytes_per_step"] / (pre["attn_ms"] / 1e3) / 1e9
+        r = {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": gbs / peaks["hbm_gbs"],
+             "peak_source": f"{peaks_src} copy bandwidth", "kernel": "prefill attention (k-mer-local)",
+             "tflops": achieved, "bytes_per_launch": pre["bytes_per_step"] / n_launch}
+    else:
+        r = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+             "frac": achieved / peaks["bf16_tflops"], "peak_source": f"{peaks_src} bf16 dense burst",
+             "frac_of_sustained": achieved / peaks["bf16_tflops_sustained"], "kernel": "prefill attention"}
+    r.update(common)
+    if pre.get("rotate_ms") is not None:
+        r["rotation_pass_ms"] = pre["rotate_ms"]
+    return r
+
+
+# the other named workloads timed beside the headline: (key, workload, steps, warm-up)
+CONFIG_LEGS = [("ksweep", "prefill_256kb_ksweep_h32_d128", 10, 3),
+               ("causal", "causal_128kb_h32_d128", 3, 3),
+               ("stream", "stream_1mb_b4_h32_d128", 2, 3)]
+
+
+def run_config_leg(args, name, steps, warmup, world, rank, local, peaks, peaks_src):
+    """One of the other named workloads at the default options (appendix mask,
+    no rotary embedding, one query head per K/V head), timed like the headline
+    step; returns its object for the bench line."""
+    import copy
+    from paper_2511_14694_gb300.workloads import WORKLOADS
+    cfg = WORKLOADS[name]
+    a = copy.copy(args)
+    a.steps, a.warmup, a.no_e2e, a.no_cpu_baseline = steps, warmup, True, True
+    a.rope, a.q_per_kv, a.mask, a.prefill_flags = 0.0, 1, "appendix", 0
+    pre = (run_stream_leg if cfg["mode"] == "stream" else run_prefill_leg)(a, cfg, world, rank, local)
+    obj = {"workload": name, "value": weak_scaling_value(cfg["B"] * cfg["N"], world, pre["step_ms"] / 1e3),
+           "unit": "nt/s", "ms_per_step": pre["step_ms"], "steps": steps, "warmup": warmup,
+           "augmented_tokens_per_s": world * cfg["B"] * pre["T"] / (pre["step_ms"] / 1e3),
+           "step": pre["step_desc"], "config": workload_config(a, cfg, pre["T"], pre["R"], name=name),
+           "roofline": prefill_roofline(pre, peaks, peaks_src), "clocks": pre["clocks"],
+           "gpu_launches": pre["launches"]}
+    if pre.get("window_compaction") is not None:
+        obj["window_compaction"] = pre["window_compaction"]
+    return obj
+
+
+def run_compact_leg(args, world, rank, local, peaks, peaks_src):
+    """Bulk focus_kv_compact at the 1 Mb x 4 workload's size: the FOCUS rows of
+    all 1,000 windows (10,000 per (sequence, head), 128 (sequence, head) pairs)
+    gathered from the augmented K/V (B=4, H=32, T=1,010,000, d=128) into the
+    ring: 655 MB read and 655 MB written per launch, both above L2. The source
+    values are never read as numbers (a bit copy), so it is left uninitialised."""
+    import torch
+    from paper_2511_14694_gb300 import focus
+    from paper_2511_14694_gb300.workloads import WORKLOADS
+    cfg = WORKLOADS["stream_1mb_b4_h32_d128"]
+    B, N, W, H, d = cfg["B"], cfg["N"], cfg["W"], cfg["H"], cfg["d"]
+    dev = torch.device("cuda", local)
+    L = focus.layout(N, W, list(cfg["k"]), device=dev)
+    src_k = torch.empty((B, H, L["T"], d), dtype=torch.bfloat16, device=dev)
+    src_v = torch.empty_like(src_k)
+    cache = focus.Cache(B, H, d, C_ring=L["R"], device=dev)
+    stream = torch.cuda.current_stream(dev)
+    for _ in range(3):
+        focus.kv_compact_bulk(cache, src_k, src_v, L, 0, L["M"], stream=stream)
+    reps = 10
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+    torch.cuda.synchronize(dev)
+    for e0, e1 in ev:
+        e0.record(stream)
+        focus.kv_compact_bulk(cache, src_k, src_v, L, 0, L["M"], stream=stream)
+        e1.record(stream)
+    torch.cuda.synchronize(dev)
+    assert focus.device_status(clear=True) == 0
+    ms = statistics.median(a.elapsed_time(b) for a, b in ev)
+    nbytes = float(L["R"] * B * H * 2 * (2 * d) * 2)
+    gbs = nbytes / (ms / 1e3) / 1e9
+    del src_k, src_v, cache
+    torch.cuda.empty_cache()
+    return {"kernel": "focus_kv_compact (bulk)", "workload": "ring of stream_1mb_b4_h32_d128 (R = %d rows per "
+            "(sequence, head), B = %d, H = %d, d = %d)" % (L["R"], B, H, d), "avg_launch_ms": ms,
+            "bytes_per_launch": nbytes, "launches": reps,
+            "timing": "CUDA events around each of %d launches (median); source rows and ring above L2" % reps,
+            "roofline": {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                         "frac": gbs / peaks["hbm_gbs"], "peak_source": f"{peaks_src} copy bandwidth"}}
+
+
 def run_focus(args, world, rank, local):
     import torch
     from paper_2511_14694_gb300.workloads import WORKLOADS
@@ -605,13 +719,18 @@ def run_focus(args, world, rank, local):
     if not args.no_decode:
         dec = run_decode_leg(args, WORKLOADS[args.decode_workload], world, rank, local)
     emb = None if args.embed_d <= 0 else run_embed_leg(args, world, rank, local)
+    legs = {}
+    if not args.no_configs:
+        for key, name, steps, warmup in CONFIG_LEGS:
+            if name != args.workload:
+                legs[key] = run_config_leg(args, name, steps, warmup, world, rank, local, peaks, peaks_src)
+    big_compact = None if args.no_configs else run_compact_leg(args, world, rank, local, peaks, peaks_src)
     if rank != 0:
         return
     value = weak_scaling_value(cfg["B"] * cfg["N"], world, pre["step_ms"] / 1e3)
-    achieved = pre["flops_per_step"] / (pre["attn_ms"] / 1e3) / 1e12
     local_mask = pre.get("local_mask", False)
     # committed DRAM counters exist for the 128 kb workload's appendix-mask kernel
-    # (persistent) and k-mer-local kernel (one CTA per item), default heads
+    # (persistent) and k-mer-local kernel, default heads
     traffic_key = {("tcgen05 persistent", False): ("prefill_attention", "prefill_tc_persistent.cu"),
                    ("tcgen05, one CTA per work item", True): ("prefill_attention_kmer_local", "prefill_tc.cu")
                    }.get((pre["kernel"], local_mask))
@@ -624,45 +743,14 @@ def run_focus(args, world, rank, local):
         "value": value, "unit": "nt/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": pre["step_ms"], "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16", "data": "synthetic (seeded N(0,1)/sqrt(d) bf16 Q/K/V, uniform A/C/G/T ids)",
-        "config": {"workload": args.workload, "B": cfg["B"], "N": cfg["N"], "W": cfg["W"], "k": list(cfg["k"]),
-                   "H": cfg["H"], "d": cfg["d"], "T_augmented": pre["T"], "R_retained": pre["R"],
-                   "step": ("per window: focus_kv_compact(window) + focus_attn_prefill(window), consecutive "
-                            "windows' attention overlapping on two streams; all windows; rate over the whole step"
-                            if cfg["mode"] == "stream" else
-                            "focus_layout + focus_kv_compact(bulk) + focus_attn_prefill(masked-parallel)"),
-                   "l2": ("inputs larger than L2 (pool of %d windows' Q/K/V %.2f GB, ring %.2f GB)" % (
-                       cfg.get("pool", 0), 3 * cfg.get("pool", 0) * cfg["B"] * cfg["H"] * (pre["T"] // max(1, -(-cfg["N"] // cfg["W"]))) * cfg["d"] * 2 / 1e9,
-                       2 * cfg["B"] * cfg["H"] * pre["R"] * cfg["d"] * 2 / 1e9) if cfg["mode"] == "stream" else
-                          "inputs larger than L2 (Q/K/V %.2f GB per step)" % (3 * cfg["B"] * pre["T"] * cfg["H"] * cfg["d"] * 2 / 1e9)),
-                   "prefill_kernel": pre["kernel"],
-                   "mask": "k-mer-local (Sec. 3.2)" if local_mask else "appendix (App. A, Eq. focus-attn)",
-                   "rope_theta": args.rope or None,
-                   "q_per_kv": args.q_per_kv},
+        "config": workload_config(args, cfg, pre["T"], pre["R"]),
+        "step": pre["step_desc"],
         "augmented_tokens_per_s": world * cfg["B"] * pre["T"] / (pre["step_ms"] / 1e3),
-        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
-                     "frac": achieved / peaks["bf16_tflops"], "traffic": traffic,
-                     "peak_source": f"{peaks_src} bf16 dense burst",
-                     "frac_of_sustained": achieved / peaks["bf16_tflops_sustained"],
-                     "kernel": "prefill attention",
-                     "flop_per_launch": pre["flops_per_step"] / (pre["launches"] // (2 * args.steps)
-                                                                 if cfg["mode"] == "stream" else 1),
-                     "visible_pairs": pre["pairs"], "avg_launch_ms": pre.get("per_launch_ms", pre["attn_ms"]),
-                     "launches_per_step": (pre["launches"] // (2 * args.steps)) if cfg["mode"] == "stream" else 1},
+        "roofline": prefill_roofline(pre, peaks, peaks_src, traffic),
         "clocks": pre["clocks"],
         "e2e": pre["e2e"],
         "gpu_launches": pre["launches"],
     }
-    if local_mask:
-        # a few visible keys per row: the launch moves far more bytes than it does FLOPs
-        gbs = pre["bytes_per_step"] / (pre["attn_ms"] / 1e3) / 1e9
-        line["roofline"] = {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                            "frac": gbs / peaks["hbm_gbs"], "traffic": traffic,
-                            "peak_source": f"{peaks_src} copy bandwidth", "kernel": "prefill attention (k-mer-local)",
-                            "tflops": achieved, "visible_pairs": pre["pairs"]}
-        n_launch = (pre["launches"] // (2 * args.steps)) if cfg["mode"] == "stream" else 1
-        line["roofline"].update(bytes_per_launch=pre["bytes_per_step"] / n_launch,
-                                flop_per_launch=pre["flops_per_step"] / n_launch,
-                                avg_launch_ms=pre.get("per_launch_ms", pre["attn_ms"]), launches_per_step=n_launch)
     if "compact_ms" in pre:
         cgbs = pre["compact_bytes"] / (pre["compact_ms"] / 1e3) / 1e9
         line["compaction"] = {"kernel": "focus_kv_compact (bulk)", "avg_launch_ms": pre["compact_ms"],
@@ -672,6 +760,8 @@ def run_focus(args, world, rank, local):
                               "roofline": {"bound": "hbm", "achieved": cgbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                                            "frac": cgbs / peaks["hbm_gbs"],
                                            "peak_source": f"{peaks_src} copy bandwidth"}}
+    if big_compact is not None:
+        line["compaction_1mb_ring"] = big_compact
     if emb is not None:
         egbs = emb["bytes"] / (emb["ms"] / 1e3) / 1e9
         line["embedding"] = {"kernel": "focus_embed_tokens", "rows": emb["T"], "D": emb["D"],
@@ -694,6 +784,7 @@ def run_focus(args, world, rank, local):
             "clocks": dec["clocks"],
         }
         line["decode"]["gpu_launches"] = dec["launches"]
+    line.update(legs)
     if pre["host_sample"] is not None and (args.rope or args.q_per_kv > 1):
         line["cpu_baseline"] = None      # the oracle baseline times the default path only
     elif pre["host_sample"] is not None:
@@ -701,27 +792,32 @@ def run_focus(args, world, rank, local):
         if local_mask:
             from oracle import focus_oracle as fo
             hs["kmer"] = fo.layout_kmer(cfg["N"], cfg["W"], hs["k_sched"])
-            full_s, desc, cores = oracle_local_sample(cfg, hs, hs["k_sched"], hs["q"], hs["k"], hs["v"],
-                                                      budget_s=args.cpu_budget)
-        else:
-            full_s, desc, cores = oracle_prefill_sample(cfg, hs, hs["q"], hs["k"], hs["v"], budget_s=args.cpu_budget)
-        line["cpu_baseline"] = {"value": cfg["B"] * cfg["N"] / full_s, "unit": "nt/s", "cores": cores,
-                                "kind": "oracle", "sample": desc}
+        secs = oracle_head_times(cfg, hs, hs["k_sched"], hs["q"], hs["k"], hs["v"], args.cpu_heads,
+                                 mask=args.mask)
+        val, desc, _ = oracle_baseline(cfg, secs, args.mask)
+        line["cpu_baseline"] = {"value": val, "unit": "nt/s", "cores": os.cpu_count(), "kind": "oracle",
+                                "sample": desc}
     print(json.dumps(line), flush=True)
 
 
 # ----------------------------------------------------------------------------- reference arm (the oracle)
 
 def run_reference(args, world, rank, local):
-    """The fp64 CPU oracle timed on the host cores, on the same workload, metric
-    and unit; each step is a bounded sample extrapolated by visible pairs."""
+    """The fp64 CPU oracle timed on the host cores, on the same workload, metric,
+    unit and config as the library arm: each step is one whole (sequence, head)
+    pass (every window and row), the workload's time that pass times B x H (every
+    pass does the same visible pairs), the same sampler as the library arm's
+    cpu_baseline."""
     if rank != 0:
         return
-    import torch
     from oracle import focus_oracle as fo
     from paper_2511_14694_gb300 import inputs
     from paper_2511_14694_gb300.workloads import WORKLOADS
     cfg = WORKLOADS[args.workload]
+    if cfg["mode"] == "stream":
+        print(json.dumps({"impl": "reference", "unavailable": "the reference arm times the masked-parallel "
+                          "workloads only"}), flush=True)
+        return
     B, N, W, H, d = cfg["B"], cfg["N"], cfg["W"], cfg["H"], cfg["d"]
     M = -(-N // W)
     k_s = inputs.k_schedule(M, cfg["k"], seed=inputs.DEFAULT_SEED)
@@ -729,25 +825,19 @@ def run_reference(args, world, rank, local):
     # two heads of inputs, drawn with the same generator recipe on the CPU
     q, k, v = inputs.qkv((2, L["T"], d), std=cfg["std"], seed=inputs.DEFAULT_SEED, device="cpu")
     hs = dict(win_off=L["win_off"], ring_off=L["ring_off"], keep=L["keep"], kind=L["kind"], win=L["win"])
-    budget = max(2.0, args.cpu_budget / max(1, args.steps + args.warmup))
     if args.mask == "kmer_local":
         hs["kmer"] = fo.layout_kmer(N, W, k_s)
-        sample = lambda: oracle_local_sample(cfg, hs, k_s, q, k, v, budget_s=budget, max_windows=4)  # noqa: E731
-    else:
-        sample = lambda: oracle_prefill_sample(cfg, hs, q, k, v, budget_s=budget, max_windows=4)  # noqa: E731
-    for _ in range(args.warmup):
-        sample()
-    secs, desc = [], ""
-    for _ in range(args.steps):
-        full_s, desc, cores = sample()
-        secs.append(full_s)
-    full_s = statistics.median(secs)
-    value = B * N / full_s
+    oracle_head_times(cfg, hs, k_s, q, k, v, args.warmup, mask=args.mask)
+    secs = oracle_head_times(cfg, hs, k_s, q, k, v, args.steps, mask=args.mask)
+    value, desc, full_s = oracle_baseline(cfg, secs, args.mask)
+    per_pass = statistics.median(secs)
     line = {"metric": METRIC, "value": value, "unit": "nt/s", "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": full_s * 1e3, "higher_is_better": True, "scaling": "weak",
+            "warmup": args.warmup, "ms_per_step": per_pass * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
-            "config": {"workload": args.workload, "B": B, "N": N, "W": W, "k": list(cfg["k"]), "H": H, "d": d,
-                       "mask": args.mask},
+            "config": workload_config(args, cfg, int(L["win_off"][-1]), int(L["ring_off"][-1])),
+            "step": "one whole (sequence, head) pass of the oracle: 1/%d of the workload; value = B N / "
+                    "(%d x ms_per_step)" % (B * H, B * H),
+            "workload_s": full_s,
             "cpu_baseline": {"value": value, "unit": "nt/s", "cores": os.cpu_count(), "kind": "oracle",
                              "sample": desc},
             "e2e": {"value": value, "unit": "nt/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -855,7 +945,10 @@ def main():
     ap.add_argument("--e2e-groups", type=int, default=16,
                     help="head (or sequence) groups of the pipelined host-buffer prefill timed as e2e")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--cpu-heads", type=int, default=8,
+                    help="whole (sequence, head) oracle passes timed for the cpu_baseline (8 of 32 = 25%%)")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the other named workloads and the 1 Mb ring compaction (profiling runs)")
     ap.add_argument("--no-clock-wait", action="store_true",
                     help="do not extend the load after a short timed region (profiling runs)")
     ap.add_argument("--legacy", action="store_true", help="time the legacy mma.sync prefill kernel")

@@ -86,7 +86,7 @@ def prefill_masked_parallel_host(cache: focus.Cache, L: dict, host: dict, dev: d
 
 
 def prefill_streaming(cache: focus.Cache, L: dict, window_qkv, outs, lses, w_begin: int = 0, w_end: int | None = None,
-                      scale=None, flags=0, stream=None, events=None):
+                      scale=None, flags=0, stream=None, events=None, compact_events=None):
     """Streaming prefill (App. A.2) of windows [w_begin, w_end) with the
     attention of consecutive windows overlapping. window_qkv(w) gives window w's
     (q, k, v) ([B, H, T_w, d] each); window w writes outs[i] and lses[i],
@@ -101,7 +101,8 @@ def prefill_streaming(cache: focus.Cache, L: dict, window_qkv, outs, lses, w_beg
     that share a buffer share a stream, so a buffer is never written by two
     launches at once).
     ``events``: optional list of (start, end) CUDA events per window, recorded
-    around each attention launch on its stream. Work is only enqueued; when
+    around each attention launch on its stream; ``compact_events`` the same
+    around each compaction launch on ``stream``. Work is only enqueued; when
     ``stream`` is done, so is everything."""
     cur = stream if stream is not None else torch.cuda.current_stream()
     key = cur.device
@@ -114,7 +115,11 @@ def prefill_streaming(cache: focus.Cache, L: dict, window_qkv, outs, lses, w_beg
         s_.wait_stream(cur)                    # inputs and buffers written before the call
     for w in range(w_begin, w_end):
         q, k, v = window_qkv(w)
+        if compact_events is not None:
+            compact_events[w - w_begin][0].record(cur)
         focus.kv_compact_bulk(cache, k, v, L, w, w + 1, src_row0=int(off[w]), stream=cur)
+        if compact_events is not None:
+            compact_events[w - w_begin][1].record(cur)
         i = w % len(outs)
         s_ = side[i % 2]
         s_.wait_stream(cur)                    # ring rows of windows <= w are in place

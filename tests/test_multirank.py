@@ -58,7 +58,7 @@ def test_reference_arm_two_ranks_prints_one_line():
     env = dict(os.environ, FOCUS_DIST_BACKEND="gloo", OMP_NUM_THREADS="2")
     cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
            "--master-addr", "127.0.0.1", "--master-port", str(port), "bench.py", "--impl", "reference",
-           "--gpus", "2", "--steps", "1", "--warmup", "0", "--cpu-budget", "1",
+           "--gpus", "2", "--steps", "1", "--warmup", "0",
            "--workload", "prefill_4kb_h4_d64"]
     r = subprocess.run(cmd, cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
     assert r.returncode == 0, r.stderr[-2000:]
