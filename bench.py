@@ -287,7 +287,9 @@ def run_prefill_leg(args, cfg, world, rank, local):
     o = torch.empty_like(q)
     lse = torch.empty((B, H, L["T"]), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
-    kernel_name = focus.prefill_kernel(cache, q, k, v, L, flags=args.prefill_flags, o=o)
+    # device workspace the fastest kernel asks for (the rotary embedding's rotated q and k), allocated once
+    ws = focus.new_prefill_workspace(cache, q, k, v, L, flags=args.prefill_flags)
+    kernel_name = focus.prefill_kernel(cache, q, k, v, L, flags=args.prefill_flags, o=o, workspace=ws)
 
     def front(evc=None):
         focus.layout_run(L, nt, stream=stream)
@@ -298,7 +300,8 @@ def run_prefill_leg(args, cfg, world, rank, local):
             evc[1].record(stream)
 
     def attn():
-        focus.attn_prefill(cache, q, k, v, L, 0, L["M"], o=o, lse=lse, stream=stream, flags=args.prefill_flags)
+        focus.attn_prefill(cache, q, k, v, L, 0, L["M"], o=o, lse=lse, stream=stream, flags=args.prefill_flags,
+                           workspace=ws)
 
     for _ in range(args.warmup):
         front()
@@ -392,7 +395,7 @@ def run_prefill_leg(args, cfg, world, rank, local):
                bytes_per_step=bytes_per_step, local_mask=local_mask, compact_ms=compact_ms,
                compact_bytes=compact_bytes,
                clocks=clk.summary(), launches=launches, e2e=e2e, host_sample=host_sample, extra_steps=extra)
-    del q, k, v, o, lse, cache
+    del q, k, v, o, lse, cache, ws
     torch.cuda.empty_cache()
     return res
 

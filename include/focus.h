@@ -200,7 +200,21 @@ typedef struct focus_prefill_args {
     int32_t     max_rows;     /* >= every window's augmented row count in the span */
     float       scale;        /* softmax scale > 0, usually 1/sqrt(d) */
     uint32_t    flags;        /* FOCUS_PREFILL_* */
+    void*       workspace;    /* device scratch, 16-byte aligned, or NULL (see focus_prefill_workspace_size) */
+    size_t      workspace_bytes;  /* its size in bytes */
 } focus_prefill_args;
+
+/* Device workspace that lets focus_attn_prefill use its fastest kernel for these
+ * arguments; 0 when none helps. Host only, no CUDA call; 0 also for arguments that
+ * focus_attn_prefill would reject. Today only the rotary embedding
+ * (cache->rope_theta > 0) on short work items (the persistent kernel's case,
+ * below) asks for one: 256 bytes of per-head counters plus a rotated copy of the
+ * span's q and k, B x H x (q_per_kv + 1) x T_span x d bf16. With it, the q and k
+ * rows are each rotated once, by otherwise idle warps of the attention kernel
+ * itself, a head ahead of their use; without it (NULL, or fewer bytes) the call
+ * still succeeds and every CTA rotates the tiles it loads. The contents need no
+ * initialisation and are scratch afterwards; the caller owns the memory. */
+size_t focus_prefill_workspace_size(const focus_cache* cache, const focus_prefill_args* args);
 
 /* Use the legacy mma.sync kernel instead of the tcgen05/TMEM kernel (kept as the
  * comparison baseline; same results within rounding). It has no rotary
@@ -240,11 +254,13 @@ focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_ar
  *   FOCUS_PREFILL_KERNEL_LEGACY      the mma.sync kernel (FOCUS_PREFILL_LEGACY_MMA),
  *   FOCUS_PREFILL_KERNEL_PERSISTENT  the tcgen05 kernel with one CTA per SM walking
  *                                    the work items (two 128-row Q tiles of a window
- *                                    each): appendix mask, no rotary embedding, and
+ *                                    each): appendix mask and
  *                                    cache->C_ring + args->max_rows <= 4096 (short
  *                                    items, whose start-up and epilogue it overlaps),
  *   FOCUS_PREFILL_KERNEL_PER_ITEM    the tcgen05 kernel with one CTA per work item
  *                                    (every other case).
+ * The persistent kernel also takes the rotary-embedding case when args carries
+ * focus_prefill_workspace_size(cache, args) bytes of workspace.
  * Both tcgen05 kernels compute the same rows (within rounding order). */
 #define FOCUS_PREFILL_KERNEL_LEGACY 0
 #define FOCUS_PREFILL_KERNEL_PER_ITEM 1

@@ -55,13 +55,8 @@ focus_status check_cache(const focus_cache* c, bool need_window) {
 namespace focus {
 
 void rope_table_fill(RopeTable* t, int d, float base) {
-    const int h = d / 2, G = 1024 / d;
-    for (int i = 0; i < kRopeMaxPairs; ++i) {
-        const double theta = i < h ? pow((double)base, -2.0 * i / d) : 0.0;
-        t->theta[i] = theta;
-        for (int g = 0; g < kRopeOffRows; ++g)
-            t->off[g][i] = g <= G ? make_float2((float)cos(g * theta), (float)sin(g * theta)) : make_float2(1.f, 0.f);
-    }
+    const int h = d / 2;
+    for (int i = 0; i < kRopeMaxPairs; ++i) t->theta[i] = i < h ? pow((double)base, -2.0 * i / d) : 0.0;
 }
 
 }  // namespace focus
@@ -191,6 +186,7 @@ static focus_status check_prefill(const focus_cache* cache, const focus_prefill_
         return FOCUS_ERR_INVALID_ARG;
     if (!isfinite(a->scale) || !(a->scale > 0.f)) return FOCUS_ERR_INVALID_ARG;
     if (!aligned16(a->q) || !aligned16(a->k) || !aligned16(a->v) || !aligned16(a->o)) return FOCUS_ERR_UNSUPPORTED;
+    if (a->workspace && !aligned16(a->workspace)) return FOCUS_ERR_UNSUPPORTED;
     if (a->flags & ~(uint32_t)(FOCUS_PREFILL_LEGACY_MMA | FOCUS_PREFILL_KMER_LOCAL)) return FOCUS_ERR_INVALID_ARG;
     if ((a->flags & FOCUS_PREFILL_LEGACY_MMA) && (cache->rope_theta > 0.f || cache->q_per_kv > 1))
         return FOCUS_ERR_UNSUPPORTED;
@@ -208,6 +204,11 @@ focus_status focus_prefill_kernel(const focus_cache* cache, const focus_prefill_
     if (s != FOCUS_OK) return s;
     *kernel = focus::prefill_kernel_choice(*cache, *a);
     return FOCUS_OK;
+}
+
+size_t focus_prefill_workspace_size(const focus_cache* cache, const focus_prefill_args* a) {
+    if (check_prefill(cache, a) != FOCUS_OK) return 0;
+    return focus::prefill_workspace_bytes(*cache, *a);
 }
 
 focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_args* a, cudaStream_t stream) {

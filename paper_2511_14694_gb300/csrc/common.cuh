@@ -45,14 +45,13 @@ __host__ __device__ __forceinline__ int64_t tail_start(int64_t n, int32_t tail) 
 // Positions reach ~10^6, where an fp32 angle p * theta_i is off by up to ~0.1 rad,
 // so every angle a kernel starts from is formed and reduced modulo 2 pi in fp64
 // and only the reduced angle goes to the fp32 sin/cos. Along a tile, rows step by
-// a fixed offset whose cos/sin come from a host table (fp64 there), so a kernel
-// needs one fp64 angle per pair and tile start, not per element.
+// small fixed offsets (|angle| <= 16 rad, accurate in fp32), so a kernel needs one
+// fp64 angle per pair and tile start, not per element.
 constexpr int kRopeMaxPairs = 64;         // d/2 for d <= 128
-constexpr int kRopeOffRows = 17;          // offsets g = 0..G, G = 1024 / d <= 16
 
+// The frequencies, computed once on the host in fp64 (a 512-byte kernel argument).
 struct RopeTable {
     double theta[kRopeMaxPairs];          // theta_i
-    float2 off[kRopeOffRows][kRopeMaxPairs];   // (cos, sin)(g * theta_i)
 };
 
 // Host: fill the table for head dimension d (even, <= 128) and base > 0.
@@ -118,6 +117,8 @@ cudaError_t launch_prefill_mma(const focus_cache& c, const focus_prefill_args& a
                                cudaStream_t stream);
 // FOCUS_PREFILL_KERNEL_* that launch_prefill_tc (or the legacy flag) selects.
 int32_t prefill_kernel_choice(const focus_cache& c, const focus_prefill_args& a);
+// Workspace bytes the fastest prefill kernel wants for these arguments (0: none).
+size_t prefill_workspace_bytes(const focus_cache& c, const focus_prefill_args& a);
 cudaError_t launch_prefill_tc(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
                               cudaStream_t stream);
 

@@ -105,77 +105,6 @@ constexpr int kRegsSoftmax = D == 128 ? 216 : 224;
 static_assert(128 * kRegsIssue<128> + 256 * kRegsSoftmax<128> <= kThreads * kLaunchRegs, "register split over budget");
 static_assert(128 * kRegsIssue<64> + 256 * kRegsSoftmax<64> <= kThreads * kLaunchRegs, "register split over budget");
 
-// Kernel argument: the rotary table only for the ROPE variants.
-template <bool ROPE>
-struct RopeArg {
-    RopeTable t;
-};
-template <>
-struct RopeArg<false> {
-    int unused;
-};
-
-// Rotation of eight column pairs (one 16-byte chunk and its partner d/2 columns
-// on), as four packed pairs of element pairs: c = cos, s = sin, n = -sin.
-struct Rot8 {
-    uint64_t c[4], s[4], n[4];
-};
-
-__device__ __forceinline__ Rot8 rot8_make(const float2* cs) {
-    Rot8 r;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        r.c[k] = f2_pack(cs[2 * k].x, cs[2 * k + 1].x);
-        r.s[k] = f2_pack(cs[2 * k].y, cs[2 * k + 1].y);
-        r.n[k] = f2_pack(-cs[2 * k].y, -cs[2 * k + 1].y);
-    }
-    return r;
-}
-
-// y_lo = x_lo c - x_hi s, y_hi = x_hi c + x_lo s on bf16 chunks, rounded once to bf16.
-__device__ __forceinline__ void rot8_apply(uint4& lo, uint4& hi, const Rot8& r) {
-    uint32_t* l = reinterpret_cast<uint32_t*>(&lo);
-    uint32_t* h = reinterpret_cast<uint32_t*>(&hi);
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const uint64_t xl = f2_pack(__uint_as_float(l[k] << 16), __uint_as_float(l[k] & 0xffff0000u));
-        const uint64_t xh = f2_pack(__uint_as_float(h[k] << 16), __uint_as_float(h[k] & 0xffff0000u));
-        const uint64_t yl = f2_fma(xh, r.n[k], f2_mul(xl, r.c[k]));
-        const uint64_t yh = f2_fma(xl, r.s[k], f2_mul(xh, r.c[k]));
-        float a, b;
-        f2_unpack(yl, a, b);
-        l[k] = pack_bf16x2(a, b);
-        f2_unpack(yh, a, b);
-        h[k] = pack_bf16x2(a, b);
-    }
-}
-
-// r <- r turned further by the angles of st.
-__device__ __forceinline__ void rot8_step(Rot8& r, const Rot8& st) {
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const uint64_t c = f2_fma(r.c[k], st.c[k], f2_mul(r.s[k], st.n[k]));
-        const uint64_t sn = f2_fma(r.s[k], st.c[k], f2_mul(r.c[k], st.s[k]));
-        const uint64_t n = f2_fma(r.n[k], st.c[k], f2_mul(r.c[k], st.n[k]));
-        r.c[k] = c;
-        r.s[k] = sn;
-        r.n[k] = n;
-    }
-}
-
-// (cos, sin) of the small angles g theta_i and G theta_i (|angle| <= 16) for the
-// eight pairs i0..i0+7: fp32 is accurate to ~1e-6 rad here.
-__device__ __forceinline__ void rope_offsets(const RopeTable& t, int i0, int g, int G, float2* off, Rot8& step) {
-    float2 st[8];
-#pragma unroll
-    for (int e = 0; e < 8; ++e) {
-        const float th = (float)t.theta[i0 + e];
-        __sincosf((float)g * th, &off[e].y, &off[e].x);
-        __sincosf((float)G * th, &st[e].y, &st[e].x);
-    }
-    step = rot8_make(st);
-}
-
 // Q/O/LSE row of this CTA's query head, read afresh from the block index where
 // it is used (keeping it in a register across the softmax loop costs spills).
 __device__ __forceinline__ int32_t query_head_row(int32_t H, int32_t q_per_kv) {
@@ -367,7 +296,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
             const int jj = tau % HALF, g = tau / HALF;
             float2 off[8];
             Rot8 step;
-            rope_offsets(rope.t, 8 * jj, g, G, off, step);
+            rope_offsets(rope.t.theta, 8 * jj, g, G, off, step);
             const double theta_own = tau < D / 2 ? rope.t.theta[tau] : 0.0;
             for (int j = 0; j < n_kv_max; ++j) {
                 const int st = j & 1, slot = 2 * st + 1;        // K_j: stage j % 2, second slot
@@ -434,7 +363,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kernel(
             const int jj = tau % HALF, g = (tau / HALF) % G;
             float2 off[8];
             Rot8 step;
-            rope_offsets(rope.t, 8 * jj, g, G, off, step);
+            rope_offsets(rope.t.theta, 8 * jj, g, G, off, step);
             named_bar_sync(2, 256);
             float2 cs[8];
 #pragma unroll
@@ -621,11 +550,25 @@ cudaError_t dispatch(const focus_cache& c, const focus_prefill_args& a, int32_t*
 // them better, and that kernel's per-tile loop is ~4% faster.
 constexpr int64_t kPersistentMaxRows = 4096;
 
+// The rotary embedding takes the persistent kernel only with the workspace for
+// its once-rotated q and k; without it, the one-CTA-per-item kernel rotates the
+// tiles each CTA loads.
+bool prefill_persistent_case(const focus_cache& c, const focus_prefill_args& a) {
+    const bool local = (a.flags & FOCUS_PREFILL_KMER_LOCAL) != 0;
+    return !(a.flags & FOCUS_PREFILL_LEGACY_MMA) && !local && (int64_t)c.C_ring + a.max_rows <= kPersistentMaxRows;
+}
+
 int32_t prefill_kernel_choice(const focus_cache& c, const focus_prefill_args& a) {
     if (a.flags & FOCUS_PREFILL_LEGACY_MMA) return FOCUS_PREFILL_KERNEL_LEGACY;
-    const bool local = (a.flags & FOCUS_PREFILL_KMER_LOCAL) != 0, rope = c.rope_theta > 0.f;
-    if (!local && !rope && (int64_t)c.C_ring + a.max_rows <= kPersistentMaxRows) return FOCUS_PREFILL_KERNEL_PERSISTENT;
+    if (prefill_persistent_case(c, a)) {
+        const size_t need = prefill::persistent_workspace_bytes(c, a);
+        if (need == 0 || (a.workspace && a.workspace_bytes >= need)) return FOCUS_PREFILL_KERNEL_PERSISTENT;
+    }
     return FOCUS_PREFILL_KERNEL_PER_ITEM;
+}
+
+size_t prefill_workspace_bytes(const focus_cache& c, const focus_prefill_args& a) {
+    return prefill_persistent_case(c, a) ? prefill::persistent_workspace_bytes(c, a) : 0;
 }
 
 cudaError_t launch_prefill_tc(const focus_cache& c, const focus_prefill_args& a, int32_t* status,

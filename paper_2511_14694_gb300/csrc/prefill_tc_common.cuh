@@ -25,6 +25,10 @@ constexpr int kBoxBytes = 128 * 128;   // one TMA box: 128 rows x 64 bf16 (128 B
 constexpr uint64_t kWaitNs = 2000000000ull;   // 2 s bound on any wait
 constexpr float kRescaleThreshold = 8.0f;     // log2 units: rescale O only if the max grows by > 2^8
 
+// Shared scratch of one 64-thread group rotating q/k rows in the persistent
+// kernel: 64 unit start angles and 64 x 8 row offsets (float2).
+constexpr int kRopeGroupScratch = 64 * 8 + 64 * 8 * 8;
+
 template <int D>
 struct Cfg {
     static constexpr int kBoxes = D / 64;                       // TMA boxes per 128-row tile
@@ -37,6 +41,9 @@ struct Cfg {
     // persistent kernel: no rotary bases; O staging of 8 warps x 32 rows x 64 B
     static constexpr int kStageOff = kBarOff + 256;
     static constexpr int kSmemPersistent = kStageOff + 8 * 2048 + 1024;
+    // persistent kernel with the rotary embedding: one rotating group's scratch
+    static constexpr int kRopeScratchOff = kStageOff + 8 * 2048;
+    static constexpr int kSmemPersistentRope = kRopeScratchOff + kRopeGroupScratch + 1024;
 };
 
 struct Bars {
@@ -164,12 +171,89 @@ __device__ __forceinline__ void softmax_tile(const float* s, uint32_t s_addr, ui
     }
 }
 
+// ---------------------------------------------------------------- rotary embedding
+
+// Kernel argument: the rotary table only for the ROPE variants.
+template <bool ROPE>
+struct RopeArg {
+    RopeTable t;
+};
+template <>
+struct RopeArg<false> {
+    int unused;
+};
+
+// Rotation of eight column pairs (one 16-byte chunk and its partner d/2 columns
+// on), as four packed pairs of element pairs: c = cos, s = sin, n = -sin.
+struct Rot8 {
+    uint64_t c[4], s[4], n[4];
+};
+
+__device__ __forceinline__ Rot8 rot8_make(const float2* cs) {
+    Rot8 r;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        r.c[k] = f2_pack(cs[2 * k].x, cs[2 * k + 1].x);
+        r.s[k] = f2_pack(cs[2 * k].y, cs[2 * k + 1].y);
+        r.n[k] = f2_pack(-cs[2 * k].y, -cs[2 * k + 1].y);
+    }
+    return r;
+}
+
+// y_lo = x_lo c - x_hi s, y_hi = x_hi c + x_lo s on bf16 chunks, rounded once to bf16.
+__device__ __forceinline__ void rot8_apply(uint4& lo, uint4& hi, const Rot8& r) {
+    uint32_t* l = reinterpret_cast<uint32_t*>(&lo);
+    uint32_t* h = reinterpret_cast<uint32_t*>(&hi);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const uint64_t xl = f2_pack(__uint_as_float(l[k] << 16), __uint_as_float(l[k] & 0xffff0000u));
+        const uint64_t xh = f2_pack(__uint_as_float(h[k] << 16), __uint_as_float(h[k] & 0xffff0000u));
+        const uint64_t yl = f2_fma(xh, r.n[k], f2_mul(xl, r.c[k]));
+        const uint64_t yh = f2_fma(xl, r.s[k], f2_mul(xh, r.c[k]));
+        float a, b;
+        f2_unpack(yl, a, b);
+        l[k] = pack_bf16x2(a, b);
+        f2_unpack(yh, a, b);
+        h[k] = pack_bf16x2(a, b);
+    }
+}
+
+// r <- r turned further by the angles of st.
+__device__ __forceinline__ void rot8_step(Rot8& r, const Rot8& st) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const uint64_t c = f2_fma(r.c[k], st.c[k], f2_mul(r.s[k], st.n[k]));
+        const uint64_t sn = f2_fma(r.s[k], st.c[k], f2_mul(r.c[k], st.s[k]));
+        const uint64_t n = f2_fma(r.n[k], st.c[k], f2_mul(r.c[k], st.n[k]));
+        r.c[k] = c;
+        r.s[k] = sn;
+        r.n[k] = n;
+    }
+}
+
+// (cos, sin) of the small angles g theta_i and G theta_i (|angle| <= 16) for the
+// eight pairs i0..i0+7: fp32 is accurate to ~1e-6 rad here.
+__device__ __forceinline__ void rope_offsets(const double* theta, int i0, int g, int G, float2* off, Rot8& step) {
+    float2 st[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        const float th = (float)theta[i0 + e];
+        __sincosf((float)g * th, &off[e].y, &off[e].x);
+        __sincosf((float)G * th, &st[e].y, &st[e].x);
+    }
+    step = rot8_make(st);
+}
+
 // 3-D map over a [BH][rows][d] bf16 tensor, box = 128 rows x 64 columns, 128-byte swizzle.
 cudaError_t make_map(CUtensorMap* m, const void* ptr, int d, int64_t rows, int64_t bh);
 
-// The persistent kernel (appendix mask, no rotary embedding).
+// The persistent kernel (appendix mask). With the rotary embedding it needs the
+// caller's workspace (persistent_workspace_bytes) for the rotated Q and K rows.
 cudaError_t launch_prefill_tc_persistent(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
                                          cudaStream_t stream);
+// Workspace bytes of the persistent kernel: 0 without the rotary embedding; with
+// it a 256-byte block of per-head counters, then Q and K of the span, rotated.
+size_t persistent_workspace_bytes(const focus_cache& c, const focus_prefill_args& a);
 
 }  // namespace prefill
 }  // namespace focus

@@ -16,7 +16,9 @@
 //   warp 1     MMA issuer: per item as in prefill_tc.cu, but with one stage wait
 //              and one stage release per iteration; an item's first PV into O_t
 //              waits until the previous item's epilogue has read O_t (o_free)
-//   warps 2-3  idle
+//   warps 2-3  idle; with the rotary embedding (ROPE) they rotate the span's Q
+//              and K rows once, into a caller workspace that the Q/K tensor maps
+//              read (rotate_span below), one head ahead of the attention
 //   warps 4-11 softmax per tile (the shared softmax_tile), then the epilogue:
 //              O_t / l to bf16 through a per-warp staging buffer (the Q buffers may
 //              already hold the next item's Q), arrive on o_free once O_t is read
@@ -36,8 +38,15 @@ namespace focus {
 namespace prefill {
 namespace {
 
-constexpr int kRegsIssue = 104, kRegsSoftmax = 200;
-static_assert(128 * kRegsIssue + 256 * kRegsSoftmax <= kThreads * kLaunchRegs, "register split over budget");
+// Register split: warpgroup 0 (TMA, MMA and, with the rotary embedding, the
+// rotating warps 2-3) and the two softmax warpgroups; the counts sum to the
+// launch's 384 x 168.
+template <bool ROPE>
+constexpr int kRegsIssue = ROPE ? 136 : 104;
+template <bool ROPE>
+constexpr int kRegsSoftmax = ROPE ? 184 : 200;
+static_assert(128 * kRegsIssue<false> + 256 * kRegsSoftmax<false> <= kThreads * kLaunchRegs, "register split over budget");
+static_assert(128 * kRegsIssue<true> + 256 * kRegsSoftmax<true> <= kThreads * kLaunchRegs, "register split over budget");
 
 // Geometry of one work item: two 128-row Q tiles of one (sequence, head,
 // window). Items are numbered head by head (sequences, then K/V heads, outermost;
@@ -86,14 +95,159 @@ __device__ __forceinline__ ItemGeom item_geom(int64_t idx, int32_t per_head, int
     return I;
 }
 
-template <int D, bool GQA>
+// Rotary embedding of the span (ROPE variants). Work unit = 64 consecutive
+// positions of one K/V head bh: its 64 K rows and the 64 rows of each of its g
+// query heads at the same positions (one 16 KB block per row set at d = 128),
+// which share every rotation angle. Units are numbered head-major (unit u: head
+// u / n_chunks, rows 64 (u % n_chunks) ..), so they finish in the order the items
+// use them. A group of 64 threads (tau = 0..63, its own named barrier and
+// kRopeGroupScratch bytes of shared memory) takes units u0, u0 + du, ... below
+// u1; after a unit, rot_done[bh] is incremented (release), and the producer
+// loads a head's Q/K tiles once rot_done[bh] reaches n_chunks. Row i of the span
+// has position id p_span0 + i (the span's rows are consecutive augmented rows).
+//
+// Thread tau owns pair chunk jj (pairs 8 jj .. 8 jj + 7: the 16-byte chunk jj and
+// its partner D/2 columns on) of rows gg, gg + G, ... of each row set: the unit's
+// start angle is formed per pair in fp64 and reduced modulo 2 pi (rope_cs, one
+// per thread), the row offset gg theta and the stride G theta are small fp32
+// angles, and the rows follow by the angle-addition recurrence.
+//
+// Rows move through registers only: the attention's MMAs read their operands
+// from shared memory at a high rate, and staging the rows there (cp.async) made
+// the rotation several times slower next to them. Each thread keeps the loads
+// of kRotRows rows of two row sets in flight, and each group prefetches its next
+// unit's rows into L2.
+template <int D>
+struct RopeSpan {
+    static constexpr int HALF = D / 16, G = 64 / HALF, RPT = 64 / G, CPR = D / 8;
+    static constexpr int kRotRows = 2;
+
+    const double* theta;
+    const uint4* q_src;
+    const uint4* k_src;
+    uint4* q_dst;
+    uint4* k_dst;
+    int32_t* rot_done;
+    int64_t T_span;
+    int32_t g;
+    int32_t p_span0;
+    int32_t BH;                                        // K/V heads of the span (sequences x heads)
+
+    __device__ __forceinline__ int32_t n_chunks() const { return (int32_t)((T_span + 63) / 64); }
+
+    // bulk prefetch into L2 of the K and Q rows of unit (bh, chunk)
+    __device__ __forceinline__ void prefetch(int32_t bh, int32_t chunk) const {
+        const int64_t row0 = (int64_t)chunk * 64;
+        const int64_t rows = T_span - row0 < 64 ? T_span - row0 : 64;
+        const uint32_t bytes = (uint32_t)(rows * D * 2);
+        asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;"
+                     ::"l"(reinterpret_cast<uint64_t>(k_src + ((int64_t)bh * T_span + row0) * CPR)), "r"(bytes)
+                     : "memory");
+        for (int m = 0; m < g; ++m)
+            asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;"
+                         ::"l"(reinterpret_cast<uint64_t>(q_src + (((int64_t)bh * g + m) * T_span + row0) * CPR)),
+                         "r"(bytes)
+                         : "memory");
+    }
+
+    // Rows gg + G m, m in [m0, m0 + kRotRows), of row sets s0 and s0 + 1 (set 0: K,
+    // set 1 + i: query head i of the group) of the unit at span row row0: loads
+    // first, then each row rotated by rot, which steps G positions after each.
+    __device__ __forceinline__ void rows_apply(int32_t bh, int64_t row0, int gg, int m0, int rows, int s0, int jj,
+                                               Rot8& rot, const Rot8& step) const {
+        const bool two = s0 + 1 <= g;
+        const int64_t h0 = s0 == 0 ? (int64_t)bh : (int64_t)bh * g + (s0 - 1);
+        const int64_t base0 = (h0 * T_span + row0 + gg + G * m0) * CPR + jj;
+        const int64_t base1 = (((int64_t)bh * g + s0) * T_span + row0 + gg + G * m0) * CPR + jj;
+        const uint4* src0 = (s0 == 0 ? k_src : q_src) + base0;
+        uint4* dst0 = (s0 == 0 ? k_dst : q_dst) + base0;
+        uint4 lo0[kRotRows], hi0[kRotRows], lo1[kRotRows], hi1[kRotRows];
+#pragma unroll
+        for (int i = 0; i < kRotRows; ++i) {
+            if (gg + G * (m0 + i) < rows) {
+                lo0[i] = src0[i * G * CPR];
+                hi0[i] = src0[i * G * CPR + HALF];
+                if (two) {
+                    lo1[i] = q_src[base1 + i * G * CPR];
+                    hi1[i] = q_src[base1 + i * G * CPR + HALF];
+                }
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < kRotRows; ++i) {
+            if (gg + G * (m0 + i) < rows) {
+                rot8_apply(lo0[i], hi0[i], rot);
+                dst0[i * G * CPR] = lo0[i];
+                dst0[i * G * CPR + HALF] = hi0[i];
+                if (two) {
+                    rot8_apply(lo1[i], hi1[i], rot);
+                    q_dst[base1 + i * G * CPR] = lo1[i];
+                    q_dst[base1 + i * G * CPR + HALF] = hi1[i];
+                }
+            }
+            rot8_step(rot, step);
+        }
+    }
+
+    // scratch: kb[64] unit start angles, then 64 x 8 row offsets (float2)
+    __device__ __forceinline__ void run(int32_t u0, int32_t u1, int32_t du, int tau, uint32_t bar,
+                                        float2* kb) const {
+        const int jj = tau % HALF, gg = tau / HALF;
+        float2* off = kb + 64 + tau * 8;
+        Rot8 step;
+        {
+            float2 o[8];
+            rope_offsets(theta, 8 * jj, gg, G, o, step);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) off[e] = o[e];
+        }
+        const int32_t nck = n_chunks();
+        if (u1 > nck * BH) u1 = nck * BH;              // units exist for heads < BH only
+        // unit u = (bh, chunk), advanced incrementally (du may exceed nck)
+        int32_t bh = u0 / nck, chunk = u0 % nck;
+        const int32_t dbh = du / nck, dch = du % nck;
+        if (tau == 0 && u0 < u1) prefetch(bh, chunk);
+        for (int32_t u = u0; u < u1; u += du) {
+            int32_t nbh = bh + dbh, nch = chunk + dch;
+            if (nch >= nck) {
+                nch -= nck;
+                ++nbh;
+            }
+            if (tau == 0 && u + du < u1) prefetch(nbh, nch);
+            const int64_t row0 = (int64_t)chunk * 64;
+            const int rows = (int)(T_span - row0 < 64 ? T_span - row0 : 64);
+            if (tau < D / 2) kb[tau] = rope_cs((double)(p_span0 + row0) * theta[tau]);
+            named_bar_sync(bar, 64);
+            // row sets in pairs (K with the first query head, then query heads two at
+            // a time), each pair's rows from the unit's start rotation
+            for (int s0 = 0; s0 <= g; s0 += 2) {
+                float2 cs[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) cs[e] = rope_mul(kb[8 * jj + e], off[e]);
+                Rot8 rot = rot8_make(cs);
+#pragma unroll 1
+                for (int m0 = 0; m0 < RPT; m0 += kRotRows) rows_apply(bh, row0, gg, m0, rows, s0, jj, rot, step);
+            }
+            fence_proxy_async_global();
+            __threadfence();
+            named_bar_sync(bar, 64);                   // the unit's rows are stored; kb may be rewritten
+            if (tau == 0) red_release_add(rot_done + bh, 1);
+            bh = nbh;
+            chunk = nch;
+        }
+    }
+};
+
+template <int D, bool GQA, bool ROPE>
 __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
         const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
         const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_rk,
         const __grid_constant__ CUtensorMap tm_rv, __nv_bfloat16* __restrict__ o, float* __restrict__ lse,
         int64_t T_span, const int32_t* __restrict__ win_off, const int32_t* __restrict__ ring_off, int32_t w_begin,
         int32_t w_end, int32_t ctas_pw, int32_t H, int32_t C_ring, float scale_log2, int32_t* status,
-        int32_t q_per_kv, int64_t n_items) {
+        int32_t q_per_kv, int64_t n_items, const __grid_constant__ RopeArg<ROPE> rope,
+        const uint4* __restrict__ q_src, const uint4* __restrict__ k_src, uint4* __restrict__ q_rot,
+        uint4* __restrict__ k_rot, int32_t* __restrict__ rot_done, int32_t BHk, int32_t rope_pro_heads) {
     using C = Cfg<D>;
     extern __shared__ unsigned char smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -153,8 +307,22 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
     tc_fence_after();
     const uint32_t tmem = bars->tmem;
 
+    if constexpr (ROPE) {
+        // prologue: all six 64-thread groups of every CTA rotate the first
+        // rope_pro_heads K/V heads' units (their K and Q rows) at the full rate of the
+        // SM, so that the attention can start on them while warps 2-3 go on with the
+        // rest; shared scratch in the K/V stages, which no copy has touched yet
+        const RopeSpan<D> rs{rope.t.theta, q_src, k_src, q_rot, k_rot, rot_done, T_span, q_per_kv,
+                             win_off[w_begin], BHk};
+        const int grp = threadIdx.x >> 6;
+        rs.run((int32_t)blockIdx.x * (kThreads / 64) + grp, rs.n_chunks() * rope_pro_heads,
+               (int32_t)gridDim.x * (kThreads / 64), threadIdx.x & 63, 1 + grp,
+               reinterpret_cast<float2*>(smem + C::kSlotOff + grp * kRopeGroupScratch));
+        __syncthreads();                               // the stage scratch is free for the copies
+    }
+
     if (warp < 4) {
-        setmaxnreg_dec<kRegsIssue>();
+        setmaxnreg_dec<kRegsIssue<ROPE>>();
         if (warp == 0 && lane == 0) {
             // ============================================= TMA producer
             prefetch_tmap(&tm_q);
@@ -166,6 +334,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
             int64_t n_issued = 0;                        // K/V groups issued (one per MMA iteration), across items
             int it = 0;                                  // valid items started
             bool ok = true;
+            int32_t ready_bh = -1;                       // ROPE: last head seen fully rotated
             int64_t k = 0;
             ItemGeom I = next_valid(k, true);
             while (ok && I.valid && !aborted(bars)) {
@@ -176,6 +345,16 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
                 if (it > 0 && !mbar_wait(smem_addr(&bars->q_free), (it - 1) & 1, kWaitNs)) {
                     fail(bars, status);
                     break;
+                }
+                if constexpr (ROPE) {
+                    // this head's rotated Q and K rows are all in the workspace
+                    if (I.bh != ready_bh) {
+                        if (!wait_count(rot_done + I.bh, (int32_t)((T_span + 63) / 64), kWaitNs)) {
+                            fail(bars, status);
+                            break;
+                        }
+                        ready_bh = I.bh;
+                    }
                 }
                 mbar_expect_tx(bq, 2 * C::kTileBytes);
                 const int32_t qrow = GQA ? I.bh * q_per_kv + I.member : I.bh;
@@ -286,10 +465,19 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
             // drain: all issued MMAs complete before TMEM is freed
             mma_commit(smem_addr(&bars->drain));
             mbar_wait(smem_addr(&bars->drain), 0, kWaitNs);
+        } else if (ROPE && (warp == 2 || warp == 3)) {
+            // ============================================= rotary embedding of the span
+            if constexpr (ROPE) {
+                const RopeSpan<D> rs{rope.t.theta, q_src, k_src, q_rot, k_rot, rot_done, T_span, q_per_kv,
+                                     win_off[w_begin], BHk};
+                const int32_t p0 = rs.n_chunks() * rope_pro_heads;   // the prologue's heads
+                rs.run(p0 + (int32_t)blockIdx.x, rs.n_chunks() * BHk, (int32_t)gridDim.x, threadIdx.x - 64, 7,
+                       reinterpret_cast<float2*>(smem + C::kRopeScratchOff));
+            }
         }
     } else {
         // ================================================= softmax / epilogue
-        setmaxnreg_inc<kRegsSoftmax>();
+        setmaxnreg_inc<kRegsSoftmax<ROPE>>();
         const int t = (warp - 4) >> 2;                    // 0: warps 4-7, 1: warps 8-11
         const int quarter = warp & 3;                     // TMEM lanes this warp may access
         const int r = quarter * 32 + lane;                // row within the Q tile
@@ -404,14 +592,37 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
     }
 }
 
-template <int D, bool GQA>
+// Workspace layout (ROPE): int32 rot_done[B H] (padded to 256 bytes), then the
+// rotated Q [B][H g][T_span][d] and K [B][H][T_span][d], bf16.
+size_t rope_counter_bytes(const focus_cache& c) { return ((size_t)c.B * c.H * 4 + 255) & ~(size_t)255; }
+
+// K/V heads rotated in the kernel's prologue by all warps (the rest by warps 2-3
+// beside the attention). One: at 128 kb, 32 heads, one head took 2.907 ms per
+// launch, 2 / 5 of the heads 2.97 ms and all of them (a rotation pass before the
+// attention, ~0.87 ms of it) 3.035 ms.
+int32_t rope_prologue_heads(int64_t BH) { return BH < 1 ? 0 : 1; }
+
+template <int D, bool GQA, bool ROPE>
 cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t* status, cudaStream_t stream) {
     const int64_t BH = (int64_t)c.B * c.H;
     const int32_t g = c.q_per_kv > 1 ? c.q_per_kv : 1;
-    CUtensorMap tq, tk, tv, trk, trv;
+    const void* qmap = a.q;
+    const void* kmap = a.k;
+    int32_t* rot_done = nullptr;
+    uint4 *q_rot = nullptr, *k_rot = nullptr;
     cudaError_t e;
-    if ((e = make_map(&tq, a.q, D, a.T_span, BH * g)) != cudaSuccess) return e;
-    if ((e = make_map(&tk, a.k, D, a.T_span, BH)) != cudaSuccess) return e;
+    if constexpr (ROPE) {
+        char* ws = static_cast<char*>(a.workspace);
+        rot_done = reinterpret_cast<int32_t*>(ws);
+        q_rot = reinterpret_cast<uint4*>(ws + rope_counter_bytes(c));
+        k_rot = q_rot + BH * g * a.T_span * D / 8;
+        qmap = q_rot;
+        kmap = k_rot;
+        if ((e = cudaMemsetAsync(rot_done, 0, (size_t)BH * 4, stream)) != cudaSuccess) return e;
+    }
+    CUtensorMap tq, tk, tv, trk, trv;
+    if ((e = make_map(&tq, qmap, D, a.T_span, BH * g)) != cudaSuccess) return e;
+    if ((e = make_map(&tk, kmap, D, a.T_span, BH)) != cudaSuccess) return e;
     if ((e = make_map(&tv, a.v, D, a.T_span, BH)) != cudaSuccess) return e;
     if (c.C_ring > 0) {
         if ((e = make_map(&trk, c.ring_k, D, c.C_ring, BH)) != cudaSuccess) return e;
@@ -420,8 +631,8 @@ cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t*
         trk = tk;
         trv = tv;
     }
-    const int smem = Cfg<D>::kSmemPersistent;
-    auto* kernel = prefill_tc_persistent_kernel<D, GQA>;
+    const int smem = ROPE ? Cfg<D>::kSmemPersistentRope : Cfg<D>::kSmemPersistent;
+    auto* kernel = prefill_tc_persistent_kernel<D, GQA, ROPE>;
     if ((e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
         return e;
     // the register split needs the launch registers it was sized for: with fewer,
@@ -435,20 +646,47 @@ cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t*
     const int ctas_pw = (a.max_rows + 2 * BM - 1) / (2 * BM);
     // one CTA per SM, each walking every gridDim.x-th work item
     const int64_t n_items = (int64_t)(a.w_end - a.w_begin) * ctas_pw * g * c.H * c.B;
-    const dim3 grid((unsigned)(n_items < sms ? n_items : sms));
-    kernel<<<grid, kThreads, smem, stream>>>(tq, tk, tv, trk, trv, (__nv_bfloat16*)a.o, a.lse, a.T_span,
-                                             a.d_win_off, a.d_ring_off, a.w_begin, a.w_end, ctas_pw, c.H, c.C_ring,
-                                             a.scale * 1.4426950408889634f, status, g, n_items);
+    RopeArg<ROPE> rope;
+    if constexpr (ROPE) rope_table_fill(&rope.t, D, c.rope_theta);
+    else rope.unused = 0;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(n_items < sms ? n_items : sms));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    // ROPE: a CTA's producer waits for rows that the other CTAs' rotating warps
+    // write, so every CTA must be resident at once: a cooperative launch
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = ROPE ? 1 : 0;
+    e = cudaLaunchKernelEx(&cfg, kernel, tq, tk, tv, trk, trv, (__nv_bfloat16*)a.o, a.lse, a.T_span, a.d_win_off,
+                           a.d_ring_off, a.w_begin, a.w_end, ctas_pw, c.H, c.C_ring,
+                           a.scale * 1.4426950408889634f, status, g, n_items, rope,
+                           (const uint4*)a.q, (const uint4*)a.k, q_rot, k_rot, rot_done, (int32_t)BH,
+                           rope_prologue_heads(BH));
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 
 }  // namespace
 
+size_t persistent_workspace_bytes(const focus_cache& c, const focus_prefill_args& a) {
+    if (!(c.rope_theta > 0.f)) return 0;
+    const size_t g = c.q_per_kv > 1 ? (size_t)c.q_per_kv : 1;
+    return rope_counter_bytes(c) + (size_t)c.B * c.H * (g + 1) * (size_t)a.T_span * c.d * 2;
+}
+
 cudaError_t launch_prefill_tc_persistent(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
                                          cudaStream_t stream) {
-    const bool gqa = c.q_per_kv > 1;
-    if (c.d == 128) return gqa ? launch_d<128, true>(c, a, status, stream) : launch_d<128, false>(c, a, status, stream);
-    return gqa ? launch_d<64, true>(c, a, status, stream) : launch_d<64, false>(c, a, status, stream);
+    const bool gqa = c.q_per_kv > 1, rope = c.rope_theta > 0.f;
+    if (c.d == 128) {
+        if (rope) return gqa ? launch_d<128, true, true>(c, a, status, stream) : launch_d<128, false, true>(c, a, status, stream);
+        return gqa ? launch_d<128, true, false>(c, a, status, stream) : launch_d<128, false, false>(c, a, status, stream);
+    }
+    if (rope) return gqa ? launch_d<64, true, true>(c, a, status, stream) : launch_d<64, false, true>(c, a, status, stream);
+    return gqa ? launch_d<64, true, false>(c, a, status, stream) : launch_d<64, false, false>(c, a, status, stream);
 }
 
 }  // namespace prefill

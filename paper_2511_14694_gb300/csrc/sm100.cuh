@@ -64,6 +64,36 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint64_
     }
 }
 
+// ---------------------------------------------------------------- cross-CTA counters
+// A count published by generic-proxy stores of other CTAs and consumed by TMA
+// loads (async proxy): the writer orders its stores before the release with a
+// proxy fence and a gpu-scope fence; the reader acquires the count, then fences
+// the async proxy before issuing its copies.
+__device__ __forceinline__ void fence_proxy_async_global() {
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+__device__ __forceinline__ void red_release_add(int32_t* p, int32_t v) {
+    asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ int32_t ld_acquire(const int32_t* p) {
+    int32_t v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+// Wait until *p >= target, giving up after limit_ns (returns false then);
+// then make the counted rows visible to this thread's later TMA loads.
+__device__ __forceinline__ bool wait_count(const int32_t* p, int32_t target, uint64_t limit_ns) {
+    if (ld_acquire(p) < target) {
+        const uint64_t t0 = globaltimer_ns();
+        while (ld_acquire(p) < target) {
+            if (globaltimer_ns() - t0 > limit_ns) return false;
+            __nanosleep(128);
+        }
+    }
+    fence_proxy_async_global();
+    return true;
+}
+
 // ---------------------------------------------------------------- TMA
 
 // 3-D tiled load of a box into shared memory, completing on an mbarrier.

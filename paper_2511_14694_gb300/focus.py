@@ -50,8 +50,7 @@ class CacheDesc(ctypes.Structure):
 class PrefillArgs(ctypes.Structure):
     _fields_ = [("q", _P), ("k", _P), ("v", _P), ("o", _P), ("lse", _P), ("T_span", _i64), ("d_win_off", _P),
                 ("d_ring_off", _P), ("n_windows", _i32), ("w_begin", _i32), ("w_end", _i32), ("max_rows", _i32),
-                ("scale", _f32),
-                ("flags", _u32)]
+                ("scale", _f32), ("flags", _u32), ("workspace", _P), ("workspace_bytes", ctypes.c_size_t)]
 
 
 class CompactArgs(ctypes.Structure):
@@ -91,6 +90,8 @@ def load() -> ctypes.CDLL:
     lib.focus_attn_prefill.argtypes = [ctypes.POINTER(CacheDesc), ctypes.POINTER(PrefillArgs), _P]
     lib.focus_prefill_kernel.restype = ctypes.c_int
     lib.focus_prefill_kernel.argtypes = [ctypes.POINTER(CacheDesc), ctypes.POINTER(PrefillArgs), _P]
+    lib.focus_prefill_workspace_size.restype = ctypes.c_size_t
+    lib.focus_prefill_workspace_size.argtypes = [ctypes.POINTER(CacheDesc), ctypes.POINTER(PrefillArgs)]
     lib.focus_decode_workspace_size.restype = ctypes.c_size_t
     lib.focus_decode_workspace_size.argtypes = [ctypes.POINTER(CacheDesc)]
     lib.focus_attn_decode.restype = ctypes.c_int
@@ -312,10 +313,35 @@ def _check_heads(cache: Cache, q, k, v):
                          f"(want {cache.H})")
 
 
+def _prefill_args(q, k, v, o, lse, L: dict, w_begin: int, w_end: int, scale: float, flags: int, workspace=None):
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    return PrefillArgs(_ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse), q.shape[2], _ptr(L["win_off"]),
+                       _ptr(L["ring_off"]), L["M"], w_begin, w_end, int(L["max_rows"]), scale, flags,
+                       _ptr(workspace), ws_bytes)
+
+
+def prefill_workspace_bytes(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | None = None,
+                            flags: int = 0) -> int:
+    """focus_prefill_workspace_size: device workspace bytes that let these
+    arguments use the fastest kernel (0: none needed)."""
+    w_end = L["M"] if w_end is None else w_end
+    a = _prefill_args(q, k, v, q, None, L, w_begin, w_end, 1.0 / math.sqrt(q.shape[3]), flags)
+    return int(load().focus_prefill_workspace_size(ctypes.byref(cache.desc), ctypes.byref(a)))
+
+
+def new_prefill_workspace(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | None = None,
+                          flags: int = 0):
+    """A device buffer of prefill_workspace_bytes (None when none is needed)."""
+    n = prefill_workspace_bytes(cache, q, k, v, L, w_begin, w_end, flags)
+    return None if n == 0 else torch.empty(n, dtype=torch.uint8, device=q.device)
+
+
 def attn_prefill(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | None = None, scale=None,
-                 o=None, lse=None, flags: int = 0, stream=None):
+                 o=None, lse=None, flags: int = 0, stream=None, workspace="auto"):
     """focus_attn_prefill over windows [w_begin, w_end). q/k/v: bf16 [B, H, T_span, d]
-    holding the augmented rows of those windows. Returns (o, lse)."""
+    holding the augmented rows of those windows. Returns (o, lse).
+    ``workspace``: a device buffer for the library (see prefill_workspace_bytes),
+    None for none, or "auto" to allocate one when the arguments can use it."""
     lib = load()
     w_end = L["M"] if w_end is None else w_end
     for name, t in (("q", q), ("k", k), ("v", v)):
@@ -327,8 +353,11 @@ def attn_prefill(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | 
     if lse is None:
         lse = torch.empty((B, H, T_span), dtype=torch.float32, device=q.device)
     scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
-    a = PrefillArgs(_ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse), T_span, _ptr(L["win_off"]), _ptr(L["ring_off"]),
-                    L["M"], w_begin, w_end, int(L["max_rows"]), scale, flags)
+    if isinstance(workspace, str):
+        workspace = new_prefill_workspace(cache, q, k, v, L, w_begin, w_end, flags)
+    elif workspace is not None:
+        _cuda(workspace, "workspace")
+    a = _prefill_args(q, k, v, o, lse, L, w_begin, w_end, scale, flags, workspace)
     _check("focus_attn_prefill", lib.focus_attn_prefill(ctypes.byref(cache.desc), ctypes.byref(a), _stream(stream)))
     return o, lse
 
@@ -337,15 +366,18 @@ PREFILL_KERNELS = {0: "legacy mma.sync", 1: "tcgen05, one CTA per work item", 2:
 
 
 def prefill_kernel(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | None = None, flags: int = 0,
-                   o=None) -> str:
+                   o=None, workspace="auto") -> str:
     """Name of the kernel focus_attn_prefill would launch for these arguments
-    (focus_prefill_kernel: host only, nothing runs on the device)."""
+    (focus_prefill_kernel: host only, nothing runs on the device). ``workspace``
+    as for attn_prefill; "auto" assumes the workspace attn_prefill would allocate."""
     lib = load()
     w_end = L["M"] if w_end is None else w_end
-    T_span = q.shape[2]
-    a = PrefillArgs(_ptr(q), _ptr(k), _ptr(v), _ptr(q if o is None else o), 0, T_span, _ptr(L["win_off"]),
-                    _ptr(L["ring_off"]), L["M"], w_begin, w_end, int(L["max_rows"]), 1.0 / math.sqrt(q.shape[3]),
-                    flags)
+    a = _prefill_args(q, k, v, q if o is None else o, None, L, w_begin, w_end, 1.0 / math.sqrt(q.shape[3]), flags)
+    if isinstance(workspace, str):
+        a.workspace_bytes = prefill_workspace_bytes(cache, q, k, v, L, w_begin, w_end, flags)
+        a.workspace = 16 if a.workspace_bytes else None        # a placeholder address: nothing is launched
+    elif workspace is not None:
+        a.workspace, a.workspace_bytes = _ptr(workspace), workspace.numel() * workspace.element_size()
     out = ctypes.c_int32()
     _check("focus_prefill_kernel", lib.focus_prefill_kernel(ctypes.byref(cache.desc), ctypes.byref(a),
                                                            ctypes.byref(out)))

@@ -24,9 +24,10 @@ from . import focus
 
 
 def prefill_masked_parallel(cache: focus.Cache, q, k, v, L: dict, scale=None, o=None, lse=None, flags=0,
-                            stream=None):
+                            stream=None, workspace="auto"):
     focus.kv_compact_bulk(cache, k, v, L, 0, L["M"], src_row0=0, stream=stream)
-    return focus.attn_prefill(cache, q, k, v, L, 0, L["M"], scale=scale, o=o, lse=lse, flags=flags, stream=stream)
+    return focus.attn_prefill(cache, q, k, v, L, 0, L["M"], scale=scale, o=o, lse=lse, flags=flags, stream=stream,
+                              workspace=workspace)
 
 
 _side_streams: dict = {}

@@ -34,7 +34,7 @@ def test_struct_sizes_match_c_layout():
     # 2 x int64 + 8 pointers; 8 pointers + 7 int32 (+pad); see focus.h
     assert ctypes.sizeof(focus.LayoutOut) == 16 + 10 * 8
     assert ctypes.sizeof(focus.CacheDesc) == 8 * 8 + 8 * 4 + 8 + 8 + 8 + 8
-    assert ctypes.sizeof(focus.PrefillArgs) == 5 * 8 + 8 + 2 * 8 + 6 * 4
+    assert ctypes.sizeof(focus.PrefillArgs) == 5 * 8 + 8 + 2 * 8 + 6 * 4 + 2 * 8
     assert ctypes.sizeof(focus.CompactArgs) == 2 * 8 + 2 * 8 + 2 * 8 + 3 * 4 + 4
 
 
@@ -157,9 +157,25 @@ def test_prefill_kernel_choice_needs_no_gpu():
     c.k_per_window, c.n_windows = 4096, 128
     assert choice(1_280, 1_010, focus.PREFILL_KMER_LOCAL) == (0, 1)
     c.rope_theta = 10_000.0
-    assert choice(1_280, 1_010) == (0, 1)
+    assert choice(1_280, 1_010) == (0, 1)            # rotary embedding without a workspace
+    # with the workspace focus_prefill_workspace_size asks for: the persistent kernel,
+    # which rotates q and k once into it (counters + rotated q and k of the span)
+    c.C_ring, a.max_rows, a.flags = 1_280, 1_010, 0
+    need = lib.focus_prefill_workspace_size(ctypes.byref(c), ctypes.byref(a))
+    assert need == 256 + c.B * c.H * 2 * a.T_span * c.d * 2
+    a.workspace, a.workspace_bytes = 4096, need
+    assert choice(1_280, 1_010) == (0, 2)
+    a.workspace_bytes = need - 1
+    assert choice(1_280, 1_010) == (0, 1)            # too small: the per-item kernel
+    a.workspace, a.workspace_bytes = 4100, need
+    assert choice(1_280, 1_010)[0] == 2              # misaligned workspace
+    a.workspace, a.workspace_bytes = 4096, need
+    assert choice(10_000, 1_010) == (0, 1)           # long items: no workspace wanted
+    assert lib.focus_prefill_workspace_size(ctypes.byref(c), ctypes.byref(a)) == 0
+    a.workspace, a.workspace_bytes = None, 0
     assert choice(1_280, 1_010, focus.PREFILL_LEGACY_MMA)[0] == 2      # legacy has no rotary embedding
     c.rope_theta = 0.0
+    assert lib.focus_prefill_workspace_size(ctypes.byref(c), ctypes.byref(a)) == 0
     assert choice(1_280, 1_010, 8)[0] == 1                              # unknown flag bit
     assert lib.focus_prefill_kernel(ctypes.byref(c), ctypes.byref(a), None) == 1
 

@@ -71,10 +71,15 @@ ROPE_CASES = [
 ]
 
 
+# with the workspace the persistent kernel rotates q and k once (warps 2-3 of
+# every CTA, a head ahead of the attention); without it the one-CTA-per-item
+# kernel rotates each tile it loads
+@pytest.mark.parametrize("ws,kernel", [("auto", "tcgen05 persistent"), (None, "tcgen05, one CTA per work item")])
 @pytest.mark.parametrize("N,W,ks,B,H,d,theta", ROPE_CASES)
-def test_prefill_rope_masked_parallel_matches_oracle(N, W, ks, B, H, d, theta):
+def test_prefill_rope_masked_parallel_matches_oracle(N, W, ks, B, H, d, theta, ws, kernel):
     L, k, q, kk, v, cache = _case(N, W, ks, B, H, d, theta, seed=N + 3)
-    o, lse = pipeline.prefill_masked_parallel(cache, q, kk, v, L)
+    assert focus.prefill_kernel(cache, q, kk, v, L, workspace=ws) == kernel
+    o, lse = pipeline.prefill_masked_parallel(cache, q, kk, v, L, workspace=ws)
     torch.cuda.synchronize()
     o_ref, lse_ref, kf, ref_L = _ref_all_rows(N, W, k, q, kk, v, theta)
     assert_attn_close(o, lse, o_ref, lse_ref, f"rope N={N} W={W} k={ks}")
@@ -82,6 +87,38 @@ def test_prefill_rope_masked_parallel_matches_oracle(N, W, ks, B, H, d, theta):
     R = L["R"]
     assert_keys_close(cache.ring_k[:, :, :R], kf[:, :, ref_L["sum_idx"]], "ring K", rel=2.0 ** -7)
     assert np.array_equal(bits(cache.ring_v)[:, :, :R], bits(v)[:, :, ref_L["sum_idx"]])
+
+
+@pytest.mark.parametrize("ws", ["auto", None])
+@pytest.mark.parametrize("g,d", [(4, 128), (3, 64)])
+def test_prefill_rope_grouped_heads_match_oracle(g, d, ws):
+    """Grouped-query heads with the rotary embedding: query head hq uses K/V head
+    hq // g; every query head and K/V head is rotated at the layout's positions."""
+    N, W, ks, B, Hk, theta = 3_000, 1_000, [100, 50, 7], 2, 2, 10_000.0
+    M = -(-N // W)
+    k = np.resize(np.asarray(ks, np.int32), M)
+    L = focus.layout(N, W, k)
+    q = inputs.normal_bf16((B, Hk * g, L["T"], d), 1.0, seed=81, device="cuda")
+    kk = inputs.normal_bf16((B, Hk, L["T"], d), 1.0, seed=82, device="cuda")
+    v = inputs.normal_bf16((B, Hk, L["T"], d), 1.0, seed=83, device="cuda")
+    cache = focus.Cache(B, Hk, d, C_ring=L["R"], k_sched=k, rope_theta=theta, q_per_kv=g)
+    o, lse = pipeline.prefill_masked_parallel(cache, q, kk, v, L, workspace=ws)
+    torch.cuda.synchronize()
+    T = L["T"]
+    ref_L = fo.layout(N, W, k)
+    pos = np.arange(T)
+    qf = fo.rope(q.reshape(B * Hk * g, T, d).cpu(), pos, theta, round_bf16=True)
+    kf = fo.rope(kk.reshape(B * Hk, T, d).cpu(), pos, theta, round_bf16=True)
+    kv_of = np.arange(B * Hk * g) // g                  # K/V head of each (sequence, query head)
+    kf_q = kf[kv_of]
+    v_q = v.reshape(B * Hk, T, d).cpu()[torch.from_numpy(kv_of)]
+    rows = np.arange(0, T, 3)
+    heads = np.repeat(np.arange(B * Hk * g), rows.size)
+    o_ref, lse_ref = fo.attn_rows_f64(qf, kf_q, v_q, ref_L["keep"], ref_L["win"], 1.0 / math.sqrt(d), heads,
+                                      np.tile(rows, B * Hk * g))
+    assert_attn_close(o.reshape(B * Hk * g, T, d)[:, rows], lse.reshape(B * Hk * g, T)[:, rows],
+                      o_ref.reshape(B * Hk * g, rows.size, d), lse_ref.reshape(B * Hk * g, rows.size),
+                      f"rope gqa g={g} ws={ws}")
 
 
 @pytest.mark.parametrize("d", [64, 128])
