@@ -275,7 +275,7 @@ def run_prefill_leg(args, cfg, world, rank, local):
     from paper_2511_14694_gb300 import focus, inputs, pipeline
 
     B, N, W, H, d = cfg["B"], cfg["N"], cfg["W"], cfg["H"], cfg["d"]
-    M = -(-N // W)
+    M = focus.n_windows(N, W)
     k_s = inputs.k_schedule(M, cfg["k"], seed=inputs.DEFAULT_SEED)
     dev = torch.device("cuda", local)
     nt = inputs.nucleotides(B, N, seed=inputs.DEFAULT_SEED, device=dev)
@@ -409,7 +409,7 @@ def run_stream_leg(args, cfg, world, rank, local):
     from paper_2511_14694_gb300 import focus, inputs, pipeline
 
     B, N, W, H, d, P = cfg["B"], cfg["N"], cfg["W"], cfg["H"], cfg["d"], cfg["pool"]
-    M = -(-N // W)
+    M = focus.n_windows(N, W)
     k_s = inputs.k_schedule(M, cfg["k"], seed=inputs.DEFAULT_SEED)
     dev = torch.device("cuda", local)
     L = focus.layout(N, W, k_s, device=dev)
@@ -503,7 +503,7 @@ def run_embed_leg(args, world, rank, local):
     from paper_2511_14694_gb300.workloads import WORKLOADS
     cfg = WORKLOADS["prefill_128kb_h32_d128"]
     N, W, D = cfg["N"], cfg["W"], args.embed_d
-    M = -(-N // W)
+    M = focus.n_windows(N, W)
     k_s = inputs.k_schedule(M, cfg["k"], seed=inputs.DEFAULT_SEED)
     dev = torch.device("cuda", local)
     nt = inputs.nucleotides(1, N, seed=inputs.DEFAULT_SEED + rank, device=dev)
@@ -822,7 +822,7 @@ def run_reference(args, world, rank, local):
                           "workloads only"}), flush=True)
         return
     B, N, W, H, d = cfg["B"], cfg["N"], cfg["W"], cfg["H"], cfg["d"]
-    M = -(-N // W)
+    M = fo.n_windows(N, W)
     k_s = inputs.k_schedule(M, cfg["k"], seed=inputs.DEFAULT_SEED)
     L = fo.layout(N, W, k_s)
     # two heads of inputs, drawn with the same generator recipe on the CPU

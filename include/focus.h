@@ -83,6 +83,19 @@ focus_status focus_get_device_status(int32_t* host_status, int32_t clear, cudaSt
 /* position of its own); Sec. 3.3 (augmented sequence y_1..y_N').           */
 /* ------------------------------------------------------------------------ */
 
+/* Host-only arithmetic: the number of windows M that cover n_nt >= 0 bases with
+ * windows of W >= 1 bases, M = ceil(n_nt / W) (App. A); 0 for n_nt = 0.
+ * FOCUS_ERR_INVALID_ARG for a negative n_nt, W < 1, a NULL M or an M above INT32_MAX. */
+focus_status focus_layout_windows(int64_t n_nt, int32_t W, int32_t* M);
+
+/* Adaptive windowing (see focus_layout_size_sched): of a window-length schedule
+ * h_W[0..n_sched) (HOST), the number M of leading windows whose lengths first
+ * reach n_nt bases in total, i.e. the windows that cover the sequence (the last
+ * one may be only partly used); 0 for n_nt = 0. FOCUS_ERR_INVALID_ARG if a length
+ * among them is < 1, if all n_sched lengths cover fewer than n_nt bases, or for
+ * NULL pointers. */
+focus_status focus_layout_windows_sched(int64_t n_nt, int32_t n_sched, const int32_t* h_W, int32_t* M);
+
 /* Host-only arithmetic: sizes of the augmented layout.
  *   n_nt        N >= 0 bases
  *   W           window length in bases, W >= 1

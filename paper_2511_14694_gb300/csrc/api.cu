@@ -156,6 +156,26 @@ focus_status layout_impl(int64_t n_nt, int32_t W, bool sched, const int32_t* d_W
 
 extern "C" {
 
+focus_status focus_layout_windows(int64_t n_nt, int32_t W, int32_t* M) {
+    if (!M || n_nt < 0 || W < 1) return FOCUS_ERR_INVALID_ARG;
+    const int64_t m = focus::ceil_div64(n_nt, W);
+    if (m > INT32_MAX) return FOCUS_ERR_INVALID_ARG;
+    *M = (int32_t)m;
+    return FOCUS_OK;
+}
+
+focus_status focus_layout_windows_sched(int64_t n_nt, int32_t n_sched, const int32_t* h_W, int32_t* M) {
+    if (!M || n_nt < 0 || n_sched < 0 || (n_sched > 0 && !h_W)) return FOCUS_ERR_INVALID_ARG;
+    int64_t covered = 0;
+    int32_t m = 0;
+    while (covered < n_nt) {
+        if (m >= n_sched || h_W[m] < 1) return FOCUS_ERR_INVALID_ARG;
+        covered += h_W[m++];
+    }
+    *M = m;
+    return FOCUS_OK;
+}
+
 focus_status focus_layout_size(int64_t n_nt, int32_t W, int32_t n_windows, const int32_t* h_k, uint32_t flags,
                                int32_t tail, int64_t* T, int64_t* R, int32_t* max_rows) {
     return layout_size_impl(n_nt, W, false, nullptr, n_windows, h_k, flags, tail, T, R, max_rows);

@@ -78,6 +78,10 @@ def load() -> ctypes.CDLL:
     lib.focus_status_string.argtypes = [ctypes.c_int]
     lib.focus_get_device_status.restype = ctypes.c_int
     lib.focus_get_device_status.argtypes = [_P, _i32, _P]
+    lib.focus_layout_windows.restype = ctypes.c_int
+    lib.focus_layout_windows.argtypes = [_i64, _i32, _P]
+    lib.focus_layout_windows_sched.restype = ctypes.c_int
+    lib.focus_layout_windows_sched.argtypes = [_i64, _i32, _P, _P]
     lib.focus_layout_size.restype = ctypes.c_int
     lib.focus_layout_size.argtypes = [_i64, _i32, _i32, _P, _u32, _i32, _P, _P, _P]
     lib.focus_layout.restype = ctypes.c_int
@@ -136,19 +140,28 @@ def _cuda(t: torch.Tensor, name: str, dtype=None):
 
 # ----------------------------------------------------------------------------- layout
 
+def n_windows(N: int, W) -> int:
+    """M, the windows that cover N bases (focus_layout_windows, or
+    focus_layout_windows_sched for a per-window sequence W)."""
+    lib = load()
+    M = _i32()
+    if np.ndim(W) == 0:
+        _check("focus_layout_windows", lib.focus_layout_windows(int(N), int(W), ctypes.byref(M)))
+    else:
+        Ws = np.ascontiguousarray(np.asarray(W, dtype=np.int32).reshape(-1))
+        _check("focus_layout_windows_sched",
+               lib.focus_layout_windows_sched(int(N), int(Ws.size), Ws.ctypes.data, ctypes.byref(M)))
+    return M.value
+
+
 def window_lengths(N: int, W):
     """None for windows of one integer length W; for a per-window sequence W
-    (adaptive windowing) the int32 lengths of the windows that cover N bases: the
-    shortest prefix whose sum reaches N."""
+    (adaptive windowing) the int32 lengths of the windows that cover N bases (the
+    library's count of them, focus_layout_windows_sched)."""
     if np.ndim(W) == 0:
         return None
-    Ws = np.asarray(W, dtype=np.int64).reshape(-1)
-    if N == 0:
-        return np.zeros(0, np.int32)
-    cover = np.cumsum(Ws)
-    if cover.size == 0 or cover[-1] < N:
-        raise ValueError("window lengths do not cover the sequence")
-    return np.ascontiguousarray(Ws[:int(np.searchsorted(cover, N)) + 1].astype(np.int32))
+    Ws = np.asarray(W, dtype=np.int32).reshape(-1)
+    return np.ascontiguousarray(Ws[:n_windows(N, Ws)])
 
 
 def layout_size(N: int, W, k_sched, close_tail: bool = True, tail: int = 0):
@@ -156,7 +169,7 @@ def layout_size(N: int, W, k_sched, close_tail: bool = True, tail: int = 0):
     library). W: one window length, or a per-window sequence."""
     lib = load()
     Ws = window_lengths(N, W)
-    M = -(-N // int(W)) if Ws is None else int(Ws.size)
+    M = n_windows(N, W) if Ws is None else int(Ws.size)
     k = np.ascontiguousarray(np.broadcast_to(np.asarray(k_sched, dtype=np.int32), (M,)))
     T, R, mx = _i64(), _i64(), _i32()
     flags = LAYOUT_CLOSE_TAIL if close_tail else 0

@@ -300,3 +300,38 @@ def test_decode_bindings_check_head_counts_before_any_call(monkeypatch):
             fn(cache, q, kv, kv)
     with pytest.raises(ValueError, match="heads"):
         focus.attn_decode_noalloc(cache, torch.zeros((2, 16, 128)), kv[:, :2], kv)
+
+
+@pytest.mark.parametrize("N,W", [(0, 1_000), (1, 1), (4_000, 1_000), (4_001, 1_000), (128_000, 1_000), (77, 100),
+                                 (1_000_000, 1_000), (10, 4)])
+def test_layout_windows_matches_oracle(N, W):
+    lib = focus.load()
+    M = ctypes.c_int32(-1)
+    assert lib.focus_layout_windows(N, W, ctypes.byref(M)) == 0
+    assert M.value == fo.n_windows(N, W) == len(fo.window_schedule(N, W))
+
+
+@pytest.mark.parametrize("N,Ws", [(0, [5]), (10, [10]), (10, [3, 3, 3, 3, 3]), (9, [3, 3, 3, 3]),
+                                  (1_000, [400, 100, 700, 1]), (5, [1, 1, 1, 1, 1, 9, 9])])
+def test_layout_windows_sched_matches_oracle(N, Ws):
+    lib = focus.load()
+    W = np.asarray(Ws, np.int32)
+    M = ctypes.c_int32(-1)
+    assert lib.focus_layout_windows_sched(N, W.size, W.ctypes.data, ctypes.byref(M)) == 0
+    assert M.value == len(fo.window_schedule(N, W))
+    assert np.array_equal(focus.window_lengths(N, W), fo.window_schedule(N, W))
+
+
+def test_layout_windows_rejects_bad_arguments():
+    lib = focus.load()
+    M = ctypes.c_int32()
+    assert lib.focus_layout_windows(-1, 10, ctypes.byref(M)) == 1
+    assert lib.focus_layout_windows(10, 0, ctypes.byref(M)) == 1
+    assert lib.focus_layout_windows(10, 10, None) == 1
+    short = np.array([3, 3], np.int32)
+    assert lib.focus_layout_windows_sched(7, 2, short.ctypes.data, ctypes.byref(M)) == 1     # does not cover
+    bad = np.array([3, 0, 9], np.int32)
+    assert lib.focus_layout_windows_sched(7, 3, bad.ctypes.data, ctypes.byref(M)) == 1       # empty window
+    assert lib.focus_layout_windows_sched(7, 3, None, ctypes.byref(M)) == 1
+    with pytest.raises(focus.FocusError):
+        focus.window_lengths(7, short)
