@@ -380,8 +380,8 @@ def run_prefill_leg(args, cfg, world, rank, local):
         d2h = h_o.numel() * h_o.element_size() + h_lse.numel() * h_lse.element_size()
         e2e = {"value": world * B * N / (e2e_ms / 1e3), "unit": "nt/s", "ms_per_step": e2e_ms,
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps_e2e,
-               "api": "pipeline.prefill_masked_parallel_host (%d head groups; copies overlap kernels)"
-                      % args.e2e_groups}
+               "api": "focus_prefill_host (C ABI, host buffers in and out; %d head groups, each group's "
+                      "copies on two side streams overlapping the other groups' kernels)" % args.e2e_groups}
         del h_q, h_k, h_v, h_o, h_lse, host
 
     host_sample = None

@@ -281,6 +281,65 @@ focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_ar
 focus_status focus_prefill_kernel(const focus_cache* cache, const focus_prefill_args* args, int32_t* kernel);
 
 /* ------------------------------------------------------------------------ */
+/* focus_prefill_host — the masked-parallel prefill (App. A.1) of a layer    */
+/* whose inputs and outputs are in host memory.                             */
+/* ------------------------------------------------------------------------ */
+typedef struct focus_prefill_host_args {
+    /* host memory; pinned (cudaHostAlloc / cudaHostRegister) for the copies to
+     * overlap the kernels. Shapes as for focus_layout and focus_attn_prefill over
+     * all windows (T = layout->T, g = cache->q_per_kv, at least 1): */
+    const uint8_t* h_nt;      /* [B][n_nt] nucleotide ids */
+    const void*    h_q;       /* bf16 [B][H g][T][d] */
+    const void*    h_k;       /* bf16 [B][H][T][d] */
+    const void*    h_v;       /* bf16 [B][H][T][d] */
+    void*          h_o;       /* bf16 [B][H g][T][d], written */
+    float*         h_lse;     /* fp32 [B][H g][T], written; may be NULL (then d_lse may be too) */
+    /* device buffers of the same shapes, caller-owned (reused across calls) */
+    uint8_t* d_nt;
+    void*    d_q;
+    void*    d_k;
+    void*    d_v;
+    void*    d_o;
+    float*   d_lse;
+    /* the layout, as for focus_layout / focus_layout_sched (d_W_sched NULL: windows
+     * of W bases); layout->tok is written from d_nt (B rows) */
+    int64_t  n_nt;
+    int32_t  W;
+    const int32_t* d_W_sched;
+    int32_t  n_windows;
+    const int32_t* d_k_sched;
+    uint32_t layout_flags;
+    int32_t  tail;
+    const focus_layout_out* layout;
+    int32_t  max_rows;        /* from focus_layout_size */
+    float    scale;           /* softmax scale > 0 */
+    uint32_t prefill_flags;   /* FOCUS_PREFILL_* */
+    void*    workspace;       /* as in focus_prefill_args, shared by the parts in turn (its size for the
+                                 whole cache covers every part), or NULL */
+    size_t   workspace_bytes;
+    int32_t  groups;          /* parts the heads (B = 1) or the sequences (B > 1) are cut into, >= 1 */
+    cudaStream_t copy_in;     /* two streams of the caller, other than `stream`, for the copies in and out */
+    cudaStream_t copy_out;
+} focus_prefill_host_args;
+
+/* The same computation as focus_layout + focus_kv_compact (bulk, all windows) +
+ * focus_attn_prefill (all windows), from and to host memory: the token ids are
+ * copied in and the layout built once; then for each of `groups` parts (K/V heads
+ * [h0, h1) of the one sequence when B = 1, else sequences [b0, b1)) the part's q,
+ * k, v are copied in on copy_in, its compaction and attention run on `stream`,
+ * and its o and lse are copied out on copy_out, so that one part's copies overlap
+ * the other parts' kernels and copies. One cudaMemcpyAsync per tensor and part
+ * (a part is contiguous in every tensor). Outputs equal those of the device-buffer
+ * calls bit for bit. Asynchronous: once `stream` has reached the end of the call,
+ * so have the copies out (the call makes `stream` wait for copy_out); the device
+ * buffers may be reused from there. The call creates and releases its own CUDA
+ * events (no device memory). Argument errors as for the three calls it makes,
+ * plus FOCUS_ERR_INVALID_ARG for missing pointers, groups < 1, or copy streams
+ * equal to `stream`. Passage: App. A.1 "Cross-window consistency" (the
+ * masked-parallel form) and App. A, "KV compression and budget". */
+focus_status focus_prefill_host(const focus_cache* cache, const focus_prefill_host_args* args, cudaStream_t stream);
+
+/* ------------------------------------------------------------------------ */
 /* focus_attn_decode — one new token per sequence against the compressed    */
 /* cache (App. A.2; decoding keeps the base decoder's interface).           */
 /* ------------------------------------------------------------------------ */

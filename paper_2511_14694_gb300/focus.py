@@ -53,6 +53,15 @@ class PrefillArgs(ctypes.Structure):
                 ("scale", _f32), ("flags", _u32), ("workspace", _P), ("workspace_bytes", ctypes.c_size_t)]
 
 
+class PrefillHostArgs(ctypes.Structure):
+    _fields_ = [("h_nt", _P), ("h_q", _P), ("h_k", _P), ("h_v", _P), ("h_o", _P), ("h_lse", _P),
+                ("d_nt", _P), ("d_q", _P), ("d_k", _P), ("d_v", _P), ("d_o", _P), ("d_lse", _P),
+                ("n_nt", _i64), ("W", _i32), ("d_W_sched", _P), ("n_windows", _i32), ("d_k_sched", _P),
+                ("layout_flags", _u32), ("tail", _i32), ("layout", ctypes.POINTER(LayoutOut)), ("max_rows", _i32),
+                ("scale", _f32), ("prefill_flags", _u32), ("workspace", _P), ("workspace_bytes", ctypes.c_size_t),
+                ("groups", _i32), ("copy_in", _P), ("copy_out", _P)]
+
+
 class CompactArgs(ctypes.Structure):
     _fields_ = [("src_k", _P), ("src_v", _P), ("src_T", _i64), ("src_row0", _i64), ("d_sum_idx", _P),
                 ("d_ring_off", _P), ("n_windows", _i32), ("w_begin", _i32), ("w_end", _i32)]
@@ -96,6 +105,8 @@ def load() -> ctypes.CDLL:
     lib.focus_prefill_kernel.argtypes = [ctypes.POINTER(CacheDesc), ctypes.POINTER(PrefillArgs), _P]
     lib.focus_prefill_workspace_size.restype = ctypes.c_size_t
     lib.focus_prefill_workspace_size.argtypes = [ctypes.POINTER(CacheDesc), ctypes.POINTER(PrefillArgs)]
+    lib.focus_prefill_host.restype = ctypes.c_int
+    lib.focus_prefill_host.argtypes = [ctypes.POINTER(CacheDesc), ctypes.POINTER(PrefillHostArgs), _P]
     lib.focus_decode_workspace_size.restype = ctypes.c_size_t
     lib.focus_decode_workspace_size.argtypes = [ctypes.POINTER(CacheDesc)]
     lib.focus_attn_decode.restype = ctypes.c_int
@@ -204,6 +215,12 @@ def layout_alloc(N: int, W, k_sched, B: int = 0, close_tail: bool = True, device
     return out
 
 
+def _layout_desc(L: dict, with_tok: bool) -> LayoutOut:
+    return LayoutOut(L["T"], L["R"], _ptr(L["kind"]), _ptr(L["src"]), _ptr(L["pos"]), _ptr(L["win"]),
+                     _ptr(L["tok"]) if with_tok else None, _ptr(L["keep"]), _ptr(L["win_off"]),
+                     _ptr(L["ring_off"]), _ptr(L["sum_idx_buf"]), _ptr(L["base_off"]))
+
+
 def layout_run(L: dict, nt: torch.Tensor | None = None, stream=None) -> None:
     """Launch focus_layout into buffers from layout_alloc (asynchronous)."""
     lib = load()
@@ -211,9 +228,7 @@ def layout_run(L: dict, nt: torch.Tensor | None = None, stream=None) -> None:
         _cuda(nt, "nt", torch.uint8)
         if L["tok"] is None or tuple(nt.shape) != (L["B"], L["N"]):
             raise ValueError("nt shape does not match the allocated layout")
-    desc = LayoutOut(L["T"], L["R"], _ptr(L["kind"]), _ptr(L["src"]), _ptr(L["pos"]), _ptr(L["win"]),
-                     _ptr(L["tok"]) if nt is not None else None, _ptr(L["keep"]), _ptr(L["win_off"]),
-                     _ptr(L["ring_off"]), _ptr(L["sum_idx_buf"]), _ptr(L["base_off"]))
+    desc = _layout_desc(L, nt is not None)
     flags = LAYOUT_CLOSE_TAIL if L["close_tail"] else 0
     B = 0 if nt is None else L["B"]
     if L["W_dev"] is None:
@@ -373,6 +388,44 @@ def attn_prefill(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | 
     a = _prefill_args(q, k, v, o, lse, L, w_begin, w_end, scale, flags, workspace)
     _check("focus_attn_prefill", lib.focus_attn_prefill(ctypes.byref(cache.desc), ctypes.byref(a), _stream(stream)))
     return o, lse
+
+
+def prefill_host(cache: Cache, L: dict, host: dict, dev: dict, copy_in, copy_out, groups: int = 8, scale=None,
+                 flags: int = 0, workspace="auto", stream=None):
+    """focus_prefill_host: the masked-parallel prefill of a layer whose inputs and
+    outputs are in (pinned) host memory. host["nt"] (uint8 [B, N]),
+    host["q"/"k"/"v"] (bf16 [B, H, T, d]) in; host["o"] (bf16) and host["lse"]
+    (fp32 [B, H, T], or None) out; ``dev`` holds device tensors of the same
+    shapes; L from layout_alloc (its tok is written). The library copies each
+    group of heads (B = 1) or sequences in on ``copy_in``, runs its compaction and
+    attention on ``stream`` and copies it out on ``copy_out``; work is only
+    enqueued, and once ``stream`` is done, so is everything."""
+    lib = load()
+    for name in ("nt", "q", "k", "v", "o"):
+        if not (isinstance(host[name], torch.Tensor) and not host[name].is_cuda and host[name].is_contiguous()):
+            raise ValueError(f"host[{name!r}] must be a contiguous host tensor")
+        _cuda(dev[name], f"dev[{name!r}]")
+        if tuple(host[name].shape) != tuple(dev[name].shape):
+            raise ValueError(f"host[{name!r}] and dev[{name!r}] differ in shape")
+    _check_heads(cache, dev["q"], dev["k"], dev["v"])
+    if tuple(dev["nt"].shape) != (L["B"], L["N"]) or L["tok"] is None:
+        raise ValueError("nt shape does not match the allocated layout")
+    d = dev["q"].shape[-1]
+    scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
+    if isinstance(workspace, str):
+        workspace = new_prefill_workspace(cache, dev["q"], dev["k"], dev["v"], L, flags=flags)
+    desc = _layout_desc(L, True)
+    lse_h, lse_d = host.get("lse"), dev.get("lse")
+    a = PrefillHostArgs(_ptr(host["nt"]), _ptr(host["q"]), _ptr(host["k"]), _ptr(host["v"]), _ptr(host["o"]),
+                        _ptr(lse_h), _ptr(dev["nt"]), _ptr(dev["q"]), _ptr(dev["k"]), _ptr(dev["v"]),
+                        _ptr(dev["o"]), _ptr(lse_d) if lse_h is not None else None, L["N"],
+                        0 if L["W_dev"] is not None else int(L["W"]), _ptr(L["W_dev"]), L["M"], _ptr(L["k"]),
+                        LAYOUT_CLOSE_TAIL if L["close_tail"] else 0, int(L["tail"]), ctypes.pointer(desc),
+                        int(L["max_rows"]), scale, flags, _ptr(workspace),
+                        0 if workspace is None else workspace.numel() * workspace.element_size(), int(groups),
+                        copy_in.cuda_stream, copy_out.cuda_stream)
+    _check("focus_prefill_host", lib.focus_prefill_host(ctypes.byref(cache.desc), ctypes.byref(a), _stream(stream)))
+    return host["o"], lse_h
 
 
 PREFILL_KERNELS = {0: "legacy mma.sync", 1: "tcgen05, one CTA per work item", 2: "tcgen05 persistent"}

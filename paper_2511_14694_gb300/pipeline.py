@@ -34,11 +34,12 @@ _side_streams: dict = {}
 
 
 def prefill_masked_parallel_host(cache: focus.Cache, L: dict, host: dict, dev: dict, groups: int = 8, scale=None,
-                                 flags=0, stream=None):
+                                 flags=0, stream=None, workspace="auto"):
     """Masked-parallel prefill of a layer whose inputs and outputs live in pinned
-    host memory: host["nt"] (uint8 [B, N]), host["q"/"k"/"v"] (bf16 [B, H, T, d])
-    in, host["o"] (bf16) and host["lse"] (fp32 [B, H, T]) out; ``dev`` holds
-    device tensors of the same shapes, reused across calls.
+    host memory, through the library's focus_prefill_host: host["nt"] (uint8
+    [B, N]), host["q"/"k"/"v"] (bf16 [B, H, T, d]) in, host["o"] (bf16) and
+    host["lse"] (fp32 [B, H, T]) out; ``dev`` holds device tensors of the same
+    shapes, reused across calls.
 
     The layout runs once; then the K/V heads (one sequence) or the sequences go
     in ``groups`` parts, and part i's Q/K/V copy in on one side stream, its
@@ -51,39 +52,8 @@ def prefill_masked_parallel_host(cache: focus.Cache, L: dict, host: dict, dev: d
     if key not in _side_streams:
         _side_streams[key] = (torch.cuda.Stream(device=key), torch.cuda.Stream(device=key))
     s_in, s_out = _side_streams[key]
-    B, H, g = cache.B, cache.H, max(cache.q_per_kv, 1)
-    by_head = B == 1
-    n = H if by_head else B
-    groups = max(1, min(groups, n))
-    bounds = [n * i // groups for i in range(groups + 1)]
-    # the previous call's compute and copy-out are done with the device buffers
-    s_in.wait_stream(cur)
-    s_in.wait_stream(s_out)
-    with torch.cuda.stream(s_in):
-        dev["nt"].copy_(host["nt"], non_blocking=True)
-    cur.wait_stream(s_in)
-    focus.layout_run(L, dev["nt"], stream=cur)
-    for lo, hi in zip(bounds[:-1], bounds[1:]):
-        if by_head:
-            part = cache.part(h0=lo, h1=hi)
-            kv, qo = (slice(None), slice(lo, hi)), (slice(None), slice(lo * g, hi * g))
-        else:
-            part = cache.part(b0=lo, b1=hi)
-            kv = qo = (slice(lo, hi),)
-        with torch.cuda.stream(s_in):
-            dev["q"][qo].copy_(host["q"][qo], non_blocking=True)
-            dev["k"][kv].copy_(host["k"][kv], non_blocking=True)
-            dev["v"][kv].copy_(host["v"][kv], non_blocking=True)
-        cur.wait_stream(s_in)
-        focus.kv_compact_bulk(part, dev["k"][kv], dev["v"][kv], L, 0, L["M"], src_row0=0, stream=cur)
-        focus.attn_prefill(part, dev["q"][qo], dev["k"][kv], dev["v"][kv], L, 0, L["M"], scale=scale,
-                           o=dev["o"][qo], lse=dev["lse"][qo], flags=flags, stream=cur)
-        s_out.wait_stream(cur)
-        with torch.cuda.stream(s_out):
-            host["o"][qo].copy_(dev["o"][qo], non_blocking=True)
-            host["lse"][qo].copy_(dev["lse"][qo], non_blocking=True)
-    cur.wait_stream(s_out)
-    return host["o"], host["lse"]
+    return focus.prefill_host(cache, L, host, dev, s_in, s_out, groups=groups, scale=scale, flags=flags,
+                              workspace=workspace, stream=cur)
 
 
 def prefill_streaming(cache: focus.Cache, L: dict, window_qkv, outs, lses, w_begin: int = 0, w_end: int | None = None,

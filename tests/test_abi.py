@@ -36,6 +36,9 @@ def test_struct_sizes_match_c_layout():
     assert ctypes.sizeof(focus.CacheDesc) == 8 * 8 + 8 * 4 + 8 + 8 + 8 + 8
     assert ctypes.sizeof(focus.PrefillArgs) == 5 * 8 + 8 + 2 * 8 + 6 * 4 + 2 * 8
     assert ctypes.sizeof(focus.CompactArgs) == 2 * 8 + 2 * 8 + 2 * 8 + 3 * 4 + 4
+    # 12 buffer pointers, n_nt, W (+pad), d_W_sched, n_windows (+pad), d_k_sched, flags, tail, layout,
+    # max_rows, scale, prefill_flags (+pad), workspace, its size, groups (+pad), two streams
+    assert ctypes.sizeof(focus.PrefillHostArgs) == 12 * 8 + 8 + 8 + 8 + 8 + 8 + 8 + 8 + 16 + 8 + 8 + 8 + 16
 
 
 def test_version_and_status_strings():
@@ -335,3 +338,27 @@ def test_layout_windows_rejects_bad_arguments():
     assert lib.focus_layout_windows_sched(7, 3, None, ctypes.byref(M)) == 1
     with pytest.raises(focus.FocusError):
         focus.window_lengths(7, short)
+
+
+def test_prefill_host_rejects_bad_arguments_before_any_cuda_call():
+    lib = focus.load()
+    c = focus.CacheDesc()
+    c.B, c.H, c.d = 1, 2, 128
+    L = focus.LayoutOut()
+    a = focus.PrefillHostArgs()
+    for f in ("h_nt", "h_q", "h_k", "h_v", "h_o", "d_nt", "d_q", "d_k", "d_v", "d_o"):
+        setattr(a, f, 4096)
+    a.layout = ctypes.pointer(L)
+    a.n_nt, a.W, a.n_windows, a.groups = 1_000, 1_000, 1, 2
+    a.copy_in, a.copy_out = 8, 16
+    assert lib.focus_prefill_host(None, ctypes.byref(a), 24) == 1
+    a.groups = 0
+    assert lib.focus_prefill_host(ctypes.byref(c), ctypes.byref(a), 24) == 1       # groups < 1
+    a.groups = 2
+    assert lib.focus_prefill_host(ctypes.byref(c), ctypes.byref(a), 8) == 1        # copy_in is the stream
+    a.copy_out = 8
+    assert lib.focus_prefill_host(ctypes.byref(c), ctypes.byref(a), 24) == 1       # one copy stream for both
+    a.copy_out, a.h_lse = 16, 4096
+    assert lib.focus_prefill_host(ctypes.byref(c), ctypes.byref(a), 24) == 1       # lse out without a device lse
+    a.h_lse, a.d_q = None, None
+    assert lib.focus_prefill_host(ctypes.byref(c), ctypes.byref(a), 24) == 1       # missing device buffer

@@ -1,5 +1,5 @@
-"""The masked-parallel prefill from pinned host memory (pipeline.
-prefill_masked_parallel_host) runs the same kernels per group of heads or
+"""The masked-parallel prefill from pinned host memory (focus_prefill_host,
+through pipeline.prefill_masked_parallel_host) runs the same kernels per group of heads or
 sequences, with the copies on side streams: its outputs must equal, bit for bit,
 those of the all-at-once device path on the same inputs, and the ring must hold
 the same rows."""
@@ -24,8 +24,9 @@ def _clean_status():
     assert focus.device_status(clear=True) == 0, "a kernel reported an error"
 
 
-@pytest.mark.parametrize("B,H,d,g,groups", [(1, 4, 64, 1, 3), (3, 2, 128, 1, 2), (1, 2, 128, 2, 2), (2, 2, 64, 1, 8)])
-def test_host_pipeline_matches_device_path(B, H, d, g, groups):
+@pytest.mark.parametrize("B,H,d,g,groups,rope", [(1, 4, 64, 1, 3, 0.0), (3, 2, 128, 1, 2, 0.0), (1, 2, 128, 2, 2, 0.0),
+                                                 (2, 2, 64, 1, 8, 0.0), (1, 4, 128, 1, 2, 10_000.0)])
+def test_host_pipeline_matches_device_path(B, H, d, g, groups, rope):
     N, W = 5_000, 1_000
     k = inputs.k_schedule(-(-N // W), [100, 10, 50], seed=3)
     L_dev = focus.layout_alloc(N, W, k, B=B)
@@ -35,7 +36,7 @@ def test_host_pipeline_matches_device_path(B, H, d, g, groups):
     q, kk, v = inputs.qkv((B, H * g, T, d), std=1.0, seed=7, device="cuda", q_per_kv=g)
     # the device path
     focus.layout_run(L_dev, nt)
-    c_dev = focus.Cache(B, H, d, C_ring=L_dev["R"], k_sched=k, q_per_kv=g)
+    c_dev = focus.Cache(B, H, d, C_ring=L_dev["R"], k_sched=k, q_per_kv=g, rope_theta=rope)
     o_dev, lse_dev = pipeline.prefill_masked_parallel(c_dev, q, kk, v, L_dev)
     # the host path
     pin = lambda t: t.cpu().pin_memory()                                  # noqa: E731
@@ -43,7 +44,7 @@ def test_host_pipeline_matches_device_path(B, H, d, g, groups):
                 lse=torch.empty((B, H * g, T), dtype=torch.float32).pin_memory())
     dev = dict(nt=torch.empty_like(nt), q=torch.empty_like(q), k=torch.empty_like(kk), v=torch.empty_like(v),
                o=torch.empty_like(q), lse=torch.empty((B, H * g, T), dtype=torch.float32, device="cuda"))
-    c_host = focus.Cache(B, H, d, C_ring=L_host["R"], k_sched=k, q_per_kv=g)
+    c_host = focus.Cache(B, H, d, C_ring=L_host["R"], k_sched=k, q_per_kv=g, rope_theta=rope)
     pipeline.prefill_masked_parallel_host(c_host, L_host, host, dev, groups=groups)
     torch.cuda.synchronize()
     assert np.array_equal(bits(host["o"]), bits(o_dev))
