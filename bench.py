@@ -734,12 +734,12 @@ def run_focus(args, world, rank, local):
     local_mask = pre.get("local_mask", False)
     # committed DRAM counters exist for the 128 kb workload's appendix-mask kernel
     # (persistent) and k-mer-local kernel, default heads
-    traffic_key = {("tcgen05 persistent", False): ("prefill_attention", "prefill_tc_persistent.cu"),
-                   ("tcgen05, one CTA per work item", True): ("prefill_attention_kmer_local", "prefill_tc.cu")
-                   }.get((pre["kernel"], local_mask))
+    traffic_key = {("tcgen05 persistent", False, False): ("prefill_attention", "prefill_tc_persistent.cu"),
+                   ("tcgen05 persistent", False, True): ("prefill_attention_rope", "prefill_tc_persistent.cu"),
+                   ("tcgen05, one CTA per work item", True, False): ("prefill_attention_kmer_local", "prefill_tc.cu")
+                   }.get((pre["kernel"], local_mask, bool(args.rope)))
     traffic = None
-    if (traffic_key and not args.rope and args.q_per_kv == 1
-            and cfg is WORKLOADS["prefill_128kb_h32_d128"]):
+    if traffic_key and args.q_per_kv == 1 and cfg is WORKLOADS["prefill_128kb_h32_d128"]:
         traffic = kernel_traffic(traffic_key[0], "paper_2511_14694_gb300/csrc/" + traffic_key[1])
     line = {
         "metric": METRIC,
