@@ -215,6 +215,10 @@ typedef struct focus_prefill_args {
     uint32_t    flags;        /* FOCUS_PREFILL_* */
     void*       workspace;    /* device scratch, 16-byte aligned, or NULL (see focus_prefill_workspace_size) */
     size_t      workspace_bytes;  /* its size in bytes */
+    const int32_t* h_k_per_window; /* optional HOST copy of cache->k_per_window (entries w_begin .. w_end-1
+                                      read), or NULL; lets FOCUS_PREFILL_KMER_LOCAL use its k-mer-tiled
+                                      kernel (below). Must hold the same values as the device schedule: a
+                                      kernel that finds them different reports FOCUS_ERR_INVALID_ARG */
 } focus_prefill_args;
 
 /* Device workspace that lets focus_attn_prefill use its fastest kernel for these
@@ -272,12 +276,21 @@ focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_ar
  *                                    items, whose start-up and epilogue it overlaps),
  *   FOCUS_PREFILL_KERNEL_PER_ITEM    the tcgen05 kernel with one CTA per work item
  *                                    (every other case).
+ *   FOCUS_PREFILL_KERNEL_KMER        the FOCUS_PREFILL_KMER_LOCAL mode with query tiles cut at
+ *                                    k-mer boundaries (one CTA per SM walking them): each tile's
+ *                                    keys, its k-mers' rows plus the few ring rows they see, fit one
+ *                                    128-row K/V tile. Taken when args->h_k_per_window is given, no
+ *                                    rotary embedding is on, and over the span's windows every k-mer
+ *                                    has at most 128 - RB rows, where RB (a multiple of 8, <= 64)
+ *                                    bounds the ring rows a tile sees: the boundary plus one FOCUS
+ *                                    row per k bases, 1 + ceil(max_rows / k_w).
  * The persistent kernel also takes the rotary-embedding case when args carries
  * focus_prefill_workspace_size(cache, args) bytes of workspace.
  * Both tcgen05 kernels compute the same rows (within rounding order). */
 #define FOCUS_PREFILL_KERNEL_LEGACY 0
 #define FOCUS_PREFILL_KERNEL_PER_ITEM 1
 #define FOCUS_PREFILL_KERNEL_PERSISTENT 2
+#define FOCUS_PREFILL_KERNEL_KMER 3
 focus_status focus_prefill_kernel(const focus_cache* cache, const focus_prefill_args* args, int32_t* kernel);
 
 /* ------------------------------------------------------------------------ */

@@ -71,14 +71,15 @@ cudaError_t get_encode(PFN_cuTensorMapEncodeTiled_v12000* out) {
 
 }  // namespace
 
-// 3-D map over a [BH][rows][d] bf16 tensor, box = 128 rows x 64 columns, 128-byte swizzle.
-cudaError_t make_map(CUtensorMap* m, const void* ptr, int d, int64_t rows, int64_t bh) {
+// 3-D map over a [BH][rows][d] bf16 tensor, box = box_rows rows x 64 columns
+// (a multiple of 8, <= 128), 128-byte swizzle.
+cudaError_t make_map(CUtensorMap* m, const void* ptr, int d, int64_t rows, int64_t bh, int box_rows) {
     PFN_cuTensorMapEncodeTiled_v12000 enc;
     cudaError_t e = get_encode(&enc);
     if (e != cudaSuccess) return e;
     cuuint64_t dims[3] = {(cuuint64_t)d, (cuuint64_t)rows, (cuuint64_t)bh};
     cuuint64_t strides[2] = {(cuuint64_t)d * 2, (cuuint64_t)d * 2 * (cuuint64_t)rows};
-    cuuint32_t box[3] = {64, 128, 1};
+    cuuint32_t box[3] = {64, (cuuint32_t)box_rows, 1};
     cuuint32_t es[3] = {1, 1, 1};
     CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box, es,
                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -560,6 +561,9 @@ bool prefill_persistent_case(const focus_cache& c, const focus_prefill_args& a) 
 
 int32_t prefill_kernel_choice(const focus_cache& c, const focus_prefill_args& a) {
     if (a.flags & FOCUS_PREFILL_LEGACY_MMA) return FOCUS_PREFILL_KERNEL_LEGACY;
+    int32_t RB, tiles;
+    if ((a.flags & FOCUS_PREFILL_KMER_LOCAL) && !(c.rope_theta > 0.f) && prefill::kmer_tiling(c, a, &RB, &tiles))
+        return FOCUS_PREFILL_KERNEL_KMER;
     if (prefill_persistent_case(c, a)) {
         const size_t need = prefill::persistent_workspace_bytes(c, a);
         if (need == 0 || (a.workspace && a.workspace_bytes >= need)) return FOCUS_PREFILL_KERNEL_PERSISTENT;
@@ -574,8 +578,9 @@ size_t prefill_workspace_bytes(const focus_cache& c, const focus_prefill_args& a
 cudaError_t launch_prefill_tc(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
                               cudaStream_t stream) {
     const bool local = (a.flags & FOCUS_PREFILL_KMER_LOCAL) != 0, rope = c.rope_theta > 0.f;
-    if (prefill_kernel_choice(c, a) == FOCUS_PREFILL_KERNEL_PERSISTENT)
-        return prefill::launch_prefill_tc_persistent(c, a, status, stream);
+    const int32_t kernel = prefill_kernel_choice(c, a);
+    if (kernel == FOCUS_PREFILL_KERNEL_PERSISTENT) return prefill::launch_prefill_tc_persistent(c, a, status, stream);
+    if (kernel == FOCUS_PREFILL_KERNEL_KMER) return prefill::launch_prefill_tc_kmer(c, a, status, stream);
     if (c.q_per_kv > 1) return dispatch<true>(c, a, status, stream, local, rope);
     return dispatch<false>(c, a, status, stream, local, rope);
 }

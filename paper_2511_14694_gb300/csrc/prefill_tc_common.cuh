@@ -244,13 +244,21 @@ __device__ __forceinline__ void rope_offsets(const double* theta, int i0, int g,
     step = rot8_make(st);
 }
 
-// 3-D map over a [BH][rows][d] bf16 tensor, box = 128 rows x 64 columns, 128-byte swizzle.
-cudaError_t make_map(CUtensorMap* m, const void* ptr, int d, int64_t rows, int64_t bh);
+// 3-D map over a [BH][rows][d] bf16 tensor, box = box_rows rows x 64 columns
+// (a multiple of 8, <= 128; a tile's 128 rows by default), 128-byte swizzle.
+cudaError_t make_map(CUtensorMap* m, const void* ptr, int d, int64_t rows, int64_t bh, int box_rows = 128);
 
 // The persistent kernel (appendix mask). With the rotary embedding it needs the
 // caller's workspace (persistent_workspace_bytes) for the rotated Q and K rows.
 cudaError_t launch_prefill_tc_persistent(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
                                          cudaStream_t stream);
+// The k-mer-local kernel with query tiles cut at k-mer boundaries
+// (prefill_tc_kmer.cu): whether the span qualifies (needs args.h_k_per_window),
+// and then its ring rows per tile (RB) and tiles per window.
+bool kmer_tiling(const focus_cache& c, const focus_prefill_args& a, int32_t* RB, int32_t* max_tiles);
+cudaError_t launch_prefill_tc_kmer(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
+                                   cudaStream_t stream);
+
 // Workspace bytes of the persistent kernel: 0 without the rotary embedding; with
 // it a 256-byte block of per-head counters, then Q and K of the span, rotated.
 size_t persistent_workspace_bytes(const focus_cache& c, const focus_prefill_args& a);

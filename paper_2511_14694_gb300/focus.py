@@ -50,7 +50,8 @@ class CacheDesc(ctypes.Structure):
 class PrefillArgs(ctypes.Structure):
     _fields_ = [("q", _P), ("k", _P), ("v", _P), ("o", _P), ("lse", _P), ("T_span", _i64), ("d_win_off", _P),
                 ("d_ring_off", _P), ("n_windows", _i32), ("w_begin", _i32), ("w_end", _i32), ("max_rows", _i32),
-                ("scale", _f32), ("flags", _u32), ("workspace", _P), ("workspace_bytes", ctypes.c_size_t)]
+                ("scale", _f32), ("flags", _u32), ("workspace", _P), ("workspace_bytes", ctypes.c_size_t),
+                ("h_k_per_window", _P)]
 
 
 class PrefillHostArgs(ctypes.Structure):
@@ -341,11 +342,13 @@ def _check_heads(cache: Cache, q, k, v):
                          f"(want {cache.H})")
 
 
-def _prefill_args(q, k, v, o, lse, L: dict, w_begin: int, w_end: int, scale: float, flags: int, workspace=None):
+def _prefill_args(q, k, v, o, lse, L: dict, w_begin: int, w_end: int, scale: float, flags: int, workspace=None,
+                  host_schedule: bool = True):
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    # the host copy of the cadence schedule lets the k-mer-local mode pick its k-mer-tiled kernel
     return PrefillArgs(_ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse), q.shape[2], _ptr(L["win_off"]),
                        _ptr(L["ring_off"]), L["M"], w_begin, w_end, int(L["max_rows"]), scale, flags,
-                       _ptr(workspace), ws_bytes)
+                       _ptr(workspace), ws_bytes, _ptr(L["k_host"]) if host_schedule else None)
 
 
 def prefill_workspace_bytes(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | None = None,
@@ -365,11 +368,13 @@ def new_prefill_workspace(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_en
 
 
 def attn_prefill(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | None = None, scale=None,
-                 o=None, lse=None, flags: int = 0, stream=None, workspace="auto"):
+                 o=None, lse=None, flags: int = 0, stream=None, workspace="auto", host_schedule: bool = True):
     """focus_attn_prefill over windows [w_begin, w_end). q/k/v: bf16 [B, H, T_span, d]
     holding the augmented rows of those windows. Returns (o, lse).
     ``workspace``: a device buffer for the library (see prefill_workspace_bytes),
-    None for none, or "auto" to allocate one when the arguments can use it."""
+    None for none, or "auto" to allocate one when the arguments can use it.
+    ``host_schedule``: pass the layout's host copy of the k schedule
+    (h_k_per_window), which the k-mer-local mode's k-mer-tiled kernel needs."""
     lib = load()
     w_end = L["M"] if w_end is None else w_end
     for name, t in (("q", q), ("k", k), ("v", v)):
@@ -385,7 +390,7 @@ def attn_prefill(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | 
         workspace = new_prefill_workspace(cache, q, k, v, L, w_begin, w_end, flags)
     elif workspace is not None:
         _cuda(workspace, "workspace")
-    a = _prefill_args(q, k, v, o, lse, L, w_begin, w_end, scale, flags, workspace)
+    a = _prefill_args(q, k, v, o, lse, L, w_begin, w_end, scale, flags, workspace, host_schedule)
     _check("focus_attn_prefill", lib.focus_attn_prefill(ctypes.byref(cache.desc), ctypes.byref(a), _stream(stream)))
     return o, lse
 
@@ -428,17 +433,19 @@ def prefill_host(cache: Cache, L: dict, host: dict, dev: dict, copy_in, copy_out
     return host["o"], lse_h
 
 
-PREFILL_KERNELS = {0: "legacy mma.sync", 1: "tcgen05, one CTA per work item", 2: "tcgen05 persistent"}
+PREFILL_KERNELS = {0: "legacy mma.sync", 1: "tcgen05, one CTA per work item", 2: "tcgen05 persistent",
+                   3: "tcgen05 k-mer tiles"}
 
 
 def prefill_kernel(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | None = None, flags: int = 0,
-                   o=None, workspace="auto") -> str:
+                   o=None, workspace="auto", host_schedule: bool = True) -> str:
     """Name of the kernel focus_attn_prefill would launch for these arguments
     (focus_prefill_kernel: host only, nothing runs on the device). ``workspace``
     as for attn_prefill; "auto" assumes the workspace attn_prefill would allocate."""
     lib = load()
     w_end = L["M"] if w_end is None else w_end
-    a = _prefill_args(q, k, v, q if o is None else o, None, L, w_begin, w_end, 1.0 / math.sqrt(q.shape[3]), flags)
+    a = _prefill_args(q, k, v, q if o is None else o, None, L, w_begin, w_end, 1.0 / math.sqrt(q.shape[3]), flags,
+                      host_schedule=host_schedule)
     if isinstance(workspace, str):
         a.workspace_bytes = prefill_workspace_bytes(cache, q, k, v, L, w_begin, w_end, flags)
         a.workspace = 16 if a.workspace_bytes else None        # a placeholder address: nothing is launched

@@ -34,7 +34,7 @@ def test_struct_sizes_match_c_layout():
     # 2 x int64 + 8 pointers; 8 pointers + 7 int32 (+pad); see focus.h
     assert ctypes.sizeof(focus.LayoutOut) == 16 + 10 * 8
     assert ctypes.sizeof(focus.CacheDesc) == 8 * 8 + 8 * 4 + 8 + 8 + 8 + 8
-    assert ctypes.sizeof(focus.PrefillArgs) == 5 * 8 + 8 + 2 * 8 + 6 * 4 + 2 * 8
+    assert ctypes.sizeof(focus.PrefillArgs) == 5 * 8 + 8 + 2 * 8 + 6 * 4 + 2 * 8 + 8
     assert ctypes.sizeof(focus.CompactArgs) == 2 * 8 + 2 * 8 + 2 * 8 + 3 * 4 + 4
     # 12 buffer pointers, n_nt, W (+pad), d_W_sched, n_windows (+pad), d_k_sched, flags, tail, layout,
     # max_rows, scale, prefill_flags (+pad), workspace, its size, groups (+pad), two streams
@@ -158,7 +158,17 @@ def test_prefill_kernel_choice_needs_no_gpu():
     assert choice(1, 128_000) == (0, 1)              # one long window
     assert choice(1_280, 1_010, focus.PREFILL_LEGACY_MMA) == (0, 0)
     c.k_per_window, c.n_windows = 4096, 128
+    assert choice(1_280, 1_010, focus.PREFILL_KMER_LOCAL) == (0, 1)       # no host schedule
+    ks = np.full(128, 100, np.int32)
+    a.h_k_per_window = ks.ctypes.data
+    assert choice(1_280, 1_010, focus.PREFILL_KMER_LOCAL) == (0, 3)       # k-mers of 101 rows, <= 12 ring rows
+    ks[5] = 10                                                            # ~100 ring rows in a tile: too many
     assert choice(1_280, 1_010, focus.PREFILL_KMER_LOCAL) == (0, 1)
+    ks[5] = 150                                                           # a k-mer of 151 rows: too long
+    assert choice(1_280, 1_010, focus.PREFILL_KMER_LOCAL) == (0, 1)
+    ks[5] = 50                                                            # 21 ring rows: RB = 24, 104-row k-mer room
+    assert choice(1_280, 1_010, focus.PREFILL_KMER_LOCAL) == (0, 3)
+    a.h_k_per_window = None
     c.rope_theta = 10_000.0
     assert choice(1_280, 1_010) == (0, 1)            # rotary embedding without a workspace
     # with the workspace focus_prefill_workspace_size asks for: the persistent kernel,

@@ -181,13 +181,24 @@ def _local_ref(N, W, k, q, kk, v, heads, rows):
                                    heads, rows)
 
 
+# the cases whose k-mers and visible ring rows fit one 128-row K/V tile run the
+# k-mer-tiled kernel when the host schedule is passed; without it (and for the
+# other cases) the one-CTA-per-item kernel runs
+LOCAL_TILED = {(4_000, 1_000), (5_000, 1_024), (20_000, 200), (300, 64)}
+
+
+@pytest.mark.parametrize("host_schedule", [True, False])
 @pytest.mark.parametrize("N,W,ks,B,H,d,std", LOCAL_PREFILL_CASES)
-def test_prefill_kmer_local_matches_oracle(N, W, ks, B, H, d, std):
+def test_prefill_kmer_local_matches_oracle(N, W, ks, B, H, d, std, host_schedule):
     L, k, q, kk, v, cache = _local_case(N, W, ks, B, H, d, std, seed=N + 7)
+    fl = focus.PREFILL_KMER_LOCAL
+    want = "tcgen05 k-mer tiles" if host_schedule and (N, W) in LOCAL_TILED else "tcgen05, one CTA per work item"
+    assert focus.prefill_kernel(cache, q, kk, v, L, flags=fl, host_schedule=host_schedule) == want
     n = q.numel()
     canary = torch.full((n + 4096,), 7.0, dtype=torch.bfloat16, device="cuda")
     o = canary[:n].view(q.shape)
-    o, lse = pipeline.prefill_masked_parallel(cache, q, kk, v, L, o=o, flags=focus.PREFILL_KMER_LOCAL)
+    focus.kv_compact_bulk(cache, kk, v, L)
+    o, lse = focus.attn_prefill(cache, q, kk, v, L, o=o, flags=fl, host_schedule=host_schedule)
     torch.cuda.synchronize()
     assert bool((canary[n:] == 7.0).all()), "prefill wrote past its output"
     T = L["T"]
