@@ -556,7 +556,11 @@ constexpr int64_t kPersistentMaxRows = 4096;
 // tiles each CTA loads.
 bool prefill_persistent_case(const focus_cache& c, const focus_prefill_args& a) {
     const bool local = (a.flags & FOCUS_PREFILL_KMER_LOCAL) != 0;
-    return !(a.flags & FOCUS_PREFILL_LEGACY_MMA) && !local && (int64_t)c.C_ring + a.max_rows <= kPersistentMaxRows;
+    // the persistent kernel numbers its work items with 32-bit arithmetic
+    const int64_t g = c.q_per_kv > 1 ? c.q_per_kv : 1;
+    const int64_t items = (int64_t)(a.w_end - a.w_begin) * ((a.max_rows + 2 * BM - 1) / (2 * BM)) * g * c.H * c.B;
+    return !(a.flags & FOCUS_PREFILL_LEGACY_MMA) && !local && (int64_t)c.C_ring + a.max_rows <= kPersistentMaxRows &&
+           items <= INT32_MAX;
 }
 
 int32_t prefill_kernel_choice(const focus_cache& c, const focus_prefill_args& a) {

@@ -59,23 +59,25 @@ struct ItemGeom {
     bool valid, cap_err;
 };
 
+// idx < n_items < 2^31 (the host's condition for this kernel), so the index
+// arithmetic is 32-bit: every role forms an item's geometry at every item.
+// w0 = win_off[w_begin]; span_ok: the span's rows fit T_span (per launch).
 template <bool GQA>
-__device__ __forceinline__ ItemGeom item_geom(int64_t idx, int32_t per_head, int32_t ctas_pw, int32_t q_per_kv,
-                                              int32_t H, const int32_t* __restrict__ win_off,
-                                              const int32_t* __restrict__ ring_off, int32_t w_begin,
-                                              int32_t w_end, int32_t C_ring, int64_t T_span) {
+__device__ __forceinline__ ItemGeom item_geom(int64_t idx, uint32_t per_head, uint32_t ctas_pw, uint32_t q_per_kv,
+                                              uint32_t H, const int32_t* __restrict__ win_off,
+                                              const int32_t* __restrict__ ring_off, int32_t w0, bool span_ok,
+                                              int32_t w_end, int32_t C_ring) {
     ItemGeom I;
     // per_head: items of one K/V head = windows x pairs (x query heads per group)
-    const uint32_t x = (uint32_t)(idx % per_head);
-    const int64_t rest = idx / per_head;
-    const int32_t h = (int32_t)(rest % H), b = (int32_t)(rest / H);
-    const uint32_t item = GQA ? x / (uint32_t)q_per_kv : x;
-    I.member = GQA ? (int32_t)(x % (uint32_t)q_per_kv) : 0;
-    const int32_t wi = item / ctas_pw;
-    I.cta = ctas_pw - 1 - (int32_t)(item % ctas_pw);
-    I.w = w_end - 1 - wi;
-    I.bh = b * H + h;
-    const int32_t w0 = win_off[w_begin];
+    const uint32_t u = (uint32_t)idx;
+    const uint32_t rest = u / per_head, x = u - rest * per_head;
+    const uint32_t b = rest / H, h = rest - b * H;
+    const uint32_t item = GQA ? x / q_per_kv : x;
+    I.member = GQA ? (int32_t)(x - item * q_per_kv) : 0;
+    const uint32_t wi = item / ctas_pw;
+    I.cta = (int32_t)(ctas_pw - 1 - (item - wi * ctas_pw));
+    I.w = w_end - 1 - (int32_t)wi;
+    I.bh = (int32_t)(b * H + h);
     const int32_t w_first = win_off[I.w];
     I.Tw = win_off[I.w + 1] - w_first;
     I.a0 = I.cta * 2 * BM;
@@ -83,7 +85,7 @@ __device__ __forceinline__ ItemGeom item_geom(int64_t idx, int32_t per_head, int
     I.cap_err = false;
     I.Rw = ring_off[I.w];
     I.n_ring = (I.Rw + BN - 1) / BN;
-    if (I.valid && (I.Rw > C_ring || (int64_t)(win_off[w_end] - w0) > T_span)) {
+    if (I.valid && (I.Rw > C_ring || !span_ok)) {
         I.cap_err = true;
         I.valid = false;
     }
@@ -256,8 +258,11 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
     // that a systematic stall costs one round of bounded waits.
     if (*(volatile int32_t*)status == FOCUS_ERR_TIMEOUT) return;
     const int32_t per_head = (w_end - w_begin) * ctas_pw * (GQA ? q_per_kv : 1);
+    const int32_t w0 = win_off[w_begin];
+    const bool span_ok = (int64_t)(win_off[w_end] - w0) <= T_span;
     auto geom = [&](int64_t idx) {
-        return item_geom<GQA>(idx, per_head, ctas_pw, q_per_kv, H, win_off, ring_off, w_begin, w_end, C_ring, T_span);
+        return item_geom<GQA>(idx, (uint32_t)per_head, (uint32_t)ctas_pw, (uint32_t)q_per_kv, (uint32_t)H, win_off,
+                              ring_off, w0, span_ok, w_end, C_ring);
     };
     // round k of a CTA: positions k G .. k G + G - 1 of the longest-first order, in
     // snake order (forward on even rounds, backward on odd) to balance the CTAs
