@@ -632,32 +632,54 @@ def prefill_roofline(pre, peaks, peaks_src, traffic=None):
     return r
 
 
-# the other named workloads timed beside the headline: (key, workload, steps, warm-up)
-CONFIG_LEGS = [("ksweep", "prefill_256kb_ksweep_h32_d128", 10, 3),
-               ("causal", "causal_128kb_h32_d128", 3, 3),
-               ("stream", "stream_1mb_b4_h32_d128", 2, 3)]
+# the other named workloads and options timed beside the headline:
+# (key, workload, steps, warm-up, options: mask, rotary base)
+CONFIG_LEGS = [("ksweep", "prefill_256kb_ksweep_h32_d128", 10, 3, {}),
+               ("causal", "causal_128kb_h32_d128", 3, 3, {}),
+               ("stream", "stream_1mb_b4_h32_d128", 2, 3, {}),
+               ("kmer_local", "prefill_128kb_h32_d128", 20, 3, {"mask": "kmer_local"}),
+               ("rope", "prefill_128kb_h32_d128", 20, 3, {"rope": 500000.0}),
+               ("stream_kmer_local", "stream_1mb_b4_h32_d128", 2, 3, {"mask": "kmer_local"})]
 
 
-def run_config_leg(args, name, steps, warmup, world, rank, local, peaks, peaks_src):
-    """One of the other named workloads at the default options (appendix mask,
-    no rotary embedding, one query head per K/V head), timed like the headline
-    step; returns its object for the bench line."""
+def run_config_leg(args, name, steps, warmup, world, rank, local, peaks, peaks_src, opts=None):
+    """One of the other named workloads, at the default options (appendix mask,
+    no rotary embedding, one query head per K/V head) unless ``opts`` sets the
+    mask or the rotary base, timed like the headline step; returns its object for
+    the bench line."""
     import copy
     from paper_2511_14694_gb300.workloads import WORKLOADS
     cfg = WORKLOADS[name]
+    opts = opts or {}
     a = copy.copy(args)
     a.steps, a.warmup, a.no_e2e, a.no_cpu_baseline = steps, warmup, True, True
-    a.rope, a.q_per_kv, a.mask, a.prefill_flags = 0.0, 1, "appendix", 0
+    a.rope, a.q_per_kv, a.mask = float(opts.get("rope", 0.0)), 1, opts.get("mask", "appendix")
+    a.prefill_flags = 2 if a.mask == "kmer_local" else 0
     pre = (run_stream_leg if cfg["mode"] == "stream" else run_prefill_leg)(a, cfg, world, rank, local)
     obj = {"workload": name, "value": weak_scaling_value(cfg["B"] * cfg["N"], world, pre["step_ms"] / 1e3),
            "unit": "nt/s", "ms_per_step": pre["step_ms"], "steps": steps, "warmup": warmup,
            "augmented_tokens_per_s": world * cfg["B"] * pre["T"] / (pre["step_ms"] / 1e3),
            "step": pre["step_desc"], "config": workload_config(a, cfg, pre["T"], pre["R"], name=name),
-           "roofline": prefill_roofline(pre, peaks, peaks_src), "clocks": pre["clocks"],
+           "roofline": prefill_roofline(pre, peaks, peaks_src, leg_traffic(pre, a, cfg)), "clocks": pre["clocks"],
            "gpu_launches": pre["launches"]}
     if pre.get("window_compaction") is not None:
         obj["window_compaction"] = pre["window_compaction"]
     return obj
+
+
+def leg_traffic(pre, args, cfg):
+    """DRAM bytes per launch from the committed ncu counters, which exist for the
+    128 kb workload (default heads) on the appendix-mask persistent kernel, its
+    rotary variant and the k-mer-tiled kernel; None elsewhere or once the
+    kernel's source has changed since the capture."""
+    from paper_2511_14694_gb300.workloads import WORKLOADS
+    key = {("tcgen05 persistent", False, False): ("prefill_attention", "prefill_tc_persistent.cu"),
+           ("tcgen05 persistent", False, True): ("prefill_attention_rope", "prefill_tc_persistent.cu"),
+           ("tcgen05 k-mer tiles", True, False): ("prefill_attention_kmer_local", "prefill_tc_kmer.cu"),
+           }.get((pre["kernel"], pre.get("local_mask", False), bool(args.rope)))
+    if not key or args.q_per_kv != 1 or cfg is not WORKLOADS["prefill_128kb_h32_d128"]:
+        return None
+    return kernel_traffic(key[0], "paper_2511_14694_gb300/csrc/" + key[1])
 
 
 def run_compact_leg(args, world, rank, local, peaks, peaks_src):
@@ -724,23 +746,15 @@ def run_focus(args, world, rank, local):
     emb = None if args.embed_d <= 0 else run_embed_leg(args, world, rank, local)
     legs = {}
     if not args.no_configs:
-        for key, name, steps, warmup in CONFIG_LEGS:
-            if name != args.workload:
-                legs[key] = run_config_leg(args, name, steps, warmup, world, rank, local, peaks, peaks_src)
+        for key, name, steps, warmup, opts in CONFIG_LEGS:
+            if name != args.workload or opts.get("mask", "appendix") != args.mask or \
+                    float(opts.get("rope", 0.0)) != float(args.rope):
+                legs[key] = run_config_leg(args, name, steps, warmup, world, rank, local, peaks, peaks_src, opts)
     big_compact = None if args.no_configs else run_compact_leg(args, world, rank, local, peaks, peaks_src)
     if rank != 0:
         return
     value = weak_scaling_value(cfg["B"] * cfg["N"], world, pre["step_ms"] / 1e3)
-    local_mask = pre.get("local_mask", False)
-    # committed DRAM counters exist for the 128 kb workload's appendix-mask kernel
-    # (persistent) and k-mer-local kernel, default heads
-    traffic_key = {("tcgen05 persistent", False, False): ("prefill_attention", "prefill_tc_persistent.cu"),
-                   ("tcgen05 persistent", False, True): ("prefill_attention_rope", "prefill_tc_persistent.cu"),
-                   ("tcgen05, one CTA per work item", True, False): ("prefill_attention_kmer_local", "prefill_tc.cu")
-                   }.get((pre["kernel"], local_mask, bool(args.rope)))
-    traffic = None
-    if traffic_key and args.q_per_kv == 1 and cfg is WORKLOADS["prefill_128kb_h32_d128"]:
-        traffic = kernel_traffic(traffic_key[0], "paper_2511_14694_gb300/csrc/" + traffic_key[1])
+    traffic = leg_traffic(pre, args, cfg)
     line = {
         "metric": METRIC,
         "value": value, "unit": "nt/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
@@ -792,7 +806,7 @@ def run_focus(args, world, rank, local):
         line["cpu_baseline"] = None      # the oracle baseline times the default path only
     elif pre["host_sample"] is not None:
         hs = pre["host_sample"]
-        if local_mask:
+        if pre.get("local_mask", False):
             from oracle import focus_oracle as fo
             hs["kmer"] = fo.layout_kmer(cfg["N"], cfg["W"], hs["k_sched"])
         secs = oracle_head_times(cfg, hs, hs["k_sched"], hs["q"], hs["k"], hs["v"], args.cpu_heads,

@@ -283,7 +283,8 @@ focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_ar
  *                                    rotary embedding is on, and over the span's windows every k-mer
  *                                    has at most 128 - RB rows, where RB (a multiple of 8, <= 64)
  *                                    bounds the ring rows a tile sees: the boundary plus one FOCUS
- *                                    row per k bases, 1 + ceil(max_rows / k_w).
+ *                                    row per k bases, 1 + ceil(max_rows / k_w); and the launch has at
+ *                                    least 2,048 work items (tiles x query heads x sequences).
  * The persistent kernel also takes the rotary-embedding case when args carries
  * focus_prefill_workspace_size(cache, args) bytes of workspace.
  * Both tcgen05 kernels compute the same rows (within rounding order). */

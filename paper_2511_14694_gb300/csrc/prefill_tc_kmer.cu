@@ -38,6 +38,7 @@ namespace {
 
 constexpr int kRegsIssue = 72, kRegsSoftmax = 216;
 constexpr int64_t kKmerMaxRingRows = 64;   // ring rows a tile may hold (the window box keeps >= 64 rows)
+constexpr int64_t kKmerMinItems = 2048;    // work items a launch needs for this kernel (~13 per SM)
 static_assert(128 * kRegsIssue + 256 * kRegsSoftmax <= kThreads * kLaunchRegs, "register split over budget");
 
 struct KBars {
@@ -417,7 +418,7 @@ bool kmer_tiling(const focus_cache& c, const focus_prefill_args& a, int32_t* RB,
     if (!a.h_k_per_window || a.max_rows <= 0) return false;
     // ring rows a tile needs: the carried boundary + the FOCUS rows of its earlier
     // k-mers, at most one per k bases of the window (+1 for an open last k-mer)
-    int64_t ring = 1, kdiv_max = 1, kdiv_min = 1 << 30;
+    int64_t ring = 1, kdiv_max = 1;
     for (int32_t w = a.w_begin; w < a.w_end; ++w) {
         const int64_t k = a.h_k_per_window[w];
         if (k < 0) return false;
@@ -425,15 +426,27 @@ bool kmer_tiling(const focus_cache& c, const focus_prefill_args& a, int32_t* RB,
         const int64_t r = k > 0 ? (a.max_rows + k - 1) / k + 1 : 1;
         if (r > ring) ring = r;
         if (kdiv > kdiv_max) kdiv_max = kdiv;
-        if (kdiv < kdiv_min) kdiv_min = kdiv;
     }
     const int64_t rb = (ring + 7) / 8 * 8;
     if (rb > kKmerMaxRingRows || kdiv_max > 128 - rb) return false;
+    // tiles per window: a tile holds (128 - RB) / kdiv whole k-mers, which is not
+    // monotonic in the k-mer length, so take the most over the windows (a device
+    // k-mer is never longer than the host's bound here, so its tiles are no more)
+    int64_t tiles = 1;
+    for (int32_t w = a.w_begin; w < a.w_end; ++w) {
+        const int64_t k = a.h_k_per_window[w];
+        const int64_t kdiv = (k > 0 && k < a.max_rows ? k : a.max_rows) + 1;
+        const int64_t nq = ((128 - rb) / kdiv) * kdiv;
+        const int64_t t = (a.max_rows + nq - 1) / nq;
+        if (t > tiles) tiles = t;
+    }
+    // a launch with few items (one window of a stream) does not fill the per-SM
+    // pipelines of this persistent kernel: one 1 kb window at batch 4 (1,280
+    // items) ran 50.8 us per launch against 47.3 for the one-CTA-per-item kernel
+    const int64_t g = c.q_per_kv > 1 ? c.q_per_kv : 1;
+    if ((int64_t)(a.w_end - a.w_begin) * tiles * g * c.H * c.B < kKmerMinItems) return false;
     *RB = (int32_t)rb;
-    // tiles per window: the shortest k-mers give the most
-    const int64_t nq_min = ((128 - rb) / kdiv_min) * kdiv_min;
-    *max_tiles = (int32_t)((a.max_rows + nq_min - 1) / nq_min);
-    (void)c;
+    *max_tiles = (int32_t)tiles;
     return true;
 }
 

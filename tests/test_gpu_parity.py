@@ -181,18 +181,26 @@ def _local_ref(N, W, k, q, kk, v, heads, rows):
                                    heads, rows)
 
 
-# the cases whose k-mers and visible ring rows fit one 128-row K/V tile run the
-# k-mer-tiled kernel when the host schedule is passed; without it (and for the
-# other cases) the one-CTA-per-item kernel runs
-LOCAL_TILED = {(4_000, 1_000), (5_000, 1_024), (20_000, 200), (300, 64)}
+# cases whose k-mers and visible ring rows fit one 128-row K/V tile, with at
+# least 2,048 work items: the k-mer-tiled kernel runs when the host schedule is
+# passed, the one-CTA-per-item kernel without it (and for the cases above)
+LOCAL_TILED_CASES = [
+    (16_000, 1_000, [100], 1, 32, 64, 1.0),                   # 10 one-k-mer tiles per window, RB = 16
+    (5_000, 1_024, [100], 2, 32, 128, 1.0),                   # partial k-mer closes every window
+    (20_000, 200, [10], 1, 16, 128, 1.0 / math.sqrt(128)),    # 9 k-mers per tile, RB = 24, ragged tiles
+    (9_000, 1_000, [100, 50, 60], 1, 32, 128, 1.0),           # k per window: tiles of 1 or 2 k-mers, RB = 24;
+                                                              # k = 60 gives the most tiles (17 of 61 rows)
+]
+LOCAL_TILED = {(N, W, B, H) for N, W, ks, B, H, *_ in LOCAL_TILED_CASES}
 
 
 @pytest.mark.parametrize("host_schedule", [True, False])
-@pytest.mark.parametrize("N,W,ks,B,H,d,std", LOCAL_PREFILL_CASES)
+@pytest.mark.parametrize("N,W,ks,B,H,d,std", LOCAL_PREFILL_CASES + LOCAL_TILED_CASES)
 def test_prefill_kmer_local_matches_oracle(N, W, ks, B, H, d, std, host_schedule):
     L, k, q, kk, v, cache = _local_case(N, W, ks, B, H, d, std, seed=N + 7)
     fl = focus.PREFILL_KMER_LOCAL
-    want = "tcgen05 k-mer tiles" if host_schedule and (N, W) in LOCAL_TILED else "tcgen05, one CTA per work item"
+    tiled = host_schedule and (N, W, B, H) in LOCAL_TILED
+    want = "tcgen05 k-mer tiles" if tiled else "tcgen05, one CTA per work item"
     assert focus.prefill_kernel(cache, q, kk, v, L, flags=fl, host_schedule=host_schedule) == want
     n = q.numel()
     canary = torch.full((n + 4096,), 7.0, dtype=torch.bfloat16, device="cuda")
