@@ -402,13 +402,18 @@ def run_prefill_leg(args, cfg, world, rank, local):
 
 def run_stream_leg(args, cfg, world, rank, local):
     """Streaming prefill (App. A.2): for each window in order, focus_kv_compact of
-    that window, then focus_attn_prefill over it against the ring, consecutive
-    windows' attention overlapping on two streams (pipeline.prefill_streaming).
-    Each window's Q/K/V is one of a pool of seeded windows (cycled)."""
+    that window; the attention per chunk of args.stream_chunk windows (one
+    focus_attn_prefill over the chunk against the ring), consecutive chunks'
+    attention overlapping on two streams (pipeline.prefill_streaming). The Q/K/V
+    come from a seeded pool of windows (cycled), held as pool / chunk contiguous
+    chunk tensors."""
     import torch
     from paper_2511_14694_gb300 import focus, inputs, pipeline
 
     B, N, W, H, d, P = cfg["B"], cfg["N"], cfg["W"], cfg["H"], cfg["d"], cfg["pool"]
+    C = args.stream_chunk
+    if C < 1 or P % C:
+        raise ValueError(f"--stream-chunk must divide the pool of {P} windows")
     M = focus.n_windows(N, W)
     k_s = inputs.k_schedule(M, cfg["k"], seed=inputs.DEFAULT_SEED)
     dev = torch.device("cuda", local)
@@ -418,29 +423,35 @@ def run_stream_leg(args, cfg, world, rank, local):
     if not (np.diff(off) == Tw).all():
         raise ValueError("the streaming leg expects windows of equal augmented size")
     g = args.q_per_kv
-    if g == 1:
-        pq, pk, pv = inputs.qkv((P, B, H, Tw, d), std=cfg["std"], seed=inputs.DEFAULT_SEED + rank, device=dev)
-    else:                            # grouped-query heads: K/V with H / g heads
-        pq = inputs.normal_bf16((P, B, H, Tw, d), cfg["std"], seed=3 * (inputs.DEFAULT_SEED + rank) + 1, device=dev)
-        pk, pv = (inputs.normal_bf16((P, B, H // g, Tw, d), cfg["std"], seed=3 * (inputs.DEFAULT_SEED + rank) + i,
-                                     device=dev) for i in (2, 3))
+    n_slots = P // C                  # chunk tensors in the pool, each [B, H(, /g), C Tw, d]
+    seed = inputs.DEFAULT_SEED + rank
+    pq = [inputs.normal_bf16((B, H, C * Tw, d), cfg["std"], seed=3 * seed + 1 + 10 * j, device=dev)
+          for j in range(n_slots)]
+    pk = [inputs.normal_bf16((B, H // g, C * Tw, d), cfg["std"], seed=3 * seed + 2 + 10 * j, device=dev)
+          for j in range(n_slots)]
+    pv = [inputs.normal_bf16((B, H // g, C * Tw, d), cfg["std"], seed=3 * seed + 3 + 10 * j, device=dev)
+          for j in range(n_slots)]
     cache = focus.Cache(B, H // g, d, C_ring=max(L["R"], 1), device=dev, k_sched=k_s, rope_theta=args.rope,
                         q_per_kv=g)
     local_mask = bool(args.prefill_flags & focus.PREFILL_KMER_LOCAL)
-    outs = [torch.empty((B, H, Tw, d), dtype=torch.bfloat16, device=dev) for _ in range(2)]
-    lses = [torch.empty((B, H, Tw), dtype=torch.float32, device=dev) for _ in range(2)]
+    outs = [torch.empty((B, H, C * Tw, d), dtype=torch.bfloat16, device=dev) for _ in range(2)]
+    lses = [torch.empty((B, H, C * Tw), dtype=torch.float32, device=dev) for _ in range(2)]
     stream = torch.cuda.current_stream(dev)
-    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(M)]
-    kernel_name = focus.prefill_kernel(cache, pq[0], pk[0], pv[0], L, M - 1, M, flags=args.prefill_flags, o=outs[0])
+    n_calls = -(-M // C)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_calls)]
+    kernel_name = focus.prefill_kernel(cache, pq[0], pk[0], pv[0], L, M - C, M, flags=args.prefill_flags, o=outs[0])
+
+    def span(w0, w1=None):
+        j = (w0 // C) % n_slots
+        return pq[j], pk[j], pv[j]
 
     cevs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(M)]
 
     def step(timed=False):
-        # each window's compaction, then its attention on one of two side streams:
-        # consecutive windows' launches overlap (pipeline.prefill_streaming)
-        pipeline.prefill_streaming(cache, L, lambda w: (pq[w % P], pk[w % P], pv[w % P]), outs, lses,
-                                   flags=args.prefill_flags, stream=stream, events=evs if timed else None,
-                                   compact_events=cevs if timed else None)
+        # each window's compaction, then the attention per chunk on one of two side
+        # streams: consecutive chunks' launches overlap (pipeline.prefill_streaming)
+        pipeline.prefill_streaming(cache, L, span, outs, lses, flags=args.prefill_flags, stream=stream,
+                                   events=evs if timed else None, compact_events=cevs if timed else None, chunk=C)
 
     for _ in range(args.warmup):
         step()
@@ -466,8 +477,9 @@ def run_stream_leg(args, cfg, world, rank, local):
     n_alone = min(M, 100)
     aev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_alone)]
     for w, (a, b) in enumerate(aev):
+        _, ck, cv = span(w - w % C)
         a.record(stream)
-        focus.kv_compact_bulk(cache, pk[w % P], pv[w % P], L, w, w + 1, src_row0=int(off[w]), stream=stream)
+        focus.kv_compact_bulk(cache, ck, cv, L, w, w + 1, src_row0=int(off[w - w % C]), stream=stream)
         b.record(stream)
     torch.cuda.synchronize(dev)
     alone_ms = statistics.median(a.elapsed_time(b) for a, b in aev)
@@ -478,9 +490,11 @@ def run_stream_leg(args, cfg, world, rank, local):
     # per-window compaction: the window's kept rows of every (sequence, K/V head), read and written
     wc_ms = compact_ms / args.steps / M
     wc_bytes = float((L["R"] / M) * B * (H // g) * 2 * (2 * d) * 2)
-    return dict(kernel=kernel_name, attn_launches_per_step=M,
-                step_desc=("per window: focus_kv_compact(window) + focus_attn_prefill(window), consecutive "
-                           "windows' attention overlapping on two streams; all windows; rate over the whole step"),
+    return dict(kernel=kernel_name, attn_launches_per_step=n_calls,
+                step_desc=("per window: focus_kv_compact(window); per chunk of %d windows: focus_attn_prefill(chunk) "
+                           "(the masked-parallel form over the chunk), consecutive chunks' attention overlapping on "
+                           "two streams; all windows; rate over the whole step" % C),
+                stream_chunk=C,
                 window_compaction={"kernel": "focus_kv_compact (one window)", "bytes_per_launch": wc_bytes,
                                    "in_step_ms": wc_ms,
                                    "in_step_note": "CUDA events on the main stream inside the step: includes "
@@ -489,8 +503,8 @@ def run_stream_leg(args, cfg, world, rank, local):
                                    "alone_note": "median of %d launches with nothing else running: a ~1 MB "
                                                  "launch, launch-latency bound" % n_alone},
                 step_ms=step_ms, attn_ms=step_ms, flops_per_step=4.0 * d * H * B * pairs, pairs=pairs,
-                T=L["T"], R=L["R"], clocks=clk.summary(), launches=2 * M * args.steps, e2e=None, host_sample=None,
-                per_launch_ms=attn_ms / args.steps / M, local_mask=local_mask,
+                T=L["T"], R=L["R"], clocks=clk.summary(), launches=(M + n_calls) * args.steps, e2e=None, host_sample=None,
+                per_launch_ms=attn_ms / args.steps / n_calls, local_mask=local_mask,
                 bytes_per_step=float(B * L["T"] * (H * (4 * d + 4) + (H // g) * 4 * d)))
 
 
@@ -964,6 +978,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-heads", type=int, default=8,
                     help="whole (sequence, head) oracle passes timed for the cpu_baseline (8 of 32 = 25%%)")
+    ap.add_argument("--stream-chunk", type=int, default=8,
+                    help="windows per attention call in the streaming legs (divides the pool of 8; 1 = per window)")
     ap.add_argument("--no-configs", action="store_true",
                     help="skip the other named workloads and the 1 Mb ring compaction (profiling runs)")
     ap.add_argument("--no-clock-wait", action="store_true",

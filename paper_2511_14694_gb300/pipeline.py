@@ -9,7 +9,8 @@ sequences of C-ABI calls. No arithmetic happens here; each step is a kernel.
   heads (or sequences), with the host-device copies of one group on side
   streams overlapping the kernels of the others;
 - streaming with overlapping windows: each window's compaction first, then its
-  attention on one of two side streams, so consecutive windows' launches overlap.
+  attention on one of two side streams, so consecutive windows' launches overlap;
+  optionally several windows per attention call.
 
 Under the k-mer-local mask (``focus.PREFILL_KMER_LOCAL``, Sec. 3.2) a row also
 reads its own window's FOCUS rows from the ring, so the streaming step compacts
@@ -57,24 +58,32 @@ def prefill_masked_parallel_host(cache: focus.Cache, L: dict, host: dict, dev: d
 
 
 def prefill_streaming(cache: focus.Cache, L: dict, window_qkv, outs, lses, w_begin: int = 0, w_end: int | None = None,
-                      scale=None, flags=0, stream=None, events=None, compact_events=None):
+                      scale=None, flags=0, stream=None, events=None, compact_events=None, chunk: int = 1):
     """Streaming prefill (App. A.2) of windows [w_begin, w_end) with the
-    attention of consecutive windows overlapping. window_qkv(w) gives window w's
-    (q, k, v) ([B, H, T_w, d] each); window w writes outs[i] and lses[i],
-    i = w % len(outs) (two buffers suffice; one per window keeps every output).
+    attention of consecutive windows (or chunks of windows) overlapping.
 
-    Window w's FOCUS rows are compacted into the ring before its attention (a
-    copy of input rows: window w reads ring rows [0, ring_off[w]) only, so the
-    order changes no value), all compactions in order on ``stream``. The
-    attention of window w then needs only the compaction of window w - 1, not the
-    attention of window w - 1: it runs on side stream i % 2 after that
-    compaction, so the tail of one launch overlaps the start of the next (windows
-    that share a buffer share a stream, so a buffer is never written by two
-    launches at once).
-    ``events``: optional list of (start, end) CUDA events per window, recorded
-    around each attention launch on its stream; ``compact_events`` the same
-    around each compaction launch on ``stream``. Work is only enqueued; when
-    ``stream`` is done, so is everything."""
+    ``chunk`` = 1: window_qkv(w) gives window w's (q, k, v) ([B, H, T_w, d] each)
+    and window w writes outs[i] and lses[i], i = w % len(outs) (two buffers
+    suffice; one per window keeps every output). ``chunk`` = c > 1: the windows go
+    in chunks of c, window_qkv(w0, w1) gives the rows of windows [w0, w1)
+    ([B, H, win_off[w1] - win_off[w0], d]) and chunk n writes outs[n % len(outs)].
+
+    Each window's FOCUS rows are compacted into the ring, window by window in
+    order on ``stream``, before the attention that reads them (a copy of input
+    rows: window w reads ring rows [0, ring_off[w]) only, so the order changes no
+    value). One attention call then covers the window (or the chunk: the
+    masked-parallel form of App. A.1 over the chunk's windows, the same rows as
+    one call per window). It needs only the compactions before it, not the
+    previous attention: it runs on side stream i % 2, so the tail of one launch
+    overlaps the start of the next (launches that share a buffer share a stream,
+    so a buffer is never written by two launches at once). Larger chunks mean
+    fewer, fuller launches and c windows' inputs resident at once.
+    ``events``: optional list of (start, end) CUDA events per attention call,
+    recorded around it on its stream; ``compact_events`` the same per window
+    around each compaction on ``stream``. Work is only enqueued; when ``stream``
+    is done, so is everything."""
+    if chunk < 1:
+        raise ValueError("chunk must be >= 1")
     cur = stream if stream is not None else torch.cuda.current_stream()
     key = cur.device
     if key not in _side_streams:
@@ -84,22 +93,23 @@ def prefill_streaming(cache: focus.Cache, L: dict, window_qkv, outs, lses, w_beg
     off = L["win_off_host"]
     for s_ in side:
         s_.wait_stream(cur)                    # inputs and buffers written before the call
-    for w in range(w_begin, w_end):
-        q, k, v = window_qkv(w)
-        if compact_events is not None:
-            compact_events[w - w_begin][0].record(cur)
-        focus.kv_compact_bulk(cache, k, v, L, w, w + 1, src_row0=int(off[w]), stream=cur)
-        if compact_events is not None:
-            compact_events[w - w_begin][1].record(cur)
-        i = w % len(outs)
+    for n, w0 in enumerate(range(w_begin, w_end, chunk)):
+        w1 = min(w0 + chunk, w_end)
+        q, k, v = window_qkv(w0) if chunk == 1 else window_qkv(w0, w1)
+        for w in range(w0, w1):
+            if compact_events is not None:
+                compact_events[w - w_begin][0].record(cur)
+            focus.kv_compact_bulk(cache, k, v, L, w, w + 1, src_row0=int(off[w0]), stream=cur)
+            if compact_events is not None:
+                compact_events[w - w_begin][1].record(cur)
+        i = (w0 if chunk == 1 else n) % len(outs)
         s_ = side[i % 2]
-        s_.wait_stream(cur)                    # ring rows of windows <= w are in place
+        s_.wait_stream(cur)                    # ring rows of windows < w1 are in place
         if events is not None:
-            events[w - w_begin][0].record(s_)
-        focus.attn_prefill(cache, q, k, v, L, w, w + 1, scale=scale, o=outs[i], lse=lses[i], flags=flags,
-                           stream=s_)
+            events[n][0].record(s_)
+        focus.attn_prefill(cache, q, k, v, L, w0, w1, scale=scale, o=outs[i], lse=lses[i], flags=flags, stream=s_)
         if events is not None:
-            events[w - w_begin][1].record(s_)
+            events[n][1].record(s_)
     for s_ in side:
         cur.wait_stream(s_)
     return outs, lses

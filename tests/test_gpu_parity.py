@@ -286,8 +286,9 @@ def test_prefill_streaming_matches_sequential_oracle(d, tail):
 @pytest.mark.parametrize("d,tail,flags", [(128, 0, 0), (64, 3, 0), (128, 0, focus.PREFILL_KMER_LOCAL)])
 def test_prefill_streaming_overlapped_equals_sequential(d, tail, flags):
     """pipeline.prefill_streaming (compaction first, consecutive windows' attention
-    overlapping on two streams) gives, bit for bit, the outputs and ring of the
-    one-window-at-a-time loop (which the test above pins to the oracle)."""
+    overlapping on two streams; one window or a chunk of windows per attention
+    call) gives, bit for bit, the outputs and ring of the one-window-at-a-time loop
+    (which the test above pins to the oracle)."""
     N, W, ks, B, H = 3_000, 500, [10, 50, 100, 7], 2, 2
     M = -(-N // W)
     k_s = inputs.k_schedule(M, ks, seed=4)
@@ -308,6 +309,24 @@ def test_prefill_streaming_overlapped_equals_sequential(d, tail, flags):
         assert torch.equal(lses[w], seq[w][1]), f"window {w}"
     assert np.array_equal(bits(c_ovl.ring_k), bits(c_seq.ring_k))
     assert np.array_equal(bits(c_ovl.ring_v), bits(c_seq.ring_v))
+    # chunks of windows per attention call (each window still compacted on its own):
+    # the same items on the same kernel, so the same bits
+    for chunk in (2, 4):
+        c_chk = focus.Cache(B, H, d, C_ring=L["R"], k_sched=k_s, tail=tail)
+        spn = lambda t, w0, w1: t[:, :, int(off[w0]):int(off[w1])].contiguous()  # noqa: E731
+        spans = {w0: (spn(q, w0, min(w0 + chunk, M)), spn(k, w0, min(w0 + chunk, M)), spn(v, w0, min(w0 + chunk, M)))
+                 for w0 in range(0, M, chunk)}
+        outs = [torch.empty_like(spans[w0][0]) for w0 in range(0, M, chunk)]
+        lses = [torch.empty(x.shape[:3], dtype=torch.float32, device="cuda") for x in outs]
+        pipeline.prefill_streaming(c_chk, L, lambda w0, w1: spans[w0], outs, lses, flags=flags, chunk=chunk)
+        torch.cuda.synchronize()
+        for n, w0 in enumerate(range(0, M, chunk)):
+            for w in range(w0, min(w0 + chunk, M)):
+                a, e = int(off[w] - off[w0]), int(off[w + 1] - off[w0])
+                assert np.array_equal(bits(outs[n][:, :, a:e]), bits(seq[w][0])), f"chunk {chunk} window {w}"
+                assert torch.equal(lses[n][:, :, a:e], seq[w][1]), f"chunk {chunk} window {w}"
+        assert np.array_equal(bits(c_chk.ring_k), bits(c_seq.ring_k))
+        assert np.array_equal(bits(c_chk.ring_v), bits(c_seq.ring_v))
 
 
 # ----------------------------------------------------------------------------- decode
