@@ -102,6 +102,28 @@ def test_adaptive_prefill_streaming_and_kmer_local():
         assert_attn_close(o, lse, o_ref.reshape(B, H, T, d), lse_ref.reshape(B, H, T), f"adaptive flags={flags}")
 
 
+def test_adaptive_kmer_tiled_prefill_matches_oracle():
+    """Window lengths 700..1,200 and cadences 90..110 with the k-mer-local mask, at a
+    size that selects the k-mer-tiled kernel (its tile count is the most any window
+    needs, so the shorter windows carry empty tiles); ragged last window."""
+    N, Ws, ks = 16_037, [700, 1_200, 900, 1_000], [90, 110, 100, 95, 105]
+    W, k = _sched(N, Ws, ks)
+    B, H, d = 1, 16, 64
+    L = focus.layout(N, W, k)
+    T = L["T"]
+    q, kk, v = inputs.qkv((B, H, T, d), seed=17, device="cuda")
+    cache = focus.Cache(B, H, d, C_ring=L["R"], k_sched=k)
+    fl = focus.PREFILL_KMER_LOCAL
+    assert focus.prefill_kernel(cache, q, kk, v, L, flags=fl) == "tcgen05 k-mer tiles"
+    o, lse = pipeline.prefill_masked_parallel(cache, q, kk, v, L, flags=fl)
+    torch.cuda.synchronize()
+    ref = fo.layout(N, W, k)
+    heads, rows = np.repeat(np.arange(H), T), np.tile(np.arange(T), H)
+    o_ref, lse_ref = fo.attn_rows_kmer_local(q[0].cpu(), kk[0].cpu(), v[0].cpu(), ref["kind"], ref["win"],
+                                             fo.layout_kmer(N, W, k), 1 / math.sqrt(d), heads, rows)
+    assert_attn_close(o, lse, o_ref.reshape(B, H, T, d), lse_ref.reshape(B, H, T), "adaptive k-mer tiles")
+
+
 def test_adaptive_decode_rolls_over_windows_of_different_lengths():
     """Decode with a per-window length schedule: each sequence fills its window
     to T_w = W_w + ceil(W_w / k_w) rows, then window-mode compaction keeps its

@@ -72,6 +72,30 @@ def test_gqa_prefill_masked_parallel_matches_oracle(g, d, flags, rope, c_ring):
         assert np.array_equal(bits(cache.ring_k)[:, :, :L["R"]], bits(kk)[:, :, ref["sum_idx"]])
 
 
+def test_gqa_kmer_tiled_prefill_matches_oracle():
+    """The k-mer-local mask at a size that selects the k-mer-tiled kernel (16 windows
+    x 10 tiles x 16 query heads = 2,560 items, above its 2,048-item threshold), with
+    four query heads per K/V head and a ragged last window; every row is checked."""
+    N, W, k_, B, H, g, d = 16_037, 1_000, 100, 1, 4, 4, 64
+    k = np.full(-(-N // W), k_, np.int32)
+    L = focus.layout(N, W, k)
+    T = L["T"]
+    q = inputs.normal_bf16((B, H * g, T, d), 1.0, seed=31, device="cuda")
+    kk, v = (inputs.normal_bf16((B, H, T, d), 1.0, seed=s, device="cuda") for s in (32, 33))
+    cache = focus.Cache(B, H, d, C_ring=L["R"], k_sched=k, q_per_kv=g)
+    fl = focus.PREFILL_KMER_LOCAL
+    assert focus.prefill_kernel(cache, q, kk, v, L, flags=fl) == "tcgen05 k-mer tiles"
+    o, lse = pipeline.prefill_masked_parallel(cache, q, kk, v, L, flags=fl)
+    torch.cuda.synchronize()
+    ref = fo.layout(N, W, k)
+    Hq = H * g
+    heads, rows = np.repeat(np.arange(Hq), T), np.tile(np.arange(T), Hq)
+    o_ref, lse_ref = fo.attn_rows_kmer_local(q[0].cpu(), _expand(kk, g)[0].cpu(), _expand(v, g)[0].cpu(),
+                                             ref["kind"], ref["win"], fo.layout_kmer(N, W, k), 1 / math.sqrt(d),
+                                             heads, rows)
+    assert_attn_close(o, lse, o_ref.reshape(B, Hq, T, d), lse_ref.reshape(B, Hq, T), "gqa k-mer tiles")
+
+
 def test_gqa_prefill_streaming_matches_oracle():
     N, W, ks, B, H, g, d = 3_000, 500, [10, 50, 0, 7, 100, 500], 2, 2, 4, 64
     k = np.resize(np.asarray(ks, np.int32), 6)
