@@ -238,9 +238,18 @@ def oracle_head_times(cfg, L_host, k_sched, q, k, v, n_heads, mask="appendix"):
 
 
 def oracle_baseline(cfg, secs, mask):
-    """(nt/s of the whole workload, description) from per-head oracle passes."""
+    """(nt/s of the whole workload, description) from per-head oracle passes: the
+    sum of the passes when all B x H of them ran (the workload timed in full),
+    else B x H x the median pass."""
     per_head = statistics.median(secs)
-    full_s = per_head * cfg["B"] * cfg["H"]
+    n_pass = cfg["B"] * cfg["H"]
+    if len(secs) == n_pass:
+        full_s = sum(secs)
+        desc = ("fp64 oracle (%s), all %d (sequence, head) passes, every window and row: the workload timed in "
+                "full, %.1f s (%.3f s per pass, median)" % ("k-mer-local rows" if mask == "kmer_local" else
+                                                            "sequential prefill", n_pass, full_s, per_head))
+        return cfg["B"] * cfg["N"] / full_s, desc, full_s
+    full_s = per_head * n_pass
     desc = ("fp64 oracle (%s), %d whole (sequence, head) passes of %d, every window and row; %.3f s per pass "
             "(median); the workload's %d passes do the same visible pairs each, so its time is %d x that "
             "(extrapolated by passes)" % ("k-mer-local rows" if mask == "kmer_local" else "sequential prefill",
@@ -386,9 +395,11 @@ def run_prefill_leg(args, cfg, world, rank, local):
 
     host_sample = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        # the heads' own inputs for up to --cpu-heads passes (at least two, cycled)
+        nh = max(2, min(args.cpu_heads, q.shape[1]))
         host_sample = dict(win_off=win_off, ring_off=ring_off, kind=L["kind"].cpu().numpy(),
                            win=L["win"].cpu().numpy(), keep=L["keep"].cpu().numpy(), k_sched=k_s,
-                           q=q[0, :2].cpu(), k=k[0, :2].cpu(), v=v[0, :2].cpu())
+                           q=q[0, :nh].cpu(), k=k[0, :nh].cpu(), v=v[0, :nh].cpu())
     res = dict(kernel=kernel_name, attn_launches_per_step=1,
                step_desc="focus_layout + focus_kv_compact(bulk) + focus_attn_prefill(masked-parallel)",
                step_ms=step_ms, attn_ms=attn_ms, flops_per_step=flops_per_step, pairs=pairs, T=L["T"], R=L["R"],
