@@ -472,10 +472,26 @@ def run_stream_leg(args, cfg, world, rank, local):
              else visible_pairs(off, L["ring_off_host"]))
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     attn_ms = compact_ms = 0.0
+    use_graph = not args.no_stream_graph
+    if use_graph:
+        # the per-call split (attention launches, in-step compactions) from one eager
+        # step with events; the timed steps replay the step captured as one CUDA graph
+        step(timed=True)
+        torch.cuda.synchronize(dev)
+        attn_ms = sum(a.elapsed_time(b) for a, b in evs) * args.steps
+        compact_ms = sum(a.elapsed_time(b) for a, b in cevs) * args.steps
+        graph = pipeline.StreamingGraph(cache, L, span, outs, lses, flags=args.prefill_flags, chunk=C)
+        for _ in range(max(1, args.warmup)):
+            graph.replay()
+        torch.cuda.synchronize(dev)
+        assert focus.device_status(clear=True) == 0
     barrier(world)
     with ClockSampler(local) as clk:
         t0.record(stream)
         for _ in range(args.steps):
+            if use_graph:
+                graph.replay()
+                continue
             step(timed=True)
             torch.cuda.synchronize(dev)
             attn_ms += sum(a.elapsed_time(b) for a, b in evs)
@@ -504,7 +520,9 @@ def run_stream_leg(args, cfg, world, rank, local):
     return dict(kernel=kernel_name, attn_launches_per_step=n_calls,
                 step_desc=("per window: focus_kv_compact(window); per chunk of %d windows: focus_attn_prefill(chunk) "
                            "(the masked-parallel form over the chunk), consecutive chunks' attention overlapping on "
-                           "two streams; all windows; rate over the whole step" % C),
+                           "two streams; all windows; rate over the whole step%s" %
+                           (C, "; the step captured once as a CUDA graph (pipeline.StreamingGraph) and replayed, "
+                               "per-launch figures from one eager step" if use_graph else "")),
                 stream_chunk=C,
                 window_compaction={"kernel": "focus_kv_compact (one window)", "bytes_per_launch": wc_bytes,
                                    "in_step_ms": wc_ms,
@@ -989,6 +1007,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-heads", type=int, default=8,
                     help="whole (sequence, head) oracle passes timed for the cpu_baseline (8 of 32 = 25%%)")
+    ap.add_argument("--no-stream-graph", action="store_true",
+                    help="stream legs: enqueue every step from the host instead of replaying its CUDA graph")
     ap.add_argument("--stream-chunk", type=int, default=8,
                     help="windows per attention call in the streaming legs (divides the pool of 8; 1 = per window)")
     ap.add_argument("--no-configs", action="store_true",

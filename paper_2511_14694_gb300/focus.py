@@ -388,6 +388,10 @@ def attn_prefill(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | 
     scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
     if isinstance(workspace, str):
         workspace = new_prefill_workspace(cache, q, k, v, L, w_begin, w_end, flags)
+        if workspace is not None and stream is not None:
+            # allocated on the current stream, used on `stream`: keep the caching
+            # allocator from reusing it before the launch there is done
+            workspace.record_stream(stream)
     elif workspace is not None:
         _cuda(workspace, "workspace")
     a = _prefill_args(q, k, v, o, lse, L, w_begin, w_end, scale, flags, workspace, host_schedule)
@@ -419,6 +423,8 @@ def prefill_host(cache: Cache, L: dict, host: dict, dev: dict, copy_in, copy_out
     scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
     if isinstance(workspace, str):
         workspace = new_prefill_workspace(cache, dev["q"], dev["k"], dev["v"], L, flags=flags)
+        if workspace is not None and stream is not None:
+            workspace.record_stream(stream)          # used on `stream`, allocated on the current one
     desc = _layout_desc(L, True)
     lse_h, lse_d = host.get("lse"), dev.get("lse")
     a = PrefillHostArgs(_ptr(host["nt"]), _ptr(host["q"]), _ptr(host["k"]), _ptr(host["v"]), _ptr(host["o"]),

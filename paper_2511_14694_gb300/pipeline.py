@@ -10,7 +10,8 @@ sequences of C-ABI calls. No arithmetic happens here; each step is a kernel.
   streams overlapping the kernels of the others;
 - streaming with overlapping windows: each window's compaction first, then its
   attention on one of two side streams, so consecutive windows' launches overlap;
-  optionally several windows per attention call.
+  optionally several windows per attention call; captured once as a CUDA graph
+  and replayed (StreamingGraph).
 
 Under the k-mer-local mask (``focus.PREFILL_KMER_LOCAL``, Sec. 3.2) a row also
 reads its own window's FOCUS rows from the ring, so the streaming step compacts
@@ -58,7 +59,8 @@ def prefill_masked_parallel_host(cache: focus.Cache, L: dict, host: dict, dev: d
 
 
 def prefill_streaming(cache: focus.Cache, L: dict, window_qkv, outs, lses, w_begin: int = 0, w_end: int | None = None,
-                      scale=None, flags=0, stream=None, events=None, compact_events=None, chunk: int = 1):
+                      scale=None, flags=0, stream=None, events=None, compact_events=None, chunk: int = 1,
+                      workspaces=None):
     """Streaming prefill (App. A.2) of windows [w_begin, w_end) with the
     attention of consecutive windows (or chunks of windows) overlapping.
 
@@ -80,8 +82,10 @@ def prefill_streaming(cache: focus.Cache, L: dict, window_qkv, outs, lses, w_beg
     fewer, fuller launches and c windows' inputs resident at once.
     ``events``: optional list of (start, end) CUDA events per attention call,
     recorded around it on its stream; ``compact_events`` the same per window
-    around each compaction on ``stream``. Work is only enqueued; when ``stream``
-    is done, so is everything."""
+    around each compaction on ``stream``. ``workspaces``: optional pair of
+    attention workspaces, one per side stream (each of the largest call's
+    prefill_workspace_bytes); by default each call allocates its own. Work is
+    only enqueued; when ``stream`` is done, so is everything."""
     if chunk < 1:
         raise ValueError("chunk must be >= 1")
     cur = stream if stream is not None else torch.cuda.current_stream()
@@ -107,12 +111,58 @@ def prefill_streaming(cache: focus.Cache, L: dict, window_qkv, outs, lses, w_beg
         s_.wait_stream(cur)                    # ring rows of windows < w1 are in place
         if events is not None:
             events[n][0].record(s_)
-        focus.attn_prefill(cache, q, k, v, L, w0, w1, scale=scale, o=outs[i], lse=lses[i], flags=flags, stream=s_)
+        if workspaces is None:
+            # allocated on this stream's behalf: the caching allocator must not hand
+            # the block to another call before this launch on s_ is done with it
+            ws = focus.new_prefill_workspace(cache, q, k, v, L, w0, w1, flags)
+            if ws is not None:
+                ws.record_stream(s_)
+        else:
+            ws = workspaces[i % 2]
+        focus.attn_prefill(cache, q, k, v, L, w0, w1, scale=scale, o=outs[i], lse=lses[i], flags=flags, stream=s_,
+                           workspace=ws)
         if events is not None:
             events[n][1].record(s_)
     for s_ in side:
         cur.wait_stream(s_)
     return outs, lses
+
+
+class StreamingGraph:
+    """prefill_streaming over windows [w_begin, w_end) captured once as a CUDA
+    graph and replayed: one graph launch instead of one host call per
+    compaction and attention (about 1,100 per 1 Mb x 4 step at chunks of 8), so
+    the step no longer waits on the host to enqueue it.
+
+    The graph holds the addresses it was captured with: window_qkv's tensors, the
+    outputs, the cache and the layout. A caller streams new windows by copying
+    them into those tensors before a replay. Construction runs the step once
+    eagerly (the library's one-time set-up: the device status word, the driver's
+    tensor-map entry point, the kernels' attributes) and allocates one attention
+    workspace per side stream, so nothing is allocated inside the capture."""
+
+    def __init__(self, cache: focus.Cache, L: dict, window_qkv, outs, lses, w_begin: int = 0,
+                 w_end: int | None = None, scale=None, flags=0, chunk: int = 1):
+        w_end = L["M"] if w_end is None else w_end
+        need = 0
+        for w0 in range(w_begin, w_end, chunk):
+            w1 = min(w0 + chunk, w_end)
+            q, k, v = window_qkv(w0) if chunk == 1 else window_qkv(w0, w1)
+            need = max(need, focus.prefill_workspace_bytes(cache, q, k, v, L, w0, w1, flags))
+        dev = outs[0].device
+        self.workspaces = ([torch.empty(need, dtype=torch.uint8, device=dev) for _ in range(2)] if need
+                           else [None, None])
+        args = (cache, L, window_qkv, outs, lses, w_begin, w_end, scale, flags)
+        prefill_streaming(*args, chunk=chunk, workspaces=self.workspaces)
+        torch.cuda.synchronize(dev)
+        self.graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(self.graph):
+            prefill_streaming(*args, stream=torch.cuda.current_stream(), chunk=chunk, workspaces=self.workspaces)
+        torch.cuda.synchronize(dev)
+
+    def replay(self):
+        """Enqueue the whole step on the current stream."""
+        self.graph.replay()
 
 
 def prefill_window(cache: focus.Cache, q_w, k_w, v_w, L: dict, w: int, scale=None, o=None, lse=None, flags=0,
