@@ -423,8 +423,9 @@ def run_stream_leg(args, cfg, world, rank, local):
 
     B, N, W, H, d, P = cfg["B"], cfg["N"], cfg["W"], cfg["H"], cfg["d"], cfg["pool"]
     C = args.stream_chunk
-    if C < 1 or P % C:
-        raise ValueError(f"--stream-chunk must divide the pool of {P} windows")
+    if C < 1:
+        raise ValueError("--stream-chunk must be >= 1")
+    P = -(-max(P, C) // C) * C        # the pool holds whole chunks, at least the workload's pool
     M = focus.n_windows(N, W)
     k_s = inputs.k_schedule(M, cfg["k"], seed=inputs.DEFAULT_SEED)
     dev = torch.device("cuda", local)
