@@ -109,6 +109,10 @@ def prefill_streaming(cache: focus.Cache, L: dict, window_qkv, outs, lses, w_beg
         i = (w0 if chunk == 1 else n) % len(outs)
         s_ = side[i % 2]
         s_.wait_stream(cur)                    # ring rows of windows < w1 are in place
+        for t in (q, k, v):
+            # window_qkv may return tensors made for this call: keep the caching
+            # allocator from reusing them before the launch on s_ has read them
+            t.record_stream(s_)
         if events is not None:
             events[n][0].record(s_)
         if workspaces is None:
