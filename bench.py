@@ -237,6 +237,36 @@ def oracle_head_times(cfg, L_host, k_sched, q, k, v, n_heads, mask="appendix"):
     return secs
 
 
+def oracle_decode_times(host, fill0, R, W, Tw, n_steps, S, scale):
+    """Times the fp64 oracle's decode (App. A.2) on the decode leg's first
+    n_steps of S steps: every (sequence, K/V head) stream attends over its ring
+    rows and window rows, whose counts follow the leg's own evolution (fill + 1
+    per step; a full window of Tw rows retires its Tw - W FOCUS rows to the ring).
+    host: uint16 bf16 bits of the cache (ring_k/ring_v [B, H, C_ring, d],
+    win_k/win_v [B, H, C_win, d]) and of the steps' q, k_new, v_new ([S, B, H, d]).
+    The oracle's time depends on the row counts only, so the cache contents the
+    GPU leg left are used as they are. Returns the per-step seconds."""
+    from oracle import focus_oracle as fo
+    B, H, C_ring, d = host["ring_k"].shape
+    C_win = host["win_k"].shape[2]
+    rk, rv = host["ring_k"].reshape(B * H, C_ring, d), host["ring_v"].reshape(B * H, C_ring, d)
+    wk, wv = host["win_k"].reshape(B * H, C_win, d), host["win_v"].reshape(B * H, C_win, d)
+    fill = fill0.astype(np.int64).copy()
+    Rb = np.full(B, R, np.int64)
+    secs = []
+    for s in range(min(n_steps, S)):
+        q = host["q"][s].reshape(B * H, d)
+        kn, vn = host["k"][s].reshape(B * H, d), host["v"][s].reshape(B * H, d)
+        t0 = time.perf_counter()
+        fo.decode(q, kn, vn, rk, rv, np.repeat(Rb, H), wk, wv, np.repeat(fill, H), scale)
+        secs.append(time.perf_counter() - t0)
+        fill += 1
+        full = fill == Tw
+        Rb[full] += Tw - W
+        fill[full] = 0
+    return secs
+
+
 def oracle_baseline(cfg, secs, mask):
     """(nt/s of the whole workload, description) from per-head oracle passes: the
     sum of the passes when all B x H of them ran (the workload timed in full),
@@ -647,8 +677,22 @@ def run_decode_leg(args, cfg, world, rank, local):
     assert focus.device_status(clear=True) == 0
     leg_ms = max_over_ranks(sum(times) / reps, world)
     dec_ms = sum(a.elapsed_time(b) for rr in evs for a, b in rr) / reps
+    cpu = None
+    if rank == 0 and world == 1 and args.decode_cpu_steps > 0 and not args.rope and g == 1:
+        bits = lambda t: t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)  # noqa: E731
+        host = dict(ring_k=bits(cache.ring_k), ring_v=bits(cache.ring_v), win_k=bits(cache.win_k),
+                    win_v=bits(cache.win_v), q=bits(qs), k=bits(ks_), v=bits(vs))
+        secs = oracle_decode_times(host, fill0, R, W, Tw, args.decode_cpu_steps, S, 1.0 / math.sqrt(d))
+        total = sum(secs) * (S / len(secs))
+        full = len(secs) == S
+        cpu = {"value": B * S / total, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+               "sample": ("fp64 oracle decode (every stream over its ring and window rows), %s of the leg's %d "
+                          "steps (B=%d x H=%d streams each), %.2f s per step (mean)%s" %
+                          ("all" if full else "the first %d" % len(secs), S, B, H, sum(secs) / len(secs),
+                           "" if full else "; the leg's time is %d x the mean step (extrapolated by steps)" % S))}
+        del host
     return dict(leg_ms=leg_ms, decode_kernels_ms=dec_ms, bytes_leg=bytes_leg, steps=S, B=B,
-                clocks=clk.summary(), launches=3 * S * reps)
+                clocks=clk.summary(), launches=3 * S * reps, cpu_baseline=cpu)
 
 
 def prefill_roofline(pre, peaks, peaks_src, traffic=None):
@@ -845,6 +889,8 @@ def run_focus(args, world, rank, local):
             "clocks": dec["clocks"],
         }
         line["decode"]["gpu_launches"] = dec["launches"]
+        if dec.get("cpu_baseline") is not None:
+            line["decode"]["cpu_baseline"] = dec["cpu_baseline"]
     line.update(legs)
     if pre["host_sample"] is not None and (args.rope or args.q_per_kv > 1):
         line["cpu_baseline"] = None      # the oracle baseline times the default path only
@@ -1016,6 +1062,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-heads", type=int, default=8,
                     help="whole (sequence, head) oracle passes timed for the cpu_baseline (8 of 32 = 25%%)")
+    ap.add_argument("--decode-cpu-steps", type=int, default=8,
+                    help="decode steps the fp64 oracle runs for the decode leg's cpu_baseline (0 = none; the leg's "
+                         "256 = in full)")
     ap.add_argument("--no-stream-graph", action="store_true",
                     help="stream legs: enqueue every step from the host instead of replaying its CUDA graph")
     ap.add_argument("--stream-chunk", type=int, default=8,
