@@ -267,6 +267,33 @@ def oracle_decode_times(host, fill0, R, W, Tw, n_steps, S, scale):
     return secs
 
 
+def oracle_stream_sample(cfg, L_off, ring_off, keep, pool_q, pool_k, pool_v, n_random, seed):
+    """The fp64 oracle's sequential prefill (App. A.2) on a sample of the streaming
+    workload: batch 0, every head, the rows of the last window and of n_random
+    other windows (seeded), each head over the whole sequence (retention runs for
+    every window; only the sampled windows' rows are computed). The sequence's
+    rows are the leg's pool of windows repeated, as the GPU leg cycles it.
+    Returns (seconds, sampled visible pairs, all visible pairs) over the heads."""
+    from oracle import focus_oracle as fo
+    M = L_off.size - 1
+    rng = np.random.default_rng(seed)
+    pick = np.zeros(M, np.uint8)
+    pick[M - 1] = 1
+    pick[rng.choice(M - 1, size=min(n_random, M - 1), replace=False)] = 1
+    tw = np.diff(L_off).astype(np.int64)
+    pairs_w = tw * (tw + 1) // 2 + tw * ring_off[:-1].astype(np.int64)
+    H, P_rows, d = pool_q.shape
+    reps = -(-int(L_off[-1]) // P_rows)
+    scale = 1.0 / math.sqrt(d)
+    secs = 0.0
+    for h in range(H):
+        q, k, v = (np.tile(p[h], (reps, 1))[: int(L_off[-1])] for p in (pool_q, pool_k, pool_v))
+        t0 = time.perf_counter()
+        fo.prefill_sequential(q, k, v, L_off, keep, scale, want=pick)
+        secs += time.perf_counter() - t0
+    return secs, H * int(pairs_w[pick == 1].sum()), H * int(pairs_w.sum()), int(pick.sum())
+
+
 def oracle_baseline(cfg, secs, mask):
     """(nt/s of the whole workload, description) from per-head oracle passes: the
     sum of the passes when all B x H of them ran (the workload timed in full),
@@ -545,6 +572,21 @@ def run_stream_leg(args, cfg, world, rank, local):
     step_ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, world)
     # the attention launches overlap, so the rate is taken over the whole step
     # (compactions and gaps included); per_launch_ms is each launch on its stream
+    cpu = None
+    if rank == 0 and world == 1 and args.stream_cpu_windows > 0 and not local_mask and not args.rope and g == 1:
+        bits = lambda t: t[0].contiguous().view(torch.int16).cpu().numpy().view(np.uint16)  # noqa: E731
+        # the pool as the leg cycles it: window w is pool window w mod P
+        pool = [np.concatenate([bits(t[j]) for j in range(n_slots)], axis=1) for t in (pq, pk, pv)]
+        secs, sp, ap_, nw = oracle_stream_sample(cfg, np.asarray(off), np.asarray(L["ring_off_host"]),
+                                                 L["keep"].cpu().numpy(), pool[0], pool[1], pool[2],
+                                                 args.stream_cpu_windows, inputs.DEFAULT_SEED)
+        full_s = secs * ap_ / sp * B               # every sequence has the same windows and pairs
+        cpu = {"value": B * N / full_s, "unit": "nt/s", "cores": os.cpu_count(), "kind": "oracle",
+               "sample": "fp64 oracle (sequential prefill with retention), batch 0, all %d heads, the rows of %d "
+                         "windows (the last and %d seeded others) of %d: %.1f s for %.3g of the %.3g visible "
+                         "pairs per sequence; the workload's time is that per pair x all pairs x %d sequences "
+                         "(extrapolated)" % (H, nw, nw - 1, M, secs, sp, ap_, B)}
+        del pool
     # per-window compaction: the window's kept rows of every (sequence, K/V head), read and written
     wc_ms = compact_ms / args.steps / M
     wc_bytes = float((L["R"] / M) * B * (H // g) * 2 * (2 * d) * 2)
@@ -564,6 +606,7 @@ def run_stream_leg(args, cfg, world, rank, local):
                                                  "launch, launch-latency bound" % n_alone},
                 step_ms=step_ms, attn_ms=step_ms, flops_per_step=4.0 * d * H * B * pairs, pairs=pairs,
                 T=L["T"], R=L["R"], clocks=clk.summary(), launches=(M + n_calls) * args.steps, e2e=None, host_sample=None,
+                cpu_baseline=cpu,
                 per_launch_ms=attn_ms / args.steps / n_calls, local_mask=local_mask,
                 bytes_per_step=float(B * L["T"] * (H * (4 * d + 4) + (H // g) * 4 * d)))
 
@@ -752,6 +795,8 @@ def run_config_leg(args, name, steps, warmup, world, rank, local, peaks, peaks_s
            "gpu_launches": pre["launches"]}
     if pre.get("window_compaction") is not None:
         obj["window_compaction"] = pre["window_compaction"]
+    if pre.get("cpu_baseline") is not None:
+        obj["cpu_baseline"] = pre["cpu_baseline"]
     return obj
 
 
@@ -892,6 +937,8 @@ def run_focus(args, world, rank, local):
         if dec.get("cpu_baseline") is not None:
             line["decode"]["cpu_baseline"] = dec["cpu_baseline"]
     line.update(legs)
+    if pre.get("cpu_baseline") is not None:          # a stream workload's oracle sample
+        line["cpu_baseline"] = pre["cpu_baseline"]
     if pre["host_sample"] is not None and (args.rope or args.q_per_kv > 1):
         line["cpu_baseline"] = None      # the oracle baseline times the default path only
     elif pre["host_sample"] is not None:
@@ -1065,6 +1112,9 @@ def main():
     ap.add_argument("--decode-cpu-steps", type=int, default=8,
                     help="decode steps the fp64 oracle runs for the decode leg's cpu_baseline (0 = none; the leg's "
                          "256 = in full)")
+    ap.add_argument("--stream-cpu-windows", type=int, default=8,
+                    help="stream legs (appendix mask): windows besides the last on which the fp64 oracle runs for "
+                         "the leg's cpu_baseline (0 = none)")
     ap.add_argument("--no-stream-graph", action="store_true",
                     help="stream legs: enqueue every step from the host instead of replaying its CUDA graph")
     ap.add_argument("--stream-chunk", type=int, default=8,
