@@ -765,7 +765,7 @@ def prefill_roofline(pre, peaks, peaks_src, traffic=None):
 
 # the other named workloads and options timed beside the headline:
 # (key, workload, steps, warm-up, options: mask, rotary base)
-CONFIG_LEGS = [("ksweep", "prefill_256kb_ksweep_h32_d128", 10, 3, {}),
+CONFIG_LEGS = [("ksweep", "prefill_256kb_ksweep_h32_d128", 10, 3, {"cpu_heads": 1}),
                ("causal", "causal_128kb_h32_d128", 3, 3, {}),
                ("stream", "stream_1mb_b4_h32_d128", 2, 3, {}),
                ("kmer_local", "prefill_128kb_h32_d128", 20, 3, {"mask": "kmer_local"}),
@@ -783,7 +783,10 @@ def run_config_leg(args, name, steps, warmup, world, rank, local, peaks, peaks_s
     cfg = WORKLOADS[name]
     opts = opts or {}
     a = copy.copy(args)
-    a.steps, a.warmup, a.no_e2e, a.no_cpu_baseline = steps, warmup, True, True
+    a.steps, a.warmup, a.no_e2e = steps, warmup, True
+    # an oracle sample for the legs that ask for one (whole (sequence, head) passes)
+    a.cpu_heads = int(opts.get("cpu_heads", 0)) if opts else 0
+    a.no_cpu_baseline = a.cpu_heads == 0 or args.no_cpu_baseline
     a.rope, a.q_per_kv, a.mask = float(opts.get("rope", 0.0)), 1, opts.get("mask", "appendix")
     a.prefill_flags = 2 if a.mask == "kmer_local" else 0
     pre = (run_stream_leg if cfg["mode"] == "stream" else run_prefill_leg)(a, cfg, world, rank, local)
@@ -797,6 +800,12 @@ def run_config_leg(args, name, steps, warmup, world, rank, local, peaks, peaks_s
         obj["window_compaction"] = pre["window_compaction"]
     if pre.get("cpu_baseline") is not None:
         obj["cpu_baseline"] = pre["cpu_baseline"]
+    if pre.get("host_sample") is not None:
+        hs = pre["host_sample"]
+        secs = oracle_head_times(cfg, hs, hs["k_sched"], hs["q"], hs["k"], hs["v"], a.cpu_heads, mask=a.mask)
+        val, desc, _ = oracle_baseline(cfg, secs, a.mask)
+        obj["cpu_baseline"] = {"value": val, "unit": "nt/s", "cores": os.cpu_count(), "kind": "oracle",
+                               "sample": desc}
     return obj
 
 
