@@ -329,26 +329,28 @@ def test_prefill_streaming_overlapped_equals_sequential(d, tail, flags):
         assert np.array_equal(bits(c_chk.ring_v), bits(c_seq.ring_v))
 
 
-@pytest.mark.parametrize("d,flags,rope,chunk", [(128, 0, 0.0, 3), (64, 0, 0.0, 1),
-                                                (128, focus.PREFILL_KMER_LOCAL, 0.0, 4), (128, 0, 10_000.0, 2)])
-def test_prefill_streaming_graph_equals_eager(d, flags, rope, chunk):
+@pytest.mark.parametrize("d,flags,rope,chunk,g", [(128, 0, 0.0, 3, 1), (64, 0, 0.0, 1, 1),
+                                                  (128, focus.PREFILL_KMER_LOCAL, 0.0, 4, 1),
+                                                  (128, 0, 10_000.0, 2, 1), (64, 0, 0.0, 2, 4)])
+def test_prefill_streaming_graph_equals_eager(d, flags, rope, chunk, g):
     """pipeline.StreamingGraph (the streaming step captured once as a CUDA graph)
     replays to the eager pipeline.prefill_streaming's outputs and ring, bit for
     bit, and rewrites them on every replay (outputs and ring are cleared between
     replays); chunk 3 leaves a partial last chunk, the rotary case allocates its
-    workspaces before the capture."""
+    workspaces before the capture, g = 4 groups the query heads."""
     N, W, ks, B, H = 6_000, 500, [10, 50, 100, 7], 2, 2
     M = -(-N // W)
     k_s = inputs.k_schedule(M, ks, seed=5)
     L = focus.layout(N, W, k_s)
-    q, k, v = inputs.qkv((B, H, L["T"], d), seed=29, device="cuda")
+    q = inputs.normal_bf16((B, H * g, L["T"], d), 1.0, seed=29, device="cuda")
+    k, v = (inputs.normal_bf16((B, H, L["T"], d), 1.0, seed=s, device="cuda") for s in (30, 31))
     off = L["win_off_host"]
     spn = lambda t, w0, w1: t[:, :, int(off[w0]):int(off[w1])].contiguous()  # noqa: E731
     spans = {w0: tuple(spn(t, w0, min(w0 + chunk, M)) for t in (q, k, v)) for w0 in range(0, M, chunk)}
     qkv = (lambda w0: spans[w0]) if chunk == 1 else (lambda w0, w1: spans[w0])
     runs = {}
     for mode in ("eager", "graph"):
-        cache = focus.Cache(B, H, d, C_ring=L["R"], k_sched=k_s, rope_theta=rope)
+        cache = focus.Cache(B, H, d, C_ring=L["R"], k_sched=k_s, rope_theta=rope, q_per_kv=g)
         outs = [torch.empty_like(spans[w0][0]) for w0 in range(0, M, chunk)]
         lses = [torch.empty(x.shape[:3], dtype=torch.float32, device="cuda") for x in outs]
         if mode == "eager":
