@@ -31,6 +31,15 @@
  *     word; the affected work is skipped, never trapped. Read and clear it with
  *     focus_get_device_status().
  *   - Supported head dimensions: d = 64 and d = 128.
+ *   - CUDA graphs: focus_layout, focus_kv_compact, focus_attn_prefill,
+ *     focus_attn_decode(_noalloc) and focus_embed_tokens enqueue kernels on the
+ *     given stream only, allocate nothing and never synchronize, so they can be
+ *     captured (stream capture) and the graph replayed. A graph keeps the
+ *     pointers it was captured with; the cache's lengths live in device memory,
+ *     so replays of a decode step advance them. Make each call once outside the
+ *     capture first: the first call per device sets up the status word, the
+ *     driver's tensor-map entry point and the kernels' attributes.
+ *     focus_get_device_status synchronizes and cannot be captured.
  */
 #ifndef FOCUS_H_
 #define FOCUS_H_
