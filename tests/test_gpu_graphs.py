@@ -1,11 +1,9 @@
 """CUDA-graph capture of the library's entry points: the layout, the
-masked-parallel prefill (bulk compaction + attention) and decode steps with
-window roll-overs, captured once and replayed, give the eager calls' results
-bit for bit (the entry points enqueue work on the given stream only, allocate
-nothing and never synchronize). The streaming prefill's graph is covered in
-test_gpu_parity.py."""
-import math
-
+masked-parallel prefill (bulk compaction + attention), decode steps with window
+roll-overs, the allocation-free decode and the token-embedding gather, captured
+once and replayed, give the eager calls' results bit for bit (the entry points
+enqueue work on the given stream only, allocate nothing and never synchronize).
+The streaming prefill's graph is covered in test_gpu_parity.py."""
 import numpy as np
 import pytest
 import torch
@@ -127,3 +125,51 @@ def test_decode_step_graph_replay(g_heads, rope):
         assert torch.equal(a, b)
     assert np.array_equal(bits(ce.ring_k), bits(cg.ring_k))
     assert np.array_equal(bits(ce.win_k), bits(cg.win_k))
+
+
+def test_embed_tokens_graph_replay():
+    N, W = 5_000, 1_000
+    nt = inputs.nucleotides(1, N, seed=8, device="cuda")
+    L = focus.layout(N, W, [100], nt=nt)
+    table = inputs.normal_bf16((5, 512), 1.0, seed=9, device="cuda")
+    ref = focus.embed_tokens(L["tok"], table)
+    out = torch.empty_like(ref)
+    g = _capture(lambda: focus.embed_tokens(L["tok"], table, out=out))
+    out.zero_()
+    g.replay()
+    torch.cuda.synchronize()
+    assert np.array_equal(bits(out), bits(ref))
+
+
+def test_decode_noalloc_graph_replay():
+    """The allocation-free decode (library-owned scratch) captured and replayed
+    equals focus_attn_decode with a caller workspace."""
+    B, H, d, W = 2, 4, 128, 50
+    k_sched = np.full(64, 10, np.int32)
+    caches = [focus.Cache(B, H, d, C_ring=256, C_win=64, W=W, k_sched=k_sched) for _ in range(2)]
+    gen = torch.Generator(device="cuda").manual_seed(17)
+    for t in (caches[0].ring_k, caches[0].ring_v, caches[0].win_k, caches[0].win_v):
+        t.copy_(torch.randn(t.shape, generator=gen, device="cuda").bfloat16())
+    for a, b in zip((caches[0].ring_k, caches[0].ring_v, caches[0].win_k, caches[0].win_v),
+                    (caches[1].ring_k, caches[1].ring_v, caches[1].win_k, caches[1].win_v)):
+        b.copy_(a)
+    for c in caches:
+        c.ring_len.fill_(100)
+        c.win_idx.fill_(10)
+        c.win_fill.fill_(7)
+    q, kn, vn = (inputs.normal_bf16((B, H, d), 1.0, seed=30 + i, device="cuda") for i in range(3))
+    o_e, l_e = focus.attn_decode(caches[0], q, kn, vn, workspace=caches[0].new_workspace())
+    o_g = torch.empty_like(q)
+    l_g = torch.empty((B, H), dtype=torch.float32, device="cuda")
+    warm = focus.Cache(B, H, d, C_ring=256, C_win=64, W=W, k_sched=k_sched)
+    focus.attn_decode_noalloc(warm, q, kn, vn, o=o_g, lse=l_g)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        focus.attn_decode_noalloc(caches[1], q, kn, vn, o=o_g, lse=l_g)
+    o_g.zero_()
+    g.replay()
+    torch.cuda.synchronize()
+    assert np.array_equal(bits(o_g), bits(o_e))
+    assert torch.equal(l_g, l_e)
+    assert torch.equal(caches[0].win_fill, caches[1].win_fill)
