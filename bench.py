@@ -267,29 +267,30 @@ def oracle_decode_times(host, fill0, R, W, Tw, n_steps, S, scale):
     return secs
 
 
-def oracle_stream_sample(cfg, L_off, ring_off, keep, pool_q, pool_k, pool_v, n_random, seed):
+def oracle_stream_sample(win_off, ring_off, keep, pool_q, pool_k, pool_v, n_random, seed):
     """The fp64 oracle's sequential prefill (App. A.2) on a sample of the streaming
     workload: batch 0, every head, the rows of the last window and of n_random
     other windows (seeded), each head over the whole sequence (retention runs for
     every window; only the sampled windows' rows are computed). The sequence's
     rows are the leg's pool of windows repeated, as the GPU leg cycles it.
-    Returns (seconds, sampled visible pairs, all visible pairs) over the heads."""
+    Returns (seconds, sampled visible pairs, all visible pairs, windows sampled),
+    pairs over the heads."""
     from oracle import focus_oracle as fo
-    M = L_off.size - 1
+    M = win_off.size - 1
     rng = np.random.default_rng(seed)
     pick = np.zeros(M, np.uint8)
     pick[M - 1] = 1
     pick[rng.choice(M - 1, size=min(n_random, M - 1), replace=False)] = 1
-    tw = np.diff(L_off).astype(np.int64)
+    tw = np.diff(win_off).astype(np.int64)
     pairs_w = tw * (tw + 1) // 2 + tw * ring_off[:-1].astype(np.int64)
     H, P_rows, d = pool_q.shape
-    reps = -(-int(L_off[-1]) // P_rows)
+    reps = -(-int(win_off[-1]) // P_rows)
     scale = 1.0 / math.sqrt(d)
     secs = 0.0
     for h in range(H):
-        q, k, v = (np.tile(p[h], (reps, 1))[: int(L_off[-1])] for p in (pool_q, pool_k, pool_v))
+        q, k, v = (np.tile(p[h], (reps, 1))[: int(win_off[-1])] for p in (pool_q, pool_k, pool_v))
         t0 = time.perf_counter()
-        fo.prefill_sequential(q, k, v, L_off, keep, scale, want=pick)
+        fo.prefill_sequential(q, k, v, win_off, keep, scale, want=pick)
         secs += time.perf_counter() - t0
     return secs, H * int(pairs_w[pick == 1].sum()), H * int(pairs_w.sum()), int(pick.sum())
 
@@ -577,7 +578,7 @@ def run_stream_leg(args, cfg, world, rank, local):
         bits = lambda t: t[0].contiguous().view(torch.int16).cpu().numpy().view(np.uint16)  # noqa: E731
         # the pool as the leg cycles it: window w is pool window w mod P
         pool = [np.concatenate([bits(t[j]) for j in range(n_slots)], axis=1) for t in (pq, pk, pv)]
-        secs, sp, ap_, nw = oracle_stream_sample(cfg, np.asarray(off), np.asarray(L["ring_off_host"]),
+        secs, sp, ap_, nw = oracle_stream_sample(np.asarray(off), np.asarray(L["ring_off_host"]),
                                                  L["keep"].cpu().numpy(), pool[0], pool[1], pool[2],
                                                  args.stream_cpu_windows, inputs.DEFAULT_SEED)
         full_s = secs * ap_ / sp * B               # every sequence has the same windows and pairs
