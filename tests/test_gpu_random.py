@@ -4,7 +4,9 @@ length, fixed or adaptive windows, per-window cadences (including k = 0, k = 1 a
 k > W), boundary tail, mask (App. A's appendix mask or Sec. 3.2's k-mer-local
 mask), rotary embedding and ring capacity (which selects the persistent or the
 one-CTA-per-item kernel). The layout must match bit for bit and every output row
-must meet the parity tolerance."""
+must meet the parity tolerance. A second sweep draws random decode caches
+(per-sequence ring lengths, fills and window indices, W, cadences, tails, grouped
+heads) and checks 40 decode steps each."""
 import math
 
 import numpy as np
@@ -87,3 +89,58 @@ def test_random_prefill_matches_oracle(seed):
     else:
         o_ref, lse_ref = fo.attn_rows(qh, kh, vh, ref["keep"], ref["win"], scale, heads, rows)
     assert_attn_close(o, lse, o_ref.reshape(B, Hq, T, d), lse_ref.reshape(B, Hq, T), str(c))
+
+
+@pytest.mark.parametrize("seed", range(24))
+def test_random_decode_matches_oracle(seed):
+    """Decode steps (App. A.2) on random caches: per-sequence ring lengths, window
+    fills and window indices, window length W, cadences (k = 0: no summary rows),
+    boundary tails and grouped heads; 40 steps against the oracle with the cache
+    evolved on the host (the window's kept rows join the ring when it is full)."""
+    r = np.random.default_rng(10_000 + seed)
+    d, B, H = int(r.choice([64, 128])), int(r.integers(1, 5)), int(r.integers(1, 4))
+    g, W, tail = int(r.choice([1, 2, 3, 4, 8])), int(r.integers(8, 100)), int(r.choice([0, 0, 2]))
+    k_sched = np.asarray(r.choice([0, 1, 2, 3, 5, 10, W, W + 7], size=64), np.int32)
+    Tws = np.array([W + (-(-W // kk) if kk > 0 else 0) for kk in k_sched])
+    widx = r.integers(0, 8, size=B).astype(np.int32)
+    fill = np.array([r.integers(0, Tws[w]) for w in widx], np.int32)
+    R = r.integers(0, 300, size=B).astype(np.int32)
+    cache = focus.Cache(B, H, d, C_ring=int(R.max()) + 2 * W + 128, C_win=int(Tws.max()) + 8, W=W, k_sched=k_sched,
+                        tail=tail, q_per_kv=g)
+    gen = torch.Generator(device="cuda").manual_seed(seed)
+    for t in (cache.ring_k, cache.ring_v, cache.win_k, cache.win_v):
+        t.copy_(torch.randn(t.shape, generator=gen, device="cuda").bfloat16())
+    cache.ring_len.copy_(torch.from_numpy(R))
+    cache.win_idx.copy_(torch.from_numpy(widx))
+    cache.win_fill.copy_(torch.from_numpy(fill))
+    bits_ = lambda t: t.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16)  # noqa: E731
+    rk, rv, wk, wv = (bits_(t).copy() for t in (cache.ring_k, cache.ring_v, cache.win_k, cache.win_v))
+    Rm, fm, wm = R.astype(np.int64), fill.astype(np.int64), widx.astype(np.int64)
+    ws = cache.new_workspace()
+    e = np.arange(H * g) // g                      # K/V head of each query head
+    scale = 1 / math.sqrt(d)
+    for step in range(40):
+        q = inputs.normal_bf16((B, H * g, d), 1.0, seed=20_000 + 97 * seed + step, device="cuda")
+        kn, vn = (inputs.normal_bf16((B, H, d), 1.0, seed=30_000 + 97 * seed + 2 * step + i, device="cuda")
+                  for i in (0, 1))
+        o, lse = focus.attn_decode(cache, q, kn, vn, workspace=ws)
+        focus.kv_compact_window(cache)
+        qb, kb, vb = bits_(q), bits_(kn), bits_(vn)
+        o_ref, lse_ref = np.zeros((B, H * g, d)), np.zeros((B, H * g))
+        for b in range(B):
+            o_ref[b], lse_ref[b] = fo.decode(qb[b], kb[b][e], vb[b][e], rk[b][e], rv[b][e], [Rm[b]] * (H * g),
+                                             wk[b][e], wv[b][e], [fm[b]] * (H * g), scale)
+            wk[b, :, fm[b]], wv[b, :, fm[b]] = kb[b], vb[b]
+            fm[b] += 1
+            kw = int(k_sched[wm[b]])
+            if fm[b] == Tws[wm[b]]:                # window complete: its kept rows join the ring
+                keep = fo.window_retained_rows(W, kw, True, tail)
+                rk[b, :, Rm[b]:Rm[b] + keep.size] = wk[b][:, keep]
+                rv[b, :, Rm[b]:Rm[b] + keep.size] = wv[b][:, keep]
+                Rm[b] += keep.size
+                fm[b] = 0
+                wm[b] += 1
+        assert_attn_close(o, lse, o_ref, lse_ref, f"seed {seed} step {step}: d={d} B={B} H={H} g={g} W={W} tail={tail}")
+    torch.cuda.synchronize()
+    assert np.array_equal(cache.ring_len.cpu().numpy(), Rm)
+    assert np.array_equal(cache.win_fill.cpu().numpy(), fm)
