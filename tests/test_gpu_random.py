@@ -6,8 +6,10 @@ mask), rotary embedding and ring capacity (which selects the persistent or the
 one-CTA-per-item kernel). The layout must match bit for bit and every output row
 must meet the parity tolerance. A second sweep draws random decode caches
 (per-sequence ring lengths, fills and window indices, W, cadences, tails, grouped
-heads) and checks 40 decode steps each."""
+heads) and checks 40 decode steps each. FOCUS_RANDOM_PREFILL_SEEDS and
+FOCUS_RANDOM_DECODE_SEEDS widen the sweeps (the same generators, more seeds)."""
 import math
+import os
 
 import numpy as np
 import pytest
@@ -20,6 +22,8 @@ from test_gpu_parity import PER_ITEM_C_RING, assert_attn_close
 pytestmark = pytest.mark.gpu
 
 K_CHOICES = [0, 1, 2, 3, 7, 10, 50, 100, 5_000]
+N_PREFILL = int(os.environ.get("FOCUS_RANDOM_PREFILL_SEEDS", "128"))
+N_DECODE = int(os.environ.get("FOCUS_RANDOM_DECODE_SEEDS", "48"))
 
 
 @pytest.fixture(autouse=True)
@@ -52,7 +56,7 @@ def _draw(seed):
     return case
 
 
-@pytest.mark.parametrize("seed", range(64))
+@pytest.mark.parametrize("seed", range(N_PREFILL))
 def test_random_prefill_matches_oracle(seed):
     c = _draw(seed)
     d, B, H, g, N, W, k, tail = c["d"], c["B"], c["H"], c["g"], c["N"], c["W"], c["k"], c["tail"]
@@ -91,7 +95,7 @@ def test_random_prefill_matches_oracle(seed):
     assert_attn_close(o, lse, o_ref.reshape(B, Hq, T, d), lse_ref.reshape(B, Hq, T), str(c))
 
 
-@pytest.mark.parametrize("seed", range(24))
+@pytest.mark.parametrize("seed", range(N_DECODE))
 def test_random_decode_matches_oracle(seed):
     """Decode steps (App. A.2) on random caches: per-sequence ring lengths, window
     fills and window indices, window length W, cadences (k = 0: no summary rows),
