@@ -98,25 +98,31 @@ def test_random_prefill_matches_oracle(seed):
 @pytest.mark.parametrize("seed", range(N_DECODE))
 def test_random_decode_matches_oracle(seed):
     """Decode steps (App. A.2) on random caches: per-sequence ring lengths, window
-    fills and window indices, window length W, cadences (k = 0: no summary rows),
-    boundary tails and grouped heads; 40 steps against the oracle with the cache
-    evolved on the host (the window's kept rows join the ring when it is full)."""
+    fills, window indices and (with the rotary embedding) first positions, window
+    length W, cadences (k = 0: no summary rows), boundary tails and grouped heads;
+    40 steps against the oracle with the cache evolved on the host (the window's
+    kept rows join the ring when it is full)."""
     r = np.random.default_rng(10_000 + seed)
     d, B, H = int(r.choice([64, 128])), int(r.integers(1, 5)), int(r.integers(1, 4))
     g, W, tail = int(r.choice([1, 2, 3, 4, 8])), int(r.integers(8, 100)), int(r.choice([0, 0, 2]))
     k_sched = np.asarray(r.choice([0, 1, 2, 3, 5, 10, W, W + 7], size=64), np.int32)
+    theta = float(r.choice([0.0, 0.0, 10_000.0, 500_000.0]))
     Tws = np.array([W + (-(-W // kk) if kk > 0 else 0) for kk in k_sched])
     widx = r.integers(0, 8, size=B).astype(np.int32)
     fill = np.array([r.integers(0, Tws[w]) for w in widx], np.int32)
     R = r.integers(0, 300, size=B).astype(np.int32)
     cache = focus.Cache(B, H, d, C_ring=int(R.max()) + 2 * W + 128, C_win=int(Tws.max()) + 8, W=W, k_sched=k_sched,
-                        tail=tail, q_per_kv=g)
+                        tail=tail, q_per_kv=g, rope_theta=theta)
     gen = torch.Generator(device="cuda").manual_seed(seed)
     for t in (cache.ring_k, cache.ring_v, cache.win_k, cache.win_v):
         t.copy_(torch.randn(t.shape, generator=gen, device="cuda").bfloat16())
     cache.ring_len.copy_(torch.from_numpy(R))
     cache.win_idx.copy_(torch.from_numpy(widx))
     cache.win_fill.copy_(torch.from_numpy(fill))
+    if theta:
+        cache.pos_base.copy_(torch.from_numpy(r.integers(0, 1_000_000, size=B).astype(np.int32)))
+        _rope_decode_steps(cache, W, k_sched, theta, tail, g, seed)
+        return
     bits_ = lambda t: t.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16)  # noqa: E731
     rk, rv, wk, wv = (bits_(t).copy() for t in (cache.ring_k, cache.ring_v, cache.win_k, cache.win_v))
     Rm, fm, wm = R.astype(np.int64), fill.astype(np.int64), widx.astype(np.int64)
@@ -148,3 +154,26 @@ def test_random_decode_matches_oracle(seed):
     torch.cuda.synchronize()
     assert np.array_equal(cache.ring_len.cpu().numpy(), Rm)
     assert np.array_equal(cache.win_fill.cpu().numpy(), fm)
+
+
+def _rope_decode_steps(cache, W, k_sched, theta, tail, g, seed):
+    """The rotary case of the sweep: q and k_new rotated at pos_base + fill, the
+    host mirror of test_gpu_rope.py evolving the rotated keys."""
+    from test_gpu_rope import RopeDecodeModel
+    B, H, d = cache.B, cache.H, cache.d
+    model = RopeDecodeModel(cache, W, k_sched, theta, tail)
+    ws = cache.new_workspace()
+    scale = 1 / math.sqrt(d)
+    for step in range(40):
+        q = inputs.normal_bf16((B, H * g, d), 1.0, seed=20_000 + 97 * seed + step, device="cuda")
+        kn, vn = (inputs.normal_bf16((B, H, d), 1.0, seed=30_000 + 97 * seed + 2 * step + i, device="cuda")
+                  for i in (0, 1))
+        o, lse = focus.attn_decode(cache, q, kn, vn, workspace=ws)
+        focus.kv_compact_window(cache)
+        o_ref, lse_ref = model.step(q, kn, vn, scale)
+        assert_attn_close(o, lse, o_ref, lse_ref, f"seed {seed} step {step}: rope {theta} d={d} B={B} H={H} g={g} "
+                                                  f"W={W} tail={tail}")
+    torch.cuda.synchronize()
+    assert np.array_equal(cache.ring_len.cpu().numpy(), model.R)
+    assert np.array_equal(cache.win_fill.cpu().numpy(), model.fill)
+    assert np.array_equal(cache.pos_base.cpu().numpy(), model.pos)

@@ -143,9 +143,10 @@ def test_prefill_rope_streaming_matches_oracle(d):
 class RopeDecodeModel:
     """Host mirror of the decode cache with fp64 (rotated) keys, evolved with the
     oracle's rules (App. A.2): each step rotates q and k_new at the new row's
-    position id pos_base + fill, appends, and retires full windows."""
+    position id pos_base + fill, appends, and retires full windows (their summary
+    rows and the last `tail` ordinary rows join the ring)."""
 
-    def __init__(self, cache, W, k_sched, theta):
+    def __init__(self, cache, W, k_sched, theta, tail=0):
         B, H = cache.B, cache.H
         self.g = max(cache.q_per_kv, 1)          # query heads per K/V head
         self.rk = cache.ring_k.float().cpu().double().numpy().copy()
@@ -156,7 +157,7 @@ class RopeDecodeModel:
         self.fill = cache.win_fill.cpu().numpy().copy()
         self.widx = cache.win_idx.cpu().numpy().copy()
         self.pos = cache.pos_base.cpu().numpy().astype(np.int64).copy()
-        self.W, self.k, self.theta, self.H = W, np.asarray(k_sched), theta, H
+        self.W, self.k, self.theta, self.H, self.tail = W, np.asarray(k_sched), theta, H, tail
 
     def step(self, q, kn, vn, scale):
         B, Hq, d = q.shape
@@ -174,7 +175,7 @@ class RopeDecodeModel:
             kw = int(self.k[self.widx[b]])
             Tw = self.W + (-(-self.W // kw) if kw > 0 else 0)
             if self.fill[b] == Tw:
-                rows = fo.window_retained_rows(self.W, kw, True, 0)
+                rows = fo.window_retained_rows(self.W, kw, True, self.tail)
                 r = self.R[b]
                 self.rk[b, :, r:r + rows.size] = self.wk[b][:, rows]
                 self.rv[b, :, r:r + rows.size] = self.wv[b][:, rows]
