@@ -416,7 +416,8 @@ def run_prefill_leg(args, cfg, world, rank, local):
     compact_ms = sum(a.elapsed_time(b) for a, b in evc) / args.steps
     # compaction moves R rows of K and V per K/V head: read once, written once
     compact_bytes = float(L["R"] * B * (H // g) * 2 * (2 * d) * 2)
-    launches = 4 * args.steps   # layout scan + layout rows + bulk compaction + prefill
+    # layout scan + layout rows + bulk compaction + prefill (+ the rotary embedding's pass)
+    launches = (4 + kernel_name.startswith("rotation pass")) * args.steps
 
     # end to end through the public API with host buffers: the pipelined host-buffer
     # prefill (copies of one head group overlap the kernels of the others)
@@ -606,7 +607,7 @@ def run_stream_leg(args, cfg, world, rank, local):
                                    "alone_note": "median of %d launches with nothing else running: a ~1 MB "
                                                  "launch, launch-latency bound" % n_alone},
                 step_ms=step_ms, attn_ms=step_ms, flops_per_step=4.0 * d * H * B * pairs, pairs=pairs,
-                T=L["T"], R=L["R"], clocks=clk.summary(), launches=(M + n_calls) * args.steps, e2e=None, host_sample=None,
+                T=L["T"], R=L["R"], clocks=clk.summary(), launches=(M + n_calls * (1 + kernel_name.startswith("rotation pass"))) * args.steps, e2e=None, host_sample=None,
                 cpu_baseline=cpu,
                 per_launch_ms=attn_ms / args.steps / n_calls, local_mask=local_mask,
                 bytes_per_step=float(B * L["T"] * (H * (4 * d + 4) + (H // g) * 4 * d)))
@@ -759,8 +760,9 @@ def prefill_roofline(pre, peaks, peaks_src, traffic=None):
              "frac": achieved / peaks["bf16_tflops"], "peak_source": f"{peaks_src} bf16 dense burst",
              "frac_of_sustained": achieved / peaks["bf16_tflops_sustained"], "kernel": "prefill attention"}
     r.update(common)
-    if pre.get("rotate_ms") is not None:
-        r["rotation_pass_ms"] = pre["rotate_ms"]
+    if pre["kernel"].startswith("rotation pass"):
+        # the rotary embedding's pass runs inside each timed call, before the attention
+        r["kernel"] += " with the rotation pass before it (both launches in the timed call)"
     return r
 
 
@@ -812,12 +814,13 @@ def run_config_leg(args, name, steps, warmup, world, rank, local, peaks, peaks_s
 
 def leg_traffic(pre, args, cfg):
     """DRAM bytes per launch from the committed ncu counters, which exist for the
-    128 kb workload (default heads) on the appendix-mask persistent kernel, its
-    rotary variant and the k-mer-tiled kernel; None elsewhere or once the
-    kernel's source has changed since the capture."""
+    128 kb workload (default heads) on the appendix-mask persistent kernel, the
+    rotary embedding's pass with that kernel after it (the two launches of one
+    call) and the k-mer-tiled kernel; None elsewhere or once a kernel's source has
+    changed since the capture."""
     from paper_2511_14694_gb300.workloads import WORKLOADS
     key = {("tcgen05 persistent", False, False): ("prefill_attention", "prefill_tc_persistent.cu"),
-           ("tcgen05 persistent", False, True): ("prefill_attention_rope", "prefill_tc_persistent.cu"),
+           ("rotation pass + tcgen05 persistent", False, True): ("prefill_attention_rope", "rope.cu"),
            ("tcgen05 k-mer tiles", True, False): ("prefill_attention_kmer_local", "prefill_tc_kmer.cu"),
            }.get((pre["kernel"], pre.get("local_mask", False), bool(args.rope)))
     if not key or args.q_per_kv != 1 or cfg is not WORKLOADS["prefill_128kb_h32_d128"]:

@@ -230,16 +230,19 @@ typedef struct focus_prefill_args {
                                       kernel that finds them different reports FOCUS_ERR_INVALID_ARG */
 } focus_prefill_args;
 
-/* Device workspace that lets focus_attn_prefill use its fastest kernel for these
+/* Device workspace that lets focus_attn_prefill use its fastest kernels for these
  * arguments; 0 when none helps. Host only, no CUDA call; 0 also for arguments that
  * focus_attn_prefill would reject. Today only the rotary embedding
- * (cache->rope_theta > 0) on short work items (the persistent kernel's case,
- * below) asks for one: 256 bytes of per-head counters plus a rotated copy of the
- * span's q and k, B x H x (q_per_kv + 1) x T_span x d bf16. With it, the q and k
- * rows are each rotated once, by otherwise idle warps of the attention kernel
- * itself, a head ahead of their use; without it (NULL, or fewer bytes) the call
- * still succeeds and every CTA rotates the tiles it loads. The contents need no
- * initialisation and are scratch afterwards; the caller owns the memory. */
+ * (cache->rope_theta > 0) asks for one: 256 bytes of per-head counters plus a
+ * rotated copy of the span's q and k, B x H x (q_per_kv + 1) x T_span x d bf16.
+ * With it, the q and k rows are each rotated once: by a pass of their own before
+ * the attention (HBM-bound; the attention then runs as without the embedding, on
+ * any kernel), or, for grouped-query heads (q_per_kv >= 2) on short work items
+ * (the persistent kernel's case), by otherwise idle warps of the persistent
+ * kernel itself, a head ahead of their use. Without it (NULL, or fewer bytes) the
+ * call still succeeds and every CTA of the one-CTA-per-item kernel rotates the
+ * tiles it loads. The contents need no initialisation and are scratch afterwards;
+ * the caller owns the memory. */
 size_t focus_prefill_workspace_size(const focus_cache* cache, const focus_prefill_args* args);
 
 /* Use the legacy mma.sync kernel instead of the tcgen05/TMEM kernel (kept as the
@@ -294,13 +297,18 @@ focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_ar
  *                                    bounds the ring rows a tile sees: the boundary plus one FOCUS
  *                                    row per k bases, 1 + ceil(max_rows / k_w); and the launch has at
  *                                    least 2,048 work items (tiles x query heads x sequences).
- * The persistent kernel also takes the rotary-embedding case when args carries
- * focus_prefill_workspace_size(cache, args) bytes of workspace.
- * Both tcgen05 kernels compute the same rows (within rounding order). */
+ * With the rotary embedding and focus_prefill_workspace_size(cache, args) bytes of
+ * workspace, the kernel is the one the same arguments take without the embedding,
+ * and FOCUS_PREFILL_KERNEL_ROTATION_PASS is or-ed into *kernel when a rotation
+ * pass runs before it (every case but grouped-query heads on the persistent
+ * kernel, which rotates q and k itself). Without the workspace the rotary
+ * embedding takes the one-CTA-per-item kernel.
+ * The tcgen05 kernels compute the same rows (within rounding order). */
 #define FOCUS_PREFILL_KERNEL_LEGACY 0
 #define FOCUS_PREFILL_KERNEL_PER_ITEM 1
 #define FOCUS_PREFILL_KERNEL_PERSISTENT 2
 #define FOCUS_PREFILL_KERNEL_KMER 3
+#define FOCUS_PREFILL_KERNEL_ROTATION_PASS 16
 focus_status focus_prefill_kernel(const focus_cache* cache, const focus_prefill_args* args, int32_t* kernel);
 
 /* ------------------------------------------------------------------------ */

@@ -90,9 +90,10 @@ __global__ void __launch_bounds__(32) compact_bulk_kernel(
 }
 
 // Bulk mode with the rotary embedding: ring K rows are stored rotated at their
-// position id p = sum_idx[r]. One thread owns one ring row and one pair of
-// 16-byte chunks (columns 8j.. and 8j + d/2..), forms the eight angles p theta_i
-// once (fp64) and applies them to every (sequence, head); V is copied as is.
+// position id p = sum_idx[r]. One thread owns one ring row, one pair of 16-byte
+// chunks (columns 8j.. and 8j + d/2..) and a group of four (sequence, head)
+// pairs: it forms the eight angles p theta_i (fp64 product, reduced) and applies
+// them to each pair of the group; V is copied as is.
 template <int D>
 __global__ void __launch_bounds__(256) compact_bulk_rope_kernel(
         uint4* __restrict__ ring_k, uint4* __restrict__ ring_v, const uint4* __restrict__ src_k,
@@ -106,8 +107,14 @@ __global__ void __launch_bounds__(256) compact_bulk_rope_kernel(
         if (blockIdx.x == 0 && threadIdx.x == 0) report(status, FOCUS_ERR_CAPACITY);
         return;
     }
-    for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < rows * HALF;
-         u += (int64_t)gridDim.x * blockDim.x) {
+    // work unit: (group of U (sequence, head) pairs, ring row, chunk pair), the
+    // group outermost, so that a warp covers whole ring rows of one group and the
+    // launch has rows x d/16 x ceil(BH / U) threads' worth of units
+    constexpr int U = 4;
+    const int64_t units = rows * HALF, n_groups = (BH + U - 1) / U;
+    for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < units * n_groups;
+         x += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t grp = x / units, u = x - grp * units;
         const int j = (int)(u % HALF);
         const int64_t r = r0 + u / HALF;
         const int64_t p = sum_idx[r];
@@ -119,14 +126,36 @@ __global__ void __launch_bounds__(256) compact_bulk_rope_kernel(
         float2 cs[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) cs[e] = rope_cs((double)p * rope.theta[8 * j + e]);
-        for (int64_t bh = 0; bh < BH; ++bh) {
-            const int64_t so = (bh * src_T + srow) * CPR, d_o = (bh * C_ring + r) * CPR;
-            uint4 lo = src_k[so + j], hi = src_k[so + j + HALF];
-            rope_rotate8(lo, hi, cs);
-            ring_k[d_o + j] = lo;
-            ring_k[d_o + j + HALF] = hi;
-            ring_v[d_o + j] = src_v[so + j];
-            ring_v[d_o + j + HALF] = src_v[so + j + HALF];
+        const int64_t bh0 = grp * U;
+        if (bh0 + U <= BH) {                     // U rows' loads in flight
+            uint4 klo[U], khi[U], vlo[U], vhi[U];
+#pragma unroll
+            for (int e = 0; e < U; ++e) {
+                const int64_t so = ((bh0 + e) * src_T + srow) * CPR;
+                klo[e] = src_k[so + j];
+                khi[e] = src_k[so + j + HALF];
+                vlo[e] = src_v[so + j];
+                vhi[e] = src_v[so + j + HALF];
+            }
+#pragma unroll
+            for (int e = 0; e < U; ++e) {
+                const int64_t d_o = ((bh0 + e) * C_ring + r) * CPR;
+                rope_rotate8(klo[e], khi[e], cs);
+                ring_k[d_o + j] = klo[e];
+                ring_k[d_o + j + HALF] = khi[e];
+                ring_v[d_o + j] = vlo[e];
+                ring_v[d_o + j + HALF] = vhi[e];
+            }
+        } else {
+            for (int64_t bh = bh0; bh < BH; ++bh) {
+                const int64_t so = (bh * src_T + srow) * CPR, d_o = (bh * C_ring + r) * CPR;
+                uint4 lo = src_k[so + j], hi = src_k[so + j + HALF];
+                rope_rotate8(lo, hi, cs);
+                ring_k[d_o + j] = lo;
+                ring_k[d_o + j + HALF] = hi;
+                ring_v[d_o + j] = src_v[so + j];
+                ring_v[d_o + j + HALF] = src_v[so + j + HALF];
+            }
         }
     }
     if (blockIdx.x == 0)

@@ -248,8 +248,9 @@ __device__ __forceinline__ void rope_offsets(const double* theta, int i0, int g,
 // (a multiple of 8, <= 128; a tile's 128 rows by default), 128-byte swizzle.
 cudaError_t make_map(CUtensorMap* m, const void* ptr, int d, int64_t rows, int64_t bh, int box_rows = 128);
 
-// The persistent kernel (appendix mask). With the rotary embedding it needs the
-// caller's workspace (persistent_workspace_bytes) for the rotated Q and K rows.
+// The persistent kernel (appendix mask). With the rotary embedding (grouped-query
+// heads) it rotates Q and K itself, into the caller's workspace
+// (persistent_workspace_bytes).
 cudaError_t launch_prefill_tc_persistent(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
                                          cudaStream_t stream);
 // The k-mer-local kernel with query tiles cut at k-mer boundaries
@@ -259,9 +260,19 @@ bool kmer_tiling(const focus_cache& c, const focus_prefill_args& a, int32_t* RB,
 cudaError_t launch_prefill_tc_kmer(const focus_cache& c, const focus_prefill_args& a, int32_t* status,
                                    cudaStream_t stream);
 
-// Workspace bytes of the persistent kernel: 0 without the rotary embedding; with
-// it a 256-byte block of per-head counters, then Q and K of the span, rotated.
+// Workspace bytes for the rotary embedding (the persistent kernel's own rotation
+// and the pass share the layout): 0 without it; with it a 256-byte block of
+// per-head counters, then Q and K of the span, rotated.
 size_t persistent_workspace_bytes(const focus_cache& c, const focus_prefill_args& a);
+
+// Bytes of the per-head counters at the start of that workspace.
+size_t rope_counter_bytes(const focus_cache& c);
+
+// The rotary embedding as a pass before the attention (rope.cu): writes the span's
+// rotated q rows to q_rot ([B][H g][T_span][d] bf16) and its k rows to k_rot
+// ([B][H][T_span][d]).
+cudaError_t launch_rope_rotate(const focus_cache& c, const focus_prefill_args& a, void* q_rot, void* k_rot,
+                               cudaStream_t stream);
 
 }  // namespace prefill
 }  // namespace focus

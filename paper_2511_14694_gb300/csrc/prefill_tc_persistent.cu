@@ -16,9 +16,11 @@
 //   warp 1     MMA issuer: per item as in prefill_tc.cu, but with one stage wait
 //              and one stage release per iteration; an item's first PV into O_t
 //              waits until the previous item's epilogue has read O_t (o_free)
-//   warps 2-3  idle; with the rotary embedding (ROPE) they rotate the span's Q
-//              and K rows once, into a caller workspace that the Q/K tensor maps
-//              read (rotate_span below), one head ahead of the attention
+//   warps 2-3  idle; with the rotary embedding (ROPE, taken for grouped-query
+//              heads; otherwise rope.cu's pass rotates q and k before this kernel)
+//              they rotate the span's Q and K rows once, into a caller workspace
+//              that the Q/K tensor maps read (RopeSpan below), one head ahead of
+//              the attention
 //   warps 4-11 softmax per tile (the shared softmax_tile), then the epilogue:
 //              O_t / l to bf16 through a per-warp staging buffer (the Q buffers may
 //              already hold the next item's Q), arrive on o_free once O_t is read
@@ -599,12 +601,11 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_persistent_kernel(
 
 // Workspace layout (ROPE): int32 rot_done[B H] (padded to 256 bytes), then the
 // rotated Q [B][H g][T_span][d] and K [B][H][T_span][d], bf16.
-size_t rope_counter_bytes(const focus_cache& c) { return ((size_t)c.B * c.H * 4 + 255) & ~(size_t)255; }
 
 // K/V heads rotated in the kernel's prologue by all warps (the rest by warps 2-3
-// beside the attention). One: at 128 kb, 32 heads, one head took 2.907 ms per
-// launch, 2 / 5 of the heads 2.97 ms and all of them (a rotation pass before the
-// attention, ~0.87 ms of it) 3.035 ms.
+// beside the attention). One: at 128 kb, 32 query heads of one K/V head each,
+// one head took 2.907 ms per launch, 2 / 5 of the heads 2.97 ms and all of them
+// 3.035 ms.
 int32_t rope_prologue_heads(int64_t BH) { return BH < 1 ? 0 : 1; }
 
 template <int D, bool GQA, bool ROPE>
@@ -676,6 +677,8 @@ cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t*
 }
 
 }  // namespace
+
+size_t rope_counter_bytes(const focus_cache& c) { return ((size_t)c.B * c.H * 4 + 255) & ~(size_t)255; }
 
 size_t persistent_workspace_bytes(const focus_cache& c, const focus_prefill_args& a) {
     if (!(c.rope_theta > 0.f)) return 0;

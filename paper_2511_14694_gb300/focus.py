@@ -441,12 +441,14 @@ def prefill_host(cache: Cache, L: dict, host: dict, dev: dict, copy_in, copy_out
 
 PREFILL_KERNELS = {0: "legacy mma.sync", 1: "tcgen05, one CTA per work item", 2: "tcgen05 persistent",
                    3: "tcgen05 k-mer tiles"}
+PREFILL_KERNEL_ROTATION_PASS = 16
 
 
 def prefill_kernel(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | None = None, flags: int = 0,
                    o=None, workspace="auto", host_schedule: bool = True) -> str:
     """Name of the kernel focus_attn_prefill would launch for these arguments
-    (focus_prefill_kernel: host only, nothing runs on the device). ``workspace``
+    (focus_prefill_kernel: host only, nothing runs on the device), prefixed with
+    "rotation pass + " when a rotary-embedding pass runs before it. ``workspace``
     as for attn_prefill; "auto" assumes the workspace attn_prefill would allocate."""
     lib = load()
     w_end = L["M"] if w_end is None else w_end
@@ -460,7 +462,8 @@ def prefill_kernel(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int 
     out = ctypes.c_int32()
     _check("focus_prefill_kernel", lib.focus_prefill_kernel(ctypes.byref(cache.desc), ctypes.byref(a),
                                                            ctypes.byref(out)))
-    return PREFILL_KERNELS[out.value]
+    name = PREFILL_KERNELS[out.value & ~PREFILL_KERNEL_ROTATION_PASS]
+    return "rotation pass + " + name if out.value & PREFILL_KERNEL_ROTATION_PASS else name
 
 
 def embed_tokens(tok, table, out=None, stream=None):

@@ -171,20 +171,36 @@ def test_prefill_kernel_choice_needs_no_gpu():
     a.h_k_per_window = None
     c.rope_theta = 10_000.0
     assert choice(1_280, 1_010) == (0, 1)            # rotary embedding without a workspace
-    # with the workspace focus_prefill_workspace_size asks for: the persistent kernel,
-    # which rotates q and k once into it (counters + rotated q and k of the span)
+    # with the workspace focus_prefill_workspace_size asks for (per-head counters,
+    # then the span's q and k, rotated there by a pass): the kernel the arguments
+    # take without the embedding
     c.C_ring, a.max_rows, a.flags = 1_280, 1_010, 0
     need = lib.focus_prefill_workspace_size(ctypes.byref(c), ctypes.byref(a))
     assert need == 256 + c.B * c.H * 2 * a.T_span * c.d * 2
     a.workspace, a.workspace_bytes = 4096, need
-    assert choice(1_280, 1_010) == (0, 2)
+    rp = focus.PREFILL_KERNEL_ROTATION_PASS
+    assert choice(1_280, 1_010) == (0, rp | 2)
     a.workspace_bytes = need - 1
-    assert choice(1_280, 1_010) == (0, 1)            # too small: the per-item kernel
+    assert choice(1_280, 1_010) == (0, 1)            # too small: the per-item kernel rotating its tiles
     a.workspace, a.workspace_bytes = 4100, need
     assert choice(1_280, 1_010)[0] == 2              # misaligned workspace
     a.workspace, a.workspace_bytes = 4096, need
-    assert choice(10_000, 1_010) == (0, 1)           # long items: no workspace wanted
-    assert lib.focus_prefill_workspace_size(ctypes.byref(c), ctypes.byref(a)) == 0
+    assert choice(10_000, 1_010) == (0, rp | 1)      # long items: the per-item kernel, on the rotated rows
+    assert lib.focus_prefill_workspace_size(ctypes.byref(c), ctypes.byref(a)) == need
+    a.h_k_per_window = ks.ctypes.data
+    assert choice(1_280, 1_010, focus.PREFILL_KMER_LOCAL) == (0, rp | 3)  # k-mer tiles on the rotated rows
+    a.workspace_bytes = need - 1
+    assert choice(1_280, 1_010, focus.PREFILL_KMER_LOCAL) == (0, 1)
+    a.h_k_per_window = None
+    # grouped-query heads on short items: the persistent kernel rotates into the
+    # workspace itself (counters + q of the 4 query heads and k of each K/V head)
+    c.q_per_kv = 4
+    need4 = lib.focus_prefill_workspace_size(ctypes.byref(c), ctypes.byref(a))
+    assert need4 == 256 + c.B * c.H * 5 * a.T_span * c.d * 2
+    a.workspace_bytes = need4
+    assert choice(1_280, 1_010) == (0, 2)            # no pass: the persistent kernel rotates
+    assert choice(10_000, 1_010) == (0, rp | 1)
+    c.q_per_kv = 1
     a.workspace, a.workspace_bytes = None, 0
     assert choice(1_280, 1_010, focus.PREFILL_LEGACY_MMA)[0] == 2      # legacy has no rotary embedding
     c.rope_theta = 0.0

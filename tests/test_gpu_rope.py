@@ -71,10 +71,10 @@ ROPE_CASES = [
 ]
 
 
-# with the workspace the persistent kernel rotates q and k once (warps 2-3 of
-# every CTA, a head ahead of the attention); without it the one-CTA-per-item
-# kernel rotates each tile it loads
-@pytest.mark.parametrize("ws,kernel", [("auto", "tcgen05 persistent"), (None, "tcgen05, one CTA per work item")])
+# with the workspace a pass rotates q and k once before the attention; without it
+# the one-CTA-per-item kernel rotates each tile it loads
+@pytest.mark.parametrize("ws,kernel", [("auto", "rotation pass + tcgen05 persistent"),
+                                       (None, "tcgen05, one CTA per work item")])
 @pytest.mark.parametrize("N,W,ks,B,H,d,theta", ROPE_CASES)
 def test_prefill_rope_masked_parallel_matches_oracle(N, W, ks, B, H, d, theta, ws, kernel):
     L, k, q, kk, v, cache = _case(N, W, ks, B, H, d, theta, seed=N + 3)
