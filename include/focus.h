@@ -233,8 +233,9 @@ typedef struct focus_prefill_args {
 /* Device workspace that lets focus_attn_prefill use its fastest kernels for these
  * arguments; 0 when none helps. Host only, no CUDA call; 0 also for arguments that
  * focus_attn_prefill would reject. Today only the rotary embedding
- * (cache->rope_theta > 0) asks for one: 256 bytes of per-head counters plus a
- * rotated copy of the span's q and k, B x H x (q_per_kv + 1) x T_span x d bf16.
+ * (cache->rope_theta > 0), outside the k-mer-tiled kernel's case (which rotates
+ * in place), asks for one: 256 bytes of per-head counters plus a rotated copy of
+ * the span's q and k, B x H x (q_per_kv + 1) x T_span x d bf16.
  * With it, the q and k rows are each rotated once: by a pass of their own before
  * the attention (HBM-bound; the attention then runs as without the embedding, on
  * any kernel), or, for grouped-query heads (q_per_kv >= 2) on short work items
@@ -291,18 +292,19 @@ focus_status focus_attn_prefill(const focus_cache* cache, const focus_prefill_ar
  *   FOCUS_PREFILL_KERNEL_KMER        the FOCUS_PREFILL_KMER_LOCAL mode with query tiles cut at
  *                                    k-mer boundaries (one CTA per SM walking them): each tile's
  *                                    keys, its k-mers' rows plus the few ring rows they see, fit one
- *                                    128-row K/V tile. Taken when args->h_k_per_window is given, no
- *                                    rotary embedding is on, and over the span's windows every k-mer
+ *                                    128-row K/V tile. Taken when args->h_k_per_window is given and
+ *                                    over the span's windows every k-mer
  *                                    has at most 128 - RB rows, where RB (a multiple of 8, <= 64)
  *                                    bounds the ring rows a tile sees: the boundary plus one FOCUS
  *                                    row per k bases, 1 + ceil(max_rows / k_w); and the launch has at
  *                                    least 2,048 work items (tiles x query heads x sequences).
- * With the rotary embedding and focus_prefill_workspace_size(cache, args) bytes of
- * workspace, the kernel is the one the same arguments take without the embedding,
- * and FOCUS_PREFILL_KERNEL_ROTATION_PASS is or-ed into *kernel when a rotation
- * pass runs before it (every case but grouped-query heads on the persistent
- * kernel, which rotates q and k itself). Without the workspace the rotary
- * embedding takes the one-CTA-per-item kernel.
+ * With the rotary embedding the k-mer-tiled kernel rotates its tiles in place
+ * (no workspace). Otherwise, with focus_prefill_workspace_size(cache, args) bytes
+ * of workspace, the kernel is the one the same arguments take without the
+ * embedding, and FOCUS_PREFILL_KERNEL_ROTATION_PASS is or-ed into *kernel when a
+ * rotation pass runs before it (every case but grouped-query heads on the
+ * persistent kernel, which rotates q and k itself); without the workspace the
+ * rotary embedding takes the one-CTA-per-item kernel.
  * The tcgen05 kernels compute the same rows (within rounding order). */
 #define FOCUS_PREFILL_KERNEL_LEGACY 0
 #define FOCUS_PREFILL_KERNEL_PER_ITEM 1

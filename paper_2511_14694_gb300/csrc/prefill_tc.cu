@@ -569,10 +569,11 @@ namespace {
 //   every angle, and there are fewer K rows to rotate, so the rotation keeps ahead
 //   of the attention: 128 kb with g = 2, 2.34 ms against 2.61 ms with the pass);
 // - otherwise a pass rotates them there first and the attention runs as without
-//   the embedding, on any kernel (128 kb with g = 1: 2.79 ms against 2.99 ms with
-//   the rotation inside the persistent kernel).
-// Without the workspace, the one-CTA-per-item kernel rotates the tiles each CTA
-// loads.
+//   the embedding (128 kb with g = 1: 2.79 ms against 2.99 ms with the rotation
+//   inside the persistent kernel);
+// except for the k-mer-tiled kernel, which rotates its tiles in place and needs no
+// workspace. Without the workspace, the one-CTA-per-item kernel rotates the
+// tiles each CTA loads.
 constexpr int32_t kRopeFusedMinGroup = 2;
 
 bool rope_workspace_ok(const focus_cache& c, const focus_prefill_args& a) {
@@ -584,14 +585,22 @@ bool rope_fused(const focus_cache& c, const focus_prefill_args& a) {
     return rope_workspace_ok(c, a) && c.q_per_kv >= kRopeFusedMinGroup && prefill_persistent_case(c, a);
 }
 
-bool rope_pass(const focus_cache& c, const focus_prefill_args& a) { return rope_workspace_ok(c, a) && !rope_fused(c, a); }
+// The k-mer-tiled kernel (which rotates q and k in place itself: it reads each
+// window row in one work item per query head).
+bool kmer_case(const focus_cache& c, const focus_prefill_args& a) {
+    int32_t RB, tiles;
+    return !(a.flags & FOCUS_PREFILL_LEGACY_MMA) && (a.flags & FOCUS_PREFILL_KMER_LOCAL) &&
+           prefill::kmer_tiling(c, a, &RB, &tiles);
+}
+
+bool rope_pass(const focus_cache& c, const focus_prefill_args& a) {
+    return rope_workspace_ok(c, a) && !rope_fused(c, a) && !kmer_case(c, a);
+}
 
 int32_t prefill_kernel_choice_plain(const focus_cache& c, const focus_prefill_args& a) {
     if (a.flags & FOCUS_PREFILL_LEGACY_MMA) return FOCUS_PREFILL_KERNEL_LEGACY;
     const bool rope = c.rope_theta > 0.f;
-    int32_t RB, tiles;
-    if ((a.flags & FOCUS_PREFILL_KMER_LOCAL) && !rope && prefill::kmer_tiling(c, a, &RB, &tiles))
-        return FOCUS_PREFILL_KERNEL_KMER;
+    if (kmer_case(c, a)) return FOCUS_PREFILL_KERNEL_KMER;
     if ((!rope || rope_fused(c, a)) && prefill_persistent_case(c, a)) return FOCUS_PREFILL_KERNEL_PERSISTENT;
     return FOCUS_PREFILL_KERNEL_PER_ITEM;
 }
@@ -608,7 +617,7 @@ int32_t prefill_kernel_choice(const focus_cache& c, const focus_prefill_args& a)
 }
 
 size_t prefill_workspace_bytes(const focus_cache& c, const focus_prefill_args& a) {
-    return (a.flags & FOCUS_PREFILL_LEGACY_MMA) ? 0 : prefill::persistent_workspace_bytes(c, a);
+    return (a.flags & FOCUS_PREFILL_LEGACY_MMA) || kmer_case(c, a) ? 0 : prefill::persistent_workspace_bytes(c, a);
 }
 
 namespace {

@@ -26,7 +26,14 @@
 //   warp 0     TMA producer: item i's Q and K once slot t's previous QK has
 //              completed, its V once that item's PV has completed
 //   warp 1     TMEM owner + MMA issuer: QK of item i, then PV of item i - 1
-//   warps 2-3  idle
+//   warps 2-3  idle; with the rotary embedding (ROPE) they rotate each item's Q
+//              tile and the window rows of its K tile in shared memory, between
+//              their TMA arrival and the item's QK (q and k rows are each read by
+//              one item per query head here, so the rotation adds no HBM traffic;
+//              the ring rows arrive rotated). A window row's position is
+//              win_off[w] + its in-window row, and the K tile's window rows start
+//              at the Q tile's first row, so Q row m and K row RB + m share every
+//              angle.
 //   warps 4-7 / 8-11  softmax + epilogue of the items of slot 0 / slot 1
 // Every mbarrier wait is bounded; on timeout the kernel reports
 // FOCUS_ERR_TIMEOUT, drains its own copies/MMAs (bounded), frees TMEM, returns.
@@ -36,10 +43,16 @@ namespace focus {
 namespace prefill {
 namespace {
 
-constexpr int kRegsIssue = 72, kRegsSoftmax = 216;
+// register split: warpgroup 0 (TMA, MMA and, with the rotary embedding, the
+// rotating warps 2-3) and the two softmax warpgroups
+template <bool ROPE>
+constexpr int kRegsIssue = ROPE ? 152 : 72;
+template <bool ROPE>
+constexpr int kRegsSoftmax = ROPE ? 176 : 216;
 constexpr int64_t kKmerMaxRingRows = 64;   // ring rows a tile may hold (the window box keeps >= 64 rows)
 constexpr int64_t kKmerMinItems = 2048;    // work items a launch needs for this kernel (~13 per SM)
-static_assert(128 * kRegsIssue + 256 * kRegsSoftmax <= kThreads * kLaunchRegs, "register split over budget");
+static_assert(128 * kRegsIssue<false> + 256 * kRegsSoftmax<false> <= kThreads * kLaunchRegs, "register split over budget");
+static_assert(128 * kRegsIssue<true> + 256 * kRegsSoftmax<true> <= kThreads * kLaunchRegs, "register split over budget");
 
 struct KBars {
     uint64_t ld_qk[2];   // Q and K of the slot's item landed
@@ -50,6 +63,7 @@ struct KBars {
     uint64_t p_full[2];
     uint64_t o_full[2];
     uint64_t o_free[2];  // the epilogue has read O_t
+    uint64_t rot[2];     // ROPE: the slot's Q tile and K window rows are rotated
     uint64_t drain;
     uint32_t tmem;
     int32_t abort;
@@ -64,7 +78,8 @@ struct KCfg {
     static constexpr int kVOff = 4 * kTile;          // V_0, V_1
     static constexpr int kBarOff = 6 * kTile;
     static constexpr int kStageOff = kBarOff + 256;  // O staging: 8 warps x 32 rows x 64 B
-    static constexpr int kSmem = kStageOff + 8 * 2048 + 1024;
+    static constexpr int kRopeOff = kStageOff + 8 * 2048;  // ROPE: the item's start angles, 64 x float2
+    static constexpr int kSmem = kRopeOff + 512 + 1024;
 };
 
 // Position in the item space (sequence b, K/V head h, window w, query tile,
@@ -112,14 +127,27 @@ struct KCursor {
     __device__ __forceinline__ int32_t rows() const { return nq < Tw - tile * nq ? nq : Tw - tile * nq; }
 };
 
-template <int D, bool GQA>
+// Barrier `id` over `count` threads that also ORs a predicate over them: every
+// participating thread gets the same result.
+__device__ __forceinline__ bool named_bar_or(uint32_t id, uint32_t count, bool pred) {
+    uint32_t r;
+    asm volatile(
+        "{\n .reg .pred p, q;\n setp.ne.u32 q, %1, 0;\n bar.red.or.pred p, %2, %3, q;\n selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(r)
+        : "r"((uint32_t)pred), "r"(id), "r"(count)
+        : "memory");
+    return r != 0;
+}
+
+template <int D, bool GQA, bool ROPE>
 __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kmer_kernel(
         const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kw,
         const __grid_constant__ CUtensorMap tm_vw, const __grid_constant__ CUtensorMap tm_rk,
         const __grid_constant__ CUtensorMap tm_rv, __nv_bfloat16* __restrict__ o, float* __restrict__ lse,
         int64_t T_span, const int32_t* __restrict__ win_off, const int32_t* __restrict__ ring_off,
         const int32_t* __restrict__ k_per_window, int32_t w_begin, int32_t w_end, int32_t max_tiles, int32_t RB,
-        int32_t H, int32_t C_ring, float scale_log2, int32_t* status, int32_t q_per_kv, int64_t n_items) {
+        int32_t H, int32_t C_ring, float scale_log2, int32_t* status, int32_t q_per_kv, int64_t n_items,
+        const __grid_constant__ RopeArg<ROPE> rope) {
     using C = KCfg<D>;
     extern __shared__ unsigned char smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -168,6 +196,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kmer_kernel(
             mbar_init(smem_addr(&bars->p_full[t]), BM);
             mbar_init(smem_addr(&bars->o_full[t]), 1);
             mbar_init(smem_addr(&bars->o_free[t]), BM);
+            mbar_init(smem_addr(&bars->rot[t]), 1);
         }
         mbar_init(smem_addr(&bars->drain), 1);
         bars->abort = 0;
@@ -188,7 +217,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kmer_kernel(
     auto aborted_k = [&]() { return *(volatile int32_t*)&bars->abort != 0; };
 
     if (warp < 4) {
-        setmaxnreg_dec<kRegsIssue>();
+        setmaxnreg_dec<kRegsIssue<ROPE>>();
         if (warp == 0 && lane == 0) {
             // ============================================= TMA producer
             prefetch_tmap(&tm_q);
@@ -260,7 +289,8 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kmer_kernel(
                 if (!I.valid()) continue;
                 const int t = (int)(i & 1);
                 const int64_t u = i >> 1;
-                if (!mbar_wait(smem_addr(&bars->ld_qk[t]), (uint32_t)(u & 1), kWaitNs)) {
+                // Q and K landed (and, with the rotary embedding, are rotated)
+                if (!mbar_wait(smem_addr(ROPE ? &bars->rot[t] : &bars->ld_qk[t]), (uint32_t)(u & 1), kWaitNs)) {
                     ok = false;
                     break;
                 }
@@ -279,10 +309,70 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kmer_kernel(
             if (!ok) fail_k();
             mma_commit(smem_addr(&bars->drain));
             mbar_wait(smem_addr(&bars->drain), 0, kWaitNs);
+        } else if (ROPE && (warp == 2 || warp == 3)) {
+            // ============================================= rotary embedding (warps 2-3)
+            if constexpr (ROPE) {
+                // thread tau owns pair chunk jj (columns 8 jj .. and D/2 + 8 jj ..) of
+                // rows g, g + G, ... of the item's Q tile and of its K tile's window rows
+                constexpr int HALF = D / 16, G = 64 / HALF;
+                const int tau = threadIdx.x - 64, jj = tau % HALF, gg = tau / HALF;
+                float2* kb = reinterpret_cast<float2*>(smem + C::kRopeOff);
+                float2 off[8];
+                Rot8 step;
+                rope_offsets(rope.t.theta, 8 * jj, gg, G, off, step);
+                const double theta_own = tau < D / 2 ? rope.t.theta[tau] : 0.0;
+                const int64_t w0 = win_off[w_begin];
+                const int clo = 8 * jj, chi = 8 * jj + D / 2;
+                int64_t i = 0;
+                KCursor I = start(false);
+                for (int64_t idx = i0; idx < i1; ++idx, advance(I, false)) {
+                    if (!I.valid()) continue;
+                    const int t = (int)(i & 1);
+                    const int64_t u = i >> 1;
+                    ++i;
+                    const bool landed = mbar_wait(smem_addr(&bars->ld_qk[t]), (uint32_t)(u & 1), kWaitNs);
+                    // position of the tile's first row; the item's start angles
+                    if (landed && tau < D / 2) kb[tau] = rope_cs((double)(w0 + I.row_base + I.s()) * theta_own);
+                    // one decision for all 64 threads: a bounded wait may give up in some only
+                    if (named_bar_or(1, 64, !landed || aborted_k())) {
+                        if (!landed) fail_k();
+                        break;
+                    }
+                    float2 cs[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) cs[e] = rope_mul(kb[8 * jj + e], off[e]);
+                    Rot8 rot = rot8_make(cs);
+                    uint8_t* qt = smem + C::kQOff + t * C::kTile;
+                    uint8_t* kt = smem + C::kKOff + t * C::kTile;
+#pragma unroll 1
+                    for (int m = gg; m < 128 - RB; m += G) {
+                        const int rk = RB + m;
+                        uint4* qlo = reinterpret_cast<uint4*>(qt + (clo / 64) * kBoxBytes + m * 128 +
+                                                              ((((clo % 64) / 8) ^ (m & 7)) << 4));
+                        uint4* qhi = reinterpret_cast<uint4*>(qt + (chi / 64) * kBoxBytes + m * 128 +
+                                                              ((((chi % 64) / 8) ^ (m & 7)) << 4));
+                        uint4* klo = reinterpret_cast<uint4*>(kt + (clo / 64) * kBoxBytes + rk * 128 +
+                                                              ((((clo % 64) / 8) ^ (rk & 7)) << 4));
+                        uint4* khi = reinterpret_cast<uint4*>(kt + (chi / 64) * kBoxBytes + rk * 128 +
+                                                              ((((chi % 64) / 8) ^ (rk & 7)) << 4));
+                        uint4 a = *qlo, b = *qhi, c = *klo, d = *khi;
+                        rot8_apply(a, b, rot);
+                        rot8_apply(c, d, rot);
+                        *qlo = a;
+                        *qhi = b;
+                        *klo = c;
+                        *khi = d;
+                        rot8_step(rot, step);
+                    }
+                    fence_proxy_async_smem();             // the MMA reads these rows through the async proxy
+                    named_bar_sync(1, 64);                 // every row rotated; kb free for the next item
+                    if (tau == 0) mbar_arrive(smem_addr(&bars->rot[t]));
+                }
+            }
         }
     } else {
         // ================================================= softmax / epilogue
-        setmaxnreg_inc<kRegsSoftmax>();
+        setmaxnreg_inc<kRegsSoftmax<ROPE>>();
         const int t = (warp - 4) >> 2;                    // slot of this warpgroup
         const int quarter = warp & 3;
         const int r = quarter * 32 + lane;                // row within the Q tile
@@ -376,7 +466,7 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kmer_kernel(
     }
 }
 
-template <int D, bool GQA>
+template <int D, bool GQA, bool ROPE>
 cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t RB, int32_t max_tiles,
                      int32_t* status, cudaStream_t stream) {
     const int64_t BH = (int64_t)c.B * c.H;
@@ -394,7 +484,7 @@ cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t 
         if ((e = make_map(&trv, a.v, D, a.T_span, BH, RB)) != cudaSuccess) return e;
     }
     const int smem = KCfg<D>::kSmem;
-    auto* kernel = prefill_tc_kmer_kernel<D, GQA>;
+    auto* kernel = prefill_tc_kmer_kernel<D, GQA, ROPE>;
     if ((e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
         return e;
     cudaFuncAttributes fa;
@@ -405,10 +495,13 @@ cudaError_t launch_d(const focus_cache& c, const focus_prefill_args& a, int32_t 
     if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
     const int64_t n_items = (int64_t)(a.w_end - a.w_begin) * max_tiles * g * c.H * c.B;
     const dim3 grid((unsigned)(n_items < sms ? n_items : sms));
+    RopeArg<ROPE> rope;
+    if constexpr (ROPE) rope_table_fill(&rope.t, D, c.rope_theta);
+    else rope.unused = 0;
     kernel<<<grid, kThreads, smem, stream>>>(tq, tkw, tvw, trk, trv, (__nv_bfloat16*)a.o, a.lse, a.T_span,
                                              a.d_win_off, a.d_ring_off, c.k_per_window, a.w_begin, a.w_end,
                                              max_tiles, RB, c.H, c.C_ring, a.scale * 1.4426950408889634f, status, g,
-                                             n_items);
+                                             n_items, rope);
     return cudaGetLastError();
 }
 
@@ -454,12 +547,19 @@ cudaError_t launch_prefill_tc_kmer(const focus_cache& c, const focus_prefill_arg
                                    cudaStream_t stream) {
     int32_t RB = 0, max_tiles = 0;
     if (!kmer_tiling(c, a, &RB, &max_tiles)) return cudaErrorInvalidValue;
-    const bool gqa = c.q_per_kv > 1;
-    if (c.d == 128)
-        return gqa ? launch_d<128, true>(c, a, RB, max_tiles, status, stream)
-                   : launch_d<128, false>(c, a, RB, max_tiles, status, stream);
-    return gqa ? launch_d<64, true>(c, a, RB, max_tiles, status, stream)
-               : launch_d<64, false>(c, a, RB, max_tiles, status, stream);
+    const bool gqa = c.q_per_kv > 1, rope = c.rope_theta > 0.f;
+    if (c.d == 128) {
+        if (rope)
+            return gqa ? launch_d<128, true, true>(c, a, RB, max_tiles, status, stream)
+                       : launch_d<128, false, true>(c, a, RB, max_tiles, status, stream);
+        return gqa ? launch_d<128, true, false>(c, a, RB, max_tiles, status, stream)
+                   : launch_d<128, false, false>(c, a, RB, max_tiles, status, stream);
+    }
+    if (rope)
+        return gqa ? launch_d<64, true, true>(c, a, RB, max_tiles, status, stream)
+                   : launch_d<64, false, true>(c, a, RB, max_tiles, status, stream);
+    return gqa ? launch_d<64, true, false>(c, a, RB, max_tiles, status, stream)
+               : launch_d<64, false, false>(c, a, RB, max_tiles, status, stream);
 }
 
 }  // namespace prefill

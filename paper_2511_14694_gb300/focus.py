@@ -352,18 +352,19 @@ def _prefill_args(q, k, v, o, lse, L: dict, w_begin: int, w_end: int, scale: flo
 
 
 def prefill_workspace_bytes(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | None = None,
-                            flags: int = 0) -> int:
+                            flags: int = 0, host_schedule: bool = True) -> int:
     """focus_prefill_workspace_size: device workspace bytes that let these
     arguments use the fastest kernel (0: none needed)."""
     w_end = L["M"] if w_end is None else w_end
-    a = _prefill_args(q, k, v, q, None, L, w_begin, w_end, 1.0 / math.sqrt(q.shape[3]), flags)
+    a = _prefill_args(q, k, v, q, None, L, w_begin, w_end, 1.0 / math.sqrt(q.shape[3]), flags,
+                      host_schedule=host_schedule)
     return int(load().focus_prefill_workspace_size(ctypes.byref(cache.desc), ctypes.byref(a)))
 
 
 def new_prefill_workspace(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | None = None,
-                          flags: int = 0):
+                          flags: int = 0, host_schedule: bool = True):
     """A device buffer of prefill_workspace_bytes (None when none is needed)."""
-    n = prefill_workspace_bytes(cache, q, k, v, L, w_begin, w_end, flags)
+    n = prefill_workspace_bytes(cache, q, k, v, L, w_begin, w_end, flags, host_schedule)
     return None if n == 0 else torch.empty(n, dtype=torch.uint8, device=q.device)
 
 
@@ -387,7 +388,7 @@ def attn_prefill(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int | 
         lse = torch.empty((B, H, T_span), dtype=torch.float32, device=q.device)
     scale = 1.0 / math.sqrt(d) if scale is None else float(scale)
     if isinstance(workspace, str):
-        workspace = new_prefill_workspace(cache, q, k, v, L, w_begin, w_end, flags)
+        workspace = new_prefill_workspace(cache, q, k, v, L, w_begin, w_end, flags, host_schedule)
         if workspace is not None and stream is not None:
             # allocated on the current stream, used on `stream`: keep the caching
             # allocator from reusing it before the launch there is done
@@ -455,7 +456,7 @@ def prefill_kernel(cache: Cache, q, k, v, L: dict, w_begin: int = 0, w_end: int 
     a = _prefill_args(q, k, v, q if o is None else o, None, L, w_begin, w_end, 1.0 / math.sqrt(q.shape[3]), flags,
                       host_schedule=host_schedule)
     if isinstance(workspace, str):
-        a.workspace_bytes = prefill_workspace_bytes(cache, q, k, v, L, w_begin, w_end, flags)
+        a.workspace_bytes = prefill_workspace_bytes(cache, q, k, v, L, w_begin, w_end, flags, host_schedule)
         a.workspace = 16 if a.workspace_bytes else None        # a placeholder address: nothing is launched
     elif workspace is not None:
         a.workspace, a.workspace_bytes = _ptr(workspace), workspace.numel() * workspace.element_size()

@@ -188,9 +188,13 @@ def test_prefill_kernel_choice_needs_no_gpu():
     assert choice(10_000, 1_010) == (0, rp | 1)      # long items: the per-item kernel, on the rotated rows
     assert lib.focus_prefill_workspace_size(ctypes.byref(c), ctypes.byref(a)) == need
     a.h_k_per_window = ks.ctypes.data
-    assert choice(1_280, 1_010, focus.PREFILL_KMER_LOCAL) == (0, rp | 3)  # k-mer tiles on the rotated rows
-    a.workspace_bytes = need - 1
-    assert choice(1_280, 1_010, focus.PREFILL_KMER_LOCAL) == (0, 1)
+    # the k-mer-tiled kernel rotates its tiles in place: no pass, no workspace
+    assert choice(1_280, 1_010, focus.PREFILL_KMER_LOCAL) == (0, 3)
+    assert lib.focus_prefill_workspace_size(ctypes.byref(c), ctypes.byref(a)) == 0
+    a.workspace, a.workspace_bytes = None, 0
+    assert choice(1_280, 1_010, focus.PREFILL_KMER_LOCAL) == (0, 3)
+    a.flags = 0
+    a.workspace, a.workspace_bytes = 4096, need
     a.h_k_per_window = None
     # grouped-query heads on short items: the persistent kernel rotates into the
     # workspace itself (counters + q of the 4 query heads and k of each K/V head)

@@ -292,3 +292,38 @@ def test_full_size_streaming_rope_sampled():
             o_ref, lse_ref = fo.attn_rows_f64(qf[None], kf[None], vv[None], keep, win, 1.0 / math.sqrt(d),
                                               np.zeros(rows.size, np.int64), rows)
             assert_attn_close(got[w][0][i], got[w][1][i], o_ref, lse_ref, f"rope stream w={w} h={h}")
+
+
+@pytest.mark.parametrize("g,d,B,H", [(1, 128, 1, 16), (4, 64, 1, 4), (1, 64, 2, 8)])
+def test_prefill_rope_kmer_tiled_matches_oracle(g, d, B, H):
+    """The k-mer-local mask (Sec. 3.2) with the rotary embedding on the k-mer-tiled
+    kernel (17 windows x 10 tiles x 16 query heads per sequence: above its 2,048-item
+    threshold), which rotates each item's Q tile and the window rows of its K tile
+    in shared memory and needs no workspace; the ring rows come rotated from the
+    compaction. Every row against the oracle on the rows rotated at their positions
+    and rounded to bf16, including a ragged last window."""
+    N, W, k_, theta = 16_037, 1_000, 100, 500_000.0
+    k = np.full(-(-N // W), k_, np.int32)
+    L = focus.layout(N, W, k)
+    T = L["T"]
+    q = inputs.normal_bf16((B, H * g, T, d), 1.0, seed=91, device="cuda")
+    kk, v = (inputs.normal_bf16((B, H, T, d), 1.0, seed=s, device="cuda") for s in (92, 93))
+    cache = focus.Cache(B, H, d, C_ring=L["R"], k_sched=k, q_per_kv=g, rope_theta=theta)
+    fl = focus.PREFILL_KMER_LOCAL
+    assert focus.prefill_workspace_bytes(cache, q, kk, v, L, flags=fl) == 0
+    assert focus.prefill_kernel(cache, q, kk, v, L, flags=fl) == "tcgen05 k-mer tiles"
+    o, lse = pipeline.prefill_masked_parallel(cache, q, kk, v, L, flags=fl)
+    torch.cuda.synchronize()
+    ref = fo.layout(N, W, k)
+    Hq = H * g
+    pos = np.arange(T)
+    qf = fo.rope(q.reshape(B * Hq, T, d).cpu(), pos, theta, round_bf16=True)
+    kf = fo.rope(kk.reshape(B * H, T, d).cpu(), pos, theta, round_bf16=True)
+    kv_of = np.arange(B * Hq) // g                      # K/V head of each (sequence, query head)
+    to_bf16 = lambda x: torch.from_numpy(x.astype(np.float32)).bfloat16()  # noqa: E731 (exact: rounded rows)
+    heads, rows = np.repeat(np.arange(B * Hq), T), np.tile(np.arange(T), B * Hq)
+    o_ref, lse_ref = fo.attn_rows_kmer_local(to_bf16(qf), to_bf16(kf[kv_of]),
+                                             v.reshape(B * H, T, d).cpu()[torch.from_numpy(kv_of)],
+                                             ref["kind"], ref["win"], fo.layout_kmer(N, W, k), 1 / math.sqrt(d),
+                                             heads, rows)
+    assert_attn_close(o, lse, o_ref.reshape(B, Hq, T, d), lse_ref.reshape(B, Hq, T), f"rope k-mer tiles g={g} d={d}")
