@@ -344,8 +344,11 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kmer_kernel(
                     Rot8 rot = rot8_make(cs);
                     uint8_t* qt = smem + C::kQOff + t * C::kTile;
                     uint8_t* kt = smem + C::kKOff + t * C::kTile;
+                    // the item's query rows and the window keys they can see (its own
+                    // k-mers: window rows below s + rows)
+                    const int n_rows = I.rows();
 #pragma unroll 1
-                    for (int m = gg; m < 128 - RB; m += G) {
+                    for (int m = gg; m < n_rows; m += G) {
                         const int rk = RB + m;
                         uint4* qlo = reinterpret_cast<uint4*>(qt + (clo / 64) * kBoxBytes + m * 128 +
                                                               ((((clo % 64) / 8) ^ (m & 7)) << 4));
