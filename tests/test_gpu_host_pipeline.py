@@ -24,9 +24,16 @@ def _clean_status():
     assert focus.device_status(clear=True) == 0, "a kernel reported an error"
 
 
-@pytest.mark.parametrize("B,H,d,g,groups,rope", [(1, 4, 64, 1, 3, 0.0), (3, 2, 128, 1, 2, 0.0), (1, 2, 128, 2, 2, 0.0),
-                                                 (2, 2, 64, 1, 8, 0.0), (1, 4, 128, 1, 2, 10_000.0)])
-def test_host_pipeline_matches_device_path(B, H, d, g, groups, rope):
+@pytest.mark.parametrize("B,H,d,g,groups,rope,local", [(1, 4, 64, 1, 3, 0.0, False), (3, 2, 128, 1, 2, 0.0, False),
+                                                       (1, 2, 128, 2, 2, 0.0, False), (2, 2, 64, 1, 8, 0.0, False),
+                                                       (1, 4, 128, 1, 2, 10_000.0, False),
+                                                       (1, 4, 128, 2, 2, 10_000.0, False),
+                                                       (2, 2, 64, 1, 2, 0.0, True), (1, 4, 128, 1, 4, 10_000.0, True)])
+def test_host_pipeline_matches_device_path(B, H, d, g, groups, rope, local):
+    """The host-buffer entry point gives the device path's outputs and ring bit for
+    bit, with grouped heads, the rotary embedding (a pass per part, or the
+    persistent kernel rotating in place for grouped heads) and the k-mer-local
+    mask; the workspace sized for the whole cache serves every part in turn."""
     N, W = 5_000, 1_000
     k = inputs.k_schedule(-(-N // W), [100, 10, 50], seed=3)
     L_dev = focus.layout_alloc(N, W, k, B=B)
@@ -37,7 +44,8 @@ def test_host_pipeline_matches_device_path(B, H, d, g, groups, rope):
     # the device path
     focus.layout_run(L_dev, nt)
     c_dev = focus.Cache(B, H, d, C_ring=L_dev["R"], k_sched=k, q_per_kv=g, rope_theta=rope)
-    o_dev, lse_dev = pipeline.prefill_masked_parallel(c_dev, q, kk, v, L_dev)
+    fl = focus.PREFILL_KMER_LOCAL if local else 0
+    o_dev, lse_dev = pipeline.prefill_masked_parallel(c_dev, q, kk, v, L_dev, flags=fl)
     # the host path
     pin = lambda t: t.cpu().pin_memory()                                  # noqa: E731
     host = dict(nt=pin(nt), q=pin(q), k=pin(kk), v=pin(v), o=torch.empty(q.shape, dtype=torch.bfloat16).pin_memory(),
@@ -45,7 +53,7 @@ def test_host_pipeline_matches_device_path(B, H, d, g, groups, rope):
     dev = dict(nt=torch.empty_like(nt), q=torch.empty_like(q), k=torch.empty_like(kk), v=torch.empty_like(v),
                o=torch.empty_like(q), lse=torch.empty((B, H * g, T), dtype=torch.float32, device="cuda"))
     c_host = focus.Cache(B, H, d, C_ring=L_host["R"], k_sched=k, q_per_kv=g, rope_theta=rope)
-    pipeline.prefill_masked_parallel_host(c_host, L_host, host, dev, groups=groups)
+    pipeline.prefill_masked_parallel_host(c_host, L_host, host, dev, groups=groups, flags=fl)
     torch.cuda.synchronize()
     assert np.array_equal(bits(host["o"]), bits(o_dev))
     assert np.array_equal(host["lse"].numpy(), lse_dev.cpu().numpy())
