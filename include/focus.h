@@ -234,8 +234,9 @@ typedef struct focus_prefill_args {
  * arguments; 0 when none helps. Host only, no CUDA call; 0 also for arguments that
  * focus_attn_prefill would reject. Today only the rotary embedding
  * (cache->rope_theta > 0), outside the k-mer-tiled kernel's case (which rotates
- * in place), asks for one: 256 bytes of per-head counters plus a rotated copy of
- * the span's q and k, B x H x (q_per_kv + 1) x T_span x d bf16.
+ * in place), asks for one: 256 bytes of per-head counters (B x H int32, rounded up
+ * to 256 bytes) followed by a rotated copy of the span's q rows ([B][H q_per_kv]
+ * [T_span][d] bf16) and k rows ([B][H][T_span][d]).
  * With it, the q and k rows are each rotated once: by a pass of their own before
  * the attention (HBM-bound; the attention then runs as without the embedding, on
  * any kernel), or, for grouped-query heads (q_per_kv >= 2) on short work items

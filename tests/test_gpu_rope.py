@@ -327,3 +327,34 @@ def test_prefill_rope_kmer_tiled_matches_oracle(g, d, B, H):
                                              ref["kind"], ref["win"], fo.layout_kmer(N, W, k), 1 / math.sqrt(d),
                                              heads, rows)
     assert_attn_close(o, lse, o_ref.reshape(B, Hq, T, d), lse_ref.reshape(B, Hq, T), f"rope k-mer tiles g={g} d={d}")
+
+
+def test_rotation_pass_rows_match_oracle():
+    """The rotation pass on its own: after a call that takes it (one query head per
+    K/V head, a span of windows 2..4 so that positions start at win_off[2]), the
+    workspace holds the span's q and k rows rotated at their position ids (its
+    documented layout: counters, then q, then k), each within one bf16 step of the
+    oracle's rotation rounded to bf16."""
+    N, W, ks, B, H, d, theta = 5_000, 1_000, [100, 7, 50], 2, 2, 128, 500_000.0
+    M = -(-N // W)
+    k = np.resize(np.asarray(ks, np.int32), M)
+    L = focus.layout(N, W, k)
+    off = L["win_off_host"]
+    w0, w1 = 2, 5
+    a, e = int(off[w0]), int(off[w1])
+    q, kk, v = inputs.qkv((B, H, e - a, d), std=1.0, seed=61, device="cuda")
+    cache = focus.Cache(B, H, d, C_ring=L["R"], k_sched=k, rope_theta=theta)
+    ws = focus.new_prefill_workspace(cache, q, kk, v, L, w0, w1)
+    assert focus.prefill_kernel(cache, q, kk, v, L, w0, w1, workspace=ws).startswith("rotation pass + ")
+    focus.attn_prefill(cache, q, kk, v, L, w0, w1, workspace=ws)
+    torch.cuda.synchronize()
+    T = e - a
+    counters = (B * H * 4 + 255) // 256 * 256
+    n = B * H * T * d * 2
+    q_rot = ws[counters:counters + n].view(torch.bfloat16).reshape(B * H, T, d)
+    k_rot = ws[counters + n:counters + 2 * n].view(torch.bfloat16).reshape(B * H, T, d)
+    pos = a + np.arange(T)                               # the span's rows are consecutive augmented rows
+    qf = fo.rope(q.reshape(B * H, T, d).cpu(), pos, theta, round_bf16=True)
+    kf = fo.rope(kk.reshape(B * H, T, d).cpu(), pos, theta, round_bf16=True)
+    assert_keys_close(q_rot, qf, "rotated q", rel=2.0 ** -7)
+    assert_keys_close(k_rot, kf, "rotated k", rel=2.0 ** -7)
