@@ -84,6 +84,13 @@ MUTANTS = [
      "static int64_t window_bases(int64_t N, int64_t start, int32_t W) { (void)N; (void)start; return W; }",
      [lambda: pins.test_layout_sizes_closed_form(5_000, 1_024, [100]),
       lambda: pins.test_adaptive_windows_sizes_and_offsets_closed_form(1_037, [64, 1_000, 1_000], [8, 100, 3])]),
+    ("summary_src_next_base", "kind[t] = 1; src[t] = (int32_t)base; pos[t] = (int32_t)t; win[t] = w;",
+     "kind[t] = 1; src[t] = (int32_t)(base + 1); pos[t] = (int32_t)t; win[t] = w;",
+     [lambda: pins.test_layout_fig1_golden()]),
+    ("summary_token_id", "tok[(int64_t)b * T_total + t] = FO_SUMMARY_TOKEN;", "tok[(int64_t)b * T_total + t] = 0;",
+     [lambda: pins.test_layout_matches_string_construction(*pins.LAYOUT_CASES[0], True)]),
+    ("ring_offsets_one_ahead", "        ring_off[w] = (int32_t)r;", "        ring_off[w] = (int32_t)(r + 1);",
+     [lambda: pins.test_layout_positions_closed_form(10), lambda: pins.test_layout_fig1_golden()]),
     ("decode_skips_self", "        kr[c] = k_new + (size_t)s * d;\n        vr[c] = v_new + (size_t)s * d;\n        c += 1;\n"
      "        softmax_row(d,", "        softmax_row(d,", [lambda: pins.test_decode_equals_prefill_row()]),
 ]
