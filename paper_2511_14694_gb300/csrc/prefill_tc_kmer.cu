@@ -436,14 +436,19 @@ __global__ void __launch_bounds__(kThreads, 1) prefill_tc_kmer_kernel(
                     tc_fence_before();
                     mbar_arrive(smem_addr(&bars->o_free[t]));
                 }
+                const uint64_t il2 = f2_pack(inv_l, inv_l);
 #pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
-                    uint4 v;
-                    v.x = pack_bf16x2(__uint_as_float(orr[q4 * 8 + 0]) * inv_l, __uint_as_float(orr[q4 * 8 + 1]) * inv_l);
-                    v.y = pack_bf16x2(__uint_as_float(orr[q4 * 8 + 2]) * inv_l, __uint_as_float(orr[q4 * 8 + 3]) * inv_l);
-                    v.z = pack_bf16x2(__uint_as_float(orr[q4 * 8 + 4]) * inv_l, __uint_as_float(orr[q4 * 8 + 5]) * inv_l);
-                    v.w = pack_bf16x2(__uint_as_float(orr[q4 * 8 + 6]) * inv_l, __uint_as_float(orr[q4 * 8 + 7]) * inv_l);
-                    *reinterpret_cast<uint4*>(stage + lane * 64 + ((q4 ^ ((lane >> 1) & 3)) << 4)) = v;
+                for (int q4 = 0; q4 < 4; ++q4) {              // O / l, scaled in pairs
+                    uint32_t w4[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        float lo, hi;
+                        f2_unpack(f2_mul(f2_pack(__uint_as_float(orr[q4 * 8 + 2 * e]),
+                                                 __uint_as_float(orr[q4 * 8 + 2 * e + 1])), il2), lo, hi);
+                        w4[e] = pack_bf16x2(lo, hi);
+                    }
+                    *reinterpret_cast<uint4*>(stage + lane * 64 + ((q4 ^ ((lane >> 1) & 3)) << 4)) =
+                        make_uint4(w4[0], w4[1], w4[2], w4[3]);
                 }
                 __syncwarp();
 #pragma unroll
