@@ -392,3 +392,20 @@ def test_prefill_host_rejects_bad_arguments_before_any_cuda_call():
     assert lib.focus_prefill_host(ctypes.byref(c), ctypes.byref(a), 24) == 1       # lse out without a device lse
     a.h_lse, a.d_q = None, None
     assert lib.focus_prefill_host(ctypes.byref(c), ctypes.byref(a), 24) == 1       # missing device buffer
+
+
+def test_binding_constants_match_the_header():
+    """The binding's flag, token and kernel constants are the header's #defines."""
+    src = open(HEADER).read()
+    defs = {m[0]: int(m[1]) for m in re.findall(r"^#define (FOCUS_[A-Z_]+) (\d+)u?\s*$", src, re.M)}
+    assert defs["FOCUS_SUMMARY_TOKEN"] == focus.SUMMARY_TOKEN
+    assert defs["FOCUS_LAYOUT_CLOSE_TAIL"] == focus.LAYOUT_CLOSE_TAIL
+    assert defs["FOCUS_PREFILL_LEGACY_MMA"] == focus.PREFILL_LEGACY_MMA
+    assert defs["FOCUS_PREFILL_KMER_LOCAL"] == focus.PREFILL_KMER_LOCAL
+    assert defs["FOCUS_PREFILL_KERNEL_ROTATION_PASS"] == focus.PREFILL_KERNEL_ROTATION_PASS
+    names = {"FOCUS_PREFILL_KERNEL_LEGACY": "legacy mma.sync", "FOCUS_PREFILL_KERNEL_PER_ITEM":
+             "tcgen05, one CTA per work item", "FOCUS_PREFILL_KERNEL_PERSISTENT": "tcgen05 persistent",
+             "FOCUS_PREFILL_KERNEL_KMER": "tcgen05 k-mer tiles"}
+    for define, name in names.items():
+        assert focus.PREFILL_KERNELS[defs[define]] == name
+    assert all(not defs["FOCUS_PREFILL_KERNEL_ROTATION_PASS"] & k for k in focus.PREFILL_KERNELS)  # a bit of its own
